@@ -1,0 +1,181 @@
+/*
+ * deepshift.h -- C ABI of the DeepShift shift-operator library for GB300 (sm_103a).
+ *
+ * DeepShift (Elhoushi et al., "DeepShift: Towards Multiplication-Less Neural
+ * Networks") replaces every multiply of a fully-connected or convolutional
+ * layer by a bitwise shift and a sign flip (Sec. 3, Eq. 1-3).  With weight
+ * codes s in {-1, 0, +1} (Eq. 2) and p in [-15, 0] (Sec. 4) and int32
+ * activations / biases in 32-bit fixed point with 16 fraction bits (Sec. 4),
+ * every operator of this library computes, per output,
+ *
+ *     y = ReLU?( sat32( b + sum_k s_k * (x_k >> -p_k) ) )
+ *
+ * with ">>" the two's-complement arithmetic right shift (floor division by
+ * 2^-p, Eq. 1), the shift applied before the flip, the sum exact and the
+ * result saturated to the int32 range.
+ *
+ * Conventions for every entry point:
+ *   - Tensor pointers are DEVICE pointers owned by the caller.  The library
+ *     allocates no memory in any call.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Compute calls are asynchronous and stream-ordered; only
+ *     ds_pack_shift_weights synchronises its stream.
+ *   - Arguments are validated before anything is launched.  On an error the
+ *     call returns a non-zero ds_status, launches nothing, writes no output,
+ *     and ds_last_error() describes the problem.  A failed launch returns
+ *     DS_ERR_CUDA.
+ *   - Activation / output base pointers must be 16-byte aligned
+ *     (DS_ERR_ALIGNMENT otherwise).  Any positive size is accepted; tails are
+ *     handled inside the kernels.
+ */
+#ifndef DEEPSHIFT_H
+#define DEEPSHIFT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  DS_OK = 0,
+  DS_ERR_INVALID_ARG = 1,      /* null pointer, bad flag, inconsistent descriptor */
+  DS_ERR_SHAPE = 2,            /* non-positive or inconsistent dimension */
+  DS_ERR_CODE_RANGE = 3,       /* s not in {-1,0,1} or p not in [-15,0] */
+  DS_ERR_ALIGNMENT = 4,        /* pointer not 16-byte aligned */
+  DS_ERR_BUFFER_TOO_SMALL = 5, /* caller buffer smaller than required */
+  DS_ERR_UNSUPPORTED = 6,      /* valid but not supported (e.g. too large) */
+  DS_ERR_CUDA = 7              /* a CUDA runtime call or launch failed */
+} ds_status;
+
+/* Description of the last error on the calling thread ("" if none). */
+const char* ds_last_error(void);
+
+/* Library version: major * 10000 + minor * 100 + patch. */
+int ds_version(void);
+
+/* ---------------------------------------------------------------------------
+ * Flags of the compute calls
+ * ------------------------------------------------------------------------- */
+#define DS_RELU 1u      /* y = max(y, 0) after saturation (and after the residual add) */
+#define DS_AMAX_IN 2u   /* amax_io[0] already holds max|x| of the input: skip the pre-pass */
+#define DS_AMAX_OUT 4u  /* write max|y| over this call's outputs into amax_io[1] */
+#define DS_RESIDUAL 8u  /* conv only: y = sat32(sat32(conv) + residual) before the ReLU */
+#define DS_FORCE_INT64 16u /* always use the 64-bit accumulator path (testing / worst case) */
+
+/* ---------------------------------------------------------------------------
+ * Packed weights.
+ *
+ * A layer's codes are given as two int8 matrices s[n_out][k_red] and
+ * p[n_out][k_red], row-major (a conv layer's OIHW codes flattened, so
+ * k_red = C*R*S in (c, r, s) order).  They are packed once into a blob of
+ * ds_packed_weight_bytes(n_out, k_red) bytes in caller-owned device memory.
+ *
+ * Blob layout (format DS_FORMAT_PLANES6, all offsets in bytes, little endian):
+ *   [0, 256)          header written by the pack kernel:
+ *                       u32 magic (0x31575344 "DSW1"), u32 format,
+ *                       i64 n_out, i64 k_red, i64 n_chunks,
+ *                       u32 invalid_count, u32 nnz_max, u64 a_max
+ *   nib  @ 256        n_chunks x n_out records of 4 u32: for chunk g, column n,
+ *                     word w holds in bits 4i..4i+3 the value -p (0..15) of
+ *                     reduction index k = 32g + 8w + i
+ *   bits @ nib + n_chunks*n_out*16
+ *                     n_chunks x n_out records of 2 u32 {sign, nz}: bit j of
+ *                     `sign` is set iff s = -1 and bit j of `nz` iff s != 0,
+ *                     for k = 32g + j
+ *   colA @ bits + n_chunks*n_out*8
+ *                     n_out u64: A[n] = sum_k |s| * 2^(15 + p)  (sum of |w| in
+ *                     units of 2^-15; used to prove int32 accumulation exact)
+ *   nnz  @ colA + n_out*8
+ *                     n_out u32: number of non-zero codes of column n
+ * Entries with k >= k_red are zero codes.  n_chunks = ceil(k_red / 32).
+ * Storage is 6 bits per weight: 4 shift bits + sign + non-zero.  The paper's
+ * 5-bit count (Sec. 4) has 32 states, one short of the 33 states of a ternary
+ * sign times 16 shifts, so the non-zero plane is the sixth bit.
+ * ------------------------------------------------------------------------- */
+#define DS_FORMAT_PLANES6 1u
+#define DS_WEIGHTS_MAGIC 0x31575344u
+
+typedef struct ds_weights {
+  uint32_t magic;       /* DS_WEIGHTS_MAGIC once filled by ds_pack_shift_weights */
+  uint32_t format;      /* DS_FORMAT_PLANES6 */
+  int64_t n_out;        /* output columns (FC: N, conv: K) */
+  int64_t k_red;        /* reduction length (FC: K, conv: C*R*S) */
+  int64_t n_chunks;     /* ceil(k_red / 32) */
+  const void* packed;   /* device pointer to the blob (caller-owned, must outlive use) */
+  size_t packed_bytes;  /* size of the blob */
+  uint64_t a_max;       /* max over columns of A[n] */
+  uint32_t nnz_max;     /* max over columns of the non-zero count */
+  uint32_t reserved;
+} ds_weights;
+
+/* Bytes needed for the packed blob of an n_out x k_red code matrix (0 if invalid). */
+size_t ds_packed_weight_bytes(int64_t n_out, int64_t k_red);
+
+/*
+ * Pack codes (Eq. 3's shift matrix P and sign matrix S, Sec. 4 range).
+ *   s, p       device int8 [n_out][k_red], row-major.
+ *   packed     device buffer of at least ds_packed_weight_bytes(n_out, k_red)
+ *              bytes, 256-byte aligned (cudaMalloc / torch allocations are).
+ *   desc       host struct filled on success.
+ * Synchronises `stream` (an offline call) so that it can report
+ * DS_ERR_CODE_RANGE when any s is outside {-1,0,1} or p outside [-15,0]
+ * (the blob is then unusable and desc is not filled).
+ */
+ds_status ds_pack_shift_weights(const int8_t* s, const int8_t* p, int64_t n_out, int64_t k_red,
+                                void* packed, size_t packed_bytes, ds_weights* desc, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * Accumulator width.  Each compute call proves, on the device and with no
+ * host round trip, whether 32-bit accumulation is exact:
+ *     ceil(amax * A[n] / 2^15) + nnz[n] + |b[n]| <= 2^31 - 1   for every n
+ * where amax = max|x| of the input.  If so the 32-bit path runs (no
+ * wrap-around and no saturation can occur); otherwise a 64-bit path runs and
+ * the exact sum is saturated.  amax comes from amax_io[0] when DS_AMAX_IN is
+ * set, else from a pre-pass over x that writes it to amax_io[0].  amax_io
+ * (device, 2 x u32) may be NULL only with DS_FORCE_INT64 unset and then the
+ * 64-bit path is always taken.
+ * ------------------------------------------------------------------------- */
+
+/*
+ * LinearShift forward (Eq. 3, Y = flip(2^P, S) X + b; Sec. 4 fixed point):
+ *   y[m][n] = sat32( bias[n] + sum_k s[n][k] * (x[m][k] >> -p[n][k]) ), ReLU if DS_RELU.
+ *   x     device int32 [M][K] row-major (Q16.16)
+ *   w     packed weights with n_out == N and k_red == K
+ *   bias  device int32 [N] or NULL (zero bias)
+ *   y     device int32 [M][N] row-major; must not overlap x
+ *   amax_io device u32[2] or NULL (see above); DS_AMAX_OUT writes max|y| to amax_io[1]
+ */
+ds_status ds_linear_shift(const int32_t* x, const ds_weights* w, const int32_t* bias, int32_t* y,
+                          int64_t M, int64_t K, int64_t N, uint32_t flags, uint32_t* amax_io,
+                          void* stream);
+
+/*
+ * ConvShift forward (Eq. 3, Y = flip(2^P, S) (*) X + b; cross-correlation with
+ * zero padding, as the paper's PyTorch operator):
+ *   y[n][k][oh][ow] = sat32( bias[k] + sum_{c,r,q} s[k][c][r][q] *
+ *                            (xpad[n][c][oh*sh + r][ow*sw + q] >> -p[k][c][r][q]) )
+ *   then, with DS_RESIDUAL, y = sat32(y + residual[n][k][oh][ow]); then ReLU if DS_RELU.
+ *   x        device int32 NCHW [N][C][H][W]
+ *   w        packed weights with n_out == K and k_red == C*R*S
+ *   bias     device int32 [K] or NULL
+ *   residual device int32 NCHW [N][K][OH][OW], required iff DS_RESIDUAL
+ *   y        device int32 NCHW [N][K][OH][OW], OH = (H + 2*pad_h - R)/stride_h + 1
+ *   amax_io  as for ds_linear_shift
+ */
+ds_status ds_conv2d_shift(const int32_t* x, const ds_weights* w, const int32_t* bias,
+                          const int32_t* residual, int32_t* y, int N, int C, int H, int W, int K,
+                          int R, int S, int stride_h, int stride_w, int pad_h, int pad_w,
+                          uint32_t flags, uint32_t* amax_io, void* stream);
+
+/*
+ * max |x| over n int32 values, written to *amax (device u32; |INT32_MIN| = 2^31).
+ */
+ds_status ds_absmax(const int32_t* x, int64_t n, uint32_t* amax, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DEEPSHIFT_H */

@@ -1,0 +1,386 @@
+"""CPU oracle for the DeepShift inference operators.  TEST INFRASTRUCTURE ONLY.
+
+Only the tests, the smoke check and the benchmark's CPU-baseline leg may
+import this module.  The CUDA library never calls it, and it shares no code
+with the CUDA path.  It is plain and slow on purpose: every function spells
+out the definition it follows in exact integer (int64 / Python int) or
+float64 arithmetic, so a reader can check it against the paper by eye.
+
+Definitions (DeepShift, Elhoushi et al.):
+
+* Eq. 1 -- a shift by p (p <= 0 here, Sec. 4 clips p to [-15, 0]) of a
+  fixed-point integer x is the two's-complement arithmetic right shift by -p,
+  i.e. floor(x / 2^-p).
+* Eq. 2 -- the ternary sign flip: flip(v, s) = -v, 0, v for s = -1, 0, +1.
+* Eq. 3 -- LinearShift / ConvShift replace the weight W by flip(2^P, S):
+  Y = flip(2^P, S) X + b and Y = flip(2^P, S) (*) X + b.
+* Sec. 4 -- activations and bias are 32-bit fixed point with 16 fraction bits.
+
+Readings taken where the paper is silent (each is listed in the design doc):
+
+* R-order: the integer term is s * (x >> -p): shift first, then flip.
+* R-acc: the sum is exact (int64), then saturated to int32, then the
+  optional ReLU is applied.
+* R-conv: convolution is cross-correlation (PyTorch conv2d semantics), OIHW
+  weights, zero padding, reduction index order (c, r, s).
+* R-pool: max-pool ignores padded taps; average pool is floor(sum / count).
+
+Parity status: every function here is pinned by tests under
+``tests/test_oracle_pins.py`` (brute force, float64 library routines on exact
+cases, closed forms and invariants), except where a docstring says
+"parity unpinned".
+"""
+from __future__ import annotations
+
+import numpy as np
+
+INT32_MIN = -(1 << 31)
+INT32_MAX = (1 << 31) - 1
+P_MIN = -15  # Sec. 4: shifts clipped to [-15, 0]
+P_MAX = 0
+
+
+# --------------------------------------------------------------------------
+# Eq. 1 and Eq. 2 on one term
+# --------------------------------------------------------------------------
+
+def shift(x: int, p: int) -> int:
+    """Eq. 1 for p <= 0: 2^p * x on a two's-complement integer = floor(x / 2^-p)."""
+    if p > 0:
+        raise ValueError("p > 0 is outside the Sec. 4 shift range")
+    return x // (1 << (-p))
+
+
+def flip(v: int, s: int) -> int:
+    """Eq. 2: ternary sign flip."""
+    if s == -1:
+        return -v
+    if s == 0:
+        return 0
+    if s == 1:
+        return v
+    raise ValueError("s must be -1, 0 or +1")
+
+
+def term(x: int, s: int, p: int) -> int:
+    """One shift-op term s * (x >> -p) (reading R-order: shift, then flip)."""
+    return flip(shift(x, p), s)
+
+
+def sat32(v):
+    """Saturate to the int32 range (reading R-acc)."""
+    return np.clip(v, INT32_MIN, INT32_MAX)
+
+
+def _check_codes(s: np.ndarray, p: np.ndarray) -> None:
+    if s.shape != p.shape:
+        raise ValueError("s and p must have the same shape")
+    if not np.isin(s, (-1, 0, 1)).all():
+        raise ValueError("sign codes must be in {-1, 0, +1} (Eq. 2)")
+    if ((p < P_MIN) | (p > P_MAX)).any():
+        raise ValueError("shift codes must be in [-15, 0] (Sec. 4)")
+
+
+# --------------------------------------------------------------------------
+# LinearShift (Eq. 3, fully-connected form)
+# --------------------------------------------------------------------------
+
+def linear_shift_acc(x: np.ndarray, s: np.ndarray, p: np.ndarray, b=None) -> np.ndarray:
+    """Exact int64 accumulator of LinearShift before saturation.
+
+    acc[m, n] = b[n] + sum_k s[n, k] * floor(x[m, k] / 2^-p[n, k]).
+    x: [M, K] integer; s, p: [N, K]; b: [N] or None.  Returns int64 [M, N].
+    The loop runs over k; each step adds one term to every (m, n).
+    """
+    x = np.asarray(x, dtype=np.int64)
+    s = np.asarray(s, dtype=np.int64)
+    p = np.asarray(p, dtype=np.int64)
+    _check_codes(s, p)
+    M, K = x.shape
+    N, K2 = s.shape
+    if K != K2:
+        raise ValueError("x and codes disagree on K")
+    acc = np.zeros((M, N), dtype=np.int64)
+    if b is not None:
+        acc += np.asarray(b, dtype=np.int64)[None, :]
+    for k in range(K):
+        divisor = np.left_shift(np.int64(1), -p[:, k])          # 2^-p per output column
+        shifted = np.floor_divide(x[:, k][:, None], divisor[None, :])  # Eq. 1
+        acc += s[:, k][None, :] * shifted                         # Eq. 2 flip, then sum
+    return acc
+
+
+def linear_shift(x, s, p, b=None, relu: bool = False) -> np.ndarray:
+    """LinearShift forward on Q16.16 int32: sat32(acc), then optional ReLU.  Returns int32."""
+    y = sat32(linear_shift_acc(x, s, p, b))
+    if relu:
+        y = np.maximum(y, 0)
+    return y.astype(np.int32)
+
+
+# --------------------------------------------------------------------------
+# ConvShift (Eq. 3, convolutional form)
+# --------------------------------------------------------------------------
+
+def conv_out_size(h: int, r: int, stride: int, pad: int) -> int:
+    return (h + 2 * pad - r) // stride + 1
+
+
+def conv2d_shift_acc(x, s, p, b=None, stride=(1, 1), pad=(0, 0)) -> np.ndarray:
+    """Exact int64 accumulator of ConvShift before saturation.
+
+    acc[n, k, oh, ow] = b[k] + sum_{c, r, q} s[k, c, r, q] *
+        floor(xpad[n, c, oh*sh + r, ow*sw + q] / 2^-p[k, c, r, q])
+    with xpad the input zero-padded by pad on each side (reading R-conv).
+    x: [N, C, H, W]; s, p: [K, C, R, S]; returns int64 [N, K, OH, OW].
+    """
+    x = np.asarray(x, dtype=np.int64)
+    s = np.asarray(s, dtype=np.int64)
+    p = np.asarray(p, dtype=np.int64)
+    _check_codes(s, p)
+    N, C, H, W = x.shape
+    K, C2, R, S = s.shape
+    if C != C2:
+        raise ValueError("x and codes disagree on C")
+    sh, sw = stride
+    ph, pw = pad
+    OH = conv_out_size(H, R, sh, ph)
+    OW = conv_out_size(W, S, sw, pw)
+    xpad = np.zeros((N, C, H + 2 * ph, W + 2 * pw), dtype=np.int64)
+    xpad[:, :, ph:ph + H, pw:pw + W] = x
+    acc = np.zeros((N, K, OH, OW), dtype=np.int64)
+    if b is not None:
+        acc += np.asarray(b, dtype=np.int64)[None, :, None, None]
+    for c in range(C):
+        for r in range(R):
+            for q in range(S):
+                # input tap seen by every output pixel for this (c, r, q): [N, OH, OW]
+                tap = xpad[:, c, r:r + sh * (OH - 1) + 1:sh, q:q + sw * (OW - 1) + 1:sw]
+                divisor = np.left_shift(np.int64(1), -p[:, c, r, q])   # [K]
+                shifted = np.floor_divide(tap[:, None, :, :], divisor[None, :, None, None])
+                acc += s[:, c, r, q][None, :, None, None] * shifted
+    return acc
+
+
+def conv2d_shift(x, s, p, b=None, stride=(1, 1), pad=(0, 0), relu: bool = False) -> np.ndarray:
+    """ConvShift forward on Q16.16 int32 NCHW: sat32(acc), then optional ReLU.  Returns int32."""
+    y = sat32(conv2d_shift_acc(x, s, p, b, stride, pad))
+    if relu:
+        y = np.maximum(y, 0)
+    return y.astype(np.int32)
+
+
+def conv2d_shift_at(x, s, p, b, stride, pad, n: int, k: int, oh: int, ow: int) -> int:
+    """One output element of ConvShift (before saturation), as a Python int.
+
+    Used to check sampled outputs of full-size launches one by one.
+    """
+    N, C, H, W = x.shape
+    _, _, R, S = s.shape
+    acc = int(b[k]) if b is not None else 0
+    for c in range(C):
+        for r in range(R):
+            for q in range(S):
+                ih = oh * stride[0] + r - pad[0]
+                iw = ow * stride[1] + q - pad[1]
+                v = int(x[n, c, ih, iw]) if (0 <= ih < H and 0 <= iw < W) else 0
+                acc += term(v, int(s[k, c, r, q]), int(p[k, c, r, q]))
+    return acc
+
+
+def linear_shift_at(x, s, p, b, m: int, n: int) -> int:
+    """One output element of LinearShift (before saturation), as a Python int."""
+    acc = int(b[n]) if b is not None else 0
+    for k in range(x.shape[1]):
+        acc += term(int(x[m, k]), int(s[n, k]), int(p[n, k]))
+    return acc
+
+
+# --------------------------------------------------------------------------
+# Accumulator-width bound (reading R-acc): when int32 accumulation is exact
+# --------------------------------------------------------------------------
+
+def absmax(x) -> int:
+    """max |x| over an int32 tensor, as a non-negative Python int (|INT32_MIN| = 2^31)."""
+    x = np.asarray(x, dtype=np.int64)
+    return int(np.abs(x).max()) if x.size else 0
+
+
+def column_constants(s, p):
+    """Per output column n (rows of the [N, Kred] code matrix):
+
+    A[n]   = sum_k |s[n,k]| * 2^(15 + p[n,k])   (sum of |weights| in units of 2^-15)
+    nnz[n] = #{k : s[n,k] != 0}
+    """
+    s = np.asarray(s, dtype=np.int64).reshape(np.shape(s)[0], -1)
+    p = np.asarray(p, dtype=np.int64).reshape(np.shape(p)[0], -1)
+    A = (np.abs(s) * np.left_shift(np.int64(1), 15 + p)).sum(axis=1)
+    nnz = (s != 0).sum(axis=1)
+    return A.astype(np.int64), nnz.astype(np.int64)
+
+
+def int32_accumulation_is_exact(amax: int, A: int, nnz: int, babs: int) -> bool:
+    """True when |b| + sum |s * (x >> -p)| <= INT32_MAX for every |x| <= amax.
+
+    |floor(x / 2^k)| <= ceil(|x| / 2^k) <= |x| / 2^k + 1 - 2^-k, so the sum is at
+    most ceil(amax * A / 2^15) + nnz + |b|.
+    """
+    return ((amax * A + (1 << 15) - 1) >> 15) + nnz + babs <= INT32_MAX
+
+
+# --------------------------------------------------------------------------
+# Chain operators (pools, residual) for ResNet / VGG shaped forwards
+# --------------------------------------------------------------------------
+
+def maxpool2d(x, k: int, stride: int, pad: int) -> np.ndarray:
+    """Integer max-pool; padded taps are ignored (reading R-pool)."""
+    x = np.asarray(x, dtype=np.int64)
+    N, C, H, W = x.shape
+    OH = conv_out_size(H, k, stride, pad)
+    OW = conv_out_size(W, k, stride, pad)
+    out = np.full((N, C, OH, OW), np.iinfo(np.int64).min, dtype=np.int64)
+    for r in range(k):
+        for q in range(k):
+            for oh in range(OH):
+                ih = oh * stride + r - pad
+                if not 0 <= ih < H:
+                    continue
+                for ow in range(OW):
+                    iw = ow * stride + q - pad
+                    if 0 <= iw < W:
+                        out[:, :, oh, ow] = np.maximum(out[:, :, oh, ow], x[:, :, ih, iw])
+    return out.astype(np.int32)
+
+
+def avgpool_floor(x, k: int, stride: int) -> np.ndarray:
+    """Integer average pool without padding: floor(sum / (k*k)) (reading R-pool)."""
+    x = np.asarray(x, dtype=np.int64)
+    N, C, H, W = x.shape
+    OH = (H - k) // stride + 1
+    OW = (W - k) // stride + 1
+    out = np.zeros((N, C, OH, OW), dtype=np.int64)
+    for oh in range(OH):
+        for ow in range(OW):
+            win = x[:, :, oh * stride:oh * stride + k, ow * stride:ow * stride + k]
+            out[:, :, oh, ow] = np.floor_divide(win.sum(axis=(2, 3)), k * k)
+    return out.astype(np.int32)
+
+
+def add_relu(a, b) -> np.ndarray:
+    """Residual join: ReLU(sat32(a + b)) on int32 tensors."""
+    v = sat32(np.asarray(a, dtype=np.int64) + np.asarray(b, dtype=np.int64))
+    return np.maximum(v, 0).astype(np.int32)
+
+
+# --------------------------------------------------------------------------
+# Float variant (bf16 activations, weights s * 2^p, float64 reference)
+# --------------------------------------------------------------------------
+
+def linear_shift_float(x_f64, s, p, b=None) -> np.ndarray:
+    """y[m, n] = b[n] + sum_k s[n,k] * 2^p[n,k] * x[m,k] in float64 (Eq. 3 with W = flip(2^P, S)).
+
+    x_f64 holds the exact values of the bf16 activations.  Also returns nothing
+    else: the tolerance scale sum |terms| comes from :func:`linear_shift_float_absterms`.
+    """
+    x = np.asarray(x_f64, dtype=np.float64)
+    s = np.asarray(s, dtype=np.int64)
+    p = np.asarray(p, dtype=np.int64)
+    _check_codes(s, p)
+    M, K = x.shape
+    N = s.shape[0]
+    y = np.zeros((M, N), dtype=np.float64)
+    if b is not None:
+        y += np.asarray(b, dtype=np.float64)[None, :]
+    for k in range(K):
+        w = s[:, k].astype(np.float64) * np.ldexp(1.0, p[:, k])   # flip(2^p, s)
+        y += x[:, k][:, None] * w[None, :]
+    return y
+
+
+def linear_shift_float_absterms(x_f64, s, p) -> np.ndarray:
+    """sum_k |s * 2^p * x| per output, the scale of the float variant's tolerance."""
+    x = np.abs(np.asarray(x_f64, dtype=np.float64))
+    w = np.abs(np.asarray(s, dtype=np.float64)) * np.ldexp(1.0, np.asarray(p, dtype=np.int64))
+    return x @ w.T
+
+
+# --------------------------------------------------------------------------
+# Packed weight blob (the library's storage format for the codes of Eq. 3;
+# layout documented in include/deepshift.h, format "planes6")
+# --------------------------------------------------------------------------
+
+BLOB_HEADER = 256
+BLOB_MAGIC = 0x31575344
+FORMAT_PLANES6 = 1
+
+
+def blob_layout(n_out: int, k_red: int) -> dict:
+    """Byte offsets of the regions of a planes6 blob."""
+    n_chunks = (k_red + 31) // 32
+    nib = BLOB_HEADER
+    bits = nib + n_chunks * n_out * 16
+    col_a = bits + n_chunks * n_out * 8
+    nnz = col_a + n_out * 8
+    end = nnz + n_out * 4
+    total = (end + 255) // 256 * 256
+    return dict(n_chunks=n_chunks, nib=nib, bits=bits, col_a=col_a, nnz=nnz, total=total)
+
+
+def pack_planes6(s, p) -> np.ndarray:
+    """Pack [n_out, k_red] codes into the planes6 blob, one weight at a time.
+
+    Returns the blob as uint8 [total].  The header carries magic, format, dims,
+    invalid_count = 0, nnz_max and a_max.
+    """
+    s = np.asarray(s, dtype=np.int64)
+    p = np.asarray(p, dtype=np.int64)
+    _check_codes(s, p)
+    n_out, k_red = s.shape
+    L = blob_layout(n_out, k_red)
+    nch = L["n_chunks"]
+    nib = np.zeros((nch, n_out, 4), dtype=np.uint32)
+    bits = np.zeros((nch, n_out, 2), dtype=np.uint32)
+    for n in range(n_out):
+        for k in range(k_red):
+            g, j = divmod(k, 32)
+            w, i = divmod(j, 8)
+            nib[g, n, w] |= np.uint32((-p[n, k]) << (4 * i))
+            if s[n, k] == -1:
+                bits[g, n, 0] |= np.uint32(1 << j)
+            if s[n, k] != 0:
+                bits[g, n, 1] |= np.uint32(1 << j)
+    A, nnz = column_constants(s, p)
+    blob = np.zeros(L["total"], dtype=np.uint8)
+    hdr = np.zeros(BLOB_HEADER, dtype=np.uint8)
+    hdr[0:4] = np.frombuffer(np.uint32(BLOB_MAGIC).tobytes(), np.uint8)
+    hdr[4:8] = np.frombuffer(np.uint32(FORMAT_PLANES6).tobytes(), np.uint8)
+    hdr[8:32] = np.frombuffer(np.array([n_out, k_red, nch], dtype=np.int64).tobytes(), np.uint8)
+    hdr[32:36] = 0  # invalid_count
+    hdr[36:40] = np.frombuffer(np.uint32(int(nnz.max()) if n_out else 0).tobytes(), np.uint8)
+    hdr[40:48] = np.frombuffer(np.uint64(int(A.max()) if n_out else 0).tobytes(), np.uint8)
+    blob[:BLOB_HEADER] = hdr
+    blob[L["nib"]:L["bits"]] = np.frombuffer(nib.tobytes(), np.uint8)
+    blob[L["bits"]:L["col_a"]] = np.frombuffer(bits.tobytes(), np.uint8)
+    blob[L["col_a"]:L["nnz"]] = np.frombuffer(A.astype(np.uint64).tobytes(), np.uint8)
+    blob[L["nnz"]:L["nnz"] + 4 * n_out] = np.frombuffer(nnz.astype(np.uint32).tobytes(), np.uint8)
+    return blob
+
+
+def unpack_planes6(blob, n_out: int, k_red: int):
+    """Inverse of pack_planes6 for the code regions: returns (s, p) int8 [n_out, k_red]."""
+    blob = np.asarray(blob, dtype=np.uint8)
+    L = blob_layout(n_out, k_red)
+    nch = L["n_chunks"]
+    nib = np.frombuffer(blob[L["nib"]:L["bits"]].tobytes(), np.uint32).reshape(nch, n_out, 4)
+    bits = np.frombuffer(blob[L["bits"]:L["col_a"]].tobytes(), np.uint32).reshape(nch, n_out, 2)
+    s = np.zeros((n_out, k_red), dtype=np.int8)
+    p = np.zeros((n_out, k_red), dtype=np.int8)
+    for n in range(n_out):
+        for k in range(k_red):
+            g, j = divmod(k, 32)
+            w, i = divmod(j, 8)
+            p[n, k] = -int((int(nib[g, n, w]) >> (4 * i)) & 15)
+            neg = (int(bits[g, n, 0]) >> j) & 1
+            nz = (int(bits[g, n, 1]) >> j) & 1
+            s[n, k] = 0 if not nz else (-1 if neg else 1)
+    return s, p

@@ -1,0 +1,414 @@
+"""Pins of the CPU oracle against what the paper and mathematics fix.
+
+No test here compares the oracle with a retyped copy of itself.  Each pin
+reaches the expected value another way: hand-derived values (golden
+fixtures), exact rational arithmetic, two's-complement bit strings, float64
+library routines on inputs where the shift is exact, closed forms and
+invariants.  A plausible mistake in the oracle (a dropped term, a wrong sign,
+shift direction or rounding, a transposed operand, a misplaced tap, a missing
+bias or clamp) fails at least one of them.
+"""
+import math
+import os
+from fractions import Fraction
+
+import numpy as np
+import pytest
+import torch
+import torch.nn.functional as F
+
+import synth_inputs as si
+from oracle import deepshift_oracle as O
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _read_golden(name):
+    rows = []
+    with open(os.path.join(GOLDEN, name)) as f:
+        for line in f:
+            line = line.split("#", 1)[0].strip()
+            if line:
+                rows.append(line.split())
+    return rows
+
+
+def _golden_layer(case):
+    d = {}
+    for row in _read_golden("layer_cases.txt"):
+        if row[0] == case:
+            d[row[1]] = [int(v) for v in row[2:]]
+    return d
+
+
+# --------------------------------------------------------------------------
+# Single term: Eq. 1 and Eq. 2
+# --------------------------------------------------------------------------
+
+def test_term_golden_cases():
+    rows = _read_golden("term_cases.txt")
+    assert len(rows) >= 20
+    for x, p, s, want in rows:
+        assert O.term(int(x), int(s), int(p)) == int(want), (x, p, s)
+
+
+EDGE_X = [-(1 << 31), -(1 << 31) + 1, -(1 << 16) - 1, -(1 << 16), -(1 << 15) - 1, -(1 << 15),
+          -(1 << 15) + 1, -3, -2, -1, 0, 1, 2, 3, (1 << 15) - 1, 1 << 15, (1 << 15) + 1,
+          (1 << 20) - 1, (1 << 31) - 2, (1 << 31) - 1]
+
+
+def _twos_complement_shift(x: int, k: int) -> int:
+    """Arithmetic right shift done on the 32-bit two's-complement bit string."""
+    bits = format(x & 0xFFFFFFFF, "032b")
+    shifted = bits[0] * k + bits[:32 - k]          # replicate the sign bit
+    v = int(shifted, 2)
+    return v - (1 << 32) if shifted[0] == "1" else v
+
+
+def test_term_exhaustive_codes_vs_rational_floor_and_bit_strings():
+    """All 33 code states x edge activations: Eq. 1 as exact rational floor and as a bit-string shift."""
+    for p in range(-15, 1):
+        for s in (-1, 0, 1):
+            for x in EDGE_X:
+                want_rational = s * math.floor(Fraction(x, 2 ** (-p)))
+                want_bits = s * _twos_complement_shift(x, -p)
+                got = O.term(x, s, p)
+                assert got == want_rational == want_bits, (x, s, p)
+
+
+def test_term_rejects_out_of_range_codes():
+    with pytest.raises(ValueError):
+        O.shift(5, 1)
+    with pytest.raises(ValueError):
+        O.flip(5, 2)
+    x = np.zeros((1, 2), np.int32)
+    with pytest.raises(ValueError):
+        O.linear_shift(x, np.array([[1, 2]]), np.array([[0, 0]]))
+    with pytest.raises(ValueError):
+        O.linear_shift(x, np.array([[1, 1]]), np.array([[0, -16]]))
+
+
+# --------------------------------------------------------------------------
+# LinearShift (Eq. 3)
+# --------------------------------------------------------------------------
+
+def test_linear_golden_cases():
+    for case in ("fc1", "sat1"):
+        g = _golden_layer(case)
+        x = np.array([g["x"]], np.int64)
+        K = x.shape[1]
+        N = len(g["b"])
+        s = np.array(g["s"], np.int64).reshape(N, K)
+        p = np.array(g["p"], np.int64).reshape(N, K)
+        b = np.array(g["b"], np.int64)
+        assert O.linear_shift(x, s, p, b).ravel().tolist() == g["y"]
+        assert O.linear_shift(x, s, p, b, relu=True).ravel().tolist() == g["y_relu"]
+
+
+def test_linear_brute_force_tiny():
+    """Every output of random tiny layers equals the sum of rational-floor terms."""
+    rng = np.random.default_rng(7)
+    for _ in range(25):
+        M, K, N = rng.integers(1, 5, size=3)
+        x = rng.choice(EDGE_X, size=(M, K)).astype(np.int64)
+        s = rng.integers(-1, 2, size=(N, K))
+        p = rng.integers(-15, 1, size=(N, K))
+        b = rng.integers(-(1 << 31), 1 << 31, size=N)
+        acc = O.linear_shift_acc(x, s, p, b)
+        for m in range(M):
+            for n in range(N):
+                want = int(b[n]) + sum(int(s[n, k]) * math.floor(Fraction(int(x[m, k]), 2 ** int(-p[n, k])))
+                                       for k in range(K))
+                assert acc[m, n] == want
+                assert O.linear_shift_at(x, s, p, b, m, n) == want
+
+
+def test_linear_exact_float64_when_x_multiple_of_2_15():
+    """x = 2^15 u makes every shift exact, so acc - b equals the float64 matmul with W = s 2^p."""
+    rng = np.random.default_rng(11)
+    M, K, N = 13, 77, 9
+    u = rng.integers(-(1 << 16), 1 << 16, size=(M, K))
+    x = u * (1 << 15)
+    s = rng.integers(-1, 2, size=(N, K))
+    p = rng.integers(-15, 1, size=(N, K))
+    b = rng.integers(-(1 << 16), 1 << 16, size=N)
+    W = s.astype(np.float64) * np.ldexp(1.0, p)
+    want = torch.from_numpy(x.astype(np.float64)) @ torch.from_numpy(W).T
+    got = O.linear_shift_acc(x, s, p, b) - b[None, :]
+    assert np.array_equal(got.astype(np.float64), want.numpy())
+
+
+def test_linear_ternary_p0_is_int_matmul():
+    rng = np.random.default_rng(12)
+    x = rng.integers(-(1 << 20), 1 << 20, size=(6, 50))
+    s = rng.integers(-1, 2, size=(7, 50))
+    p = np.zeros_like(s)
+    assert np.array_equal(O.linear_shift_acc(x, s, p), np.matmul(x, s.T))
+
+
+def test_linear_negation_invariance():
+    """s -> -s negates acc - b exactly; x -> -x does not (floor), which is documented here."""
+    x, s, p, b = si.fc_layer(3, 8, 40, 6, -(1 << 20), 1 << 20)
+    b = b.astype(np.int64)
+    a = O.linear_shift_acc(x, s, p, b) - b
+    a_neg = O.linear_shift_acc(x, -s, p, b) - b
+    assert np.array_equal(a_neg, -a)
+    a_xneg = O.linear_shift_acc(-x.astype(np.int64), s, p, b) - b
+    assert not np.array_equal(a_xneg, -a)
+
+
+def test_linear_split_k_additive():
+    x, s, p, b = si.fc_layer(4, 5, 70, 3, -(1 << 20), 1 << 20)
+    full = O.linear_shift_acc(x, s, p)
+    part = O.linear_shift_acc(x[:, :33], s[:, :33], p[:, :33]) + O.linear_shift_acc(x[:, 33:], s[:, 33:], p[:, 33:])
+    assert np.array_equal(full, part)
+
+
+def test_linear_trivial_weights():
+    x, s, p, b = si.fc_layer(5, 4, 30, 5, -(1 << 31), 1 << 31)
+    # all-zero signs: y = sat(b)
+    assert np.array_equal(O.linear_shift(x, np.zeros_like(s), p, b), np.broadcast_to(b, (4, 5)))
+    # one-hot code at k0 with shift q: y = x[:, k0] >> q
+    for q in (0, 1, 7, 15):
+        s1 = np.zeros_like(s)
+        s1[:, 3] = 1
+        p1 = np.full_like(p, -q)
+        want = np.floor_divide(x[:, 3].astype(np.int64), 1 << q)
+        got = O.linear_shift(x, s1, p1)
+        assert np.array_equal(got, np.repeat(want[:, None], 5, axis=1))
+
+
+def test_linear_saturation_boundaries():
+    # exact sum lands on INT32_MAX, INT32_MAX + 1, INT32_MIN, INT32_MIN - 1
+    x = np.array([[(1 << 30), (1 << 30) - 1, 1]], np.int64)
+    s = np.array([[1, 1, 0], [1, 1, 1], [-1, -1, -1], [-1, -1, -1]])
+    p = np.zeros_like(s)
+    b = np.array([0, 0, 0, -1])
+    y = O.linear_shift(x, s, p, b)
+    assert y.ravel().tolist() == [(1 << 31) - 1, (1 << 31) - 1, -(1 << 31), -(1 << 31)]
+    acc = O.linear_shift_acc(x, s, p, b).ravel().tolist()
+    assert acc == [(1 << 31) - 1, 1 << 31, -(1 << 31), -(1 << 31) - 1]
+
+
+def test_accumulation_bound_holds_and_is_tight():
+    rng = np.random.default_rng(21)
+    for _ in range(30):
+        M, K, N = 4, int(rng.integers(1, 60)), 3
+        amax_bits = int(rng.integers(1, 32))
+        x = rng.integers(-(1 << amax_bits), 1 << amax_bits, size=(M, K))
+        x = np.clip(x, -(1 << 31), (1 << 31) - 1)
+        s = rng.integers(-1, 2, size=(N, K))
+        p = rng.integers(-15, 1, size=(N, K))
+        b = rng.integers(-(1 << 20), 1 << 20, size=N)
+        A, nnz = O.column_constants(s, p)
+        amax = O.absmax(x)
+        acc = O.linear_shift_acc(x, s, p, b)
+        for n in range(N):
+            bound = ((amax * int(A[n]) + (1 << 15) - 1) >> 15) + int(nnz[n]) + abs(int(b[n]))
+            assert np.abs(acc[:, n]).max() <= bound
+    # worst case attains ceil(amax / 2^k) per term
+    amax = (1 << 20) + 5
+    ks = np.arange(16)
+    x = np.full((1, 16), -amax)
+    s = -np.ones((1, 16), np.int64)
+    p = -ks[None, :]
+    acc = int(O.linear_shift_acc(x, s, p)[0, 0])
+    assert acc == sum(-(-amax // (1 << int(k))) for k in ks)
+    A, nnz = O.column_constants(s, p)
+    assert acc <= ((amax * int(A[0]) + (1 << 15) - 1) >> 15) + int(nnz[0])
+    # -INT32_MIN with s = -1 does not fit int32: the bound must refuse it
+    assert not O.int32_accumulation_is_exact(1 << 31, 1 << 15, 1, 0)
+    assert O.int32_accumulation_is_exact((1 << 31) - 2, 1 << 15, 1, 0)
+
+
+def test_column_constants_closed_forms():
+    K = 37
+    s = np.ones((3, K), np.int64)
+    p = np.stack([np.zeros(K), np.full(K, -15), np.full(K, -3)]).astype(np.int64)
+    A, nnz = O.column_constants(s, p)
+    assert A.tolist() == [K << 15, K, K << 12]
+    assert nnz.tolist() == [K, K, K]
+    s[1, ::2] = 0
+    A, nnz = O.column_constants(s, p)
+    assert A[1] == K // 2 and nnz[1] == K // 2
+
+
+# --------------------------------------------------------------------------
+# ConvShift (Eq. 3, convolution form)
+# --------------------------------------------------------------------------
+
+def test_conv_golden_cases():
+    x = np.arange(1, 10, dtype=np.int64).reshape(1, 1, 3, 3)
+    s = np.zeros((1, 1, 3, 3), np.int64)
+    s[0, 0, 0, 2] = 1
+    p = np.zeros_like(s)
+    y = O.conv2d_shift(x, s, p, None, (1, 1), (1, 1))
+    assert y.ravel().tolist() == _golden_layer("conv_xcorr")["y"]
+    g = _golden_layer("conv_half")
+    y = O.conv2d_shift(x, np.ones_like(s), -np.ones_like(s), None, (1, 1), (1, 1))[0, 0]
+    for key, (i, j) in {"y00": (0, 0), "y01": (0, 1), "y10": (1, 0), "y11": (1, 1), "y22": (2, 2)}.items():
+        assert y[i, j] == g[key][0]
+    # 1x1 stride 2: subsampling
+    x = np.arange(16, dtype=np.int64).reshape(1, 1, 4, 4)
+    y = O.conv2d_shift(x, np.ones((1, 1, 1, 1)), np.zeros((1, 1, 1, 1)), None, (2, 2), (0, 0))
+    assert y.ravel().tolist() == [0, 2, 8, 10]
+
+
+@pytest.mark.parametrize("geom", [(2, 3, 7, 6, 4, 3, 3, 1, 1, 1, 1), (1, 2, 9, 9, 3, 3, 3, 2, 2, 1, 1),
+                                  (2, 3, 11, 10, 2, 7, 7, 2, 2, 3, 3), (1, 4, 6, 5, 3, 1, 1, 2, 2, 0, 0),
+                                  (1, 2, 5, 7, 2, 3, 1, 1, 2, 0, 2)])
+def test_conv_exact_float64_when_x_multiple_of_2_15(geom):
+    """x = 2^15 u: acc - b equals torch's float64 conv2d with W = s 2^p (cross-correlation)."""
+    N, C, H, W, K, R, S, sh, sw, ph, pw = geom
+    rng = np.random.default_rng(sum(geom))
+    x = rng.integers(-(1 << 16), 1 << 16, size=(N, C, H, W)) * (1 << 15)
+    s = rng.integers(-1, 2, size=(K, C, R, S))
+    p = rng.integers(-15, 1, size=(K, C, R, S))
+    b = rng.integers(-(1 << 16), 1 << 16, size=K)
+    Wt = torch.from_numpy(s.astype(np.float64) * np.ldexp(1.0, p))
+    want = F.conv2d(torch.from_numpy(x.astype(np.float64)), Wt, stride=(sh, sw), padding=(ph, pw))
+    got = O.conv2d_shift_acc(x, s, p, b, (sh, sw), (ph, pw)) - b[None, :, None, None]
+    assert got.shape == tuple(want.shape)
+    assert np.array_equal(got.astype(np.float64), want.numpy())
+
+
+def _im2col(x, R, S, stride, pad):
+    """Explicit patch gather: rows = (n, oh, ow), columns = (c, r, q), zero outside the image."""
+    N, C, H, W = x.shape
+    OH = (H + 2 * pad[0] - R) // stride[0] + 1
+    OW = (W + 2 * pad[1] - S) // stride[1] + 1
+    cols = np.zeros((N * OH * OW, C * R * S), dtype=np.int64)
+    for n in range(N):
+        for oh in range(OH):
+            for ow in range(OW):
+                row = (n * OH + oh) * OW + ow
+                for c in range(C):
+                    for r in range(R):
+                        for q in range(S):
+                            ih = oh * stride[0] - pad[0] + r
+                            iw = ow * stride[1] - pad[1] + q
+                            if 0 <= ih < H and 0 <= iw < W:
+                                cols[row, (c * R + r) * S + q] = x[n, c, ih, iw]
+    return cols, OH, OW
+
+
+@pytest.mark.parametrize("geom", [(2, 3, 6, 5, 4, 3, 3, 1, 1, 1, 1), (1, 2, 9, 8, 3, 7, 7, 2, 2, 3, 3),
+                                  (1, 3, 7, 7, 2, 3, 3, 2, 2, 1, 1)])
+def test_conv_equals_im2col_plus_linear(geom):
+    N, C, H, W, K, R, S, sh, sw, ph, pw = geom
+    x, s, p, b = si.conv_layer(sum(geom), N, C, H, W, K, R, S, -(1 << 20), 1 << 20)
+    cols, OH, OW = _im2col(x.astype(np.int64), R, S, (sh, sw), (ph, pw))
+    lin = O.linear_shift_acc(cols, s.reshape(K, -1), p.reshape(K, -1), b)
+    lin = lin.reshape(N, OH, OW, K).transpose(0, 3, 1, 2)
+    assert np.array_equal(O.conv2d_shift_acc(x, s, p, b, (sh, sw), (ph, pw)), lin)
+
+
+def test_conv_identity_and_sampled_elements():
+    x, s, p, b = si.conv_layer(9, 2, 4, 6, 6, 4, 1, 1, -(1 << 31), 1 << 31)
+    eye_s = np.eye(4, dtype=np.int64).reshape(4, 4, 1, 1)
+    y = O.conv2d_shift(x, eye_s, np.zeros_like(eye_s), None)
+    assert np.array_equal(y, x)
+    x, s, p, b = si.conv_layer(10, 2, 3, 7, 6, 5, 3, 3)
+    acc = O.conv2d_shift_acc(x, s, p, b, (2, 1), (1, 0))
+    for (n, k, oh, ow) in [(0, 0, 0, 0), (1, 4, 3, 3), (0, 2, 1, 2), (1, 1, 3, 0)]:
+        assert acc[n, k, oh, ow] == O.conv2d_shift_at(x, s, p, b, (2, 1), (1, 0), n, k, oh, ow)
+
+
+def test_conv_negation_invariance():
+    x, s, p, b = si.conv_layer(13, 1, 3, 6, 6, 4, 3, 3, -(1 << 20), 1 << 20)
+    bb = b.astype(np.int64)[None, :, None, None]
+    a = O.conv2d_shift_acc(x, s, p, b, (1, 1), (1, 1)) - bb
+    assert np.array_equal(O.conv2d_shift_acc(x, -s, p, b, (1, 1), (1, 1)) - bb, -a)
+
+
+# --------------------------------------------------------------------------
+# Chain operators
+# --------------------------------------------------------------------------
+
+def test_maxpool_golden_and_library():
+    x = np.array([[[[-1, -2], [-3, -4]]]], np.int32)
+    assert O.maxpool2d(x, 3, 2, 1).ravel().tolist() == _golden_layer("maxpool_neg")["y"]
+    rng = np.random.default_rng(3)
+    x = rng.integers(-(1 << 31), 1 << 31, size=(2, 3, 11, 10)).astype(np.int32)
+    want = F.max_pool2d(torch.from_numpy(x.astype(np.float64)), 3, 2, 1).numpy()
+    assert np.array_equal(O.maxpool2d(x, 3, 2, 1).astype(np.float64), want)
+    want2 = F.max_pool2d(torch.from_numpy(x.astype(np.float64)), 2, 2, 0).numpy()
+    assert np.array_equal(O.maxpool2d(x, 2, 2, 0).astype(np.float64), want2)
+
+
+def test_avgpool_floor_golden_and_library():
+    g = _golden_layer("avgpool_floor")
+    for key in ("a", "b"):
+        x = np.array(g[key], np.int32).reshape(1, 1, 2, 2)
+        assert O.avgpool_floor(x, 2, 2).ravel().tolist() == g[key + "_y"]
+    rng = np.random.default_rng(4)
+    x = rng.integers(-(1 << 31), 1 << 31, size=(2, 5, 7, 7)).astype(np.int32)
+    mean = F.avg_pool2d(torch.from_numpy(x.astype(np.float64)), 7).numpy()
+    assert np.array_equal(O.avgpool_floor(x, 7, 7).astype(np.float64), np.floor(mean))
+
+
+def test_add_relu_golden():
+    g = _golden_layer("add_relu")
+    assert O.add_relu(np.array(g["a"], np.int32), np.array(g["b"], np.int32)).tolist() == g["y"]
+
+
+# --------------------------------------------------------------------------
+# Float variant
+# --------------------------------------------------------------------------
+
+def test_float_variant_exact_on_small_integers_and_near_library():
+    rng = np.random.default_rng(5)
+    M, K, N = 9, 64, 7
+    xi = rng.integers(-100, 100, size=(M, K))
+    s = rng.integers(-1, 2, size=(N, K))
+    p = rng.integers(-15, 1, size=(N, K))
+    got = O.linear_shift_float(xi.astype(np.float64), s, p)
+    for m in range(M):
+        for n in range(N):
+            want = sum(Fraction(int(s[n, k]) * int(xi[m, k])) * Fraction(1, 2 ** int(-p[n, k])) for k in range(K))
+            assert Fraction(got[m, n]) == want
+    x = si.bits_to_f64(si.bf16_bits(rng.uniform(-(1 << 20), 1 << 20, size=(M, K))))
+    b = rng.uniform(-1, 1, size=N)
+    W = s.astype(np.float64) * np.ldexp(1.0, p)
+    lib = x @ W.T + b
+    got = O.linear_shift_float(x, s, p, b)
+    scale = O.linear_shift_float_absterms(x, s, p) + np.abs(b)
+    assert np.all(np.abs(got - lib) <= 1e-13 * scale)
+
+
+# --------------------------------------------------------------------------
+# Packed blob (storage format of the codes)
+# --------------------------------------------------------------------------
+
+def test_pack_golden_tiny_blob():
+    g = {r[0]: [int(v) for v in r[1:]] for r in _read_golden("pack_tiny.txt")}
+    s = np.array(g["s"]).reshape(2, 3)
+    p = np.array(g["p"]).reshape(2, 3)
+    blob = O.pack_planes6(s, p)
+    L = O.blob_layout(2, 3)
+    nib = np.frombuffer(blob[L["nib"]:L["bits"]].tobytes(), np.uint32).reshape(1, 2, 4)
+    bits = np.frombuffer(blob[L["bits"]:L["col_a"]].tobytes(), np.uint32).reshape(1, 2, 2)
+    assert nib[0, 0].tolist() == g["nib0"] and nib[0, 1].tolist() == g["nib1"]
+    assert bits[0, 0].tolist() == g["bits0"] and bits[0, 1].tolist() == g["bits1"]
+    colA = np.frombuffer(blob[L["col_a"]:L["nnz"]].tobytes(), np.uint64)
+    nnz = np.frombuffer(blob[L["nnz"]:L["nnz"] + 8].tobytes(), np.uint32)
+    assert colA.tolist() == g["colA"] and nnz.tolist() == g["nnz"]
+    hdr = blob[:48]
+    assert int(np.frombuffer(hdr[0:4].tobytes(), np.uint32)[0]) == 0x31575344
+    assert np.frombuffer(hdr[8:32].tobytes(), np.int64).tolist() == [2, 3, 1]
+    assert int(np.frombuffer(hdr[36:40].tobytes(), np.uint32)[0]) == 3
+    assert int(np.frombuffer(hdr[40:48].tobytes(), np.uint64)[0]) == 32769
+
+
+def test_pack_round_trip_and_sizes():
+    for n_out, k_red in [(1, 1), (3, 31), (5, 32), (4, 33), (2, 100)]:
+        s = si.sign_codes(n_out * 1000 + k_red, (n_out, k_red))
+        p = si.shift_codes_uniform(n_out * 1000 + k_red, (n_out, k_red))
+        blob = O.pack_planes6(s, p)
+        L = O.blob_layout(n_out, k_red)
+        assert blob.size == L["total"] and L["total"] % 256 == 0
+        assert L["bits"] - L["nib"] == ((k_red + 31) // 32) * n_out * 16
+        s2, p2 = O.unpack_planes6(blob, n_out, k_red)
+        assert np.array_equal(s2, s)
+        # a zero code's shift is still stored
+        assert np.array_equal(p2, p)
