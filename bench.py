@@ -1,0 +1,308 @@
+"""Benchmark of the DeepShift shift-operator hot path on GB300.
+
+Default workload: the ResNet18 conv2_x-shaped ConvShift layer (N=32, C=K=64,
+56x56, 3x3, stride 1, pad 1) on int32 Q16.16 activations with 6-bit packed
+codes.  One step = the whole hot path of one layer forward: max|x| pre-pass
+(accumulator-width proof) + ConvShift with its fused bias/saturate epilogue.
+
+Prints one JSON line (rank 0).  `--impl reference` times the CPU oracle on a
+bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth_inputs as si  # noqa: E402
+
+METRIC = "Gshift-ops/s"
+L2_BYTES = 129 * 1024 * 1024
+SMS = 152
+INT_OPS_PER_CLK_PER_SM = 128  # 4 SMSPs x 32 lanes: 16-lane ALU pipe + 16-lane FMA pipe (IMAD)
+ALG_INT_OPS_PER_TERM = 2      # one shift + one add/subtract per term (Fig. 1a: MAC -> shift + add)
+
+
+def workload_conv2x(batch: int):
+    """ResNet18 conv2_x-shaped ConvShift layer: batch x 64 x 56 x 56, 3x3/1/1, 64 channels."""
+    N, C, H, W, K, R, S = batch, 64, 56, 56, 64, 3, 3
+    return dict(name="resnet18_conv2x_convshift_3x3", N=N, C=C, H=H, W=W, K=K, R=R, S=S, stride=1, pad=1,
+                terms=N * K * H * W * C * R * S)
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            return json.load(f), "measured"
+    return {"hbm_gbs": 6800.0, "sm_max_mhz": 2070.0, "bf16_tflops": 1900.0}, "fallback"
+
+
+class ClockSampler:
+    """Samples nvidia-smi SM clocks and throttle reasons while the timed region runs."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        mhz, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                mhz.append(float(parts[1]))
+                mx = float(parts[2])
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        return {"sm_mhz": float(np.median(mhz)) if mhz else None, "sm_max_mhz": mx,
+                "reasons": sorted(reasons), "samples": len(mhz)}
+
+
+def oracle_conv_sample(wl, n_images: int, seed: int):
+    """Times the CPU oracle on n_images of the workload; returns (seconds, terms)."""
+    from oracle import deepshift_oracle as O
+    x, s, p, b = si.conv_layer(seed, n_images, wl["C"], wl["H"], wl["W"], wl["K"], wl["R"], wl["S"])
+    t0 = time.perf_counter()
+    O.conv2d_shift(x, s, p, b, (wl["stride"], wl["stride"]), (wl["pad"], wl["pad"]))
+    dt = time.perf_counter() - t0
+    terms = wl["terms"] // wl["N"] * n_images
+    return dt, terms
+
+
+def cpu_baseline(wl, n_images: int = 16):
+    dt, terms = oracle_conv_sample(wl, n_images, si.SEED_BASE + 2)
+    return {"value": terms / dt / 1e9, "unit": METRIC, "cores": 1, "kind": "oracle",
+            "sample": f"{n_images} of {wl['N']} images of the same layer (numpy int64 oracle, 1 thread), "
+                      f"{dt:.1f} s"}
+
+
+def run_reference(args, wl, rank, world):
+    if rank != 0:
+        return
+    n_images = 1
+    times = []
+    for i in range(args.warmup + args.steps):
+        dt, terms = oracle_conv_sample(wl, n_images, si.SEED_BASE + 2)
+        if i >= args.warmup:
+            times.append(dt)
+    t = float(np.sum(times))
+    value = terms * len(times) / t / 1e9
+    out = {"impl": "reference", "metric": METRIC, "value": value, "unit": METRIC, "n_gpus": args.gpus,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": t / len(times) * 1e3,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
+           "data": "synthetic",
+           "config": {"workload": wl["name"], "batch": wl["N"], "C": wl["C"], "H": wl["H"], "W": wl["W"],
+                      "K": wl["K"], "kernel": "3x3", "stride": 1, "pad": 1,
+                      "reference_sample": f"{n_images} image per step"},
+           "cpu_baseline": {"value": value, "unit": METRIC, "cores": 1, "kind": "oracle",
+                            "sample": f"{n_images} of {wl['N']} images per step"},
+           "e2e": {"value": value, "unit": METRIC, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def run_gpu(args, wl, rank, world, local_rank):
+    import torch
+    import paper_1905_13298_gb300 as ds
+    from paper_1905_13298_gb300 import build as dsb
+
+    dsb.build_library()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+
+    N, C, H, W, K, R, S = (wl[k] for k in ("N", "C", "H", "W", "K", "R", "S"))
+    seed = si.SEED_BASE + 2 + 1000 * rank
+    x, s, p, b = si.conv_layer(seed, N, C, H, W, K, R, S)
+    w = ds.pack_shift_weights(torch.from_numpy(s).to(dev), torch.from_numpy(p).to(dev))
+    bd = torch.from_numpy(b).to(dev)
+    per_step_bytes = x.nbytes * 2
+    n_rot = max(2, int(np.ceil(2 * L2_BYTES / per_step_bytes)))
+    xs = [torch.from_numpy(x).to(dev) for _ in range(n_rot)]
+    ys = [torch.empty((N, K, H, W), dtype=torch.int32, device=dev) for _ in range(n_rot)]
+    amax_io = torch.zeros(2 * n_rot, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream()
+    st = stream.cuda_stream
+
+    def step(i, ev=None):
+        j = i % n_rot
+        a = amax_io[2 * j:2 * j + 2]
+        ds.ds_absmax(xs[j], xs[j].numel(), a, st)
+        if ev is not None:
+            ev[0].record(stream)
+        ds.ds_conv2d_shift(xs[j], w.desc, bd, None, ys[j], N, C, H, W, K, R, S, 1, 1, 1, 1, ds.DS_AMAX_IN, a, st)
+        if ev is not None:
+            ev[1].record(stream)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(local_rank) if rank == 0 else None
+    if sampler:
+        sampler.start()
+        time.sleep(0.3)
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_start.record(stream)
+    for i in range(args.steps):
+        step(i, evs[i])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    clocks = sampler.stop() if sampler else None
+    ms_total = t_start.elapsed_time(t_end)
+    kern_ms = float(np.mean([a.elapsed_time(b) for a, b in evs]))
+    if dist:
+        tt = torch.tensor([ms_total, kern_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms_total, kern_ms = float(tt[0]), float(tt[1])
+
+    # end to end through the public API with host buffers
+    xh = torch.from_numpy(x).pin_memory()
+    yh = torch.empty((N, K, H, W), dtype=torch.int32).pin_memory()
+    xd, yd = xs[0], ys[0]
+    a = amax_io[0:2]
+
+    def e2e_step():
+        xd.copy_(xh, non_blocking=True)
+        ds.ds_conv2d_shift(xd, w.desc, bd, None, yd, N, C, H, W, K, R, S, 1, 1, 1, 1, 0, a, st)
+        yh.copy_(yd, non_blocking=True)
+
+    for _ in range(max(1, args.warmup)):
+        e2e_step()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    if dist:
+        dist.barrier()
+    e0.record(stream)
+    for _ in range(args.steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1)
+    if dist:
+        tt = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_ms = float(tt[0])
+
+    # parity spot check of the timed output (whole-tensor parity lives in tests/)
+    if rank == 0:
+        from oracle import deepshift_oracle as O
+        got = ys[(args.steps - 1) % n_rot][0:1].cpu().numpy()
+        want = O.conv2d_shift(x[0:1], s, p, b, (1, 1), (1, 1))
+        parity = bool(np.array_equal(got, want))
+    else:
+        parity = None
+
+    if rank == 0:
+        peaks, peak_kind = measured_peaks()
+        terms_total = wl["terms"] * args.steps * world
+        value = terms_total / (ms_total / 1e3) / 1e9
+        sm_max = float(peaks.get("sm_max_mhz", 2070.0))
+        alu_peak = SMS * INT_OPS_PER_CLK_PER_SM * sm_max * 1e6 / 1e12  # T int-ops/s
+        achieved = ALG_INT_OPS_PER_TERM * wl["terms"] / (kern_ms / 1e3) / 1e12
+        alg_bytes = 4 * (N * C * H * W + N * K * H * W) + ds.ds_packed_weight_bytes(K, C * R * S) + 4 * K
+        out = {
+            "metric": METRIC, "value": value, "unit": METRIC, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_total / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "int32", "data": "synthetic",
+            "config": {"workload": wl["name"], "batch": N, "C": C, "H": H, "W": W, "K": K, "kernel": "3x3",
+                       "stride": 1, "pad": 1, "codes": "p geometric around -6, P(s=0)=0.1",
+                       "activations": "uniform [0, 2^20) int32 Q16.16",
+                       "l2": f"rotating {n_rot} input/output sets ({n_rot * per_step_bytes / 2**20:.0f} MiB > L2)",
+                       "step": "absmax pre-pass + ConvShift (fused bias/saturate epilogue)"},
+            "roofline": {"bound": "alu", "achieved": achieved, "peak": alu_peak, "unit": "Tintop/s",
+                         "frac": achieved / alu_peak, "traffic": None,
+                         "kernel": "shift_gemm_kernel<conv>", "kernel_ms": kern_ms,
+                         "peak_basis": f"{SMS} SMs x {INT_OPS_PER_CLK_PER_SM} int32 ops/clk x {sm_max:.0f} MHz "
+                                       f"(sm_max_mhz, {peak_kind})",
+                         "alg_int_ops_per_launch": ALG_INT_OPS_PER_TERM * wl["terms"],
+                         "hbm_gbs": alg_bytes / (kern_ms / 1e3) / 1e9,
+                         "hbm_frac": alg_bytes / (kern_ms / 1e3) / 1e9 / float(peaks.get("hbm_gbs", 6800.0))},
+            "e2e": {"value": wl["terms"] * args.steps * world / (e2e_ms / 1e3) / 1e9, "unit": METRIC,
+                    "h2d_bytes_per_step": int(x.nbytes), "d2h_bytes_per_step": int(x.nbytes // C * K)},
+            "gpu_launches": 2 * args.steps,
+            "clocks": clocks,
+            "parity_spot_check": parity,
+        }
+        if not args.no_cpu_baseline:
+            out["cpu_baseline"] = cpu_baseline(wl)
+        print(json.dumps(out), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--batch", type=int, default=32)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    wl = workload_conv2x(args.batch)
+    if args.impl == "reference":
+        run_reference(args, wl, rank, world)
+    else:
+        run_gpu(args, wl, rank, world, local_rank)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,206 @@
+"""DeepShift shift operators on GB300: thin Python binding of libdeepshift.so.
+
+The functions named ``ds_*`` mirror the C ABI of ``include/deepshift.h`` one
+to one (argument marshalling only: every step runs in the library's CUDA
+kernels).  PyTorch supplies device memory and the current CUDA stream.  There
+is no CPU fallback: importing works without a GPU, but every compute call
+needs the built library and a CUDA device, and fails loudly otherwise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libdeepshift.so")
+
+# status codes (deepshift.h)
+DS_OK = 0
+DS_ERR_INVALID_ARG = 1
+DS_ERR_SHAPE = 2
+DS_ERR_CODE_RANGE = 3
+DS_ERR_ALIGNMENT = 4
+DS_ERR_BUFFER_TOO_SMALL = 5
+DS_ERR_UNSUPPORTED = 6
+DS_ERR_CUDA = 7
+STATUS_NAMES = {0: "DS_OK", 1: "DS_ERR_INVALID_ARG", 2: "DS_ERR_SHAPE", 3: "DS_ERR_CODE_RANGE",
+                4: "DS_ERR_ALIGNMENT", 5: "DS_ERR_BUFFER_TOO_SMALL", 6: "DS_ERR_UNSUPPORTED",
+                7: "DS_ERR_CUDA"}
+
+# flags
+DS_RELU = 1
+DS_AMAX_IN = 2
+DS_AMAX_OUT = 4
+DS_RESIDUAL = 8
+DS_FORCE_INT64 = 16
+
+DS_WEIGHTS_MAGIC = 0x31575344
+DS_FORMAT_PLANES6 = 1
+
+
+class DsError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"{STATUS_NAMES.get(status, status)}: {msg}")
+        self.status = status
+
+
+class ds_weights(ctypes.Structure):
+    _fields_ = [("magic", ctypes.c_uint32), ("format", ctypes.c_uint32),
+                ("n_out", ctypes.c_int64), ("k_red", ctypes.c_int64), ("n_chunks", ctypes.c_int64),
+                ("packed", ctypes.c_void_p), ("packed_bytes", ctypes.c_size_t),
+                ("a_max", ctypes.c_uint64), ("nnz_max", ctypes.c_uint32), ("reserved", ctypes.c_uint32)]
+
+
+_lib = None
+
+_SIGNATURES = {
+    "ds_last_error": (ctypes.c_char_p, []),
+    "ds_version": (ctypes.c_int, []),
+    "ds_packed_weight_bytes": (ctypes.c_size_t, [ctypes.c_int64, ctypes.c_int64]),
+    "ds_pack_shift_weights": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64,
+                                             ctypes.c_void_p, ctypes.c_size_t, ctypes.POINTER(ds_weights),
+                                             ctypes.c_void_p]),
+    "ds_linear_shift": (ctypes.c_int, [ctypes.c_void_p, ctypes.POINTER(ds_weights), ctypes.c_void_p,
+                                       ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
+                                       ctypes.c_uint32, ctypes.c_void_p, ctypes.c_void_p]),
+    "ds_conv2d_shift": (ctypes.c_int, [ctypes.c_void_p, ctypes.POINTER(ds_weights), ctypes.c_void_p,
+                                       ctypes.c_void_p, ctypes.c_void_p] + [ctypes.c_int] * 11 +
+                        [ctypes.c_uint32, ctypes.c_void_p, ctypes.c_void_p]),
+    "ds_absmax": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]),
+}
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded library; raises if it has not been built (there is no fallback)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise ImportError(f"{LIB_PATH} is missing: build it with paper_1905_13298_gb300.build.build_library()")
+        L = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in _SIGNATURES.items():
+            fn = getattr(L, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = L
+    return _lib
+
+
+def ds_last_error() -> str:
+    return lib().ds_last_error().decode()
+
+
+def _check(status: int) -> None:
+    if status != DS_OK:
+        raise DsError(status, ds_last_error())
+
+
+def _ptr(t) -> int | None:
+    """Device (or host) address of a tensor, None for None; ints pass through."""
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def _stream(stream) -> int | None:
+    if stream is not None:
+        return stream if isinstance(stream, int) else stream.cuda_stream
+    import torch
+    return torch.cuda.current_stream().cuda_stream
+
+
+# ---------------------------------------------------------------------------
+# One-to-one wrappers of the C ABI
+# ---------------------------------------------------------------------------
+
+def ds_packed_weight_bytes(n_out: int, k_red: int) -> int:
+    return int(lib().ds_packed_weight_bytes(n_out, k_red))
+
+
+def ds_pack_shift_weights(s, p, n_out: int, k_red: int, packed, packed_bytes: int, stream=None) -> ds_weights:
+    desc = ds_weights()
+    _check(lib().ds_pack_shift_weights(_ptr(s), _ptr(p), n_out, k_red, _ptr(packed), packed_bytes,
+                                       ctypes.byref(desc), _stream(stream)))
+    return desc
+
+
+def ds_linear_shift(x, w: ds_weights, bias, y, M: int, K: int, N: int, flags: int = 0, amax_io=None,
+                    stream=None) -> None:
+    _check(lib().ds_linear_shift(_ptr(x), ctypes.byref(w), _ptr(bias), _ptr(y), M, K, N, flags,
+                                 _ptr(amax_io), _stream(stream)))
+
+
+def ds_conv2d_shift(x, w: ds_weights, bias, residual, y, N, C, H, W, K, R, S, stride_h, stride_w,
+                    pad_h, pad_w, flags: int = 0, amax_io=None, stream=None) -> None:
+    _check(lib().ds_conv2d_shift(_ptr(x), ctypes.byref(w), _ptr(bias), _ptr(residual), _ptr(y), N, C, H,
+                                 W, K, R, S, stride_h, stride_w, pad_h, pad_w, flags, _ptr(amax_io),
+                                 _stream(stream)))
+
+
+def ds_absmax(x, n: int, amax, stream=None) -> None:
+    _check(lib().ds_absmax(_ptr(x), n, _ptr(amax), _stream(stream)))
+
+
+# ---------------------------------------------------------------------------
+# Tensor-level helpers (allocate outputs with torch, then call the ABI)
+# ---------------------------------------------------------------------------
+
+class PackedShiftWeights:
+    """A packed blob (device uint8 tensor) plus its ds_weights descriptor."""
+
+    def __init__(self, blob, desc: ds_weights):
+        self.blob = blob
+        self.desc = desc
+
+    @property
+    def n_out(self) -> int:
+        return int(self.desc.n_out)
+
+    @property
+    def k_red(self) -> int:
+        return int(self.desc.k_red)
+
+
+def pack_shift_weights(s, p, stream=None) -> PackedShiftWeights:
+    """Packs int8 sign/shift code tensors [n_out, ...] (device) into a new blob."""
+    import torch
+    if s.device.type != "cuda" or p.device.type != "cuda":
+        raise ValueError("codes must be CUDA tensors")
+    n_out = s.shape[0]
+    k_red = s[0].numel() if n_out else 0
+    s2 = s.reshape(n_out, k_red).to(torch.int8).contiguous()
+    p2 = p.reshape(n_out, k_red).to(torch.int8).contiguous()
+    nbytes = ds_packed_weight_bytes(n_out, k_red)
+    if nbytes == 0:
+        raise DsError(DS_ERR_SHAPE, "invalid code matrix shape")
+    blob = torch.empty(nbytes, dtype=torch.uint8, device=s.device)
+    desc = ds_pack_shift_weights(s2, p2, n_out, k_red, blob, nbytes, stream)
+    return PackedShiftWeights(blob, desc)
+
+
+def linear_shift(x, w: PackedShiftWeights, bias=None, relu: bool = False, amax_io=None, flags: int = 0,
+                 out=None, stream=None):
+    """y = sat32(bias + sum s * (x >> -p)) [ReLU] for int32 x [M, K] on the GPU."""
+    import torch
+    M, K = x.shape
+    N = w.n_out
+    y = out if out is not None else torch.empty((M, N), dtype=torch.int32, device=x.device)
+    ds_linear_shift(x, w.desc, bias, y, M, K, N, flags | (DS_RELU if relu else 0), amax_io, stream)
+    return y
+
+
+def conv2d_shift(x, w: PackedShiftWeights, kernel_size, bias=None, stride=(1, 1), padding=(0, 0),
+                 relu: bool = False, residual=None, amax_io=None, flags: int = 0, out=None, stream=None):
+    """ConvShift forward on int32 NCHW x; w packed from OIHW codes."""
+    import torch
+    N, C, H, W = x.shape
+    R, S = kernel_size
+    K = w.n_out
+    OH = (H + 2 * padding[0] - R) // stride[0] + 1
+    OW = (W + 2 * padding[1] - S) // stride[1] + 1
+    y = out if out is not None else torch.empty((N, K, OH, OW), dtype=torch.int32, device=x.device)
+    f = flags | (DS_RELU if relu else 0) | (DS_RESIDUAL if residual is not None else 0)
+    ds_conv2d_shift(x, w.desc, bias, residual, y, N, C, H, W, K, R, S, stride[0], stride[1], padding[0],
+                    padding[1], f, amax_io, stream)
+    return y

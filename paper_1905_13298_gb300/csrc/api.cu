@@ -1,0 +1,239 @@
+// C ABI entry points: argument validation, then stream-ordered launches.
+// Nothing is launched and no output is written when validation fails.
+#include <stdarg.h>
+#include <stdio.h>
+
+#include <string>
+
+#include "ds_common.cuh"
+
+namespace ds {
+
+static thread_local std::string g_last_error;
+
+void set_error(const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+}
+
+void clear_error() { g_last_error.clear(); }
+
+ds_status fail(ds_status st, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return st;
+}
+
+ds_status cuda_check(cudaError_t e, const char* what) {
+  if (e == cudaSuccess) return DS_OK;
+  return fail(DS_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+// Checks a descriptor filled by ds_pack_shift_weights against the call's dims.
+static ds_status check_weights(const ds_weights* w, int64_t n_out, int64_t k_red) {
+  if (w == nullptr) return fail(DS_ERR_INVALID_ARG, "weights descriptor is NULL");
+  if (w->magic != DS_WEIGHTS_MAGIC || w->format != DS_FORMAT_PLANES6)
+    return fail(DS_ERR_INVALID_ARG, "weights descriptor was not filled by ds_pack_shift_weights");
+  if (w->packed == nullptr) return fail(DS_ERR_INVALID_ARG, "weights descriptor has no blob");
+  if (w->n_out != n_out || w->k_red != k_red)
+    return fail(DS_ERR_SHAPE, "weights are %lld x %lld, call needs %lld x %lld", (long long)w->n_out,
+                (long long)w->k_red, (long long)n_out, (long long)k_red);
+  const BlobLayout L = blob_layout(n_out, k_red);
+  if (w->n_chunks != L.n_chunks || w->packed_bytes < (size_t)L.total)
+    return fail(DS_ERR_INVALID_ARG, "weights descriptor is inconsistent with its dims");
+  if ((reinterpret_cast<uintptr_t>(w->packed) & 255) != 0)
+    return fail(DS_ERR_ALIGNMENT, "packed blob must be 256-byte aligned");
+  return DS_OK;
+}
+
+static void fill_blob_offsets(GemmParams& p, const ds_weights* w) {
+  const BlobLayout L = blob_layout(w->n_out, w->k_red);
+  p.blob = static_cast<const uint8_t*>(w->packed);
+  p.n_chunks = L.n_chunks;
+  p.off_nib = L.nib;
+  p.off_bits = L.bits;
+  p.off_cola = L.col_a;
+  p.off_nnz = L.nnz;
+}
+
+// Resolves the amax slots: computes max|x| into amax_io[0] unless the caller
+// provided it, and zeroes amax_io[1] when the call reports the output amax.
+static ds_status prepare_amax(const int32_t* x, int64_t nx, uint32_t flags, uint32_t* amax_io,
+                              cudaStream_t st, GemmParams& p) {
+  p.amax_in = nullptr;
+  p.amax_out = nullptr;
+  if (amax_io == nullptr) return DS_OK;
+  if (!(flags & DS_AMAX_IN)) {
+    ds_status s = cuda_check(launch_absmax(x, nx, amax_io, st), "absmax pre-pass");
+    if (s != DS_OK) return s;
+  }
+  p.amax_in = amax_io;
+  if (flags & DS_AMAX_OUT) {
+    ds_status s = cuda_check(cudaMemsetAsync(amax_io + 1, 0, sizeof(uint32_t), st), "amax_out reset");
+    if (s != DS_OK) return s;
+    p.amax_out = amax_io + 1;
+  }
+  return DS_OK;
+}
+
+constexpr uint32_t kKnownFlags = DS_RELU | DS_AMAX_IN | DS_AMAX_OUT | DS_RESIDUAL | DS_FORCE_INT64;
+
+}  // namespace ds
+
+using namespace ds;
+
+extern "C" {
+
+const char* ds_last_error(void) { return g_last_error.c_str(); }
+
+int ds_version(void) { return 100; }
+
+size_t ds_packed_weight_bytes(int64_t n_out, int64_t k_red) {
+  if (n_out <= 0 || k_red <= 0) return 0;
+  if (n_out > (int64_t(1) << 31) || k_red > (int64_t(1) << 40)) return 0;
+  return (size_t)blob_layout(n_out, k_red).total;
+}
+
+ds_status ds_pack_shift_weights(const int8_t* s, const int8_t* p, int64_t n_out, int64_t k_red,
+                                void* packed, size_t packed_bytes, ds_weights* desc, void* stream) {
+  clear_error();
+  if (!s || !p || !packed || !desc) return fail(DS_ERR_INVALID_ARG, "NULL pointer argument");
+  if (n_out <= 0 || k_red <= 0) return fail(DS_ERR_SHAPE, "n_out and k_red must be positive");
+  const size_t need = ds_packed_weight_bytes(n_out, k_red);
+  if (need == 0) return fail(DS_ERR_UNSUPPORTED, "code matrix too large");
+  if (packed_bytes < need)
+    return fail(DS_ERR_BUFFER_TOO_SMALL, "packed buffer has %zu bytes, needs %zu", packed_bytes, need);
+  if ((reinterpret_cast<uintptr_t>(packed) & 255) != 0)
+    return fail(DS_ERR_ALIGNMENT, "packed buffer must be 256-byte aligned");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  uint8_t* blob = static_cast<uint8_t*>(packed);
+  ds_status r = cuda_check(launch_pack(s, p, n_out, k_red, blob, st), "pack launch");
+  if (r != DS_OK) return r;
+  BlobHeader h;
+  r = cuda_check(cudaMemcpyAsync(&h, blob, sizeof(h), cudaMemcpyDeviceToHost, st), "header read");
+  if (r != DS_OK) return r;
+  r = cuda_check(cudaStreamSynchronize(st), "pack synchronise");
+  if (r != DS_OK) return r;
+  if (h.invalid_count != 0)
+    return fail(DS_ERR_CODE_RANGE, "%u codes outside s in {-1,0,1} or p in [-15,0]", h.invalid_count);
+  desc->magic = DS_WEIGHTS_MAGIC;
+  desc->format = DS_FORMAT_PLANES6;
+  desc->n_out = n_out;
+  desc->k_red = k_red;
+  desc->n_chunks = h.n_chunks;
+  desc->packed = packed;
+  desc->packed_bytes = need;
+  desc->a_max = h.a_max;
+  desc->nnz_max = h.nnz_max;
+  desc->reserved = 0;
+  return DS_OK;
+}
+
+ds_status ds_absmax(const int32_t* x, int64_t n, uint32_t* amax, void* stream) {
+  clear_error();
+  if (!x || !amax) return fail(DS_ERR_INVALID_ARG, "NULL pointer argument");
+  if (n <= 0) return fail(DS_ERR_SHAPE, "n must be positive");
+  return cuda_check(launch_absmax(x, n, amax, static_cast<cudaStream_t>(stream)), "absmax launch");
+}
+
+ds_status ds_linear_shift(const int32_t* x, const ds_weights* w, const int32_t* bias, int32_t* y,
+                          int64_t M, int64_t K, int64_t N, uint32_t flags, uint32_t* amax_io,
+                          void* stream) {
+  clear_error();
+  if (!x || !y) return fail(DS_ERR_INVALID_ARG, "NULL x or y");
+  if (M <= 0 || K <= 0 || N <= 0) return fail(DS_ERR_SHAPE, "M, K and N must be positive");
+  if (M > (int64_t(1) << 40) || N > 65535LL * 64) return fail(DS_ERR_UNSUPPORTED, "M or N too large");
+  if (flags & ~kKnownFlags) return fail(DS_ERR_INVALID_ARG, "unknown flag bits 0x%x", flags & ~kKnownFlags);
+  if (flags & DS_RESIDUAL) return fail(DS_ERR_INVALID_ARG, "DS_RESIDUAL applies to ds_conv2d_shift only");
+  if ((flags & (DS_AMAX_IN | DS_AMAX_OUT)) && amax_io == nullptr)
+    return fail(DS_ERR_INVALID_ARG, "DS_AMAX_IN / DS_AMAX_OUT need amax_io");
+  if (!aligned16(x) || !aligned16(y)) return fail(DS_ERR_ALIGNMENT, "x and y must be 16-byte aligned");
+  ds_status r = check_weights(w, N, K);
+  if (r != DS_OK) return r;
+  const int64_t xb = M * K * 4, yb = M * N * 4;
+  const char* xa = reinterpret_cast<const char*>(x);
+  const char* ya = reinterpret_cast<const char*>(y);
+  if (xa < ya + yb && ya < xa + xb) return fail(DS_ERR_INVALID_ARG, "y must not overlap x");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  GemmParams p{};
+  p.x = x;
+  p.bias = bias;
+  p.residual = nullptr;
+  p.y = y;
+  p.rows = M;
+  p.kred = K;
+  p.cols = N;
+  p.flags = flags;
+  fill_blob_offsets(p, w);
+  r = prepare_amax(x, M * K, flags, amax_io, st, p);
+  if (r != DS_OK) return r;
+  return cuda_check(launch_linear_shift(p, st), "linear_shift launch");
+}
+
+ds_status ds_conv2d_shift(const int32_t* x, const ds_weights* w, const int32_t* bias,
+                          const int32_t* residual, int32_t* y, int N, int C, int H, int W, int K,
+                          int R, int S, int stride_h, int stride_w, int pad_h, int pad_w,
+                          uint32_t flags, uint32_t* amax_io, void* stream) {
+  clear_error();
+  if (!x || !y) return fail(DS_ERR_INVALID_ARG, "NULL x or y");
+  if (N <= 0 || C <= 0 || H <= 0 || W <= 0 || K <= 0 || R <= 0 || S <= 0)
+    return fail(DS_ERR_SHAPE, "N, C, H, W, K, R, S must be positive");
+  if (stride_h <= 0 || stride_w <= 0 || pad_h < 0 || pad_w < 0)
+    return fail(DS_ERR_SHAPE, "strides must be positive and pads non-negative");
+  if (H + 2 * pad_h < R || W + 2 * pad_w < S) return fail(DS_ERR_SHAPE, "kernel larger than padded input");
+  if (flags & ~kKnownFlags) return fail(DS_ERR_INVALID_ARG, "unknown flag bits 0x%x", flags & ~kKnownFlags);
+  if ((flags & DS_RESIDUAL) && residual == nullptr)
+    return fail(DS_ERR_INVALID_ARG, "DS_RESIDUAL needs a residual tensor");
+  if ((flags & (DS_AMAX_IN | DS_AMAX_OUT)) && amax_io == nullptr)
+    return fail(DS_ERR_INVALID_ARG, "DS_AMAX_IN / DS_AMAX_OUT need amax_io");
+  if (!aligned16(x) || !aligned16(y)) return fail(DS_ERR_ALIGNMENT, "x and y must be 16-byte aligned");
+  const int OH = (H + 2 * pad_h - R) / stride_h + 1;
+  const int OW = (W + 2 * pad_w - S) / stride_w + 1;
+  const int64_t kred = (int64_t)C * R * S;
+  ds_status r = check_weights(w, K, kred);
+  if (r != DS_OK) return r;
+  const int64_t nx = (int64_t)N * C * H * W;
+  const int64_t ny = (int64_t)N * K * OH * OW;
+  const char* xa = reinterpret_cast<const char*>(x);
+  const char* ya = reinterpret_cast<const char*>(y);
+  if (xa < ya + ny * 4 && ya < xa + nx * 4) return fail(DS_ERR_INVALID_ARG, "y must not overlap x");
+  if ((int64_t)OH * OW > (int64_t)1 << 30 || (int64_t)C * H * W > (int64_t)1 << 31)
+    return fail(DS_ERR_UNSUPPORTED, "image too large");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  GemmParams p{};
+  p.x = x;
+  p.bias = bias;
+  p.residual = (flags & DS_RESIDUAL) ? residual : nullptr;
+  p.y = y;
+  p.rows = (int64_t)N * OH * OW;
+  p.kred = kred;
+  p.cols = K;
+  p.flags = flags;
+  p.C = C;
+  p.H = H;
+  p.W = W;
+  p.R = R;
+  p.S = S;
+  p.sh = stride_h;
+  p.sw = stride_w;
+  p.ph = pad_h;
+  p.pw = pad_w;
+  p.OH = OH;
+  p.OW = OW;
+  fill_blob_offsets(p, w);
+  r = prepare_amax(x, nx, flags, amax_io, st, p);
+  if (r != DS_OK) return r;
+  return cuda_check(launch_conv2d_shift(p, st), "conv2d_shift launch");
+}
+
+}  // extern "C"

@@ -1,0 +1,85 @@
+// Shared definitions of the DeepShift CUDA library (sm_103a).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "deepshift.h"
+
+namespace ds {
+
+// ---------------------------------------------------------------------------
+// Error reporting (thread-local last error, see ds_last_error()).
+// ---------------------------------------------------------------------------
+void set_error(const char* fmt, ...);
+void clear_error();
+ds_status fail(ds_status st, const char* fmt, ...);
+ds_status cuda_check(cudaError_t e, const char* what);
+
+// ---------------------------------------------------------------------------
+// Packed blob geometry (format DS_FORMAT_PLANES6, documented in deepshift.h).
+// ---------------------------------------------------------------------------
+constexpr int64_t kBlobHeader = 256;
+constexpr int kChunk = 32;  // reduction indices per packed chunk
+
+struct BlobLayout {
+  int64_t n_chunks, nib, bits, col_a, nnz, total;
+};
+
+__host__ __device__ inline BlobLayout blob_layout(int64_t n_out, int64_t k_red) {
+  BlobLayout L;
+  L.n_chunks = (k_red + kChunk - 1) / kChunk;
+  L.nib = kBlobHeader;
+  L.bits = L.nib + L.n_chunks * n_out * 16;
+  L.col_a = L.bits + L.n_chunks * n_out * 8;
+  L.nnz = L.col_a + n_out * 8;
+  int64_t end = L.nnz + n_out * 4;
+  L.total = (end + 255) / 256 * 256;
+  return L;
+}
+
+// Header written on the device by the pack kernel.
+struct BlobHeader {
+  uint32_t magic;
+  uint32_t format;
+  int64_t n_out;
+  int64_t k_red;
+  int64_t n_chunks;
+  uint32_t invalid_count;
+  uint32_t nnz_max;
+  unsigned long long a_max;
+};
+static_assert(sizeof(BlobHeader) == 48, "header layout");
+
+// ---------------------------------------------------------------------------
+// Parameters of the shift-GEMM kernels (FC and conv implicit GEMM).
+// The GEMM view: rows = FC rows m or conv output pixels (n, oh, ow);
+// columns = output features / channels; reduction = K or (c, r, s).
+// ---------------------------------------------------------------------------
+struct GemmParams {
+  const int32_t* x;
+  const uint8_t* blob;
+  const int32_t* bias;      // nullable
+  const int32_t* residual;  // nullable (conv, DS_RESIDUAL)
+  int32_t* y;
+  const uint32_t* amax_in;  // nullable: then the 64-bit path is taken
+  uint32_t* amax_out;       // nullable
+  int64_t rows;             // FC: M; conv: N*OH*OW
+  int64_t kred;             // FC: K; conv: C*R*S
+  int64_t cols;             // FC: N; conv: K
+  int64_t n_chunks;
+  int64_t off_nib, off_bits, off_cola, off_nnz;
+  // conv geometry (unused by FC)
+  int C, H, W, R, S, sh, sw, ph, pw, OH, OW;
+  uint32_t flags;
+};
+
+// Launchers (defined in shift_gemm.cu).
+cudaError_t launch_linear_shift(const GemmParams& p, cudaStream_t st);
+cudaError_t launch_conv2d_shift(const GemmParams& p, cudaStream_t st);
+// Defined in misc_kernels.cu.
+cudaError_t launch_absmax(const int32_t* x, int64_t n, uint32_t* out, cudaStream_t st);
+cudaError_t launch_pack(const int8_t* s, const int8_t* p, int64_t n_out, int64_t k_red,
+                        uint8_t* blob, cudaStream_t st);
+
+}  // namespace ds

@@ -1,0 +1,113 @@
+// Weight packing and the max|x| pre-pass.
+//
+// Packing follows Eq. 3 of DeepShift (the weight matrix is replaced by the
+// shift matrix P and the sign matrix S) with the Sec. 4 range p in [-15, 0];
+// the blob layout is the library's own (deepshift.h, DS_FORMAT_PLANES6).
+#include "ds_common.cuh"
+
+namespace ds {
+
+// One thread per output column: walks the column's reduction range chunk by
+// chunk, validates the codes, writes the nibble and bit-plane records and the
+// column constants A[n] and nnz[n], and folds them into the header maxima.
+__global__ void pack_kernel(const int8_t* __restrict__ s, const int8_t* __restrict__ p,
+                            int64_t n_out, int64_t k_red, uint8_t* __restrict__ blob) {
+  const BlobLayout L = blob_layout(n_out, k_red);
+  BlobHeader* hdr = reinterpret_cast<BlobHeader*>(blob);
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    hdr->magic = DS_WEIGHTS_MAGIC;
+    hdr->format = DS_FORMAT_PLANES6;
+    hdr->n_out = n_out;
+    hdr->k_red = k_red;
+    hdr->n_chunks = L.n_chunks;
+  }
+  const int64_t n = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (n >= n_out) return;
+  const int8_t* srow = s + n * k_red;
+  const int8_t* prow = p + n * k_red;
+  uint4* nib = reinterpret_cast<uint4*>(blob + L.nib);
+  uint2* bits = reinterpret_cast<uint2*>(blob + L.bits);
+  unsigned long long a_sum = 0;
+  uint32_t nnz = 0, invalid = 0;
+  for (int64_t g = 0; g < L.n_chunks; ++g) {
+    uint32_t w[4] = {0u, 0u, 0u, 0u};
+    uint32_t neg = 0u, nz = 0u;
+    for (int j = 0; j < kChunk; ++j) {
+      const int64_t k = g * kChunk + j;
+      if (k >= k_red) break;
+      const int sv = srow[k];
+      const int pv = prow[k];
+      if (sv < -1 || sv > 1 || pv < -15 || pv > 0) {
+        ++invalid;
+        continue;
+      }
+      w[j >> 3] |= (uint32_t)(-pv) << (4 * (j & 7));
+      if (sv == -1) neg |= 1u << j;
+      if (sv != 0) {
+        nz |= 1u << j;
+        ++nnz;
+        a_sum += 1ull << (15 + pv);
+      }
+    }
+    nib[g * n_out + n] = make_uint4(w[0], w[1], w[2], w[3]);
+    bits[g * n_out + n] = make_uint2(neg, nz);
+  }
+  reinterpret_cast<unsigned long long*>(blob + L.col_a)[n] = a_sum;
+  reinterpret_cast<uint32_t*>(blob + L.nnz)[n] = nnz;
+  if (invalid) atomicAdd(&hdr->invalid_count, invalid);
+  atomicMax(&hdr->nnz_max, nnz);
+  atomicMax(&hdr->a_max, a_sum);
+}
+
+cudaError_t launch_pack(const int8_t* s, const int8_t* p, int64_t n_out, int64_t k_red,
+                        uint8_t* blob, cudaStream_t st) {
+  // zero the whole blob: header counters, and the tail padding stays defined
+  cudaError_t e = cudaMemsetAsync(blob, 0, (size_t)blob_layout(n_out, k_red).total, st);
+  if (e != cudaSuccess) return e;
+  const int threads = 128;
+  const int64_t blocks = (n_out + threads - 1) / threads;
+  pack_kernel<<<(unsigned)blocks, threads, 0, st>>>(s, p, n_out, k_red, blob);
+  return cudaGetLastError();
+}
+
+// max |x| (as u32, |INT32_MIN| = 2^31).  Grid-stride over 16-byte vectors,
+// warp reduction, one atomicMax per warp.  The target is zeroed first.
+__device__ __forceinline__ uint32_t uabs32(int32_t v) {
+  return v < 0 ? (uint32_t)0 - (uint32_t)v : (uint32_t)v;
+}
+
+__global__ void absmax_kernel(const int32_t* __restrict__ x, int64_t n, uint32_t* out) {
+  uint32_t m = 0;
+  const int64_t tid = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const bool vec = ((reinterpret_cast<uintptr_t>(x) & 15) == 0);
+  if (vec) {
+    const int64_t nv = n >> 2;
+    const int4* xv = reinterpret_cast<const int4*>(x);
+    for (int64_t i = tid; i < nv; i += stride) {
+      int4 v = __ldg(xv + i);
+      m = max(m, max(max(uabs32(v.x), uabs32(v.y)), max(uabs32(v.z), uabs32(v.w))));
+    }
+    for (int64_t i = (nv << 2) + tid; i < n; i += stride) m = max(m, uabs32(x[i]));
+  } else {
+    for (int64_t i = tid; i < n; i += stride) m = max(m, uabs32(x[i]));
+  }
+  m = __reduce_max_sync(0xffffffffu, m);
+  if ((threadIdx.x & 31) == 0 && m) atomicMax(out, m);
+}
+
+cudaError_t launch_absmax(const int32_t* x, int64_t n, uint32_t* out, cudaStream_t st) {
+  cudaError_t e = cudaMemsetAsync(out, 0, sizeof(uint32_t), st);
+  if (e != cudaSuccess) return e;
+  int dev = 0, sms = 152;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int threads = 256;
+  int64_t want = (n / 4 + threads - 1) / threads;
+  int64_t blocks = want < (int64_t)sms * 8 ? want : (int64_t)sms * 8;
+  if (blocks < 1) blocks = 1;
+  absmax_kernel<<<(unsigned)blocks, threads, 0, st>>>(x, n, out);
+  return cudaGetLastError();
+}
+
+}  // namespace ds

@@ -8,3 +8,19 @@ if ROOT not in sys.path:
 
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (GB300, sm_103a) and the built library")
+
+
+import pytest
+
+
+@pytest.fixture(scope="session")
+def dslib():
+    """The built CUDA library and its binding (GPU tests only)."""
+    import torch
+    if not torch.cuda.is_available():
+        pytest.fail("GPU test collected without a CUDA device")
+    from paper_1905_13298_gb300 import build
+    build.build_library()
+    import paper_1905_13298_gb300 as ds
+    ds.lib()
+    return ds

@@ -1,0 +1,103 @@
+"""Host-side checks of the C ABI: the library loads without a GPU, exports
+every entry point its header declares, and rejects bad arguments before it
+touches CUDA."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+from oracle import deepshift_oracle as O
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def ds():
+    from paper_1905_13298_gb300 import build
+    build.build_library()
+    import paper_1905_13298_gb300 as ds
+    ds.lib()
+    return ds
+
+
+def _declared_functions():
+    names = set()
+    for hdr in os.listdir(os.path.join(ROOT, "include")):
+        if not hdr.endswith(".h"):
+            continue
+        text = open(os.path.join(ROOT, "include", hdr)).read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", "", text)
+        names |= set(re.findall(r"\b(ds_\w+)\s*\(", text))
+    return sorted(names)
+
+
+def test_every_declared_symbol_is_exported(ds):
+    names = _declared_functions()
+    assert "ds_linear_shift" in names and "ds_conv2d_shift" in names and "ds_pack_shift_weights" in names
+    L = ds.lib()
+    for n in names:
+        assert hasattr(L, n), n
+        assert n in ds._SIGNATURES or n.startswith("ds_"), n
+
+
+def test_binding_covers_every_declared_symbol(ds):
+    for n in _declared_functions():
+        assert n in ds._SIGNATURES, f"{n} has no ctypes signature in the binding"
+
+
+def test_packed_bytes_match_documented_layout(ds):
+    for n_out, k_red in [(1, 1), (64, 576), (512, 784), (4096, 4096), (1000, 512), (3, 33)]:
+        assert ds.ds_packed_weight_bytes(n_out, k_red) == O.blob_layout(n_out, k_red)["total"]
+    assert ds.ds_packed_weight_bytes(0, 5) == 0
+    assert ds.ds_packed_weight_bytes(5, -1) == 0
+
+
+def test_weights_struct_layout(ds):
+    assert ctypes.sizeof(ds.ds_weights) == 64
+    assert ds.ds_weights.packed.offset == 32
+
+
+def test_validation_happens_before_cuda(ds):
+    L = ds.lib()
+    w = ds.ds_weights()
+    # NULL pointers
+    assert L.ds_linear_shift(None, ctypes.byref(w), None, None, 1, 1, 1, 0, None, None) == ds.DS_ERR_INVALID_ARG
+    assert "NULL" in ds.ds_last_error()
+    # bad shapes
+    assert L.ds_linear_shift(16, ctypes.byref(w), None, 4096, 0, 1, 1, 0, None, None) == ds.DS_ERR_SHAPE
+    assert L.ds_conv2d_shift(16, ctypes.byref(w), None, None, 4096, 1, 1, 3, 3, 1, 3, 3, 0, 1, 1, 1, 0, None,
+                             None) == ds.DS_ERR_SHAPE
+    # misaligned pointers
+    assert L.ds_linear_shift(20, ctypes.byref(w), None, 4096, 1, 1, 1, 0, None, None) == ds.DS_ERR_ALIGNMENT
+    # unfilled descriptor
+    assert L.ds_linear_shift(16, ctypes.byref(w), None, 4096, 1, 1, 1, 0, None, None) == ds.DS_ERR_INVALID_ARG
+    assert "ds_pack_shift_weights" in ds.ds_last_error()
+    # unknown flags, residual on FC, amax flags without a buffer
+    assert L.ds_linear_shift(16, ctypes.byref(w), None, 4096, 1, 1, 1, 1 << 20, None, None) == ds.DS_ERR_INVALID_ARG
+    assert L.ds_linear_shift(16, ctypes.byref(w), None, 4096, 1, 1, 1, ds.DS_RESIDUAL, None, None) == ds.DS_ERR_INVALID_ARG
+    assert L.ds_linear_shift(16, ctypes.byref(w), None, 4096, 1, 1, 1, ds.DS_AMAX_IN, None, None) == ds.DS_ERR_INVALID_ARG
+    # pack: buffer too small, misaligned blob
+    d = ds.ds_weights()
+    assert L.ds_pack_shift_weights(16, 16, 4, 4, 256, 10, ctypes.byref(d), None) == ds.DS_ERR_BUFFER_TOO_SMALL
+    assert L.ds_pack_shift_weights(16, 16, 4, 4, 272, 4096, ctypes.byref(d), None) == ds.DS_ERR_ALIGNMENT
+    assert L.ds_pack_shift_weights(16, 16, 0, 4, 256, 4096, ctypes.byref(d), None) == ds.DS_ERR_SHAPE
+    assert d.magic == 0
+    # descriptor/dims mismatch
+    w2 = ds.ds_weights(magic=ds.DS_WEIGHTS_MAGIC, format=ds.DS_FORMAT_PLANES6, n_out=8, k_red=8, n_chunks=1,
+                       packed=256, packed_bytes=ds.ds_packed_weight_bytes(8, 8))
+    assert L.ds_linear_shift(16, ctypes.byref(w2), None, 4096, 2, 9, 8, 0, None, None) == ds.DS_ERR_SHAPE
+    # overlap of x and y
+    assert L.ds_linear_shift(4096, ctypes.byref(w2), None, 4096, 2, 8, 8, 0, None, None) == ds.DS_ERR_INVALID_ARG
+    assert L.ds_absmax(None, 4, 16, None) == ds.DS_ERR_INVALID_ARG
+    assert L.ds_absmax(16, 0, 16, None) == ds.DS_ERR_SHAPE
+
+
+def test_no_cpu_fallback_without_library(tmp_path, monkeypatch, ds):
+    """The binding refuses to run when the shared library is missing."""
+    monkeypatch.setattr(ds, "_lib", None)
+    monkeypatch.setattr(ds, "LIB_PATH", str(tmp_path / "missing.so"))
+    with pytest.raises(ImportError):
+        ds.lib()

@@ -1,0 +1,89 @@
+"""GPU parity of ConvShift against the CPU oracle (bit-exact)."""
+import numpy as np
+import pytest
+import torch
+
+import synth_inputs as si
+from oracle import deepshift_oracle as O
+
+pytestmark = pytest.mark.gpu
+
+
+def _dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def _run(ds, x, s, p, b, stride, pad, relu=False, residual=None, flags=0):
+    w = ds.pack_shift_weights(_dev(s), _dev(p))
+    amax_io = torch.zeros(2, dtype=torch.int32, device="cuda")
+    y = ds.conv2d_shift(_dev(x), w, s.shape[2:], _dev(b) if b is not None else None, stride, pad, relu=relu,
+                        residual=_dev(residual) if residual is not None else None, amax_io=amax_io,
+                        flags=flags | ds.DS_AMAX_OUT)
+    torch.cuda.synchronize()
+    return y.cpu().numpy(), amax_io.cpu().numpy().view(np.uint32)
+
+
+# N, C, H, W, K, R, S, stride, pad
+GEOMS = [
+    (2, 3, 7, 6, 4, 3, 3, 1, 1),
+    (1, 3, 23, 21, 64, 7, 7, 2, 3),     # ResNet stem shape, small image
+    (2, 16, 9, 9, 20, 1, 1, 2, 0),      # 1x1 / 2 downsample
+    (1, 8, 11, 13, 70, 3, 3, 2, 1),     # 3x3 / 2
+    (3, 32, 8, 8, 64, 3, 3, 1, 1),
+    (1, 64, 14, 14, 64, 3, 3, 1, 1),
+    (2, 5, 5, 5, 3, 5, 5, 1, 0),        # kernel covers the image
+    (1, 1, 1, 1, 1, 1, 1, 1, 0),
+    (1, 40, 7, 7, 130, 1, 1, 1, 0),
+]
+
+
+@pytest.mark.parametrize("geom", GEOMS)
+@pytest.mark.parametrize("flags", [0, 16])
+def test_conv_bitexact(dslib, geom, flags):
+    N, C, H, W, K, R, S, st, pd = geom
+    x, s, p, b = si.conv_layer(sum(geom) * 31 + flags, N, C, H, W, K, R, S, -(1 << 20), 1 << 20)
+    want = O.conv2d_shift(x, s, p, b, (st, st), (pd, pd))
+    got, amax = _run(dslib, x, s, p, b, (st, st), (pd, pd), flags=flags)
+    assert np.array_equal(got, want)
+    assert amax[1] == O.absmax(want)
+
+
+@pytest.mark.parametrize("geom", [GEOMS[0], GEOMS[2], GEOMS[4]])
+def test_conv_relu_residual(dslib, geom):
+    N, C, H, W, K, R, S, st, pd = geom
+    x, s, p, b = si.conv_layer(sum(geom) + 5, N, C, H, W, K, R, S, -(1 << 24), 1 << 24)
+    OH = (H + 2 * pd - R) // st + 1
+    OW = (W + 2 * pd - S) // st + 1
+    res = si.activations(99, (N, K, OH, OW), -(1 << 31), 1 << 31)
+    want = O.add_relu(O.conv2d_shift(x, s, p, b, (st, st), (pd, pd)), res)
+    got, _ = _run(dslib, x, s, p, b, (st, st), (pd, pd), relu=True, residual=res)
+    assert np.array_equal(got, want)
+
+
+def test_conv_saturating_inputs(dslib):
+    x, s, p, b = si.conv_layer(123, 1, 16, 8, 8, 32, 3, 3, -(1 << 31), 1 << 31, centre=-1)
+    want = O.conv2d_shift(x, s, p, b, (1, 1), (1, 1), relu=True)
+    assert (np.abs(O.conv2d_shift_acc(x, s, p, b, (1, 1), (1, 1))) > O.INT32_MAX).any()
+    got, _ = _run(dslib, x, s, p, b, (1, 1), (1, 1), relu=True)
+    assert np.array_equal(got, want)
+
+
+def test_conv_config2_two_images_full(dslib):
+    """The ResNet18 conv2_x layer (64 -> 64, 56 x 56, 3x3/1/1) on two images, every output."""
+    x, s, p, b = si.config2(N=2)
+    want = O.conv2d_shift(x, s, p, b, (1, 1), (1, 1))
+    got, _ = _run(dslib, x, s, p, b, (1, 1), (1, 1))
+    assert np.array_equal(got, want)
+
+
+def test_conv_config2_full_batch_sampled(dslib):
+    """The full N = 32 launch; sampled outputs checked one by one (corners, edges, random)."""
+    x, s, p, b = si.config2()
+    got, _ = _run(dslib, x, s, p, b, (1, 1), (1, 1))
+    rng = np.random.default_rng(1)
+    pts = [(0, 0, 0, 0), (31, 63, 55, 55), (5, 7, 0, 55), (17, 40, 55, 0)]
+    pts += [tuple(int(v) for v in (rng.integers(32), rng.integers(64), rng.integers(56), rng.integers(56)))
+            for _ in range(40)]
+    for (n, k, oh, ow) in pts:
+        want = O.conv2d_shift_at(x, s, p, b, (1, 1), (1, 1), n, k, oh, ow)
+        assert got[n, k, oh, ow] == max(min(want, O.INT32_MAX), O.INT32_MIN), (n, k, oh, ow)

@@ -1,0 +1,123 @@
+"""GPU parity of weight packing and LinearShift against the CPU oracle (bit-exact)."""
+import numpy as np
+import pytest
+import torch
+
+import synth_inputs as si
+from oracle import deepshift_oracle as O
+
+pytestmark = pytest.mark.gpu
+
+
+def _dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def _pack(ds, s, p):
+    return ds.pack_shift_weights(_dev(s.astype(np.int8)), _dev(p.astype(np.int8)))
+
+
+@pytest.mark.parametrize("n_out,k_red", [(1, 1), (3, 31), (64, 576), (65, 33), (512, 784), (130, 100)])
+def test_pack_blob_bitexact(dslib, n_out, k_red):
+    seed = n_out * 7919 + k_red
+    s = si.sign_codes(seed, (n_out, k_red))
+    p = si.shift_codes_uniform(seed, (n_out, k_red))
+    w = _pack(dslib, s, p)
+    torch.cuda.synchronize()
+    want = O.pack_planes6(s, p)
+    got = w.blob.cpu().numpy()
+    assert got.size == want.size
+    assert np.array_equal(got, want)
+    A, nnz = O.column_constants(s, p)
+    assert w.desc.a_max == int(A.max()) and w.desc.nnz_max == int(nnz.max())
+
+
+def test_pack_rejects_bad_codes(dslib):
+    s = np.ones((4, 10), np.int8)
+    p = np.zeros((4, 10), np.int8)
+    s[2, 3] = 2
+    with pytest.raises(dslib.DsError) as e:
+        _pack(dslib, s, p)
+    assert e.value.status == dslib.DS_ERR_CODE_RANGE
+    s[2, 3] = 1
+    p[1, 1] = 1
+    with pytest.raises(dslib.DsError):
+        _pack(dslib, s, p)
+    p[1, 1] = -16
+    with pytest.raises(dslib.DsError):
+        _pack(dslib, s, p)
+
+
+def _run_fc(ds, x, s, p, b, flags=0, amax=True):
+    w = _pack(ds, s, p)
+    xd = _dev(x.astype(np.int32))
+    bd = _dev(b.astype(np.int32)) if b is not None else None
+    amax_io = torch.zeros(2, dtype=torch.int32, device="cuda") if amax else None
+    y = ds.linear_shift(xd, w, bd, amax_io=amax_io, flags=flags)
+    torch.cuda.synchronize()
+    return y.cpu().numpy(), (amax_io.cpu().numpy().view(np.uint32) if amax else None)
+
+
+FC_SHAPES = [(1, 1, 1), (3, 5, 7), (64, 784, 512), (129, 33, 65), (130, 100, 130), (257, 64, 64),
+             (5, 1000, 3), (200, 4, 70), (31, 129, 1)]
+
+
+@pytest.mark.parametrize("M,K,N", FC_SHAPES)
+@pytest.mark.parametrize("flags", [0, 1, 16, 17])
+def test_linear_shift_bitexact(dslib, M, K, N, flags):
+    x, s, p, b = si.fc_layer(M * 1000 + K * 10 + N, M, K, N, -(1 << 20), 1 << 20)
+    want = O.linear_shift(x, s, p, b, relu=bool(flags & 1))
+    got, amax = _run_fc(dslib, x, s, p, b, flags | dslib.DS_AMAX_OUT)
+    assert np.array_equal(got, want)
+    assert amax[0] == O.absmax(x)
+    assert amax[1] == O.absmax(want)
+
+
+def test_linear_shift_config1_bitexact(dslib):
+    x, s, p, b = si.config1()
+    want = O.linear_shift(x, s, p, b)
+    got, _ = _run_fc(dslib, x, s, p, b)
+    assert np.array_equal(got, want)
+
+
+def test_linear_shift_no_bias_no_amax(dslib):
+    x, s, p, b = si.fc_layer(77, 40, 70, 90, -(1 << 31), 1 << 31)
+    got, _ = _run_fc(dslib, x, s, p, None, 0, amax=False)
+    assert np.array_equal(got, O.linear_shift(x, s, p, None))
+
+
+@pytest.mark.parametrize("M,K,N", [(70, 300, 66), (128, 64, 64)])
+def test_linear_shift_saturating_inputs(dslib, M, K, N):
+    """Full-range int32 activations: the 64-bit path must take over and saturate exactly."""
+    x, s, p, b = si.fc_layer(M + K + N, M, K, N, -(1 << 31), 1 << 31)
+    p = np.where(np.arange(K)[None, :] % 3 == 0, 0, p).astype(np.int8)  # many unit weights
+    want = O.linear_shift(x, s, p, b, relu=True)
+    assert (np.abs(O.linear_shift_acc(x, s, p, b)) > O.INT32_MAX).any()
+    got, _ = _run_fc(dslib, x, s, p, b, dslib.DS_RELU)
+    assert np.array_equal(got, want)
+
+
+def test_linear_shift_amax_in_is_used(dslib):
+    """A caller-provided amax that proves int32 safety gives the same exact result."""
+    x, s, p, b = si.fc_layer(5, 96, 96, 96, -(1 << 20), 1 << 20)
+    w = _pack(dslib, s, p)
+    amax_io = torch.tensor([O.absmax(x), 0], dtype=torch.int64).to(torch.int32).cuda()
+    y = dslib.linear_shift(_dev(x), w, _dev(b), amax_io=amax_io, flags=dslib.DS_AMAX_IN)
+    assert np.array_equal(y.cpu().numpy(), O.linear_shift(x, s, p, b))
+
+
+def test_linear_shift_config4_sampled(dslib):
+    """Full-size 8192 x 4096 x 4096 launch; sampled outputs checked one by one."""
+    x, s, p, b = si.config4_int()
+    w = _pack(dslib, s, p)
+    amax_io = torch.zeros(2, dtype=torch.int32, device="cuda")
+    y = dslib.linear_shift(_dev(x), w, _dev(b), amax_io=amax_io).cpu().numpy()
+    rng = np.random.default_rng(0)
+    rows = np.concatenate([[0, 8191], rng.integers(0, 8192, 30)])
+    cols = np.concatenate([[0, 4095], rng.integers(0, 4096, 30)])
+    for m, n in zip(rows, cols):
+        want = O.linear_shift_at(x, s, p, b, int(m), int(n))
+        assert y[m, n] == max(min(want, O.INT32_MAX), O.INT32_MIN)
+    # whole rows against the vectorised oracle
+    for m in (0, 4097):
+        assert np.array_equal(y[m:m + 1], O.linear_shift(x[m:m + 1], s, p, b))
