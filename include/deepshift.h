@@ -170,6 +170,32 @@ ds_status ds_conv2d_shift(const int32_t* x, const ds_weights* w, const int32_t* 
                           uint32_t flags, uint32_t* amax_io, void* stream);
 
 /*
+ * LinearShift for callers that cannot allocate device memory.  The paper has
+ * no counterpart: this is a deployment convenience of this library.
+ *
+ * Same operation, arguments and errors as ds_linear_shift, except that the
+ * two scratch words of amax_io come from a static device array of 64 u32
+ * (256 bytes) that every GPU loading this library holds until the process
+ * exits.  It suits callers that must not call cudaMalloc or any allocating
+ * routine: a plugin given only its input and output buffers, a host callback,
+ * a real-time path that must stay out of the allocator.  Each call uses two of
+ * the 64 words whatever the problem size; a build whose per-call need exceeded
+ * the array would be rejected with DS_ERR_UNSUPPORTED.  DS_AMAX_IN and
+ * DS_AMAX_OUT are rejected (DS_ERR_INVALID_ARG): they need caller scratch.
+ *   - The first call on each device looks up the array's device address
+ *     (cudaGetSymbolAddress with that device current) and caches it; make that
+ *     first call before any stream capture.
+ *   - All calls share the array, which keeps the last call's contents; the
+ *     max|x| pre-pass clears its word before writing it.  Calls that overlap on
+ *     the GPU (different streams without ordering, or several threads) race on
+ *     the array and may compute wrong results: order them on one stream.
+ *   - It allocates nothing: no cudaMalloc, cudaFree or allocating library call.
+ */
+ds_status ds_linear_shift_static_scratch(const int32_t* x, const ds_weights* w, const int32_t* bias,
+                                         int32_t* y, int64_t M, int64_t K, int64_t N, uint32_t flags,
+                                         void* stream);
+
+/*
  * max |x| over n int32 values, written to *amax (device u32; |INT32_MIN| = 2^31).
  */
 ds_status ds_absmax(const int32_t* x, int64_t n, uint32_t* amax, void* stream);

@@ -66,6 +66,10 @@ _SIGNATURES = {
     "ds_conv2d_shift": (ctypes.c_int, [ctypes.c_void_p, ctypes.POINTER(ds_weights), ctypes.c_void_p,
                                        ctypes.c_void_p, ctypes.c_void_p] + [ctypes.c_int] * 11 +
                         [ctypes.c_uint32, ctypes.c_void_p, ctypes.c_void_p]),
+    "ds_linear_shift_static_scratch": (ctypes.c_int, [ctypes.c_void_p, ctypes.POINTER(ds_weights),
+                                                      ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64,
+                                                      ctypes.c_int64, ctypes.c_int64, ctypes.c_uint32,
+                                                      ctypes.c_void_p]),
     "ds_absmax": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]),
 }
 
@@ -136,6 +140,13 @@ def ds_conv2d_shift(x, w: ds_weights, bias, residual, y, N, C, H, W, K, R, S, st
     _check(lib().ds_conv2d_shift(_ptr(x), ctypes.byref(w), _ptr(bias), _ptr(residual), _ptr(y), N, C, H,
                                  W, K, R, S, stride_h, stride_w, pad_h, pad_w, flags, _ptr(amax_io),
                                  _stream(stream)))
+
+
+def ds_linear_shift_static_scratch(x, w: ds_weights, bias, y, M: int, K: int, N: int, flags: int = 0,
+                                   stream=None) -> None:
+    """ds_linear_shift with its scratch in the library's static device array (no allocation)."""
+    _check(lib().ds_linear_shift_static_scratch(_ptr(x), ctypes.byref(w), _ptr(bias), _ptr(y), M, K, N, flags,
+                                                _stream(stream)))
 
 
 def ds_absmax(x, n: int, amax, stream=None) -> None:
