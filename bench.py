@@ -266,7 +266,7 @@ def run_gpu(args, wl, rank, world, local_rank):
                        "step": "absmax pre-pass + ConvShift (fused bias/saturate epilogue)"},
             "roofline": {"bound": "alu", "achieved": achieved, "peak": alu_peak, "unit": "Tintop/s",
                          "frac": achieved / alu_peak, "traffic": None,
-                         "kernel": "shift_gemm_kernel<conv>", "kernel_ms": kern_ms,
+                         "kernel": "conv_direct_kernel<1,3>", "kernel_ms": kern_ms,
                          "peak_basis": f"{SMS} SMs x {INT_OPS_PER_CLK_PER_SM} int32 ops/clk x {sm_max:.0f} MHz "
                                        f"(sm_max_mhz, {peak_kind})",
                          "alg_int_ops_per_launch": ALG_INT_OPS_PER_TERM * wl["terms"],

@@ -63,6 +63,8 @@ int ds_version(void);
 #define DS_AMAX_OUT 4u  /* write max|y| over this call's outputs into amax_io[1] */
 #define DS_RESIDUAL 8u  /* conv only: y = sat32(sat32(conv) + residual) before the ReLU */
 #define DS_FORCE_INT64 16u /* always use the 64-bit accumulator path (testing / worst case) */
+#define DS_CONV_IM2COL 32u /* conv only: use the implicit-GEMM (im2col gather) kernel instead of the
+                              direct halo-tile kernel (testing / comparison) */
 
 /* ---------------------------------------------------------------------------
  * Packed weights.

@@ -33,6 +33,7 @@ DS_AMAX_IN = 2
 DS_AMAX_OUT = 4
 DS_RESIDUAL = 8
 DS_FORCE_INT64 = 16
+DS_CONV_IM2COL = 32
 
 DS_WEIGHTS_MAGIC = 0x31575344
 DS_FORMAT_PLANES6 = 1

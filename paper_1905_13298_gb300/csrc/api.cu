@@ -86,7 +86,8 @@ static ds_status prepare_amax(const int32_t* x, int64_t nx, uint32_t flags, uint
   return DS_OK;
 }
 
-constexpr uint32_t kKnownFlags = DS_RELU | DS_AMAX_IN | DS_AMAX_OUT | DS_RESIDUAL | DS_FORCE_INT64;
+constexpr uint32_t kKnownFlags =
+    DS_RELU | DS_AMAX_IN | DS_AMAX_OUT | DS_RESIDUAL | DS_FORCE_INT64 | DS_CONV_IM2COL;
 
 }  // namespace ds
 
@@ -154,7 +155,8 @@ ds_status ds_linear_shift(const int32_t* x, const ds_weights* w, const int32_t* 
   if (M <= 0 || K <= 0 || N <= 0) return fail(DS_ERR_SHAPE, "M, K and N must be positive");
   if (M > (int64_t(1) << 40) || N > 65535LL * 64) return fail(DS_ERR_UNSUPPORTED, "M or N too large");
   if (flags & ~kKnownFlags) return fail(DS_ERR_INVALID_ARG, "unknown flag bits 0x%x", flags & ~kKnownFlags);
-  if (flags & DS_RESIDUAL) return fail(DS_ERR_INVALID_ARG, "DS_RESIDUAL applies to ds_conv2d_shift only");
+  if (flags & (DS_RESIDUAL | DS_CONV_IM2COL))
+    return fail(DS_ERR_INVALID_ARG, "DS_RESIDUAL / DS_CONV_IM2COL apply to ds_conv2d_shift only");
   if ((flags & (DS_AMAX_IN | DS_AMAX_OUT)) && amax_io == nullptr)
     return fail(DS_ERR_INVALID_ARG, "DS_AMAX_IN / DS_AMAX_OUT need amax_io");
   if (!aligned16(x) || !aligned16(y)) return fail(DS_ERR_ALIGNMENT, "x and y must be 16-byte aligned");
@@ -233,7 +235,9 @@ ds_status ds_conv2d_shift(const int32_t* x, const ds_weights* w, const int32_t* 
   fill_blob_offsets(p, w);
   r = prepare_amax(x, nx, flags, amax_io, st, p);
   if (r != DS_OK) return r;
-  return cuda_check(launch_conv2d_shift(p, st), "conv2d_shift launch");
+  if (!(flags & DS_CONV_IM2COL) && conv_direct_supported(p))
+    return cuda_check(launch_conv2d_direct(p, st), "conv2d_shift (direct) launch");
+  return cuda_check(launch_conv2d_shift(p, st), "conv2d_shift (implicit GEMM) launch");
 }
 
 }  // extern "C"

@@ -77,6 +77,9 @@ struct GemmParams {
 // Launchers (defined in shift_gemm.cu).
 cudaError_t launch_linear_shift(const GemmParams& p, cudaStream_t st);
 cudaError_t launch_conv2d_shift(const GemmParams& p, cudaStream_t st);
+// Defined in conv_direct.cu.
+bool conv_direct_supported(const GemmParams& p);
+cudaError_t launch_conv2d_direct(const GemmParams& p, cudaStream_t st);
 // Defined in misc_kernels.cu.
 cudaError_t launch_absmax(const int32_t* x, int64_t n, uint32_t* out, cudaStream_t st);
 cudaError_t launch_pack(const int8_t* s, const int8_t* p, int64_t n_out, int64_t k_red,

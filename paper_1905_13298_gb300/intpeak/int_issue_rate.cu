@@ -1,0 +1,88 @@
+// Integer issue-rate microbenchmark for the roofline denominator of the
+// shift kernels (built as its own small library, not part of the C ABI).
+//
+// Each kernel runs a register-resident loop of one instruction mix with
+// enough independent chains to hide latency, one full wave of CTAs, and
+// reports per-CTA SM cycles from clock64().  ops/clk/SM = thread instructions
+// of the mix executed by the CTAs of one SM / cycles.
+//   kind 0: SHF only        (shr.s32, ALU pipe)
+//   kind 1: IMAD only       (mad.lo.s32, FMA pipe)
+//   kind 2: SHF + IMAD      (the shift-GEMM inner loop: t = x >> s; acc += g * t)
+//   kind 3: IADD3 only      (add.s32 chains)
+//   kind 4: LOP3 only       (xor/and chains)
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace {
+
+template <int KIND>
+__global__ void __launch_bounds__(256) mix_kernel(const int* __restrict__ seed, int iters, int* out,
+                                                  long long* cycles) {
+  int x[8], s[8], g[8], acc[8][8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    x[i] = seed[(threadIdx.x + i) & 63];
+    s[i] = seed[64 + i] & 15;
+    g[i] = seed[72 + i];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc[i][j] = i ^ j;
+  }
+  __syncthreads();
+  const long long t0 = clock64();
+  for (int it = 0; it < iters; ++it) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        if (KIND == 0) {
+          asm volatile("shr.s32 %0, %0, %1;" : "+r"(acc[i][j]) : "r"(s[j]));
+        } else if (KIND == 1) {
+          asm volatile("mad.lo.s32 %0, %0, %1, %2;" : "+r"(acc[i][j]) : "r"(g[j]), "r"(x[i]));
+        } else if (KIND == 2) {
+          int t;
+          asm volatile("shr.s32 %0, %1, %2;" : "=r"(t) : "r"(x[i]), "r"(s[j]));
+          asm volatile("mad.lo.s32 %0, %1, %2, %0;" : "+r"(acc[i][j]) : "r"(g[j]), "r"(t));
+        } else if (KIND == 3) {
+          asm volatile("add.s32 %0, %0, %1;" : "+r"(acc[i][j]) : "r"(x[i]));
+        } else {
+          asm volatile("xor.b32 %0, %0, %1;" : "+r"(acc[i][j]) : "r"(g[j]));
+        }
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) x[i] += acc[i][i];
+  }
+  const long long t1 = clock64();
+  int r = 0;
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) r ^= acc[i][j];
+  out[blockIdx.x * blockDim.x + threadIdx.x] = r;
+  if (threadIdx.x == 0) cycles[blockIdx.x] = t1 - t0;
+}
+
+}  // namespace
+
+// Runs one mix; writes the mean CTA cycle count and the kernel time (ms).
+// out must hold blocks*threads ints, cycles `blocks` long longs, seed 80 ints.
+extern "C" int ds_probe_int_mix(int kind, int blocks, int threads, int iters, const int* seed, int* out,
+                                long long* cycles, float* ms) {
+  cudaEvent_t a, b;
+  cudaEventCreate(&a);
+  cudaEventCreate(&b);
+  cudaEventRecord(a);
+  switch (kind) {
+    case 0: mix_kernel<0><<<blocks, threads>>>(seed, iters, out, cycles); break;
+    case 1: mix_kernel<1><<<blocks, threads>>>(seed, iters, out, cycles); break;
+    case 2: mix_kernel<2><<<blocks, threads>>>(seed, iters, out, cycles); break;
+    case 3: mix_kernel<3><<<blocks, threads>>>(seed, iters, out, cycles); break;
+    default: mix_kernel<4><<<blocks, threads>>>(seed, iters, out, cycles); break;
+  }
+  cudaEventRecord(b);
+  cudaError_t e = cudaEventSynchronize(b);
+  cudaEventElapsedTime(ms, a, b);
+  cudaEventDestroy(a);
+  cudaEventDestroy(b);
+  return e == cudaSuccess ? (int)cudaGetLastError() : (int)e;
+}

@@ -38,7 +38,7 @@ GEOMS = [
 
 
 @pytest.mark.parametrize("geom", GEOMS)
-@pytest.mark.parametrize("flags", [0, 16])
+@pytest.mark.parametrize("flags", [0, 16, 32, 48])  # direct / forced 64-bit / implicit GEMM / both
 def test_conv_bitexact(dslib, geom, flags):
     N, C, H, W, K, R, S, st, pd = geom
     x, s, p, b = si.conv_layer(sum(geom) * 31 + flags, N, C, H, W, K, R, S, -(1 << 20), 1 << 20)
@@ -49,23 +49,49 @@ def test_conv_bitexact(dslib, geom, flags):
 
 
 @pytest.mark.parametrize("geom", [GEOMS[0], GEOMS[2], GEOMS[4]])
-def test_conv_relu_residual(dslib, geom):
+@pytest.mark.parametrize("flags", [0, 32])
+def test_conv_relu_residual(dslib, geom, flags):
     N, C, H, W, K, R, S, st, pd = geom
     x, s, p, b = si.conv_layer(sum(geom) + 5, N, C, H, W, K, R, S, -(1 << 24), 1 << 24)
     OH = (H + 2 * pd - R) // st + 1
     OW = (W + 2 * pd - S) // st + 1
     res = si.activations(99, (N, K, OH, OW), -(1 << 31), 1 << 31)
     want = O.add_relu(O.conv2d_shift(x, s, p, b, (st, st), (pd, pd)), res)
-    got, _ = _run(dslib, x, s, p, b, (st, st), (pd, pd), relu=True, residual=res)
+    got, _ = _run(dslib, x, s, p, b, (st, st), (pd, pd), relu=True, residual=res, flags=flags)
     assert np.array_equal(got, want)
 
 
-def test_conv_saturating_inputs(dslib):
+@pytest.mark.parametrize("flags", [0, 32])
+def test_conv_saturating_inputs(dslib, flags):
     x, s, p, b = si.conv_layer(123, 1, 16, 8, 8, 32, 3, 3, -(1 << 31), 1 << 31, centre=-1)
     want = O.conv2d_shift(x, s, p, b, (1, 1), (1, 1), relu=True)
     assert (np.abs(O.conv2d_shift_acc(x, s, p, b, (1, 1), (1, 1))) > O.INT32_MAX).any()
-    got, _ = _run(dslib, x, s, p, b, (1, 1), (1, 1), relu=True)
+    got, _ = _run(dslib, x, s, p, b, (1, 1), (1, 1), relu=True, flags=flags)
     assert np.array_equal(got, want)
+
+
+# ResNet18 / ResNet50 / VGG16 layer shapes at a small batch, both kernels
+NET_GEOMS = [
+    (1, 3, 224, 224, 64, 7, 7, 2, 3),    # stem 7x7/2
+    (2, 64, 56, 56, 64, 3, 3, 1, 1),     # conv2_x
+    (2, 64, 56, 56, 128, 3, 3, 2, 1),    # conv3_1 3x3/2
+    (2, 64, 56, 56, 128, 1, 1, 2, 0),    # downsample 1x1/2
+    (2, 128, 28, 28, 128, 3, 3, 1, 1),
+    (2, 256, 14, 14, 256, 3, 3, 1, 1),
+    (2, 512, 7, 7, 512, 3, 3, 1, 1),
+    (2, 64, 56, 56, 256, 1, 1, 1, 0),    # bottleneck expand
+    (1, 3, 32, 32, 64, 3, 3, 1, 1),      # VGG first conv (small image)
+]
+
+
+@pytest.mark.parametrize("geom", NET_GEOMS)
+def test_conv_network_layer_shapes(dslib, geom):
+    N, C, H, W, K, R, S, st, pd = geom
+    x, s, p, b = si.conv_layer(sum(geom) * 7, N, C, H, W, K, R, S, 0, 1 << 20)
+    want = O.conv2d_shift(x, s, p, b, (st, st), (pd, pd), relu=True)
+    for flags in (0, 32):
+        got, _ = _run(dslib, x, s, p, b, (st, st), (pd, pd), relu=True, flags=flags)
+        assert np.array_equal(got, want), flags
 
 
 def test_conv_config2_two_images_full(dslib):
