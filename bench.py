@@ -160,7 +160,7 @@ def run_gpu(args, wl, rank, world, local_rank):
     N, C, H, W, K, R, S = (wl[k] for k in ("N", "C", "H", "W", "K", "R", "S"))
     seed = si.SEED_BASE + 2 + 1000 * rank
     x, s, p, b = si.conv_layer(seed, N, C, H, W, K, R, S)
-    w = ds.pack_shift_weights(torch.from_numpy(s).to(dev), torch.from_numpy(p).to(dev))
+    w = ds.pack_shift_weights(torch.from_numpy(s).to(dev), torch.from_numpy(p).to(dev), expand=True)
     bd = torch.from_numpy(b).to(dev)
     per_step_bytes = x.nbytes * 2
     n_rot = max(2, int(np.ceil(2 * L2_BYTES / per_step_bytes)))
@@ -260,13 +260,13 @@ def run_gpu(args, wl, rank, world, local_rank):
             "warmup": args.warmup, "ms_per_step": ms_total / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "int32", "data": "synthetic",
             "config": {"workload": wl["name"], "batch": N, "C": C, "H": H, "W": W, "K": K, "kernel": "3x3",
-                       "stride": 1, "pad": 1, "codes": "p geometric around -6, P(s=0)=0.1",
+                       "stride": 1, "pad": 1, "codes": "p geometric around -6, P(s=0)=0.1; 6-bit packed blob + expanded execution layout",
                        "activations": "uniform [0, 2^20) int32 Q16.16",
                        "l2": f"rotating {n_rot} input/output sets ({n_rot * per_step_bytes / 2**20:.0f} MiB > L2)",
                        "step": "absmax pre-pass + ConvShift (fused bias/saturate epilogue)"},
             "roofline": {"bound": "alu", "achieved": achieved, "peak": alu_peak, "unit": "Tintop/s",
                          "frac": achieved / alu_peak, "traffic": None,
-                         "kernel": "conv_direct_kernel<1,3>", "kernel_ms": kern_ms,
+                         "kernel": "conv_direct_kernel<1,3,7,32>", "kernel_ms": kern_ms,
                          "peak_basis": f"{SMS} SMs x {INT_OPS_PER_CLK_PER_SM} int32 ops/clk x {sm_max:.0f} MHz "
                                        f"(sm_max_mhz, {peak_kind})",
                          "alg_int_ops_per_launch": ALG_INT_OPS_PER_TERM * wl["terms"],

@@ -110,6 +110,8 @@ typedef struct ds_weights {
   uint64_t a_max;       /* max over columns of A[n] */
   uint32_t nnz_max;     /* max over columns of the non-zero count */
   uint32_t reserved;
+  const void* expanded; /* NULL, or the execution layout set by ds_expand_shift_weights */
+  size_t expanded_bytes;
 } ds_weights;
 
 /* Bytes needed for the packed blob of an n_out x k_red code matrix (0 if invalid). */
@@ -129,6 +131,32 @@ ds_status ds_pack_shift_weights(const int8_t* s, const int8_t* p, int64_t n_out,
                                 void* packed, size_t packed_bytes, ds_weights* desc, void* stream);
 
 /* ---------------------------------------------------------------------------
+ * Expanded execution layout (optional).  The packed blob is the storage
+ * format; decoding it inside every CTA of every launch costs a measurable
+ * share of the integer issue slots of these ALU-bound kernels.  A layer may
+ * therefore be expanded once into 32-bit shift / sign words laid out as the
+ * kernels stage them:
+ *   int32 [ceil(n_out / 32)][k_red][64]: for column block cb and reduction
+ *   index k, words 0..31 hold -p and words 32..63 hold s of columns
+ *   32*cb .. 32*cb + 31 (zero beyond n_out).
+ * 8 bytes per weight (plus padding of the last column block).  Kernels use
+ * it when desc->expanded is set and decode the blob otherwise; results are
+ * identical either way.
+ * ------------------------------------------------------------------------- */
+
+/* Bytes of the expanded layout of an n_out x k_red code matrix (0 if invalid). */
+size_t ds_expanded_weight_bytes(int64_t n_out, int64_t k_red);
+
+/*
+ * Expand packed weights into `expanded` (device, 16-byte aligned, at least
+ * ds_expanded_weight_bytes bytes, caller-owned and outliving every use) and
+ * record it in *w (w->expanded, w->expanded_bytes).  Stream-ordered and
+ * asynchronous; the blob must stay valid.  Errors: DS_ERR_INVALID_ARG for an
+ * unfilled descriptor, DS_ERR_BUFFER_TOO_SMALL, DS_ERR_ALIGNMENT.
+ */
+ds_status ds_expand_shift_weights(ds_weights* w, void* expanded, size_t expanded_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------
  * Accumulator width.  Each compute call proves, on the device and with no
  * host round trip, whether 32-bit accumulation is exact:
  *     ceil(amax * A[n] / 2^15) + nnz[n] + |b[n]| <= 2^31 - 1   for every n
@@ -136,8 +164,8 @@ ds_status ds_pack_shift_weights(const int8_t* s, const int8_t* p, int64_t n_out,
  * wrap-around and no saturation can occur); otherwise a 64-bit path runs and
  * the exact sum is saturated.  amax comes from amax_io[0] when DS_AMAX_IN is
  * set, else from a pre-pass over x that writes it to amax_io[0].  amax_io
- * (device, 2 x u32) may be NULL only with DS_FORCE_INT64 unset and then the
- * 64-bit path is always taken.
+ * (device, 2 x u32) may be NULL: then no bound is available and the 64-bit
+ * path is always taken (DS_AMAX_IN and DS_AMAX_OUT need amax_io).
  * ------------------------------------------------------------------------- */
 
 /*

@@ -384,3 +384,19 @@ def unpack_planes6(blob, n_out: int, k_red: int):
             nz = (int(bits[g, n, 1]) >> j) & 1
             s[n, k] = 0 if not nz else (-1 if neg else 1)
     return s, p
+
+
+def expand_codes(s, p) -> np.ndarray:
+    """Expanded execution layout of [n_out, k_red] codes (documented in include/deepshift.h):
+    int32 [ceil(n_out/32)][k_red][64], words 0..31 = -p and 32..63 = s of columns 32*cb + c."""
+    s = np.asarray(s, dtype=np.int64)
+    p = np.asarray(p, dtype=np.int64)
+    _check_codes(s, p)
+    n_out, k_red = s.shape
+    nb = (n_out + 31) // 32
+    out = np.zeros((nb, k_red, 64), dtype=np.int32)
+    for n in range(n_out):
+        cb, c = divmod(n, 32)
+        out[cb, :, c] = -p[n, :]
+        out[cb, :, 32 + c] = s[n, :]
+    return out

@@ -49,7 +49,8 @@ class ds_weights(ctypes.Structure):
     _fields_ = [("magic", ctypes.c_uint32), ("format", ctypes.c_uint32),
                 ("n_out", ctypes.c_int64), ("k_red", ctypes.c_int64), ("n_chunks", ctypes.c_int64),
                 ("packed", ctypes.c_void_p), ("packed_bytes", ctypes.c_size_t),
-                ("a_max", ctypes.c_uint64), ("nnz_max", ctypes.c_uint32), ("reserved", ctypes.c_uint32)]
+                ("a_max", ctypes.c_uint64), ("nnz_max", ctypes.c_uint32), ("reserved", ctypes.c_uint32),
+                ("expanded", ctypes.c_void_p), ("expanded_bytes", ctypes.c_size_t)]
 
 
 _lib = None
@@ -71,6 +72,9 @@ _SIGNATURES = {
                                                       ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64,
                                                       ctypes.c_int64, ctypes.c_int64, ctypes.c_uint32,
                                                       ctypes.c_void_p]),
+    "ds_expanded_weight_bytes": (ctypes.c_size_t, [ctypes.c_int64, ctypes.c_int64]),
+    "ds_expand_shift_weights": (ctypes.c_int, [ctypes.POINTER(ds_weights), ctypes.c_void_p, ctypes.c_size_t,
+                                               ctypes.c_void_p]),
     "ds_absmax": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]),
 }
 
@@ -130,6 +134,14 @@ def ds_pack_shift_weights(s, p, n_out: int, k_red: int, packed, packed_bytes: in
     return desc
 
 
+def ds_expanded_weight_bytes(n_out: int, k_red: int) -> int:
+    return int(lib().ds_expanded_weight_bytes(n_out, k_red))
+
+
+def ds_expand_shift_weights(w: ds_weights, expanded, expanded_bytes: int, stream=None) -> None:
+    _check(lib().ds_expand_shift_weights(ctypes.byref(w), _ptr(expanded), expanded_bytes, _stream(stream)))
+
+
 def ds_linear_shift(x, w: ds_weights, bias, y, M: int, K: int, N: int, flags: int = 0, amax_io=None,
                     stream=None) -> None:
     _check(lib().ds_linear_shift(_ptr(x), ctypes.byref(w), _ptr(bias), _ptr(y), M, K, N, flags,
@@ -159,11 +171,13 @@ def ds_absmax(x, n: int, amax, stream=None) -> None:
 # ---------------------------------------------------------------------------
 
 class PackedShiftWeights:
-    """A packed blob (device uint8 tensor) plus its ds_weights descriptor."""
+    """A packed blob (device uint8 tensor) plus its ds_weights descriptor and,
+    optionally, the expanded execution layout (device int32 tensor)."""
 
     def __init__(self, blob, desc: ds_weights):
         self.blob = blob
         self.desc = desc
+        self.expanded = None
 
     @property
     def n_out(self) -> int:
@@ -174,8 +188,19 @@ class PackedShiftWeights:
         return int(self.desc.k_red)
 
 
-def pack_shift_weights(s, p, stream=None) -> PackedShiftWeights:
-    """Packs int8 sign/shift code tensors [n_out, ...] (device) into a new blob."""
+def expand_shift_weights(w: PackedShiftWeights, stream=None) -> PackedShiftWeights:
+    """Adds the expanded execution layout to packed weights (8 bytes per weight)."""
+    import torch
+    nbytes = ds_expanded_weight_bytes(w.n_out, w.k_red)
+    buf = torch.empty(nbytes // 4, dtype=torch.int32, device=w.blob.device)
+    ds_expand_shift_weights(w.desc, buf, nbytes, stream)
+    w.expanded = buf
+    return w
+
+
+def pack_shift_weights(s, p, stream=None, expand: bool = False) -> PackedShiftWeights:
+    """Packs int8 sign/shift code tensors [n_out, ...] (device) into a new blob;
+    with expand=True also builds the expanded execution layout."""
     import torch
     if s.device.type != "cuda" or p.device.type != "cuda":
         raise ValueError("codes must be CUDA tensors")
@@ -188,7 +213,10 @@ def pack_shift_weights(s, p, stream=None) -> PackedShiftWeights:
         raise DsError(DS_ERR_SHAPE, "invalid code matrix shape")
     blob = torch.empty(nbytes, dtype=torch.uint8, device=s.device)
     desc = ds_pack_shift_weights(s2, p2, n_out, k_red, blob, nbytes, stream)
-    return PackedShiftWeights(blob, desc)
+    w = PackedShiftWeights(blob, desc)
+    if expand:
+        expand_shift_weights(w, stream)
+    return w
 
 
 def linear_shift(x, w: PackedShiftWeights, bias=None, relu: bool = False, amax_io=None, flags: int = 0,

@@ -59,6 +59,10 @@ static ds_status check_weights(const ds_weights* w, int64_t n_out, int64_t k_red
 static void fill_blob_offsets(GemmParams& p, const ds_weights* w) {
   const BlobLayout L = blob_layout(w->n_out, w->k_red);
   p.blob = static_cast<const uint8_t*>(w->packed);
+  p.xcodes = (w->expanded != nullptr &&
+              w->expanded_bytes >= (size_t)expanded_words(w->n_out, w->k_red) * sizeof(int32_t))
+                 ? static_cast<const int32_t*>(w->expanded)
+                 : nullptr;
   p.n_chunks = L.n_chunks;
   p.off_nib = L.nib;
   p.off_bits = L.bits;
@@ -137,6 +141,33 @@ ds_status ds_pack_shift_weights(const int8_t* s, const int8_t* p, int64_t n_out,
   desc->a_max = h.a_max;
   desc->nnz_max = h.nnz_max;
   desc->reserved = 0;
+  desc->expanded = nullptr;
+  desc->expanded_bytes = 0;
+  return DS_OK;
+}
+
+size_t ds_expanded_weight_bytes(int64_t n_out, int64_t k_red) {
+  if (n_out <= 0 || k_red <= 0) return 0;
+  if (n_out > (int64_t(1) << 31) || k_red > (int64_t(1) << 36)) return 0;
+  return (size_t)expanded_words(n_out, k_red) * sizeof(int32_t);
+}
+
+ds_status ds_expand_shift_weights(ds_weights* w, void* expanded, size_t expanded_bytes, void* stream) {
+  clear_error();
+  if (w == nullptr || expanded == nullptr) return fail(DS_ERR_INVALID_ARG, "NULL pointer argument");
+  ds_status r = check_weights(w, w->n_out, w->k_red);
+  if (r != DS_OK) return r;
+  const size_t need = ds_expanded_weight_bytes(w->n_out, w->k_red);
+  if (need == 0) return fail(DS_ERR_UNSUPPORTED, "code matrix too large to expand");
+  if (expanded_bytes < need)
+    return fail(DS_ERR_BUFFER_TOO_SMALL, "expanded buffer has %zu bytes, needs %zu", expanded_bytes, need);
+  if (!aligned16(expanded)) return fail(DS_ERR_ALIGNMENT, "expanded buffer must be 16-byte aligned");
+  r = cuda_check(launch_expand(static_cast<const uint8_t*>(w->packed), w->n_out, w->k_red,
+                               static_cast<int32_t*>(expanded), static_cast<cudaStream_t>(stream)),
+                 "expand launch");
+  if (r != DS_OK) return r;
+  w->expanded = expanded;
+  w->expanded_bytes = need;
   return DS_OK;
 }
 

@@ -3,14 +3,16 @@
 //   y[n][k][oh][ow] = sat32( b[k] + sum_{c,r,s} s_w * (xpad[n][c][oh*sig + r][ow*sig + s] >> -p) )
 //
 // CTA tile: one image, TH output rows x GW groups of TM consecutive output
-// columns, NT output channels.  A thread owns one group (TM pixels of one
-// row) and TN = 4 channels.  Per chunk of CC input channels (one pipeline
-// stage) the CTA stages into shared memory
+// columns, NT output channels (256 threads, 8 warps).  A thread owns one
+// group (TM pixels of one row) and TN = 4 channels.  Per chunk of CC input
+// channels (one pipeline stage) the CTA stages into shared memory
 //   * the input window of every group, zero outside the image, as a "slot"
 //     of WSP words (WS = (TM-1)*sig + S values, padded to 16 bytes), so that
 //     a thread reads the window of one kernel row with WSP/4 vector loads;
-//   * the decoded codes of the chunk's taps, shift and sign as 32-bit words,
-//     one row of NT channels per tap.
+//   * the codes of the chunk's taps as 32-bit shift / sign words, one row of
+//     NT channels per tap: copied with 16-byte cp.async from the expanded
+//     execution layout when the layer has one, else decoded from the packed
+//     blob (one item of at most 16 taps of one channel per thread).
 // For each (c, r) a thread loads its window once and reuses it for the S
 // taps of that row (sliding window); per term the hot loop issues one
 // arithmetic right shift (ALU pipe) and one multiply-add by the sign (FMA
@@ -23,22 +25,19 @@
 namespace ds {
 namespace {
 
-constexpr int TN = 4;            // output channels per thread
-constexpr int kThreads = 256;    // 8 warps: every SM sub-partition gets the same share
+constexpr int TN = 4;                   // output channels per thread
+constexpr int kThreads = 256;           // 8 warps: every SM sub-partition gets the same share
 constexpr int kSmemBudget = 74 * 1024;  // 3 CTAs per SM
 
 struct DirectGeom {
-  int NT, CG;        // channels per CTA, channel groups (NT / TN)
   int TH, GW;        // output rows and pixel groups per row per CTA
-  int WSP;           // slot words per group
   int CC;            // input channels per stage
   int HR;            // halo rows
   int taps;          // CC * R * S
   int n_stages;      // ceil(C / CC)
   int halo_words;    // CC * HR * GW * WSP
-  int code_words;    // taps * NT
-  int run;           // taps per decode item
-  int threads;       // TH * GW * CG
+  int code_words;    // taps * 2 * NT
+  int run;           // taps per decode item (blob path)
   int tiles_w, tiles_h;
 };
 
@@ -46,6 +45,11 @@ __device__ __forceinline__ void cp_async4(void* smem_dst, const void* gsrc, bool
   const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
   const int n = valid ? 4 : 0;
   asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(d), "l"(gsrc), "r"(n));
+}
+__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gsrc, bool valid) {
+  const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
+  const int n = valid ? 16 : 0;
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(gsrc), "r"(n));
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::); }
@@ -58,38 +62,66 @@ __device__ __forceinline__ uint32_t uabs(int32_t v) {
   return v < 0 ? (uint32_t)0 - (uint32_t)v : (uint32_t)v;
 }
 
-// Stage the group windows of input channels [c0, c0 + CC): one warp per
-// (channel, halo row), lanes over (group, offset).  Zero outside the image
+template <int SIG, int S, int TM>
+struct Win {
+  static constexpr int WS = (TM - 1) * SIG + S;  // window values
+  static constexpr int WSP = (WS + 3) / 4 * 4;   // slot words
+  static constexpr int WV = WSP / 4;             // 16-byte loads per window
+};
+
+// Stage the group windows of input channels [c0, c0 + CC): one slot
+// (channel, halo row, group) per thread at a time; zero outside the image
 // and for channels >= C.
 template <int SIG, int S, int TM>
 __device__ __forceinline__ void stage_halo(const GemmParams& P, const DirectGeom G, int32_t* halo,
                                            int64_t img_base, int ih0, int iw0, int c0) {
-  constexpr int WS = (TM - 1) * SIG + S;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int nwarps = G.threads >> 5;
+  using WN = Win<SIG, S, TM>;
   const int64_t HW = (int64_t)P.H * P.W;
-  const int per_row = G.GW * WS;
-  for (int row = warp; row < G.CC * G.HR; row += nwarps) {
+  const int nslots = G.CC * G.HR * G.GW;
+  for (int sl = threadIdx.x; sl < nslots; sl += kThreads) {
+    const int row = sl / G.GW;          // (channel, halo row)
+    const int g = sl - row * G.GW;
     const int cl = row / G.HR;
     const int hr = row - cl * G.HR;
     const int c = c0 + cl;
     const int ih = ih0 + hr;
+    const int iws = iw0 + g * TM * SIG;
+    int32_t* dst = halo + sl * WN::WSP;
     const bool row_ok = (c < P.C) && ((unsigned)ih < (unsigned)P.H);
-    const int32_t* src_row = P.x + img_base + (int64_t)c * HW + (int64_t)ih * P.W;
-    int32_t* dst_row = halo + row * (G.GW * G.WSP);
-    for (int e = lane; e < per_row; e += 32) {
-      const int g = e / WS;
-      const int i = e - g * WS;
-      const int iw = iw0 + g * TM * SIG + i;
-      const bool ok = row_ok && ((unsigned)iw < (unsigned)P.W);
-      cp_async4(dst_row + g * G.WSP + i, ok ? (const void*)(src_row + iw) : (const void*)P.x, ok);
+    const int32_t* src = P.x + img_base + (int64_t)c * HW + (int64_t)ih * P.W + iws;
+    if (row_ok && iws >= 0 && iws + WN::WS <= P.W) {
+#pragma unroll
+      for (int i = 0; i < WN::WS; ++i) cp_async4(dst + i, src + i, true);
+    } else {
+#pragma unroll
+      for (int i = 0; i < WN::WS; ++i) {
+        const bool ok = row_ok && ((unsigned)(iws + i) < (unsigned)P.W);
+        cp_async4(dst + i, ok ? (const void*)(src + i) : (const void*)P.x, ok);
+      }
     }
   }
 }
 
-// Decode the codes of taps [kb, kb + taps) of the CTA's NT channels into shift
-// / sign words.  Work item = (channel, run of G.run <= 16 taps); the host
-// picks the run so that a thread owns at most one item.
+// Codes of taps [kb, kb + taps) of the CTA's NT channels.  Shared-memory row
+// per tap: NT/32 blocks of 64 words (32 shifts, then 32 signs).
+template <int NT>
+__device__ __forceinline__ void stage_codes_expanded(const GemmParams& P, const DirectGeom G, int32_t* code,
+                                                     int64_t col0, int64_t kb) {
+  constexpr int NB = NT / 32;
+  const int64_t nblocks = (P.cols + 31) / 32;
+  const int per_block = G.taps * 16;  // 16-byte pieces per block
+#pragma unroll
+  for (int b = 0; b < NB; ++b) {
+    const int64_t cb = col0 / 32 + b;
+    for (int e = threadIdx.x; e < per_block; e += kThreads) {
+      const int tap = e >> 4, q = e & 15;
+      const bool ok = (cb < nblocks) && (kb + tap < P.kred);
+      const int32_t* src = ok ? P.xcodes + ((cb * P.kred + kb + tap) * 64 + q * 4) : P.xcodes;
+      cp_async16(code + (tap * NB + b) * 64 + q * 4, src, ok);
+    }
+  }
+}
+
 __device__ __forceinline__ uint32_t nib_word(const GemmParams& P, int64_t col, int64_t k) {
   const int64_t rec = (k >> 5) * P.cols + col;
   return __ldg(reinterpret_cast<const uint32_t*>(P.blob + P.off_nib + rec * 16) + ((k >> 3) & 3));
@@ -99,13 +131,15 @@ __device__ __forceinline__ uint2 bit_words(const GemmParams& P, int64_t col, int
   return __ldg(reinterpret_cast<const uint2*>(P.blob + P.off_bits + rec * 8));
 }
 
-__device__ __forceinline__ void decode_codes(const GemmParams& P, const DirectGeom G, int32_t* sh_s,
-                                             int32_t* sg_s, int64_t col0, int64_t kb) {
+template <int NT>
+__device__ __forceinline__ void decode_codes(const GemmParams& P, const DirectGeom G, int32_t* code,
+                                             int64_t col0, int64_t kb) {
+  constexpr int NB = NT / 32;
   const int item = threadIdx.x;
   const int runs = (G.taps + G.run - 1) / G.run;
-  if (item >= runs * G.NT) return;
-  const int n = item % G.NT;
-  const int tl0 = (item / G.NT) * G.run;
+  if (item >= runs * NT) return;
+  const int n = item % NT;
+  const int tl0 = (item / NT) * G.run;
   const int64_t col = col0 + n;
   const int64_t ks = kb + tl0;
   uint32_t lo = 0u, hi = 0u, neg = 0u, nz = 0u;
@@ -125,6 +159,7 @@ __device__ __forceinline__ void decode_codes(const GemmParams& P, const DirectGe
   }
   const int nvalid_k = (int)((P.kred - ks) < 16 ? (P.kred - ks) : 16);
   const int nloc = (G.taps - tl0) < G.run ? (G.taps - tl0) : G.run;
+  int32_t* base = code + (n >> 5) * 64 + (n & 31);
 #pragma unroll
   for (int i = 0; i < 16; ++i) {
     if (i < nloc) {
@@ -132,31 +167,29 @@ __device__ __forceinline__ void decode_codes(const GemmParams& P, const DirectGe
       const uint32_t w = i < 8 ? lo : hi;
       const int sh = valid ? (int)((w >> (4 * (i & 7))) & 15u) : 0;
       const int sg = valid ? (int)((nz >> i) & 1u) - 2 * (int)((neg >> i) & 1u) : 0;
-      sh_s[(tl0 + i) * G.NT + n] = sh;
-      sg_s[(tl0 + i) * G.NT + n] = sg;
+      base[(tl0 + i) * NB * 64] = sh;
+      base[(tl0 + i) * NB * 64 + 32] = sg;
     }
   }
 }
 
-// The hot loop over one stage.
-template <int SIG, int S, int TM, int I0, int NI, typename Acc>
-__device__ __forceinline__ void compute_stage(const DirectGeom G, const int32_t* halo, const int32_t* sh_s,
-                                              const int32_t* sg_s, int oh_l, int g, int cg,
-                                              Acc (&acc)[NI][TN]) {
+// The hot loop over one stage.  hp: this thread's window slot in channel 0
+// of the stage; cp: this thread's 4 channels in tap 0 of the stage.
+template <int SIG, int S, int TM, int NT, int I0, int NI, typename Acc>
+__device__ __forceinline__ void compute_stage(const DirectGeom G, const int32_t* hp, const int32_t* cp,
+                                              int rowstride, Acc (&acc)[NI][TN]) {
+  using WN = Win<SIG, S, TM>;
   constexpr int R = S;  // square kernels
-  constexpr int WS = (TM - 1) * SIG + S;
-  constexpr int WV = (WS + 3) / 4;
-  const int rowstride = G.GW * G.WSP;
-  const int32_t* hbase = halo + (oh_l * SIG) * rowstride + g * G.WSP;
-  const int32_t* shb = sh_s + cg * TN;
-  const int32_t* sgb = sg_s + cg * TN;
+  constexpr int TAPW = 2 * NT;  // words per tap row
+  const int cstride = G.HR * rowstride;
+#pragma unroll 1
   for (int cl = 0; cl < G.CC; ++cl) {
 #pragma unroll
     for (int r = 0; r < R; ++r) {
-      const int4* wp = reinterpret_cast<const int4*>(hbase + (cl * G.HR + r) * rowstride);
-      int w[4 * WV];
+      const int4* wp = reinterpret_cast<const int4*>(hp + r * rowstride);
+      int w[4 * WN::WV];
 #pragma unroll
-      for (int v = 0; v < WV; ++v) {
+      for (int v = 0; v < WN::WV; ++v) {
         const int4 t = wp[v];
         w[4 * v] = t.x;
         w[4 * v + 1] = t.y;
@@ -165,9 +198,8 @@ __device__ __forceinline__ void compute_stage(const DirectGeom G, const int32_t*
       }
 #pragma unroll
       for (int s = 0; s < S; ++s) {
-        const int tap = (cl * R + r) * S + s;
-        const int4 shv = *reinterpret_cast<const int4*>(shb + tap * G.NT);
-        const int4 sgv = *reinterpret_cast<const int4*>(sgb + tap * G.NT);
+        const int4 shv = *reinterpret_cast<const int4*>(cp + (r * S + s) * TAPW);
+        const int4 sgv = *reinterpret_cast<const int4*>(cp + (r * S + s) * TAPW + 32);
         const int sh[TN] = {shv.x, shv.y, shv.z, shv.w};
         const int sg[TN] = {sgv.x, sgv.y, sgv.z, sgv.w};
 #pragma unroll
@@ -185,24 +217,32 @@ __device__ __forceinline__ void compute_stage(const DirectGeom G, const int32_t*
         }
       }
     }
+    hp += cstride;
+    cp += R * S * TAPW;
   }
 }
 
-template <int SIG, int S, int TM, int I0, int NI, typename Acc>
+template <int SIG, int S, int TM, int NT, int I0, int NI, typename Acc>
 __device__ __forceinline__ void run_direct(const GemmParams& P, const DirectGeom G, unsigned char* smem,
                                            int n_img, int oh0, int ow0, int64_t col0,
                                            uint32_t& amax_local) {
+  using WN = Win<SIG, S, TM>;
+  constexpr int CG = NT / TN;
   const int t = threadIdx.x;
-  const int cg = t % G.CG;
-  const int pg = t / G.CG;
+  const int cg = t % CG;
+  const int pg = t / CG;
   const int g = pg % G.GW;
   const int oh_l = pg / G.GW;
   const int64_t img_base = (int64_t)n_img * P.C * P.H * P.W;
   const int ih0 = oh0 * SIG - P.ph;
   const int iw0 = ow0 * SIG - P.pw;
+  const int rowstride = G.GW * WN::WSP;
 
   int32_t* const halo_base = reinterpret_cast<int32_t*>(smem);
   int32_t* const code_base = halo_base + 2 * G.halo_words;
+  const int hoff = (oh_l * SIG) * rowstride + g * WN::WSP;
+  const int coff = (cg >> 3) * 64 + (cg & 7) * TN;
+  const bool expanded = P.xcodes != nullptr;
 
   Acc acc[NI][TN];
 #pragma unroll
@@ -212,29 +252,31 @@ __device__ __forceinline__ void run_direct(const GemmParams& P, const DirectGeom
 
   // Stage st reads buffers st % 2.  After the barrier of stage st every
   // thread has finished stage st - 1, so the other buffers are free: the
-  // halo copies of stage st + 1 are issued there and its codes decoded there
-  // after the compute; each thread waits for its own copies before the next
-  // barrier, which then makes all of stage st + 1 visible.
+  // copies of stage st + 1 are issued there (and, without the expanded
+  // layout, its codes decoded there after the compute); each thread waits
+  // for its own copies before the next barrier, which then makes all of
+  // stage st + 1 visible.
   const int64_t taps_per_c = (int64_t)S * S;
   stage_halo<SIG, S, TM>(P, G, halo_base, img_base, ih0, iw0, 0);
+  if (expanded) stage_codes_expanded<NT>(P, G, code_base, col0, 0);
   cp_async_commit();
-  decode_codes(P, G, code_base, code_base + G.code_words, col0, 0);
+  if (!expanded) decode_codes<NT>(P, G, code_base, col0, 0);
   cp_async_wait_all();
   for (int st = 0; st < G.n_stages; ++st) {
     const int b = st & 1;
     const bool more = st + 1 < G.n_stages;
+    const int64_t kb1 = (int64_t)(st + 1) * G.CC * taps_per_c;
     __syncthreads();
     if (more) {
       stage_halo<SIG, S, TM>(P, G, halo_base + (b ^ 1) * G.halo_words, img_base, ih0, iw0,
                              (st + 1) * G.CC);
+      if (expanded) stage_codes_expanded<NT>(P, G, code_base + (b ^ 1) * G.code_words, col0, kb1);
       cp_async_commit();
     }
-    const int32_t* cc = code_base + b * 2 * G.code_words;
-    compute_stage<SIG, S, TM, I0, NI, Acc>(G, halo_base + b * G.halo_words, cc, cc + G.code_words, oh_l,
-                                           g, cg, acc);
+    compute_stage<SIG, S, TM, NT, I0, NI, Acc>(G, halo_base + b * G.halo_words + hoff,
+                                               code_base + b * G.code_words + coff, rowstride, acc);
     if (more) {
-      int32_t* cn = code_base + (b ^ 1) * 2 * G.code_words;
-      decode_codes(P, G, cn, cn + G.code_words, col0, (int64_t)(st + 1) * G.CC * taps_per_c);
+      if (!expanded) decode_codes<NT>(P, G, code_base + (b ^ 1) * G.code_words, col0, kb1);
       cp_async_wait_all();
     }
   }
@@ -276,12 +318,12 @@ __device__ __forceinline__ void run_direct(const GemmParams& P, const DirectGeom
   }
 }
 
-__device__ __forceinline__ bool tile_int32_exact(const GemmParams& P, const DirectGeom G, int64_t col0) {
+__device__ __forceinline__ bool tile_int32_exact(const GemmParams& P, int NT, int64_t col0) {
   bool unsafe = false;
   const int t = threadIdx.x;
   if (P.amax_in == nullptr || (P.flags & DS_FORCE_INT64)) {
     unsafe = true;
-  } else if (t < G.NT) {
+  } else if (t < NT) {
     const int64_t col = col0 + t;
     if (col < P.cols) {
       const unsigned long long amax = *P.amax_in;
@@ -300,7 +342,7 @@ __device__ __forceinline__ bool tile_int32_exact(const GemmParams& P, const Dire
   return !__syncthreads_or(unsafe);
 }
 
-template <int SIG, int S, int TM>
+template <int SIG, int S, int TM, int NT>
 __global__ void __launch_bounds__(kThreads, 3) conv_direct_kernel(const GemmParams P, const DirectGeom G) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   int bx = blockIdx.x;
@@ -308,16 +350,16 @@ __global__ void __launch_bounds__(kThreads, 3) conv_direct_kernel(const GemmPara
   bx /= G.tiles_w;
   const int th = bx % G.tiles_h;
   const int n_img = bx / G.tiles_h;
-  const int64_t col0 = (int64_t)blockIdx.y * G.NT;
+  const int64_t col0 = (int64_t)blockIdx.y * NT;
   const int oh0 = th * G.TH, ow0 = tw * TM * G.GW;
 
   uint32_t amax_local = 0;
-  if (tile_int32_exact(P, G, col0)) {
-    run_direct<SIG, S, TM, 0, TM, uint32_t>(P, G, smem_raw, n_img, oh0, ow0, col0, amax_local);
+  if (tile_int32_exact(P, NT, col0)) {
+    run_direct<SIG, S, TM, NT, 0, TM, uint32_t>(P, G, smem_raw, n_img, oh0, ow0, col0, amax_local);
   } else {
     constexpr int H1 = TM / 2;
-    run_direct<SIG, S, TM, 0, H1, int64_t>(P, G, smem_raw, n_img, oh0, ow0, col0, amax_local);
-    run_direct<SIG, S, TM, H1, TM - H1, int64_t>(P, G, smem_raw, n_img, oh0, ow0, col0, amax_local);
+    run_direct<SIG, S, TM, NT, 0, H1, int64_t>(P, G, smem_raw, n_img, oh0, ow0, col0, amax_local);
+    run_direct<SIG, S, TM, NT, H1, TM - H1, int64_t>(P, G, smem_raw, n_img, oh0, ow0, col0, amax_local);
   }
   if (P.amax_out != nullptr) {
     amax_local = __reduce_max_sync(0xffffffffu, amax_local);
@@ -325,42 +367,45 @@ __global__ void __launch_bounds__(kThreads, 3) conv_direct_kernel(const GemmPara
   }
 }
 
+struct Choice {
+  DirectGeom G;
+  int TM, NT;
+};
+
 size_t direct_smem_bytes(const DirectGeom& G) {
-  return (size_t)2 * (G.halo_words + 2 * (size_t)G.code_words) * sizeof(int32_t);
+  return (size_t)2 * (G.halo_words + (size_t)G.code_words) * sizeof(int32_t);
 }
 
 // Tile choice.  TM = 7 when the output width is a multiple of 7 (every
 // ResNet / VGG feature map: 112, 56, 28, 14, 7), else 8.  Groups per row at
 // most 8; rows so that the CTA has 256 threads; 32 channels per CTA, or 64
 // when the pixel tile is too small for 256 threads with 8 channel groups.
-bool choose_geom(const GemmParams& p, int TM, DirectGeom& G) {
-  G.NT = 32;
-  G.CG = G.NT / TN;
-  int gw = (p.OW + TM - 1) / TM;
+bool choose_geom(const GemmParams& p, Choice& ch) {
+  DirectGeom& G = ch.G;
+  ch.TM = (p.OW % 7 == 0) ? 7 : 8;
+  const int WS = (ch.TM - 1) * p.sw + p.S;
+  const int WSP = (WS + 3) / 4 * 4;
+  ch.NT = 32;
+  int gw = (p.OW + ch.TM - 1) / ch.TM;
   if (gw > 8) {
     const int pieces = (gw + 7) / 8;
     gw = (gw + pieces - 1) / pieces;
   }
   G.GW = gw;
-  G.TH = kThreads / (G.GW * G.CG);
+  G.TH = kThreads / (G.GW * (ch.NT / TN));
   if (G.TH > p.OH) {
     // small image: widen the channel tile instead of idling threads
-    G.NT = 64;
-    G.CG = 16;
-    G.TH = kThreads / (G.GW * G.CG);
+    ch.NT = 64;
+    G.TH = kThreads / (G.GW * (ch.NT / TN));
     if (G.TH < 1 || G.TH > p.OH) return false;
   }
-  if (G.TH * G.GW * G.CG != kThreads) return false;
-  const int WS = (TM - 1) * p.sw + p.S;
-  G.WSP = (WS + 3) / 4 * 4;
+  if (G.TH * G.GW * (ch.NT / TN) != kThreads) return false;
   G.HR = (G.TH - 1) * p.sh + p.R;
-  G.threads = kThreads;
-  const int per_c_words = G.HR * G.GW * G.WSP + 2 * p.R * p.S * G.NT;
+  const int per_c_words = G.HR * G.GW * WSP + 2 * p.R * p.S * ch.NT;
   int cc = kSmemBudget / (2 * 4 * per_c_words);
   if (cc < 1) return false;
   if (cc > p.C) cc = p.C;
-  // prefer a chunk that divides C
-  for (int d = cc; d >= 1; --d)
+  for (int d = cc; d >= 1; --d)  // prefer a chunk that divides C
     if (p.C % d == 0 && 2 * d >= cc) {
       cc = d;
       break;
@@ -368,39 +413,41 @@ bool choose_geom(const GemmParams& p, int TM, DirectGeom& G) {
   G.CC = cc;
   G.taps = G.CC * p.R * p.S;
   G.n_stages = (p.C + G.CC - 1) / G.CC;
-  G.halo_words = G.CC * G.HR * G.GW * G.WSP;
-  G.code_words = G.taps * G.NT;
-  // decode run: smallest run with at most one item per thread
-  int run = (G.taps * G.NT + kThreads - 1) / kThreads;
+  G.halo_words = G.CC * G.HR * G.GW * WSP;
+  G.code_words = G.taps * 2 * ch.NT;
+  int run = (G.taps * ch.NT + kThreads - 1) / kThreads;  // decode: at most one item per thread
   if (run < 1) run = 1;
   if (run > 16) return false;
   G.run = run;
-  G.tiles_w = (p.OW + TM * G.GW - 1) / (TM * G.GW);
+  G.tiles_w = (p.OW + ch.TM * G.GW - 1) / (ch.TM * G.GW);
   G.tiles_h = (p.OH + G.TH - 1) / G.TH;
   return direct_smem_bytes(G) <= (size_t)kSmemBudget;
 }
 
-template <int SIG, int S, int TM>
+template <int SIG, int S, int TM, int NT>
 cudaError_t launch_direct(const GemmParams& p, const DirectGeom& G, cudaStream_t st) {
   const size_t smem = direct_smem_bytes(G);
-  cudaError_t e = cudaFuncSetAttribute(conv_direct_kernel<SIG, S, TM>,
+  cudaError_t e = cudaFuncSetAttribute(conv_direct_kernel<SIG, S, TM, NT>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   const int64_t n_img = p.rows / ((int64_t)p.OH * p.OW);
   const int64_t nb = (int64_t)G.tiles_w * G.tiles_h * n_img;
-  dim3 grid((unsigned)nb, (unsigned)((p.cols + G.NT - 1) / G.NT));
-  conv_direct_kernel<SIG, S, TM><<<grid, G.threads, smem, st>>>(p, G);
+  dim3 grid((unsigned)nb, (unsigned)((p.cols + NT - 1) / NT));
+  conv_direct_kernel<SIG, S, TM, NT><<<grid, kThreads, smem, st>>>(p, G);
   return cudaGetLastError();
 }
 
-template <int SIG, int TM>
+template <int SIG, int TM, int NT>
 cudaError_t launch_by_s(const GemmParams& p, const DirectGeom& G, cudaStream_t st) {
-  if (p.S == 1) return launch_direct<SIG, 1, TM>(p, G, st);
-  if (p.S == 3) return launch_direct<SIG, 3, TM>(p, G, st);
-  return launch_direct<SIG, 7, TM>(p, G, st);
+  if (p.S == 1) return launch_direct<SIG, 1, TM, NT>(p, G, st);
+  if (p.S == 3) return launch_direct<SIG, 3, TM, NT>(p, G, st);
+  return launch_direct<SIG, 7, TM, NT>(p, G, st);
 }
 
-int pick_tm(const GemmParams& p) { return (p.OW % 7 == 0) ? 7 : 8; }
+template <int SIG, int TM>
+cudaError_t launch_by_nt(const GemmParams& p, const Choice& ch, cudaStream_t st) {
+  return ch.NT == 32 ? launch_by_s<SIG, TM, 32>(p, ch.G, st) : launch_by_s<SIG, TM, 64>(p, ch.G, st);
+}
 
 }  // namespace
 
@@ -408,16 +455,15 @@ bool conv_direct_supported(const GemmParams& p) {
   if (p.sh != p.sw || !(p.sh == 1 || p.sh == 2)) return false;
   if (!(p.S == 1 || p.S == 3 || p.S == 7) || p.R != p.S) return false;
   if ((p.rows / ((int64_t)p.OH * p.OW)) >= ((int64_t)1 << 24)) return false;
-  DirectGeom G;
-  return choose_geom(p, pick_tm(p), G);
+  Choice ch;
+  return choose_geom(p, ch);
 }
 
 cudaError_t launch_conv2d_direct(const GemmParams& p, cudaStream_t st) {
-  DirectGeom G;
-  const int TM = pick_tm(p);
-  if (!choose_geom(p, TM, G)) return cudaErrorInvalidConfiguration;
-  if (TM == 7) return p.sh == 1 ? launch_by_s<1, 7>(p, G, st) : launch_by_s<2, 7>(p, G, st);
-  return p.sh == 1 ? launch_by_s<1, 8>(p, G, st) : launch_by_s<2, 8>(p, G, st);
+  Choice ch;
+  if (!choose_geom(p, ch)) return cudaErrorInvalidConfiguration;
+  if (ch.TM == 7) return p.sh == 1 ? launch_by_nt<1, 7>(p, ch, st) : launch_by_nt<2, 7>(p, ch, st);
+  return p.sh == 1 ? launch_by_nt<1, 8>(p, ch, st) : launch_by_nt<2, 8>(p, ch, st);
 }
 
 }  // namespace ds

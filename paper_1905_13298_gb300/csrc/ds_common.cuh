@@ -59,6 +59,7 @@ static_assert(sizeof(BlobHeader) == 48, "header layout");
 struct GemmParams {
   const int32_t* x;
   const uint8_t* blob;
+  const int32_t* xcodes;    // nullable: expanded layout [ceil(cols/32)][kred][64]
   const int32_t* bias;      // nullable
   const int32_t* residual;  // nullable (conv, DS_RESIDUAL)
   int32_t* y;
@@ -84,5 +85,10 @@ cudaError_t launch_conv2d_direct(const GemmParams& p, cudaStream_t st);
 cudaError_t launch_absmax(const int32_t* x, int64_t n, uint32_t* out, cudaStream_t st);
 cudaError_t launch_pack(const int8_t* s, const int8_t* p, int64_t n_out, int64_t k_red,
                         uint8_t* blob, cudaStream_t st);
+cudaError_t launch_expand(const uint8_t* blob, int64_t n_out, int64_t k_red, int32_t* out, cudaStream_t st);
+
+__host__ __device__ inline int64_t expanded_words(int64_t n_out, int64_t k_red) {
+  return ((n_out + 31) / 32) * k_red * 64;
+}
 
 }  // namespace ds

@@ -70,6 +70,43 @@ cudaError_t launch_pack(const int8_t* s, const int8_t* p, int64_t n_out, int64_t
   return cudaGetLastError();
 }
 
+// Expanded execution layout: out[cb][k][c] = -p (c < 32) or s (c >= 32) of
+// column 32*cb + (c & 31) at reduction index k; zero beyond n_out.
+__global__ void expand_kernel(const uint8_t* __restrict__ blob, int64_t n_out, int64_t k_red,
+                              int32_t* __restrict__ out) {
+  const BlobLayout L = blob_layout(n_out, k_red);
+  const int64_t total = ((n_out + 31) / 32) * k_red * 32;  // (cb, k, c32) triples
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const int c32 = (int)(e & 31);
+    const int64_t kc = e >> 5;  // cb * k_red + k
+    const int64_t cb = kc / k_red;
+    const int64_t k = kc - cb * k_red;
+    const int64_t col = cb * 32 + c32;
+    int32_t sh = 0, sg = 0;
+    if (col < n_out) {
+      const int64_t rec = (k >> 5) * n_out + col;
+      const uint32_t nib = reinterpret_cast<const uint32_t*>(blob + L.nib + rec * 16)[(k >> 3) & 3];
+      const uint2 b = reinterpret_cast<const uint2*>(blob + L.bits + rec * 8)[0];
+      const int j = (int)(k & 31);
+      sh = (int32_t)((nib >> (4 * (k & 7))) & 15u);
+      sg = (int32_t)((b.y >> j) & 1u) - 2 * (int32_t)((b.x >> j) & 1u);
+    }
+    int32_t* row = out + kc * 64;
+    row[c32] = sh;
+    row[32 + c32] = sg;
+  }
+}
+
+cudaError_t launch_expand(const uint8_t* blob, int64_t n_out, int64_t k_red, int32_t* out, cudaStream_t st) {
+  const int threads = 256;
+  const int64_t total = ((n_out + 31) / 32) * k_red * 32;
+  int64_t blocks = (total + threads - 1) / threads;
+  if (blocks > 65535 * 8) blocks = 65535 * 8;
+  expand_kernel<<<(unsigned)blocks, threads, 0, st>>>(blob, n_out, k_red, out);
+  return cudaGetLastError();
+}
+
 // max |x| (as u32, |INT32_MIN| = 2^31).  Grid-stride over 16-byte vectors,
 // warp reduction, one atomicMax per warp.  The target is zeroed first.
 __device__ __forceinline__ uint32_t uabs32(int32_t v) {

@@ -56,7 +56,7 @@ def test_packed_bytes_match_documented_layout(ds):
 
 
 def test_weights_struct_layout(ds):
-    assert ctypes.sizeof(ds.ds_weights) == 64
+    assert ctypes.sizeof(ds.ds_weights) == 80
     assert ds.ds_weights.packed.offset == 32
 
 

@@ -13,8 +13,8 @@ def _dev(a):
     return torch.from_numpy(np.ascontiguousarray(a)).cuda()
 
 
-def _run(ds, x, s, p, b, stride, pad, relu=False, residual=None, flags=0):
-    w = ds.pack_shift_weights(_dev(s), _dev(p))
+def _run(ds, x, s, p, b, stride, pad, relu=False, residual=None, flags=0, expand=False):
+    w = ds.pack_shift_weights(_dev(s), _dev(p), expand=expand)
     amax_io = torch.zeros(2, dtype=torch.int32, device="cuda")
     y = ds.conv2d_shift(_dev(x), w, s.shape[2:], _dev(b) if b is not None else None, stride, pad, relu=relu,
                         residual=_dev(residual) if residual is not None else None, amax_io=amax_io,
@@ -39,11 +39,12 @@ GEOMS = [
 
 @pytest.mark.parametrize("geom", GEOMS)
 @pytest.mark.parametrize("flags", [0, 16, 32, 48])  # direct / forced 64-bit / implicit GEMM / both
-def test_conv_bitexact(dslib, geom, flags):
+@pytest.mark.parametrize("expand", [False, True])
+def test_conv_bitexact(dslib, geom, flags, expand):
     N, C, H, W, K, R, S, st, pd = geom
     x, s, p, b = si.conv_layer(sum(geom) * 31 + flags, N, C, H, W, K, R, S, -(1 << 20), 1 << 20)
     want = O.conv2d_shift(x, s, p, b, (st, st), (pd, pd))
-    got, amax = _run(dslib, x, s, p, b, (st, st), (pd, pd), flags=flags)
+    got, amax = _run(dslib, x, s, p, b, (st, st), (pd, pd), flags=flags, expand=expand)
     assert np.array_equal(got, want)
     assert amax[1] == O.absmax(want)
 
@@ -89,23 +90,25 @@ def test_conv_network_layer_shapes(dslib, geom):
     N, C, H, W, K, R, S, st, pd = geom
     x, s, p, b = si.conv_layer(sum(geom) * 7, N, C, H, W, K, R, S, 0, 1 << 20)
     want = O.conv2d_shift(x, s, p, b, (st, st), (pd, pd), relu=True)
-    for flags in (0, 32):
-        got, _ = _run(dslib, x, s, p, b, (st, st), (pd, pd), relu=True, flags=flags)
-        assert np.array_equal(got, want), flags
+    for flags, expand in ((0, False), (0, True), (32, False), (16, True)):
+        got, _ = _run(dslib, x, s, p, b, (st, st), (pd, pd), relu=True, flags=flags, expand=expand)
+        assert np.array_equal(got, want), (flags, expand)
 
 
-def test_conv_config2_two_images_full(dslib):
+@pytest.mark.parametrize("expand", [False, True])
+def test_conv_config2_two_images_full(dslib, expand):
     """The ResNet18 conv2_x layer (64 -> 64, 56 x 56, 3x3/1/1) on two images, every output."""
     x, s, p, b = si.config2(N=2)
     want = O.conv2d_shift(x, s, p, b, (1, 1), (1, 1))
-    got, _ = _run(dslib, x, s, p, b, (1, 1), (1, 1))
+    got, _ = _run(dslib, x, s, p, b, (1, 1), (1, 1), expand=expand)
     assert np.array_equal(got, want)
 
 
-def test_conv_config2_full_batch_sampled(dslib):
-    """The full N = 32 launch; sampled outputs checked one by one (corners, edges, random)."""
+@pytest.mark.parametrize("expand", [False, True])
+def test_conv_config2_full_batch_sampled(dslib, expand):
+    """The full N = 32 launch (as timed by the benchmark); sampled outputs checked one by one."""
     x, s, p, b = si.config2()
-    got, _ = _run(dslib, x, s, p, b, (1, 1), (1, 1))
+    got, _ = _run(dslib, x, s, p, b, (1, 1), (1, 1), expand=expand)
     rng = np.random.default_rng(1)
     pts = [(0, 0, 0, 0), (31, 63, 55, 55), (5, 7, 0, 55), (17, 40, 55, 0)]
     pts += [tuple(int(v) for v in (rng.integers(32), rng.integers(64), rng.integers(56), rng.integers(56)))

@@ -32,6 +32,19 @@ def test_pack_blob_bitexact(dslib, n_out, k_red):
     assert w.desc.a_max == int(A.max()) and w.desc.nnz_max == int(nnz.max())
 
 
+@pytest.mark.parametrize("n_out,k_red", [(1, 1), (33, 31), (64, 576), (70, 100)])
+def test_expand_bitexact(dslib, n_out, k_red):
+    seed = n_out * 31 + k_red
+    s = si.sign_codes(seed, (n_out, k_red))
+    p = si.shift_codes_uniform(seed, (n_out, k_red))
+    w = dslib.pack_shift_weights(_dev(s), _dev(p), expand=True)
+    torch.cuda.synchronize()
+    want = O.expand_codes(s, p)
+    got = w.expanded.cpu().numpy().reshape(want.shape)
+    assert np.array_equal(got, want)
+    assert w.desc.expanded == w.expanded.data_ptr()
+
+
 def test_pack_rejects_bad_codes(dslib):
     s = np.ones((4, 10), np.int8)
     p = np.zeros((4, 10), np.int8)

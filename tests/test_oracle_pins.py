@@ -412,3 +412,17 @@ def test_pack_round_trip_and_sizes():
         assert np.array_equal(s2, s)
         # a zero code's shift is still stored
         assert np.array_equal(p2, p)
+
+
+def test_expand_layout_closed_form():
+    """Expanded layout: word c of row (cb, k) is -p of column 32 cb + c, word 32 + c its sign."""
+    s = np.array([[1, -1, 0], [0, 1, -1]])
+    p = np.array([[0, -15, -3], [-1, -2, -4]])
+    e = O.expand_codes(s, p)
+    assert e.shape == (1, 3, 64)
+    assert e[0, :, 0].tolist() == [0, 15, 3] and e[0, :, 1].tolist() == [1, 2, 4]
+    assert e[0, :, 32].tolist() == [1, -1, 0] and e[0, :, 33].tolist() == [0, 1, -1]
+    assert not e[0, :, 2:32].any() and not e[0, :, 34:].any()
+    s2 = np.ones((40, 2), np.int64)
+    e2 = O.expand_codes(s2, np.zeros_like(s2))
+    assert e2.shape == (2, 2, 64) and e2[1, :, 32:40].all() and not e2[1, :, 40:].any()
