@@ -225,6 +225,57 @@ ds_status ds_linear_shift_static_scratch(const int32_t* x, const ds_weights* w, 
                                          int32_t* y, int64_t M, int64_t K, int64_t N, uint32_t flags,
                                          void* stream);
 
+/* ---------------------------------------------------------------------------
+ * Chained forward (ResNet / VGG shaped networks of shift layers).
+ *
+ * A network is an array of ds_layer run in order on one stream.  Tensors
+ * live in numbered slots: slot 0 is the network input x, slot 1 the network
+ * output y, slots >= 2 are carved from the caller's workspace.  Activations
+ * are NCHW int32 Q16.16; an FC layer reads its input slot as [batch][C*H*W].
+ * The ops are the paper's operators (Eq. 3: DS_OP_CONV, DS_OP_FC with the
+ * fused bias / saturation / residual / ReLU epilogue) plus the integer pools
+ * that ResNet and VGG need (DS_OP_MAXPOOL: max over the window, padded taps
+ * ignored; DS_OP_AVGPOOL: floor(sum / (R*S)), no padding).  Each shift layer
+ * proves its accumulator width on the device from the max|x| that its
+ * producer wrote (the network input gets one pre-pass), so the whole forward
+ * runs without a host round trip and can be captured in a CUDA graph.
+ * ------------------------------------------------------------------------- */
+#define DS_OP_CONV 1
+#define DS_OP_FC 2
+#define DS_OP_MAXPOOL 3
+#define DS_OP_AVGPOOL 4
+
+typedef struct ds_layer {
+  int32_t op;          /* DS_OP_* */
+  int32_t in;          /* input slot */
+  int32_t aux;         /* residual slot (DS_RESIDUAL), else -1 */
+  int32_t out;         /* output slot (not 0; distinct from in and aux) */
+  int32_t C, H, W;     /* input channels and spatial size, per image */
+  int32_t K;           /* conv / FC: output channels or features (pools: ignored) */
+  int32_t R, S;        /* conv / pool window */
+  int32_t stride, pad; /* conv / pool */
+  uint32_t flags;      /* DS_RELU, DS_RESIDUAL (conv only) */
+  const ds_weights* w; /* conv / FC weights (n_out = K, k_red = C*R*S or C*H*W) */
+  const int32_t* bias; /* conv / FC bias (device int32 [K]) or NULL */
+} ds_layer;
+
+/*
+ * Workspace bytes for running n layers at the given batch (0 if invalid):
+ * every slot >= 2 sized for the largest tensor written to it, plus the
+ * max|x| words.  Validates the program like ds_shift_forward.
+ */
+size_t ds_shift_forward_workspace_bytes(const ds_layer* layers, int n, int batch);
+
+/*
+ * Runs the program: x = slot 0 (device, [batch][C0][H0][W0] of layer 0),
+ * y = slot 1 (device, the tensor of the last layer that writes slot 1),
+ * ws = workspace (device, 256-byte aligned, >= the bytes above).
+ * Validation errors (DS_ERR_SHAPE, DS_ERR_INVALID_ARG, ...) are reported
+ * before anything is launched.  Asynchronous, stream-ordered, no allocation.
+ */
+ds_status ds_shift_forward(const ds_layer* layers, int n, const int32_t* x, int32_t* y, void* ws,
+                           size_t ws_bytes, int batch, void* stream);
+
 /*
  * max |x| over n int32 values, written to *amax (device u32; |INT32_MIN| = 2^31).
  */

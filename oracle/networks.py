@@ -1,0 +1,93 @@
+"""CPU oracle of chained DeepShift forwards.  TEST INFRASTRUCTURE ONLY.
+
+Every conv and FC layer of the network is a shift layer (Eq. 3 with the
+Sec. 4 fixed point; DeepShift converts all layers, including the first and the
+last), composed with the integer pools of ``deepshift_oracle``.  BatchNorm is
+omitted (reading R-bn: it is not a shift op and the codes are synthetic).
+The architectures follow the standard definitions that the paper evaluates:
+
+* ResNet18 / ResNet50 (He et al.): 7x7/2 stem conv + ReLU, 3x3/2 max-pool
+  (pad 1), four stages of basic (18) or bottleneck (50) blocks, floor
+  average pool over the final 7x7 map, FC to 1000.  A block computes
+  ReLU(sat32(main + shortcut)); the shortcut is the identity or a 1x1 conv
+  with the block's stride (no ReLU); in bottleneck blocks the stride sits on
+  the 3x3 conv.
+* VGG16 (Simonyan and Zisserman): thirteen 3x3/1/1 convs + ReLU with 2x2/2
+  max-pools, then FC 25088 -> 4096 -> 4096 (ReLU) -> 1000.
+
+Parameter order (``params`` is a list of (s, p, b) per shift layer):
+ResNet: stem; then per block conv1, conv2 (, conv3 for bottleneck) and the
+downsample conv if the block has one; then the FC.  VGG16: the 13 convs,
+then the 3 FCs.
+
+parity unpinned beyond composition: the chain is checked only through its
+pinned parts (conv, FC, pools, residual join) and one library special case
+(tests/test_oracle_pins.py::test_resnet_chain_matches_float64_library_case).
+"""
+from __future__ import annotations
+
+import numpy as np
+
+from . import deepshift_oracle as O
+
+RESNET_STAGES = {"resnet18": ("basic", [2, 2, 2, 2]), "resnet50": ("bottleneck", [3, 4, 6, 3])}
+VGG16_CFG = [64, 64, "M", 128, 128, "M", 256, 256, 256, "M", 512, 512, 512, "M", 512, 512, 512, "M"]
+
+
+def _conv(x, prm, stride, pad, relu, residual=None):
+    s, p, b = prm
+    y = O.conv2d_shift(x, s, p, b, (stride, stride), (pad, pad), relu=False)
+    if residual is not None:
+        return O.add_relu(y, residual)
+    return np.maximum(y, 0).astype(np.int32) if relu else y
+
+
+def resnet_forward(x, params, arch: str = "resnet18"):
+    """Forward of an all-shift ResNet; x int32 [N, 3, 224, 224]; returns int32 [N, 1000]."""
+    kind, blocks = RESNET_STAGES[arch]
+    it = iter(params)
+    x = _conv(x, next(it), 2, 3, relu=True)
+    x = O.maxpool2d(x, 3, 2, 1)
+    for stage, nb in enumerate(blocks):
+        for bi in range(nb):
+            stride = 2 if (stage > 0 and bi == 0) else 1
+            planes = 64 * (2 ** stage)
+            out_c = planes if kind == "basic" else planes * 4
+            need_ds = stride != 1 or x.shape[1] != out_c
+            if kind == "basic":
+                c1, c2 = next(it), next(it)
+                ds = next(it) if need_ds else None
+                t = _conv(x, c1, stride, 1, relu=True)
+                sc = _conv(x, ds, stride, 0, relu=False) if ds is not None else x
+                x = _conv(t, c2, 1, 1, relu=True, residual=sc)
+            else:
+                c1, c2, c3 = next(it), next(it), next(it)
+                ds = next(it) if need_ds else None
+                t = _conv(x, c1, 1, 0, relu=True)
+                t = _conv(t, c2, stride, 1, relu=True)
+                sc = _conv(x, ds, stride, 0, relu=False) if ds is not None else x
+                x = _conv(t, c3, 1, 0, relu=True, residual=sc)
+    k = x.shape[2]
+    x = O.avgpool_floor(x, k, k)
+    s, p, b = next(it)
+    y = O.linear_shift(x.reshape(x.shape[0], -1), s.reshape(s.shape[0], -1), p.reshape(p.shape[0], -1), b)
+    if next(it, None) is not None:
+        raise ValueError("unused parameters")
+    return y
+
+
+def vgg16_forward(x, params):
+    """Forward of an all-shift VGG16; x int32 [N, 3, 224, 224]; returns int32 [N, 1000]."""
+    it = iter(params)
+    for v in VGG16_CFG:
+        if v == "M":
+            x = O.maxpool2d(x, 2, 2, 0)
+        else:
+            x = _conv(x, next(it), 1, 1, relu=True)
+    x = x.reshape(x.shape[0], -1)
+    for i in range(3):
+        s, p, b = next(it)
+        x = O.linear_shift(x, s.reshape(s.shape[0], -1), p.reshape(p.shape[0], -1), b, relu=(i < 2))
+    if next(it, None) is not None:
+        raise ValueError("unused parameters")
+    return x

@@ -35,6 +35,11 @@ DS_RESIDUAL = 8
 DS_FORCE_INT64 = 16
 DS_CONV_IM2COL = 32
 
+DS_OP_CONV = 1
+DS_OP_FC = 2
+DS_OP_MAXPOOL = 3
+DS_OP_AVGPOOL = 4
+
 DS_WEIGHTS_MAGIC = 0x31575344
 DS_FORMAT_PLANES6 = 1
 
@@ -51,6 +56,13 @@ class ds_weights(ctypes.Structure):
                 ("packed", ctypes.c_void_p), ("packed_bytes", ctypes.c_size_t),
                 ("a_max", ctypes.c_uint64), ("nnz_max", ctypes.c_uint32), ("reserved", ctypes.c_uint32),
                 ("expanded", ctypes.c_void_p), ("expanded_bytes", ctypes.c_size_t)]
+
+
+class ds_layer(ctypes.Structure):
+    _fields_ = [("op", ctypes.c_int32), ("in_", ctypes.c_int32), ("aux", ctypes.c_int32), ("out", ctypes.c_int32),
+                ("C", ctypes.c_int32), ("H", ctypes.c_int32), ("W", ctypes.c_int32), ("K", ctypes.c_int32),
+                ("R", ctypes.c_int32), ("S", ctypes.c_int32), ("stride", ctypes.c_int32), ("pad", ctypes.c_int32),
+                ("flags", ctypes.c_uint32), ("w", ctypes.POINTER(ds_weights)), ("bias", ctypes.c_void_p)]
 
 
 _lib = None
@@ -75,6 +87,9 @@ _SIGNATURES = {
     "ds_expanded_weight_bytes": (ctypes.c_size_t, [ctypes.c_int64, ctypes.c_int64]),
     "ds_expand_shift_weights": (ctypes.c_int, [ctypes.POINTER(ds_weights), ctypes.c_void_p, ctypes.c_size_t,
                                                ctypes.c_void_p]),
+    "ds_shift_forward_workspace_bytes": (ctypes.c_size_t, [ctypes.POINTER(ds_layer), ctypes.c_int, ctypes.c_int]),
+    "ds_shift_forward": (ctypes.c_int, [ctypes.POINTER(ds_layer), ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p,
+                                        ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int, ctypes.c_void_p]),
     "ds_absmax": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]),
 }
 
@@ -160,6 +175,14 @@ def ds_linear_shift_static_scratch(x, w: ds_weights, bias, y, M: int, K: int, N:
     """ds_linear_shift with its scratch in the library's static device array (no allocation)."""
     _check(lib().ds_linear_shift_static_scratch(_ptr(x), ctypes.byref(w), _ptr(bias), _ptr(y), M, K, N, flags,
                                                 _stream(stream)))
+
+
+def ds_shift_forward_workspace_bytes(layers, n: int, batch: int) -> int:
+    return int(lib().ds_shift_forward_workspace_bytes(layers, n, batch))
+
+
+def ds_shift_forward(layers, n: int, x, y, ws, ws_bytes: int, batch: int, stream=None) -> None:
+    _check(lib().ds_shift_forward(layers, n, _ptr(x), _ptr(y), _ptr(ws), ws_bytes, batch, _stream(stream)))
 
 
 def ds_absmax(x, n: int, amax, stream=None) -> None:

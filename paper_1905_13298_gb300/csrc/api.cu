@@ -40,7 +40,7 @@ ds_status cuda_check(cudaError_t e, const char* what) {
 static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
 // Checks a descriptor filled by ds_pack_shift_weights against the call's dims.
-static ds_status check_weights(const ds_weights* w, int64_t n_out, int64_t k_red) {
+ds_status check_weights(const ds_weights* w, int64_t n_out, int64_t k_red) {
   if (w == nullptr) return fail(DS_ERR_INVALID_ARG, "weights descriptor is NULL");
   if (w->magic != DS_WEIGHTS_MAGIC || w->format != DS_FORMAT_PLANES6)
     return fail(DS_ERR_INVALID_ARG, "weights descriptor was not filled by ds_pack_shift_weights");
@@ -88,6 +88,55 @@ static ds_status prepare_amax(const int32_t* x, int64_t nx, uint32_t flags, uint
     p.amax_out = amax_io + 1;
   }
   return DS_OK;
+}
+
+ds_status conv_launch(const int32_t* x, const ds_weights* w, const int32_t* bias, const int32_t* residual,
+                      int32_t* y, int N, int C, int H, int W, int K, int R, int S, int stride, int pad,
+                      uint32_t flags, const uint32_t* amax_in, uint32_t* amax_out, cudaStream_t st) {
+  GemmParams p{};
+  p.x = x;
+  p.bias = bias;
+  p.residual = (flags & DS_RESIDUAL) ? residual : nullptr;
+  p.y = y;
+  p.OH = (H + 2 * pad - R) / stride + 1;
+  p.OW = (W + 2 * pad - S) / stride + 1;
+  p.rows = (int64_t)N * p.OH * p.OW;
+  p.kred = (int64_t)C * R * S;
+  p.cols = K;
+  p.flags = flags;
+  p.C = C;
+  p.H = H;
+  p.W = W;
+  p.R = R;
+  p.S = S;
+  p.sh = stride;
+  p.sw = stride;
+  p.ph = pad;
+  p.pw = pad;
+  fill_blob_offsets(p, w);
+  p.amax_in = amax_in;
+  p.amax_out = amax_out;
+  if (!(flags & DS_CONV_IM2COL) && conv_direct_supported(p))
+    return cuda_check(launch_conv2d_direct(p, st), "conv2d_shift (direct) launch");
+  return cuda_check(launch_conv2d_shift(p, st), "conv2d_shift (implicit GEMM) launch");
+}
+
+ds_status fc_launch(const int32_t* x, const ds_weights* w, const int32_t* bias, int32_t* y, int64_t M,
+                    int64_t K, int64_t N, uint32_t flags, const uint32_t* amax_in, uint32_t* amax_out,
+                    cudaStream_t st) {
+  GemmParams p{};
+  p.x = x;
+  p.bias = bias;
+  p.residual = nullptr;
+  p.y = y;
+  p.rows = M;
+  p.kred = K;
+  p.cols = N;
+  p.flags = flags;
+  fill_blob_offsets(p, w);
+  p.amax_in = amax_in;
+  p.amax_out = amax_out;
+  return cuda_check(launch_linear_shift(p, st), "linear_shift launch");
 }
 
 constexpr uint32_t kKnownFlags =

@@ -1,0 +1,73 @@
+// Integer pooling for the chained forward of ResNet / VGG shaped networks.
+// Max-pool ignores padded taps; average pool is floor(sum / (R*S)) over a
+// window without padding (floor division, also for negative sums).
+#include "ds_common.cuh"
+
+namespace ds {
+
+__global__ void maxpool_kernel(const int32_t* __restrict__ x, int32_t* __restrict__ y, int64_t planes,
+                               int H, int W, int OH, int OW, int R, int S, int stride, int pad) {
+  const int64_t total = planes * OH * OW;
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const int ow = (int)(e % OW);
+    const int64_t t = e / OW;
+    const int oh = (int)(t % OH);
+    const int64_t pl = t / OH;
+    const int32_t* xp = x + pl * H * W;
+    int32_t m = INT32_MIN;
+    for (int r = 0; r < R; ++r) {
+      const int ih = oh * stride - pad + r;
+      if ((unsigned)ih >= (unsigned)H) continue;
+      for (int s = 0; s < S; ++s) {
+        const int iw = ow * stride - pad + s;
+        if ((unsigned)iw >= (unsigned)W) continue;
+        m = max(m, __ldg(xp + (int64_t)ih * W + iw));
+      }
+    }
+    y[e] = m;
+  }
+}
+
+__global__ void avgpool_floor_kernel(const int32_t* __restrict__ x, int32_t* __restrict__ y, int64_t planes,
+                                     int H, int W, int OH, int OW, int R, int S, int stride) {
+  const int64_t total = planes * OH * OW;
+  const int64_t d = (int64_t)R * S;
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const int ow = (int)(e % OW);
+    const int64_t t = e / OW;
+    const int oh = (int)(t % OH);
+    const int64_t pl = t / OH;
+    const int32_t* xp = x + pl * H * W + (int64_t)oh * stride * W + (int64_t)ow * stride;
+    int64_t sum = 0;
+    for (int r = 0; r < R; ++r)
+      for (int s = 0; s < S; ++s) sum += __ldg(xp + (int64_t)r * W + s);
+    int64_t q = sum / d;
+    if (sum % d != 0 && sum < 0) --q;  // floor
+    y[e] = (int32_t)q;
+  }
+}
+
+static int64_t pool_blocks(int64_t total, int threads) {
+  int64_t b = (total + threads - 1) / threads;
+  return b > 152 * 32 ? 152 * 32 : (b < 1 ? 1 : b);
+}
+
+cudaError_t launch_maxpool(const int32_t* x, int32_t* y, int64_t planes, int H, int W, int OH, int OW, int R,
+                           int S, int stride, int pad, cudaStream_t st) {
+  const int threads = 256;
+  maxpool_kernel<<<(unsigned)pool_blocks(planes * OH * OW, threads), threads, 0, st>>>(x, y, planes, H, W, OH, OW,
+                                                                                       R, S, stride, pad);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_avgpool_floor(const int32_t* x, int32_t* y, int64_t planes, int H, int W, int OH, int OW,
+                                 int R, int S, int stride, cudaStream_t st) {
+  const int threads = 256;
+  avgpool_floor_kernel<<<(unsigned)pool_blocks(planes * OH * OW, threads), threads, 0, st>>>(
+      x, y, planes, H, W, OH, OW, R, S, stride);
+  return cudaGetLastError();
+}
+
+}  // namespace ds

@@ -81,6 +81,19 @@ cudaError_t launch_conv2d_shift(const GemmParams& p, cudaStream_t st);
 // Defined in conv_direct.cu.
 bool conv_direct_supported(const GemmParams& p);
 cudaError_t launch_conv2d_direct(const GemmParams& p, cudaStream_t st);
+// Defined in chain_ops.cu.
+cudaError_t launch_maxpool(const int32_t* x, int32_t* y, int64_t planes, int H, int W, int OH, int OW, int R,
+                           int S, int stride, int pad, cudaStream_t st);
+cudaError_t launch_avgpool_floor(const int32_t* x, int32_t* y, int64_t planes, int H, int W, int OH, int OW,
+                                 int R, int S, int stride, cudaStream_t st);
+// Defined in api.cu: launches after validation, with explicit amax slots.
+ds_status check_weights(const ds_weights* w, int64_t n_out, int64_t k_red);
+ds_status conv_launch(const int32_t* x, const ds_weights* w, const int32_t* bias, const int32_t* residual,
+                      int32_t* y, int N, int C, int H, int W, int K, int R, int S, int stride, int pad,
+                      uint32_t flags, const uint32_t* amax_in, uint32_t* amax_out, cudaStream_t st);
+ds_status fc_launch(const int32_t* x, const ds_weights* w, const int32_t* bias, int32_t* y, int64_t M,
+                    int64_t K, int64_t N, uint32_t flags, const uint32_t* amax_in, uint32_t* amax_out,
+                    cudaStream_t st);
 // Defined in misc_kernels.cu.
 cudaError_t launch_absmax(const int32_t* x, int64_t n, uint32_t* out, cudaStream_t st);
 cudaError_t launch_pack(const int8_t* s, const int8_t* p, int64_t n_out, int64_t k_red,

@@ -1,0 +1,196 @@
+// Chained forward: runs a program of shift layers and integer pools on one
+// stream (ResNet / VGG shaped networks built from the operators of Eq. 3).
+//
+// Host side: one validation pass computes every slot's shape, the workspace
+// layout and the device max|x| word that bounds each layer's input.  Device
+// side: one memset of the max|x| words, one max|x| pre-pass over the network
+// input, then one launch per layer.  A shift layer reads the max|x| word of
+// its producer (pools pass their input's bound through, since max-pool and
+// floor-average never exceed it) and writes max|y| into its own word, so the
+// accumulator-width proof of every layer happens on the device.
+#include <algorithm>
+#include <vector>
+
+#include "ds_common.cuh"
+
+namespace ds {
+namespace {
+
+struct Shape {
+  int C = 0, H = 0, W = 0;
+  int64_t elems() const { return (int64_t)C * H * W; }
+};
+
+struct Plan {
+  std::vector<Shape> out_shape;   // per layer
+  std::vector<int64_t> slot_elems;  // per slot, per image (slots >= 2)
+  std::vector<size_t> slot_off;   // byte offsets in the workspace
+  size_t amax_bytes = 0;
+  size_t total = 0;
+  int n_slots = 0;
+};
+
+ds_status plan_program(const ds_layer* L, int n, int batch, Plan& P) {
+  if (L == nullptr || n <= 0) return fail(DS_ERR_INVALID_ARG, "empty layer program");
+  if (batch <= 0) return fail(DS_ERR_SHAPE, "batch must be positive");
+  int max_slot = 1;
+  for (int i = 0; i < n; ++i) {
+    if (L[i].in < 0 || L[i].out < 1 || L[i].aux < -1)
+      return fail(DS_ERR_INVALID_ARG, "layer %d: bad slot numbers", i);
+    max_slot = std::max(max_slot, std::max(L[i].in, std::max(L[i].out, L[i].aux)));
+  }
+  if (max_slot > 64) return fail(DS_ERR_UNSUPPORTED, "at most 64 slots");
+  P.n_slots = max_slot + 1;
+  std::vector<Shape> slot(P.n_slots);
+  std::vector<bool> defined(P.n_slots, false);
+  P.slot_elems.assign(P.n_slots, 0);
+  P.out_shape.assign(n, Shape{});
+  slot[0] = Shape{L[0].C, L[0].H, L[0].W};
+  defined[0] = true;
+  bool wrote_y = false;
+  for (int i = 0; i < n; ++i) {
+    const ds_layer& l = L[i];
+    if (!defined[l.in]) return fail(DS_ERR_INVALID_ARG, "layer %d reads slot %d before it is written", i, l.in);
+    if (l.out == l.in || l.out == l.aux) return fail(DS_ERR_INVALID_ARG, "layer %d: output slot aliases an input", i);
+    const Shape in = slot[l.in];
+    Shape out;
+    switch (l.op) {
+      case DS_OP_CONV: {
+        if (in.C != l.C || in.H != l.H || in.W != l.W)
+          return fail(DS_ERR_SHAPE, "layer %d: input %dx%dx%d, slot holds %dx%dx%d", i, l.C, l.H, l.W, in.C,
+                      in.H, in.W);
+        if (l.K <= 0 || l.R <= 0 || l.S <= 0 || l.stride <= 0 || l.pad < 0)
+          return fail(DS_ERR_SHAPE, "layer %d: bad conv geometry", i);
+        if (l.H + 2 * l.pad < l.R || l.W + 2 * l.pad < l.S) return fail(DS_ERR_SHAPE, "layer %d: kernel too big", i);
+        ds_status r = check_weights(l.w, l.K, (int64_t)l.C * l.R * l.S);
+        if (r != DS_OK) return r;
+        out = Shape{l.K, (l.H + 2 * l.pad - l.R) / l.stride + 1, (l.W + 2 * l.pad - l.S) / l.stride + 1};
+        break;
+      }
+      case DS_OP_FC: {
+        if (in.elems() != (int64_t)l.C * l.H * l.W)
+          return fail(DS_ERR_SHAPE, "layer %d: FC input of %lld features, slot holds %lld", i,
+                      (long long)((int64_t)l.C * l.H * l.W), (long long)in.elems());
+        if (l.K <= 0) return fail(DS_ERR_SHAPE, "layer %d: bad FC width", i);
+        if (l.flags & DS_RESIDUAL) return fail(DS_ERR_INVALID_ARG, "layer %d: residual on FC", i);
+        ds_status r = check_weights(l.w, l.K, in.elems());
+        if (r != DS_OK) return r;
+        out = Shape{l.K, 1, 1};
+        break;
+      }
+      case DS_OP_MAXPOOL:
+      case DS_OP_AVGPOOL: {
+        if (in.C != l.C || in.H != l.H || in.W != l.W) return fail(DS_ERR_SHAPE, "layer %d: pool input shape", i);
+        const int pad = l.op == DS_OP_MAXPOOL ? l.pad : 0;
+        if (l.op == DS_OP_AVGPOOL && l.pad != 0) return fail(DS_ERR_UNSUPPORTED, "layer %d: padded avgpool", i);
+        if (l.R <= 0 || l.S <= 0 || l.stride <= 0 || pad < 0 || pad >= l.R || pad >= l.S)
+          return fail(DS_ERR_SHAPE, "layer %d: bad pool geometry", i);
+        if (l.H + 2 * pad < l.R || l.W + 2 * pad < l.S) return fail(DS_ERR_SHAPE, "layer %d: window too big", i);
+        if (l.flags != 0) return fail(DS_ERR_INVALID_ARG, "layer %d: flags on a pool", i);
+        out = Shape{l.C, (l.H + 2 * pad - l.R) / l.stride + 1, (l.W + 2 * pad - l.S) / l.stride + 1};
+        break;
+      }
+      default:
+        return fail(DS_ERR_INVALID_ARG, "layer %d: unknown op %d", i, l.op);
+    }
+    if (l.flags & ~(DS_RELU | DS_RESIDUAL)) return fail(DS_ERR_INVALID_ARG, "layer %d: unsupported flags", i);
+    if (l.flags & DS_RESIDUAL) {
+      if (l.aux < 0 || !defined[l.aux]) return fail(DS_ERR_INVALID_ARG, "layer %d: residual slot not written", i);
+      const Shape a = slot[l.aux];
+      if (a.C != out.C || a.H != out.H || a.W != out.W)
+        return fail(DS_ERR_SHAPE, "layer %d: residual shape differs from the output", i);
+    }
+    P.out_shape[i] = out;
+    slot[l.out] = out;
+    defined[l.out] = true;
+    if (l.out == 1) wrote_y = true;
+    if (l.out >= 2) P.slot_elems[l.out] = std::max(P.slot_elems[l.out], out.elems());
+  }
+  if (!wrote_y) return fail(DS_ERR_INVALID_ARG, "no layer writes the output slot 1");
+  P.amax_bytes = ((size_t)(n + 1) * sizeof(uint32_t) + 255) / 256 * 256;
+  P.slot_off.assign(P.n_slots, 0);
+  size_t off = P.amax_bytes;
+  for (int s = 2; s < P.n_slots; ++s) {
+    P.slot_off[s] = off;
+    off += ((size_t)P.slot_elems[s] * batch * sizeof(int32_t) + 255) / 256 * 256;
+  }
+  P.total = off;
+  return DS_OK;
+}
+
+}  // namespace
+}  // namespace ds
+
+using namespace ds;
+
+extern "C" {
+
+size_t ds_shift_forward_workspace_bytes(const ds_layer* layers, int n, int batch) {
+  clear_error();
+  Plan P;
+  if (plan_program(layers, n, batch, P) != DS_OK) return 0;
+  return P.total;
+}
+
+ds_status ds_shift_forward(const ds_layer* L, int n, const int32_t* x, int32_t* y, void* ws, size_t ws_bytes,
+                           int batch, void* stream) {
+  clear_error();
+  if (!x || !y || !ws) return fail(DS_ERR_INVALID_ARG, "NULL x, y or workspace");
+  Plan P;
+  ds_status r = plan_program(L, n, batch, P);
+  if (r != DS_OK) return r;
+  if (ws_bytes < P.total)
+    return fail(DS_ERR_BUFFER_TOO_SMALL, "workspace has %zu bytes, needs %zu", ws_bytes, P.total);
+  if ((reinterpret_cast<uintptr_t>(ws) & 255) != 0) return fail(DS_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
+  if ((reinterpret_cast<uintptr_t>(x) & 15) != 0 || (reinterpret_cast<uintptr_t>(y) & 15) != 0)
+    return fail(DS_ERR_ALIGNMENT, "x and y must be 16-byte aligned");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  unsigned char* base = static_cast<unsigned char*>(ws);
+  uint32_t* amax = reinterpret_cast<uint32_t*>(base);
+  std::vector<int32_t*> slot_ptr(P.n_slots, nullptr);
+  std::vector<const uint32_t*> slot_amax(P.n_slots, nullptr);
+  slot_ptr[0] = const_cast<int32_t*>(x);
+  slot_ptr[1] = y;
+  for (int s = 2; s < P.n_slots; ++s) slot_ptr[s] = reinterpret_cast<int32_t*>(base + P.slot_off[s]);
+
+  r = cuda_check(cudaMemsetAsync(amax, 0, (size_t)(n + 1) * sizeof(uint32_t), st), "amax reset");
+  if (r != DS_OK) return r;
+  const Shape in0{L[0].C, L[0].H, L[0].W};
+  r = cuda_check(launch_absmax(x, in0.elems() * batch, amax + n, st), "input max|x| pre-pass");
+  if (r != DS_OK) return r;
+  slot_amax[0] = amax + n;
+
+  for (int i = 0; i < n; ++i) {
+    const ds_layer& l = L[i];
+    const int32_t* xin = slot_ptr[l.in];
+    int32_t* yout = slot_ptr[l.out];
+    switch (l.op) {
+      case DS_OP_CONV:
+        r = conv_launch(xin, l.w, l.bias, l.aux >= 0 ? slot_ptr[l.aux] : nullptr, yout, batch, l.C, l.H, l.W,
+                        l.K, l.R, l.S, l.stride, l.pad, l.flags, slot_amax[l.in], amax + i, st);
+        slot_amax[l.out] = amax + i;
+        break;
+      case DS_OP_FC:
+        r = fc_launch(xin, l.w, l.bias, yout, batch, (int64_t)l.C * l.H * l.W, l.K, l.flags & DS_RELU,
+                      slot_amax[l.in], amax + i, st);
+        slot_amax[l.out] = amax + i;
+        break;
+      case DS_OP_MAXPOOL:
+        r = cuda_check(launch_maxpool(xin, yout, (int64_t)batch * l.C, l.H, l.W, P.out_shape[i].H,
+                                      P.out_shape[i].W, l.R, l.S, l.stride, l.pad, st),
+                       "maxpool launch");
+        slot_amax[l.out] = slot_amax[l.in];
+        break;
+      default:
+        r = cuda_check(launch_avgpool_floor(xin, yout, (int64_t)batch * l.C, l.H, l.W, P.out_shape[i].H,
+                                            P.out_shape[i].W, l.R, l.S, l.stride, st),
+                       "avgpool launch");
+        slot_amax[l.out] = slot_amax[l.in];
+        break;
+    }
+    if (r != DS_OK) return r;
+  }
+  return DS_OK;
+}
+
+}  // extern "C"

@@ -121,11 +121,21 @@ __global__ void absmax_kernel(const int32_t* __restrict__ x, int64_t n, uint32_t
   if (vec) {
     const int64_t nv = n >> 2;
     const int4* xv = reinterpret_cast<const int4*>(x);
-    for (int64_t i = tid; i < nv; i += stride) {
-      int4 v = __ldg(xv + i);
-      m = max(m, max(max(uabs32(v.x), uabs32(v.y)), max(uabs32(v.z), uabs32(v.w))));
+    int64_t i = tid;
+    // four independent 16-byte loads in flight per thread
+    for (; i + 3 * stride < nv; i += 4 * stride) {
+      const int4 a = __ldg(xv + i), b = __ldg(xv + i + stride);
+      const int4 c = __ldg(xv + i + 2 * stride), d = __ldg(xv + i + 3 * stride);
+      m = max(m, max(max(uabs32(a.x), uabs32(a.y)), max(uabs32(a.z), uabs32(a.w))));
+      m = max(m, max(max(uabs32(b.x), uabs32(b.y)), max(uabs32(b.z), uabs32(b.w))));
+      m = max(m, max(max(uabs32(c.x), uabs32(c.y)), max(uabs32(c.z), uabs32(c.w))));
+      m = max(m, max(max(uabs32(d.x), uabs32(d.y)), max(uabs32(d.z), uabs32(d.w))));
     }
-    for (int64_t i = (nv << 2) + tid; i < n; i += stride) m = max(m, uabs32(x[i]));
+    for (; i < nv; i += stride) {
+      const int4 a = __ldg(xv + i);
+      m = max(m, max(max(uabs32(a.x), uabs32(a.y)), max(uabs32(a.z), uabs32(a.w))));
+    }
+    for (int64_t j = (nv << 2) + tid; j < n; j += stride) m = max(m, uabs32(x[j]));
   } else {
     for (int64_t i = tid; i < n; i += stride) m = max(m, uabs32(x[i]));
   }
@@ -140,8 +150,8 @@ cudaError_t launch_absmax(const int32_t* x, int64_t n, uint32_t* out, cudaStream
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const int threads = 256;
-  int64_t want = (n / 4 + threads - 1) / threads;
-  int64_t blocks = want < (int64_t)sms * 8 ? want : (int64_t)sms * 8;
+  int64_t want = (n / 16 + threads - 1) / threads;
+  int64_t blocks = want < (int64_t)sms * 4 ? want : (int64_t)sms * 4;
   if (blocks < 1) blocks = 1;
   absmax_kernel<<<(unsigned)blocks, threads, 0, st>>>(x, n, out);
   return cudaGetLastError();

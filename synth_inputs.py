@@ -196,3 +196,28 @@ def layer_centre(c_in: int, r: int, s: int) -> int:
     """Per-layer shift centre -round(log2(C*R*S)/2) - 4 that keeps a chain in range."""
     fan_in = c_in * r * s
     return -int(np.floor(0.5 * np.log2(fan_in) + 0.5)) - 4
+
+
+def network_params(shapes, seed: int):
+    """Codes and biases for every shift layer of a network, in the given order.
+
+    shapes: list of (K, C, R, S) for conv layers or (N, K) for FC layers.
+    Layer i uses seed + i; shifts are geometric around the per-layer centre
+    -round(log2(fan_in) / 2) - 4 (fan_in = C*R*S or K), which keeps chained
+    activations inside the int32 range; signs as in every config.
+    """
+    params = []
+    for i, shp in enumerate(shapes):
+        sd = seed + i
+        fan_in = int(np.prod(shp[1:]))
+        centre = -int(np.floor(0.5 * np.log2(fan_in) + 0.5)) - 4
+        s = sign_codes(sd, shp)
+        p = shift_codes_geometric(sd, shp, centre)
+        b = bias(sd, shp[0])
+        params.append((s, p, b))
+    return params
+
+
+def image_batch(seed: int, n: int, c: int = 3, h: int = 224, w: int = 224):
+    """Network input stand-in for ImageNet images: int32 uniform in [-2^17, 2^17) (signed, like normalised pixels)."""
+    return activations(seed, (n, c, h, w), -(1 << 17), 1 << 17)

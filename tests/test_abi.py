@@ -101,3 +101,37 @@ def test_no_cpu_fallback_without_library(tmp_path, monkeypatch, ds):
     monkeypatch.setattr(ds, "LIB_PATH", str(tmp_path / "missing.so"))
     with pytest.raises(ImportError):
         ds.lib()
+
+
+def test_forward_program_validation_without_gpu(ds):
+    """Programs are validated on the host: bad shapes and slots are rejected before anything runs."""
+    from paper_1905_13298_gb300 import networks as PN
+    specs, shapes = PN.resnet_program("resnet18")
+    ws = [ds.ds_weights(magic=ds.DS_WEIGHTS_MAGIC, format=ds.DS_FORMAT_PLANES6, n_out=shp[0],
+                        k_red=int(np.prod(shp[1:])), n_chunks=(int(np.prod(shp[1:])) + 31) // 32, packed=4096,
+                        packed_bytes=ds.ds_packed_weight_bytes(shp[0], int(np.prod(shp[1:]))))
+          for shp in shapes]
+    layers = (ds.ds_layer * len(specs))()
+    for i, sp in enumerate(specs):
+        L = layers[i]
+        L.op, L.in_, L.aux, L.out = sp.op, sp.inp, sp.aux, sp.out
+        L.C, L.H, L.W, L.K, L.R, L.S, L.stride, L.pad, L.flags = (sp.C, sp.H, sp.W, sp.K, sp.R, sp.S, sp.stride,
+                                                                  sp.pad, sp.flags)
+        if sp.param >= 0:
+            L.w = ctypes.pointer(ws[sp.param])
+    n = len(specs)
+    good = ds.ds_shift_forward_workspace_bytes(layers, n, 32)
+    # the largest slot is the stem output 64 x 112 x 112 per image
+    assert good >= 32 * 64 * 112 * 112 * 4
+    assert ds.ds_shift_forward_workspace_bytes(layers, n, 0) == 0
+    layers[3].C += 1                   # a conv whose input channels disagree with its producer
+    assert ds.ds_shift_forward_workspace_bytes(layers, n, 32) == 0
+    assert "input" in ds.ds_last_error()
+    layers[3].C -= 1
+    saved = layers[n - 1].out
+    layers[n - 1].out = 7              # nobody writes the output slot
+    assert ds.ds_shift_forward_workspace_bytes(layers, n, 32) == 0
+    layers[n - 1].out = saved
+    assert ds.ds_shift_forward_workspace_bytes(layers, n, 32) == good
+    L = ds.lib()
+    assert L.ds_shift_forward(layers, n, 16, 16, 256, good - 1, 32, None) == ds.DS_ERR_BUFFER_TOO_SMALL

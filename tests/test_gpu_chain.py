@@ -1,0 +1,65 @@
+"""GPU parity of the chained forward (ds_shift_forward) against the CPU oracle (bit-exact)."""
+import numpy as np
+import pytest
+import torch
+
+import synth_inputs as si
+from oracle import networks as ON
+
+pytestmark = pytest.mark.gpu
+
+
+def _run(program, params, x, expand=True):
+    from paper_1905_13298_gb300.networks import ShiftNetwork
+    specs, _ = program
+    net = ShiftNetwork(specs, params, batch=x.shape[0], expand=expand)
+    y = net.forward(torch.from_numpy(x).cuda())
+    torch.cuda.synchronize()
+    return y.cpu().numpy().reshape(x.shape[0], -1)
+
+
+@pytest.mark.parametrize("expand", [True, False])
+def test_resnet18_small_images(dslib, expand):
+    from paper_1905_13298_gb300 import networks as PN
+    prog = PN.resnet_program("resnet18", 64, 64)
+    params = si.network_params(prog[1], 100)
+    x = si.image_batch(7, 2, 3, 64, 64)
+    assert np.array_equal(_run(prog, params, x, expand), ON.resnet_forward(x, params, "resnet18"))
+
+
+def test_resnet50_small_image(dslib):
+    from paper_1905_13298_gb300 import networks as PN
+    prog = PN.resnet_program("resnet50", 64, 64)
+    params = si.network_params(prog[1], 200)
+    x = si.image_batch(8, 1, 3, 64, 64)
+    assert np.array_equal(_run(prog, params, x), ON.resnet_forward(x, params, "resnet50"))
+
+
+def test_vgg16_small_images(dslib):
+    from paper_1905_13298_gb300 import networks as PN
+    prog = PN.vgg16_program(32, 32)
+    params = si.network_params(prog[1], 300)
+    x = si.image_batch(9, 2, 3, 32, 32)
+    assert np.array_equal(_run(prog, params, x), ON.vgg16_forward(x, params))
+
+
+def test_resnet18_stress_codes_saturate_exactly(dslib):
+    """Codes centred at -6 in every layer (the stress law): activations saturate; results stay exact."""
+    from paper_1905_13298_gb300 import networks as PN
+    prog = PN.resnet_program("resnet18", 32, 32)
+    params = []
+    for i, shp in enumerate(prog[1]):
+        params.append((si.sign_codes(400 + i, shp), si.shift_codes_geometric(400 + i, shp, -6), si.bias(400 + i, shp[0])))
+    x = si.image_batch(10, 2, 3, 32, 32)
+    want = ON.resnet_forward(x, params, "resnet18")
+    assert (np.abs(want) == 2 ** 31 - 1).any() or (want == -(2 ** 31)).any()
+    assert np.array_equal(_run(prog, params, x), want)
+
+
+def test_resnet18_full_size_batch1(dslib):
+    """The ResNet18-architecture forward at 224 x 224, batch 1: every output."""
+    from paper_1905_13298_gb300 import networks as PN
+    prog = PN.resnet_program("resnet18")
+    params = si.network_params(prog[1], si.SEED_BASE + 3)
+    x = si.image_batch(si.SEED_BASE + 3, 1)
+    assert np.array_equal(_run(prog, params, x), ON.resnet_forward(x, params, "resnet18"))

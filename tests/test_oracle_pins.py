@@ -426,3 +426,67 @@ def test_expand_layout_closed_form():
     s2 = np.ones((40, 2), np.int64)
     e2 = O.expand_codes(s2, np.zeros_like(s2))
     assert e2.shape == (2, 2, 64) and e2[1, :, 32:40].all() and not e2[1, :, 40:].any()
+
+
+# --------------------------------------------------------------------------
+# Chained forward: the ResNet composition against float64 library routines
+# --------------------------------------------------------------------------
+
+def _one_hot_params(shapes, seed):
+    """p = 0 and exactly one non-zero sign per output channel: every term is exact, activations stay bounded."""
+    rng = np.random.default_rng(seed)
+    params = []
+    for shp in shapes:
+        K = shp[0]
+        fan = int(np.prod(shp[1:]))
+        s = np.zeros((K, fan), np.int64)
+        s[np.arange(K), rng.integers(0, fan, K)] = rng.choice([-1, 1], K)
+        params.append((s.reshape(shp), np.zeros(shp, np.int64), rng.integers(-(1 << 10), 1 << 10, K)))
+    return params
+
+
+def _torch_resnet(x, params, kind, blocks):
+    """float64 torch restatement (library conv2d / pools / linear) of the same ResNet topology."""
+    t = lambda a: torch.from_numpy(np.asarray(a, dtype=np.float64))
+    it = iter(params)
+
+    def conv(v, prm, stride, pad):
+        s, p, b = prm
+        return F.conv2d(v, t(s * np.ldexp(1.0, p)), t(b), stride=stride, padding=pad)
+
+    v = F.relu(conv(t(x), next(it), 2, 3))
+    v = F.max_pool2d(v, 3, 2, 1)
+    for stage, nb in enumerate(blocks):
+        planes = 64 * 2 ** stage
+        out_c = planes if kind == "basic" else 4 * planes
+        for bi in range(nb):
+            stride = 2 if (stage > 0 and bi == 0) else 1
+            need_ds = stride != 1 or v.shape[1] != out_c
+            if kind == "basic":
+                c1, c2 = next(it), next(it)
+                ds = next(it) if need_ds else None
+                m = conv(F.relu(conv(v, c1, stride, 1)), c2, 1, 1)
+            else:
+                c1, c2, c3 = next(it), next(it), next(it)
+                ds = next(it) if need_ds else None
+                m = conv(F.relu(conv(F.relu(conv(v, c1, 1, 0)), c2, stride, 1)), c3, 1, 0)
+            sc = conv(v, ds, stride, 0) if ds is not None else v
+            v = F.relu(m + sc)
+    v = torch.floor(F.avg_pool2d(v, v.shape[2]))
+    s, p, b = next(it)
+    return F.linear(v.reshape(v.shape[0], -1), t(s.reshape(s.shape[0], -1) * np.ldexp(1.0, p.reshape(p.shape[0], -1))),
+                    t(b))
+
+
+@pytest.mark.parametrize("arch,kind,blocks", [("resnet18", "basic", [2, 2, 2, 2]),
+                                              ("resnet50", "bottleneck", [3, 4, 6, 3])])
+def test_resnet_chain_matches_float64_library_case(arch, kind, blocks):
+    from oracle import networks as ON
+    from paper_1905_13298_gb300 import networks as PN   # layer shapes only (no library call)
+    _, shapes = PN.resnet_program(arch, 32, 32)
+    params = _one_hot_params(shapes, 3)
+    x = si.image_batch(5, 2, 3, 32, 32)
+    got = ON.resnet_forward(x, params, arch)
+    want = _torch_resnet(x, params, kind, blocks).numpy()
+    assert np.abs(want).max() < 2 ** 31
+    assert np.array_equal(got.astype(np.float64), want)
