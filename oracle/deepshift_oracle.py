@@ -16,7 +16,7 @@ Definitions (DeepShift, Elhoushi et al.):
   Y = flip(2^P, S) X + b and Y = flip(2^P, S) (*) X + b.
 * Sec. 4 -- activations and bias are 32-bit fixed point with 16 fraction bits.
 
-Readings taken where the paper is silent (each is listed in the design doc):
+Readings taken where the paper is silent:
 
 * R-order: the integer term is s * (x >> -p): shift first, then flip.
 * R-acc: the sum is exact (int64), then saturated to int32, then the
