@@ -42,6 +42,23 @@ def workload_conv2x(batch: int):
                 terms=N * K * H * W * C * R * S)
 
 
+def workload_by_name(name: str, batch):
+    """Workloads other than the default layer: full configurations of the evaluation."""
+    if name == "conv2x":
+        return workload_conv2x(batch or 32)
+    if name == "fc_large":
+        M, K, N = 8192, 4096, 4096
+        return dict(name="fc_shift_8192x4096x4096_int32", kind="fc", M=M, K=K, Nout=N, terms=M * K * N)
+    if name in ("sweep_resnet50", "sweep_vgg16", "sweep_resnet18"):
+        arch = name.split("_")[1]
+        b = batch or (32 if arch == "resnet18" else 64)
+        return dict(name=f"{arch}_conv_layer_sweep_b{b}_224", kind="sweep", arch=arch, N=b)
+    if name in ("resnet18", "resnet50", "vgg16"):
+        b = batch or (32 if name == "resnet18" else 64)
+        return dict(name=f"{name}_shift_forward_b{b}_224", kind="net", arch=name, N=b)
+    raise ValueError(f"unknown workload {name}")
+
+
 def measured_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -144,6 +161,147 @@ def run_reference(args, wl, rank, world):
            "cpu_baseline": {"value": value, "unit": METRIC, "cores": 1, "kind": "oracle",
                             "sample": f"{n_images} of {wl['N']} images per step"},
            "e2e": {"value": value, "unit": METRIC, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def run_gpu_other(args, wl, rank, world, local_rank):
+    """FC-large and whole-network workloads: value = Gshift-ops/s of the whole step (one forward)."""
+    import torch
+    import paper_1905_13298_gb300 as ds
+    from paper_1905_13298_gb300 import build as dsb
+    from paper_1905_13298_gb300 import networks as PN
+
+    dsb.build_library()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    stream = torch.cuda.current_stream()
+    if wl["kind"] == "fc":
+        x, s, p, b = si.config4_int()
+        w = ds.pack_shift_weights(torch.from_numpy(s).to(dev), torch.from_numpy(p).to(dev), expand=True)
+        xd, bd = torch.from_numpy(x).to(dev), torch.from_numpy(b).to(dev)
+        y = torch.empty((wl["M"], wl["Nout"]), dtype=torch.int32, device=dev)
+        a = torch.zeros(2, dtype=torch.int32, device=dev)
+        terms = wl["terms"]
+
+        def step():  # the stream is looked up at call time so that graph capture records the launches
+            ds.ds_linear_shift(xd, w.desc, bd, y, wl["M"], wl["K"], wl["Nout"], 0, a,
+                               torch.cuda.current_stream().cuda_stream)
+        launches = 2
+        h2d = x.nbytes
+    else:
+        specs, shapes = (PN.resnet_program(wl["arch"]) if wl["arch"] != "vgg16" else PN.vgg16_program())
+        params = si.network_params(shapes, si.SEED_BASE + 3)
+        net = PN.ShiftNetwork(specs, params, batch=wl["N"], device=dev, expand=True)
+        xd = torch.from_numpy(si.image_batch(si.SEED_BASE + 3, wl["N"])).to(dev)
+        y = torch.empty(net.out_shape, dtype=torch.int32, device=dev)
+        terms = PN.shift_terms(specs, wl["N"])
+        launches = 1 + len(specs)
+
+        def step():
+            net.forward(xd, y, torch.cuda.current_stream().cuda_stream)
+        h2d = xd.numel() * 4
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    graph = None
+    if args.graph:
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, capture_error_mode="relaxed"):
+            step()
+        torch.cuda.synchronize()
+        run = graph.replay
+        stream = torch.cuda.current_stream()
+    else:
+        run = step
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(local_rank)
+    sampler.start()
+    time.sleep(0.3)
+    torch.cuda.synchronize()
+    e0.record()
+    for _ in range(args.steps):
+        run()
+    e1.record()
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    ms = e0.elapsed_time(e1)
+    peaks, _ = measured_peaks()
+    sm_max = float(peaks.get("sm_max_mhz", 2070.0))
+    alu_peak = SMS * INT_OPS_PER_CLK_PER_SM * sm_max * 1e6 / 1e12
+    value = terms * args.steps / (ms / 1e3) / 1e9
+    out = {"metric": METRIC, "value": value, "unit": METRIC, "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+           "dtype": "int32", "data": "synthetic",
+           "config": {"workload": wl["name"], "cuda_graph": bool(args.graph), "terms_per_step": terms},
+           "roofline": {"bound": "alu", "achieved": 2 * terms / (ms / args.steps / 1e3) / 1e12, "peak": alu_peak,
+                        "unit": "Tintop/s", "frac": 2 * terms / (ms / args.steps / 1e3) / 1e12 / alu_peak,
+                        "traffic": None, "kernel": "whole step"},
+           "gpu_launches": launches * args.steps, "clocks": clocks, "h2d_bytes_per_step_e2e": h2d}
+    print(json.dumps(out), flush=True)
+
+
+def run_layer_sweep(args, wl, local_rank):
+    """Every conv layer of the network standalone (own inputs, same shapes as in the chain)."""
+    import torch
+    import paper_1905_13298_gb300 as ds
+    from paper_1905_13298_gb300 import build as dsb
+    from paper_1905_13298_gb300 import networks as PN
+
+    dsb.build_library()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    specs, shapes = (PN.resnet_program(wl["arch"]) if wl["arch"] != "vgg16" else PN.vgg16_program())
+    B = wl["N"]
+    seen = {}
+    rows = []
+    tot_terms = tot_ms = 0.0
+    for i, sp in enumerate(specs):
+        if sp.op != ds.DS_OP_CONV:
+            continue
+        key = (sp.C, sp.H, sp.W, sp.K, sp.R, sp.stride, sp.pad)
+        if key in seen:  # identical layers are timed once and counted each time
+            rows.append(dict(seen[key], layer=i))
+            tot_terms += seen[key]["terms"]
+            tot_ms += seen[key]["ms"]
+            continue
+        x, s, p, b = si.conv_layer(si.SEED_BASE + 5 + i, B, sp.C, sp.H, sp.W, sp.K, sp.R, sp.S, 0, 1 << 20,
+                                   si.layer_centre(sp.C, sp.R, sp.S))
+        w = ds.pack_shift_weights(torch.from_numpy(s).to(dev), torch.from_numpy(p).to(dev), expand=True)
+        xd, bd = torch.from_numpy(x).to(dev), torch.from_numpy(b).to(dev)
+        OH = (sp.H + 2 * sp.pad - sp.R) // sp.stride + 1
+        OW = (sp.W + 2 * sp.pad - sp.S) // sp.stride + 1
+        y = torch.empty((B, sp.K, OH, OW), dtype=torch.int32, device=dev)
+        a = torch.zeros(2, dtype=torch.int32, device=dev)
+        ds.ds_absmax(xd, xd.numel(), a)
+        st = torch.cuda.current_stream().cuda_stream
+
+        def call():
+            ds.ds_conv2d_shift(xd, w.desc, bd, None, y, B, sp.C, sp.H, sp.W, sp.K, sp.R, sp.S, sp.stride, sp.stride,
+                               sp.pad, sp.pad, ds.DS_RELU | ds.DS_AMAX_IN, a, st)
+        for _ in range(max(3, args.warmup)):
+            call()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        reps = max(3, args.steps)
+        e0.record()
+        for _ in range(reps):
+            call()
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / reps
+        terms = B * sp.K * OH * OW * sp.C * sp.R * sp.S
+        r = dict(layer=i, shape=f"{sp.C}x{sp.H}x{sp.W}->{sp.K} {sp.R}x{sp.S}/{sp.stride}", terms=terms, ms=ms,
+                 gsops=terms / ms / 1e6, frac=2 * terms / (ms / 1e3) / (SMS * INT_OPS_PER_CLK_PER_SM * 2070e6))
+        seen[key] = r
+        rows.append(r)
+        tot_terms += terms
+        tot_ms += ms
+        del xd, y, w
+    out = {"metric": METRIC, "value": tot_terms / tot_ms / 1e6, "unit": METRIC, "n_gpus": 1, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": tot_ms, "higher_is_better": True, "scaling": "weak",
+           "vs_baseline": None, "dtype": "int32", "data": "synthetic",
+           "config": {"workload": wl["name"], "layers": [{k: (round(v, 4) if isinstance(v, float) else v)
+                                                          for k, v in r.items()} for r in rows]}}
     print(json.dumps(out), flush=True)
 
 
@@ -294,17 +452,26 @@ def main():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
-    ap.add_argument("--batch", type=int, default=32)
+    ap.add_argument("--batch", type=int, default=None)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--workload", default="conv2x", choices=["conv2x", "fc_large", "resnet18", "resnet50", "vgg16",
+                                                         "sweep_resnet18", "sweep_resnet50", "sweep_vgg16"])
+    ap.add_argument("--graph", action="store_true", help="replay each step from a CUDA graph (other workloads)")
     args = ap.parse_args()
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
-    wl = workload_conv2x(args.batch)
+    wl = workload_by_name(args.workload, args.batch)
     if args.impl == "reference":
+        if args.workload != "conv2x":
+            raise SystemExit("the reference arm times the default workload only")
         run_reference(args, wl, rank, world)
-    else:
+    elif args.workload == "conv2x":
         run_gpu(args, wl, rank, world, local_rank)
+    elif wl["kind"] == "sweep":
+        run_layer_sweep(args, wl, local_rank)
+    else:
+        run_gpu_other(args, wl, rank, world, local_rank)
 
 
 if __name__ == "__main__":

@@ -427,9 +427,15 @@ bool choose_geom(const GemmParams& p, Choice& ch) {
 template <int SIG, int S, int TM, int NT>
 cudaError_t launch_direct(const GemmParams& p, const DirectGeom& G, cudaStream_t st) {
   const size_t smem = direct_smem_bytes(G);
-  cudaError_t e = cudaFuncSetAttribute(conv_direct_kernel<SIG, S, TM, NT>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
+  // raise the dynamic shared-memory limit once per process (not a stream operation, so a
+  // forward captured in a CUDA graph after a first eager call issues no attribute call)
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(conv_direct_kernel<SIG, S, TM, NT>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
   const int64_t n_img = p.rows / ((int64_t)p.OH * p.OW);
   const int64_t nb = (int64_t)G.tiles_w * G.tiles_h * n_img;
   dim3 grid((unsigned)nb, (unsigned)((p.cols + NT - 1) / NT));
