@@ -55,6 +55,10 @@ const char* ds_last_error(void);
 /* Library version: major * 10000 + minor * 100 + patch. */
 int ds_version(void);
 
+/* sizeof of the ABI structs as compiled into the library (0: ds_weights, 1: ds_layer), so that
+ * bindings can check their layout; 0 for any other argument. */
+size_t ds_abi_struct_size(int which);
+
 /* ---------------------------------------------------------------------------
  * Flags of the compute calls
  * ------------------------------------------------------------------------- */
@@ -112,6 +116,8 @@ typedef struct ds_weights {
   uint32_t reserved;
   const void* expanded; /* NULL, or the execution layout set by ds_expand_shift_weights */
   size_t expanded_bytes;
+  const void* weights_bf16; /* NULL, or the bf16 weights set by ds_expand_shift_weights_bf16 */
+  size_t weights_bf16_bytes;
 } ds_weights;
 
 /* Bytes needed for the packed blob of an n_out x k_red code matrix (0 if invalid). */
@@ -155,6 +161,42 @@ size_t ds_expanded_weight_bytes(int64_t n_out, int64_t k_red);
  * unfilled descriptor, DS_ERR_BUFFER_TOO_SMALL, DS_ERR_ALIGNMENT.
  */
 ds_status ds_expand_shift_weights(ds_weights* w, void* expanded, size_t expanded_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * Float variant (bf16 activations, fp32 accumulation on the tensor cores).
+ *
+ * With x in bf16 the product x * s * 2^p is exact (s * 2^p is a power of two
+ * with p in [-15, 0]), so LinearShift is an ordinary dense contraction
+ *     y[m][n] = ReLU?( bias[n] + sum_k x[m][k] * W[n][k] ),  W = flip(2^P, S)  (Eq. 3)
+ * with fp32 accumulation.  Its result is not bit-exact: the sum is rounded
+ * in an implementation-defined order; |y - exact| <= 1e-5 * (sum_k |x W| + |bias|)
+ * is the tolerance the tests hold it to.
+ * ------------------------------------------------------------------------- */
+
+/* Bytes of the bf16 weight layout: bf16 [n_out][kpad], kpad = ceil(k_red / 8) * 8. */
+size_t ds_bf16_weight_bytes(int64_t n_out, int64_t k_red);
+
+/*
+ * Decode packed weights into bf16 W[n][k] = s * 2^p (sign bit, exponent 127 + p,
+ * zero mantissa; +0 for s = 0) in `buf` (device, 16-byte aligned, caller-owned)
+ * and record it in w->weights_bf16.  Stream-ordered, asynchronous.
+ */
+ds_status ds_expand_shift_weights_bf16(ds_weights* w, void* buf, size_t bytes, void* stream);
+
+/*
+ * Float LinearShift on tcgen05 tensor cores (TMA-fed, TMEM accumulator).
+ *   x     device bf16 bit patterns (uint16) [M][K], row-major, K % 8 == 0
+ *   w     weights with w->weights_bf16 set, n_out == N, k_red == K
+ *   bias  device fp32 [N] or NULL
+ *   y     device fp32 [M][N]
+ *   flags DS_RELU or 0
+ * Errors: DS_ERR_UNSUPPORTED when K % 8 != 0 or the bf16 weights are missing.
+ */
+ds_status ds_linear_shift_bf16(const uint16_t* x, const ds_weights* w, const float* bias, float* y, int64_t M,
+                               int64_t K, int64_t N, uint32_t flags, void* stream);
+
+/* 1 if a bounded wait of the float kernel gave up (a fault record; 0 normally, -1 if unreadable). */
+int ds_bf16_fault_flag(void);
 
 /* ---------------------------------------------------------------------------
  * Accumulator width.  Each compute call proves, on the device and with no

@@ -400,3 +400,12 @@ def expand_codes(s, p) -> np.ndarray:
         out[cb, :, c] = -p[n, :]
         out[cb, :, 32 + c] = s[n, :]
     return out
+
+
+def weights_bf16_bits(s, p) -> np.ndarray:
+    """bf16 bit patterns of W = flip(2^P, S) (Eq. 3): sign bit of s, exponent 127 + p, zero mantissa; +0 for s = 0."""
+    s = np.asarray(s, dtype=np.int64)
+    p = np.asarray(p, dtype=np.int64)
+    _check_codes(s, p)
+    bits = ((s < 0).astype(np.int64) << 15) | ((127 + p) << 7)
+    return np.where(s == 0, 0, bits).astype(np.uint16)

@@ -55,7 +55,8 @@ class ds_weights(ctypes.Structure):
                 ("n_out", ctypes.c_int64), ("k_red", ctypes.c_int64), ("n_chunks", ctypes.c_int64),
                 ("packed", ctypes.c_void_p), ("packed_bytes", ctypes.c_size_t),
                 ("a_max", ctypes.c_uint64), ("nnz_max", ctypes.c_uint32), ("reserved", ctypes.c_uint32),
-                ("expanded", ctypes.c_void_p), ("expanded_bytes", ctypes.c_size_t)]
+                ("expanded", ctypes.c_void_p), ("expanded_bytes", ctypes.c_size_t),
+                ("weights_bf16", ctypes.c_void_p), ("weights_bf16_bytes", ctypes.c_size_t)]
 
 
 class ds_layer(ctypes.Structure):
@@ -70,6 +71,7 @@ _lib = None
 _SIGNATURES = {
     "ds_last_error": (ctypes.c_char_p, []),
     "ds_version": (ctypes.c_int, []),
+    "ds_abi_struct_size": (ctypes.c_size_t, [ctypes.c_int]),
     "ds_packed_weight_bytes": (ctypes.c_size_t, [ctypes.c_int64, ctypes.c_int64]),
     "ds_pack_shift_weights": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64,
                                              ctypes.c_void_p, ctypes.c_size_t, ctypes.POINTER(ds_weights),
@@ -90,6 +92,13 @@ _SIGNATURES = {
     "ds_shift_forward_workspace_bytes": (ctypes.c_size_t, [ctypes.POINTER(ds_layer), ctypes.c_int, ctypes.c_int]),
     "ds_shift_forward": (ctypes.c_int, [ctypes.POINTER(ds_layer), ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p,
                                         ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int, ctypes.c_void_p]),
+    "ds_bf16_weight_bytes": (ctypes.c_size_t, [ctypes.c_int64, ctypes.c_int64]),
+    "ds_expand_shift_weights_bf16": (ctypes.c_int, [ctypes.POINTER(ds_weights), ctypes.c_void_p, ctypes.c_size_t,
+                                                    ctypes.c_void_p]),
+    "ds_linear_shift_bf16": (ctypes.c_int, [ctypes.c_void_p, ctypes.POINTER(ds_weights), ctypes.c_void_p,
+                                            ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
+                                            ctypes.c_uint32, ctypes.c_void_p]),
+    "ds_bf16_fault_flag": (ctypes.c_int, []),
     "ds_absmax": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]),
 }
 
@@ -105,6 +114,9 @@ def lib() -> ctypes.CDLL:
             fn = getattr(L, name)
             fn.restype = res
             fn.argtypes = args
+        for which, st in ((0, ds_weights), (1, ds_layer)):
+            if L.ds_abi_struct_size(which) != ctypes.sizeof(st):
+                raise ImportError(f"{st.__name__} layout differs between the binding and {LIB_PATH}")
         _lib = L
     return _lib
 
@@ -185,6 +197,22 @@ def ds_shift_forward(layers, n: int, x, y, ws, ws_bytes: int, batch: int, stream
     _check(lib().ds_shift_forward(layers, n, _ptr(x), _ptr(y), _ptr(ws), ws_bytes, batch, _stream(stream)))
 
 
+def ds_bf16_weight_bytes(n_out: int, k_red: int) -> int:
+    return int(lib().ds_bf16_weight_bytes(n_out, k_red))
+
+
+def ds_expand_shift_weights_bf16(w: ds_weights, buf, nbytes: int, stream=None) -> None:
+    _check(lib().ds_expand_shift_weights_bf16(ctypes.byref(w), _ptr(buf), nbytes, _stream(stream)))
+
+
+def ds_linear_shift_bf16(x, w: ds_weights, bias, y, M: int, K: int, N: int, flags: int = 0, stream=None) -> None:
+    _check(lib().ds_linear_shift_bf16(_ptr(x), ctypes.byref(w), _ptr(bias), _ptr(y), M, K, N, flags, _stream(stream)))
+
+
+def ds_bf16_fault_flag() -> int:
+    return int(lib().ds_bf16_fault_flag())
+
+
 def ds_absmax(x, n: int, amax, stream=None) -> None:
     _check(lib().ds_absmax(_ptr(x), n, _ptr(amax), _stream(stream)))
 
@@ -201,6 +229,7 @@ class PackedShiftWeights:
         self.blob = blob
         self.desc = desc
         self.expanded = None
+        self.bf16 = None
 
     @property
     def n_out(self) -> int:
@@ -219,6 +248,26 @@ def expand_shift_weights(w: PackedShiftWeights, stream=None) -> PackedShiftWeigh
     ds_expand_shift_weights(w.desc, buf, nbytes, stream)
     w.expanded = buf
     return w
+
+
+def expand_shift_weights_bf16(w: PackedShiftWeights, stream=None) -> PackedShiftWeights:
+    """Adds the bf16 weight layout W = s * 2^p used by the float variant."""
+    import torch
+    nbytes = ds_bf16_weight_bytes(w.n_out, w.k_red)
+    buf = torch.empty(nbytes, dtype=torch.uint8, device=w.blob.device)
+    ds_expand_shift_weights_bf16(w.desc, buf, nbytes, stream)
+    w.bf16 = buf
+    return w
+
+
+def linear_shift_bf16(x, w: PackedShiftWeights, bias=None, relu: bool = False, out=None, stream=None):
+    """Float LinearShift: fp32 y = bias + x @ W^T (ReLU) for bf16 x [M, K] on the tensor cores."""
+    import torch
+    M, K = x.shape
+    N = w.n_out
+    y = out if out is not None else torch.empty((M, N), dtype=torch.float32, device=x.device)
+    ds_linear_shift_bf16(x, w.desc, bias, y, M, K, N, DS_RELU if relu else 0, stream)
+    return y
 
 
 def pack_shift_weights(s, p, stream=None, expand: bool = False) -> PackedShiftWeights:

@@ -152,6 +152,10 @@ const char* ds_last_error(void) { return g_last_error.c_str(); }
 
 int ds_version(void) { return 100; }
 
+size_t ds_abi_struct_size(int which) {
+  return which == 0 ? sizeof(ds_weights) : (which == 1 ? sizeof(ds_layer) : 0);
+}
+
 size_t ds_packed_weight_bytes(int64_t n_out, int64_t k_red) {
   if (n_out <= 0 || k_red <= 0) return 0;
   if (n_out > (int64_t(1) << 31) || k_red > (int64_t(1) << 40)) return 0;
@@ -192,6 +196,8 @@ ds_status ds_pack_shift_weights(const int8_t* s, const int8_t* p, int64_t n_out,
   desc->reserved = 0;
   desc->expanded = nullptr;
   desc->expanded_bytes = 0;
+  desc->weights_bf16 = nullptr;
+  desc->weights_bf16_bytes = 0;
   return DS_OK;
 }
 
@@ -219,6 +225,50 @@ ds_status ds_expand_shift_weights(ds_weights* w, void* expanded, size_t expanded
   w->expanded_bytes = need;
   return DS_OK;
 }
+
+size_t ds_bf16_weight_bytes(int64_t n_out, int64_t k_red) {
+  if (n_out <= 0 || k_red <= 0) return 0;
+  if (n_out > (int64_t(1) << 31) || k_red > (int64_t(1) << 36)) return 0;
+  return (size_t)(n_out * bf16_kpad(k_red) * 2 + 255) / 256 * 256;
+}
+
+ds_status ds_expand_shift_weights_bf16(ds_weights* w, void* buf, size_t bytes, void* stream) {
+  clear_error();
+  if (w == nullptr || buf == nullptr) return fail(DS_ERR_INVALID_ARG, "NULL pointer argument");
+  ds_status r = check_weights(w, w->n_out, w->k_red);
+  if (r != DS_OK) return r;
+  const size_t need = ds_bf16_weight_bytes(w->n_out, w->k_red);
+  if (need == 0) return fail(DS_ERR_UNSUPPORTED, "code matrix too large");
+  if (bytes < need) return fail(DS_ERR_BUFFER_TOO_SMALL, "bf16 buffer has %zu bytes, needs %zu", bytes, need);
+  if (!aligned16(buf)) return fail(DS_ERR_ALIGNMENT, "bf16 buffer must be 16-byte aligned");
+  r = cuda_check(launch_expand_bf16(static_cast<const uint8_t*>(w->packed), w->n_out, w->k_red,
+                                    static_cast<uint16_t*>(buf), static_cast<cudaStream_t>(stream)),
+                 "bf16 expand launch");
+  if (r != DS_OK) return r;
+  w->weights_bf16 = buf;
+  w->weights_bf16_bytes = need;
+  return DS_OK;
+}
+
+ds_status ds_linear_shift_bf16(const uint16_t* x, const ds_weights* w, const float* bias, float* y, int64_t M,
+                               int64_t K, int64_t N, uint32_t flags, void* stream) {
+  clear_error();
+  if (!x || !y) return fail(DS_ERR_INVALID_ARG, "NULL x or y");
+  if (M <= 0 || K <= 0 || N <= 0) return fail(DS_ERR_SHAPE, "M, K and N must be positive");
+  if (M > ((int64_t)1 << 31) - 256 || N > ((int64_t)1 << 31) - 256) return fail(DS_ERR_UNSUPPORTED, "M or N too large");
+  if (flags & ~DS_RELU) return fail(DS_ERR_INVALID_ARG, "only DS_RELU applies to the float variant");
+  if (!aligned16(x) || !aligned16(y)) return fail(DS_ERR_ALIGNMENT, "x and y must be 16-byte aligned");
+  if (K % 8 != 0) return fail(DS_ERR_UNSUPPORTED, "K must be a multiple of 8 (16-byte bf16 rows)");
+  ds_status r = check_weights(w, N, K);
+  if (r != DS_OK) return r;
+  if (w->weights_bf16 == nullptr || w->weights_bf16_bytes < ds_bf16_weight_bytes(N, K))
+    return fail(DS_ERR_UNSUPPORTED, "bf16 weights missing: call ds_expand_shift_weights_bf16 first");
+  return cuda_check(launch_linear_bf16(x, static_cast<const uint16_t*>(w->weights_bf16), bias, y, M, K, N, flags,
+                                       static_cast<cudaStream_t>(stream)),
+                    "linear_shift_bf16 launch");
+}
+
+int ds_bf16_fault_flag(void) { return read_bf16_fault_flag(); }
 
 ds_status ds_absmax(const int32_t* x, int64_t n, uint32_t* amax, void* stream) {
   clear_error();

@@ -55,8 +55,11 @@ def test_packed_bytes_match_documented_layout(ds):
     assert ds.ds_packed_weight_bytes(5, -1) == 0
 
 
-def test_weights_struct_layout(ds):
-    assert ctypes.sizeof(ds.ds_weights) == 80
+def test_struct_layouts_match_library(ds):
+    L = ds.lib()
+    assert L.ds_abi_struct_size(0) == ctypes.sizeof(ds.ds_weights) == 96
+    assert L.ds_abi_struct_size(1) == ctypes.sizeof(ds.ds_layer)
+    assert L.ds_abi_struct_size(7) == 0
     assert ds.ds_weights.packed.offset == 32
 
 

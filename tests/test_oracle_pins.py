@@ -490,3 +490,13 @@ def test_resnet_chain_matches_float64_library_case(arch, kind, blocks):
     want = _torch_resnet(x, params, kind, blocks).numpy()
     assert np.abs(want).max() < 2 ** 31
     assert np.array_equal(got.astype(np.float64), want)
+
+
+def test_bf16_weight_bits_decode_to_s_times_power_of_two():
+    """bf16 patterns of the float variant's weights decode (via float32 bit casts) to s * 2^p exactly."""
+    s = np.array([[1, -1, 0, 1], [-1, 1, 1, 0]])
+    p = np.array([[0, -15, -3, -7], [-1, -2, 0, -15]])
+    bits = O.weights_bf16_bits(s, p)
+    assert bits[0, 0] == 0x3F80 and bits[0, 1] == 0xB800 and bits[0, 2] == 0 and bits[1, 2] == 0x3F80
+    vals = si.bits_to_f64(bits)
+    assert np.array_equal(vals, s * np.ldexp(1.0, p))
