@@ -46,6 +46,9 @@ def workload_by_name(name: str, batch):
     """Workloads other than the default layer: full configurations of the evaluation."""
     if name == "conv2x":
         return workload_conv2x(batch or 32)
+    if name == "fc_large_bf16":
+        M, K, N = 8192, 4096, 4096
+        return dict(name="fc_shift_8192x4096x4096_bf16", kind="fc16", M=M, K=K, Nout=N, terms=M * K * N)
     if name == "fc_large":
         M, K, N = 8192, 4096, 4096
         return dict(name="fc_shift_8192x4096x4096_int32", kind="fc", M=M, K=K, Nout=N, terms=M * K * N)
@@ -175,7 +178,24 @@ def run_gpu_other(args, wl, rank, world, local_rank):
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
     stream = torch.cuda.current_stream()
-    if wl["kind"] == "fc":
+    if wl["kind"] == "fc16":
+        rng = np.random.default_rng(si.SEED_BASE + 44)
+        bits = si.bf16_bits(rng.uniform(-(1 << 20), 1 << 20, size=(wl["M"], wl["K"])))
+        s = si.sign_codes(si.SEED_BASE + 44, (wl["Nout"], wl["K"]))
+        p = si.shift_codes_uniform(si.SEED_BASE + 44, (wl["Nout"], wl["K"]))
+        w = ds.pack_shift_weights(torch.from_numpy(s).to(dev), torch.from_numpy(p).to(dev))
+        ds.expand_shift_weights_bf16(w)
+        xd = torch.from_numpy(bits.view(np.int16)).to(dev).view(torch.bfloat16)
+        bd = torch.zeros(wl["Nout"], dtype=torch.float32, device=dev)
+        y = torch.empty((wl["M"], wl["Nout"]), dtype=torch.float32, device=dev)
+        terms = wl["terms"]
+
+        def step():
+            ds.ds_linear_shift_bf16(xd, w.desc, bd, y, wl["M"], wl["K"], wl["Nout"], 0,
+                                    torch.cuda.current_stream().cuda_stream)
+        launches = 1
+        h2d = xd.numel() * 2
+    elif wl["kind"] == "fc":
         x, s, p, b = si.config4_int()
         w = ds.pack_shift_weights(torch.from_numpy(s).to(dev), torch.from_numpy(p).to(dev), expand=True)
         xd, bd = torch.from_numpy(x).to(dev), torch.from_numpy(b).to(dev)
@@ -229,13 +249,20 @@ def run_gpu_other(args, wl, rank, world, local_rank):
     sm_max = float(peaks.get("sm_max_mhz", 2070.0))
     alu_peak = SMS * INT_OPS_PER_CLK_PER_SM * sm_max * 1e6 / 1e12
     value = terms * args.steps / (ms / 1e3) / 1e9
+    if wl["kind"] == "fc16":
+        tflops = 2 * terms / (ms / args.steps / 1e3) / 1e12
+        peak = float(peaks.get("bf16_tflops", 1894.4))
+        roof = {"bound": "tensor", "achieved": tflops, "peak": peak, "unit": "TFLOP/s", "frac": tflops / peak,
+                "traffic": None, "kernel": "linear_bf16_kernel", "peak_basis": "bf16_tflops (burst), measured"}
+    else:
+        roof = {"bound": "alu", "achieved": 2 * terms / (ms / args.steps / 1e3) / 1e12, "peak": alu_peak,
+                "unit": "Tintop/s", "frac": 2 * terms / (ms / args.steps / 1e3) / 1e12 / alu_peak,
+                "traffic": None, "kernel": "whole step"}
     out = {"metric": METRIC, "value": value, "unit": METRIC, "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
            "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-           "dtype": "int32", "data": "synthetic",
+           "dtype": "bf16" if wl["kind"] == "fc16" else "int32", "data": "synthetic",
            "config": {"workload": wl["name"], "cuda_graph": bool(args.graph), "terms_per_step": terms},
-           "roofline": {"bound": "alu", "achieved": 2 * terms / (ms / args.steps / 1e3) / 1e12, "peak": alu_peak,
-                        "unit": "Tintop/s", "frac": 2 * terms / (ms / args.steps / 1e3) / 1e12 / alu_peak,
-                        "traffic": None, "kernel": "whole step"},
+           "roofline": roof,
            "gpu_launches": launches * args.steps, "clocks": clocks, "h2d_bytes_per_step_e2e": h2d}
     print(json.dumps(out), flush=True)
 
@@ -454,7 +481,7 @@ def main():
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--batch", type=int, default=None)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--workload", default="conv2x", choices=["conv2x", "fc_large", "resnet18", "resnet50", "vgg16",
+    ap.add_argument("--workload", default="conv2x", choices=["conv2x", "fc_large", "fc_large_bf16", "resnet18", "resnet50", "vgg16",
                                                          "sweep_resnet18", "sweep_resnet50", "sweep_vgg16"])
     ap.add_argument("--graph", action="store_true", help="replay each step from a CUDA graph (other workloads)")
     args = ap.parse_args()
