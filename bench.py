@@ -62,6 +62,26 @@ def workload_by_name(name: str, batch):
     raise ValueError(f"unknown workload {name}")
 
 
+def reduce_max_over_ranks(values, device=None):
+    """Element-wise max of a list of floats over all ranks (identity without a process group).
+
+    Every rank runs its own replica on its own batch (weak scaling, no data-path collective); the job time is the
+    slowest rank's, so value = units of all ranks / max time.
+    """
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return list(values)
+    t = torch.tensor(list(values), dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t.tolist()]
+
+
+def replica_seed(base: int, rank: int) -> int:
+    """Seed of rank r's replica: distinct inputs per rank, identical across runs."""
+    return base + 1000 * rank
+
+
 def measured_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -346,7 +366,7 @@ def run_gpu(args, wl, rank, world, local_rank):
         dist.init_process_group("nccl", device_id=dev)
 
     N, C, H, W, K, R, S = (wl[k] for k in ("N", "C", "H", "W", "K", "R", "S"))
-    seed = si.SEED_BASE + 2 + 1000 * rank
+    seed = replica_seed(si.SEED_BASE + 2, rank)
     x, s, p, b = si.conv_layer(seed, N, C, H, W, K, R, S)
     w = ds.pack_shift_weights(torch.from_numpy(s).to(dev), torch.from_numpy(p).to(dev), expand=True)
     bd = torch.from_numpy(b).to(dev)
@@ -392,10 +412,7 @@ def run_gpu(args, wl, rank, world, local_rank):
     clocks = sampler.stop() if sampler else None
     ms_total = t_start.elapsed_time(t_end)
     kern_ms = float(np.mean([a.elapsed_time(b) for a, b in evs]))
-    if dist:
-        tt = torch.tensor([ms_total, kern_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms_total, kern_ms = float(tt[0]), float(tt[1])
+    ms_total, kern_ms = reduce_max_over_ranks([ms_total, kern_ms], dev)
 
     # end to end through the public API with host buffers
     xh = torch.from_numpy(x).pin_memory()
@@ -421,10 +438,7 @@ def run_gpu(args, wl, rank, world, local_rank):
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1)
-    if dist:
-        tt = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_ms = float(tt[0])
+    e2e_ms = reduce_max_over_ranks([e2e_ms], dev)[0]
 
     # parity spot check of the timed output (whole-tensor parity lives in tests/)
     if rank == 0:
