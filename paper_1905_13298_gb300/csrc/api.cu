@@ -90,20 +90,14 @@ static ds_status prepare_amax(const int32_t* x, int64_t nx, uint32_t flags, uint
   return DS_OK;
 }
 
-ds_status conv_launch(const int32_t* x, const ds_weights* w, const int32_t* bias, const int32_t* residual,
-                      int32_t* y, int N, int C, int H, int W, int K, int R, int S, int stride, int pad,
-                      uint32_t flags, const uint32_t* amax_in, uint32_t* amax_out, cudaStream_t st) {
+GemmParams conv_params(const ds_weights* w, int N, int C, int H, int W, int K, int R, int S, int stride,
+                       int pad) {
   GemmParams p{};
-  p.x = x;
-  p.bias = bias;
-  p.residual = (flags & DS_RESIDUAL) ? residual : nullptr;
-  p.y = y;
   p.OH = (H + 2 * pad - R) / stride + 1;
   p.OW = (W + 2 * pad - S) / stride + 1;
   p.rows = (int64_t)N * p.OH * p.OW;
   p.kred = (int64_t)C * R * S;
   p.cols = K;
-  p.flags = flags;
   p.C = C;
   p.H = H;
   p.W = W;
@@ -114,10 +108,26 @@ ds_status conv_launch(const int32_t* x, const ds_weights* w, const int32_t* bias
   p.ph = pad;
   p.pw = pad;
   fill_blob_offsets(p, w);
+  return p;
+}
+
+ds_status conv_launch(const int32_t* x, const ds_weights* w, const int32_t* bias, const int32_t* residual,
+                      int32_t* y, int N, int C, int H, int W, int K, int R, int S, int stride, int pad,
+                      uint32_t flags, const uint32_t* amax_in, uint32_t* amax_out, cudaStream_t st,
+                      int64_t* split_acc, size_t split_capacity) {
+  GemmParams p = conv_params(w, N, C, H, W, K, R, S, stride, pad);
+  p.x = x;
+  p.bias = bias;
+  p.residual = (flags & DS_RESIDUAL) ? residual : nullptr;
+  p.y = y;
+  p.flags = flags;
   p.amax_in = amax_in;
   p.amax_out = amax_out;
+  p.split_acc = split_acc;
+  p.split_capacity = split_capacity;
   if (!(flags & DS_CONV_IM2COL) && conv_direct_supported(p))
     return cuda_check(launch_conv2d_direct(p, st), "conv2d_shift (direct) launch");
+  p.split_acc = nullptr;
   return cuda_check(launch_conv2d_shift(p, st), "conv2d_shift (implicit GEMM) launch");
 }
 

@@ -20,25 +20,39 @@
 //
 // Accumulator width as in shift_gemm.cu: 32-bit when the launch bound proves
 // it exact for the CTA's channels, else a 64-bit pass per half of the pixels.
+#include <algorithm>
+
 #include "ds_common.cuh"
 
 namespace ds {
 namespace {
 
 constexpr int TN = 4;                   // output channels per thread
-constexpr int kThreads = 256;           // 8 warps: every SM sub-partition gets the same share
+constexpr int NT = 32;                  // output channels per CTA
+constexpr int CG = NT / TN;             // channel groups per CTA
+constexpr int kMaxThreads = 256;        // 8 warps: every SM sub-partition gets the same share
 constexpr int kSmemBudget = 74 * 1024;  // 3 CTAs per SM
+constexpr int kSlots = 152 * 3;         // resident CTAs on a GB300
 
+// The CTA tiles run over the stacked output rows gr = n * OH + oh of all
+// images, so a tile may span image boundaries (small feature maps, batch 1).
+// In "stacked input" coordinates image n's zero-padded rows are
+// n * HP + ihp (HP = H + 2 * pad); output row (n, oh) reads stacked rows
+// n * HP + oh * sig + r.  A tile's halo is the contiguous stacked range its
+// rows read, HR rows at most.
 struct DirectGeom {
   int TH, GW;        // output rows and pixel groups per row per CTA
+  int threads;       // TH * GW * CG
   int CC;            // input channels per stage
-  int HR;            // halo rows
+  int HR, HP;        // halo rows per tile, padded input height
+  int N;             // images
   int taps;          // CC * R * S
   int n_stages;      // ceil(C / CC)
   int halo_words;    // CC * HR * GW * WSP
   int code_words;    // taps * 2 * NT
   int run;           // taps per decode item (blob path)
   int tiles_w, tiles_h;
+  int splits, stages_per_split;  // split reduction over the stages
 };
 
 __device__ __forceinline__ void cp_async4(void* smem_dst, const void* gsrc, bool valid) {
@@ -69,26 +83,29 @@ struct Win {
   static constexpr int WV = WSP / 4;             // 16-byte loads per window
 };
 
-// Stage the group windows of input channels [c0, c0 + CC): one slot
-// (channel, halo row, group) per thread at a time; zero outside the image
-// and for channels >= C.
+// Stage the group windows of input channels [c0, c0 + CC) for halo rows
+// s_lo .. s_lo + HR - 1 (stacked coordinates): one slot (channel, halo row,
+// group) per thread at a time; zero in padding rows, outside the image and
+// for channels >= C.
 template <int SIG, int S, int TM>
-__device__ __forceinline__ void stage_halo(const GemmParams& P, const DirectGeom G, int32_t* halo,
-                                           int64_t img_base, int ih0, int iw0, int c0) {
+__device__ __forceinline__ void stage_halo(const GemmParams& P, const DirectGeom G, int32_t* halo, int64_t s_lo,
+                                           int iw0, int c0) {
   using WN = Win<SIG, S, TM>;
   const int64_t HW = (int64_t)P.H * P.W;
   const int nslots = G.CC * G.HR * G.GW;
-  for (int sl = threadIdx.x; sl < nslots; sl += kThreads) {
-    const int row = sl / G.GW;          // (channel, halo row)
+  for (int sl = threadIdx.x; sl < nslots; sl += G.threads) {
+    const int row = sl / G.GW;  // (channel, halo row)
     const int g = sl - row * G.GW;
     const int cl = row / G.HR;
     const int hr = row - cl * G.HR;
     const int c = c0 + cl;
-    const int ih = ih0 + hr;
+    const int64_t sr = s_lo + hr;
+    const int64_t ni = sr / G.HP;
+    const int ih = (int)(sr - ni * G.HP) - P.ph;
     const int iws = iw0 + g * TM * SIG;
     int32_t* dst = halo + sl * WN::WSP;
-    const bool row_ok = (c < P.C) && ((unsigned)ih < (unsigned)P.H);
-    const int32_t* src = P.x + img_base + (int64_t)c * HW + (int64_t)ih * P.W + iws;
+    const bool row_ok = (c < P.C) && (ni < G.N) && ((unsigned)ih < (unsigned)P.H);
+    const int32_t* src = P.x + (ni * P.C + c) * HW + (int64_t)ih * P.W + iws;
     if (row_ok && iws >= 0 && iws + WN::WS <= P.W) {
 #pragma unroll
       for (int i = 0; i < WN::WS; ++i) cp_async4(dst + i, src + i, true);
@@ -104,7 +121,6 @@ __device__ __forceinline__ void stage_halo(const GemmParams& P, const DirectGeom
 
 // Codes of taps [kb, kb + taps) of the CTA's NT channels.  Shared-memory row
 // per tap: NT/32 blocks of 64 words (32 shifts, then 32 signs).
-template <int NT>
 __device__ __forceinline__ void stage_codes_expanded(const GemmParams& P, const DirectGeom G, int32_t* code,
                                                      int64_t col0, int64_t kb) {
   constexpr int NB = NT / 32;
@@ -113,7 +129,7 @@ __device__ __forceinline__ void stage_codes_expanded(const GemmParams& P, const 
 #pragma unroll
   for (int b = 0; b < NB; ++b) {
     const int64_t cb = col0 / 32 + b;
-    for (int e = threadIdx.x; e < per_block; e += kThreads) {
+    for (int e = threadIdx.x; e < per_block; e += G.threads) {
       const int tap = e >> 4, q = e & 15;
       const bool ok = (cb < nblocks) && (kb + tap < P.kred);
       const int32_t* src = ok ? P.xcodes + ((cb * P.kred + kb + tap) * 64 + q * 4) : P.xcodes;
@@ -131,7 +147,6 @@ __device__ __forceinline__ uint2 bit_words(const GemmParams& P, int64_t col, int
   return __ldg(reinterpret_cast<const uint2*>(P.blob + P.off_bits + rec * 8));
 }
 
-template <int NT>
 __device__ __forceinline__ void decode_codes(const GemmParams& P, const DirectGeom G, int32_t* code,
                                              int64_t col0, int64_t kb) {
   constexpr int NB = NT / 32;
@@ -175,7 +190,7 @@ __device__ __forceinline__ void decode_codes(const GemmParams& P, const DirectGe
 
 // The hot loop over one stage.  hp: this thread's window slot in channel 0
 // of the stage; cp: this thread's 4 channels in tap 0 of the stage.
-template <int SIG, int S, int TM, int NT, int I0, int NI, typename Acc>
+template <int SIG, int S, int TM, int I0, int NI, typename Acc>
 __device__ __forceinline__ void compute_stage(const DirectGeom G, const int32_t* hp, const int32_t* cp,
                                               int rowstride, Acc (&acc)[NI][TN]) {
   using WN = Win<SIG, S, TM>;
@@ -222,25 +237,31 @@ __device__ __forceinline__ void compute_stage(const DirectGeom G, const int32_t*
   }
 }
 
-template <int SIG, int S, int TM, int NT, int I0, int NI, typename Acc>
+template <int SIG, int S, int TM, int I0, int NI, typename Acc>
 __device__ __forceinline__ void run_direct(const GemmParams& P, const DirectGeom G, unsigned char* smem,
-                                           int n_img, int oh0, int ow0, int64_t col0,
+                                           int64_t gr0, int ow0, int64_t col0, int st_begin, int st_end,
                                            uint32_t& amax_local) {
   using WN = Win<SIG, S, TM>;
-  constexpr int CG = NT / TN;
   const int t = threadIdx.x;
   const int cg = t % CG;
   const int pg = t / CG;
   const int g = pg % G.GW;
   const int oh_l = pg / G.GW;
-  const int64_t img_base = (int64_t)n_img * P.C * P.H * P.W;
-  const int ih0 = oh0 * SIG - P.ph;
+  // the tile's first stacked halo row, and this thread's halo row offset
+  const int64_t n0 = gr0 / P.OH;
+  const int64_t s_lo = n0 * G.HP + (gr0 - n0 * P.OH) * SIG;
+  int srow;
+  {
+    const int64_t gr = gr0 + oh_l;
+    const int64_t ni = gr / P.OH;
+    srow = gr < (int64_t)G.N * P.OH ? (int)(ni * G.HP + (gr - ni * P.OH) * SIG - s_lo) : 0;
+  }
   const int iw0 = ow0 * SIG - P.pw;
   const int rowstride = G.GW * WN::WSP;
 
   int32_t* const halo_base = reinterpret_cast<int32_t*>(smem);
   int32_t* const code_base = halo_base + 2 * G.halo_words;
-  const int hoff = (oh_l * SIG) * rowstride + g * WN::WSP;
+  const int hoff = srow * rowstride + g * WN::WSP;
   const int coff = (cg >> 3) * 64 + (cg & 7) * TN;
   const bool expanded = P.xcodes != nullptr;
 
@@ -257,46 +278,71 @@ __device__ __forceinline__ void run_direct(const GemmParams& P, const DirectGeom
   // for its own copies before the next barrier, which then makes all of
   // stage st + 1 visible.
   const int64_t taps_per_c = (int64_t)S * S;
-  stage_halo<SIG, S, TM>(P, G, halo_base, img_base, ih0, iw0, 0);
-  if (expanded) stage_codes_expanded<NT>(P, G, code_base, col0, 0);
-  cp_async_commit();
-  if (!expanded) decode_codes<NT>(P, G, code_base, col0, 0);
-  cp_async_wait_all();
-  for (int st = 0; st < G.n_stages; ++st) {
-    const int b = st & 1;
-    const bool more = st + 1 < G.n_stages;
+  {
+    const int64_t kb = (int64_t)st_begin * G.CC * taps_per_c;
+    stage_halo<SIG, S, TM>(P, G, halo_base, s_lo, iw0, st_begin * G.CC);
+    if (expanded) stage_codes_expanded(P, G, code_base, col0, kb);
+    cp_async_commit();
+    if (!expanded) decode_codes(P, G, code_base, col0, kb);
+    cp_async_wait_all();
+  }
+  for (int st = st_begin; st < st_end; ++st) {
+    const int b = (st - st_begin) & 1;
+    const bool more = st + 1 < st_end;
     const int64_t kb1 = (int64_t)(st + 1) * G.CC * taps_per_c;
     __syncthreads();
     if (more) {
-      stage_halo<SIG, S, TM>(P, G, halo_base + (b ^ 1) * G.halo_words, img_base, ih0, iw0,
-                             (st + 1) * G.CC);
-      if (expanded) stage_codes_expanded<NT>(P, G, code_base + (b ^ 1) * G.code_words, col0, kb1);
+      stage_halo<SIG, S, TM>(P, G, halo_base + (b ^ 1) * G.halo_words, s_lo, iw0, (st + 1) * G.CC);
+      if (expanded) stage_codes_expanded(P, G, code_base + (b ^ 1) * G.code_words, col0, kb1);
       cp_async_commit();
     }
-    compute_stage<SIG, S, TM, NT, I0, NI, Acc>(G, halo_base + b * G.halo_words + hoff,
-                                               code_base + b * G.code_words + coff, rowstride, acc);
+    compute_stage<SIG, S, TM, I0, NI, Acc>(G, halo_base + b * G.halo_words + hoff,
+                                           code_base + b * G.code_words + coff, rowstride, acc);
     if (more) {
-      if (!expanded) decode_codes<NT>(P, G, code_base + (b ^ 1) * G.code_words, col0, kb1);
+      if (!expanded) decode_codes(P, G, code_base + (b ^ 1) * G.code_words, col0, kb1);
       cp_async_wait_all();
     }
   }
   __syncthreads();  // the next pass (64-bit path) reuses the buffers
 
-  // fused epilogue: bias, saturation (64-bit path), residual, ReLU, amax
-  const int oh = oh0 + oh_l;
-  if (oh >= P.OH) return;
-  const bool relu = (P.flags & DS_RELU) != 0;
-  const bool resid = (P.flags & DS_RESIDUAL) != 0;
+  const int64_t gr = gr0 + oh_l;  // this thread's output row (recomputed: not kept live in the loop)
+  if (gr >= (int64_t)G.N * P.OH) return;
+  const int64_t n_img = gr / P.OH;
+  const int oh = (int)(gr - n_img * P.OH);
   const int owb = ow0 + g * TM + I0;
   const int64_t OHW = (int64_t)P.OH * P.OW;
+  if (P.split_acc != nullptr) {
+    // split reduction: add this stage range's exact partial sums (no bias)
+#pragma unroll
+    for (int j = 0; j < TN; ++j) {
+      const int64_t col = col0 + cg * TN + j;
+      if (col >= P.cols) continue;
+      unsigned long long* arow = reinterpret_cast<unsigned long long*>(P.split_acc) +
+                                 (n_img * P.cols + col) * OHW + (int64_t)oh * P.OW;
+#pragma unroll
+      for (int i = 0; i < NI; ++i) {
+        if (owb + i >= P.OW) continue;
+        int64_t v;
+        if constexpr (sizeof(Acc) == 4) {
+          v = (int64_t)(int32_t)acc[i][j];  // exact: |partial| <= the proven bound < 2^31
+        } else {
+          v = acc[i][j];
+        }
+        atomicAdd(arow + owb + i, (unsigned long long)v);
+      }
+    }
+    return;
+  }
+  // fused epilogue: bias, saturation (64-bit path), residual, ReLU, amax
+  const bool relu = (P.flags & DS_RELU) != 0;
+  const bool resid = (P.flags & DS_RESIDUAL) != 0;
 #pragma unroll
   for (int j = 0; j < TN; ++j) {
     const int64_t col = col0 + cg * TN + j;
     if (col >= P.cols) continue;
     const int32_t bcol = P.bias ? __ldg(P.bias + col) : 0;
-    int32_t* yrow = P.y + ((int64_t)n_img * P.cols + col) * OHW + (int64_t)oh * P.OW;
-    const int32_t* rrow = resid ? P.residual + ((int64_t)n_img * P.cols + col) * OHW + (int64_t)oh * P.OW
-                                : nullptr;
+    int32_t* yrow = P.y + (n_img * P.cols + col) * OHW + (int64_t)oh * P.OW;
+    const int32_t* rrow = resid ? P.residual + (n_img * P.cols + col) * OHW + (int64_t)oh * P.OW : nullptr;
 #pragma unroll
     for (int i = 0; i < NI; ++i) {
       const int ow = owb + i;
@@ -342,24 +388,49 @@ __device__ __forceinline__ bool tile_int32_exact(const GemmParams& P, int NT, in
   return !__syncthreads_or(unsafe);
 }
 
-template <int SIG, int S, int TM, int NT>
-__global__ void __launch_bounds__(kThreads, 3) conv_direct_kernel(const GemmParams P, const DirectGeom G) {
+template <int SIG, int S, int TM>
+__global__ void __launch_bounds__(kMaxThreads, 3) conv_direct_kernel(const GemmParams P, const DirectGeom G) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  int bx = blockIdx.x;
+  const int bx = blockIdx.x;
   const int tw = bx % G.tiles_w;
-  bx /= G.tiles_w;
-  const int th = bx % G.tiles_h;
-  const int n_img = bx / G.tiles_h;
+  const int th = bx / G.tiles_w;
   const int64_t col0 = (int64_t)blockIdx.y * NT;
-  const int oh0 = th * G.TH, ow0 = tw * TM * G.GW;
+  const int64_t gr0 = (int64_t)th * G.TH;
+  const int ow0 = tw * TM * G.GW;
+  const int st_begin = blockIdx.z * G.stages_per_split;
+  const int st_end = min(G.n_stages, st_begin + G.stages_per_split);
 
   uint32_t amax_local = 0;
   if (tile_int32_exact(P, NT, col0)) {
-    run_direct<SIG, S, TM, NT, 0, TM, uint32_t>(P, G, smem_raw, n_img, oh0, ow0, col0, amax_local);
+    run_direct<SIG, S, TM, 0, TM, uint32_t>(P, G, smem_raw, gr0, ow0, col0, st_begin, st_end, amax_local);
   } else {
     constexpr int H1 = TM / 2;
-    run_direct<SIG, S, TM, NT, 0, H1, int64_t>(P, G, smem_raw, n_img, oh0, ow0, col0, amax_local);
-    run_direct<SIG, S, TM, NT, H1, TM - H1, int64_t>(P, G, smem_raw, n_img, oh0, ow0, col0, amax_local);
+    run_direct<SIG, S, TM, 0, H1, int64_t>(P, G, smem_raw, gr0, ow0, col0, st_begin, st_end, amax_local);
+    run_direct<SIG, S, TM, H1, TM - H1, int64_t>(P, G, smem_raw, gr0, ow0, col0, st_begin, st_end, amax_local);
+  }
+  if (P.amax_out != nullptr && P.split_acc == nullptr) {
+    amax_local = __reduce_max_sync(0xffffffffu, amax_local);
+    if ((threadIdx.x & 31) == 0 && amax_local) atomicMax(P.amax_out, amax_local);
+  }
+}
+
+// Epilogue of a split reduction: y = ReLU?(sat32(sat32(acc + bias) + residual)), amax.
+__global__ void conv_split_finalize_kernel(const GemmParams P, int64_t total) {
+  const int64_t OHW = (int64_t)P.OH * P.OW;
+  const bool relu = (P.flags & DS_RELU) != 0;
+  const bool resid = (P.flags & DS_RESIDUAL) != 0;
+  uint32_t amax_local = 0;
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t col = (e / OHW) % P.cols;
+    int64_t a = P.split_acc[e] + (P.bias ? (int64_t)__ldg(P.bias + col) : 0);
+    a = a > (int64_t)INT32_MAX ? (int64_t)INT32_MAX : a;
+    a = a < (int64_t)INT32_MIN ? (int64_t)INT32_MIN : a;
+    int32_t o = (int32_t)a;
+    if (resid) o = add_sat(o, __ldg(P.residual + e));
+    if (relu) o = max(o, 0);
+    amax_local = max(amax_local, uabs(o));
+    P.y[e] = o;
   }
   if (P.amax_out != nullptr) {
     amax_local = __reduce_max_sync(0xffffffffu, amax_local);
@@ -369,7 +440,7 @@ __global__ void __launch_bounds__(kThreads, 3) conv_direct_kernel(const GemmPara
 
 struct Choice {
   DirectGeom G;
-  int TM, NT;
+  int TM;
 };
 
 size_t direct_smem_bytes(const DirectGeom& G) {
@@ -378,30 +449,46 @@ size_t direct_smem_bytes(const DirectGeom& G) {
 
 // Tile choice.  TM = 7 when the output width is a multiple of 7 (every
 // ResNet / VGG feature map: 112, 56, 28, 14, 7), else 8.  Groups per row at
-// most 8; rows so that the CTA has 256 threads; 32 channels per CTA, or 64
-// when the pixel tile is too small for 256 threads with 8 channel groups.
-bool choose_geom(const GemmParams& p, Choice& ch) {
+// most 8; TH stacked rows so that the CTA has 256 threads (fewer only when
+// the whole batch has fewer rows).  With split_capacity > 0 the stages are
+// split over CTAs when the grid would not fill every SM slot once (targeting
+// two waves).
+bool choose_geom(const GemmParams& p, size_t split_capacity, Choice& ch) {
   DirectGeom& G = ch.G;
   ch.TM = (p.OW % 7 == 0) ? 7 : 8;
   const int WS = (ch.TM - 1) * p.sw + p.S;
   const int WSP = (WS + 3) / 4 * 4;
-  ch.NT = 32;
   int gw = (p.OW + ch.TM - 1) / ch.TM;
   if (gw > 8) {
     const int pieces = (gw + 7) / 8;
     gw = (gw + pieces - 1) / pieces;
   }
   G.GW = gw;
-  G.TH = kThreads / (G.GW * (ch.NT / TN));
-  if (G.TH > p.OH) {
-    // small image: widen the channel tile instead of idling threads
-    ch.NT = 64;
-    G.TH = kThreads / (G.GW * (ch.NT / TN));
-    if (G.TH < 1 || G.TH > p.OH) return false;
+  G.N = (int)(p.rows / ((int64_t)p.OH * p.OW));
+  const int64_t rows_total = (int64_t)G.N * p.OH;
+  int th = kMaxThreads / (G.GW * CG);
+  if (th < 1) return false;
+  if (rows_total < th) {
+    th = (int)rows_total;
+    while ((th * G.GW) % 4 != 0) ++th;  // whole warps
   }
-  if (G.TH * G.GW * (ch.NT / TN) != kThreads) return false;
-  G.HR = (G.TH - 1) * p.sh + p.R;
-  const int per_c_words = G.HR * G.GW * WSP + 2 * p.R * p.S * ch.NT;
+  G.TH = th;
+  G.threads = G.TH * G.GW * CG;
+  if (G.threads % 32 != 0 || G.threads > kMaxThreads || G.threads < NT) return false;
+  G.HP = p.H + 2 * p.ph;
+  // halo rows: the largest stacked-row span any tile reads (tile starts repeat
+  // with period OH, so OH + 1 starts cover every case)
+  const int64_t tiles_h = (rows_total + G.TH - 1) / G.TH;
+  int64_t span = 0;
+  for (int64_t k = 0; k < tiles_h && k <= p.OH; ++k) {
+    const int64_t a = k * G.TH, z = std::min(a + G.TH, rows_total) - 1;
+    const int64_t sa = (a / p.OH) * G.HP + (a % p.OH) * p.sh;
+    const int64_t sz = (z / p.OH) * G.HP + (z % p.OH) * p.sh;
+    span = std::max(span, sz - sa + p.R);
+  }
+  if (span > 4096) return false;
+  G.HR = (int)span;
+  const int per_c_words = G.HR * G.GW * WSP + 2 * p.R * p.S * NT;
   int cc = kSmemBudget / (2 * 4 * per_c_words);
   if (cc < 1) return false;
   if (cc > p.C) cc = p.C;
@@ -414,45 +501,61 @@ bool choose_geom(const GemmParams& p, Choice& ch) {
   G.taps = G.CC * p.R * p.S;
   G.n_stages = (p.C + G.CC - 1) / G.CC;
   G.halo_words = G.CC * G.HR * G.GW * WSP;
-  G.code_words = G.taps * 2 * ch.NT;
-  int run = (G.taps * ch.NT + kThreads - 1) / kThreads;  // decode: at most one item per thread
+  G.code_words = G.taps * 2 * NT;
+  int run = (G.taps * NT + G.threads - 1) / G.threads;  // decode: at most one item per thread
   if (run < 1) run = 1;
-  if (run > 16) return false;
+  if (run > 16 && p.xcodes == nullptr) return false;
   G.run = run;
   G.tiles_w = (p.OW + ch.TM * G.GW - 1) / (ch.TM * G.GW);
-  G.tiles_h = (p.OH + G.TH - 1) / G.TH;
+  G.tiles_h = (int)tiles_h;
+  // split the stages when the grid would not fill every SM slot once
+  G.splits = 1;
+  G.stages_per_split = G.n_stages;
+  const int64_t ctas = (int64_t)G.tiles_w * G.tiles_h * ((p.cols + NT - 1) / NT);
+  const size_t need = (size_t)p.rows * p.cols * sizeof(int64_t);
+  if (split_capacity >= need && ctas < kSlots && G.n_stages > 1) {
+    int want = (int)std::min<int64_t>(G.n_stages, (2 * kSlots + ctas - 1) / ctas);
+    G.stages_per_split = (G.n_stages + want - 1) / want;
+    G.splits = (G.n_stages + G.stages_per_split - 1) / G.stages_per_split;
+  }
   return direct_smem_bytes(G) <= (size_t)kSmemBudget;
 }
 
-template <int SIG, int S, int TM, int NT>
+template <int SIG, int S, int TM>
 cudaError_t launch_direct(const GemmParams& p, const DirectGeom& G, cudaStream_t st) {
   const size_t smem = direct_smem_bytes(G);
   // raise the dynamic shared-memory limit once per process (not a stream operation, so a
   // forward captured in a CUDA graph after a first eager call issues no attribute call)
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(conv_direct_kernel<SIG, S, TM, NT>,
+    cudaError_t e = cudaFuncSetAttribute(conv_direct_kernel<SIG, S, TM>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  const int64_t n_img = p.rows / ((int64_t)p.OH * p.OW);
-  const int64_t nb = (int64_t)G.tiles_w * G.tiles_h * n_img;
-  dim3 grid((unsigned)nb, (unsigned)((p.cols + NT - 1) / NT));
-  conv_direct_kernel<SIG, S, TM, NT><<<grid, kThreads, smem, st>>>(p, G);
+  GemmParams q = p;
+  if (G.splits > 1) {
+    cudaError_t e = cudaMemsetAsync(q.split_acc, 0, (size_t)p.rows * p.cols * sizeof(int64_t), st);
+    if (e != cudaSuccess) return e;
+  } else {
+    q.split_acc = nullptr;
+  }
+  dim3 grid((unsigned)((int64_t)G.tiles_w * G.tiles_h), (unsigned)((p.cols + NT - 1) / NT), (unsigned)G.splits);
+  conv_direct_kernel<SIG, S, TM><<<grid, G.threads, smem, st>>>(q, G);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess || G.splits == 1) return e;
+  const int64_t total = p.rows * p.cols;
+  int64_t blocks = (total + 255) / 256;
+  if (blocks > kSlots * 8) blocks = kSlots * 8;
+  conv_split_finalize_kernel<<<(unsigned)blocks, 256, 0, st>>>(q, total);
   return cudaGetLastError();
 }
 
-template <int SIG, int TM, int NT>
-cudaError_t launch_by_s(const GemmParams& p, const DirectGeom& G, cudaStream_t st) {
-  if (p.S == 1) return launch_direct<SIG, 1, TM, NT>(p, G, st);
-  if (p.S == 3) return launch_direct<SIG, 3, TM, NT>(p, G, st);
-  return launch_direct<SIG, 7, TM, NT>(p, G, st);
-}
-
 template <int SIG, int TM>
-cudaError_t launch_by_nt(const GemmParams& p, const Choice& ch, cudaStream_t st) {
-  return ch.NT == 32 ? launch_by_s<SIG, TM, 32>(p, ch.G, st) : launch_by_s<SIG, TM, 64>(p, ch.G, st);
+cudaError_t launch_by_s(const GemmParams& p, const DirectGeom& G, cudaStream_t st) {
+  if (p.S == 1) return launch_direct<SIG, 1, TM>(p, G, st);
+  if (p.S == 3) return launch_direct<SIG, 3, TM>(p, G, st);
+  return launch_direct<SIG, 7, TM>(p, G, st);
 }
 
 }  // namespace
@@ -462,14 +565,21 @@ bool conv_direct_supported(const GemmParams& p) {
   if (!(p.S == 1 || p.S == 3 || p.S == 7) || p.R != p.S) return false;
   if ((p.rows / ((int64_t)p.OH * p.OW)) >= ((int64_t)1 << 24)) return false;
   Choice ch;
-  return choose_geom(p, ch);
+  return choose_geom(p, p.split_acc ? p.split_capacity : 0, ch);
+}
+
+size_t conv_split_bytes(const GemmParams& p) {
+  if (!conv_direct_supported(p)) return 0;
+  Choice ch;
+  if (!choose_geom(p, ~(size_t)0, ch) || ch.G.splits <= 1) return 0;
+  return (size_t)p.rows * p.cols * sizeof(int64_t);
 }
 
 cudaError_t launch_conv2d_direct(const GemmParams& p, cudaStream_t st) {
   Choice ch;
-  if (!choose_geom(p, ch)) return cudaErrorInvalidConfiguration;
-  if (ch.TM == 7) return p.sh == 1 ? launch_by_nt<1, 7>(p, ch, st) : launch_by_nt<2, 7>(p, ch, st);
-  return p.sh == 1 ? launch_by_nt<1, 8>(p, ch, st) : launch_by_nt<2, 8>(p, ch, st);
+  if (!choose_geom(p, p.split_acc ? p.split_capacity : 0, ch)) return cudaErrorInvalidConfiguration;
+  if (ch.TM == 7) return p.sh == 1 ? launch_by_s<1, 7>(p, ch.G, st) : launch_by_s<2, 7>(p, ch.G, st);
+  return p.sh == 1 ? launch_by_s<1, 8>(p, ch.G, st) : launch_by_s<2, 8>(p, ch.G, st);
 }
 
 }  // namespace ds

@@ -73,6 +73,9 @@ struct GemmParams {
   // conv geometry (unused by FC)
   int C, H, W, R, S, sh, sw, ph, pw, OH, OW;
   uint32_t flags;
+  // split reduction (conv, chained forward only): int64 partial sums of every output, zeroed first
+  int64_t* split_acc;       // nullable
+  size_t split_capacity;    // bytes available at split_acc
 };
 
 // Launchers (defined in shift_gemm.cu).
@@ -80,6 +83,7 @@ cudaError_t launch_linear_shift(const GemmParams& p, cudaStream_t st);
 cudaError_t launch_conv2d_shift(const GemmParams& p, cudaStream_t st);
 // Defined in conv_direct.cu.
 bool conv_direct_supported(const GemmParams& p);
+size_t conv_split_bytes(const GemmParams& p);  // int64 scratch a split reduction would use (0: no split)
 cudaError_t launch_conv2d_direct(const GemmParams& p, cudaStream_t st);
 // Defined in linear_bf16.cu.
 int64_t bf16_kpad(int64_t k_red);
@@ -96,7 +100,9 @@ cudaError_t launch_avgpool_floor(const int32_t* x, int32_t* y, int64_t planes, i
 ds_status check_weights(const ds_weights* w, int64_t n_out, int64_t k_red);
 ds_status conv_launch(const int32_t* x, const ds_weights* w, const int32_t* bias, const int32_t* residual,
                       int32_t* y, int N, int C, int H, int W, int K, int R, int S, int stride, int pad,
-                      uint32_t flags, const uint32_t* amax_in, uint32_t* amax_out, cudaStream_t st);
+                      uint32_t flags, const uint32_t* amax_in, uint32_t* amax_out, cudaStream_t st,
+                      int64_t* split_acc = nullptr, size_t split_capacity = 0);
+GemmParams conv_params(const ds_weights* w, int N, int C, int H, int W, int K, int R, int S, int stride, int pad);
 ds_status fc_launch(const int32_t* x, const ds_weights* w, const int32_t* bias, int32_t* y, int64_t M,
                     int64_t K, int64_t N, uint32_t flags, const uint32_t* amax_in, uint32_t* amax_out,
                     cudaStream_t st);

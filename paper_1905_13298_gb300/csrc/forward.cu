@@ -26,6 +26,7 @@ struct Plan {
   std::vector<int64_t> slot_elems;  // per slot, per image (slots >= 2)
   std::vector<size_t> slot_off;   // byte offsets in the workspace
   size_t amax_bytes = 0;
+  size_t split_bytes = 0;  // int64 scratch of split reductions (largest layer)
   size_t total = 0;
   int n_slots = 0;
 };
@@ -65,6 +66,8 @@ ds_status plan_program(const ds_layer* L, int n, int batch, Plan& P) {
         ds_status r = check_weights(l.w, l.K, (int64_t)l.C * l.R * l.S);
         if (r != DS_OK) return r;
         out = Shape{l.K, (l.H + 2 * l.pad - l.R) / l.stride + 1, (l.W + 2 * l.pad - l.S) / l.stride + 1};
+        P.split_bytes = std::max(P.split_bytes,
+                                 conv_split_bytes(conv_params(l.w, batch, l.C, l.H, l.W, l.K, l.R, l.S, l.stride, l.pad)));
         break;
       }
       case DS_OP_FC: {
@@ -108,8 +111,9 @@ ds_status plan_program(const ds_layer* L, int n, int batch, Plan& P) {
   }
   if (!wrote_y) return fail(DS_ERR_INVALID_ARG, "no layer writes the output slot 1");
   P.amax_bytes = ((size_t)(n + 1) * sizeof(uint32_t) + 255) / 256 * 256;
+  P.split_bytes = (P.split_bytes + 255) / 256 * 256;
   P.slot_off.assign(P.n_slots, 0);
-  size_t off = P.amax_bytes;
+  size_t off = P.amax_bytes + P.split_bytes;
   for (int s = 2; s < P.n_slots; ++s) {
     P.slot_off[s] = off;
     off += ((size_t)P.slot_elems[s] * batch * sizeof(int32_t) + 255) / 256 * 256;
@@ -167,7 +171,8 @@ ds_status ds_shift_forward(const ds_layer* L, int n, const int32_t* x, int32_t* 
     switch (l.op) {
       case DS_OP_CONV:
         r = conv_launch(xin, l.w, l.bias, l.aux >= 0 ? slot_ptr[l.aux] : nullptr, yout, batch, l.C, l.H, l.W,
-                        l.K, l.R, l.S, l.stride, l.pad, l.flags, slot_amax[l.in], amax + i, st);
+                        l.K, l.R, l.S, l.stride, l.pad, l.flags, slot_amax[l.in], amax + i, st,
+                        P.split_bytes ? reinterpret_cast<int64_t*>(base + P.amax_bytes) : nullptr, P.split_bytes);
         slot_amax[l.out] = amax + i;
         break;
       case DS_OP_FC:

@@ -139,8 +139,16 @@ __global__ void absmax_kernel(const int32_t* __restrict__ x, int64_t n, uint32_t
   } else {
     for (int64_t i = tid; i < n; i += stride) m = max(m, uabs32(x[i]));
   }
+  // block reduction, then one atomic per block
+  __shared__ uint32_t wmax[32];
   m = __reduce_max_sync(0xffffffffu, m);
-  if ((threadIdx.x & 31) == 0 && m) atomicMax(out, m);
+  if ((threadIdx.x & 31) == 0) wmax[threadIdx.x >> 5] = m;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    uint32_t v = threadIdx.x < (blockDim.x >> 5) ? wmax[threadIdx.x] : 0u;
+    v = __reduce_max_sync(0xffffffffu, v);
+    if (threadIdx.x == 0 && v) atomicMax(out, v);
+  }
 }
 
 cudaError_t launch_absmax(const int32_t* x, int64_t n, uint32_t* out, cudaStream_t st) {

@@ -63,3 +63,24 @@ def test_resnet18_full_size_batch1(dslib):
     params = si.network_params(prog[1], si.SEED_BASE + 3)
     x = si.image_batch(si.SEED_BASE + 3, 1)
     assert np.array_equal(_run(prog, params, x), ON.resnet_forward(x, params, "resnet18"))
+
+
+@pytest.mark.parametrize("batch", [1, 3])
+def test_resnet18_small_batches_split_reduction(dslib, batch):
+    """Small batches: tiles span image boundaries and small layers split their reduction (int64 partials)."""
+    from paper_1905_13298_gb300 import networks as PN
+    prog = PN.resnet_program("resnet18", 64, 64)
+    params = si.network_params(prog[1], 500 + batch)
+    x = si.image_batch(11 + batch, batch, 3, 64, 64)
+    assert np.array_equal(_run(prog, params, x), ON.resnet_forward(x, params, "resnet18"))
+
+
+def test_resnet18_stress_codes_small_batch(dslib):
+    """Saturating codes at batch 1: the split reduction takes the 64-bit path and saturates exactly."""
+    from paper_1905_13298_gb300 import networks as PN
+    prog = PN.resnet_program("resnet18", 32, 32)
+    params = []
+    for i, shp in enumerate(prog[1]):
+        params.append((si.sign_codes(600 + i, shp), si.shift_codes_geometric(600 + i, shp, -6), si.bias(600 + i, shp[0])))
+    x = si.image_batch(12, 1, 3, 32, 32)
+    assert np.array_equal(_run(prog, params, x), ON.resnet_forward(x, params, "resnet18"))
