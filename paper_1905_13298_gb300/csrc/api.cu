@@ -125,8 +125,13 @@ ds_status conv_launch(const int32_t* x, const ds_weights* w, const int32_t* bias
   p.amax_out = amax_out;
   p.split_acc = split_acc;
   p.split_capacity = split_capacity;
-  if (!(flags & DS_CONV_IM2COL) && conv_direct_supported(p))
-    return cuda_check(launch_conv2d_direct(p, st), "conv2d_shift (direct) launch");
+  if (!(flags & DS_CONV_IM2COL)) {
+    if (conv_pointwise_supported(p)) {
+      p.split_acc = nullptr;
+      return cuda_check(launch_conv2d_pointwise(p, st), "conv2d_shift (pointwise) launch");
+    }
+    if (conv_direct_supported(p)) return cuda_check(launch_conv2d_direct(p, st), "conv2d_shift (direct) launch");
+  }
   p.split_acc = nullptr;
   return cuda_check(launch_conv2d_shift(p, st), "conv2d_shift (implicit GEMM) launch");
 }
@@ -375,8 +380,11 @@ ds_status ds_conv2d_shift(const int32_t* x, const ds_weights* w, const int32_t* 
   fill_blob_offsets(p, w);
   r = prepare_amax(x, nx, flags, amax_io, st, p);
   if (r != DS_OK) return r;
-  if (!(flags & DS_CONV_IM2COL) && conv_direct_supported(p))
-    return cuda_check(launch_conv2d_direct(p, st), "conv2d_shift (direct) launch");
+  if (!(flags & DS_CONV_IM2COL)) {
+    if (conv_pointwise_supported(p))
+      return cuda_check(launch_conv2d_pointwise(p, st), "conv2d_shift (pointwise) launch");
+    if (conv_direct_supported(p)) return cuda_check(launch_conv2d_direct(p, st), "conv2d_shift (direct) launch");
+  }
   return cuda_check(launch_conv2d_shift(p, st), "conv2d_shift (implicit GEMM) launch");
 }
 

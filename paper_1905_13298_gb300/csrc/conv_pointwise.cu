@@ -1,0 +1,316 @@
+// Pointwise (1x1) ConvShift as a shift GEMM over pixels (DeepShift Eq. 1-3).
+//
+//   y[n][k][oh][ow] = sat32( b[k] + sum_c s[k][c] * (x[n][c][oh*sig][ow*sig] >> -p[k][c]) )
+//
+// A 1x1 convolution has no window to reuse, so it runs as a GEMM whose rows
+// are output pixels (all images), columns are output channels and whose
+// reduction runs over input channels.  The activation tile of a stage is
+// staged channel-major ([32 channels][128 pixels]): for stride 1 every
+// 16-byte chunk of 4 pixels is one cp.async, for stride 2 four 4-byte copies.
+// A thread owns 8 pixels (two quads 64 apart, so a warp's 16-byte loads are
+// contiguous) and 8 channels; per term the hot loop is one SHF and one IMAD.
+// Codes come from the expanded execution layout (cp.async) or are decoded
+// from the packed blob per stage.  Accumulator width as in shift_gemm.cu.
+#include "ds_common.cuh"
+
+namespace ds {
+namespace {
+
+constexpr int MT = 128;       // pixels per CTA
+constexpr int NT = 64;        // channels per CTA
+constexpr int TN = 8;         // channels per thread
+constexpr int THREADS = 128;  // 16 pixel groups x 8 channel groups
+constexpr int KC = 32;        // input channels per stage (= one packed chunk)
+
+struct __align__(16) PwSmem {
+  int32_t xs[2][KC * MT];
+  int32_t cs[2][KC * 2 * NT];  // per input channel: 2 blocks of {32 shifts, 32 signs}
+};
+
+__device__ __forceinline__ void cp_async4(void* smem_dst, const void* gsrc, bool valid) {
+  const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(d), "l"(gsrc), "r"(valid ? 4 : 0));
+}
+__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gsrc, bool valid) {
+  const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(gsrc), "r"(valid ? 16 : 0));
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::); }
+__device__ __forceinline__ int32_t add_sat(int32_t a, int32_t b) {
+  int32_t r;
+  asm("add.sat.s32 %0, %1, %2;\n" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+__device__ __forceinline__ uint32_t uabs(int32_t v) { return v < 0 ? (uint32_t)0 - (uint32_t)v : (uint32_t)v; }
+
+// This thread's staging assignment: pixel quad q = t % 32 of the tile, input
+// channels t / 32 + 4 j.  Input offsets of the quad's 4 pixels (channel 0).
+struct QuadCtx {
+  int64_t off[4];
+  bool valid[4];
+  bool vec;  // the 4 pixels are consecutive and 16-byte aligned in memory
+};
+
+template <bool STRIDED>
+__device__ __forceinline__ QuadCtx quad_ctx(const GemmParams& P, int64_t m0) {
+  QuadCtx q;
+  const int64_t OHW = (int64_t)P.OH * P.OW;
+  const int64_t CHW = (int64_t)P.C * P.H * P.W;
+  const int64_t mq = m0 + 4 * (threadIdx.x & 31);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int64_t m = mq + i;
+    q.valid[i] = m < P.rows;
+    const int64_t n = q.valid[i] ? m / OHW : 0;
+    const int64_t pix = q.valid[i] ? m - n * OHW : 0;
+    if constexpr (STRIDED) {
+      const int oh = (int)(pix / P.OW), ow = (int)(pix - (pix / P.OW) * P.OW);
+      q.off[i] = n * CHW + (int64_t)oh * P.sh * P.W + (int64_t)ow * P.sw;
+    } else {
+      q.off[i] = n * CHW + pix;
+    }
+  }
+  // 16-byte copies need every channel's quad aligned: offset and channel stride multiples of 4 words
+  q.vec = !STRIDED && q.valid[3] && (q.off[3] == q.off[0] + 3) && ((q.off[0] & 3) == 0) &&
+          ((((int64_t)P.H * P.W) & 3) == 0) && ((reinterpret_cast<uintptr_t>(P.x) & 15) == 0);
+  return q;
+}
+
+template <bool STRIDED>
+__device__ __forceinline__ void stage_x(const GemmParams& P, int32_t* xs, const QuadCtx& q, int c0) {
+  const int64_t HW = (int64_t)P.H * P.W;
+  const int qi = threadIdx.x & 31;
+#pragma unroll
+  for (int j = 0; j < KC / 4; ++j) {
+    const int cl = (threadIdx.x >> 5) + 4 * j;
+    const int c = c0 + cl;
+    int32_t* dst = xs + cl * MT + 4 * qi;
+    const bool cok = c < P.C;
+    if (!STRIDED && q.vec) {
+      cp_async16(dst, cok ? (const void*)(P.x + q.off[0] + c * HW) : (const void*)P.x, cok);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const bool ok = cok && q.valid[i];
+        cp_async4(dst + i, ok ? (const void*)(P.x + q.off[i] + c * HW) : (const void*)P.x, ok);
+      }
+    }
+  }
+}
+
+// Codes of input channels [c0, c0 + KC) for columns [col0, col0 + 64).
+__device__ __forceinline__ void stage_codes_expanded(const GemmParams& P, int32_t* cs, int64_t col0, int c0) {
+  const int64_t nblocks = (P.cols + 31) / 32;
+  // 2 blocks x 32 channels x 16 pieces of 16 bytes
+  for (int e = threadIdx.x; e < 2 * KC * 16; e += THREADS) {
+    const int b = e / (KC * 16);
+    const int r = e - b * KC * 16;
+    const int cl = r >> 4, q = r & 15;
+    const int64_t cb = col0 / 32 + b;
+    const bool ok = cb < nblocks && c0 + cl < P.kred;
+    const int32_t* src = ok ? P.xcodes + ((cb * P.kred + c0 + cl) * 64 + q * 4) : P.xcodes;
+    cp_async16(cs + (cl * 2 + b) * 64 + q * 4, src, ok);
+  }
+}
+
+// Blob path: thread t decodes 16 reduction indices of column t % 64.
+__device__ __forceinline__ void decode_codes(const GemmParams& P, int32_t* cs, int64_t col0, int64_t g) {
+  const int t = threadIdx.x;
+  const int n = t & 63;
+  const int h = t >> 6;
+  const int64_t col = col0 + n;
+  uint2 nib = make_uint2(0u, 0u), bits = make_uint2(0u, 0u);
+  if (col < P.cols) {
+    const int64_t rec = g * P.cols + col;
+    nib = __ldg(reinterpret_cast<const uint2*>(P.blob + P.off_nib + rec * 16 + h * 8));
+    bits = __ldg(reinterpret_cast<const uint2*>(P.blob + P.off_bits + rec * 8));
+  }
+  int32_t* base = cs + (n >> 5) * 64 + (n & 31);
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    const int k = 16 * h + i;
+    const uint32_t w = i < 8 ? nib.x : nib.y;
+    base[k * 2 * NT] = (int)((w >> (4 * (i & 7))) & 15u);
+    base[k * 2 * NT + 32] = (int)((bits.y >> k) & 1u) - 2 * (int)((bits.x >> k) & 1u);
+  }
+}
+
+template <int I0, int NI, typename Acc>
+__device__ __forceinline__ void compute_stage(const int32_t* xs, const int32_t* cs, int tm, int tn,
+                                              Acc (&acc)[NI][TN]) {
+  const int32_t* cbase = cs + (tn >> 2) * 64 + (tn & 3) * TN;
+#pragma unroll 4
+  for (int k = 0; k < KC; ++k) {
+    int x[8];
+    {
+      const int4 a = *reinterpret_cast<const int4*>(xs + k * MT + 4 * tm);
+      const int4 b = *reinterpret_cast<const int4*>(xs + k * MT + 64 + 4 * tm);
+      x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w;
+      x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
+    }
+    const int4 s0 = *reinterpret_cast<const int4*>(cbase + k * 2 * NT);
+    const int4 s1 = *reinterpret_cast<const int4*>(cbase + k * 2 * NT + 4);
+    const int4 g0 = *reinterpret_cast<const int4*>(cbase + k * 2 * NT + 32);
+    const int4 g1 = *reinterpret_cast<const int4*>(cbase + k * 2 * NT + 36);
+    const int sh[TN] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+    const int sg[TN] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+#pragma unroll
+    for (int i = 0; i < NI; ++i) {
+      const int xv = x[I0 + i];
+#pragma unroll
+      for (int j = 0; j < TN; ++j) {
+        const int t = xv >> sh[j];  // Eq. 1
+        if constexpr (sizeof(Acc) == 4) {
+          acc[i][j] += (uint32_t)sg[j] * (uint32_t)t;  // Eq. 2 + accumulate (mod 2^32)
+        } else {
+          acc[i][j] += (int64_t)sg[j] * (int64_t)t;
+        }
+      }
+    }
+  }
+}
+
+template <bool STRIDED, int I0, int NI, typename Acc>
+__device__ __forceinline__ void run_tile(const GemmParams& P, PwSmem& sm, int64_t m0, int64_t col0,
+                                         const QuadCtx& q, uint32_t& amax_local) {
+  const int t = threadIdx.x;
+  const int tm = t & 15, tn = t >> 4;
+  const bool expanded = P.xcodes != nullptr;
+  Acc acc[NI][TN];
+#pragma unroll
+  for (int i = 0; i < NI; ++i)
+#pragma unroll
+    for (int j = 0; j < TN; ++j) acc[i][j] = 0;
+
+  const int nst = (P.C + KC - 1) / KC;
+  stage_x<STRIDED>(P, sm.xs[0], q, 0);
+  if (expanded) stage_codes_expanded(P, sm.cs[0], col0, 0);
+  cp_async_commit();
+  if (!expanded) decode_codes(P, sm.cs[0], col0, 0);
+  cp_async_wait_all();
+  for (int st = 0; st < nst; ++st) {
+    const int b = st & 1;
+    const bool more = st + 1 < nst;
+    __syncthreads();
+    if (more) {
+      stage_x<STRIDED>(P, sm.xs[b ^ 1], q, (st + 1) * KC);
+      if (expanded) stage_codes_expanded(P, sm.cs[b ^ 1], col0, (st + 1) * KC);
+      cp_async_commit();
+    }
+    compute_stage<I0, NI, Acc>(sm.xs[b], sm.cs[b], tm, tn, acc);
+    if (more) {
+      if (!expanded) decode_codes(P, sm.cs[b ^ 1], col0, st + 1);
+      cp_async_wait_all();
+    }
+  }
+  __syncthreads();  // a second pass (64-bit path) reuses the buffers
+
+  // fused epilogue: bias, saturation (64-bit path), residual, ReLU, amax
+  const bool relu = (P.flags & DS_RELU) != 0;
+  const bool resid = (P.flags & DS_RESIDUAL) != 0;
+  const int64_t OHW = (int64_t)P.OH * P.OW;
+  int32_t bcol[TN];
+#pragma unroll
+  for (int j = 0; j < TN; ++j) {
+    const int64_t col = col0 + tn * TN + j;
+    bcol[j] = (P.bias != nullptr && col < P.cols) ? __ldg(P.bias + col) : 0;
+  }
+#pragma unroll
+  for (int i = 0; i < NI; ++i) {
+    const int li = I0 + i;
+    const int64_t m = m0 + 4 * tm + (li & 3) + 64 * (li >> 2);
+    if (m >= P.rows) continue;
+    const int64_t n = m / OHW;  // once per pixel
+    const int64_t base = n * P.cols * OHW + (m - n * OHW);
+#pragma unroll
+    for (int j = 0; j < TN; ++j) {
+      const int64_t col = col0 + tn * TN + j;
+      if (col >= P.cols) continue;
+      const int64_t idx = base + col * OHW;
+      int32_t o;
+      if constexpr (sizeof(Acc) == 4) {
+        o = (int32_t)(acc[i][j] + (uint32_t)bcol[j]);
+      } else {
+        int64_t a = acc[i][j] + (int64_t)bcol[j];
+        a = a > (int64_t)INT32_MAX ? (int64_t)INT32_MAX : a;
+        a = a < (int64_t)INT32_MIN ? (int64_t)INT32_MIN : a;
+        o = (int32_t)a;
+      }
+      if (resid) o = add_sat(o, __ldg(P.residual + idx));
+      if (relu) o = max(o, 0);
+      amax_local = max(amax_local, uabs(o));
+      P.y[idx] = o;
+    }
+  }
+}
+
+__device__ __forceinline__ bool tile_int32_exact(const GemmParams& P, int64_t col0) {
+  bool unsafe = false;
+  const int t = threadIdx.x;
+  if (P.amax_in == nullptr || (P.flags & DS_FORCE_INT64)) {
+    unsafe = true;
+  } else if (t < NT) {
+    const int64_t col = col0 + t;
+    if (col < P.cols) {
+      const unsigned long long amax = *P.amax_in;
+      const unsigned long long A = reinterpret_cast<const unsigned long long*>(P.blob + P.off_cola)[col];
+      const unsigned long long nnz = reinterpret_cast<const uint32_t*>(P.blob + P.off_nnz)[col];
+      const unsigned long long b = P.bias ? (unsigned long long)uabs(P.bias[col]) : 0ull;
+      const unsigned long long hi = __umul64hi(amax, A);
+      const unsigned long long lo = amax * A;
+      unsafe = (hi != 0ull || lo > ~0ull - 32767ull) ? true
+                                                     : (((lo + 32767ull) >> 15) + nnz + b) > (unsigned long long)INT32_MAX;
+    }
+  }
+  return !__syncthreads_or(unsafe);
+}
+
+template <bool STRIDED>
+__global__ void __launch_bounds__(THREADS, 3) conv_pointwise_kernel(const GemmParams P) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  PwSmem& sm = *reinterpret_cast<PwSmem*>(smem_raw);
+  const int64_t m0 = (int64_t)blockIdx.x * MT;
+  const int64_t col0 = (int64_t)blockIdx.y * NT;
+  const QuadCtx q = quad_ctx<STRIDED>(P, m0);
+  uint32_t amax_local = 0;
+  if (tile_int32_exact(P, col0)) {
+    run_tile<STRIDED, 0, 8, uint32_t>(P, sm, m0, col0, q, amax_local);
+  } else {
+    run_tile<STRIDED, 0, 4, int64_t>(P, sm, m0, col0, q, amax_local);
+    run_tile<STRIDED, 4, 4, int64_t>(P, sm, m0, col0, q, amax_local);
+  }
+  if (P.amax_out != nullptr) {
+    amax_local = __reduce_max_sync(0xffffffffu, amax_local);
+    if ((threadIdx.x & 31) == 0 && amax_local) atomicMax(P.amax_out, amax_local);
+  }
+}
+
+template <bool STRIDED>
+cudaError_t launch_pw(const GemmParams& p, cudaStream_t st) {
+  const size_t smem = sizeof(PwSmem);
+  static bool attr_set = false;  // once per process (see conv_direct.cu)
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(conv_pointwise_kernel<STRIDED>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  dim3 grid((unsigned)((p.rows + MT - 1) / MT), (unsigned)((p.cols + NT - 1) / NT));
+  conv_pointwise_kernel<STRIDED><<<grid, THREADS, smem, st>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+bool conv_pointwise_supported(const GemmParams& p) {
+  return p.R == 1 && p.S == 1 && p.ph == 0 && p.pw == 0 && p.sh >= 1 && p.sw >= 1 && p.cols <= 65535LL * NT &&
+         p.rows < ((int64_t)1 << 40);
+}
+
+cudaError_t launch_conv2d_pointwise(const GemmParams& p, cudaStream_t st) {
+  const bool strided = p.sh != 1 || p.sw != 1;
+  return strided ? launch_pw<true>(p, st) : launch_pw<false>(p, st);
+}
+
+}  // namespace ds

@@ -84,6 +84,9 @@ cudaError_t launch_conv2d_shift(const GemmParams& p, cudaStream_t st);
 // Defined in conv_direct.cu.
 bool conv_direct_supported(const GemmParams& p);
 size_t conv_split_bytes(const GemmParams& p);  // int64 scratch a split reduction would use (0: no split)
+// Defined in conv_pointwise.cu (1x1 convolutions as a GEMM over pixels).
+bool conv_pointwise_supported(const GemmParams& p);
+cudaError_t launch_conv2d_pointwise(const GemmParams& p, cudaStream_t st);
 cudaError_t launch_conv2d_direct(const GemmParams& p, cudaStream_t st);
 // Defined in linear_bf16.cu.
 int64_t bf16_kpad(int64_t k_red);
