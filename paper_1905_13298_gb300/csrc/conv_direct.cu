@@ -197,7 +197,7 @@ __device__ __forceinline__ void compute_stage(const DirectGeom G, const int32_t*
   constexpr int R = S;  // square kernels
   constexpr int TAPW = 2 * NT;  // words per tap row
   const int cstride = G.HR * rowstride;
-#pragma unroll 1
+#pragma unroll 2
   for (int cl = 0; cl < G.CC; ++cl) {
 #pragma unroll
     for (int r = 0; r < R; ++r) {
@@ -217,12 +217,12 @@ __device__ __forceinline__ void compute_stage(const DirectGeom G, const int32_t*
         const int4 sgv = *reinterpret_cast<const int4*>(cp + (r * S + s) * TAPW + 32);
         const int sh[TN] = {shv.x, shv.y, shv.z, shv.w};
         const int sg[TN] = {sgv.x, sgv.y, sgv.z, sgv.w};
+        // channel-outer order: consecutive SHF / IMAD share their shift / sign operand
 #pragma unroll
-        for (int i = 0; i < NI; ++i) {
-          const int xv = w[(I0 + i) * SIG + s];
+        for (int j = 0; j < TN; ++j) {
 #pragma unroll
-          for (int j = 0; j < TN; ++j) {
-            const int t = xv >> sh[j];  // Eq. 1
+          for (int i = 0; i < NI; ++i) {
+            const int t = w[(I0 + i) * SIG + s] >> sh[j];  // Eq. 1
             if constexpr (sizeof(Acc) == 4) {
               acc[i][j] += (uint32_t)sg[j] * (uint32_t)t;  // Eq. 2 + accumulate (mod 2^32)
             } else {

@@ -14,9 +14,9 @@ import subprocess
 HERE = os.path.dirname(os.path.abspath(__file__))
 SRC = os.path.join(HERE, "int_issue_rate.cu")
 LIB = os.path.join(HERE, "libds_intpeak.so")
-KINDS = {0: "SHF", 1: "IMAD", 2: "SHF+IMAD", 3: "IADD", 4: "LOP"}
+KINDS = {0: "SHF", 1: "IMAD", 2: "SHF+IMAD", 3: "IADD", 4: "LOP", 5: "IMAD.HI", 6: "ADD+ADD"}
 # instructions per inner iteration: 64 of the mix (128 for SHF+IMAD) + 8 x-updates
-INSTR_PER_ITER = {0: 72, 1: 72, 2: 136, 3: 72, 4: 72}
+INSTR_PER_ITER = {0: 72, 1: 72, 2: 136, 3: 72, 4: 72, 5: 72, 6: 136}
 
 
 def build() -> str:

@@ -10,6 +10,8 @@
 //   kind 2: SHF + IMAD      (the shift-GEMM inner loop: t = x >> s; acc += g * t)
 //   kind 3: IADD3 only      (add.s32 chains)
 //   kind 4: LOP3 only       (xor/and chains)
+//   kind 5: IMAD.HI only    (mad.hi.s32: high word of x * m plus acc)
+//   kind 6: IADD3 pairs     (acc = acc + a + b, three-input adds)
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -44,6 +46,10 @@ __global__ void __launch_bounds__(256) mix_kernel(const int* __restrict__ seed, 
           asm volatile("mad.lo.s32 %0, %1, %2, %0;" : "+r"(acc[i][j]) : "r"(g[j]), "r"(t));
         } else if (KIND == 3) {
           asm volatile("add.s32 %0, %0, %1;" : "+r"(acc[i][j]) : "r"(x[i]));
+        } else if (KIND == 5) {
+          asm volatile("mad.hi.s32 %0, %1, %2, %0;" : "+r"(acc[i][j]) : "r"(x[i]), "r"(g[j]));
+        } else if (KIND == 6) {
+          asm volatile("{\n\t.reg .s32 t;\n\tadd.s32 t, %1, %2;\n\tadd.s32 %0, %0, t;\n\t}" : "+r"(acc[i][j]) : "r"(x[i]), "r"(g[j]));
         } else {
           asm volatile("xor.b32 %0, %0, %1;" : "+r"(acc[i][j]) : "r"(g[j]));
         }
@@ -77,6 +83,8 @@ extern "C" int ds_probe_int_mix(int kind, int blocks, int threads, int iters, co
     case 1: mix_kernel<1><<<blocks, threads>>>(seed, iters, out, cycles); break;
     case 2: mix_kernel<2><<<blocks, threads>>>(seed, iters, out, cycles); break;
     case 3: mix_kernel<3><<<blocks, threads>>>(seed, iters, out, cycles); break;
+    case 5: mix_kernel<5><<<blocks, threads>>>(seed, iters, out, cycles); break;
+    case 6: mix_kernel<6><<<blocks, threads>>>(seed, iters, out, cycles); break;
     default: mix_kernel<4><<<blocks, threads>>>(seed, iters, out, cycles); break;
   }
   cudaEventRecord(b);
