@@ -7,8 +7,9 @@
 // group (TM pixels of one row) and TN = 4 channels.  Per chunk of CC input
 // channels (one pipeline stage) the CTA stages into shared memory
 //   * the input window of every group, zero outside the image, as a "slot"
-//     of WSP words (WS = (TM-1)*sig + S values, padded to 16 bytes), so that
-//     a thread reads the window of one kernel row with WSP/4 vector loads;
+//     of WSP words (WS = (TM-1)*sig + S values, padded to 16 bytes and to a
+//     stride of 4 mod 8 words), so that a thread reads the window of one
+//     kernel row with ceil(WS/4) vector loads;
 //   * the codes of the chunk's taps as 32-bit shift / sign words, one row of
 //     NT channels per tap: copied with 16-byte cp.async from the expanded
 //     execution layout when the layer has one, else decoded from the packed
@@ -40,6 +41,24 @@ constexpr int kSlots = 152 * 3;         // resident CTAs on a GB300
 // n * HP + ihp (HP = H + 2 * pad); output row (n, oh) reads stacked rows
 // n * HP + oh * sig + r.  A tile's halo is the contiguous stacked range its
 // rows read, HR rows at most.
+// Division by a runtime constant d >= 1 of numerators 0 <= n < 2^31 as one
+// widening multiply and a shift (Granlund and Montgomery, "Division by
+// invariant integers using multiplication", PLDI 1994, Thm. 4.2): with
+// l = ceil(log2 d) and m = floor(2^(31+l) / d) + 1, m*d - 2^(31+l) <= d <= 2^l,
+// hence floor(n / d) = floor(n * m / 2^(31+l)) for every such n, and m < 2^32.
+struct FastDiv {
+  uint32_t m;
+  int sh;
+};
+inline FastDiv make_fastdiv(uint32_t d) {
+  int l = 0;
+  while ((1ull << l) < d) ++l;
+  return FastDiv{(uint32_t)((1ull << (31 + l)) / d + 1), 31 + l};
+}
+__device__ __forceinline__ int fdiv(int n, FastDiv f) {
+  return (int)(((uint64_t)(uint32_t)n * f.m) >> f.sh);
+}
+
 struct DirectGeom {
   int TH, GW;        // output rows and pixel groups per row per CTA
   int threads;       // TH * GW * CG
@@ -53,6 +72,7 @@ struct DirectGeom {
   int run;           // taps per decode item (blob path)
   int tiles_w, tiles_h;
   int splits, stages_per_split;  // split reduction over the stages
+  FastDiv dGW, dHR, dHP;         // dividers of the halo staging
 };
 
 __device__ __forceinline__ void cp_async4(void* smem_dst, const void* gsrc, bool valid) {
@@ -79,33 +99,37 @@ __device__ __forceinline__ uint32_t uabs(int32_t v) {
 template <int SIG, int S, int TM>
 struct Win {
   static constexpr int WS = (TM - 1) * SIG + S;  // window values
-  static constexpr int WSP = (WS + 3) / 4 * 4;   // slot words
-  static constexpr int WV = WSP / 4;             // 16-byte loads per window
+  static constexpr int WV = (WS + 3) / 4;        // 16-byte loads per window
+  // slot stride in words: 16-byte aligned and 4 mod 8, so that the 4-byte
+  // copies of 32 consecutive slots fill 8 bank groups (4-way at most) rather
+  // than 2 (16-way) when the window is a multiple of 8 words
+  static constexpr int WSP = WV * 4 + (WV % 2 == 0 ? 4 : 0);
 };
 
 // Stage the group windows of input channels [c0, c0 + CC) for halo rows
-// s_lo .. s_lo + HR - 1 (stacked coordinates): one slot (channel, halo row,
+// n0 * HP + off0 + [0, HR) (stacked coordinates): one slot (channel, halo row,
 // group) per thread at a time; zero in padding rows, outside the image and
 // for channels >= C.
 template <int SIG, int S, int TM>
-__device__ __forceinline__ void stage_halo(const GemmParams& P, const DirectGeom G, int32_t* halo, int64_t s_lo,
-                                           int iw0, int c0) {
+__device__ __forceinline__ void stage_halo(const GemmParams& P, const DirectGeom G, int32_t* halo, int n0,
+                                           int off0, int iw0, int c0) {
   using WN = Win<SIG, S, TM>;
   const int64_t HW = (int64_t)P.H * P.W;
   const int nslots = G.CC * G.HR * G.GW;
   for (int sl = threadIdx.x; sl < nslots; sl += G.threads) {
-    const int row = sl / G.GW;  // (channel, halo row)
+    const int row = fdiv(sl, G.dGW);  // (channel, halo row)
     const int g = sl - row * G.GW;
-    const int cl = row / G.HR;
+    const int cl = fdiv(row, G.dHR);
     const int hr = row - cl * G.HR;
     const int c = c0 + cl;
-    const int64_t sr = s_lo + hr;
-    const int64_t ni = sr / G.HP;
-    const int ih = (int)(sr - ni * G.HP) - P.ph;
+    const int o = off0 + hr;  // stacked row, counted from image n0's first padded row
+    const int di = fdiv(o, G.dHP);
+    const int ni = n0 + di;
+    const int ih = o - di * G.HP - P.ph;
     const int iws = iw0 + g * TM * SIG;
     int32_t* dst = halo + sl * WN::WSP;
     const bool row_ok = (c < P.C) && (ni < G.N) && ((unsigned)ih < (unsigned)P.H);
-    const int32_t* src = P.x + (ni * P.C + c) * HW + (int64_t)ih * P.W + iws;
+    const int32_t* src = P.x + ((int64_t)ni * P.C + c) * HW + (int64_t)ih * P.W + iws;
     if (row_ok && iws >= 0 && iws + WN::WS <= P.W) {
 #pragma unroll
       for (int i = 0; i < WN::WS; ++i) cp_async4(dst + i, src + i, true);
@@ -119,23 +143,19 @@ __device__ __forceinline__ void stage_halo(const GemmParams& P, const DirectGeom
   }
 }
 
-// Codes of taps [kb, kb + taps) of the CTA's NT channels.  Shared-memory row
-// per tap: NT/32 blocks of 64 words (32 shifts, then 32 signs).
+// Codes of taps [kb, kb + taps) of the CTA's NT = 32 channels: one block of
+// the expanded layout, whose rows of 64 words (32 shifts, then 32 signs) are
+// contiguous over the taps, so the stage is one flat 16-byte copy (zero fill
+// past the last tap).
 __device__ __forceinline__ void stage_codes_expanded(const GemmParams& P, const DirectGeom G, int32_t* code,
                                                      int64_t col0, int64_t kb) {
-  constexpr int NB = NT / 32;
-  const int64_t nblocks = (P.cols + 31) / 32;
-  const int per_block = G.taps * 16;  // 16-byte pieces per block
-#pragma unroll
-  for (int b = 0; b < NB; ++b) {
-    const int64_t cb = col0 / 32 + b;
-    for (int e = threadIdx.x; e < per_block; e += G.threads) {
-      const int tap = e >> 4, q = e & 15;
-      const bool ok = (cb < nblocks) && (kb + tap < P.kred);
-      const int32_t* src = ok ? P.xcodes + ((cb * P.kred + kb + tap) * 64 + q * 4) : P.xcodes;
-      cp_async16(code + (tap * NB + b) * 64 + q * 4, src, ok);
-    }
-  }
+  static_assert(NT == 32, "one 32-channel block of the expanded layout per CTA");
+  const int64_t left = P.kred - kb;
+  const int valid = (left < G.taps ? (int)left : G.taps) * 16;  // 16-byte pieces present
+  const int pieces = G.taps * 16;
+  const int32_t* src = P.xcodes + ((col0 / 32) * P.kred + kb) * 64;
+  for (int e = threadIdx.x; e < pieces; e += G.threads)
+    cp_async16(code + e * 4, e < valid ? (const void*)(src + e * 4) : (const void*)P.xcodes, e < valid);
 }
 
 __device__ __forceinline__ uint32_t nib_word(const GemmParams& P, int64_t col, int64_t k) {
@@ -197,7 +217,8 @@ __device__ __forceinline__ void compute_stage(const DirectGeom G, const int32_t*
   constexpr int R = S;  // square kernels
   constexpr int TAPW = 2 * NT;  // words per tap row
   const int cstride = G.HR * rowstride;
-#pragma unroll 2
+  constexpr int kUnrollC = S <= 3 ? 2 : 1;  // a 7-wide kernel's window already fills the registers
+#pragma unroll kUnrollC
   for (int cl = 0; cl < G.CC; ++cl) {
 #pragma unroll
     for (int r = 0; r < R; ++r) {
@@ -248,8 +269,9 @@ __device__ __forceinline__ void run_direct(const GemmParams& P, const DirectGeom
   const int g = pg % G.GW;
   const int oh_l = pg / G.GW;
   // the tile's first stacked halo row, and this thread's halo row offset
-  const int64_t n0 = gr0 / P.OH;
-  const int64_t s_lo = n0 * G.HP + (gr0 - n0 * P.OH) * SIG;
+  const int n0 = (int)(gr0 / P.OH);
+  const int off0 = (int)(gr0 - (int64_t)n0 * P.OH) * SIG;  // first halo row = stacked row n0 * HP + off0
+  const int64_t s_lo = (int64_t)n0 * G.HP + off0;
   int srow;
   {
     const int64_t gr = gr0 + oh_l;
@@ -280,7 +302,7 @@ __device__ __forceinline__ void run_direct(const GemmParams& P, const DirectGeom
   const int64_t taps_per_c = (int64_t)S * S;
   {
     const int64_t kb = (int64_t)st_begin * G.CC * taps_per_c;
-    stage_halo<SIG, S, TM>(P, G, halo_base, s_lo, iw0, st_begin * G.CC);
+    stage_halo<SIG, S, TM>(P, G, halo_base, n0, off0, iw0, st_begin * G.CC);
     if (expanded) stage_codes_expanded(P, G, code_base, col0, kb);
     cp_async_commit();
     if (!expanded) decode_codes(P, G, code_base, col0, kb);
@@ -292,7 +314,8 @@ __device__ __forceinline__ void run_direct(const GemmParams& P, const DirectGeom
     const int64_t kb1 = (int64_t)(st + 1) * G.CC * taps_per_c;
     __syncthreads();
     if (more) {
-      stage_halo<SIG, S, TM>(P, G, halo_base + (b ^ 1) * G.halo_words, s_lo, iw0, (st + 1) * G.CC);
+      stage_halo<SIG, S, TM>(P, G, halo_base + (b ^ 1) * G.halo_words, n0, off0, iw0,
+                             (st + 1) * G.CC);
       if (expanded) stage_codes_expanded(P, G, code_base + (b ^ 1) * G.code_words, col0, kb1);
       cp_async_commit();
     }
@@ -457,7 +480,7 @@ bool choose_geom(const GemmParams& p, size_t split_capacity, Choice& ch) {
   DirectGeom& G = ch.G;
   ch.TM = (p.OW % 7 == 0) ? 7 : 8;
   const int WS = (ch.TM - 1) * p.sw + p.S;
-  const int WSP = (WS + 3) / 4 * 4;
+  const int WSP = (WS + 3) / 4 * 4 + (((WS + 3) / 4) % 2 == 0 ? 4 : 0);  // as Win<>::WSP
   int gw = (p.OW + ch.TM - 1) / ch.TM;
   if (gw > 8) {
     const int pieces = (gw + 7) / 8;
@@ -506,6 +529,9 @@ bool choose_geom(const GemmParams& p, size_t split_capacity, Choice& ch) {
   if (run < 1) run = 1;
   if (run > 16 && p.xcodes == nullptr) return false;
   G.run = run;
+  G.dGW = make_fastdiv((uint32_t)G.GW);
+  G.dHR = make_fastdiv((uint32_t)G.HR);
+  G.dHP = make_fastdiv((uint32_t)G.HP);
   G.tiles_w = (p.OW + ch.TM * G.GW - 1) / (ch.TM * G.GW);
   G.tiles_h = (int)tiles_h;
   // split the stages when the grid would not fill every SM slot once
