@@ -126,14 +126,16 @@ ds_status conv_launch(const int32_t* x, const ds_weights* w, const int32_t* bias
   p.split_acc = split_acc;
   p.split_capacity = split_capacity;
   if (!(flags & DS_CONV_IM2COL)) {
-    if (conv_pointwise_supported(p)) {
-      p.split_acc = nullptr;
-      return cuda_check(launch_conv2d_pointwise(p, st), "conv2d_shift (pointwise) launch");
-    }
+    if (conv_pointwise_supported(p)) return cuda_check(launch_conv2d_pointwise(p, st), "conv2d_shift (pointwise) launch");
     if (conv_direct_supported(p)) return cuda_check(launch_conv2d_direct(p, st), "conv2d_shift (direct) launch");
   }
   p.split_acc = nullptr;
   return cuda_check(launch_conv2d_shift(p, st), "conv2d_shift (implicit GEMM) launch");
+}
+
+size_t conv_split_bytes(const GemmParams& p) {
+  if (conv_pointwise_supported(p)) return conv_pointwise_split_bytes(p);
+  return conv_direct_split_bytes(p);
 }
 
 ds_status fc_launch(const int32_t* x, const ds_weights* w, const int32_t* bias, int32_t* y, int64_t M,

@@ -570,11 +570,7 @@ cudaError_t launch_direct(const GemmParams& p, const DirectGeom& G, cudaStream_t
   conv_direct_kernel<SIG, S, TM><<<grid, G.threads, smem, st>>>(q, G);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || G.splits == 1) return e;
-  const int64_t total = p.rows * p.cols;
-  int64_t blocks = (total + 255) / 256;
-  if (blocks > kSlots * 8) blocks = kSlots * 8;
-  conv_split_finalize_kernel<<<(unsigned)blocks, 256, 0, st>>>(q, total);
-  return cudaGetLastError();
+  return launch_split_finalize(q, st);
 }
 
 template <int SIG, int TM>
@@ -594,7 +590,15 @@ bool conv_direct_supported(const GemmParams& p) {
   return choose_geom(p, p.split_acc ? p.split_capacity : 0, ch);
 }
 
-size_t conv_split_bytes(const GemmParams& p) {
+cudaError_t launch_split_finalize(const GemmParams& p, cudaStream_t st) {
+  const int64_t total = p.rows * p.cols;
+  int64_t blocks = (total + 255) / 256;
+  if (blocks > kSlots * 8) blocks = kSlots * 8;
+  conv_split_finalize_kernel<<<(unsigned)blocks, 256, 0, st>>>(p, total);
+  return cudaGetLastError();
+}
+
+size_t conv_direct_split_bytes(const GemmParams& p) {
   if (!conv_direct_supported(p)) return 0;
   Choice ch;
   if (!choose_geom(p, ~(size_t)0, ch) || ch.G.splits <= 1) return 0;

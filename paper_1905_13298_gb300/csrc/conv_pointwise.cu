@@ -5,12 +5,22 @@
 // A 1x1 convolution has no window to reuse, so it runs as a GEMM whose rows
 // are output pixels (all images), columns are output channels and whose
 // reduction runs over input channels.  The activation tile of a stage is
-// staged channel-major ([32 channels][128 pixels]): for stride 1 every
+// staged channel-major ([16 channels][128 pixels]): for stride 1 every
 // 16-byte chunk of 4 pixels is one cp.async, for stride 2 four 4-byte copies.
 // A thread owns 8 pixels (two quads 64 apart, so a warp's 16-byte loads are
 // contiguous) and 8 channels; per term the hot loop is one SHF and one IMAD.
+// 128 threads at 128 registers and 32 KB of shared memory: 4 CTAs per SM.
 // Codes come from the expanded execution layout (cp.async) or are decoded
-// from the packed blob per stage.  Accumulator width as in shift_gemm.cu.
+// from the packed blob per stage.  The epilogue writes each (quad, channel)
+// as one 16-byte store when OH*OW is a multiple of 4.  Accumulator width as
+// in shift_gemm.cu.
+//
+// Split reduction (chained forward, layers whose grid would not fill the
+// SMs, e.g. 2048 input channels on 7x7 maps): grid.z CTAs share a tile's
+// stages and add their exact partial sums into an int64 workspace with
+// 64-bit atomics; the finalize kernel of conv_direct.cu applies the epilogue.
+#include <algorithm>
+
 #include "ds_common.cuh"
 
 namespace ds {
@@ -19,12 +29,17 @@ namespace {
 constexpr int MT = 128;       // pixels per CTA
 constexpr int NT = 64;        // channels per CTA
 constexpr int TN = 8;         // channels per thread
-constexpr int THREADS = 128;  // 16 pixel groups x 8 channel groups
-constexpr int KC = 32;        // input channels per stage (= one packed chunk)
+constexpr int PG = MT / 8;    // pixel groups (two quads each)
+constexpr int THREADS = 128;  // PG x (NT / TN)
+constexpr int KC = 16;        // input channels per stage (half of a packed 32-index chunk)
+constexpr int NB = NT / 32;   // 32-channel blocks of the expanded layout per CTA
+constexpr int QUADS = MT / 4;
+constexpr int kSlots = 152 * 4;  // resident CTAs on a GB300
+static_assert(PG * (NT / TN) == THREADS && THREADS % QUADS == 0, "tile shape");
 
 struct __align__(16) PwSmem {
   int32_t xs[2][KC * MT];
-  int32_t cs[2][KC * 2 * NT];  // per input channel: 2 blocks of {32 shifts, 32 signs}
+  int32_t cs[2][KC * 2 * NT];  // per input channel: NB blocks of {32 shifts, 32 signs}
 };
 
 __device__ __forceinline__ void cp_async4(void* smem_dst, const void* gsrc, bool valid) {
@@ -57,7 +72,7 @@ __device__ __forceinline__ QuadCtx quad_ctx(const GemmParams& P, int64_t m0) {
   QuadCtx q;
   const int64_t OHW = (int64_t)P.OH * P.OW;
   const int64_t CHW = (int64_t)P.C * P.H * P.W;
-  const int64_t mq = m0 + 4 * (threadIdx.x & 31);
+  const int64_t mq = m0 + 4 * (threadIdx.x % QUADS);
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
     const int64_t m = mq + i;
@@ -80,10 +95,11 @@ __device__ __forceinline__ QuadCtx quad_ctx(const GemmParams& P, int64_t m0) {
 template <bool STRIDED>
 __device__ __forceinline__ void stage_x(const GemmParams& P, int32_t* xs, const QuadCtx& q, int c0) {
   const int64_t HW = (int64_t)P.H * P.W;
-  const int qi = threadIdx.x & 31;
+  const int qi = threadIdx.x % QUADS;
+  constexpr int ROWS = THREADS / QUADS;  // channel rows per pass
 #pragma unroll
-  for (int j = 0; j < KC / 4; ++j) {
-    const int cl = (threadIdx.x >> 5) + 4 * j;
+  for (int j = 0; j < KC / ROWS; ++j) {
+    const int cl = (int)(threadIdx.x / QUADS) + ROWS * j;
     const int c = c0 + cl;
     int32_t* dst = xs + cl * MT + 4 * qi;
     const bool cok = c < P.C;
@@ -102,59 +118,64 @@ __device__ __forceinline__ void stage_x(const GemmParams& P, int32_t* xs, const 
 // Codes of input channels [c0, c0 + KC) for columns [col0, col0 + 64).
 __device__ __forceinline__ void stage_codes_expanded(const GemmParams& P, int32_t* cs, int64_t col0, int c0) {
   const int64_t nblocks = (P.cols + 31) / 32;
-  // 2 blocks x 32 channels x 16 pieces of 16 bytes
-  for (int e = threadIdx.x; e < 2 * KC * 16; e += THREADS) {
+  for (int e = threadIdx.x; e < NB * KC * 16; e += THREADS) {  // NB blocks x KC channels x 16 pieces
     const int b = e / (KC * 16);
     const int r = e - b * KC * 16;
     const int cl = r >> 4, q = r & 15;
     const int64_t cb = col0 / 32 + b;
     const bool ok = cb < nblocks && c0 + cl < P.kred;
     const int32_t* src = ok ? P.xcodes + ((cb * P.kred + c0 + cl) * 64 + q * 4) : P.xcodes;
-    cp_async16(cs + (cl * 2 + b) * 64 + q * 4, src, ok);
+    cp_async16(cs + (cl * NB + b) * 64 + q * 4, src, ok);
   }
 }
 
-// Blob path: thread t decodes 16 reduction indices of column t % 64.
-__device__ __forceinline__ void decode_codes(const GemmParams& P, int32_t* cs, int64_t col0, int64_t g) {
+// Blob path: stage st covers reduction indices [16 st, 16 st + 16), half
+// st % 2 of packed chunk st / 2.  Thread t decodes 8 indices of column t % 64
+// (indices past k_red decode to s = 0: the blob's padding is zero).
+__device__ __forceinline__ void decode_codes(const GemmParams& P, int32_t* cs, int64_t col0, int st) {
   const int t = threadIdx.x;
   const int n = t & 63;
-  const int h = t >> 6;
+  const int h = t >> 6;                   // which 8 of the stage's 16 indices
+  const int kk0 = 16 * (st & 1) + 8 * h;  // first index within the 32-index chunk
   const int64_t col = col0 + n;
-  uint2 nib = make_uint2(0u, 0u), bits = make_uint2(0u, 0u);
+  uint32_t nib = 0u;
+  uint2 bits = make_uint2(0u, 0u);
   if (col < P.cols) {
-    const int64_t rec = g * P.cols + col;
-    nib = __ldg(reinterpret_cast<const uint2*>(P.blob + P.off_nib + rec * 16 + h * 8));
+    const int64_t rec = (int64_t)(st >> 1) * P.cols + col;
+    nib = __ldg(reinterpret_cast<const uint32_t*>(P.blob + P.off_nib + rec * 16) + (kk0 >> 3));
     bits = __ldg(reinterpret_cast<const uint2*>(P.blob + P.off_bits + rec * 8));
   }
   int32_t* base = cs + (n >> 5) * 64 + (n & 31);
 #pragma unroll
-  for (int i = 0; i < 16; ++i) {
-    const int k = 16 * h + i;
-    const uint32_t w = i < 8 ? nib.x : nib.y;
-    base[k * 2 * NT] = (int)((w >> (4 * (i & 7))) & 15u);
-    base[k * 2 * NT + 32] = (int)((bits.y >> k) & 1u) - 2 * (int)((bits.x >> k) & 1u);
+  for (int i = 0; i < 8; ++i) {
+    const int k = 8 * h + i;  // index within the stage
+    const int kk = kk0 + i;
+    base[k * 2 * NT] = (int)((nib >> (4 * i)) & 15u);
+    base[k * 2 * NT + 32] = (int)((bits.y >> kk) & 1u) - 2 * (int)((bits.x >> kk) & 1u);
   }
 }
 
 template <int I0, int NI, typename Acc>
 __device__ __forceinline__ void compute_stage(const int32_t* xs, const int32_t* cs, int tm, int tn,
                                               Acc (&acc)[NI][TN]) {
-  const int32_t* cbase = cs + (tn >> 2) * 64 + (tn & 3) * TN;
-#pragma unroll 4
+  const int32_t* cbase = cs + ((tn * TN) >> 5) * 64 + ((tn * TN) & 31);
+#pragma unroll 2
   for (int k = 0; k < KC; ++k) {
     int x[8];
     {
       const int4 a = *reinterpret_cast<const int4*>(xs + k * MT + 4 * tm);
-      const int4 b = *reinterpret_cast<const int4*>(xs + k * MT + 64 + 4 * tm);
+      const int4 b = *reinterpret_cast<const int4*>(xs + k * MT + MT / 2 + 4 * tm);
       x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w;
       x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
     }
-    const int4 s0 = *reinterpret_cast<const int4*>(cbase + k * 2 * NT);
-    const int4 s1 = *reinterpret_cast<const int4*>(cbase + k * 2 * NT + 4);
-    const int4 g0 = *reinterpret_cast<const int4*>(cbase + k * 2 * NT + 32);
-    const int4 g1 = *reinterpret_cast<const int4*>(cbase + k * 2 * NT + 36);
-    const int sh[TN] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
-    const int sg[TN] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+    int sh[TN], sg[TN];
+#pragma unroll
+    for (int v = 0; v < TN / 4; ++v) {
+      const int4 s0 = *reinterpret_cast<const int4*>(cbase + k * 2 * NT + 4 * v);
+      const int4 g0 = *reinterpret_cast<const int4*>(cbase + k * 2 * NT + 32 + 4 * v);
+      sh[4 * v] = s0.x; sh[4 * v + 1] = s0.y; sh[4 * v + 2] = s0.z; sh[4 * v + 3] = s0.w;
+      sg[4 * v] = g0.x; sg[4 * v + 1] = g0.y; sg[4 * v + 2] = g0.z; sg[4 * v + 3] = g0.w;
+    }
 #pragma unroll
     for (int i = 0; i < NI; ++i) {
       const int xv = x[I0 + i];
@@ -173,9 +194,9 @@ __device__ __forceinline__ void compute_stage(const int32_t* xs, const int32_t* 
 
 template <bool STRIDED, int I0, int NI, typename Acc>
 __device__ __forceinline__ void run_tile(const GemmParams& P, PwSmem& sm, int64_t m0, int64_t col0,
-                                         const QuadCtx& q, uint32_t& amax_local) {
+                                         const QuadCtx& q, int st_begin, int st_end, uint32_t& amax_local) {
   const int t = threadIdx.x;
-  const int tm = t & 15, tn = t >> 4;
+  const int tm = t % PG, tn = t / PG;
   const bool expanded = P.xcodes != nullptr;
   Acc acc[NI][TN];
 #pragma unroll
@@ -183,15 +204,14 @@ __device__ __forceinline__ void run_tile(const GemmParams& P, PwSmem& sm, int64_
 #pragma unroll
     for (int j = 0; j < TN; ++j) acc[i][j] = 0;
 
-  const int nst = (P.C + KC - 1) / KC;
-  stage_x<STRIDED>(P, sm.xs[0], q, 0);
-  if (expanded) stage_codes_expanded(P, sm.cs[0], col0, 0);
+  stage_x<STRIDED>(P, sm.xs[0], q, st_begin * KC);
+  if (expanded) stage_codes_expanded(P, sm.cs[0], col0, st_begin * KC);
   cp_async_commit();
-  if (!expanded) decode_codes(P, sm.cs[0], col0, 0);
+  if (!expanded) decode_codes(P, sm.cs[0], col0, st_begin);
   cp_async_wait_all();
-  for (int st = 0; st < nst; ++st) {
-    const int b = st & 1;
-    const bool more = st + 1 < nst;
+  for (int st = st_begin; st < st_end; ++st) {
+    const int b = (st - st_begin) & 1;
+    const bool more = st + 1 < st_end;
     __syncthreads();
     if (more) {
       stage_x<STRIDED>(P, sm.xs[b ^ 1], q, (st + 1) * KC);
@@ -206,38 +226,97 @@ __device__ __forceinline__ void run_tile(const GemmParams& P, PwSmem& sm, int64_
   }
   __syncthreads();  // a second pass (64-bit path) reuses the buffers
 
-  // fused epilogue: bias, saturation (64-bit path), residual, ReLU, amax
-  const bool relu = (P.flags & DS_RELU) != 0;
-  const bool resid = (P.flags & DS_RESIDUAL) != 0;
   const int64_t OHW = (int64_t)P.OH * P.OW;
+  if (P.split_acc != nullptr) {
+    // split reduction: exact partial sums (a subset of the terms, so 32-bit
+    // partials are exact whenever the full sum is) into the int64 workspace
+#pragma unroll
+    for (int i = 0; i < NI; ++i) {
+      const int li = I0 + i;
+      const int64_t m = m0 + 4 * tm + (li & 3) + (MT / 2) * (li >> 2);
+      if (m >= P.rows) continue;
+      const int64_t n = m / OHW;
+      const int64_t base = n * P.cols * OHW + (m - n * OHW);
+#pragma unroll
+      for (int j = 0; j < TN; ++j) {
+        const int64_t col = col0 + tn * TN + j;
+        if (col >= P.cols) break;
+        const int64_t v = sizeof(Acc) == 4 ? (int64_t)(int32_t)acc[i][j] : (int64_t)acc[i][j];
+        atomicAdd(reinterpret_cast<unsigned long long*>(P.split_acc + base + col * OHW), (unsigned long long)v);
+      }
+    }
+    return;
+  }
+
+  // fused epilogue: bias, saturation (64-bit path), residual, ReLU, amax.
+  // The thread's pixels are two quads of 4 consecutive output pixels.  When
+  // OH*OW is a multiple of 4 a quad lies inside one image and starts on a
+  // 16-byte boundary, so each (quad, channel) is one 16-byte load / store.
+  const bool relu = (P.flags & DS_RELU) != 0;
+  const int32_t* resid = (P.flags & DS_RESIDUAL) ? P.residual : nullptr;
+  const bool vec = ((OHW & 3) == 0) && (resid == nullptr || (reinterpret_cast<uintptr_t>(resid) & 15) == 0);
   int32_t bcol[TN];
 #pragma unroll
   for (int j = 0; j < TN; ++j) {
     const int64_t col = col0 + tn * TN + j;
     bcol[j] = (P.bias != nullptr && col < P.cols) ? __ldg(P.bias + col) : 0;
   }
+  auto finish = [](Acc a, int32_t b) -> int32_t {
+    if constexpr (sizeof(Acc) == 4) {
+      return (int32_t)(a + (uint32_t)b);
+    } else {
+      int64_t v = a + (int64_t)b;
+      v = v > (int64_t)INT32_MAX ? (int64_t)INT32_MAX : v;
+      v = v < (int64_t)INT32_MIN ? (int64_t)INT32_MIN : v;
+      return (int32_t)v;
+    }
+  };
+  if (vec) {
+#pragma unroll
+    for (int qd = 0; qd < NI / 4; ++qd) {
+      const int64_t mq = m0 + 4 * tm + (MT / 2) * ((I0 >> 2) + qd);
+      if (mq >= P.rows) continue;  // rows = N * OH * OW is a multiple of 4: quads are whole
+      const int64_t n = mq / OHW;  // once per quad
+      const int64_t base = n * P.cols * OHW + (mq - n * OHW);
+#pragma unroll
+      for (int j = 0; j < TN; ++j) {
+        const int64_t col = col0 + tn * TN + j;
+        if (col >= P.cols) break;
+        const int64_t idx = base + col * OHW;
+        int32_t o[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) o[e] = finish(acc[4 * qd + e][j], bcol[j]);
+        if (resid != nullptr) {
+          const int4 r = __ldg(reinterpret_cast<const int4*>(resid + idx));
+          o[0] = add_sat(o[0], r.x);
+          o[1] = add_sat(o[1], r.y);
+          o[2] = add_sat(o[2], r.z);
+          o[3] = add_sat(o[3], r.w);
+        }
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          if (relu) o[e] = max(o[e], 0);
+          amax_local = max(amax_local, uabs(o[e]));
+        }
+        *reinterpret_cast<int4*>(P.y + idx) = make_int4(o[0], o[1], o[2], o[3]);
+      }
+    }
+    return;
+  }
 #pragma unroll
   for (int i = 0; i < NI; ++i) {
     const int li = I0 + i;
-    const int64_t m = m0 + 4 * tm + (li & 3) + 64 * (li >> 2);
+    const int64_t m = m0 + 4 * tm + (li & 3) + (MT / 2) * (li >> 2);
     if (m >= P.rows) continue;
     const int64_t n = m / OHW;  // once per pixel
     const int64_t base = n * P.cols * OHW + (m - n * OHW);
 #pragma unroll
     for (int j = 0; j < TN; ++j) {
       const int64_t col = col0 + tn * TN + j;
-      if (col >= P.cols) continue;
+      if (col >= P.cols) break;
       const int64_t idx = base + col * OHW;
-      int32_t o;
-      if constexpr (sizeof(Acc) == 4) {
-        o = (int32_t)(acc[i][j] + (uint32_t)bcol[j]);
-      } else {
-        int64_t a = acc[i][j] + (int64_t)bcol[j];
-        a = a > (int64_t)INT32_MAX ? (int64_t)INT32_MAX : a;
-        a = a < (int64_t)INT32_MIN ? (int64_t)INT32_MIN : a;
-        o = (int32_t)a;
-      }
-      if (resid) o = add_sat(o, __ldg(P.residual + idx));
+      int32_t o = finish(acc[i][j], bcol[j]);
+      if (resid != nullptr) o = add_sat(o, __ldg(resid + idx));
       if (relu) o = max(o, 0);
       amax_local = max(amax_local, uabs(o));
       P.y[idx] = o;
@@ -267,23 +346,38 @@ __device__ __forceinline__ bool tile_int32_exact(const GemmParams& P, int64_t co
 }
 
 template <bool STRIDED>
-__global__ void __launch_bounds__(THREADS, 3) conv_pointwise_kernel(const GemmParams P) {
+__global__ void __launch_bounds__(THREADS, 4) conv_pointwise_kernel(const GemmParams P, int stages_per_split) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   PwSmem& sm = *reinterpret_cast<PwSmem*>(smem_raw);
   const int64_t m0 = (int64_t)blockIdx.x * MT;
   const int64_t col0 = (int64_t)blockIdx.y * NT;
+  const int n_stages = (P.C + KC - 1) / KC;
+  const int st_begin = blockIdx.z * stages_per_split;
+  const int st_end = min(n_stages, st_begin + stages_per_split);
   const QuadCtx q = quad_ctx<STRIDED>(P, m0);
   uint32_t amax_local = 0;
   if (tile_int32_exact(P, col0)) {
-    run_tile<STRIDED, 0, 8, uint32_t>(P, sm, m0, col0, q, amax_local);
+    run_tile<STRIDED, 0, 8, uint32_t>(P, sm, m0, col0, q, st_begin, st_end, amax_local);
   } else {
-    run_tile<STRIDED, 0, 4, int64_t>(P, sm, m0, col0, q, amax_local);
-    run_tile<STRIDED, 4, 4, int64_t>(P, sm, m0, col0, q, amax_local);
+    run_tile<STRIDED, 0, 4, int64_t>(P, sm, m0, col0, q, st_begin, st_end, amax_local);
+    run_tile<STRIDED, 4, 4, int64_t>(P, sm, m0, col0, q, st_begin, st_end, amax_local);
   }
-  if (P.amax_out != nullptr) {
+  if (P.amax_out != nullptr && P.split_acc == nullptr) {
     amax_local = __reduce_max_sync(0xffffffffu, amax_local);
     if ((threadIdx.x & 31) == 0 && amax_local) atomicMax(P.amax_out, amax_local);
   }
+}
+
+// Stages per CTA of a split reduction (n_stages: no split).  Splits only
+// when the grid would not fill every SM slot once and the workspace holds
+// the int64 partial sums; then it targets two waves.
+int pw_stages_per_split(const GemmParams& p, size_t split_capacity) {
+  const int n_stages = (p.C + KC - 1) / KC;
+  const int64_t ctas = ((p.rows + MT - 1) / MT) * ((p.cols + NT - 1) / NT);
+  const size_t need = (size_t)p.rows * p.cols * sizeof(int64_t);
+  if (split_capacity < need || ctas >= kSlots || n_stages < 2) return n_stages;
+  const int want = (int)std::min<int64_t>(n_stages, (2 * kSlots + ctas - 1) / ctas);
+  return (n_stages + want - 1) / want;
 }
 
 template <bool STRIDED>
@@ -296,16 +390,35 @@ cudaError_t launch_pw(const GemmParams& p, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  dim3 grid((unsigned)((p.rows + MT - 1) / MT), (unsigned)((p.cols + NT - 1) / NT));
-  conv_pointwise_kernel<STRIDED><<<grid, THREADS, smem, st>>>(p);
-  return cudaGetLastError();
+  const int n_stages = (p.C + KC - 1) / KC;
+  const int sps = pw_stages_per_split(p, p.split_acc ? p.split_capacity : 0);
+  const int splits = (n_stages + sps - 1) / sps;
+  GemmParams q = p;
+  if (splits > 1) {
+    cudaError_t e = cudaMemsetAsync(q.split_acc, 0, (size_t)p.rows * p.cols * sizeof(int64_t), st);
+    if (e != cudaSuccess) return e;
+  } else {
+    q.split_acc = nullptr;
+  }
+  dim3 grid((unsigned)((p.rows + MT - 1) / MT), (unsigned)((p.cols + NT - 1) / NT), (unsigned)splits);
+  conv_pointwise_kernel<STRIDED><<<grid, THREADS, smem, st>>>(q, sps);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess || splits == 1) return e;
+  return launch_split_finalize(q, st);
 }
 
 }  // namespace
 
 bool conv_pointwise_supported(const GemmParams& p) {
   return p.R == 1 && p.S == 1 && p.ph == 0 && p.pw == 0 && p.sh >= 1 && p.sw >= 1 && p.cols <= 65535LL * NT &&
-         p.rows < ((int64_t)1 << 40);
+         (p.rows + MT - 1) / MT <= (int64_t)INT32_MAX;
+}
+
+size_t conv_pointwise_split_bytes(const GemmParams& p) {
+  if (!conv_pointwise_supported(p)) return 0;
+  const int n_stages = (p.C + KC - 1) / KC;
+  if (pw_stages_per_split(p, ~(size_t)0) >= n_stages) return 0;
+  return (size_t)p.rows * p.cols * sizeof(int64_t);
 }
 
 cudaError_t launch_conv2d_pointwise(const GemmParams& p, cudaStream_t st) {

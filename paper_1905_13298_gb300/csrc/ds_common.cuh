@@ -83,11 +83,16 @@ cudaError_t launch_linear_shift(const GemmParams& p, cudaStream_t st);
 cudaError_t launch_conv2d_shift(const GemmParams& p, cudaStream_t st);
 // Defined in conv_direct.cu.
 bool conv_direct_supported(const GemmParams& p);
-size_t conv_split_bytes(const GemmParams& p);  // int64 scratch a split reduction would use (0: no split)
+size_t conv_direct_split_bytes(const GemmParams& p);  // int64 scratch a split reduction would use (0: no split)
+cudaError_t launch_conv2d_direct(const GemmParams& p, cudaStream_t st);
+// Epilogue of a split reduction: y = ReLU?(sat32(sat32(split_acc + bias) + residual)), max|y|.
+cudaError_t launch_split_finalize(const GemmParams& p, cudaStream_t st);
 // Defined in conv_pointwise.cu (1x1 convolutions as a GEMM over pixels).
 bool conv_pointwise_supported(const GemmParams& p);
+size_t conv_pointwise_split_bytes(const GemmParams& p);
 cudaError_t launch_conv2d_pointwise(const GemmParams& p, cudaStream_t st);
-cudaError_t launch_conv2d_direct(const GemmParams& p, cudaStream_t st);
+// Defined in api.cu: the split scratch of the kernel conv_launch would choose.
+size_t conv_split_bytes(const GemmParams& p);
 // Defined in linear_bf16.cu.
 int64_t bf16_kpad(int64_t k_red);
 cudaError_t launch_expand_bf16(const uint8_t* blob, int64_t n_out, int64_t k_red, uint16_t* out, cudaStream_t st);

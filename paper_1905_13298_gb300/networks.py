@@ -8,6 +8,7 @@ omitted: it is not a shift operation and the codes are synthetic.
 from __future__ import annotations
 
 import ctypes
+import math
 from dataclasses import dataclass
 
 from . import (DS_OP_AVGPOOL, DS_OP_CONV, DS_OP_FC, DS_OP_MAXPOOL, DS_RELU, DS_RESIDUAL, ds_layer,
@@ -157,6 +158,15 @@ def shift_terms(specs, batch: int) -> int:
     return total
 
 
+def output_shape(sp):
+    """(channels, height, width) a layer writes per image."""
+    if sp.op == DS_OP_FC:
+        return (sp.K, 1, 1)
+    OH = (sp.H + 2 * sp.pad - sp.R) // sp.stride + 1
+    OW = (sp.W + 2 * sp.pad - sp.S) // sp.stride + 1
+    return (sp.K if sp.op == DS_OP_CONV else sp.C, OH, OW)
+
+
 class ShiftNetwork:
     """A packed all-shift network bound to device memory, run with ds_shift_forward."""
 
@@ -181,14 +191,14 @@ class ShiftNetwork:
                 L.bias = self.biases[sp.param].data_ptr()
         nbytes = ds_shift_forward_workspace_bytes(self.layers, len(specs), batch)
         self.workspace = torch.empty(nbytes, dtype=torch.uint8, device=device)
-        last = [sp for sp in specs if sp.out == 1][-1]
-        self.out_shape = (batch, last.K if last.op in (DS_OP_CONV, DS_OP_FC) else last.C) + (
-            (1, 1) if last.op == DS_OP_FC else ())
+        self.out_shape = (batch,) + output_shape([sp for sp in specs if sp.out == 1][-1])
 
     def forward(self, x, y=None, stream=None):
         import torch
         if y is None:
             y = torch.empty(self.out_shape, dtype=torch.int32, device=x.device)
+        elif y.dtype != torch.int32 or not y.is_contiguous() or y.numel() < math.prod(self.out_shape):
+            raise ValueError(f"y must be a contiguous int32 tensor of at least {math.prod(self.out_shape)} elements")
         ds_shift_forward(self.layers, len(self.specs), x, y, self.workspace, self.workspace.numel(), self.batch,
                          stream)
         return y

@@ -138,3 +138,19 @@ def test_forward_program_validation_without_gpu(ds):
     assert ds.ds_shift_forward_workspace_bytes(layers, n, 32) == good
     L = ds.lib()
     assert L.ds_shift_forward(layers, n, 16, 16, 256, good - 1, 32, None) == ds.DS_ERR_BUFFER_TOO_SMALL
+
+
+def test_network_output_shapes(ds):
+    """ShiftNetwork sizes its output from the last layer writing the output slot (conv, pool or FC)."""
+    from paper_1905_13298_gb300 import networks as PN
+    assert PN.output_shape(PN.resnet_program("resnet18")[0][-1]) == (1000, 1, 1)
+    assert PN.output_shape(PN.vgg16_program()[0][-1]) == (1000, 1, 1)
+    b = PN._Builder(512, 7, 7)
+    b.conv(0, 96, 1, 1, 0, out=1)
+    assert PN.output_shape(b.specs[-1]) == (96, 7, 7)
+    b = PN._Builder(64, 56, 56)
+    b.conv(0, 64, 3, 2, 1, out=1)
+    assert PN.output_shape(b.specs[-1]) == (64, 28, 28)
+    b = PN._Builder(64, 56, 56)
+    b.pool(ds.DS_OP_MAXPOOL, 0, 3, 2, 1)
+    assert PN.output_shape(b.specs[-1]) == (64, 28, 28)

@@ -84,3 +84,38 @@ def test_resnet18_stress_codes_small_batch(dslib):
         params.append((si.sign_codes(600 + i, shp), si.shift_codes_geometric(600 + i, shp, -6), si.bias(600 + i, shp[0])))
     x = si.image_batch(12, 1, 3, 32, 32)
     assert np.array_equal(_run(prog, params, x), ON.resnet_forward(x, params, "resnet18"))
+
+
+def _pointwise_pair_program(C, H, W, K1):
+    """x [C,H,W] -> 1x1 conv K1 + ReLU -> 1x1 conv C, + x, ReLU (a bottleneck-style pair of 1x1 layers)."""
+    from paper_1905_13298_gb300 import networks as PN
+    b = PN._Builder(C, H, W)
+    a = b.conv(0, K1, 1, 1, 0, relu=True)
+    b.conv(a, C, 1, 1, 0, relu=True, residual=0, out=1)
+    return (b.specs, b.shapes)
+
+
+def _pointwise_pair_oracle(x, params):
+    from oracle import deepshift_oracle as O
+    (s1, p1, b1), (s2, p2, b2) = params
+    a = O.conv2d_shift(x, s1, p1, b1, (1, 1), (0, 0), relu=True)
+    return O.add_relu(O.conv2d_shift(a, s2, p2, b2, (1, 1), (0, 0)), x)
+
+
+@pytest.mark.parametrize("batch,hw", [(1, 7), (2, 5)])
+@pytest.mark.parametrize("stress", [False, True])
+def test_pointwise_split_reduction(dslib, batch, hw, stress):
+    """1x1 layers with 512 / 256 input channels on tiny maps: the chained forward splits their reduction
+    over CTAs (int64 partials, then the finalize epilogue with residual and ReLU).  Pixel tiles span
+    image boundaries (49 and 25 pixels per image).  Stress codes force the 64-bit path and saturation."""
+    prog = _pointwise_pair_program(512, hw, hw, 256)
+    if stress:
+        params = [(si.sign_codes(700 + i, shp), si.shift_codes_geometric(700 + i, shp, -1), si.bias(700 + i, shp[0]))
+                  for i, shp in enumerate(prog[1])]
+    else:
+        params = si.network_params(prog[1], 710 + batch)
+    x = si.activations(720 + batch, (batch, 512, hw, hw), -(1 << 24), 1 << 24)
+    want = _pointwise_pair_oracle(x, params).reshape(batch, -1)
+    if stress:
+        assert (np.abs(want) == 2 ** 31 - 1).any()
+    assert np.array_equal(_run(prog, params, x), want)

@@ -34,6 +34,8 @@ GEOMS = [
     (2, 5, 5, 5, 3, 5, 5, 1, 0),        # kernel covers the image
     (1, 1, 1, 1, 1, 1, 1, 1, 0),
     (1, 40, 7, 7, 130, 1, 1, 1, 0),
+    (2, 48, 8, 8, 72, 1, 1, 1, 0),      # 1x1, OH*OW % 4 == 0: 16-byte epilogue, ragged channel tile
+    (1, 20, 16, 16, 36, 1, 1, 2, 0),    # 1x1 / 2, 16-byte epilogue, channels not a multiple of 16
 ]
 
 
@@ -49,8 +51,8 @@ def test_conv_bitexact(dslib, geom, flags, expand):
     assert amax[1] == O.absmax(want)
 
 
-@pytest.mark.parametrize("geom", [GEOMS[0], GEOMS[2], GEOMS[4]])
-@pytest.mark.parametrize("flags", [0, 32])
+@pytest.mark.parametrize("geom", [GEOMS[0], GEOMS[2], GEOMS[4], GEOMS[9], GEOMS[10]])
+@pytest.mark.parametrize("flags", [0, 16, 32])
 def test_conv_relu_residual(dslib, geom, flags):
     N, C, H, W, K, R, S, st, pd = geom
     x, s, p, b = si.conv_layer(sum(geom) + 5, N, C, H, W, K, R, S, -(1 << 24), 1 << 24)
