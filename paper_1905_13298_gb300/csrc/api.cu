@@ -138,6 +138,13 @@ size_t conv_split_bytes(const GemmParams& p) {
   return conv_direct_split_bytes(p);
 }
 
+// LinearShift kernel choice: small batches split the reduction over a
+// thread-block cluster, large ones run the 128 x 64-tile shift GEMM.
+static ds_status launch_fc(const GemmParams& p, cudaStream_t st) {
+  if (linear_cluster_preferred(p)) return cuda_check(launch_linear_cluster(p, st), "linear_shift (cluster) launch");
+  return cuda_check(launch_linear_shift(p, st), "linear_shift launch");
+}
+
 ds_status fc_launch(const int32_t* x, const ds_weights* w, const int32_t* bias, int32_t* y, int64_t M,
                     int64_t K, int64_t N, uint32_t flags, const uint32_t* amax_in, uint32_t* amax_out,
                     cudaStream_t st) {
@@ -153,7 +160,7 @@ ds_status fc_launch(const int32_t* x, const ds_weights* w, const int32_t* bias, 
   fill_blob_offsets(p, w);
   p.amax_in = amax_in;
   p.amax_out = amax_out;
-  return cuda_check(launch_linear_shift(p, st), "linear_shift launch");
+  return launch_fc(p, st);
 }
 
 constexpr uint32_t kKnownFlags =
@@ -326,7 +333,7 @@ ds_status ds_linear_shift(const int32_t* x, const ds_weights* w, const int32_t* 
   fill_blob_offsets(p, w);
   r = prepare_amax(x, M * K, flags, amax_io, st, p);
   if (r != DS_OK) return r;
-  return cuda_check(launch_linear_shift(p, st), "linear_shift launch");
+  return launch_fc(p, st);
 }
 
 ds_status ds_conv2d_shift(const int32_t* x, const ds_weights* w, const int32_t* bias,

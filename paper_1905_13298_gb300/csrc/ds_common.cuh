@@ -80,6 +80,9 @@ struct GemmParams {
 
 // Launchers (defined in shift_gemm.cu).
 cudaError_t launch_linear_shift(const GemmParams& p, cudaStream_t st);
+// Defined in linear_cluster.cu (small batches: the reduction split over a thread-block cluster).
+bool linear_cluster_preferred(const GemmParams& p);
+cudaError_t launch_linear_cluster(const GemmParams& p, cudaStream_t st);
 cudaError_t launch_conv2d_shift(const GemmParams& p, cudaStream_t st);
 // Defined in conv_direct.cu.
 bool conv_direct_supported(const GemmParams& p);

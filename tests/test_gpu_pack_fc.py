@@ -13,8 +13,8 @@ def _dev(a):
     return torch.from_numpy(np.ascontiguousarray(a)).cuda()
 
 
-def _pack(ds, s, p):
-    return ds.pack_shift_weights(_dev(s.astype(np.int8)), _dev(p.astype(np.int8)))
+def _pack(ds, s, p, expand=False):
+    return ds.pack_shift_weights(_dev(s.astype(np.int8)), _dev(p.astype(np.int8)), expand=expand)
 
 
 @pytest.mark.parametrize("n_out,k_red", [(1, 1), (3, 31), (64, 576), (65, 33), (512, 784), (130, 100)])
@@ -61,8 +61,8 @@ def test_pack_rejects_bad_codes(dslib):
         _pack(dslib, s, p)
 
 
-def _run_fc(ds, x, s, p, b, flags=0, amax=True):
-    w = _pack(ds, s, p)
+def _run_fc(ds, x, s, p, b, flags=0, amax=True, expand=False):
+    w = _pack(ds, s, p, expand)
     xd = _dev(x.astype(np.int32))
     bd = _dev(b.astype(np.int32)) if b is not None else None
     amax_io = torch.zeros(2, dtype=torch.int32, device="cuda") if amax else None
@@ -71,16 +71,22 @@ def _run_fc(ds, x, s, p, b, flags=0, amax=True):
     return y.cpu().numpy(), (amax_io.cpu().numpy().view(np.uint32) if amax else None)
 
 
+# Small and medium batches take the cluster kernel (the reduction split over up
+# to 16 CTAs); (1024, 40, 3712) fills the SMs with 128 x 64 tiles and takes
+# the plain shift GEMM.  K covers < 32, non-multiples of 4 and of 32, and long
+# reductions with several chunks per CTA of a cluster.
 FC_SHAPES = [(1, 1, 1), (3, 5, 7), (64, 784, 512), (129, 33, 65), (130, 100, 130), (257, 64, 64),
-             (5, 1000, 3), (200, 4, 70), (31, 129, 1)]
+             (5, 1000, 3), (200, 4, 70), (31, 129, 1), (2, 8195, 96), (64, 4100, 200), (9, 2000, 130),
+             (1024, 40, 3712)]
 
 
 @pytest.mark.parametrize("M,K,N", FC_SHAPES)
 @pytest.mark.parametrize("flags", [0, 1, 16, 17])
-def test_linear_shift_bitexact(dslib, M, K, N, flags):
+@pytest.mark.parametrize("expand", [False, True])
+def test_linear_shift_bitexact(dslib, M, K, N, flags, expand):
     x, s, p, b = si.fc_layer(M * 1000 + K * 10 + N, M, K, N, -(1 << 20), 1 << 20)
     want = O.linear_shift(x, s, p, b, relu=bool(flags & 1))
-    got, amax = _run_fc(dslib, x, s, p, b, flags | dslib.DS_AMAX_OUT)
+    got, amax = _run_fc(dslib, x, s, p, b, flags | dslib.DS_AMAX_OUT, expand=expand)
     assert np.array_equal(got, want)
     assert amax[0] == O.absmax(x)
     assert amax[1] == O.absmax(want)
@@ -99,7 +105,7 @@ def test_linear_shift_no_bias_no_amax(dslib):
     assert np.array_equal(got, O.linear_shift(x, s, p, None))
 
 
-@pytest.mark.parametrize("M,K,N", [(70, 300, 66), (128, 64, 64)])
+@pytest.mark.parametrize("M,K,N", [(70, 300, 66), (128, 64, 64), (3, 5000, 40)])
 def test_linear_shift_saturating_inputs(dslib, M, K, N):
     """Full-range int32 activations: the 64-bit path must take over and saturate exactly."""
     x, s, p, b = si.fc_layer(M + K + N, M, K, N, -(1 << 31), 1 << 31)
