@@ -6,22 +6,26 @@
 // With few rows (a batch of 1 to a few hundred) the 128 x 64 tiles of
 // shift_gemm.cu leave most SMs idle: a 64 x 784 x 512 layer makes 8 CTAs.
 // Here a tile of MR = 8 * TMR rows x 64 columns belongs to one cluster of CS
-// CTAs (CS <= 16, a power of two) along the reduction: CTA z of the cluster sums the terms of
-// a 32-aligned slice of k.  Each CTA leaves its partial sums in its own shared
+// CTAs (CS <= 16) along the reduction: CTA z of the cluster sums the terms of
+// a 16-aligned slice of k.  Each CTA leaves its partial sums in its own shared
 // memory; after a cluster barrier CTA z reduces one share of the tile over all
 // CS partials through distributed shared memory (16-byte remote loads),
 // applies the epilogue (bias, saturation, ReLU, max|y|) and stores; a second
 // cluster barrier keeps every CTA's shared memory alive until the remote
 // reads are done.  No global scratch memory is used.
 //
-// 128 threads: thread (tm, tn) = (t % 8, t / 8) owns rows tm + 8 i (i < TMR)
-// and columns 4 tn .. 4 tn + 3.  Per reduction chunk of 32 k the CTA stages
-// x rows (16-byte cp.async when K % 4 == 0) and the chunk's codes (expanded
-// layout: 16-byte cp.async; else decoded from the packed blob).  Per term the
-// hot loop is one SHF and one IMAD, as in shift_gemm.cu.  Accumulator width
-// as in shift_gemm.cu: the bound proven for the whole sum also covers every
-// partial sum (a subset of its terms), so 32-bit partials are exact whenever
-// the 32-bit path is taken, and their wrap-around sum is the exact sum.
+// 128 threads: thread (tm, tn) = (t % 8, t / 8) owns columns 4 tn .. 4 tn + 3
+// and TMR rows: row tm (TMR = 1), rows 4 tm .. 4 tm + 3 (TMR = 4), or two such
+// quads 32 rows apart (TMR = 8), so that the 8 row groups of a warp read
+// distinct banks.  Per stage of 16 k the CTA stages x transposed ([k][row], so
+// a thread's rows at one k are one or two 16-byte loads) and the stage's
+// codes (expanded layout: 16-byte cp.async; else decoded from the packed
+// blob).  Per term the hot loop is one SHF and one IMAD, as in shift_gemm.cu;
+// at most 102 registers, 5 CTAs per SM.
+// Accumulator width as in shift_gemm.cu: the bound proven for the whole sum
+// also covers every partial sum (a subset of its terms), so 32-bit partials
+// are exact whenever the 32-bit path is taken, and their wrap-around sum is
+// the exact sum.
 #include <cooperative_groups.h>
 
 #include <algorithm>
@@ -36,17 +40,23 @@ namespace {
 constexpr int NT = 64;        // columns per tile
 constexpr int TN = 4;         // columns per thread
 constexpr int THREADS = 128;  // 8 row groups x 16 column groups
-constexpr int KC = kChunk;    // reduction indices per stage (one packed chunk)
-constexpr int XS = KC + 4;    // words per staged x row (16-byte reads of 8 rows hit distinct banks)
+constexpr int KC = 16;        // reduction indices per stage (half of a packed 32-index chunk)
 constexpr int CW = 2 * 64;    // code words per k: 2 blocks of {32 shifts, 32 signs}
-constexpr int kSlots = 152 * 4;  // resident CTAs on a GB300 at 4 per SM
+constexpr int kMinBlocks = 5;
+constexpr int kSlots = 152 * kMinBlocks;  // resident CTAs on a GB300
 constexpr int kMaxCluster = 16;
 
 template <int TMR>
 struct ClSmem {
   static constexpr int MR = 8 * TMR;
-  int32_t xs[2][MR * XS];
-  int32_t cs[2][KC * CW];
+  static constexpr int XR = MR + 4;  // words per staged k (16-byte aligned rows of the transposed tile)
+  union {
+    struct {
+      int32_t xs[2][KC * XR];
+      int32_t cs[2][KC * CW];
+    } st;
+    int64_t red[MR * NT];  // the partial sums (int64 or int32) after the reduction loop
+  };
 };
 
 __device__ __forceinline__ void cp_async4(void* smem_dst, const void* gsrc, bool valid) {
@@ -61,29 +71,22 @@ __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commi
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::); }
 __device__ __forceinline__ uint32_t uabs(int32_t v) { return v < 0 ? (uint32_t)0 - (uint32_t)v : (uint32_t)v; }
 
-// x rows [row0, row0 + MR), reduction indices [k0, k0 + 32) clipped to kend
-// (the end of this CTA's slice); zero elsewhere.
-template <int TMR, bool VEC>
+// x rows [row0, row0 + MR), reduction indices [k0, k0 + 16) clipped to kend
+// (the end of this CTA's slice), transposed into xs[k][row]; zero elsewhere.
+// Consecutive threads read consecutive k of one row (64-byte segments).
+template <int TMR>
 __device__ __forceinline__ void stage_x(const GemmParams& P, int32_t* xs, int64_t row0, int64_t k0, int64_t kend) {
-  constexpr int MR = 8 * TMR;
-  if constexpr (VEC) {
-    for (int e = threadIdx.x; e < MR * (KC / 4); e += THREADS) {
-      const int r = e / (KC / 4), q = e % (KC / 4);
-      const int64_t row = row0 + r, k = k0 + 4 * q;
-      const bool ok = row < P.rows && k < kend;  // K % 4 == 0 and kend is 32-aligned or K: whole pieces
-      cp_async16(xs + r * XS + 4 * q, ok ? (const void*)(P.x + row * P.kred + k) : (const void*)P.x, ok);
-    }
-  } else {
-    for (int e = threadIdx.x; e < MR * KC; e += THREADS) {
-      const int r = e / KC, kk = e % KC;
-      const int64_t row = row0 + r, k = k0 + kk;
-      const bool ok = row < P.rows && k < kend;
-      cp_async4(xs + r * XS + kk, ok ? (const void*)(P.x + row * P.kred + k) : (const void*)P.x, ok);
-    }
+  constexpr int MR = 8 * TMR, XR = ClSmem<TMR>::XR;
+  for (int e = threadIdx.x; e < MR * KC; e += THREADS) {
+    const int r = e / KC, kk = e % KC;
+    const int64_t row = row0 + r, k = k0 + kk;
+    const bool ok = row < P.rows && k < kend;
+    cp_async4(xs + kk * XR + r, ok ? (const void*)(P.x + row * P.kred + k) : (const void*)P.x, ok);
   }
 }
 
-// Codes of chunk k0 / 32 for columns [col0, col0 + 64) from the expanded layout.
+// Codes of reduction indices [k0, k0 + 16) for columns [col0, col0 + 64) from
+// the expanded layout.
 __device__ __forceinline__ void stage_codes_expanded(const GemmParams& P, int32_t* cs, int64_t col0, int64_t k0) {
   const int64_t nblocks = (P.cols + 31) / 32;
   for (int e = threadIdx.x; e < 2 * KC * 16; e += THREADS) {
@@ -97,56 +100,77 @@ __device__ __forceinline__ void stage_codes_expanded(const GemmParams& P, int32_
   }
 }
 
-// Blob path: thread t decodes 16 indices (half t / 64) of column t % 64 of
-// chunk g (indices past k_red decode to s = 0: the blob's padding is zero).
-__device__ __forceinline__ void decode_codes(const GemmParams& P, int32_t* cs, int64_t col0, int64_t g) {
+// Blob path: the stage starting at k0 (a multiple of 16) is half (k0 / 16) % 2
+// of packed chunk k0 / 32.  Thread t decodes 8 indices of column t % 64
+// (indices past k_red decode to s = 0: the blob's padding is zero).
+__device__ __forceinline__ void decode_codes(const GemmParams& P, int32_t* cs, int64_t col0, int64_t k0) {
   const int t = threadIdx.x;
   const int n = t & 63;
-  const int h = t >> 6;
+  const int h = t >> 6;                    // which 8 of the stage's 16 indices
+  const int kk0 = (int)(k0 & 31) + 8 * h;  // first index within the 32-index chunk
   const int64_t col = col0 + n;
-  uint2 nib = make_uint2(0u, 0u), bits = make_uint2(0u, 0u);
+  uint32_t nib = 0u;
+  uint2 bits = make_uint2(0u, 0u);
   if (col < P.cols) {
-    const int64_t rec = g * P.cols + col;
-    nib = __ldg(reinterpret_cast<const uint2*>(P.blob + P.off_nib + rec * 16 + h * 8));
+    const int64_t rec = (k0 / 32) * P.cols + col;
+    nib = __ldg(reinterpret_cast<const uint32_t*>(P.blob + P.off_nib + rec * 16) + (kk0 >> 3));
     bits = __ldg(reinterpret_cast<const uint2*>(P.blob + P.off_bits + rec * 8));
   }
   int32_t* base = cs + (n >> 5) * 64 + (n & 31);
 #pragma unroll
-  for (int i = 0; i < 16; ++i) {
-    const int k = 16 * h + i;
-    const uint32_t w = i < 8 ? nib.x : nib.y;
-    base[k * CW] = (int)((w >> (4 * (i & 7))) & 15u);
-    base[k * CW + 32] = (int)((bits.y >> k) & 1u) - 2 * (int)((bits.x >> k) & 1u);
+  for (int i = 0; i < 8; ++i) {
+    const int k = 8 * h + i;  // index within the stage
+    const int kk = kk0 + i;
+    base[k * CW] = (int)((nib >> (4 * i)) & 15u);
+    base[k * CW + 32] = (int)((bits.y >> kk) & 1u) - 2 * (int)((bits.x >> kk) & 1u);
+  }
+}
+
+// Tile row of this thread's i-th row.
+template <int TMR>
+__device__ __forceinline__ int thread_row(int tm, int i) {
+  if constexpr (TMR == 1) {
+    return tm;
+  } else {
+    return (i >> 2) * 32 + 4 * tm + (i & 3);
   }
 }
 
 template <int TMR, typename Acc>
-__device__ __forceinline__ void compute_chunk(const int32_t* xs, const int32_t* cs, int tm, int tn,
+__device__ __forceinline__ void compute_stage(const int32_t* xs, const int32_t* cs, int tm, int tn,
                                               Acc (&acc)[TMR][TN]) {
+  constexpr int XR = ClSmem<TMR>::XR;
   const int32_t* cb = cs + ((tn * TN) >> 5) * 64 + ((tn * TN) & 31);
-#pragma unroll 2
-  for (int k4 = 0; k4 < KC / 4; ++k4) {
-    int4 xv[TMR];
+  const int32_t* xb = xs + (TMR == 1 ? tm : 4 * tm);
 #pragma unroll
-    for (int i = 0; i < TMR; ++i) xv[i] = *reinterpret_cast<const int4*>(xs + (tm + 8 * i) * XS + 4 * k4);
+  for (int k = 0; k < KC; ++k) {
+    int x[TMR];
+    if constexpr (TMR % 4 == 0) {
 #pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-      const int k = 4 * k4 + kk;
-      const int4 s4 = *reinterpret_cast<const int4*>(cb + k * CW);
-      const int4 g4 = *reinterpret_cast<const int4*>(cb + k * CW + 32);
-      const int sh[TN] = {s4.x, s4.y, s4.z, s4.w};
-      const int sg[TN] = {g4.x, g4.y, g4.z, g4.w};
+      for (int v = 0; v < TMR / 4; ++v) {
+        const int4 a = *reinterpret_cast<const int4*>(xb + k * XR + 32 * v);
+        x[4 * v] = a.x;
+        x[4 * v + 1] = a.y;
+        x[4 * v + 2] = a.z;
+        x[4 * v + 3] = a.w;
+      }
+    } else {
+      static_assert(TMR == 1, "row mapping");
+      x[0] = xb[k * XR];
+    }
+    const int4 s4 = *reinterpret_cast<const int4*>(cb + k * CW);
+    const int4 g4 = *reinterpret_cast<const int4*>(cb + k * CW + 32);
+    const int sh[TN] = {s4.x, s4.y, s4.z, s4.w};
+    const int sg[TN] = {g4.x, g4.y, g4.z, g4.w};
 #pragma unroll
-      for (int i = 0; i < TMR; ++i) {
-        const int x = kk == 0 ? xv[i].x : kk == 1 ? xv[i].y : kk == 2 ? xv[i].z : xv[i].w;
+    for (int i = 0; i < TMR; ++i) {
 #pragma unroll
-        for (int j = 0; j < TN; ++j) {
-          const int t = x >> sh[j];  // Eq. 1
-          if constexpr (sizeof(Acc) == 4) {
-            acc[i][j] += (uint32_t)sg[j] * (uint32_t)t;  // Eq. 2 + accumulate (mod 2^32)
-          } else {
-            acc[i][j] += (int64_t)sg[j] * (int64_t)t;
-          }
+      for (int j = 0; j < TN; ++j) {
+        const int t = x[i] >> sh[j];  // Eq. 1
+        if constexpr (sizeof(Acc) == 4) {
+          acc[i][j] += (uint32_t)sg[j] * (uint32_t)t;  // Eq. 2 + accumulate (mod 2^32)
+        } else {
+          acc[i][j] += (int64_t)sg[j] * (int64_t)t;
         }
       }
     }
@@ -176,7 +200,7 @@ __device__ __forceinline__ bool tile_int32_exact(const GemmParams& P, int64_t co
   return !__syncthreads_or(unsafe);
 }
 
-template <int TMR, bool VEC, typename Acc>
+template <int TMR, typename Acc>
 __device__ __forceinline__ void run_cluster_tile(const GemmParams& P, ClSmem<TMR>& sm, cg::cluster_group& cl,
                                                  int64_t row0, int64_t col0, int64_t kbeg, int64_t kend,
                                                  uint32_t& amax_local) {
@@ -194,10 +218,10 @@ __device__ __forceinline__ void run_cluster_tile(const GemmParams& P, ClSmem<TMR
   // and contributes zero partial sums
   const int nst = kend > kbeg ? (int)((kend - kbeg + KC - 1) / KC) : 0;
   if (nst > 0) {
-    stage_x<TMR, VEC>(P, sm.xs[0], row0, kbeg, kend);
-    if (expanded) stage_codes_expanded(P, sm.cs[0], col0, kbeg);
+    stage_x<TMR>(P, sm.st.xs[0], row0, kbeg, kend);
+    if (expanded) stage_codes_expanded(P, sm.st.cs[0], col0, kbeg);
     cp_async_commit();
-    if (!expanded) decode_codes(P, sm.cs[0], col0, kbeg / KC);
+    if (!expanded) decode_codes(P, sm.st.cs[0], col0, kbeg);
     cp_async_wait_all();
   }
   for (int st = 0; st < nst; ++st) {
@@ -206,23 +230,23 @@ __device__ __forceinline__ void run_cluster_tile(const GemmParams& P, ClSmem<TMR
     const int64_t k1 = kbeg + (int64_t)(st + 1) * KC;
     __syncthreads();
     if (more) {
-      stage_x<TMR, VEC>(P, sm.xs[b ^ 1], row0, k1, kend);
-      if (expanded) stage_codes_expanded(P, sm.cs[b ^ 1], col0, k1);
+      stage_x<TMR>(P, sm.st.xs[b ^ 1], row0, k1, kend);
+      if (expanded) stage_codes_expanded(P, sm.st.cs[b ^ 1], col0, k1);
       cp_async_commit();
     }
-    compute_chunk<TMR, Acc>(sm.xs[b], sm.cs[b], tm, tn, acc);
+    compute_stage<TMR, Acc>(sm.st.xs[b], sm.st.cs[b], tm, tn, acc);
     if (more) {
-      if (!expanded) decode_codes(P, sm.cs[b ^ 1], col0, k1 / KC);
+      if (!expanded) decode_codes(P, sm.st.cs[b ^ 1], col0, k1);
       cp_async_wait_all();
     }
   }
   __syncthreads();  // every thread is done with the staging buffers: they hold the partials next
 
   // this CTA's partial sums, [MR][64] row-major, 16 bytes per (row, 4 columns) for 32-bit
-  Acc* red = reinterpret_cast<Acc*>(&sm);
+  Acc* red = reinterpret_cast<Acc*>(sm.red);
 #pragma unroll
   for (int i = 0; i < TMR; ++i) {
-    Acc* dst = red + (tm + 8 * i) * NT + tn * TN;
+    Acc* dst = red + thread_row<TMR>(tm, i) * NT + tn * TN;
 #pragma unroll
     for (int j = 0; j < TN; ++j) dst[j] = acc[i][j];
   }
@@ -288,8 +312,8 @@ __device__ __forceinline__ void run_cluster_tile(const GemmParams& P, ClSmem<TMR
   cl.sync();  // no CTA leaves (or reuses its shared memory) while another still reads it
 }
 
-template <int TMR, bool VEC>
-__global__ void __launch_bounds__(THREADS, 4) linear_cluster_kernel(const GemmParams P, int64_t k_per_cta) {
+template <int TMR>
+__global__ void __launch_bounds__(THREADS, kMinBlocks) linear_cluster_kernel(const GemmParams P, int64_t k_per_cta) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   ClSmem<TMR>& sm = *reinterpret_cast<ClSmem<TMR>*>(smem_raw);
   cg::cluster_group cl = cg::this_cluster();
@@ -299,9 +323,9 @@ __global__ void __launch_bounds__(THREADS, 4) linear_cluster_kernel(const GemmPa
   const int64_t kend = min(P.kred, kbeg + k_per_cta);
   uint32_t amax_local = 0;
   if (tile_int32_exact(P, col0)) {
-    run_cluster_tile<TMR, VEC, uint32_t>(P, sm, cl, row0, col0, kbeg, kend, amax_local);
+    run_cluster_tile<TMR, uint32_t>(P, sm, cl, row0, col0, kbeg, kend, amax_local);
   } else {
-    run_cluster_tile<TMR, VEC, int64_t>(P, sm, cl, row0, col0, kbeg, kend, amax_local);
+    run_cluster_tile<TMR, int64_t>(P, sm, cl, row0, col0, kbeg, kend, amax_local);
   }
   if (P.amax_out != nullptr) {
     amax_local = __reduce_max_sync(0xffffffffu, amax_local);
@@ -309,65 +333,60 @@ __global__ void __launch_bounds__(THREADS, 4) linear_cluster_kernel(const GemmPa
   }
 }
 
-// Largest cluster size (<= 16) the device can co-schedule for this kernel,
-// queried once per process.
-template <int TMR, bool VEC>
-cudaError_t prepare(size_t smem, int& max_cluster) {
-  static int cached = 0;
-  if (cached > 0) {
-    max_cluster = cached;
-    return cudaSuccess;
-  }
-  auto kern = linear_cluster_kernel<TMR, VEC>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-  if (e != cudaSuccess) return e;
-  int best = 1;
-  for (int cs = kMaxCluster; cs >= 2; cs /= 2) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(1, 1, cs);
-    cfg.blockDim = dim3(THREADS, 1, 1);
-    cfg.dynamicSmemBytes = smem;
-    cudaLaunchAttribute attr;
-    attr.id = cudaLaunchAttributeClusterDimension;
-    attr.val.clusterDim.x = 1;
-    attr.val.clusterDim.y = 1;
-    attr.val.clusterDim.z = cs;
-    cfg.attrs = &attr;
-    cfg.numAttrs = 1;
-    int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) == cudaSuccess && n > 0) {
-      best = cs;
-      break;
+// How many clusters of cs CTAs the device can hold at once (0: not
+// launchable), queried once per process and size.
+template <int TMR>
+int active_clusters(int cs) {
+  static int cache[kMaxCluster + 1] = {0};
+  static bool attrs_set = false;
+  if (cs < 1 || cs > kMaxCluster) return 0;
+  if (cache[cs] != 0) return cache[cs] > 0 ? cache[cs] : 0;
+  auto kern = linear_cluster_kernel<TMR>;
+  if (!attrs_set) {
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(ClSmem<TMR>)) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
+      (void)cudaGetLastError();
+      return 0;
     }
-    (void)cudaGetLastError();  // clear a refused query
+    attrs_set = true;
   }
-  cached = best;
-  max_cluster = best;
-  return cudaSuccess;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(1, 1, cs);
+  cfg.blockDim = dim3(THREADS, 1, 1);
+  cfg.dynamicSmemBytes = sizeof(ClSmem<TMR>);
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeClusterDimension;
+  attr.val.clusterDim.x = 1;
+  attr.val.clusterDim.y = 1;
+  attr.val.clusterDim.z = cs;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
+    (void)cudaGetLastError();  // a refused size
+    n = 0;
+  }
+  cache[cs] = n > 0 ? n : -1;
+  return n;
 }
 
-template <int TMR, bool VEC>
+template <int TMR>
 cudaError_t launch_tmr(const GemmParams& p, cudaStream_t st) {
   constexpr int MR = 8 * TMR;
-  const size_t smem = sizeof(ClSmem<TMR>);
-  static_assert(sizeof(ClSmem<TMR>) >= (size_t)MR * NT * sizeof(int64_t), "partials fit the staging buffers");
-  int max_cluster = 1;
-  cudaError_t e = prepare<TMR, VEC>(smem, max_cluster);
-  if (e != cudaSuccess) return e;
   const int64_t tiles = ((p.rows + MR - 1) / MR) * ((p.cols + NT - 1) / NT);
-  const int64_t chunks = (p.kred + KC - 1) / KC;
-  // the cluster size: a power of two that fills at most one wave of CTAs and
-  // gives every CTA at least one chunk (trailing slices may still be empty)
-  const int64_t want = std::min<int64_t>(std::min<int64_t>(kSlots / std::max<int64_t>(tiles, 1), max_cluster), chunks);
-  int64_t cs = 1;
-  while (cs * 2 <= want) cs *= 2;
-  const int64_t chunks_per_cta = (chunks + cs - 1) / cs;
+  const int64_t stages = (p.kred + KC - 1) / KC;
+  // the cluster size: at most one wave of CTAs, at least one stage per CTA,
+  // and a size the device accepts (trailing slices may still be empty)
+  int64_t cs = std::min<int64_t>(std::min<int64_t>(kSlots / std::max<int64_t>(tiles, 1), kMaxCluster), stages);
+  cs = std::max<int64_t>(cs, 1);
+  while (cs > 1 && active_clusters<TMR>((int)cs) <= 0) --cs;
+  if (active_clusters<TMR>((int)cs) <= 0) return cudaErrorLaunchOutOfResources;
+  const int64_t stages_per_cta = (stages + cs - 1) / cs;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)((p.rows + MR - 1) / MR), (unsigned)((p.cols + NT - 1) / NT), (unsigned)cs);
   cfg.blockDim = dim3(THREADS, 1, 1);
-  cfg.dynamicSmemBytes = smem;
+  cfg.dynamicSmemBytes = sizeof(ClSmem<TMR>);
   cfg.stream = st;
   cudaLaunchAttribute attr;
   attr.id = cudaLaunchAttributeClusterDimension;
@@ -376,14 +395,7 @@ cudaError_t launch_tmr(const GemmParams& p, cudaStream_t st) {
   attr.val.clusterDim.z = (unsigned)cs;
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, linear_cluster_kernel<TMR, VEC>, p, chunks_per_cta * KC);
-}
-
-template <bool VEC>
-cudaError_t launch_by_rows(const GemmParams& p, cudaStream_t st) {
-  if (p.rows <= 8) return launch_tmr<1, VEC>(p, st);
-  if (p.rows <= 32) return launch_tmr<4, VEC>(p, st);
-  return launch_tmr<8, VEC>(p, st);
+  return cudaLaunchKernelEx(&cfg, linear_cluster_kernel<TMR>, p, stages_per_cta * KC);
 }
 
 }  // namespace
@@ -395,8 +407,9 @@ bool linear_cluster_preferred(const GemmParams& p) {
 }
 
 cudaError_t launch_linear_cluster(const GemmParams& p, cudaStream_t st) {
-  const bool vec = (p.kred % 4 == 0) && ((reinterpret_cast<uintptr_t>(p.x) & 15) == 0);
-  return vec ? launch_by_rows<true>(p, st) : launch_by_rows<false>(p, st);
+  if (p.rows <= 8) return launch_tmr<1>(p, st);
+  if (p.rows <= 32) return launch_tmr<4>(p, st);
+  return launch_tmr<8>(p, st);
 }
 
 }  // namespace ds
