@@ -52,6 +52,11 @@ def workload_by_name(name: str, batch):
     if name == "fc_large":
         M, K, N = 8192, 4096, 4096
         return dict(name="fc_shift_8192x4096x4096_int32", kind="fc", M=M, K=K, Nout=N, terms=M * K * N)
+    if name == "fc_vgg16_fc1":
+        # VGG16's first FC layer at a small batch: codes geometric around the per-layer centre, as in the chain
+        M, K, N = batch or 64, 25088, 4096
+        return dict(name=f"fc_shift_vgg16_fc1_b{M}_int32", kind="fc", M=M, K=K, Nout=N, terms=M * K * N,
+                    centred=True)
     if name in ("sweep_resnet50", "sweep_vgg16", "sweep_resnet18"):
         arch = name.split("_")[1]
         b = batch or (32 if arch == "resnet18" else 64)
@@ -216,7 +221,11 @@ def run_gpu_other(args, wl, rank, world, local_rank):
         launches = 1
         h2d = xd.numel() * 2
     elif wl["kind"] == "fc":
-        x, s, p, b = si.config4_int()
+        if wl.get("centred"):
+            x, s, p, b = si.fc_layer(si.SEED_BASE + 45, wl["M"], wl["K"], wl["Nout"], 0, 1 << 20,
+                                     si.layer_centre(wl["K"], 1, 1))
+        else:
+            x, s, p, b = si.config4_int()
         w = ds.pack_shift_weights(torch.from_numpy(s).to(dev), torch.from_numpy(p).to(dev), expand=True)
         xd, bd = torch.from_numpy(x).to(dev), torch.from_numpy(b).to(dev)
         y = torch.empty((wl["M"], wl["Nout"]), dtype=torch.int32, device=dev)
@@ -287,8 +296,37 @@ def run_gpu_other(args, wl, rank, world, local_rank):
     print(json.dumps(out), flush=True)
 
 
+def time_fc_layer(args, ds, dev, seed, M, K, N):
+    """One FC-shift layer standalone: codes geometric around the per-layer centre, as in the chain."""
+    import torch
+    x, s, p, b = si.fc_layer(seed, M, K, N, 0, 1 << 20, si.layer_centre(K, 1, 1))
+    w = ds.pack_shift_weights(torch.from_numpy(s).to(dev), torch.from_numpy(p).to(dev), expand=True)
+    xd, bd = torch.from_numpy(x).to(dev), torch.from_numpy(b).to(dev)
+    y = torch.empty((M, N), dtype=torch.int32, device=dev)
+    a = torch.zeros(2, dtype=torch.int32, device=dev)
+    ds.ds_absmax(xd, xd.numel(), a)
+    st = torch.cuda.current_stream().cuda_stream
+
+    def call():
+        ds.ds_linear_shift(xd, w.desc, bd, y, M, K, N, ds.DS_AMAX_IN, a, st)
+    for _ in range(max(3, args.warmup)):
+        call()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = max(3, args.steps)
+    e0.record()
+    for _ in range(reps):
+        call()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / reps
+    terms = M * K * N
+    return dict(shape=f"FC {K}->{N}", terms=terms, ms=ms, gsops=terms / ms / 1e6,
+                frac=2 * terms / (ms / 1e3) / (SMS * INT_OPS_PER_CLK_PER_SM * 2070e6))
+
+
 def run_layer_sweep(args, wl, local_rank):
-    """Every conv layer of the network standalone (own inputs, same shapes as in the chain)."""
+    """Every conv and FC layer of the network standalone (own inputs, same shapes as in the chain)."""
     import torch
     import paper_1905_13298_gb300 as ds
     from paper_1905_13298_gb300 import build as dsb
@@ -303,6 +341,13 @@ def run_layer_sweep(args, wl, local_rank):
     rows = []
     tot_terms = tot_ms = 0.0
     for i, sp in enumerate(specs):
+        if sp.op == ds.DS_OP_FC:
+            r = time_fc_layer(args, ds, dev, si.SEED_BASE + 5 + i, B, sp.C * sp.H * sp.W, sp.K)
+            r["layer"] = i
+            rows.append(r)
+            tot_terms += r["terms"]
+            tot_ms += r["ms"]
+            continue
         if sp.op != ds.DS_OP_CONV:
             continue
         key = (sp.C, sp.H, sp.W, sp.K, sp.R, sp.stride, sp.pad)
@@ -495,7 +540,7 @@ def main():
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--batch", type=int, default=None)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--workload", default="conv2x", choices=["conv2x", "fc_large", "fc_large_bf16", "resnet18", "resnet50", "vgg16",
+    ap.add_argument("--workload", default="conv2x", choices=["conv2x", "fc_large", "fc_vgg16_fc1", "fc_large_bf16", "resnet18", "resnet50", "vgg16",
                                                          "sweep_resnet18", "sweep_resnet50", "sweep_vgg16"])
     ap.add_argument("--graph", action="store_true", help="replay each step from a CUDA graph (other workloads)")
     args = ap.parse_args()
