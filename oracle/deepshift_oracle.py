@@ -15,6 +15,9 @@ Definitions (DeepShift, Elhoushi et al.):
 * Eq. 3 -- LinearShift / ConvShift replace the weight W by flip(2^P, S):
   Y = flip(2^P, S) X + b and Y = flip(2^P, S) (*) X + b.
 * Sec. 4 -- activations and bias are 32-bit fixed point with 16 fraction bits.
+* Eq. 4-6 (DeepShift-Q) -- a float weight W becomes S = sign(W),
+  P = round(log2|W|), W_q = flip(2^P, S); Sec. 4 clips P to the supported
+  shift range ([-15, 0], or [-14, 0] for strict 5-bit codes).
 
 Readings taken where the paper is silent:
 
@@ -24,6 +27,11 @@ Readings taken where the paper is silent:
 * R-conv: convolution is cross-correlation (PyTorch conv2d semantics), OIHW
   weights, zero padding, reduction index order (c, r, s).
 * R-pool: max-pool ignores padded taps; average pool is floor(sum / count).
+* R-round: round(log2|W|) is the integer n with 2^(n - 1/2) <= |W| < 2^(n + 1/2);
+  the bound 2^(1/2) is irrational, so no float weight is a tie.  W = 0 and NaN
+  give S = 0 and P = p_min (clip of -inf); W = +-inf gives S = +-1, P = 0.
+* R-q16: the Sec. 4 rounding to fixed point is round-half-to-even of x * 2^16,
+  saturated to the int32 range; NaN becomes 0.
 
 Parity status: every function here is pinned by tests under
 ``tests/test_oracle_pins.py`` (brute force, float64 library routines on exact
@@ -409,3 +417,39 @@ def weights_bf16_bits(s, p) -> np.ndarray:
     _check_codes(s, p)
     bits = ((s < 0).astype(np.int64) << 15) | ((127 + p) << 7)
     return np.where(s == 0, 0, bits).astype(np.uint16)
+
+
+# ---------------------------------------------------------------------------
+# Float -> code and float -> Q16.16 conversion (the step before packing)
+# ---------------------------------------------------------------------------
+def quantize_weights(W, p_min: int = P_MIN):
+    """DeepShift-Q quantizer (Eq. 4-6, clipping of Sec. 4) of float32 weights.
+
+    s = sign(W); p = clip(round(log2|W|), p_min, 0) with the readings R-round.
+    Written with frexp: |W| = m 2^e, m in [1/2, 1), so |W| = (2m) 2^(e-1) with
+    2m in [1, 2) and log2|W| = (e - 1) + log2(2m); the fractional part rounds
+    up exactly when 2m >= 2^(1/2), i.e. m^2 >= 1/2 (exact in float64: m has at
+    most 24 significant bits).  Returns int8 arrays s, p of W's shape.
+    """
+    if not (P_MIN <= p_min <= P_MAX):
+        raise ValueError("p_min outside [-15, 0]")
+    w = np.asarray(W, dtype=np.float32).astype(np.float64)
+    nan = np.isnan(w)
+    s = np.where(nan, 0.0, np.sign(w)).astype(np.int8)
+    a = np.abs(np.where(nan, 0.0, w))
+    finite_nz = np.isfinite(a) & (a > 0)
+    m, e = np.frexp(np.where(finite_nz, a, 1.0))
+    r = (e.astype(np.int64) - 1) + (m * m >= 0.5)
+    p = np.clip(r, p_min, P_MAX)
+    p = np.where(np.isinf(a), P_MAX, p)
+    p = np.where(a == 0, p_min, p)  # zero and NaN (mapped to 0 above)
+    return s, p.astype(np.int8)
+
+
+def quantize_activations(x) -> np.ndarray:
+    """Float32 -> int32 Q16.16 (Sec. 4, reading R-q16): rint(x * 2^16), ties to
+    even, saturated to [-2^31, 2^31 - 1], NaN -> 0.  x * 2^16 is exact in
+    float64 for every float32 x."""
+    y = np.asarray(x, dtype=np.float32).astype(np.float64) * 65536.0
+    y = np.where(np.isnan(y), 0.0, np.rint(y))
+    return np.clip(y, INT32_MIN, INT32_MAX).astype(np.int64).astype(np.int32)

@@ -30,6 +30,7 @@ STREAM_P = 2
 STREAM_S = 3
 STREAM_B = 4
 STREAM_G2 = 5
+STREAM_F = 6
 
 
 def _mix(z: np.ndarray) -> np.ndarray:
@@ -151,6 +152,40 @@ def bits_to_f64(bits: np.ndarray) -> np.ndarray:
 # --------------------------------------------------------------------------
 # Workload recipes (shapes and distributions of the evaluated configurations)
 # --------------------------------------------------------------------------
+
+def float32_from_fields(sign, exponent, mantissa) -> np.ndarray:
+    """float32 values assembled from integer IEEE-754 fields (sign bit, unbiased
+    exponent of a normal number, 23-bit mantissa): identical on every platform."""
+    sign = np.asarray(sign, dtype=np.uint64)
+    biased = (np.asarray(exponent, dtype=np.int64) + 127).astype(np.uint64)
+    mant = np.asarray(mantissa, dtype=np.uint64)
+    bits = (sign << np.uint64(31)) | (biased << np.uint64(23)) | mant
+    return bits.astype(np.uint32).view(np.float32)
+
+
+def float_weights(seed: int, shape, e_lo: int = -20, e_hi: int = 1) -> np.ndarray:
+    """float32 weights with a random sign, a uniform 23-bit mantissa and an
+    exponent uniform in [e_lo, e_hi] (a log-uniform magnitude), built from bit
+    fields.  One word per element: bit 0 sign, bits 1-23 mantissa, bits 32-63
+    the exponent draw."""
+    n = int(np.prod(shape))
+    w = raw_u64(seed, STREAM_F, n)
+    span = e_hi - e_lo + 1
+    sign = w & np.uint64(1)
+    mant = (w >> np.uint64(1)) & np.uint64(0x7FFFFF)
+    expo = e_lo + ((w >> np.uint64(32)) % np.uint64(span)).astype(np.int64)
+    return float32_from_fields(sign, expo, mant).reshape(shape)
+
+
+def float_activations(seed: int, shape, e_lo: int = -20, e_hi: int = 17) -> np.ndarray:
+    """float32 activations as float_weights, plus exact Q16.16 rounding ties:
+    every 8th element is (2k + 1) / 2^17 for a random |k| < 2^20."""
+    x = float_weights(seed, shape, e_lo, e_hi).reshape(-1).copy()
+    k = uniform_int(seed, STREAM_X, (x.size,), -(1 << 20), 1 << 20)
+    ties = ((2 * k + 1).astype(np.float64) / float(1 << 17)).astype(np.float32)
+    x[::8] = ties[::8]
+    return x.reshape(shape)
+
 
 SEED_BASE = 0xD5000000
 

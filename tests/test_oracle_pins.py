@@ -500,3 +500,100 @@ def test_bf16_weight_bits_decode_to_s_times_power_of_two():
     assert bits[0, 0] == 0x3F80 and bits[0, 1] == 0xB800 and bits[0, 2] == 0 and bits[1, 2] == 0x3F80
     vals = si.bits_to_f64(bits)
     assert np.array_equal(vals, s * np.ldexp(1.0, p))
+
+
+# ---------------------------------------------------------------------------
+# DeepShift-Q quantizer (Eq. 4-6) and Q16.16 input rounding (Sec. 4)
+# ---------------------------------------------------------------------------
+def _exact_round_log2(a: float) -> int:
+    """round(log2 a) for a float a > 0 from exact rationals: the n with
+    2^(2n-1) <= a^2 < 2^(2n+1) (the bound 2^(n+1/2) is irrational, so no ties)."""
+    from fractions import Fraction
+    q = Fraction(a) ** 2
+    n = 0
+    while q >= Fraction(2) ** (2 * n + 1):
+        n += 1
+    while q < Fraction(2) ** (2 * n - 1):
+        n -= 1
+    return n
+
+
+def test_quantize_weights_powers_of_two_are_fixed_points():
+    """W = +-2^k quantizes to s = +-1, p = k inside [-15, 0] and to the clip bound outside it."""
+    ks = np.arange(-20, 4)
+    for sign in (1.0, -1.0):
+        w = (sign * np.ldexp(1.0, ks)).astype(np.float32)
+        s, p = O.quantize_weights(w)
+        assert (s == int(sign)).all()
+        assert np.array_equal(p, np.clip(ks, -15, 0))
+
+
+def test_quantize_weights_against_exact_rationals():
+    """Random float32 weights, and the float32 neighbours of every rounding bound 2^(n+1/2):
+    p equals the clipped exact round(log2|W|), s the sign."""
+    w = si.float_weights(31, (4000,), -19, 2)
+    bounds = []
+    for n in range(-18, 3):
+        c = np.float32(2.0 ** (n + 0.5))
+        bounds += [c, np.nextafter(c, np.float32(0)), np.nextafter(c, np.float32(10))]
+    w = np.concatenate([w, np.array(bounds, np.float32), -np.array(bounds, np.float32)])
+    for p_min in (-15, -14):
+        s, p = O.quantize_weights(w, p_min)
+        for wi, si_, pi in zip(w.tolist(), s.tolist(), p.tolist()):
+            assert si_ == (1 if wi > 0 else -1)
+            assert pi == min(max(_exact_round_log2(abs(wi)), p_min), 0), (wi, pi)
+
+
+def test_quantize_weights_matches_log2_library_away_from_bounds():
+    """np.round(np.log2(|W|)), a different route, agrees wherever log2|W| is not within 1e-6 of a half-integer."""
+    w = si.float_weights(32, (200000,), -17, 1)
+    lg = np.log2(np.abs(w.astype(np.float64)))
+    far = np.abs(lg - np.floor(lg) - 0.5) > 1e-6
+    s, p = O.quantize_weights(w)
+    assert np.array_equal(p[far], np.clip(np.round(lg[far]), -15, 0).astype(np.int8))
+    assert np.array_equal(s, np.sign(w).astype(np.int8))
+
+
+def test_quantize_weights_special_values():
+    w = np.array([0.0, -0.0, np.nan, np.inf, -np.inf, 1e-45, -1e-40, 3.0, -1.0e30], np.float32)
+    s, p = O.quantize_weights(w)
+    assert s.tolist() == [0, 0, 0, 1, -1, 1, -1, 1, -1]
+    assert p.tolist() == [-15, -15, -15, 0, 0, -15, -15, 0, 0]
+    s, p = O.quantize_weights(w, -14)
+    assert p.tolist() == [-14, -14, -14, 0, 0, -14, -14, 0, 0]
+    with pytest.raises(ValueError):
+        O.quantize_weights(w, -16)
+
+
+def test_quantize_weights_then_flip_reproduces_powers_of_two():
+    """Eq. 6: flip(2^p, s) of the codes is the nearest power of two in log scale, clipped."""
+    w = si.float_weights(33, (5000,), -14, -1)
+    s, p = O.quantize_weights(w)
+    wq = s.astype(np.float64) * np.ldexp(1.0, p.astype(np.int64))
+    ratio = np.abs(w.astype(np.float64)) / np.abs(wq)
+    assert (ratio >= 2 ** -0.5).all() and (ratio < 2 ** 0.5).all()
+
+
+def test_quantize_activations_ties_saturation_and_specials():
+    half = 1.0 / 65536
+    x = np.array([0.5 * half, 1.5 * half, 2.5 * half, -0.5 * half, -1.5 * half, -2.5 * half,
+                  32767.0, 32768.0, -32768.0, -32768.5, 1e30, -1e30, np.nan, np.inf, -np.inf], np.float32)
+    q = O.quantize_activations(x)
+    assert q.tolist() == [0, 2, 2, 0, -2, -2, 32767 << 16, 2 ** 31 - 1, -(2 ** 31), -(2 ** 31),
+                          2 ** 31 - 1, -(2 ** 31), 0, 2 ** 31 - 1, -(2 ** 31)]
+
+
+def test_quantize_activations_against_exact_rationals_and_torch_round():
+    """Exact rational round-half-even on random values (including ties), and torch.round (also half to
+    even) as a library route for values inside the range."""
+    from fractions import Fraction
+    x = si.float_activations(34, (3000,), -20, 14)
+    q = O.quantize_activations(x)
+    for xi, qi in zip(x.tolist(), q.tolist()):
+        v = Fraction(xi) * 65536
+        fl = v.numerator // v.denominator
+        d = v - fl
+        r = fl + (1 if d > Fraction(1, 2) or (d == Fraction(1, 2) and fl % 2 == 1) else 0)
+        assert qi == max(min(r, 2 ** 31 - 1), -(2 ** 31)), xi
+    t = torch.round(torch.from_numpy(x.astype(np.float64)) * 65536).to(torch.int64).numpy()
+    assert np.array_equal(q.astype(np.int64), t)
