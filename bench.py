@@ -57,6 +57,15 @@ def workload_by_name(name: str, batch):
         M, K, N = batch or 64, 25088, 4096
         return dict(name=f"fc_shift_vgg16_fc1_b{M}_int32", kind="fc", M=M, K=K, Nout=N, terms=M * K * N,
                     centred=True)
+    if name == "quantize_vgg16_fc1":
+        # float32 weights of VGG16's first FC layer -> int8 sign and shift codes (DeepShift-Q)
+        n = 4096 * 25088
+        return dict(name="quantize_weights_vgg16_fc1_4096x25088", kind="quant", n=n, bytes=n * (4 + 2))
+    if name == "q16_input":
+        # float32 network input -> Q16.16 int32 (batch 256 of 3 x 224 x 224: larger than L2 both ways)
+        b = batch or 256
+        n = b * 3 * 224 * 224
+        return dict(name=f"q16_input_b{b}_3x224x224", kind="q16", n=n, bytes=n * (4 + 4))
     if name in ("sweep_resnet50", "sweep_vgg16", "sweep_resnet18"):
         arch = name.split("_")[1]
         b = batch or (32 if arch == "resnet18" else 64)
@@ -293,6 +302,60 @@ def run_gpu_other(args, wl, rank, world, local_rank):
            "config": {"workload": wl["name"], "cuda_graph": bool(args.graph), "terms_per_step": terms},
            "roofline": roof,
            "gpu_launches": launches * args.steps, "clocks": clocks, "h2d_bytes_per_step_e2e": h2d}
+    print(json.dumps(out), flush=True)
+
+
+def run_conversion(args, wl, local_rank):
+    """Float -> code / float -> Q16.16 conversion: value = algorithmic GB/s (bytes read + written once)."""
+    import torch
+    import paper_1905_13298_gb300 as ds
+    from paper_1905_13298_gb300 import build as dsb
+
+    dsb.build_library()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    n = wl["n"]
+    if wl["kind"] == "quant":
+        src = torch.from_numpy(si.float_weights(si.SEED_BASE + 46, (n,), -18, 1)).to(dev)
+        s = torch.empty(n, dtype=torch.int8, device=dev)
+        p = torch.empty(n, dtype=torch.int8, device=dev)
+
+        def step():
+            ds.ds_quantize_shift_weights(src, n, -15, s, p, torch.cuda.current_stream().cuda_stream)
+        kernel = "quantize_weights_kernel"
+    else:
+        src = torch.from_numpy(si.float_activations(si.SEED_BASE + 47, (n,), -12, 10)).to(dev)
+        q = torch.empty(n, dtype=torch.int32, device=dev)
+
+        def step():
+            ds.ds_quantize_q16(src, n, q, torch.cuda.current_stream().cuda_stream)
+        kernel = "quantize_q16_kernel"
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(local_rank)
+    sampler.start()
+    time.sleep(0.3)
+    torch.cuda.synchronize()
+    e0.record()
+    for _ in range(args.steps):
+        step()
+    e1.record()
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    ms = e0.elapsed_time(e1) / args.steps
+    gbs = wl["bytes"] / (ms / 1e3) / 1e9
+    peaks, src_name = measured_peaks()
+    peak = float(peaks.get("hbm_gbs", 6800.0))
+    out = {"metric": "GB/s", "value": gbs, "unit": "GB/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+           "dtype": "f32->int8" if wl["kind"] == "quant" else "f32->int32", "data": "synthetic",
+           "config": {"workload": wl["name"], "elements": n, "bytes_per_step": wl["bytes"],
+                      "l2": "inputs and outputs larger than L2"},
+           "roofline": {"bound": "hbm", "achieved": gbs, "peak": peak, "unit": "GB/s", "frac": gbs / peak,
+                        "traffic": None, "kernel": kernel, "peak_basis": f"hbm_gbs, {src_name}"},
+           "gpu_launches": args.steps, "clocks": clocks}
     print(json.dumps(out), flush=True)
 
 
@@ -540,7 +603,7 @@ def main():
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--batch", type=int, default=None)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--workload", default="conv2x", choices=["conv2x", "fc_large", "fc_vgg16_fc1", "fc_large_bf16", "resnet18", "resnet50", "vgg16",
+    ap.add_argument("--workload", default="conv2x", choices=["conv2x", "fc_large", "fc_vgg16_fc1", "fc_large_bf16", "quantize_vgg16_fc1", "q16_input", "resnet18", "resnet50", "vgg16",
                                                          "sweep_resnet18", "sweep_resnet50", "sweep_vgg16"])
     ap.add_argument("--graph", action="store_true", help="replay each step from a CUDA graph (other workloads)")
     args = ap.parse_args()
@@ -556,6 +619,8 @@ def main():
         run_gpu(args, wl, rank, world, local_rank)
     elif wl["kind"] == "sweep":
         run_layer_sweep(args, wl, local_rank)
+    elif wl["kind"] in ("quant", "q16"):
+        run_conversion(args, wl, local_rank)
     else:
         run_gpu_other(args, wl, rank, world, local_rank)
 

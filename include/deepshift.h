@@ -318,6 +318,33 @@ size_t ds_shift_forward_workspace_bytes(const ds_layer* layers, int n, int batch
 ds_status ds_shift_forward(const ds_layer* layers, int n, const int32_t* x, int32_t* y, void* ws,
                            size_t ws_bytes, int batch, void* stream);
 
+/* ---------------------------------------------------------------------------
+ * Conversion of float models (the step before packing).
+ *
+ * ds_quantize_shift_weights: the DeepShift-Q quantizer (Sec. 3.1, Eq. 4-6,
+ * with the shift clipping of Sec. 4) of n float32 weights w (device, 4-byte
+ * aligned, any layout; conv weights flattened as [K][C][R][S]) into the
+ * int8 codes s (device, n bytes) and p (device, n bytes) that
+ * ds_pack_shift_weights takes:
+ *   s = sign(w) in {-1, 0, +1},  p = clip(round(log2|w|), p_min, 0).
+ * round(log2|w|) is the integer n with 2^(n-1/2) <= |w| < 2^(n+1/2), decided
+ * exactly (no float log; no float weight is a tie).  p_min is -15 (the
+ * 6-bit code format) or -14 (codes that also fit the strict 5-bit format of
+ * Sec. 4); other values in [-15, 0] are accepted.  w = 0 and NaN give s = 0,
+ * p = p_min; +-inf gives s = +-1, p = 0.  Stream-ordered, no synchronisation.
+ * Errors: DS_ERR_INVALID_ARG (NULL pointer, p_min outside [-15, 0]),
+ * DS_ERR_SHAPE (n <= 0), DS_ERR_ALIGNMENT (w not 4-byte aligned).
+ *
+ * ds_quantize_q16: Sec. 4's rounding of float inputs (and biases) to 32-bit
+ * fixed point with 16 fraction bits: q = round-half-to-even(x * 2^16),
+ * saturated to [INT32_MIN, INT32_MAX]; NaN gives 0.  x (n float32) and q
+ * (n int32) are device pointers, 4-byte aligned (16-byte alignment takes
+ * the vectorised path).  Errors: DS_ERR_INVALID_ARG, DS_ERR_SHAPE,
+ * DS_ERR_ALIGNMENT as above.
+ * ------------------------------------------------------------------------- */
+ds_status ds_quantize_shift_weights(const float* w, int64_t n, int p_min, int8_t* s, int8_t* p, void* stream);
+ds_status ds_quantize_q16(const float* x, int64_t n, int32_t* q, void* stream);
+
 /*
  * max |x| over n int32 values, written to *amax (device u32; |INT32_MIN| = 2^31).
  */

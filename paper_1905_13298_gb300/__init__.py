@@ -100,6 +100,9 @@ _SIGNATURES = {
                                             ctypes.c_uint32, ctypes.c_void_p]),
     "ds_bf16_fault_flag": (ctypes.c_int, []),
     "ds_absmax": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]),
+    "ds_quantize_shift_weights": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_void_p,
+                                                 ctypes.c_void_p, ctypes.c_void_p]),
+    "ds_quantize_q16": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]),
 }
 
 
@@ -217,6 +220,14 @@ def ds_absmax(x, n: int, amax, stream=None) -> None:
     _check(lib().ds_absmax(_ptr(x), n, _ptr(amax), _stream(stream)))
 
 
+def ds_quantize_shift_weights(w, n: int, p_min: int, s, p, stream=None) -> None:
+    _check(lib().ds_quantize_shift_weights(_ptr(w), n, p_min, _ptr(s), _ptr(p), _stream(stream)))
+
+
+def ds_quantize_q16(x, n: int, q, stream=None) -> None:
+    _check(lib().ds_quantize_q16(_ptr(x), n, _ptr(q), _stream(stream)))
+
+
 # ---------------------------------------------------------------------------
 # Tensor-level helpers (allocate outputs with torch, then call the ABI)
 # ---------------------------------------------------------------------------
@@ -268,6 +279,29 @@ def linear_shift_bf16(x, w: PackedShiftWeights, bias=None, relu: bool = False, o
     y = out if out is not None else torch.empty((M, N), dtype=torch.float32, device=x.device)
     ds_linear_shift_bf16(x, w.desc, bias, y, M, K, N, DS_RELU if relu else 0, stream)
     return y
+
+
+def quantize_shift_weights(w, p_min: int = -15, stream=None):
+    """DeepShift-Q codes (Eq. 4-6) of a float32 CUDA weight tensor: int8 tensors s, p of w's shape."""
+    import torch
+    if w.device.type != "cuda" or w.dtype != torch.float32:
+        raise ValueError("w must be a float32 CUDA tensor")
+    w = w.contiguous()
+    s = torch.empty(w.shape, dtype=torch.int8, device=w.device)
+    p = torch.empty(w.shape, dtype=torch.int8, device=w.device)
+    ds_quantize_shift_weights(w, w.numel(), p_min, s, p, stream)
+    return s, p
+
+
+def quantize_q16(x, out=None, stream=None):
+    """Q16.16 int32 tensor of a float32 CUDA tensor (Sec. 4: ties to even, saturating, NaN -> 0)."""
+    import torch
+    if x.device.type != "cuda" or x.dtype != torch.float32:
+        raise ValueError("x must be a float32 CUDA tensor")
+    x = x.contiguous()
+    q = out if out is not None else torch.empty(x.shape, dtype=torch.int32, device=x.device)
+    ds_quantize_q16(x, x.numel(), q, stream)
+    return q
 
 
 def pack_shift_weights(s, p, stream=None, expand: bool = False) -> PackedShiftWeights:

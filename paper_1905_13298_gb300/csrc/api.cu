@@ -294,6 +294,25 @@ ds_status ds_linear_shift_bf16(const uint16_t* x, const ds_weights* w, const flo
 
 int ds_bf16_fault_flag(void) { return read_bf16_fault_flag(); }
 
+ds_status ds_quantize_shift_weights(const float* w, int64_t n, int p_min, int8_t* s, int8_t* p, void* stream) {
+  clear_error();
+  if (!w || !s || !p) return fail(DS_ERR_INVALID_ARG, "NULL pointer argument");
+  if (n <= 0) return fail(DS_ERR_SHAPE, "n must be positive");
+  if (p_min < -15 || p_min > 0) return fail(DS_ERR_INVALID_ARG, "p_min %d outside [-15, 0]", p_min);
+  if ((reinterpret_cast<uintptr_t>(w) & 3) != 0) return fail(DS_ERR_ALIGNMENT, "w must be 4-byte aligned");
+  return cuda_check(launch_quantize_weights(w, n, p_min, s, p, static_cast<cudaStream_t>(stream)),
+                    "quantize_shift_weights launch");
+}
+
+ds_status ds_quantize_q16(const float* x, int64_t n, int32_t* q, void* stream) {
+  clear_error();
+  if (!x || !q) return fail(DS_ERR_INVALID_ARG, "NULL pointer argument");
+  if (n <= 0) return fail(DS_ERR_SHAPE, "n must be positive");
+  if ((reinterpret_cast<uintptr_t>(x) & 3) != 0 || (reinterpret_cast<uintptr_t>(q) & 3) != 0)
+    return fail(DS_ERR_ALIGNMENT, "x and q must be 4-byte aligned");
+  return cuda_check(launch_quantize_q16(x, n, q, static_cast<cudaStream_t>(stream)), "quantize_q16 launch");
+}
+
 ds_status ds_absmax(const int32_t* x, int64_t n, uint32_t* amax, void* stream) {
   clear_error();
   if (!x || !amax) return fail(DS_ERR_INVALID_ARG, "NULL pointer argument");

@@ -117,6 +117,9 @@ GemmParams conv_params(const ds_weights* w, int N, int C, int H, int W, int K, i
 ds_status fc_launch(const int32_t* x, const ds_weights* w, const int32_t* bias, int32_t* y, int64_t M,
                     int64_t K, int64_t N, uint32_t flags, const uint32_t* amax_in, uint32_t* amax_out,
                     cudaStream_t st);
+// Defined in quantize.cu (DeepShift-Q codes from float weights, Q16.16 from float activations).
+cudaError_t launch_quantize_weights(const float* w, int64_t n, int p_min, int8_t* s, int8_t* p, cudaStream_t st);
+cudaError_t launch_quantize_q16(const float* x, int64_t n, int32_t* q, cudaStream_t st);
 // Defined in misc_kernels.cu.
 cudaError_t launch_absmax(const int32_t* x, int64_t n, uint32_t* out, cudaStream_t st);
 cudaError_t launch_pack(const int8_t* s, const int8_t* p, int64_t n_out, int64_t k_red,

@@ -96,6 +96,16 @@ def test_validation_happens_before_cuda(ds):
     assert L.ds_linear_shift(4096, ctypes.byref(w2), None, 4096, 2, 8, 8, 0, None, None) == ds.DS_ERR_INVALID_ARG
     assert L.ds_absmax(None, 4, 16, None) == ds.DS_ERR_INVALID_ARG
     assert L.ds_absmax(16, 0, 16, None) == ds.DS_ERR_SHAPE
+    # quantizers: NULL pointers, p_min range, sizes, alignment
+    assert L.ds_quantize_shift_weights(None, 4, -15, 16, 32, None) == ds.DS_ERR_INVALID_ARG
+    assert L.ds_quantize_shift_weights(16, 4, -16, 16, 32, None) == ds.DS_ERR_INVALID_ARG
+    assert "p_min" in ds.ds_last_error()
+    assert L.ds_quantize_shift_weights(16, 4, 1, 16, 32, None) == ds.DS_ERR_INVALID_ARG
+    assert L.ds_quantize_shift_weights(16, 0, -15, 16, 32, None) == ds.DS_ERR_SHAPE
+    assert L.ds_quantize_shift_weights(18, 4, -15, 16, 32, None) == ds.DS_ERR_ALIGNMENT
+    assert L.ds_quantize_q16(16, 4, None, None) == ds.DS_ERR_INVALID_ARG
+    assert L.ds_quantize_q16(16, -1, 32, None) == ds.DS_ERR_SHAPE
+    assert L.ds_quantize_q16(16, 4, 34, None) == ds.DS_ERR_ALIGNMENT
 
 
 def test_no_cpu_fallback_without_library(tmp_path, monkeypatch, ds):
