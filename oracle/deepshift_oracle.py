@@ -32,6 +32,11 @@ Readings taken where the paper is silent:
   give S = 0 and P = p_min (clip of -inf); W = +-inf gives S = +-1, P = 0.
 * R-q16: the Sec. 4 rounding to fixed point is round-half-to-even of x * 2^16,
   saturated to the int32 range; NaN becomes 0.
+* Eq. 7 (with its footnote) -- the input gradient of LinearShift is
+  dC/dY W_q^T, of ConvShift W_q^rot180 (*) dC/dY.
+* R-bwd: the backward terms use the forward's fixed-point semantics: the
+  Q16.16 gradient dy is shifted (floor) and flipped, s * (dy >> -p), the sum
+  is exact, then saturated to int32.
 
 Parity status: every function here is pinned by tests under
 ``tests/test_oracle_pins.py`` (brute force, float64 library routines on exact
@@ -453,3 +458,74 @@ def quantize_activations(x) -> np.ndarray:
     y = np.asarray(x, dtype=np.float32).astype(np.float64) * 65536.0
     y = np.where(np.isnan(y), 0.0, np.rint(y))
     return np.clip(y, INT32_MIN, INT32_MAX).astype(np.int64).astype(np.int32)
+
+
+# ---------------------------------------------------------------------------
+# Input gradient (Eq. 7 and its footnote), reading R-bwd
+# ---------------------------------------------------------------------------
+def linear_shift_backward_x_acc(dy, s, p) -> np.ndarray:
+    """Exact int64 dC/dX of LinearShift: dx[m, k] = sum_n s[n, k] * floor(dy[m, n] / 2^-p[n, k]),
+    i.e. dC/dY W_q^T with every product a shift and a flip.  dy: [M, N]; s, p: [N, K]."""
+    dy = np.asarray(dy, dtype=np.int64)
+    s = np.asarray(s, dtype=np.int64)
+    p = np.asarray(p, dtype=np.int64)
+    _check_codes(s, p)
+    M, N = dy.shape
+    N2, K = s.shape
+    if N != N2:
+        raise ValueError("dy and codes disagree on N")
+    acc = np.zeros((M, K), dtype=np.int64)
+    for n in range(N):
+        divisor = np.left_shift(np.int64(1), -p[n])  # [K]
+        acc += s[n][None, :] * np.floor_divide(dy[:, n][:, None], divisor[None, :])
+    return acc
+
+
+def linear_shift_backward_x(dy, s, p) -> np.ndarray:
+    return sat32(linear_shift_backward_x_acc(dy, s, p)).astype(np.int32)
+
+
+def conv2d_shift_backward_x_acc(dy, s, p, in_hw, stride=(1, 1), pad=(0, 0)) -> np.ndarray:
+    """Exact int64 dC/dX of ConvShift, written as the scatter the forward gather
+    implies: output (n, k, oh, ow) read input (c, oh*sh + r - ph, ow*sw + q - pw)
+    through code (k, c, r, q), so its gradient term s * floor(dy / 2^-p) is added
+    there (positions in the padding are dropped).  dy: [N, K, OH, OW];
+    s, p: [K, C, R, S]; in_hw = (H, W); returns int64 [N, C, H, W]."""
+    dy = np.asarray(dy, dtype=np.int64)
+    s = np.asarray(s, dtype=np.int64)
+    p = np.asarray(p, dtype=np.int64)
+    _check_codes(s, p)
+    N, K, OH, OW = dy.shape
+    K2, C, R, S = s.shape
+    H, W = in_hw
+    sh, sw = stride
+    ph, pw = pad
+    if K != K2 or OH != conv_out_size(H, R, sh, ph) or OW != conv_out_size(W, S, sw, pw):
+        raise ValueError("dy, codes and geometry disagree")
+    gpad = np.zeros((N, C, H + 2 * ph + sh, W + 2 * pw + sw), dtype=np.int64)  # padded input grid
+    for k in range(K):
+        for r in range(R):
+            for q in range(S):
+                divisor = np.left_shift(np.int64(1), -p[k, :, r, q])  # [C]
+                terms = s[k, :, r, q][None, :, None, None] * np.floor_divide(
+                    dy[:, k][:, None, :, :], divisor[None, :, None, None])  # [N, C, OH, OW]
+                gpad[:, :, r:r + sh * (OH - 1) + 1:sh, q:q + sw * (OW - 1) + 1:sw] += terms
+    return gpad[:, :, ph:ph + H, pw:pw + W]
+
+
+def conv2d_shift_backward_x(dy, s, p, in_hw, stride=(1, 1), pad=(0, 0)) -> np.ndarray:
+    return sat32(conv2d_shift_backward_x_acc(dy, s, p, in_hw, stride, pad)).astype(np.int32)
+
+
+def backward_codes(s, p):
+    """Code matrix of the input-gradient pass as a forward layer (Eq. 7 footnote):
+    column c, reduction index (k, r, q) holds the code of (k, c, R-1-r, S-1-q),
+    i.e. W^rot180 with the channel axes swapped.  s, p: [K, C, R, S] (FC:
+    [N, K] is taken as [N, K, 1, 1]); returns [C, K, R, S] int8 arrays."""
+    s = np.asarray(s)
+    p = np.asarray(p)
+    if s.ndim == 2:
+        s, p = s[:, :, None, None], p[:, :, None, None]
+    st = np.ascontiguousarray(np.transpose(s[:, :, ::-1, ::-1], (1, 0, 2, 3)))
+    pt = np.ascontiguousarray(np.transpose(p[:, :, ::-1, ::-1], (1, 0, 2, 3)))
+    return st.astype(np.int8), pt.astype(np.int8)

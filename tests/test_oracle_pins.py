@@ -597,3 +597,88 @@ def test_quantize_activations_against_exact_rationals_and_torch_round():
         assert qi == max(min(r, 2 ** 31 - 1), -(2 ** 31)), xi
     t = torch.round(torch.from_numpy(x.astype(np.float64)) * 65536).to(torch.int64).numpy()
     assert np.array_equal(q.astype(np.int64), t)
+
+
+# ---------------------------------------------------------------------------
+# Input gradient (Eq. 7 and its footnote)
+# ---------------------------------------------------------------------------
+BWD_GEOMS = [  # N, C, H, W, K, R, S, stride, pad
+    (2, 3, 7, 6, 4, 3, 3, 1, 1), (2, 3, 7, 6, 4, 3, 3, 2, 1), (1, 2, 9, 9, 3, 7, 7, 2, 3),
+    (2, 5, 6, 5, 3, 1, 1, 2, 0), (1, 4, 5, 5, 2, 3, 3, 1, 0), (1, 2, 8, 7, 3, 5, 3, 2, 2),
+]
+
+
+@pytest.mark.parametrize("geom", BWD_GEOMS)
+def test_conv_backward_x_equals_float64_autograd_on_exact_inputs(geom):
+    """dy a multiple of 2^15 makes every shift exact, so dC/dX is torch's float64 autograd of conv2d with
+    W = s * 2^p (a library route through the transposed convolution)."""
+    N, C, H, W, K, R, S, st, pd = geom
+    s = si.sign_codes(sum(geom), (K, C, R, S))
+    p = si.shift_codes_uniform(sum(geom), (K, C, R, S))
+    OH, OW = O.conv_out_size(H, R, st, pd), O.conv_out_size(W, S, st, pd)
+    dy = si.uniform_int(sum(geom) + 1, si.STREAM_X, (N, K, OH, OW), -4096, 4096) * (1 << 15)
+    got = O.conv2d_shift_backward_x_acc(dy, s, p, (H, W), (st, st), (pd, pd))
+    wt = torch.tensor(s * np.ldexp(1.0, p.astype(np.int64)), dtype=torch.float64)
+    x = torch.zeros((N, C, H, W), dtype=torch.float64, requires_grad=True)
+    F.conv2d(x, wt, stride=st, padding=pd).backward(torch.tensor(dy, dtype=torch.float64))
+    assert np.array_equal(got, x.grad.numpy().astype(np.int64))
+
+
+def test_linear_backward_x_equals_float64_matmul_on_exact_inputs():
+    M, K, N = 7, 19, 11
+    s = si.sign_codes(3, (N, K))
+    p = si.shift_codes_uniform(3, (N, K))
+    dy = si.uniform_int(4, si.STREAM_X, (M, N), -4096, 4096) * (1 << 15)
+    wt = torch.tensor(s * np.ldexp(1.0, p.astype(np.int64)), dtype=torch.float64)
+    want = (torch.tensor(dy, dtype=torch.float64) @ wt).numpy().astype(np.int64)
+    assert np.array_equal(O.linear_shift_backward_x_acc(dy, s, p), want)
+
+
+@pytest.mark.parametrize("geom", BWD_GEOMS[:4])
+def test_conv_backward_x_brute_force_gather_with_floor(geom):
+    """Non-exact gradients (floor matters): each input position gathers, with Python ints, every
+    (output, tap) pair that read it in the forward pass."""
+    N, C, H, W, K, R, S, st, pd = geom
+    s = si.sign_codes(sum(geom) + 2, (K, C, R, S))
+    p = si.shift_codes_uniform(sum(geom) + 2, (K, C, R, S))
+    OH, OW = O.conv_out_size(H, R, st, pd), O.conv_out_size(W, S, st, pd)
+    dy = si.activations(sum(geom) + 3, (N, K, OH, OW), -(1 << 20), 1 << 20)
+    got = O.conv2d_shift_backward_x(dy, s, p, (H, W), (st, st), (pd, pd))
+    for n in range(N):
+        for c in range(C):
+            for i in range(H):
+                for j in range(W):
+                    acc = 0
+                    for k in range(K):
+                        for r in range(R):
+                            for q in range(S):
+                                u, v = i + pd - r, j + pd - q
+                                if u % st or v % st:
+                                    continue
+                                oh, ow = u // st, v // st
+                                if 0 <= oh < OH and 0 <= ow < OW:
+                                    acc += int(s[k, c, r, q]) * (int(dy[n, k, oh, ow]) // (1 << -int(p[k, c, r, q])))
+                    assert got[n, c, i, j] == max(min(acc, 2 ** 31 - 1), -(2 ** 31))
+
+
+@pytest.mark.parametrize("geom", [g for g in BWD_GEOMS if g[7] == 1])
+def test_conv_backward_x_stride1_is_forward_conv_with_rot180_codes(geom):
+    """For stride 1 the input gradient is the forward ConvShift of dy with the rot180 / transposed codes
+    (Eq. 7 footnote) and padding R - 1 - pad."""
+    N, C, H, W, K, R, S, st, pd = geom
+    s = si.sign_codes(sum(geom) + 4, (K, C, R, S))
+    p = si.shift_codes_uniform(sum(geom) + 4, (K, C, R, S))
+    OH, OW = O.conv_out_size(H, R, 1, pd), O.conv_out_size(W, S, 1, pd)
+    dy = si.activations(sum(geom) + 5, (N, K, OH, OW), -(1 << 24), 1 << 24)
+    sb, pb = O.backward_codes(s, p)
+    assert sb.shape == (C, K, R, S) and sb[0, 0, 0, 0] == s[0, 0, R - 1, S - 1]
+    want = O.conv2d_shift_backward_x(dy, s, p, (H, W), (1, 1), (pd, pd))
+    assert np.array_equal(O.conv2d_shift(dy, sb, pb, None, (1, 1), (R - 1 - pd, S - 1 - pd)), want)
+
+
+def test_linear_backward_x_is_forward_with_transposed_codes():
+    s = si.sign_codes(6, (13, 29))
+    p = si.shift_codes_uniform(6, (13, 29))
+    dy = si.activations(7, (5, 13), -(1 << 30), 1 << 30)
+    sb, pb = O.backward_codes(s, p)
+    assert np.array_equal(O.linear_shift(dy, sb[:, :, 0, 0], pb[:, :, 0, 0]), O.linear_shift_backward_x(dy, s, p))
