@@ -319,6 +319,41 @@ ds_status ds_shift_forward(const ds_layer* layers, int n, const int32_t* x, int3
                            size_t ws_bytes, int batch, void* stream);
 
 /* ---------------------------------------------------------------------------
+ * Input gradient (Eq. 7 and its footnote: dC/dX = dC/dY W_q^T for LinearShift,
+ * W_q^rot180 (*) dC/dY for ConvShift).  The gradient dY is int32 Q16.16 and
+ * each term is the forward's shift-then-flip, s * (dy >> -p); the exact sum
+ * is saturated to int32 (no bias, no ReLU).
+ *
+ * ds_pack_shift_weights_backward packs the code matrix of that pass from the
+ * forward codes s, p (device int8, [K][C][R][S]; an FC layer's [N][K_in] is
+ * K = N, C = K_in, R = S = 1): C columns, reduction length K*R*S, column c
+ * and index (k, r, q) holding the code of (k, c, R-1-r, S-1-q).  Buffer size
+ * ds_packed_weight_bytes(C, K*R*S); otherwise as ds_pack_shift_weights
+ * (synchronises, DS_ERR_CODE_RANGE on bad codes).
+ *
+ * ds_linear_shift_backward_x: dx [M][K] from dy [M][N] (row-major, 16-byte
+ * aligned) with w_bwd packed by ds_pack_shift_weights_backward(s, p, N, K,
+ * 1, 1).  Flags: DS_AMAX_IN / DS_AMAX_OUT (amax_io as in ds_linear_shift)
+ * and DS_FORCE_INT64 only.
+ *
+ * ds_conv2d_shift_backward_x: dx [N][C][H][W] from dy [N][K][OH][OW] of the
+ * forward geometry (H, W, R, S, strides, pads as given to ds_conv2d_shift;
+ * OH = (H + 2 pad_h - R) / stride_h + 1, likewise OW), w_bwd packed by
+ * ds_pack_shift_weights_backward(s, p, K, C, R, S).  Stride 1 runs the
+ * forward ConvShift of dy with padding R-1-pad; larger strides run the
+ * implicit GEMM whose gather reads dy at window positions divisible by the
+ * stride.  Flags: DS_AMAX_IN, DS_AMAX_OUT, DS_FORCE_INT64, and
+ * DS_CONV_IM2COL (the gather path at any stride).  Errors as ds_conv2d_shift.
+ * ------------------------------------------------------------------------- */
+ds_status ds_pack_shift_weights_backward(const int8_t* s, const int8_t* p, int K, int C, int R, int S, void* packed,
+                                         size_t packed_bytes, ds_weights* desc, void* stream);
+ds_status ds_linear_shift_backward_x(const int32_t* dy, const ds_weights* w_bwd, int32_t* dx, int64_t M, int64_t K,
+                                     int64_t N, uint32_t flags, uint32_t* amax_io, void* stream);
+ds_status ds_conv2d_shift_backward_x(const int32_t* dy, const ds_weights* w_bwd, int32_t* dx, int N, int C, int H,
+                                     int W, int K, int R, int S, int stride_h, int stride_w, int pad_h, int pad_w,
+                                     uint32_t flags, uint32_t* amax_io, void* stream);
+
+/* ---------------------------------------------------------------------------
  * Conversion of float models (the step before packing).
  *
  * ds_quantize_shift_weights: the DeepShift-Q quantizer (Sec. 3.1, Eq. 4-6,

@@ -103,6 +103,14 @@ _SIGNATURES = {
     "ds_quantize_shift_weights": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_void_p,
                                                  ctypes.c_void_p, ctypes.c_void_p]),
     "ds_quantize_q16": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]),
+    "ds_pack_shift_weights_backward": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
+                                                      ctypes.c_int, ctypes.c_int, ctypes.c_void_p, ctypes.c_size_t,
+                                                      ctypes.c_void_p, ctypes.c_void_p]),
+    "ds_linear_shift_backward_x": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64,
+                                                  ctypes.c_int64, ctypes.c_int64, ctypes.c_uint32, ctypes.c_void_p,
+                                                  ctypes.c_void_p]),
+    "ds_conv2d_shift_backward_x": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p] +
+                                   [ctypes.c_int] * 11 + [ctypes.c_uint32, ctypes.c_void_p, ctypes.c_void_p]),
 }
 
 
@@ -220,6 +228,26 @@ def ds_absmax(x, n: int, amax, stream=None) -> None:
     _check(lib().ds_absmax(_ptr(x), n, _ptr(amax), _stream(stream)))
 
 
+def ds_pack_shift_weights_backward(s, p, K: int, C: int, R: int, S: int, packed, packed_bytes: int,
+                                   stream=None) -> ds_weights:
+    desc = ds_weights()
+    _check(lib().ds_pack_shift_weights_backward(_ptr(s), _ptr(p), K, C, R, S, _ptr(packed), packed_bytes,
+                                                ctypes.byref(desc), _stream(stream)))
+    return desc
+
+
+def ds_linear_shift_backward_x(dy, w: ds_weights, dx, M: int, K: int, N: int, flags: int = 0, amax_io=None,
+                               stream=None) -> None:
+    _check(lib().ds_linear_shift_backward_x(_ptr(dy), ctypes.byref(w), _ptr(dx), M, K, N, flags, _ptr(amax_io),
+                                            _stream(stream)))
+
+
+def ds_conv2d_shift_backward_x(dy, w: ds_weights, dx, N, C, H, W, K, R, S, stride_h, stride_w, pad_h, pad_w,
+                               flags: int = 0, amax_io=None, stream=None) -> None:
+    _check(lib().ds_conv2d_shift_backward_x(_ptr(dy), ctypes.byref(w), _ptr(dx), N, C, H, W, K, R, S, stride_h,
+                                            stride_w, pad_h, pad_w, flags, _ptr(amax_io), _stream(stream)))
+
+
 def ds_quantize_shift_weights(w, n: int, p_min: int, s, p, stream=None) -> None:
     _check(lib().ds_quantize_shift_weights(_ptr(w), n, p_min, _ptr(s), _ptr(p), _stream(stream)))
 
@@ -279,6 +307,27 @@ def linear_shift_bf16(x, w: PackedShiftWeights, bias=None, relu: bool = False, o
     y = out if out is not None else torch.empty((M, N), dtype=torch.float32, device=x.device)
     ds_linear_shift_bf16(x, w.desc, bias, y, M, K, N, DS_RELU if relu else 0, stream)
     return y
+
+
+def pack_shift_weights_backward(s, p, stream=None, expand: bool = False) -> PackedShiftWeights:
+    """Packs the input-gradient codes (rot180, channels swapped) of forward int8 codes [K, C, R, S] or
+    [N, K] (device); with expand=True also builds the expanded execution layout."""
+    import torch
+    if s.device.type != "cuda" or p.device.type != "cuda":
+        raise ValueError("codes must be CUDA tensors")
+    dims = tuple(s.shape) + (1,) * (4 - s.dim())
+    K, C, R, S = dims
+    s4 = s.reshape(dims).to(torch.int8).contiguous()
+    p4 = p.reshape(dims).to(torch.int8).contiguous()
+    nbytes = ds_packed_weight_bytes(C, K * R * S)
+    if nbytes == 0:
+        raise DsError(DS_ERR_SHAPE, "invalid code matrix shape")
+    blob = torch.empty(nbytes, dtype=torch.uint8, device=s.device)
+    desc = ds_pack_shift_weights_backward(s4, p4, K, C, R, S, blob, nbytes, stream)
+    w = PackedShiftWeights(blob, desc)
+    if expand:
+        expand_shift_weights(w, stream)
+    return w
 
 
 def quantize_shift_weights(w, p_min: int = -15, stream=None):

@@ -163,6 +163,9 @@ ds_status fc_launch(const int32_t* x, const ds_weights* w, const int32_t* bias, 
   return launch_fc(p, st);
 }
 
+ds_status pack_finish(const int8_t* s, const int8_t* p, int64_t n_out, int64_t k_red, void* packed, size_t need,
+                      ds_weights* desc, cudaStream_t st, const int* bwd);
+
 constexpr uint32_t kKnownFlags =
     DS_RELU | DS_AMAX_IN | DS_AMAX_OUT | DS_RESIDUAL | DS_FORCE_INT64 | DS_CONV_IM2COL;
 
@@ -197,9 +200,18 @@ ds_status ds_pack_shift_weights(const int8_t* s, const int8_t* p, int64_t n_out,
     return fail(DS_ERR_BUFFER_TOO_SMALL, "packed buffer has %zu bytes, needs %zu", packed_bytes, need);
   if ((reinterpret_cast<uintptr_t>(packed) & 255) != 0)
     return fail(DS_ERR_ALIGNMENT, "packed buffer must be 256-byte aligned");
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  return pack_finish(s, p, n_out, k_red, packed, need, desc, static_cast<cudaStream_t>(stream), nullptr);
+}
+
+}  // extern "C"
+
+namespace ds {
+// Launches the pack, waits for it and fills the descriptor (shared by the
+// forward and the input-gradient packing).
+ds_status pack_finish(const int8_t* s, const int8_t* p, int64_t n_out, int64_t k_red, void* packed, size_t need,
+                      ds_weights* desc, cudaStream_t st, const int* bwd) {
   uint8_t* blob = static_cast<uint8_t*>(packed);
-  ds_status r = cuda_check(launch_pack(s, p, n_out, k_red, blob, st), "pack launch");
+  ds_status r = cuda_check(launch_pack(s, p, n_out, k_red, blob, st, bwd), "pack launch");
   if (r != DS_OK) return r;
   BlobHeader h;
   r = cuda_check(cudaMemcpyAsync(&h, blob, sizeof(h), cudaMemcpyDeviceToHost, st), "header read");
@@ -223,6 +235,25 @@ ds_status ds_pack_shift_weights(const int8_t* s, const int8_t* p, int64_t n_out,
   desc->weights_bf16 = nullptr;
   desc->weights_bf16_bytes = 0;
   return DS_OK;
+}
+}  // namespace ds
+
+extern "C" {
+
+ds_status ds_pack_shift_weights_backward(const int8_t* s, const int8_t* p, int K, int C, int R, int S, void* packed,
+                                         size_t packed_bytes, ds_weights* desc, void* stream) {
+  clear_error();
+  if (!s || !p || !packed || !desc) return fail(DS_ERR_INVALID_ARG, "NULL pointer argument");
+  if (K <= 0 || C <= 0 || R <= 0 || S <= 0) return fail(DS_ERR_SHAPE, "K, C, R and S must be positive");
+  const int64_t n_out = C, k_red = (int64_t)K * R * S;
+  const size_t need = ds_packed_weight_bytes(n_out, k_red);
+  if (need == 0) return fail(DS_ERR_UNSUPPORTED, "code matrix too large");
+  if (packed_bytes < need)
+    return fail(DS_ERR_BUFFER_TOO_SMALL, "packed buffer has %zu bytes, needs %zu", packed_bytes, need);
+  if ((reinterpret_cast<uintptr_t>(packed) & 255) != 0)
+    return fail(DS_ERR_ALIGNMENT, "packed buffer must be 256-byte aligned");
+  const int dims[4] = {K, C, R, S};
+  return pack_finish(s, p, n_out, k_red, packed, need, desc, static_cast<cudaStream_t>(stream), dims);
 }
 
 size_t ds_expanded_weight_bytes(int64_t n_out, int64_t k_red) {
@@ -293,6 +324,71 @@ ds_status ds_linear_shift_bf16(const uint16_t* x, const ds_weights* w, const flo
 }
 
 int ds_bf16_fault_flag(void) { return read_bf16_fault_flag(); }
+
+ds_status ds_linear_shift_backward_x(const int32_t* dy, const ds_weights* w_bwd, int32_t* dx, int64_t M, int64_t K,
+                                     int64_t N, uint32_t flags, uint32_t* amax_io, void* stream) {
+  clear_error();
+  if (flags & ~(DS_AMAX_IN | DS_AMAX_OUT | DS_FORCE_INT64))
+    return fail(DS_ERR_INVALID_ARG, "only DS_AMAX_IN, DS_AMAX_OUT and DS_FORCE_INT64 apply to a gradient");
+  // dX [M][K] = dY [M][N] times the input-gradient codes (K columns, reduction N)
+  return ds_linear_shift(dy, w_bwd, nullptr, dx, M, N, K, flags, amax_io, stream);
+}
+
+ds_status ds_conv2d_shift_backward_x(const int32_t* dy, const ds_weights* w_bwd, int32_t* dx, int N, int C, int H,
+                                     int W, int K, int R, int S, int stride_h, int stride_w, int pad_h, int pad_w,
+                                     uint32_t flags, uint32_t* amax_io, void* stream) {
+  clear_error();
+  if (!dy || !dx) return fail(DS_ERR_INVALID_ARG, "NULL dy or dx");
+  if (N <= 0 || C <= 0 || H <= 0 || W <= 0 || K <= 0 || R <= 0 || S <= 0)
+    return fail(DS_ERR_SHAPE, "N, C, H, W, K, R, S must be positive");
+  if (stride_h <= 0 || stride_w <= 0 || pad_h < 0 || pad_w < 0)
+    return fail(DS_ERR_SHAPE, "strides must be positive and pads non-negative");
+  if (H + 2 * pad_h < R || W + 2 * pad_w < S) return fail(DS_ERR_SHAPE, "kernel larger than padded input");
+  if (flags & ~(DS_AMAX_IN | DS_AMAX_OUT | DS_FORCE_INT64 | DS_CONV_IM2COL))
+    return fail(DS_ERR_INVALID_ARG, "only DS_AMAX_IN, DS_AMAX_OUT, DS_FORCE_INT64, DS_CONV_IM2COL apply here");
+  if ((flags & (DS_AMAX_IN | DS_AMAX_OUT)) && amax_io == nullptr)
+    return fail(DS_ERR_INVALID_ARG, "DS_AMAX_IN / DS_AMAX_OUT need amax_io");
+  const int OH = (H + 2 * pad_h - R) / stride_h + 1;
+  const int OW = (W + 2 * pad_w - S) / stride_w + 1;
+  // stride 1: the forward ConvShift of dY with the rot180 / transposed codes and padding R-1-pad
+  if (stride_h == 1 && stride_w == 1 && pad_h <= R - 1 && pad_w <= S - 1 && !(flags & DS_CONV_IM2COL))
+    return ds_conv2d_shift(dy, w_bwd, nullptr, nullptr, dx, N, K, OH, OW, C, R, S, 1, 1, R - 1 - pad_h,
+                           S - 1 - pad_w, flags, amax_io, stream);
+  if (!aligned16(dy) || !aligned16(dx)) return fail(DS_ERR_ALIGNMENT, "dy and dx must be 16-byte aligned");
+  ds_status r = check_weights(w_bwd, C, (int64_t)K * R * S);
+  if (r != DS_OK) return r;
+  const int64_t ny = (int64_t)N * K * OH * OW, nx = (int64_t)N * C * H * W;
+  const char* ya = reinterpret_cast<const char*>(dy);
+  const char* xa = reinterpret_cast<const char*>(dx);
+  if (xa < ya + ny * 4 && ya < xa + nx * 4) return fail(DS_ERR_INVALID_ARG, "dx must not overlap dy");
+  if ((int64_t)H * W > (int64_t)1 << 30 || (int64_t)K * OH * OW > (int64_t)1 << 31)
+    return fail(DS_ERR_UNSUPPORTED, "image too large");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  GemmParams p{};
+  p.x = dy;
+  p.y = dx;
+  p.rows = (int64_t)N * H * W;
+  p.kred = (int64_t)K * R * S;
+  p.cols = C;
+  p.flags = flags & ~DS_CONV_IM2COL;
+  p.C = K;
+  p.H = OH;
+  p.W = OW;
+  p.R = R;
+  p.S = S;
+  p.sh = 1;
+  p.sw = 1;
+  p.ph = R - 1 - pad_h;
+  p.pw = S - 1 - pad_w;
+  p.OH = H;
+  p.OW = W;
+  p.dh = stride_h;
+  p.dw = stride_w;
+  fill_blob_offsets(p, w_bwd);
+  r = prepare_amax(dy, ny, flags, amax_io, st, p);
+  if (r != DS_OK) return r;
+  return cuda_check(launch_conv2d_shift(p, st), "conv2d_shift_backward_x (implicit GEMM) launch");
+}
 
 ds_status ds_quantize_shift_weights(const float* w, int64_t n, int p_min, int8_t* s, int8_t* p, void* stream) {
   clear_error();

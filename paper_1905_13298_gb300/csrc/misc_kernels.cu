@@ -11,7 +11,8 @@ namespace ds {
 // chunk, validates the codes, writes the nibble and bit-plane records and the
 // column constants A[n] and nnz[n], and folds them into the header maxima.
 __global__ void pack_kernel(const int8_t* __restrict__ s, const int8_t* __restrict__ p,
-                            int64_t n_out, int64_t k_red, uint8_t* __restrict__ blob) {
+                            int64_t n_out, int64_t k_red, uint8_t* __restrict__ blob, int bK, int bC, int bR,
+                            int bS) {
   const BlobLayout L = blob_layout(n_out, k_red);
   BlobHeader* hdr = reinterpret_cast<BlobHeader*>(blob);
   if (blockIdx.x == 0 && threadIdx.x == 0) {
@@ -23,8 +24,15 @@ __global__ void pack_kernel(const int8_t* __restrict__ s, const int8_t* __restri
   }
   const int64_t n = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (n >= n_out) return;
-  const int8_t* srow = s + n * k_red;
-  const int8_t* prow = p + n * k_red;
+  // forward: column n's codes are row n; input-gradient pass (bK > 0): column n is
+  // input channel n, index k = (k_out, r, q) reads code (k_out, n, bR-1-r, bS-1-q)
+  const int64_t rs = (int64_t)bR * bS;
+  auto offset = [&](int64_t k) -> int64_t {
+    if (bK == 0) return n * k_red + k;
+    const int64_t ko = k / rs, rem = k - ko * rs;
+    const int64_t r = rem / bS, q = rem - r * bS;
+    return ((ko * bC + n) * bR + (bR - 1 - r)) * bS + (bS - 1 - q);
+  };
   uint4* nib = reinterpret_cast<uint4*>(blob + L.nib);
   uint2* bits = reinterpret_cast<uint2*>(blob + L.bits);
   unsigned long long a_sum = 0;
@@ -35,8 +43,9 @@ __global__ void pack_kernel(const int8_t* __restrict__ s, const int8_t* __restri
     for (int j = 0; j < kChunk; ++j) {
       const int64_t k = g * kChunk + j;
       if (k >= k_red) break;
-      const int sv = srow[k];
-      const int pv = prow[k];
+      const int64_t o = offset(k);
+      const int sv = s[o];
+      const int pv = p[o];
       if (sv < -1 || sv > 1 || pv < -15 || pv > 0) {
         ++invalid;
         continue;
@@ -60,13 +69,17 @@ __global__ void pack_kernel(const int8_t* __restrict__ s, const int8_t* __restri
 }
 
 cudaError_t launch_pack(const int8_t* s, const int8_t* p, int64_t n_out, int64_t k_red,
-                        uint8_t* blob, cudaStream_t st) {
+                        uint8_t* blob, cudaStream_t st, const int* bwd) {
   // zero the whole blob: header counters, and the tail padding stays defined
   cudaError_t e = cudaMemsetAsync(blob, 0, (size_t)blob_layout(n_out, k_red).total, st);
   if (e != cudaSuccess) return e;
   const int threads = 128;
   const int64_t blocks = (n_out + threads - 1) / threads;
-  pack_kernel<<<(unsigned)blocks, threads, 0, st>>>(s, p, n_out, k_red, blob);
+  if (bwd != nullptr) {
+    pack_kernel<<<(unsigned)blocks, threads, 0, st>>>(s, p, n_out, k_red, blob, bwd[0], bwd[1], bwd[2], bwd[3]);
+  } else {
+    pack_kernel<<<(unsigned)blocks, threads, 0, st>>>(s, p, n_out, k_red, blob, 0, 0, 1, 1);
+  }
   return cudaGetLastError();
 }
 

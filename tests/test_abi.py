@@ -96,6 +96,19 @@ def test_validation_happens_before_cuda(ds):
     assert L.ds_linear_shift(4096, ctypes.byref(w2), None, 4096, 2, 8, 8, 0, None, None) == ds.DS_ERR_INVALID_ARG
     assert L.ds_absmax(None, 4, 16, None) == ds.DS_ERR_INVALID_ARG
     assert L.ds_absmax(16, 0, 16, None) == ds.DS_ERR_SHAPE
+    # input-gradient calls: bad flags (ReLU / residual / bias-like flags do not apply), shapes, buffers
+    assert L.ds_linear_shift_backward_x(16, ctypes.byref(w), 4096, 1, 1, 1, ds.DS_RELU, None, None) == ds.DS_ERR_INVALID_ARG
+    assert L.ds_conv2d_shift_backward_x(16, ctypes.byref(w), 4096, 1, 1, 3, 3, 1, 3, 3, 1, 1, 1, 1,
+                                        ds.DS_RESIDUAL, None, None) == ds.DS_ERR_INVALID_ARG
+    assert L.ds_conv2d_shift_backward_x(None, ctypes.byref(w), 4096, 1, 1, 3, 3, 1, 3, 3, 1, 1, 1, 1, 0, None,
+                                        None) == ds.DS_ERR_INVALID_ARG
+    assert L.ds_conv2d_shift_backward_x(16, ctypes.byref(w), 4096, 1, 1, 3, 3, 1, 3, 3, 0, 1, 1, 1, 0, None,
+                                        None) == ds.DS_ERR_SHAPE
+    assert L.ds_conv2d_shift_backward_x(16, ctypes.byref(w), 4096, 1, 1, 3, 3, 1, 3, 3, 2, 2, 1, 1, 0, None,
+                                        None) == ds.DS_ERR_INVALID_ARG  # unfilled descriptor
+    assert L.ds_pack_shift_weights_backward(16, 16, 4, 4, 3, 3, 256, 10, ctypes.byref(d), None) == ds.DS_ERR_BUFFER_TOO_SMALL
+    assert L.ds_pack_shift_weights_backward(16, 16, 4, 0, 3, 3, 256, 4096, ctypes.byref(d), None) == ds.DS_ERR_SHAPE
+    assert L.ds_pack_shift_weights_backward(16, 16, 4, 4, 1, 1, 272, 4096, ctypes.byref(d), None) == ds.DS_ERR_ALIGNMENT
     # quantizers: NULL pointers, p_min range, sizes, alignment
     assert L.ds_quantize_shift_weights(None, 4, -15, 16, 32, None) == ds.DS_ERR_INVALID_ARG
     assert L.ds_quantize_shift_weights(16, 4, -16, 16, 32, None) == ds.DS_ERR_INVALID_ARG

@@ -1,0 +1,109 @@
+"""GPU parity of the input gradient (Eq. 7 and its footnote) of LinearShift and ConvShift, and of the
+input-gradient code packing, against the CPU oracle (bit-exact)."""
+import numpy as np
+import pytest
+import torch
+
+import synth_inputs as si
+from oracle import deepshift_oracle as O
+
+pytestmark = pytest.mark.gpu
+
+
+def _dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+@pytest.mark.parametrize("dims", [(1, 1, 1, 1), (5, 3, 3, 3), (64, 33, 1, 1), (7, 40, 7, 7), (3, 70, 3, 2)])
+def test_pack_backward_blob_bitexact(dslib, dims):
+    K, C, R, S = dims
+    s = si.sign_codes(sum(dims), dims)
+    p = si.shift_codes_uniform(sum(dims), dims)
+    w = dslib.pack_shift_weights_backward(_dev(s), _dev(p))
+    sb, pb = O.backward_codes(s, p)
+    want = O.pack_planes6(sb.reshape(C, -1), pb.reshape(C, -1))
+    got = w.blob.cpu().numpy()
+    assert w.n_out == C and w.k_red == K * R * S
+    assert np.array_equal(got[:want.size], want)
+
+
+FC_SHAPES = [(1, 1, 1), (3, 7, 5), (64, 784, 512), (33, 130, 65), (200, 64, 1000)]
+
+
+@pytest.mark.parametrize("M,K,N", FC_SHAPES)
+@pytest.mark.parametrize("flags", [0, 16])
+@pytest.mark.parametrize("expand", [False, True])
+def test_linear_backward_x_bitexact(dslib, M, K, N, flags, expand):
+    s = si.sign_codes(M + K + N, (N, K))
+    p = si.shift_codes_uniform(M + K + N, (N, K))
+    dy = si.activations(M * 7 + N, (M, N), -(1 << 22), 1 << 22)
+    w = dslib.pack_shift_weights_backward(_dev(s), _dev(p), expand=expand)
+    dx = torch.empty((M, K), dtype=torch.int32, device="cuda")
+    amax = torch.zeros(2, dtype=torch.int32, device="cuda")
+    dslib.ds_linear_shift_backward_x(_dev(dy), w.desc, dx, M, K, N, flags | dslib.DS_AMAX_OUT, amax)
+    want = O.linear_shift_backward_x(dy, s, p)
+    assert np.array_equal(dx.cpu().numpy(), want)
+    assert amax.cpu().numpy().view(np.uint32)[1] == O.absmax(want)
+
+
+def test_linear_backward_x_saturates(dslib):
+    M, K, N = 9, 40, 300
+    s = si.sign_codes(1, (N, K))
+    p = np.zeros((N, K), np.int8)
+    dy = si.activations(2, (M, N), -(1 << 31), 1 << 31)
+    w = dslib.pack_shift_weights_backward(_dev(s), _dev(p))
+    dx = torch.empty((M, K), dtype=torch.int32, device="cuda")
+    amax = torch.zeros(2, dtype=torch.int32, device="cuda")
+    dslib.ds_linear_shift_backward_x(_dev(dy), w.desc, dx, M, K, N, 0, amax)
+    want = O.linear_shift_backward_x(dy, s, p)
+    assert (np.abs(O.linear_shift_backward_x_acc(dy, s, p)) > O.INT32_MAX).any()
+    assert np.array_equal(dx.cpu().numpy(), want)
+
+
+# N, C, H, W, K, R, S, stride, pad
+CONV_GEOMS = [
+    (2, 3, 7, 6, 4, 3, 3, 1, 1),
+    (2, 3, 7, 6, 4, 3, 3, 2, 1),
+    (1, 3, 23, 21, 16, 7, 7, 2, 3),     # stem-shaped
+    (2, 16, 9, 9, 20, 1, 1, 2, 0),      # 1x1 / 2 downsample
+    (1, 8, 11, 13, 70, 3, 3, 2, 1),
+    (3, 32, 8, 8, 64, 3, 3, 1, 1),
+    (1, 40, 7, 7, 130, 1, 1, 1, 0),
+    (1, 5, 6, 6, 3, 1, 1, 1, 1),        # pad > R - 1: the gather path even at stride 1
+    (2, 4, 10, 9, 6, 5, 3, 2, 2),       # non-square kernel
+]
+
+
+@pytest.mark.parametrize("geom", CONV_GEOMS)
+@pytest.mark.parametrize("flags", [0, 16, 32])  # default / forced 64-bit / forced gather path
+@pytest.mark.parametrize("expand", [False, True])
+def test_conv_backward_x_bitexact(dslib, geom, flags, expand):
+    N, C, H, W, K, R, S, st, pd = geom
+    s = si.sign_codes(sum(geom) * 3, (K, C, R, S))
+    p = si.shift_codes_uniform(sum(geom) * 3, (K, C, R, S))
+    OH, OW = O.conv_out_size(H, R, st, pd), O.conv_out_size(W, S, st, pd)
+    dy = si.activations(sum(geom) + flags, (N, K, OH, OW), -(1 << 22), 1 << 22)
+    w = dslib.pack_shift_weights_backward(_dev(s), _dev(p), expand=expand)
+    dx = torch.empty((N, C, H, W), dtype=torch.int32, device="cuda")
+    amax = torch.zeros(2, dtype=torch.int32, device="cuda")
+    dslib.ds_conv2d_shift_backward_x(_dev(dy), w.desc, dx, N, C, H, W, K, R, S, st, st, pd, pd,
+                                     flags | dslib.DS_AMAX_OUT, amax)
+    want = O.conv2d_shift_backward_x(dy, s, p, (H, W), (st, st), (pd, pd))
+    assert np.array_equal(dx.cpu().numpy(), want)
+    assert amax.cpu().numpy().view(np.uint32)[1] == O.absmax(want)
+
+
+@pytest.mark.parametrize("geom", [(2, 64, 56, 56, 64, 3, 3, 1, 1), (2, 64, 56, 56, 128, 1, 1, 2, 0),
+                                  (2, 64, 56, 56, 128, 3, 3, 2, 1)])
+def test_conv_backward_x_resnet_layers(dslib, geom):
+    """ResNet18 layer shapes (conv2_x, the 1x1/2 and 3x3/2 transitions), 2 images, every output."""
+    N, C, H, W, K, R, S, st, pd = geom
+    s = si.sign_codes(sum(geom), (K, C, R, S))
+    p = si.shift_codes_geometric(sum(geom), (K, C, R, S), -6)
+    OH, OW = O.conv_out_size(H, R, st, pd), O.conv_out_size(W, S, st, pd)
+    dy = si.activations(sum(geom) + 1, (N, K, OH, OW), -(1 << 20), 1 << 20)
+    w = dslib.pack_shift_weights_backward(_dev(s), _dev(p), expand=True)
+    dx = torch.empty((N, C, H, W), dtype=torch.int32, device="cuda")
+    amax = torch.zeros(2, dtype=torch.int32, device="cuda")
+    dslib.ds_conv2d_shift_backward_x(_dev(dy), w.desc, dx, N, C, H, W, K, R, S, st, st, pd, pd, 0, amax)
+    assert np.array_equal(dx.cpu().numpy(), O.conv2d_shift_backward_x(dy, s, p, (H, W), (st, st), (pd, pd)))
