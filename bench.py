@@ -70,6 +70,11 @@ def workload_by_name(name: str, batch):
         arch = name.split("_")[1]
         b = batch or (32 if arch == "resnet18" else 64)
         return dict(name=f"{arch}_conv_layer_sweep_b{b}_224", kind="sweep", arch=arch, N=b)
+    if name in ("sweep_resnet18_backward", "sweep_resnet50_backward"):
+        # the input gradient (Eq. 7) of every conv and FC layer, standalone
+        arch = name.split("_")[1]
+        b = batch or (32 if arch == "resnet18" else 64)
+        return dict(name=f"{arch}_input_gradient_layer_sweep_b{b}_224", kind="sweep", arch=arch, N=b, backward=True)
     if name in ("resnet18", "resnet50", "vgg16"):
         b = batch or (32 if name == "resnet18" else 64)
         return dict(name=f"{name}_shift_forward_b{b}_224", kind="net", arch=name, N=b)
@@ -359,19 +364,29 @@ def run_conversion(args, wl, local_rank):
     print(json.dumps(out), flush=True)
 
 
-def time_fc_layer(args, ds, dev, seed, M, K, N):
-    """One FC-shift layer standalone: codes geometric around the per-layer centre, as in the chain."""
+def time_fc_layer(args, ds, dev, seed, M, K, N, backward=False):
+    """One FC-shift layer standalone (or its input gradient): codes geometric around the per-layer
+    centre, as in the chain."""
     import torch
     x, s, p, b = si.fc_layer(seed, M, K, N, 0, 1 << 20, si.layer_centre(K, 1, 1))
-    w = ds.pack_shift_weights(torch.from_numpy(s).to(dev), torch.from_numpy(p).to(dev), expand=True)
-    xd, bd = torch.from_numpy(x).to(dev), torch.from_numpy(b).to(dev)
-    y = torch.empty((M, N), dtype=torch.int32, device=dev)
     a = torch.zeros(2, dtype=torch.int32, device=dev)
-    ds.ds_absmax(xd, xd.numel(), a)
     st = torch.cuda.current_stream().cuda_stream
+    if backward:
+        w = ds.pack_shift_weights_backward(torch.from_numpy(s).to(dev), torch.from_numpy(p).to(dev), expand=True)
+        dy = torch.from_numpy(si.activations(seed + 1, (M, N), -(1 << 20), 1 << 20)).to(dev)
+        dx = torch.empty((M, K), dtype=torch.int32, device=dev)
+        ds.ds_absmax(dy, dy.numel(), a)
 
-    def call():
-        ds.ds_linear_shift(xd, w.desc, bd, y, M, K, N, ds.DS_AMAX_IN, a, st)
+        def call():
+            ds.ds_linear_shift_backward_x(dy, w.desc[0], dx, M, K, N, ds.DS_AMAX_IN, a, st)
+    else:
+        w = ds.pack_shift_weights(torch.from_numpy(s).to(dev), torch.from_numpy(p).to(dev), expand=True)
+        xd, bd = torch.from_numpy(x).to(dev), torch.from_numpy(b).to(dev)
+        y = torch.empty((M, N), dtype=torch.int32, device=dev)
+        ds.ds_absmax(xd, xd.numel(), a)
+
+        def call():
+            ds.ds_linear_shift(xd, w.desc, bd, y, M, K, N, ds.DS_AMAX_IN, a, st)
     for _ in range(max(3, args.warmup)):
         call()
     torch.cuda.synchronize()
@@ -403,9 +418,10 @@ def run_layer_sweep(args, wl, local_rank):
     seen = {}
     rows = []
     tot_terms = tot_ms = 0.0
+    bwd = bool(wl.get("backward"))
     for i, sp in enumerate(specs):
         if sp.op == ds.DS_OP_FC:
-            r = time_fc_layer(args, ds, dev, si.SEED_BASE + 5 + i, B, sp.C * sp.H * sp.W, sp.K)
+            r = time_fc_layer(args, ds, dev, si.SEED_BASE + 5 + i, B, sp.C * sp.H * sp.W, sp.K, backward=bwd)
             r["layer"] = i
             rows.append(r)
             tot_terms += r["terms"]
@@ -421,18 +437,30 @@ def run_layer_sweep(args, wl, local_rank):
             continue
         x, s, p, b = si.conv_layer(si.SEED_BASE + 5 + i, B, sp.C, sp.H, sp.W, sp.K, sp.R, sp.S, 0, 1 << 20,
                                    si.layer_centre(sp.C, sp.R, sp.S))
-        w = ds.pack_shift_weights(torch.from_numpy(s).to(dev), torch.from_numpy(p).to(dev), expand=True)
-        xd, bd = torch.from_numpy(x).to(dev), torch.from_numpy(b).to(dev)
         OH = (sp.H + 2 * sp.pad - sp.R) // sp.stride + 1
         OW = (sp.W + 2 * sp.pad - sp.S) // sp.stride + 1
-        y = torch.empty((B, sp.K, OH, OW), dtype=torch.int32, device=dev)
-        a = torch.zeros(2, dtype=torch.int32, device=dev)
-        ds.ds_absmax(xd, xd.numel(), a)
         st = torch.cuda.current_stream().cuda_stream
+        a = torch.zeros(2, dtype=torch.int32, device=dev)
+        if bwd:
+            # dX [B, C, H, W] from a gradient dY [B, K, OH, OW] with the rot180 / transposed codes
+            w = ds.pack_shift_weights_backward(torch.from_numpy(s).to(dev), torch.from_numpy(p).to(dev),
+                                               (sp.stride, sp.stride), expand=True)
+            xd = torch.from_numpy(si.activations(si.SEED_BASE + 6 + i, (B, sp.K, OH, OW), -(1 << 20), 1 << 20)).to(dev)
+            y = torch.empty((B, sp.C, sp.H, sp.W), dtype=torch.int32, device=dev)
+            ds.ds_absmax(xd, xd.numel(), a)
 
-        def call():
-            ds.ds_conv2d_shift(xd, w.desc, bd, None, y, B, sp.C, sp.H, sp.W, sp.K, sp.R, sp.S, sp.stride, sp.stride,
-                               sp.pad, sp.pad, ds.DS_RELU | ds.DS_AMAX_IN, a, st)
+            def call():
+                ds.ds_conv2d_shift_backward_x(xd, w.desc, y, B, sp.C, sp.H, sp.W, sp.K, sp.R, sp.S, sp.stride,
+                                              sp.stride, sp.pad, sp.pad, ds.DS_AMAX_IN, a, st)
+        else:
+            w = ds.pack_shift_weights(torch.from_numpy(s).to(dev), torch.from_numpy(p).to(dev), expand=True)
+            xd, bd = torch.from_numpy(x).to(dev), torch.from_numpy(b).to(dev)
+            y = torch.empty((B, sp.K, OH, OW), dtype=torch.int32, device=dev)
+            ds.ds_absmax(xd, xd.numel(), a)
+
+            def call():
+                ds.ds_conv2d_shift(xd, w.desc, bd, None, y, B, sp.C, sp.H, sp.W, sp.K, sp.R, sp.S, sp.stride,
+                                   sp.stride, sp.pad, sp.pad, ds.DS_RELU | ds.DS_AMAX_IN, a, st)
         for _ in range(max(3, args.warmup)):
             call()
         torch.cuda.synchronize()
@@ -604,7 +632,8 @@ def main():
     ap.add_argument("--batch", type=int, default=None)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--workload", default="conv2x", choices=["conv2x", "fc_large", "fc_vgg16_fc1", "fc_large_bf16", "quantize_vgg16_fc1", "q16_input", "resnet18", "resnet50", "vgg16",
-                                                         "sweep_resnet18", "sweep_resnet50", "sweep_vgg16"])
+                                                         "sweep_resnet18", "sweep_resnet50", "sweep_vgg16",
+                                                         "sweep_resnet18_backward", "sweep_resnet50_backward"])
     ap.add_argument("--graph", action="store_true", help="replay each step from a CUDA graph (other workloads)")
     args = ap.parse_args()
     rank = int(os.environ.get("RANK", "0"))

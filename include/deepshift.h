@@ -324,29 +324,41 @@ ds_status ds_shift_forward(const ds_layer* layers, int n, const int32_t* x, int3
  * each term is the forward's shift-then-flip, s * (dy >> -p); the exact sum
  * is saturated to int32 (no bias, no ReLU).
  *
- * ds_pack_shift_weights_backward packs the code matrix of that pass from the
- * forward codes s, p (device int8, [K][C][R][S]; an FC layer's [N][K_in] is
- * K = N, C = K_in, R = S = 1): C columns, reduction length K*R*S, column c
- * and index (k, r, q) holding the code of (k, c, R-1-r, S-1-q).  Buffer size
- * ds_packed_weight_bytes(C, K*R*S); otherwise as ds_pack_shift_weights
- * (synchronises, DS_ERR_CODE_RANGE on bad codes).
+ * ds_pack_shift_weights_backward packs the code matrices of that pass from
+ * the forward codes s, p (device int8, [K][C][R][S]; an FC layer's [N][K_in]
+ * is K = N, C = K_in, R = S = 1, strides 1).  A layer of strides (sh, sw) has
+ * sh * sw tap phases (a, b): input position i = sh i' + rho receives only the
+ * taps r = a + sh t with a = (rho + pad) mod sh, so each phase is a stride-1
+ * correlation of dY with a sub-kernel of Th(a) = ceil((R - a) / sh) x Tw(b)
+ * taps.  Phase (a, b) is packed as a matrix of C columns and reduction length
+ * K * Th * Tw (index (k, t, u) holds the code of (k, c, a + sh (Th-1-t),
+ * b + sw (Tw-1-u)); for stride 1 this is W^rot180 with the channels swapped)
+ * into desc[a * sw + b]; a phase with no taps gets a descriptor with
+ * k_red = 0 and no blob.  desc points to sh * sw caller-owned descriptors,
+ * packed to ds_packed_weight_bytes_backward(K, C, R, S, sh, sw) bytes
+ * (256-byte aligned; phases at 256-byte aligned offsets).  Synchronises its
+ * stream once per phase; DS_ERR_CODE_RANGE on bad codes; strides in [1, 16].
  *
  * ds_linear_shift_backward_x: dx [M][K] from dy [M][N] (row-major, 16-byte
  * aligned) with w_bwd packed by ds_pack_shift_weights_backward(s, p, N, K,
- * 1, 1).  Flags: DS_AMAX_IN / DS_AMAX_OUT (amax_io as in ds_linear_shift)
- * and DS_FORCE_INT64 only.
+ * 1, 1, 1, 1, ...).  Flags: DS_AMAX_IN / DS_AMAX_OUT (amax_io as in
+ * ds_linear_shift) and DS_FORCE_INT64 only.
  *
  * ds_conv2d_shift_backward_x: dx [N][C][H][W] from dy [N][K][OH][OW] of the
  * forward geometry (H, W, R, S, strides, pads as given to ds_conv2d_shift;
- * OH = (H + 2 pad_h - R) / stride_h + 1, likewise OW), w_bwd packed by
- * ds_pack_shift_weights_backward(s, p, K, C, R, S).  Stride 1 runs the
- * forward ConvShift of dy with padding R-1-pad; larger strides run the
- * implicit GEMM whose gather reads dy at window positions divisible by the
- * stride.  Flags: DS_AMAX_IN, DS_AMAX_OUT, DS_FORCE_INT64, and
- * DS_CONV_IM2COL (the gather path at any stride).  Errors as ds_conv2d_shift.
+ * OH = (H + 2 pad_h - R) / stride_h + 1, likewise OW), w_bwd the
+ * stride_h * stride_w descriptors of ds_pack_shift_weights_backward(s, p, K,
+ * C, R, S, stride_h, stride_w, ...).  Stride 1 runs the forward ConvShift of
+ * dy with padding R-1-pad (direct / pointwise kernels); larger strides run one
+ * implicit GEMM per output phase (no term of a skipped window position is
+ * computed) and zero-fill the positions no tap reaches.  Flags: DS_AMAX_IN,
+ * DS_AMAX_OUT, DS_FORCE_INT64, and DS_CONV_IM2COL (the per-phase implicit
+ * GEMM also at stride 1).  Errors as ds_conv2d_shift.
  * ------------------------------------------------------------------------- */
-ds_status ds_pack_shift_weights_backward(const int8_t* s, const int8_t* p, int K, int C, int R, int S, void* packed,
-                                         size_t packed_bytes, ds_weights* desc, void* stream);
+size_t ds_packed_weight_bytes_backward(int K, int C, int R, int S, int stride_h, int stride_w);
+ds_status ds_pack_shift_weights_backward(const int8_t* s, const int8_t* p, int K, int C, int R, int S, int stride_h,
+                                         int stride_w, void* packed, size_t packed_bytes, ds_weights* desc,
+                                         void* stream);
 ds_status ds_linear_shift_backward_x(const int32_t* dy, const ds_weights* w_bwd, int32_t* dx, int64_t M, int64_t K,
                                      int64_t N, uint32_t flags, uint32_t* amax_io, void* stream);
 ds_status ds_conv2d_shift_backward_x(const int32_t* dy, const ds_weights* w_bwd, int32_t* dx, int N, int C, int H,

@@ -529,3 +529,38 @@ def backward_codes(s, p):
     st = np.ascontiguousarray(np.transpose(s[:, :, ::-1, ::-1], (1, 0, 2, 3)))
     pt = np.ascontiguousarray(np.transpose(p[:, :, ::-1, ::-1], (1, 0, 2, 3)))
     return st.astype(np.int8), pt.astype(np.int8)
+
+
+def phase_taps(R: int, stride: int, a: int) -> int:
+    """Number of taps r = a, a + stride, ... below R."""
+    return (R - 1 - a) // stride + 1 if a < R else 0
+
+
+def backward_phase_codes(s, p, stride):
+    """Input-gradient codes of a strided layer split by tap phase (a layout,
+    following Eq. 7's footnote): input row i = sh i' + rho receives only the
+    taps r = a + sh t, a = (rho + pad) mod sh.  For each phase (a, b) returns
+    [C, K, Th, Tw] arrays whose index (k, t, u) holds the code of
+    (k, c, a + sh (Th-1-t), b + sw (Tw-1-u)) -- rot180 of the phase's taps,
+    channels swapped -- or None when no tap has that phase.  Stride 1: the
+    single phase equals backward_codes."""
+    s = np.asarray(s)
+    p = np.asarray(p)
+    if s.ndim == 2:
+        s, p = s[:, :, None, None], p[:, :, None, None]
+    K, C, R, S = s.shape
+    sh, sw = stride
+    out = {}
+    for a in range(sh):
+        for b in range(sw):
+            th, tw = phase_taps(R, sh, a), phase_taps(S, sw, b)
+            if th == 0 or tw == 0:
+                out[(a, b)] = None
+                continue
+            rows = [a + sh * (th - 1 - t) for t in range(th)]
+            cols = [b + sw * (tw - 1 - u) for u in range(tw)]
+            ss = s[:, :, rows][:, :, :, cols]
+            pp = p[:, :, rows][:, :, :, cols]
+            out[(a, b)] = (np.ascontiguousarray(np.transpose(ss, (1, 0, 2, 3))).astype(np.int8),
+                           np.ascontiguousarray(np.transpose(pp, (1, 0, 2, 3))).astype(np.int8))
+    return out

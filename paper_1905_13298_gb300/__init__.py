@@ -103,9 +103,9 @@ _SIGNATURES = {
     "ds_quantize_shift_weights": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_void_p,
                                                  ctypes.c_void_p, ctypes.c_void_p]),
     "ds_quantize_q16": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]),
-    "ds_pack_shift_weights_backward": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
-                                                      ctypes.c_int, ctypes.c_int, ctypes.c_void_p, ctypes.c_size_t,
-                                                      ctypes.c_void_p, ctypes.c_void_p]),
+    "ds_packed_weight_bytes_backward": (ctypes.c_size_t, [ctypes.c_int] * 6),
+    "ds_pack_shift_weights_backward": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p] + [ctypes.c_int] * 6 +
+                                       [ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p, ctypes.c_void_p]),
     "ds_linear_shift_backward_x": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64,
                                                   ctypes.c_int64, ctypes.c_int64, ctypes.c_uint32, ctypes.c_void_p,
                                                   ctypes.c_void_p]),
@@ -228,12 +228,17 @@ def ds_absmax(x, n: int, amax, stream=None) -> None:
     _check(lib().ds_absmax(_ptr(x), n, _ptr(amax), _stream(stream)))
 
 
-def ds_pack_shift_weights_backward(s, p, K: int, C: int, R: int, S: int, packed, packed_bytes: int,
-                                   stream=None) -> ds_weights:
-    desc = ds_weights()
-    _check(lib().ds_pack_shift_weights_backward(_ptr(s), _ptr(p), K, C, R, S, _ptr(packed), packed_bytes,
-                                                ctypes.byref(desc), _stream(stream)))
-    return desc
+def ds_packed_weight_bytes_backward(K: int, C: int, R: int, S: int, stride_h: int = 1, stride_w: int = 1) -> int:
+    return int(lib().ds_packed_weight_bytes_backward(K, C, R, S, stride_h, stride_w))
+
+
+def ds_pack_shift_weights_backward(s, p, K: int, C: int, R: int, S: int, stride_h: int, stride_w: int, packed,
+                                   packed_bytes: int, stream=None):
+    """Returns a ctypes array of stride_h * stride_w descriptors (one per tap phase)."""
+    descs = (ds_weights * (stride_h * stride_w))()
+    _check(lib().ds_pack_shift_weights_backward(_ptr(s), _ptr(p), K, C, R, S, stride_h, stride_w, _ptr(packed),
+                                                packed_bytes, descs, _stream(stream)))
+    return descs
 
 
 def ds_linear_shift_backward_x(dy, w: ds_weights, dx, M: int, K: int, N: int, flags: int = 0, amax_io=None,
@@ -242,9 +247,11 @@ def ds_linear_shift_backward_x(dy, w: ds_weights, dx, M: int, K: int, N: int, fl
                                             _stream(stream)))
 
 
-def ds_conv2d_shift_backward_x(dy, w: ds_weights, dx, N, C, H, W, K, R, S, stride_h, stride_w, pad_h, pad_w,
+def ds_conv2d_shift_backward_x(dy, w, dx, N, C, H, W, K, R, S, stride_h, stride_w, pad_h, pad_w,
                                flags: int = 0, amax_io=None, stream=None) -> None:
-    _check(lib().ds_conv2d_shift_backward_x(_ptr(dy), ctypes.byref(w), _ptr(dx), N, C, H, W, K, R, S, stride_h,
+    """w: the ctypes descriptor array of ds_pack_shift_weights_backward (or one descriptor for stride 1)."""
+    ref = w if isinstance(w, ctypes.Array) else ctypes.byref(w)
+    _check(lib().ds_conv2d_shift_backward_x(_ptr(dy), ref, _ptr(dx), N, C, H, W, K, R, S, stride_h,
                                             stride_w, pad_h, pad_w, flags, _ptr(amax_io), _stream(stream)))
 
 
@@ -309,24 +316,47 @@ def linear_shift_bf16(x, w: PackedShiftWeights, bias=None, relu: bool = False, o
     return y
 
 
-def pack_shift_weights_backward(s, p, stream=None, expand: bool = False) -> PackedShiftWeights:
-    """Packs the input-gradient codes (rot180, channels swapped) of forward int8 codes [K, C, R, S] or
-    [N, K] (device); with expand=True also builds the expanded execution layout."""
+class PackedBackwardWeights:
+    """The input-gradient codes of one layer: a device blob holding one packed matrix per tap phase,
+    the ctypes array of their descriptors, and optionally each phase's expanded layout."""
+
+    def __init__(self, blob, descs, stride):
+        self.blob = blob
+        self.desc = descs  # pass to ds_conv2d_shift_backward_x; descs[0] to ds_linear_shift_backward_x
+        self.stride = stride
+        self.expanded = []
+
+    def expand(self, stream=None):
+        import torch
+        for d in self.desc:
+            if d.k_red == 0:
+                continue
+            nbytes = ds_expanded_weight_bytes(d.n_out, d.k_red)
+            buf = torch.empty(nbytes // 4, dtype=torch.int32, device=self.blob.device)
+            ds_expand_shift_weights(d, buf, nbytes, stream)
+            self.expanded.append(buf)
+        return self
+
+
+def pack_shift_weights_backward(s, p, stride=(1, 1), stream=None, expand: bool = False) -> PackedBackwardWeights:
+    """Packs the input-gradient codes (Eq. 7 footnote: rot180, channels swapped, split into the tap phases
+    of a strided layer) of forward int8 codes [K, C, R, S] or [N, K] (device)."""
     import torch
     if s.device.type != "cuda" or p.device.type != "cuda":
         raise ValueError("codes must be CUDA tensors")
     dims = tuple(s.shape) + (1,) * (4 - s.dim())
     K, C, R, S = dims
+    sh, sw = stride
     s4 = s.reshape(dims).to(torch.int8).contiguous()
     p4 = p.reshape(dims).to(torch.int8).contiguous()
-    nbytes = ds_packed_weight_bytes(C, K * R * S)
+    nbytes = ds_packed_weight_bytes_backward(K, C, R, S, sh, sw)
     if nbytes == 0:
         raise DsError(DS_ERR_SHAPE, "invalid code matrix shape")
     blob = torch.empty(nbytes, dtype=torch.uint8, device=s.device)
-    desc = ds_pack_shift_weights_backward(s4, p4, K, C, R, S, blob, nbytes, stream)
-    w = PackedShiftWeights(blob, desc)
+    descs = ds_pack_shift_weights_backward(s4, p4, K, C, R, S, sh, sw, blob, nbytes, stream)
+    w = PackedBackwardWeights(blob, descs, (sh, sw))
     if expand:
-        expand_shift_weights(w, stream)
+        w.expand(stream)
     return w
 
 

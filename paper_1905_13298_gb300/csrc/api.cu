@@ -166,6 +166,9 @@ ds_status fc_launch(const int32_t* x, const ds_weights* w, const int32_t* bias, 
 ds_status pack_finish(const int8_t* s, const int8_t* p, int64_t n_out, int64_t k_red, void* packed, size_t need,
                       ds_weights* desc, cudaStream_t st, const int* bwd);
 
+// Taps r = a, a + stride, ... < R of tap phase a (the input-gradient decomposition of a strided layer).
+static int phase_taps(int R, int stride, int a) { return a < R ? (R - 1 - a) / stride + 1 : 0; }
+
 constexpr uint32_t kKnownFlags =
     DS_RELU | DS_AMAX_IN | DS_AMAX_OUT | DS_RESIDUAL | DS_FORCE_INT64 | DS_CONV_IM2COL;
 
@@ -240,20 +243,56 @@ ds_status pack_finish(const int8_t* s, const int8_t* p, int64_t n_out, int64_t k
 
 extern "C" {
 
-ds_status ds_pack_shift_weights_backward(const int8_t* s, const int8_t* p, int K, int C, int R, int S, void* packed,
-                                         size_t packed_bytes, ds_weights* desc, void* stream) {
+size_t ds_packed_weight_bytes_backward(int K, int C, int R, int S, int stride_h, int stride_w) {
+  if (K <= 0 || C <= 0 || R <= 0 || S <= 0 || stride_h <= 0 || stride_w <= 0) return 0;
+  size_t total = 0;
+  for (int a = 0; a < stride_h; ++a)
+    for (int b = 0; b < stride_w; ++b) {
+      const int th = phase_taps(R, stride_h, a), tw = phase_taps(S, stride_w, b);
+      if (th == 0 || tw == 0) continue;
+      const size_t one = ds_packed_weight_bytes(C, (int64_t)K * th * tw);
+      if (one == 0) return 0;
+      total += (one + 255) / 256 * 256;
+    }
+  return total;
+}
+
+ds_status ds_pack_shift_weights_backward(const int8_t* s, const int8_t* p, int K, int C, int R, int S, int stride_h,
+                                         int stride_w, void* packed, size_t packed_bytes, ds_weights* desc,
+                                         void* stream) {
   clear_error();
   if (!s || !p || !packed || !desc) return fail(DS_ERR_INVALID_ARG, "NULL pointer argument");
   if (K <= 0 || C <= 0 || R <= 0 || S <= 0) return fail(DS_ERR_SHAPE, "K, C, R and S must be positive");
-  const int64_t n_out = C, k_red = (int64_t)K * R * S;
-  const size_t need = ds_packed_weight_bytes(n_out, k_red);
+  if (stride_h <= 0 || stride_w <= 0 || stride_h > 16 || stride_w > 16)
+    return fail(DS_ERR_SHAPE, "strides must be in [1, 16]");
+  const size_t need = ds_packed_weight_bytes_backward(K, C, R, S, stride_h, stride_w);
   if (need == 0) return fail(DS_ERR_UNSUPPORTED, "code matrix too large");
   if (packed_bytes < need)
     return fail(DS_ERR_BUFFER_TOO_SMALL, "packed buffer has %zu bytes, needs %zu", packed_bytes, need);
   if ((reinterpret_cast<uintptr_t>(packed) & 255) != 0)
     return fail(DS_ERR_ALIGNMENT, "packed buffer must be 256-byte aligned");
-  const int dims[4] = {K, C, R, S};
-  return pack_finish(s, p, n_out, k_red, packed, need, desc, static_cast<cudaStream_t>(stream), dims);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  size_t off = 0;
+  for (int a = 0; a < stride_h; ++a)
+    for (int b = 0; b < stride_w; ++b) {
+      ds_weights& d = desc[a * stride_w + b];
+      const int th = phase_taps(R, stride_h, a), tw = phase_taps(S, stride_w, b);
+      if (th == 0 || tw == 0) {  // a phase no tap reaches: its input-gradient positions are zero
+        d = ds_weights{};
+        d.magic = DS_WEIGHTS_MAGIC;
+        d.format = DS_FORMAT_PLANES6;
+        d.n_out = C;
+        d.k_red = 0;
+        continue;
+      }
+      const int64_t k_red = (int64_t)K * th * tw;
+      const size_t one = ds_packed_weight_bytes(C, k_red);
+      const int map[10] = {K, C, R, S, stride_h, stride_w, a, b, th, tw};
+      ds_status r = pack_finish(s, p, C, k_red, static_cast<unsigned char*>(packed) + off, one, &d, st, map);
+      if (r != DS_OK) return r;
+      off += (one + 255) / 256 * 256;
+    }
+  return DS_OK;
 }
 
 size_t ds_expanded_weight_bytes(int64_t n_out, int64_t k_red) {
@@ -338,11 +377,11 @@ ds_status ds_conv2d_shift_backward_x(const int32_t* dy, const ds_weights* w_bwd,
                                      int W, int K, int R, int S, int stride_h, int stride_w, int pad_h, int pad_w,
                                      uint32_t flags, uint32_t* amax_io, void* stream) {
   clear_error();
-  if (!dy || !dx) return fail(DS_ERR_INVALID_ARG, "NULL dy or dx");
+  if (!dy || !dx || !w_bwd) return fail(DS_ERR_INVALID_ARG, "NULL dy, dx or weights");
   if (N <= 0 || C <= 0 || H <= 0 || W <= 0 || K <= 0 || R <= 0 || S <= 0)
     return fail(DS_ERR_SHAPE, "N, C, H, W, K, R, S must be positive");
-  if (stride_h <= 0 || stride_w <= 0 || pad_h < 0 || pad_w < 0)
-    return fail(DS_ERR_SHAPE, "strides must be positive and pads non-negative");
+  if (stride_h <= 0 || stride_w <= 0 || stride_h > 16 || stride_w > 16 || pad_h < 0 || pad_w < 0)
+    return fail(DS_ERR_SHAPE, "strides must be in [1, 16] and pads non-negative");
   if (H + 2 * pad_h < R || W + 2 * pad_w < S) return fail(DS_ERR_SHAPE, "kernel larger than padded input");
   if (flags & ~(DS_AMAX_IN | DS_AMAX_OUT | DS_FORCE_INT64 | DS_CONV_IM2COL))
     return fail(DS_ERR_INVALID_ARG, "only DS_AMAX_IN, DS_AMAX_OUT, DS_FORCE_INT64, DS_CONV_IM2COL apply here");
@@ -350,13 +389,26 @@ ds_status ds_conv2d_shift_backward_x(const int32_t* dy, const ds_weights* w_bwd,
     return fail(DS_ERR_INVALID_ARG, "DS_AMAX_IN / DS_AMAX_OUT need amax_io");
   const int OH = (H + 2 * pad_h - R) / stride_h + 1;
   const int OW = (W + 2 * pad_w - S) / stride_w + 1;
+  // one descriptor per tap phase (a, b), as ds_pack_shift_weights_backward fills them
+  bool empty_phase = false;
+  for (int a = 0; a < stride_h; ++a)
+    for (int b = 0; b < stride_w; ++b) {
+      const ds_weights& d = w_bwd[a * stride_w + b];
+      const int th = phase_taps(R, stride_h, a), tw = phase_taps(S, stride_w, b);
+      if (th == 0 || tw == 0) {
+        if (d.magic != DS_WEIGHTS_MAGIC || d.n_out != C || d.k_red != 0)
+          return fail(DS_ERR_INVALID_ARG, "phase (%d, %d): descriptor does not match the layer", a, b);
+        empty_phase = true;
+        continue;
+      }
+      ds_status r = check_weights(&d, C, (int64_t)K * th * tw);
+      if (r != DS_OK) return r;
+    }
   // stride 1: the forward ConvShift of dY with the rot180 / transposed codes and padding R-1-pad
   if (stride_h == 1 && stride_w == 1 && pad_h <= R - 1 && pad_w <= S - 1 && !(flags & DS_CONV_IM2COL))
     return ds_conv2d_shift(dy, w_bwd, nullptr, nullptr, dx, N, K, OH, OW, C, R, S, 1, 1, R - 1 - pad_h,
                            S - 1 - pad_w, flags, amax_io, stream);
   if (!aligned16(dy) || !aligned16(dx)) return fail(DS_ERR_ALIGNMENT, "dy and dx must be 16-byte aligned");
-  ds_status r = check_weights(w_bwd, C, (int64_t)K * R * S);
-  if (r != DS_OK) return r;
   const int64_t ny = (int64_t)N * K * OH * OW, nx = (int64_t)N * C * H * W;
   const char* ya = reinterpret_cast<const char*>(dy);
   const char* xa = reinterpret_cast<const char*>(dx);
@@ -364,30 +416,51 @@ ds_status ds_conv2d_shift_backward_x(const int32_t* dy, const ds_weights* w_bwd,
   if ((int64_t)H * W > (int64_t)1 << 30 || (int64_t)K * OH * OW > (int64_t)1 << 31)
     return fail(DS_ERR_UNSUPPORTED, "image too large");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  GemmParams p{};
-  p.x = dy;
-  p.y = dx;
-  p.rows = (int64_t)N * H * W;
-  p.kred = (int64_t)K * R * S;
-  p.cols = C;
-  p.flags = flags & ~DS_CONV_IM2COL;
-  p.C = K;
-  p.H = OH;
-  p.W = OW;
-  p.R = R;
-  p.S = S;
-  p.sh = 1;
-  p.sw = 1;
-  p.ph = R - 1 - pad_h;
-  p.pw = S - 1 - pad_w;
-  p.OH = H;
-  p.OW = W;
-  p.dh = stride_h;
-  p.dw = stride_w;
-  fill_blob_offsets(p, w_bwd);
-  r = prepare_amax(dy, ny, flags, amax_io, st, p);
+  GemmParams base{};
+  base.flags = flags & ~DS_CONV_IM2COL;
+  ds_status r = prepare_amax(dy, ny, flags, amax_io, st, base);
   if (r != DS_OK) return r;
-  return cuda_check(launch_conv2d_shift(p, st), "conv2d_shift_backward_x (implicit GEMM) launch");
+  if (empty_phase) {
+    r = cuda_check(cudaMemsetAsync(dx, 0, (size_t)nx * sizeof(int32_t), st), "dx reset");
+    if (r != DS_OK) return r;
+  }
+  // output phase (rh, rw): dX rows rh, rh + sh, ...; they receive the taps r = a + sh t with
+  // a = (rh + pad_h) mod sh, reading gradient row i' + c_h - t (i = sh i' + rh, c_h = (rh + pad_h - a) / sh):
+  // a stride-1 correlation of dY with the phase's Th x Tw sub-kernel and padding Th - 1 - c_h
+  for (int rh = 0; rh < stride_h && rh < H; ++rh)
+    for (int rw = 0; rw < stride_w && rw < W; ++rw) {
+      const int a = (rh + pad_h) % stride_h, b = (rw + pad_w) % stride_w;
+      const int th = phase_taps(R, stride_h, a), tw = phase_taps(S, stride_w, b);
+      if (th == 0 || tw == 0) continue;
+      const int ch = (rh + pad_h - a) / stride_h, cw = (rw + pad_w - b) / stride_w;
+      GemmParams p = base;
+      p.x = dy;
+      p.y = dx;
+      p.C = K;
+      p.H = OH;
+      p.W = OW;
+      p.R = th;
+      p.S = tw;
+      p.sh = 1;
+      p.sw = 1;
+      p.ph = th - 1 - ch;
+      p.pw = tw - 1 - cw;
+      p.OH = (H - rh + stride_h - 1) / stride_h;
+      p.OW = (W - rw + stride_w - 1) / stride_w;
+      p.rows = (int64_t)N * p.OH * p.OW;
+      p.kred = (int64_t)K * th * tw;
+      p.cols = C;
+      p.ys_h = stride_h;
+      p.ys_w = stride_w;
+      p.yph = rh;
+      p.ypw = rw;
+      p.yH = H;
+      p.yW = W;
+      fill_blob_offsets(p, &w_bwd[a * stride_w + b]);
+      r = cuda_check(launch_conv2d_shift(p, st), "conv2d_shift_backward_x (implicit GEMM) launch");
+      if (r != DS_OK) return r;
+    }
+  return DS_OK;
 }
 
 ds_status ds_quantize_shift_weights(const float* w, int64_t n, int p_min, int8_t* s, int8_t* p, void* stream) {

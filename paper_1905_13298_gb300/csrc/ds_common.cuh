@@ -72,9 +72,10 @@ struct GemmParams {
   int64_t off_nib, off_bits, off_cola, off_nnz;
   // conv geometry (unused by FC)
   int C, H, W, R, S, sh, sw, ph, pw, OH, OW;
-  // implicit GEMM, input-gradient gather: output (dX) pixel i reads window row
-  // u = i - ph + r of the gradient, row u / dh when dh divides u (0: forward gather)
-  int dh, dw;
+  // implicit GEMM output placement (0: dense): output pixel (oh, ow) is stored
+  // at (ys_h * oh + yph, ys_w * ow + ypw) of a yH x yW plane (one phase of a
+  // strided layer's input gradient)
+  int ys_h, ys_w, yph, ypw, yH, yW;
   uint32_t flags;
   // split reduction (conv, chained forward only): int64 partial sums of every output, zeroed first
   int64_t* split_acc;       // nullable
@@ -125,8 +126,9 @@ cudaError_t launch_quantize_weights(const float* w, int64_t n, int p_min, int8_t
 cudaError_t launch_quantize_q16(const float* x, int64_t n, int32_t* q, cudaStream_t st);
 // Defined in misc_kernels.cu.
 cudaError_t launch_absmax(const int32_t* x, int64_t n, uint32_t* out, cudaStream_t st);
-// bwd != nullptr: pack the input-gradient code matrix of forward codes [K][C][R][S]
-// (bwd = {K, C, R, S}; column c, index (k, r, q) reads code (k, c, R-1-r, S-1-q)).
+// bwd != nullptr: pack one phase of the input-gradient codes of forward codes
+// [K][C][R][S]: bwd = {K, C, R, S, sh, sw, a, b, Th, Tw}; column c, index
+// (k, t, u) reads code (k, c, a + sh (Th-1-t), b + sw (Tw-1-u)).
 cudaError_t launch_pack(const int8_t* s, const int8_t* p, int64_t n_out, int64_t k_red,
                         uint8_t* blob, cudaStream_t st, const int* bwd = nullptr);
 cudaError_t launch_expand(const uint8_t* blob, int64_t n_out, int64_t k_red, int32_t* out, cudaStream_t st);

@@ -10,9 +10,12 @@ namespace ds {
 // One thread per output column: walks the column's reduction range chunk by
 // chunk, validates the codes, writes the nibble and bit-plane records and the
 // column constants A[n] and nnz[n], and folds them into the header maxima.
+struct BwdMap {
+  int K, C, R, S, sh, sw, a, b, Th, Tw;  // K == 0: forward layout
+};
+
 __global__ void pack_kernel(const int8_t* __restrict__ s, const int8_t* __restrict__ p,
-                            int64_t n_out, int64_t k_red, uint8_t* __restrict__ blob, int bK, int bC, int bR,
-                            int bS) {
+                            int64_t n_out, int64_t k_red, uint8_t* __restrict__ blob, const BwdMap m) {
   const BlobLayout L = blob_layout(n_out, k_red);
   BlobHeader* hdr = reinterpret_cast<BlobHeader*>(blob);
   if (blockIdx.x == 0 && threadIdx.x == 0) {
@@ -24,14 +27,16 @@ __global__ void pack_kernel(const int8_t* __restrict__ s, const int8_t* __restri
   }
   const int64_t n = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (n >= n_out) return;
-  // forward: column n's codes are row n; input-gradient pass (bK > 0): column n is
-  // input channel n, index k = (k_out, r, q) reads code (k_out, n, bR-1-r, bS-1-q)
-  const int64_t rs = (int64_t)bR * bS;
+  // forward: column n's codes are row n.  Input-gradient phase (m.K > 0):
+  // column n is input channel n, index k = (k_out, t, u) reads the code of tap
+  // (m.a + m.sh (Th-1-t), m.b + m.sw (Tw-1-u)) of (k_out, n)
+  const int64_t tt = (int64_t)m.Th * m.Tw;
   auto offset = [&](int64_t k) -> int64_t {
-    if (bK == 0) return n * k_red + k;
-    const int64_t ko = k / rs, rem = k - ko * rs;
-    const int64_t r = rem / bS, q = rem - r * bS;
-    return ((ko * bC + n) * bR + (bR - 1 - r)) * bS + (bS - 1 - q);
+    if (m.K == 0) return n * k_red + k;
+    const int64_t ko = k / tt, rem = k - ko * tt;
+    const int64_t t = rem / m.Tw, u = rem - t * m.Tw;
+    const int64_t r = m.a + (int64_t)m.sh * (m.Th - 1 - t), q = m.b + (int64_t)m.sw * (m.Tw - 1 - u);
+    return ((ko * m.C + n) * m.R + r) * m.S + q;
   };
   uint4* nib = reinterpret_cast<uint4*>(blob + L.nib);
   uint2* bits = reinterpret_cast<uint2*>(blob + L.bits);
@@ -75,11 +80,9 @@ cudaError_t launch_pack(const int8_t* s, const int8_t* p, int64_t n_out, int64_t
   if (e != cudaSuccess) return e;
   const int threads = 128;
   const int64_t blocks = (n_out + threads - 1) / threads;
-  if (bwd != nullptr) {
-    pack_kernel<<<(unsigned)blocks, threads, 0, st>>>(s, p, n_out, k_red, blob, bwd[0], bwd[1], bwd[2], bwd[3]);
-  } else {
-    pack_kernel<<<(unsigned)blocks, threads, 0, st>>>(s, p, n_out, k_red, blob, 0, 0, 1, 1);
-  }
+  BwdMap m{0, 0, 1, 1, 1, 1, 0, 0, 1, 1};
+  if (bwd != nullptr) m = BwdMap{bwd[0], bwd[1], bwd[2], bwd[3], bwd[4], bwd[5], bwd[6], bwd[7], bwd[8], bwd[9]};
+  pack_kernel<<<(unsigned)blocks, threads, 0, st>>>(s, p, n_out, k_red, blob, m);
   return cudaGetLastError();
 }
 

@@ -112,39 +112,18 @@ __device__ __forceinline__ void stage_x(const GemmParams& P, Smem& sm, int buf, 
     int s = rem - r * P.S;
     const int64_t HW = (int64_t)P.H * P.W;
     int32_t* dst = xs + t * XS;
-    if (P.dh == 0) {
 #pragma unroll 4
-      for (int kk = 0; kk < kChunk; ++kk) {
-        const int ih = rc.ih0 + r, iw = rc.iw0 + s;
-        const bool ok = rc.valid && (k + kk < P.kred) && ((unsigned)ih < (unsigned)P.H) &&
-                        ((unsigned)iw < (unsigned)P.W);
-        const int32_t* src = ok ? (P.x + rc.img_base + (int64_t)c * HW + (int64_t)ih * P.W + iw) : P.x;
-        cp_async4(dst + kk, src, ok);
-        if (++s == P.S) {
-          s = 0;
-          if (++r == P.R) {
-            r = 0;
-            ++c;
-          }
-        }
-      }
-    } else {
-      // input-gradient gather: window position (u, v) holds gradient (u / dh, v / dw)
-      // when both divide, zero otherwise (the positions a strided forward skipped)
-#pragma unroll 4
-      for (int kk = 0; kk < kChunk; ++kk) {
-        const int u = rc.ih0 + r, v = rc.iw0 + s;
-        const int ih = u / P.dh, iw = v / P.dw;
-        const bool ok = rc.valid && (k + kk < P.kred) && u >= 0 && v >= 0 && ih * P.dh == u && iw * P.dw == v &&
-                        ih < P.H && iw < P.W;
-        const int32_t* src = ok ? (P.x + rc.img_base + (int64_t)c * HW + (int64_t)ih * P.W + iw) : P.x;
-        cp_async4(dst + kk, src, ok);
-        if (++s == P.S) {
-          s = 0;
-          if (++r == P.R) {
-            r = 0;
-            ++c;
-          }
+    for (int kk = 0; kk < kChunk; ++kk) {
+      const int ih = rc.ih0 + r, iw = rc.iw0 + s;
+      const bool ok = rc.valid && (k + kk < P.kred) && ((unsigned)ih < (unsigned)P.H) &&
+                      ((unsigned)iw < (unsigned)P.W);
+      const int32_t* src = ok ? (P.x + rc.img_base + (int64_t)c * HW + (int64_t)ih * P.W + iw) : P.x;
+      cp_async4(dst + kk, src, ok);
+      if (++s == P.S) {
+        s = 0;
+        if (++r == P.R) {
+          r = 0;
+          ++c;
         }
       }
     }
@@ -320,11 +299,18 @@ __device__ __forceinline__ void run_tile(const GemmParams& P, Smem& sm, int64_t 
     } else {
       const int64_t n = row / OHW;
       const int64_t pix = row - n * OHW;
+      // output placement: pixel (oh, ow) of this grid -> (ys_h oh + yph, ys_w ow + ypw) of a yH x yW plane
+      int64_t plane = OHW, off = pix;
+      if (P.ys_h) {
+        const int oh = (int)(pix / P.OW), ow = (int)(pix - (pix / P.OW) * P.OW);
+        plane = (int64_t)P.yH * P.yW;
+        off = (int64_t)(P.ys_h * oh + P.yph) * P.yW + P.ys_w * ow + P.ypw;
+      }
 #pragma unroll
       for (int j = 0; j < TN; ++j) {
         const int64_t col = col0 + tn * TN + j;
         if (col >= P.cols) continue;
-        const int64_t idx = (n * P.cols + col) * OHW + pix;
+        const int64_t idx = (n * P.cols + col) * plane + off;
         int32_t o = v[j];
         if (resid) o = add_sat(o, __ldg(P.residual + idx));
         if (relu) o = max(o, 0);
@@ -378,8 +364,8 @@ __global__ void __launch_bounds__(THREADS, 3) shift_gemm_kernel(const GemmParams
       const int pr = (int)(pixel - n * OHW);
       const int oh = pr / P.OW, ow = pr - (pr / P.OW) * P.OW;
       rc.img_base = n * (int64_t)P.C * P.H * P.W;
-      rc.ih0 = (P.dh ? oh : oh * P.sh) - P.ph;
-      rc.iw0 = (P.dw ? ow : ow * P.sw) - P.pw;
+      rc.ih0 = oh * P.sh - P.ph;
+      rc.iw0 = ow * P.sw - P.pw;
     }
   }
 

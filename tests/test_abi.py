@@ -104,11 +104,19 @@ def test_validation_happens_before_cuda(ds):
                                         None) == ds.DS_ERR_INVALID_ARG
     assert L.ds_conv2d_shift_backward_x(16, ctypes.byref(w), 4096, 1, 1, 3, 3, 1, 3, 3, 0, 1, 1, 1, 0, None,
                                         None) == ds.DS_ERR_SHAPE
-    assert L.ds_conv2d_shift_backward_x(16, ctypes.byref(w), 4096, 1, 1, 3, 3, 1, 3, 3, 2, 2, 1, 1, 0, None,
-                                        None) == ds.DS_ERR_INVALID_ARG  # unfilled descriptor
-    assert L.ds_pack_shift_weights_backward(16, 16, 4, 4, 3, 3, 256, 10, ctypes.byref(d), None) == ds.DS_ERR_BUFFER_TOO_SMALL
-    assert L.ds_pack_shift_weights_backward(16, 16, 4, 0, 3, 3, 256, 4096, ctypes.byref(d), None) == ds.DS_ERR_SHAPE
-    assert L.ds_pack_shift_weights_backward(16, 16, 4, 4, 1, 1, 272, 4096, ctypes.byref(d), None) == ds.DS_ERR_ALIGNMENT
+    w4 = (ds.ds_weights * 4)()
+    assert L.ds_conv2d_shift_backward_x(16, w4, 4096, 1, 1, 3, 3, 1, 3, 3, 2, 2, 1, 1, 0, None,
+                                        None) == ds.DS_ERR_INVALID_ARG  # unfilled descriptors
+    d4 = (ds.ds_weights * 4)()
+    assert L.ds_pack_shift_weights_backward(16, 16, 4, 4, 3, 3, 1, 1, 256, 10, d4, None) == ds.DS_ERR_BUFFER_TOO_SMALL
+    assert L.ds_pack_shift_weights_backward(16, 16, 4, 0, 3, 3, 1, 1, 256, 4096, d4, None) == ds.DS_ERR_SHAPE
+    assert L.ds_pack_shift_weights_backward(16, 16, 4, 4, 3, 3, 0, 1, 256, 4096, d4, None) == ds.DS_ERR_SHAPE
+    assert L.ds_pack_shift_weights_backward(16, 16, 4, 4, 1, 1, 1, 1, 272, 4096, d4, None) == ds.DS_ERR_ALIGNMENT
+    # phase sizes: a 3x3 / 2 layer has phases of 2x2, 2x1, 1x2, 1x1 taps; a 1x1 / 2 layer one non-empty phase
+    ph = [ds.ds_packed_weight_bytes(5, 4 * t) for t in (4, 2, 2, 1)]
+    assert ds.ds_packed_weight_bytes_backward(4, 5, 3, 3, 2, 2) == sum((b + 255) // 256 * 256 for b in ph)
+    assert ds.ds_packed_weight_bytes_backward(4, 5, 1, 1, 2, 2) == (ds.ds_packed_weight_bytes(5, 4) + 255) // 256 * 256
+    assert ds.ds_packed_weight_bytes_backward(4, 5, 3, 3, 0, 2) == 0
     # quantizers: NULL pointers, p_min range, sizes, alignment
     assert L.ds_quantize_shift_weights(None, 4, -15, 16, 32, None) == ds.DS_ERR_INVALID_ARG
     assert L.ds_quantize_shift_weights(16, 4, -16, 16, 32, None) == ds.DS_ERR_INVALID_ARG

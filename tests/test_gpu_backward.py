@@ -14,17 +14,26 @@ def _dev(a):
     return torch.from_numpy(np.ascontiguousarray(a)).cuda()
 
 
-@pytest.mark.parametrize("dims", [(1, 1, 1, 1), (5, 3, 3, 3), (64, 33, 1, 1), (7, 40, 7, 7), (3, 70, 3, 2)])
-def test_pack_backward_blob_bitexact(dslib, dims):
+@pytest.mark.parametrize("dims,stride", [((1, 1, 1, 1), 1), ((5, 3, 3, 3), 1), ((64, 33, 1, 1), 1),
+                                         ((7, 40, 7, 7), 2), ((3, 70, 3, 2), 2), ((6, 9, 1, 1), 2),
+                                         ((4, 5, 5, 3), 3)])
+def test_pack_backward_phase_blobs_bitexact(dslib, dims, stride):
     K, C, R, S = dims
     s = si.sign_codes(sum(dims), dims)
     p = si.shift_codes_uniform(sum(dims), dims)
-    w = dslib.pack_shift_weights_backward(_dev(s), _dev(p))
-    sb, pb = O.backward_codes(s, p)
-    want = O.pack_planes6(sb.reshape(C, -1), pb.reshape(C, -1))
-    got = w.blob.cpu().numpy()
-    assert w.n_out == C and w.k_red == K * R * S
-    assert np.array_equal(got[:want.size], want)
+    w = dslib.pack_shift_weights_backward(_dev(s), _dev(p), (stride, stride))
+    blob = w.blob.cpu().numpy()
+    for (a, b), codes in O.backward_phase_codes(s, p, (stride, stride)).items():
+        d = w.desc[a * stride + b]
+        assert d.n_out == C
+        if codes is None:
+            assert d.k_red == 0 and not d.packed
+            continue
+        sp, pp = codes
+        assert d.k_red == sp[0].size
+        want = O.pack_planes6(sp.reshape(C, -1), pp.reshape(C, -1))
+        off = d.packed - w.blob.data_ptr()
+        assert np.array_equal(blob[off:off + want.size], want)
 
 
 FC_SHAPES = [(1, 1, 1), (3, 7, 5), (64, 784, 512), (33, 130, 65), (200, 64, 1000)]
@@ -40,7 +49,7 @@ def test_linear_backward_x_bitexact(dslib, M, K, N, flags, expand):
     w = dslib.pack_shift_weights_backward(_dev(s), _dev(p), expand=expand)
     dx = torch.empty((M, K), dtype=torch.int32, device="cuda")
     amax = torch.zeros(2, dtype=torch.int32, device="cuda")
-    dslib.ds_linear_shift_backward_x(_dev(dy), w.desc, dx, M, K, N, flags | dslib.DS_AMAX_OUT, amax)
+    dslib.ds_linear_shift_backward_x(_dev(dy), w.desc[0], dx, M, K, N, flags | dslib.DS_AMAX_OUT, amax)
     want = O.linear_shift_backward_x(dy, s, p)
     assert np.array_equal(dx.cpu().numpy(), want)
     assert amax.cpu().numpy().view(np.uint32)[1] == O.absmax(want)
@@ -54,7 +63,7 @@ def test_linear_backward_x_saturates(dslib):
     w = dslib.pack_shift_weights_backward(_dev(s), _dev(p))
     dx = torch.empty((M, K), dtype=torch.int32, device="cuda")
     amax = torch.zeros(2, dtype=torch.int32, device="cuda")
-    dslib.ds_linear_shift_backward_x(_dev(dy), w.desc, dx, M, K, N, 0, amax)
+    dslib.ds_linear_shift_backward_x(_dev(dy), w.desc[0], dx, M, K, N, 0, amax)
     want = O.linear_shift_backward_x(dy, s, p)
     assert (np.abs(O.linear_shift_backward_x_acc(dy, s, p)) > O.INT32_MAX).any()
     assert np.array_equal(dx.cpu().numpy(), want)
@@ -71,6 +80,8 @@ CONV_GEOMS = [
     (1, 40, 7, 7, 130, 1, 1, 1, 0),
     (1, 5, 6, 6, 3, 1, 1, 1, 1),        # pad > R - 1: the gather path even at stride 1
     (2, 4, 10, 9, 6, 5, 3, 2, 2),       # non-square kernel
+    (1, 6, 11, 10, 5, 5, 5, 3, 2),      # stride 3
+    (2, 7, 9, 9, 4, 3, 3, 2, 0),        # stride 2, no padding: the last input row / column get no gradient
 ]
 
 
@@ -83,7 +94,7 @@ def test_conv_backward_x_bitexact(dslib, geom, flags, expand):
     p = si.shift_codes_uniform(sum(geom) * 3, (K, C, R, S))
     OH, OW = O.conv_out_size(H, R, st, pd), O.conv_out_size(W, S, st, pd)
     dy = si.activations(sum(geom) + flags, (N, K, OH, OW), -(1 << 22), 1 << 22)
-    w = dslib.pack_shift_weights_backward(_dev(s), _dev(p), expand=expand)
+    w = dslib.pack_shift_weights_backward(_dev(s), _dev(p), (st, st), expand=expand)
     dx = torch.empty((N, C, H, W), dtype=torch.int32, device="cuda")
     amax = torch.zeros(2, dtype=torch.int32, device="cuda")
     dslib.ds_conv2d_shift_backward_x(_dev(dy), w.desc, dx, N, C, H, W, K, R, S, st, st, pd, pd,
@@ -102,7 +113,7 @@ def test_conv_backward_x_resnet_layers(dslib, geom):
     p = si.shift_codes_geometric(sum(geom), (K, C, R, S), -6)
     OH, OW = O.conv_out_size(H, R, st, pd), O.conv_out_size(W, S, st, pd)
     dy = si.activations(sum(geom) + 1, (N, K, OH, OW), -(1 << 20), 1 << 20)
-    w = dslib.pack_shift_weights_backward(_dev(s), _dev(p), expand=True)
+    w = dslib.pack_shift_weights_backward(_dev(s), _dev(p), (st, st), expand=True)
     dx = torch.empty((N, C, H, W), dtype=torch.int32, device="cuda")
     amax = torch.zeros(2, dtype=torch.int32, device="cuda")
     dslib.ds_conv2d_shift_backward_x(_dev(dy), w.desc, dx, N, C, H, W, K, R, S, st, st, pd, pd, 0, amax)

@@ -682,3 +682,42 @@ def test_linear_backward_x_is_forward_with_transposed_codes():
     dy = si.activations(7, (5, 13), -(1 << 30), 1 << 30)
     sb, pb = O.backward_codes(s, p)
     assert np.array_equal(O.linear_shift(dy, sb[:, :, 0, 0], pb[:, :, 0, 0]), O.linear_shift_backward_x(dy, s, p))
+
+
+@pytest.mark.parametrize("geom", BWD_GEOMS)
+def test_conv_backward_x_phase_decomposition(geom):
+    """The input gradient equals, phase by phase, a stride-1 correlation of dy with the phase's rot180
+    sub-kernel (backward_phase_codes) and padding Th - 1 - c, placed at rows sh i' + rho (the algorithm of
+    the GPU path for strided layers), restated here with Python ints."""
+    N, C, H, W, K, R, S, st, pd = geom
+    s = si.sign_codes(sum(geom) + 8, (K, C, R, S))
+    p = si.shift_codes_uniform(sum(geom) + 8, (K, C, R, S))
+    OH, OW = O.conv_out_size(H, R, st, pd), O.conv_out_size(W, S, st, pd)
+    dy = si.activations(sum(geom) + 9, (N, K, OH, OW), -(1 << 20), 1 << 20)
+    want = O.conv2d_shift_backward_x_acc(dy, s, p, (H, W), (st, st), (pd, pd))
+    phases = O.backward_phase_codes(s, p, (st, st))
+    got = np.zeros_like(want)
+    for rh in range(min(st, H)):
+        for rw in range(min(st, W)):
+            a, b = (rh + pd) % st, (rw + pd) % st
+            if phases[(a, b)] is None:
+                continue
+            sp, pp = phases[(a, b)]
+            th, tw = sp.shape[2], sp.shape[3]
+            ph, pw = th - 1 - (rh + pd - a) // st, tw - 1 - (rw + pd - b) // st
+            for i in range((H - rh + st - 1) // st):
+                for j in range((W - rw + st - 1) // st):
+                    for n in range(N):
+                        for c in range(C):
+                            acc = 0
+                            for k in range(K):
+                                for t in range(th):
+                                    for u in range(tw):
+                                        ih, iw = i - ph + t, j - pw + u
+                                        if 0 <= ih < OH and 0 <= iw < OW:
+                                            acc += int(sp[c, k, t, u]) * (int(dy[n, k, ih, iw]) >> -int(pp[c, k, t, u]))
+                            got[n, c, st * i + rh, st * j + rw] = acc
+    assert np.array_equal(got, want)
+    if st == 1:
+        sb, pb = O.backward_codes(s, p)
+        assert np.array_equal(phases[(0, 0)][0], sb) and np.array_equal(phases[(0, 0)][1], pb)
