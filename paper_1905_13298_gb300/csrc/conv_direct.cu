@@ -21,9 +21,13 @@
 //
 // Accumulator width as in shift_gemm.cu: 32-bit when the launch bound proves
 // it exact for the CTA's channels, else a 64-bit pass per half of the pixels.
+#include <cooperative_groups.h>
+
 #include <algorithm>
 
 #include "ds_common.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace ds {
 namespace {
@@ -34,6 +38,7 @@ constexpr int CG = NT / TN;             // channel groups per CTA
 constexpr int kMaxThreads = 256;        // 8 warps: every SM sub-partition gets the same share
 constexpr int kSmemBudget = 74 * 1024;  // 3 CTAs per SM
 constexpr int kSlots = 152 * 3;         // resident CTAs on a GB300
+constexpr int kMaxCluster = 16;         // CTAs per thread-block cluster (non-portable maximum)
 
 // The CTA tiles run over the stacked output rows gr = n * OH + oh of all
 // images, so a tile may span image boundaries (small feature maps, batch 1).
@@ -72,6 +77,7 @@ struct DirectGeom {
   int run;           // taps per decode item (blob path)
   int tiles_w, tiles_h;
   int splits, stages_per_split;  // split reduction over the stages
+  int cluster;                   // > 1: the splits form one thread-block cluster (reduction in DSMEM)
   FastDiv dGW, dHR, dHP;         // dividers of the halo staging
 };
 
@@ -258,7 +264,7 @@ __device__ __forceinline__ void compute_stage(const DirectGeom G, const int32_t*
   }
 }
 
-template <int SIG, int S, int TM, int I0, int NI, typename Acc>
+template <int SIG, int S, int TM, int I0, int NI, typename Acc, bool CL>
 __device__ __forceinline__ void run_direct(const GemmParams& P, const DirectGeom G, unsigned char* smem,
                                            int64_t gr0, int ow0, int64_t col0, int st_begin, int st_end,
                                            uint32_t& amax_local) {
@@ -300,7 +306,7 @@ __device__ __forceinline__ void run_direct(const GemmParams& P, const DirectGeom
   // for its own copies before the next barrier, which then makes all of
   // stage st + 1 visible.
   const int64_t taps_per_c = (int64_t)S * S;
-  {
+  if (st_begin < st_end) {  // a trailing rank of a cluster may have no stage: zero partial sums
     const int64_t kb = (int64_t)st_begin * G.CC * taps_per_c;
     stage_halo<SIG, S, TM>(P, G, halo_base, n0, off0, iw0, st_begin * G.CC);
     if (expanded) stage_codes_expanded(P, G, code_base, col0, kb);
@@ -327,6 +333,73 @@ __device__ __forceinline__ void run_direct(const GemmParams& P, const DirectGeom
     }
   }
   __syncthreads();  // the next pass (64-bit path) reuses the buffers
+
+  if constexpr (CL) {
+    // Split over a thread-block cluster: every rank has the same tile mapping,
+    // so entry (thread, pixel slot, channel) of each rank's partial sums (a
+    // subset of the terms: 32-bit partials are exact whenever the bound holds)
+    // belongs to the same output.  Rank r sums, through distributed shared
+    // memory, the slots i = r (mod cluster) of its threads and stores them.
+    Acc* red = reinterpret_cast<Acc*>(smem);
+#pragma unroll
+    for (int i = 0; i < NI; ++i)
+#pragma unroll
+      for (int j = 0; j < TN; ++j) red[(t * TM + I0 + i) * TN + j] = acc[i][j];
+    cg::cluster_group cl = cg::this_cluster();
+    cl.sync();  // all partials written
+    const int rank = (int)cl.block_rank();
+    const int64_t grc = gr0 + oh_l;
+    const bool row_ok = grc < (int64_t)G.N * P.OH;
+    const int64_t nc = row_ok ? grc / P.OH : 0;
+    const int ohc = row_ok ? (int)(grc - nc * P.OH) : 0;
+    const int64_t OHWc = (int64_t)P.OH * P.OW;
+    const bool relu_c = (P.flags & DS_RELU) != 0;
+    const bool resid_c = (P.flags & DS_RESIDUAL) != 0;
+    for (int i = I0; i < I0 + NI; ++i) {
+      const int ow = ow0 + g * TM + i;
+      if (i % G.cluster != rank || !row_ok || ow >= P.OW) continue;
+      Acc sum[TN] = {0, 0, 0, 0};
+      for (int q = 0; q < G.cluster; ++q) {
+        const Acc* src = cl.map_shared_rank(red, q) + (t * TM + i) * TN;
+        if constexpr (sizeof(Acc) == 4) {
+          const uint4 v = *reinterpret_cast<const uint4*>(src);
+          sum[0] += v.x;
+          sum[1] += v.y;
+          sum[2] += v.z;
+          sum[3] += v.w;
+        } else {
+          const longlong2 v0 = *reinterpret_cast<const longlong2*>(src);
+          const longlong2 v1 = *reinterpret_cast<const longlong2*>(src + 2);
+          sum[0] += v0.x;
+          sum[1] += v0.y;
+          sum[2] += v1.x;
+          sum[3] += v1.y;
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < TN; ++j) {
+        const int64_t col = col0 + cg * TN + j;
+        if (col >= P.cols) continue;
+        const int64_t idx = (nc * P.cols + col) * OHWc + (int64_t)ohc * P.OW + ow;
+        const int32_t bcol = P.bias ? __ldg(P.bias + col) : 0;
+        int32_t o;
+        if constexpr (sizeof(Acc) == 4) {
+          o = (int32_t)(sum[j] + (uint32_t)bcol);
+        } else {
+          int64_t a = sum[j] + (int64_t)bcol;
+          a = a > (int64_t)INT32_MAX ? (int64_t)INT32_MAX : a;
+          a = a < (int64_t)INT32_MIN ? (int64_t)INT32_MIN : a;
+          o = (int32_t)a;
+        }
+        if (resid_c) o = add_sat(o, __ldg(P.residual + idx));
+        if (relu_c) o = max(o, 0);
+        amax_local = max(amax_local, uabs(o));
+        P.y[idx] = o;
+      }
+    }
+    cl.sync();  // no rank reuses its shared memory (next pass) or exits while another reads it
+    return;
+  }
 
   const int64_t gr = gr0 + oh_l;  // this thread's output row (recomputed: not kept live in the loop)
   if (gr >= (int64_t)G.N * P.OH) return;
@@ -411,7 +484,7 @@ __device__ __forceinline__ bool tile_int32_exact(const GemmParams& P, int NT, in
   return !__syncthreads_or(unsafe);
 }
 
-template <int SIG, int S, int TM>
+template <int SIG, int S, int TM, bool CL>
 __global__ void __launch_bounds__(kMaxThreads, 3) conv_direct_kernel(const GemmParams P, const DirectGeom G) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int bx = blockIdx.x;
@@ -425,11 +498,11 @@ __global__ void __launch_bounds__(kMaxThreads, 3) conv_direct_kernel(const GemmP
 
   uint32_t amax_local = 0;
   if (tile_int32_exact(P, NT, col0)) {
-    run_direct<SIG, S, TM, 0, TM, uint32_t>(P, G, smem_raw, gr0, ow0, col0, st_begin, st_end, amax_local);
+    run_direct<SIG, S, TM, 0, TM, uint32_t, CL>(P, G, smem_raw, gr0, ow0, col0, st_begin, st_end, amax_local);
   } else {
     constexpr int H1 = TM / 2;
-    run_direct<SIG, S, TM, 0, H1, int64_t>(P, G, smem_raw, gr0, ow0, col0, st_begin, st_end, amax_local);
-    run_direct<SIG, S, TM, H1, TM - H1, int64_t>(P, G, smem_raw, gr0, ow0, col0, st_begin, st_end, amax_local);
+    run_direct<SIG, S, TM, 0, H1, int64_t, CL>(P, G, smem_raw, gr0, ow0, col0, st_begin, st_end, amax_local);
+    run_direct<SIG, S, TM, H1, TM - H1, int64_t, CL>(P, G, smem_raw, gr0, ow0, col0, st_begin, st_end, amax_local);
   }
   if (P.amax_out != nullptr && P.split_acc == nullptr) {
     amax_local = __reduce_max_sync(0xffffffffu, amax_local);
@@ -479,6 +552,10 @@ size_t direct_smem_bytes(const DirectGeom& G) {
 bool choose_geom(const GemmParams& p, size_t split_capacity, Choice& ch) {
   DirectGeom& G = ch.G;
   ch.TM = (p.OW % 7 == 0) ? 7 : 8;
+  // Cluster split for calls without a workspace (the kernels with a cluster
+  // variant); with a workspace (the chained forward) the atomic split is
+  // used: measured faster there (ResNet18 batch 1: 0.51 vs 0.63 ms per forward).
+  const bool allow_cluster = split_capacity == 0 && ch.TM == 7 && (p.S == 3 || p.S == 7);
   const int WS = (ch.TM - 1) * p.sw + p.S;
   const int WSP = (WS + 3) / 4 * 4 + (((WS + 3) / 4) % 2 == 0 ? 4 : 0);  // as Win<>::WSP
   int gw = (p.OW + ch.TM - 1) / ch.TM;
@@ -520,6 +597,19 @@ bool choose_geom(const GemmParams& p, size_t split_capacity, Choice& ch) {
       cc = d;
       break;
     }
+  const int64_t ctas = (int64_t)((p.OW + ch.TM * G.GW - 1) / (ch.TM * G.GW)) * tiles_h * ((p.cols + NT - 1) / NT);
+  // A grid that does not fill every SM slot once splits its stages over the
+  // CTAs of a cluster: then use stages small enough that every rank gets one.
+  const int target = (int)std::min<int64_t>(kMaxCluster, ctas < kSlots ? kSlots / std::max<int64_t>(ctas, 1) : 1);
+  if (allow_cluster && target >= 2 && (p.C + cc - 1) / cc < target) {
+    int want = std::max(1, p.C / target);
+    for (int d = want; d >= 1; --d)
+      if (p.C % d == 0) {
+        want = d;
+        break;
+      }
+    cc = std::min(cc, want);
+  }
   G.CC = cc;
   G.taps = G.CC * p.R * p.S;
   G.n_stages = (p.C + G.CC - 1) / G.CC;
@@ -534,40 +624,132 @@ bool choose_geom(const GemmParams& p, size_t split_capacity, Choice& ch) {
   G.dHP = make_fastdiv((uint32_t)G.HP);
   G.tiles_w = (p.OW + ch.TM * G.GW - 1) / (ch.TM * G.GW);
   G.tiles_h = (int)tiles_h;
-  // split the stages when the grid would not fill every SM slot once
+  // split the stages when the grid would not fill every SM slot once: over a
+  // thread-block cluster (launch_direct checks the size with the device),
+  // else, with a workspace, over CTAs adding int64 partials atomically
   G.splits = 1;
   G.stages_per_split = G.n_stages;
-  const int64_t ctas = (int64_t)G.tiles_w * G.tiles_h * ((p.cols + NT - 1) / NT);
-  const size_t need = (size_t)p.rows * p.cols * sizeof(int64_t);
-  if (split_capacity >= need && ctas < kSlots && G.n_stages > 1) {
-    int want = (int)std::min<int64_t>(G.n_stages, (2 * kSlots + ctas - 1) / ctas);
-    G.stages_per_split = (G.n_stages + want - 1) / want;
-    G.splits = (G.n_stages + G.stages_per_split - 1) / G.stages_per_split;
+  G.cluster = 1;
+  if (allow_cluster && target >= 2 && G.n_stages >= 2) {
+    G.cluster = std::min(target, G.n_stages);
+    G.stages_per_split = (G.n_stages + G.cluster - 1) / G.cluster;
+    G.splits = G.cluster;
+  } else {
+    const size_t need = (size_t)p.rows * p.cols * sizeof(int64_t);
+    if (split_capacity >= need && ctas < kSlots && G.n_stages > 1) {
+      int want = (int)std::min<int64_t>(G.n_stages, (2 * kSlots + ctas - 1) / ctas);
+      G.stages_per_split = (G.n_stages + want - 1) / want;
+      G.splits = (G.n_stages + G.stages_per_split - 1) / G.stages_per_split;
+    }
   }
   return direct_smem_bytes(G) <= (size_t)kSmemBudget;
 }
 
-template <int SIG, int S, int TM>
-cudaError_t launch_direct(const GemmParams& p, const DirectGeom& G, cudaStream_t st) {
-  const size_t smem = direct_smem_bytes(G);
-  // raise the dynamic shared-memory limit once per process (not a stream operation, so a
-  // forward captured in a CUDA graph after a first eager call issues no attribute call)
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(conv_direct_kernel<SIG, S, TM>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
+// Shared memory of a launch: the staging buffers, and in cluster mode at least
+// the partial sums (threads x TM x TN, 64-bit in the worst case).
+size_t launch_smem_bytes(const DirectGeom& G, int TM) {
+  size_t smem = direct_smem_bytes(G);
+  if (G.cluster > 1) smem = std::max(smem, (size_t)G.threads * TM * TN * sizeof(int64_t));
+  return smem;
+}
+
+template <int SIG, int S, int TM, bool CL>
+bool set_attributes() {
+  // once per process (not a stream operation, so a forward captured in a CUDA
+  // graph after a first eager call issues no attribute call)
+  static int state = 0;  // 0 unset, 1 ok, -1 failed
+  if (state == 0) {
+    const bool ok = cudaFuncSetAttribute(conv_direct_kernel<SIG, S, TM, CL>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget) == cudaSuccess &&
+                    (!CL || cudaFuncSetAttribute(conv_direct_kernel<SIG, S, TM, CL>,
+                                                 cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess);
+    if (!ok) (void)cudaGetLastError();
+    state = ok ? 1 : -1;
   }
+  return state == 1;
+}
+
+// Whether the device can co-schedule a cluster of cs CTAs of this kernel
+// (cached per process and size).
+template <int SIG, int S, int TM>
+bool cluster_ok(int cs, size_t smem) {
+  if (!set_attributes<SIG, S, TM, true>()) return false;
+  static int cache[kMaxCluster + 1] = {0};
+  if (cs < 2 || cs > kMaxCluster) return false;
+  if (cache[cs] == 0) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(1, 1, cs);
+    cfg.blockDim = dim3(kMaxThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeClusterDimension;
+    attr.val.clusterDim.x = 1;
+    attr.val.clusterDim.y = 1;
+    attr.val.clusterDim.z = cs;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, conv_direct_kernel<SIG, S, TM, true>, &cfg) != cudaSuccess) {
+      (void)cudaGetLastError();
+      n = 0;
+    }
+    cache[cs] = n > 0 ? 1 : -1;
+  }
+  return cache[cs] > 0;
+}
+
+// Cluster-split variants exist for the network shapes (TM = 7; 3x3 and 7x7 kernels).
+constexpr bool has_cluster_variant(int S, int TM) { return TM == 7 && (S == 3 || S == 7); }
+
+template <int SIG, int S, int TM>
+cudaError_t launch_direct(const GemmParams& p, const DirectGeom& G0, cudaStream_t st) {
+  if (!set_attributes<SIG, S, TM, false>()) return cudaErrorInvalidValue;
+  DirectGeom G = G0;
+  if (G.cluster > 1) {
+    // the largest cluster size the device accepts; without one, no split
+    int cs = 1;
+    if constexpr (has_cluster_variant(S, TM)) {
+      cs = G.cluster;
+      while (cs >= 2 && !cluster_ok<SIG, S, TM>(cs, launch_smem_bytes(G, TM))) --cs;
+    }
+    if (cs >= 2) {
+      G.cluster = cs;
+      G.stages_per_split = (G.n_stages + cs - 1) / cs;
+      G.splits = cs;
+    } else {
+      G.cluster = 1;
+      G.splits = 1;
+      G.stages_per_split = G.n_stages;
+    }
+  }
+  const size_t smem = launch_smem_bytes(G, TM);
   GemmParams q = p;
+  const dim3 grid((unsigned)((int64_t)G.tiles_w * G.tiles_h), (unsigned)((p.cols + NT - 1) / NT), (unsigned)G.splits);
+  if (G.cluster > 1) {
+    q.split_acc = nullptr;
+    if constexpr (has_cluster_variant(S, TM)) {
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = grid;
+      cfg.blockDim = dim3(G.threads, 1, 1);
+      cfg.dynamicSmemBytes = smem;
+      cfg.stream = st;
+      cudaLaunchAttribute attr;
+      attr.id = cudaLaunchAttributeClusterDimension;
+      attr.val.clusterDim.x = 1;
+      attr.val.clusterDim.y = 1;
+      attr.val.clusterDim.z = (unsigned)G.cluster;
+      cfg.attrs = &attr;
+      cfg.numAttrs = 1;
+      return cudaLaunchKernelEx(&cfg, conv_direct_kernel<SIG, S, TM, true>, q, G);
+    }
+  }
   if (G.splits > 1) {
     cudaError_t e = cudaMemsetAsync(q.split_acc, 0, (size_t)p.rows * p.cols * sizeof(int64_t), st);
     if (e != cudaSuccess) return e;
   } else {
     q.split_acc = nullptr;
   }
-  dim3 grid((unsigned)((int64_t)G.tiles_w * G.tiles_h), (unsigned)((p.cols + NT - 1) / NT), (unsigned)G.splits);
-  conv_direct_kernel<SIG, S, TM><<<grid, G.threads, smem, st>>>(q, G);
+  conv_direct_kernel<SIG, S, TM, false><<<grid, G.threads, smem, st>>>(q, G);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || G.splits == 1) return e;
   return launch_split_finalize(q, st);
@@ -601,7 +783,7 @@ cudaError_t launch_split_finalize(const GemmParams& p, cudaStream_t st) {
 size_t conv_direct_split_bytes(const GemmParams& p) {
   if (!conv_direct_supported(p)) return 0;
   Choice ch;
-  if (!choose_geom(p, ~(size_t)0, ch) || ch.G.splits <= 1) return 0;
+  if (!choose_geom(p, ~(size_t)0, ch) || ch.G.splits <= 1 || ch.G.cluster > 1) return 0;  // clusters need none
   return (size_t)p.rows * p.cols * sizeof(int64_t);
 }
 
