@@ -520,6 +520,7 @@ __global__ void conv_split_finalize_kernel(const GemmParams P, int64_t total) {
        e += (int64_t)gridDim.x * blockDim.x) {
     const int64_t col = (e / OHW) % P.cols;
     int64_t a = P.split_acc[e] + (P.bias ? (int64_t)__ldg(P.bias + col) : 0);
+    if (e < (int64_t)(kSmallScratchBytes / sizeof(int64_t))) P.split_acc[e] = 0;  // the zero prefix
     a = a > (int64_t)INT32_MAX ? (int64_t)INT32_MAX : a;
     a = a < (int64_t)INT32_MIN ? (int64_t)INT32_MIN : a;
     int32_t o = (int32_t)a;
@@ -743,11 +744,11 @@ cudaError_t launch_direct(const GemmParams& p, const DirectGeom& G0, cudaStream_
       return cudaLaunchKernelEx(&cfg, conv_direct_kernel<SIG, S, TM, true>, q, G);
     }
   }
-  if (G.splits > 1) {
-    cudaError_t e = cudaMemsetAsync(q.split_acc, 0, (size_t)p.rows * p.cols * sizeof(int64_t), st);
-    if (e != cudaSuccess) return e;
-  } else {
+  if (G.splits == 1) {
     q.split_acc = nullptr;
+  } else {
+    cudaError_t e = prepare_split_scratch(q, st);
+    if (e != cudaSuccess) return e;
   }
   conv_direct_kernel<SIG, S, TM, false><<<grid, G.threads, smem, st>>>(q, G);
   cudaError_t e = cudaGetLastError();
@@ -770,6 +771,17 @@ bool conv_direct_supported(const GemmParams& p) {
   if ((p.rows / ((int64_t)p.OH * p.OW)) >= ((int64_t)1 << 24)) return false;
   Choice ch;
   return choose_geom(p, p.split_acc ? p.split_capacity : 0, ch);
+}
+
+cudaError_t prepare_split_scratch(const GemmParams& p, cudaStream_t st) {
+  // The first kSmallScratchBytes of the scratch are zero between layers (the
+  // chained forward resets them once, every finalize re-zeroes them), so a
+  // small region (batch 1) needs no memset launch.  A larger region is zeroed
+  // here: a memset is cheaper than re-zeroing it in the finalize (measured:
+  // ResNet18 batch 32 5.33 vs 5.50 ms per forward, batch 1 0.49 vs 0.50 ms).
+  const size_t bytes = (size_t)p.rows * p.cols * sizeof(int64_t);
+  if (bytes <= kSmallScratchBytes) return cudaSuccess;
+  return cudaMemsetAsync(p.split_acc, 0, bytes, st);
 }
 
 cudaError_t launch_split_finalize(const GemmParams& p, cudaStream_t st) {

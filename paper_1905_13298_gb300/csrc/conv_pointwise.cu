@@ -394,11 +394,11 @@ cudaError_t launch_pw(const GemmParams& p, cudaStream_t st) {
   const int sps = pw_stages_per_split(p, p.split_acc ? p.split_capacity : 0);
   const int splits = (n_stages + sps - 1) / sps;
   GemmParams q = p;
-  if (splits > 1) {
-    cudaError_t e = cudaMemsetAsync(q.split_acc, 0, (size_t)p.rows * p.cols * sizeof(int64_t), st);
-    if (e != cudaSuccess) return e;
-  } else {
+  if (splits == 1) {
     q.split_acc = nullptr;
+  } else {
+    cudaError_t e = prepare_split_scratch(q, st);
+    if (e != cudaSuccess) return e;
   }
   dim3 grid((unsigned)((p.rows + MT - 1) / MT), (unsigned)((p.cols + NT - 1) / NT), (unsigned)splits);
   conv_pointwise_kernel<STRIDED><<<grid, THREADS, smem, st>>>(q, sps);

@@ -77,7 +77,8 @@ struct GemmParams {
   // strided layer's input gradient)
   int ys_h, ys_w, yph, ypw, yH, yW;
   uint32_t flags;
-  // split reduction (conv, chained forward only): int64 partial sums of every output, zeroed first
+  // split reduction (conv, chained forward only): int64 partial sums of every
+  // output; its first kSmallScratchBytes are zero on entry and on exit
   int64_t* split_acc;       // nullable
   size_t split_capacity;    // bytes available at split_acc
 };
@@ -92,8 +93,12 @@ cudaError_t launch_conv2d_shift(const GemmParams& p, cudaStream_t st);
 bool conv_direct_supported(const GemmParams& p);
 size_t conv_direct_split_bytes(const GemmParams& p);  // int64 scratch a split reduction would use (0: no split)
 cudaError_t launch_conv2d_direct(const GemmParams& p, cudaStream_t st);
-// Epilogue of a split reduction: y = ReLU?(sat32(sat32(split_acc + bias) + residual)), max|y|.
+// Epilogue of a split reduction: y = ReLU?(sat32(sat32(split_acc + bias) + residual)), max|y|;
+// re-zeroes the first kSmallScratchBytes of the scratch.
 cudaError_t launch_split_finalize(const GemmParams& p, cudaStream_t st);
+// Before a split launch: zeroes a scratch region larger than kSmallScratchBytes (smaller ones are zero).
+constexpr size_t kSmallScratchBytes = 2u << 20;
+cudaError_t prepare_split_scratch(const GemmParams& p, cudaStream_t st);
 // Defined in conv_pointwise.cu (1x1 convolutions as a GEMM over pixels).
 bool conv_pointwise_supported(const GemmParams& p);
 size_t conv_pointwise_split_bytes(const GemmParams& p);

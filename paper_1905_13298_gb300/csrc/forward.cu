@@ -157,7 +157,10 @@ ds_status ds_shift_forward(const ds_layer* L, int n, const int32_t* x, int32_t* 
   slot_ptr[1] = y;
   for (int s = 2; s < P.n_slots; ++s) slot_ptr[s] = reinterpret_cast<int32_t*>(base + P.slot_off[s]);
 
-  r = cuda_check(cudaMemsetAsync(amax, 0, (size_t)(n + 1) * sizeof(uint32_t), st), "amax reset");
+  // one reset per forward: the max|x| words and the split-reduction scratch (its
+  // zero prefix is kept zero by the finalize kernels, larger regions are zeroed
+  // before their layer)
+  r = cuda_check(cudaMemsetAsync(amax, 0, P.amax_bytes + P.split_bytes, st), "workspace reset");
   if (r != DS_OK) return r;
   const Shape in0{L[0].C, L[0].H, L[0].W};
   r = cuda_check(launch_absmax(x, in0.elems() * batch, amax + n, st), "input max|x| pre-pass");

@@ -119,3 +119,29 @@ def test_pointwise_split_reduction(dslib, batch, hw, stress):
     if stress:
         assert (np.abs(want) == 2 ** 31 - 1).any()
     assert np.array_equal(_run(prog, params, x), want)
+
+
+def test_split_scratch_large_then_small_layers(dslib):
+    """A split layer whose int64 scratch exceeds the 2 MB zero prefix (zeroed before its launch) followed by
+    split layers that rely on the prefix being left zero (3x3 64 -> 128 on 28x28 at batch 4, then a 3x3/2 and
+    a 1x1 on 14x14), twice in a row."""
+    from paper_1905_13298_gb300 import networks as PN
+    from oracle import deepshift_oracle as O
+    b = PN._Builder(64, 28, 28)
+    a1 = b.conv(0, 128, 3, 1, 1, relu=True)
+    a2 = b.conv(a1, 128, 3, 2, 1, relu=True)
+    b.conv(a2, 256, 1, 1, 0, relu=True, out=1)
+    prog = (b.specs, b.shapes)
+    params = si.network_params(prog[1], 820)
+    x = si.activations(821, (4, 64, 28, 28), 0, 1 << 20)
+    (s1, p1, b1), (s2, p2, b2), (s3, p3, b3) = params
+    h = O.conv2d_shift(x, s1, p1, b1, (1, 1), (1, 1), relu=True)
+    h = O.conv2d_shift(h, s2, p2, b2, (2, 2), (1, 1), relu=True)
+    want = O.conv2d_shift(h, s3, p3, b3, (1, 1), (0, 0), relu=True).reshape(4, -1)
+    from paper_1905_13298_gb300.networks import ShiftNetwork
+    net = ShiftNetwork(prog[0], params, batch=4, expand=True)
+    xd = torch.from_numpy(x).cuda()
+    for _ in range(2):
+        y = net.forward(xd)
+        torch.cuda.synchronize()
+        assert np.array_equal(y.cpu().numpy().reshape(4, -1), want)
