@@ -30,9 +30,9 @@ L2_BYTES = 129 * 1024 * 1024
 SMS = 152
 INT_OPS_PER_CLK_PER_SM = 128  # 4 SMSPs x 32 lanes: 16-lane ALU pipe + 16-lane FMA pipe (IMAD)
 ALG_INT_OPS_PER_TERM = 2      # one shift + one add/subtract per term (Fig. 1a: MAC -> shift + add)
-# DRAM bytes (read + write) of one conv_direct_kernel<1,3,7> launch on this workload, from one ncu capture
+# DRAM bytes (read + write) of one conv_direct_kernel<1,3,7,0> launch on this workload, from one ncu capture
 # of the current kernel (dram__bytes_read.sum + dram__bytes_write.sum); y stays in L2 at kernel end.
-NCU_TRAFFIC_BYTES = 26.14e6
+NCU_TRAFFIC_BYTES = 26.13e6
 
 
 def workload_conv2x(batch: int):
@@ -604,7 +604,7 @@ def run_gpu(args, wl, rank, world, local_rank):
                        "step": "absmax pre-pass + ConvShift (fused bias/saturate epilogue)"},
             "roofline": {"bound": "alu", "achieved": achieved, "peak": alu_peak, "unit": "Tintop/s",
                          "frac": achieved / alu_peak, "traffic": NCU_TRAFFIC_BYTES,
-                         "kernel": "conv_direct_kernel<1,3,7>", "kernel_ms": kern_ms,
+                         "kernel": "conv_direct_kernel<1,3,7,0>", "kernel_ms": kern_ms,
                          "peak_basis": f"{SMS} SMs x {INT_OPS_PER_CLK_PER_SM} int32 ops/clk x {sm_max:.0f} MHz "
                                        f"(sm_max_mhz, {peak_kind})",
                          "alg_int_ops_per_launch": ALG_INT_OPS_PER_TERM * wl["terms"],
