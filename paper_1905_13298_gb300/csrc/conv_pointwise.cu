@@ -176,11 +176,12 @@ __device__ __forceinline__ void compute_stage(const int32_t* xs, const int32_t* 
       sh[4 * v] = s0.x; sh[4 * v + 1] = s0.y; sh[4 * v + 2] = s0.z; sh[4 * v + 3] = s0.w;
       sg[4 * v] = g0.x; sg[4 * v + 1] = g0.y; sg[4 * v + 2] = g0.z; sg[4 * v + 3] = g0.w;
     }
+    // channel-outer order: consecutive SHF / IMAD share their shift / sign operand
 #pragma unroll
-    for (int i = 0; i < NI; ++i) {
-      const int xv = x[I0 + i];
+    for (int j = 0; j < TN; ++j) {
 #pragma unroll
-      for (int j = 0; j < TN; ++j) {
+      for (int i = 0; i < NI; ++i) {
+        const int xv = x[I0 + i];
         const int t = xv >> sh[j];  // Eq. 1
         if constexpr (sizeof(Acc) == 4) {
           acc[i][j] += (uint32_t)sg[j] * (uint32_t)t;  // Eq. 2 + accumulate (mod 2^32)

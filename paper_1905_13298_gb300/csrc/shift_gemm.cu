@@ -196,11 +196,12 @@ __device__ __forceinline__ void compute_chunk(const Smem& sm, int buf, int tm, i
       const int4 g1 = *reinterpret_cast<const int4*>(sgs + k * NT + 4);
       const int sh[TN] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
       const int sg[TN] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+      // column-outer order: consecutive SHF / IMAD share their shift / sign operand
 #pragma unroll
-      for (int i = 0; i < ROWS; ++i) {
-        const int xk = kk == 0 ? xv[i].x : kk == 1 ? xv[i].y : kk == 2 ? xv[i].z : xv[i].w;
+      for (int j = 0; j < TN; ++j) {
 #pragma unroll
-        for (int j = 0; j < TN; ++j) {
+        for (int i = 0; i < ROWS; ++i) {
+          const int xk = kk == 0 ? xv[i].x : kk == 1 ? xv[i].y : kk == 2 ? xv[i].z : xv[i].w;
           const int t = xk >> sh[j];  // Eq. 1: arithmetic right shift by -p
           if constexpr (sizeof(Acc) == 4) {
             acc[i][j] += (uint32_t)sg[j] * (uint32_t)t;  // Eq. 2 flip + accumulate (mod 2^32)

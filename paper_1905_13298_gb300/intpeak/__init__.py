@@ -1,9 +1,11 @@
 """Integer issue-rate microbenchmark: the measured side of the shift kernels' ALU roofline.
 
 `measure()` builds libds_intpeak.so (nvcc, sm_103a) next to this file, runs
-each instruction mix on one full wave of CTAs, and returns thread
-instructions per SM clock for each mix (from clock64 cycles, so independent
-of the clock frequency) and the wall-clock rate.
+each instruction mix on a grid of 2 CTAs per SM, and returns thread
+instructions per SM clock for each mix and the wall-clock rate.  The per-SM
+rate divides the instructions of an SM's CTAs by that SM's span of clock64
+(first start to last end), so it stays right when a mix's register count
+lets only one CTA per SM be resident at a time.
 """
 from __future__ import annotations
 
@@ -34,19 +36,25 @@ def measure(iters: int = 4096, threads: int = 256, blocks_per_sm: int = 2):
     blocks = sms * blocks_per_sm
     seed = torch.randint(1, 1 << 20, (80,), dtype=torch.int32, device="cuda")
     out = torch.empty(blocks * threads, dtype=torch.int32, device="cuda")
-    cyc = torch.empty(blocks, dtype=torch.int64, device="cuda")
+    cyc = torch.empty(2 * blocks, dtype=torch.int64, device="cuda")
+    smid = torch.empty(blocks, dtype=torch.int32, device="cuda")
     res = {}
     for kind, name in KINDS.items():
         ms = ctypes.c_float()
         for _ in range(2):  # first run warms up
             rc = L.ds_probe_int_mix(kind, blocks, threads, iters, ctypes.c_void_p(seed.data_ptr()),
                                     ctypes.c_void_p(out.data_ptr()), ctypes.c_void_p(cyc.data_ptr()),
-                                    ctypes.byref(ms))
+                                    ctypes.c_void_p(smid.data_ptr()), ctypes.byref(ms))
             if rc != 0:
                 raise RuntimeError(f"probe kind {kind} failed with CUDA error {rc}")
-        cycles = float(cyc.double().max())
-        instr_per_sm = blocks_per_sm * threads * iters * INSTR_PER_ITER[kind]
-        res[name] = {"thread_instr_per_clk_per_sm": instr_per_sm / cycles,
+        c = cyc.view(blocks, 2).cpu().numpy()
+        sm = smid.cpu().numpy()
+        rates = []
+        for s in set(sm.tolist()):
+            sel = sm == s
+            span = float(c[sel, 1].max() - c[sel, 0].min())
+            rates.append(int(sel.sum()) * threads * iters * INSTR_PER_ITER[kind] / span)
+        res[name] = {"thread_instr_per_clk_per_sm": sum(rates) / len(rates),
                      "wall_tinstr_per_s": blocks * threads * iters * INSTR_PER_ITER[kind] / (ms.value / 1e3) / 1e12,
                      "ms": ms.value}
     return res

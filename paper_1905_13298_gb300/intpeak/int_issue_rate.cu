@@ -2,9 +2,11 @@
 // shift kernels (built as its own small library, not part of the C ABI).
 //
 // Each kernel runs a register-resident loop of one instruction mix with
-// enough independent chains to hide latency, one full wave of CTAs, and
-// reports per-CTA SM cycles from clock64().  ops/clk/SM = thread instructions
-// of the mix executed by the CTAs of one SM / cycles.
+// enough independent chains to hide latency over a grid of CTAs, and records
+// per CTA its SM and its first and last clock64() (one counter per SM).
+// ops/clk/SM = thread instructions of the mix executed by the CTAs of one SM
+// / (last end - first start on that SM), so a mix whose registers allow fewer
+// resident CTAs (which then run one after the other) is not over-counted.
 //   kind 0: SHF only        (shr.s32, ALU pipe)
 //   kind 1: IMAD only       (mad.lo.s32, FMA pipe)
 //   kind 2: SHF + IMAD      (the shift-GEMM inner loop: t = x >> s; acc += g * t)
@@ -19,7 +21,7 @@ namespace {
 
 template <int KIND>
 __global__ void __launch_bounds__(256) mix_kernel(const int* __restrict__ seed, int iters, int* out,
-                                                  long long* cycles) {
+                                                  long long* cycles, int* smid) {
   int x[8], s[8], g[8], acc[8][8];
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
@@ -65,27 +67,34 @@ __global__ void __launch_bounds__(256) mix_kernel(const int* __restrict__ seed, 
 #pragma unroll
     for (int j = 0; j < 8; ++j) r ^= acc[i][j];
   out[blockIdx.x * blockDim.x + threadIdx.x] = r;
-  if (threadIdx.x == 0) cycles[blockIdx.x] = t1 - t0;
+  if (threadIdx.x == 0) {
+    unsigned sm;
+    asm volatile("mov.u32 %0, %%smid;" : "=r"(sm));
+    cycles[2 * blockIdx.x] = t0;
+    cycles[2 * blockIdx.x + 1] = t1;
+    smid[blockIdx.x] = (int)sm;
+  }
 }
 
 }  // namespace
 
-// Runs one mix; writes the mean CTA cycle count and the kernel time (ms).
-// out must hold blocks*threads ints, cycles `blocks` long longs, seed 80 ints.
+// Runs one mix; writes per CTA its (start, end) clock64 pair and SM id, and
+// the kernel time (ms).  out must hold blocks*threads ints, cycles 2*blocks
+// long longs, smid `blocks` ints, seed 80 ints.
 extern "C" int ds_probe_int_mix(int kind, int blocks, int threads, int iters, const int* seed, int* out,
-                                long long* cycles, float* ms) {
+                                long long* cycles, int* smid, float* ms) {
   cudaEvent_t a, b;
   cudaEventCreate(&a);
   cudaEventCreate(&b);
   cudaEventRecord(a);
   switch (kind) {
-    case 0: mix_kernel<0><<<blocks, threads>>>(seed, iters, out, cycles); break;
-    case 1: mix_kernel<1><<<blocks, threads>>>(seed, iters, out, cycles); break;
-    case 2: mix_kernel<2><<<blocks, threads>>>(seed, iters, out, cycles); break;
-    case 3: mix_kernel<3><<<blocks, threads>>>(seed, iters, out, cycles); break;
-    case 5: mix_kernel<5><<<blocks, threads>>>(seed, iters, out, cycles); break;
-    case 6: mix_kernel<6><<<blocks, threads>>>(seed, iters, out, cycles); break;
-    default: mix_kernel<4><<<blocks, threads>>>(seed, iters, out, cycles); break;
+    case 0: mix_kernel<0><<<blocks, threads>>>(seed, iters, out, cycles, smid); break;
+    case 1: mix_kernel<1><<<blocks, threads>>>(seed, iters, out, cycles, smid); break;
+    case 2: mix_kernel<2><<<blocks, threads>>>(seed, iters, out, cycles, smid); break;
+    case 3: mix_kernel<3><<<blocks, threads>>>(seed, iters, out, cycles, smid); break;
+    case 5: mix_kernel<5><<<blocks, threads>>>(seed, iters, out, cycles, smid); break;
+    case 6: mix_kernel<6><<<blocks, threads>>>(seed, iters, out, cycles, smid); break;
+    default: mix_kernel<4><<<blocks, threads>>>(seed, iters, out, cycles, smid); break;
   }
   cudaEventRecord(b);
   cudaError_t e = cudaEventSynchronize(b);
