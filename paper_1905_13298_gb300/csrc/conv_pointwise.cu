@@ -11,7 +11,9 @@
 // contiguous) and 8 channels; per term the hot loop is one SHF and one IMAD.
 // 128 threads at 128 registers and 32 KB of shared memory: 4 CTAs per SM.
 // Codes come from the expanded execution layout (cp.async) or are decoded
-// from the packed blob per stage.  The epilogue writes each (quad, channel)
+// from the packed blob per stage (ExpandedCodeStager: each thread's code
+// pieces and source address are fixed, advancing by 16 channels per stage).
+// The epilogue writes each (quad, channel)
 // as one 16-byte store when OH*OW is a multiple of 4.  Accumulator width as
 // in shift_gemm.cu.
 //
@@ -97,35 +99,23 @@ __device__ __forceinline__ void stage_x(const GemmParams& P, int32_t* xs, const 
   const int64_t HW = (int64_t)P.H * P.W;
   const int qi = threadIdx.x % QUADS;
   constexpr int ROWS = THREADS / QUADS;  // channel rows per pass
+  const int cl0 = (int)(threadIdx.x / QUADS);
+  const int32_t* xc = P.x + (int64_t)(c0 + cl0) * HW;  // this thread's first channel of the stage
 #pragma unroll
   for (int j = 0; j < KC / ROWS; ++j) {
-    const int cl = (int)(threadIdx.x / QUADS) + ROWS * j;
-    const int c = c0 + cl;
+    const int cl = cl0 + ROWS * j;
+    const int32_t* xj = xc + (int64_t)(ROWS * j) * HW;
     int32_t* dst = xs + cl * MT + 4 * qi;
-    const bool cok = c < P.C;
+    const bool cok = c0 + cl < P.C;
     if (!STRIDED && q.vec) {
-      cp_async16(dst, cok ? (const void*)(P.x + q.off[0] + c * HW) : (const void*)P.x, cok);
+      cp_async16(dst, cok ? (const void*)(xj + q.off[0]) : (const void*)P.x, cok);
     } else {
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
         const bool ok = cok && q.valid[i];
-        cp_async4(dst + i, ok ? (const void*)(P.x + q.off[i] + c * HW) : (const void*)P.x, ok);
+        cp_async4(dst + i, ok ? (const void*)(xj + q.off[i]) : (const void*)P.x, ok);
       }
     }
-  }
-}
-
-// Codes of input channels [c0, c0 + KC) for columns [col0, col0 + 64).
-__device__ __forceinline__ void stage_codes_expanded(const GemmParams& P, int32_t* cs, int64_t col0, int c0) {
-  const int64_t nblocks = (P.cols + 31) / 32;
-  for (int e = threadIdx.x; e < NB * KC * 16; e += THREADS) {  // NB blocks x KC channels x 16 pieces
-    const int b = e / (KC * 16);
-    const int r = e - b * KC * 16;
-    const int cl = r >> 4, q = r & 15;
-    const int64_t cb = col0 / 32 + b;
-    const bool ok = cb < nblocks && c0 + cl < P.kred;
-    const int32_t* src = ok ? P.xcodes + ((cb * P.kred + c0 + cl) * 64 + q * 4) : P.xcodes;
-    cp_async16(cs + (cl * NB + b) * 64 + q * 4, src, ok);
   }
 }
 
@@ -205,8 +195,10 @@ __device__ __forceinline__ void run_tile(const GemmParams& P, PwSmem& sm, int64_
 #pragma unroll
     for (int j = 0; j < TN; ++j) acc[i][j] = 0;
 
+  static_assert(KC == 16 && NB == 2 && THREADS == 128, "ExpandedCodeStager's stage shape");
+  const ExpandedCodeStager cst(P.xcodes, P.cols, P.kred, col0, (int64_t)st_begin * KC);
   stage_x<STRIDED>(P, sm.xs[0], q, st_begin * KC);
-  if (expanded) stage_codes_expanded(P, sm.cs[0], col0, st_begin * KC);
+  if (expanded) cst.stage(P.xcodes, P.kred, sm.cs[0], 0);
   cp_async_commit();
   if (!expanded) decode_codes(P, sm.cs[0], col0, st_begin);
   cp_async_wait_all();
@@ -216,7 +208,7 @@ __device__ __forceinline__ void run_tile(const GemmParams& P, PwSmem& sm, int64_
     __syncthreads();
     if (more) {
       stage_x<STRIDED>(P, sm.xs[b ^ 1], q, (st + 1) * KC);
-      if (expanded) stage_codes_expanded(P, sm.cs[b ^ 1], col0, (st + 1) * KC);
+      if (expanded) cst.stage(P.xcodes, P.kred, sm.cs[b ^ 1], st + 1 - st_begin);
       cp_async_commit();
     }
     compute_stage<I0, NI, Acc>(sm.xs[b], sm.cs[b], tm, tn, acc);

@@ -142,4 +142,41 @@ __host__ __device__ inline int64_t expanded_words(int64_t n_out, int64_t k_red) 
   return ((n_out + 31) / 32) * k_red * 64;
 }
 
+#ifdef __CUDACC__
+// Staging of the expanded codes of 64 columns (two 32-column blocks) and 16
+// reduction indices per stage, by 128 threads: the stage is 512 16-byte
+// pieces, and thread t copies the pieces at index kl = t / 16 and kl + 8 of
+// both blocks, bytes 16 (t % 16) of the 64-word row, into
+// cs[kl][block][64].  The pieces are the same at every stage, so the source
+// address is computed once and advances by 16 indices per stage.
+struct ExpandedCodeStager {
+  const int32_t* src;  // (block 0, kl) at stage 0
+  int64_t kp;          // kl's reduction index at stage 0
+  bool b1;             // block 1 exists
+  __device__ __forceinline__ ExpandedCodeStager(const int32_t* xcodes, int64_t cols, int64_t kred, int64_t col0,
+                                                int64_t kbeg) {
+    const int t = threadIdx.x;
+    const int64_t cb = col0 / 32;
+    b1 = cb + 1 < (cols + 31) / 32;
+    kp = kbeg + (t >> 4);
+    src = xcodes != nullptr ? xcodes + (cb * kred + kp) * 64 + (t & 15) * 4 : xcodes;
+  }
+  // stage st (indices kbeg + 16 st ..) into cs; zero fill past kred and for an absent block
+  __device__ __forceinline__ void stage(const int32_t* xcodes, int64_t kred, int32_t* cs, int st) const {
+    const int t = threadIdx.x;
+    const int64_t k = kp + (int64_t)st * 16;
+    const int32_t* s = src + (int64_t)st * 16 * 64;
+    const uint32_t d = (uint32_t)__cvta_generic_to_shared(cs + (t >> 4) * 128 + (t & 15) * 4);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int kl8 = (u & 1) * 8, b = u >> 1;
+      const bool ok = k + kl8 < kred && (b == 0 || b1);
+      const int32_t* g = ok ? s + kl8 * 64 + b * kred * 64 : xcodes;
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d + (uint32_t)(kl8 * 128 + b * 64) * 4),
+                   "l"(g), "r"(ok ? 16 : 0));
+    }
+  }
+};
+#endif
+
 }  // namespace ds

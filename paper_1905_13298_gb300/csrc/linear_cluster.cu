@@ -20,8 +20,13 @@
 // distinct banks.  Per stage of 16 k the CTA stages x transposed ([k][row], so
 // a thread's rows at one k are one or two 16-byte loads) and the stage's
 // codes (expanded layout: 16-byte cp.async; else decoded from the packed
-// blob).  Per term the hot loop is one SHF and one IMAD, as in shift_gemm.cu;
-// at most 102 registers, 5 CTAs per SM.
+// blob; the expanded copy is ExpandedCodeStager).  x arrives in 16-byte pieces of 4 k of one row (4-byte copies when K
+// is not a multiple of 4, as rows are then not 16-byte aligned) in a row-major
+// scratch tile; once a thread's own copies have landed it writes its pieces
+// transposed, so no barrier is added.  Every thread copies the same pieces at
+// every stage: its source pointers only advance by 16 k.  Per term the hot
+// loop is one SHF and one IMAD, as in shift_gemm.cu; at most 96 registers,
+// 5 CTAs per SM.
 // Accumulator width as in shift_gemm.cu: the bound proven for the whole sum
 // also covers every partial sum (a subset of its terms), so 32-bit partials
 // are exact whenever the 32-bit path is taken, and their wrap-around sum is
@@ -54,6 +59,7 @@ struct ClSmem {
     struct {
       int32_t xs[2][KC * XR];
       int32_t cs[2][KC * CW];
+      int32_t xt[MR * KC];  // x of the stage in flight, row-major [row][16 k]
     } st;
     int64_t red[MR * NT];  // the partial sums (int64 or int32) after the reduction loop
   };
@@ -72,33 +78,63 @@ __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wai
 __device__ __forceinline__ uint32_t uabs(int32_t v) { return v < 0 ? (uint32_t)0 - (uint32_t)v : (uint32_t)v; }
 
 // x rows [row0, row0 + MR), reduction indices [k0, k0 + 16) clipped to kend
-// (the end of this CTA's slice), transposed into xs[k][row]; zero elsewhere.
-// Consecutive threads read consecutive k of one row (64-byte segments).
-template <int TMR>
-__device__ __forceinline__ void stage_x(const GemmParams& P, int32_t* xs, int64_t row0, int64_t k0, int64_t kend) {
-  constexpr int MR = 8 * TMR, XR = ClSmem<TMR>::XR;
-  for (int e = threadIdx.x; e < MR * KC; e += THREADS) {
-    const int r = e / KC, kk = e % KC;
-    const int64_t row = row0 + r, k = k0 + kk;
-    const bool ok = row < P.rows && k < kend;
-    cp_async4(xs + kk * XR + r, ok ? (const void*)(P.x + row * P.kred + k) : (const void*)P.x, ok);
+// (the end of this CTA's slice); zero elsewhere.  Piece e of a stage (e =
+// threadIdx.x + THREADS u) is 4 consecutive k of one row: row e / 4, k0 +
+// 4 (e % 4); consecutive threads read consecutive pieces of a row.  copy()
+// puts it at xt[4 e] (XV: one 16-byte copy whose source size zero-fills a
+// ragged end; else four 4-byte copies), transpose() moves the thread's own
+// landed pieces to xs[k][row].  src[u]: the piece's address at stage 0.
+template <int TMR, bool XV>
+struct XStager {
+  static constexpr int MR = 8 * TMR;
+  static constexpr int NP = MR * KC / 4;                       // pieces per stage
+  static constexpr int PIECES = (NP + THREADS - 1) / THREADS;  // per thread: 1, 1, 2
+  const int32_t* src[PIECES];
+  int64_t kp[PIECES];  // the piece's first k at stage 0, or the slice end if its row is absent
+  __device__ __forceinline__ XStager(const GemmParams& P, int64_t row0, int64_t kbeg, int64_t kend) {
+#pragma unroll
+    for (int u = 0; u < PIECES; ++u) {
+      const int e = threadIdx.x + THREADS * u;
+      const int64_t row = row0 + e / 4;
+      const bool ok = e < NP && row < P.rows;
+      kp[u] = ok ? kbeg + 4 * (e % 4) : kend;
+      src[u] = ok ? P.x + row * P.kred + kbeg + 4 * (e % 4) : P.x;
+    }
   }
-}
+  __device__ __forceinline__ void copy(const GemmParams& P, int32_t* xt, int64_t kend, int st) const {
+#pragma unroll
+    for (int u = 0; u < PIECES; ++u) {
+      const int e = threadIdx.x + THREADS * u;
+      if (e >= NP) continue;
+      const int64_t left = kend - (kp[u] + (int64_t)st * KC);  // valid k of the piece, if positive
+      const int32_t* s = src[u] + (int64_t)st * KC;
+      if constexpr (XV) {
+        const int n = left >= 4 ? 16 : (left > 0 ? 4 * (int)left : 0);
+        const uint32_t d = (uint32_t)__cvta_generic_to_shared(xt + 4 * e);
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(n ? s : P.x), "r"(n));
+      } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          cp_async4(xt + 4 * e + i, i < left ? (const void*)(s + i) : (const void*)P.x, i < left);
+      }
+    }
+  }
+  __device__ __forceinline__ void transpose(const int32_t* xt, int32_t* xs) const {
+    constexpr int XR = ClSmem<TMR>::XR;
+#pragma unroll
+    for (int u = 0; u < PIECES; ++u) {
+      const int e = threadIdx.x + THREADS * u;
+      if (e >= NP) continue;
+      const int4 v = *reinterpret_cast<const int4*>(xt + 4 * e);
+      int32_t* d = xs + (4 * (e % 4)) * XR + e / 4;
+      d[0] = v.x;
+      d[XR] = v.y;
+      d[2 * XR] = v.z;
+      d[3 * XR] = v.w;
+    }
+  }
+};
 
-// Codes of reduction indices [k0, k0 + 16) for columns [col0, col0 + 64) from
-// the expanded layout.
-__device__ __forceinline__ void stage_codes_expanded(const GemmParams& P, int32_t* cs, int64_t col0, int64_t k0) {
-  const int64_t nblocks = (P.cols + 31) / 32;
-  for (int e = threadIdx.x; e < 2 * KC * 16; e += THREADS) {
-    const int b = e / (KC * 16);
-    const int r = e - b * KC * 16;
-    const int kl = r >> 4, q = r & 15;
-    const int64_t cb = col0 / 32 + b;
-    const bool ok = cb < nblocks && k0 + kl < P.kred;
-    const int32_t* src = ok ? P.xcodes + ((cb * P.kred + k0 + kl) * 64 + q * 4) : P.xcodes;
-    cp_async16(cs + kl * CW + b * 64 + q * 4, src, ok);
-  }
-}
 
 // Blob path: the stage starting at k0 (a multiple of 16) is half (k0 / 16) % 2
 // of packed chunk k0 / 32.  Thread t decodes 8 indices of column t % 64
@@ -200,7 +236,7 @@ __device__ __forceinline__ bool tile_int32_exact(const GemmParams& P, int64_t co
   return !__syncthreads_or(unsafe);
 }
 
-template <int TMR, typename Acc>
+template <int TMR, bool XV, typename Acc>
 __device__ __forceinline__ void run_cluster_tile(const GemmParams& P, ClSmem<TMR>& sm, cg::cluster_group& cl,
                                                  int64_t row0, int64_t col0, int64_t kbeg, int64_t kend,
                                                  uint32_t& amax_local) {
@@ -217,12 +253,15 @@ __device__ __forceinline__ void run_cluster_tile(const GemmParams& P, ClSmem<TMR
   // a trailing CTA of the cluster may have an empty slice: it stages nothing
   // and contributes zero partial sums
   const int nst = kend > kbeg ? (int)((kend - kbeg + KC - 1) / KC) : 0;
+  const XStager<TMR, XV> xst(P, row0, kbeg, kend);
+  const ExpandedCodeStager cst(P.xcodes, P.cols, P.kred, col0, kbeg);
   if (nst > 0) {
-    stage_x<TMR>(P, sm.st.xs[0], row0, kbeg, kend);
-    if (expanded) stage_codes_expanded(P, sm.st.cs[0], col0, kbeg);
+    xst.copy(P, sm.st.xt, kend, 0);
+    if (expanded) cst.stage(P.xcodes, P.kred, sm.st.cs[0], 0);
     cp_async_commit();
     if (!expanded) decode_codes(P, sm.st.cs[0], col0, kbeg);
     cp_async_wait_all();
+    xst.transpose(sm.st.xt, sm.st.xs[0]);
   }
   for (int st = 0; st < nst; ++st) {
     const int b = st & 1;
@@ -230,14 +269,15 @@ __device__ __forceinline__ void run_cluster_tile(const GemmParams& P, ClSmem<TMR
     const int64_t k1 = kbeg + (int64_t)(st + 1) * KC;
     __syncthreads();
     if (more) {
-      stage_x<TMR>(P, sm.st.xs[b ^ 1], row0, k1, kend);
-      if (expanded) stage_codes_expanded(P, sm.st.cs[b ^ 1], col0, k1);
+      xst.copy(P, sm.st.xt, kend, st + 1);
+      if (expanded) cst.stage(P.xcodes, P.kred, sm.st.cs[b ^ 1], st + 1);
       cp_async_commit();
     }
     compute_stage<TMR, Acc>(sm.st.xs[b], sm.st.cs[b], tm, tn, acc);
     if (more) {
       if (!expanded) decode_codes(P, sm.st.cs[b ^ 1], col0, k1);
       cp_async_wait_all();
+      xst.transpose(sm.st.xt, sm.st.xs[b ^ 1]);
     }
   }
   __syncthreads();  // every thread is done with the staging buffers: they hold the partials next
@@ -312,7 +352,7 @@ __device__ __forceinline__ void run_cluster_tile(const GemmParams& P, ClSmem<TMR
   cl.sync();  // no CTA leaves (or reuses its shared memory) while another still reads it
 }
 
-template <int TMR>
+template <int TMR, bool XV>
 __global__ void __launch_bounds__(THREADS, kMinBlocks) linear_cluster_kernel(const GemmParams P, int64_t k_per_cta) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   ClSmem<TMR>& sm = *reinterpret_cast<ClSmem<TMR>*>(smem_raw);
@@ -323,9 +363,9 @@ __global__ void __launch_bounds__(THREADS, kMinBlocks) linear_cluster_kernel(con
   const int64_t kend = min(P.kred, kbeg + k_per_cta);
   uint32_t amax_local = 0;
   if (tile_int32_exact(P, col0)) {
-    run_cluster_tile<TMR, uint32_t>(P, sm, cl, row0, col0, kbeg, kend, amax_local);
+    run_cluster_tile<TMR, XV, uint32_t>(P, sm, cl, row0, col0, kbeg, kend, amax_local);
   } else {
-    run_cluster_tile<TMR, int64_t>(P, sm, cl, row0, col0, kbeg, kend, amax_local);
+    run_cluster_tile<TMR, XV, int64_t>(P, sm, cl, row0, col0, kbeg, kend, amax_local);
   }
   if (P.amax_out != nullptr) {
     amax_local = __reduce_max_sync(0xffffffffu, amax_local);
@@ -335,13 +375,13 @@ __global__ void __launch_bounds__(THREADS, kMinBlocks) linear_cluster_kernel(con
 
 // How many clusters of cs CTAs the device can hold at once (0: not
 // launchable), queried once per process and size.
-template <int TMR>
+template <int TMR, bool XV>
 int active_clusters(int cs) {
   static int cache[kMaxCluster + 1] = {0};
   static bool attrs_set = false;
   if (cs < 1 || cs > kMaxCluster) return 0;
   if (cache[cs] != 0) return cache[cs] > 0 ? cache[cs] : 0;
-  auto kern = linear_cluster_kernel<TMR>;
+  auto kern = linear_cluster_kernel<TMR, XV>;
   if (!attrs_set) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(ClSmem<TMR>)) !=
             cudaSuccess ||
@@ -371,7 +411,7 @@ int active_clusters(int cs) {
   return n;
 }
 
-template <int TMR>
+template <int TMR, bool XV>
 cudaError_t launch_tmr(const GemmParams& p, cudaStream_t st) {
   constexpr int MR = 8 * TMR;
   const int64_t tiles = ((p.rows + MR - 1) / MR) * ((p.cols + NT - 1) / NT);
@@ -380,8 +420,8 @@ cudaError_t launch_tmr(const GemmParams& p, cudaStream_t st) {
   // and a size the device accepts (trailing slices may still be empty)
   int64_t cs = std::min<int64_t>(std::min<int64_t>(kSlots / std::max<int64_t>(tiles, 1), kMaxCluster), stages);
   cs = std::max<int64_t>(cs, 1);
-  while (cs > 1 && active_clusters<TMR>((int)cs) <= 0) --cs;
-  if (active_clusters<TMR>((int)cs) <= 0) return cudaErrorLaunchOutOfResources;
+  while (cs > 1 && active_clusters<TMR, XV>((int)cs) <= 0) --cs;
+  if (active_clusters<TMR, XV>((int)cs) <= 0) return cudaErrorLaunchOutOfResources;
   const int64_t stages_per_cta = (stages + cs - 1) / cs;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)((p.rows + MR - 1) / MR), (unsigned)((p.cols + NT - 1) / NT), (unsigned)cs);
@@ -395,7 +435,14 @@ cudaError_t launch_tmr(const GemmParams& p, cudaStream_t st) {
   attr.val.clusterDim.z = (unsigned)cs;
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, linear_cluster_kernel<TMR>, p, stages_per_cta * KC);
+  return cudaLaunchKernelEx(&cfg, linear_cluster_kernel<TMR, XV>, p, stages_per_cta * KC);
+}
+
+template <bool XV>
+cudaError_t launch_xv(const GemmParams& p, cudaStream_t st) {
+  if (p.rows <= 8) return launch_tmr<1, XV>(p, st);
+  if (p.rows <= 32) return launch_tmr<4, XV>(p, st);
+  return launch_tmr<8, XV>(p, st);
 }
 
 }  // namespace
@@ -407,9 +454,9 @@ bool linear_cluster_preferred(const GemmParams& p) {
 }
 
 cudaError_t launch_linear_cluster(const GemmParams& p, cudaStream_t st) {
-  if (p.rows <= 8) return launch_tmr<1>(p, st);
-  if (p.rows <= 32) return launch_tmr<4>(p, st);
-  return launch_tmr<8>(p, st);
+  // 16-byte x pieces need 16-byte aligned rows: K a multiple of 4 (x itself is 16-byte aligned)
+  const bool xv = (p.kred % 4) == 0 && (reinterpret_cast<uintptr_t>(p.x) & 15) == 0;
+  return xv ? launch_xv<true>(p, st) : launch_xv<false>(p, st);
 }
 
 }  // namespace ds
