@@ -78,6 +78,7 @@ struct DirectGeom {
   int tiles_w, tiles_h;
   int splits, stages_per_split;  // split reduction over the stages
   int cluster;                   // > 1: the splits form one thread-block cluster (reduction in DSMEM)
+  int pairs;                     // stride 2: stage the halo with 8-byte copies (even W, odd padding)
   FastDiv dGW, dHR, dHP;         // dividers of the halo staging
 };
 
@@ -85,6 +86,11 @@ __device__ __forceinline__ void cp_async4(void* smem_dst, const void* gsrc, bool
   const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
   const int n = valid ? 4 : 0;
   asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(d), "l"(gsrc), "r"(n));
+}
+__device__ __forceinline__ void cp_async8(void* smem_dst, const void* gsrc, bool valid) {
+  const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
+  const int n = valid ? 8 : 0;
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;\n" ::"r"(d), "l"(gsrc), "r"(n));
 }
 __device__ __forceinline__ void cp_async16(void* smem_dst, const void* gsrc, bool valid) {
   const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
@@ -105,7 +111,12 @@ __device__ __forceinline__ uint32_t uabs(int32_t v) {
 template <int SIG, int S, int TM>
 struct Win {
   static constexpr int WS = (TM - 1) * SIG + S;  // window values
-  static constexpr int WV = (WS + 3) / 4;        // 16-byte loads per window
+  // Stride 2: the slot starts one column before the window (word D = 1 holds
+  // its first value), so that with an odd padding and an even row length
+  // (every ResNet stride-2 layer) the slot starts on an even column and is
+  // staged with 8-byte copies.
+  static constexpr int D = SIG == 2 ? 1 : 0;
+  static constexpr int WV = (WS + D + 3) / 4;  // 16-byte loads per window
   // slot stride in words: 16-byte aligned and 4 mod 8, so that the 4-byte
   // copies of 32 consecutive slots fill 8 bank groups (4-way at most) rather
   // than 2 (16-way) when the window is a multiple of 8 words
@@ -132,16 +143,35 @@ __device__ __forceinline__ void stage_halo(const GemmParams& P, const DirectGeom
     const int di = fdiv(o, G.dHP);
     const int ni = n0 + di;
     const int ih = o - di * G.HP - P.ph;
-    const int iws = iw0 + g * TM * SIG;
+    const int iws = iw0 + g * TM * SIG - WN::D;  // first staged column
     int32_t* dst = halo + sl * WN::WSP;
     const bool row_ok = (c < P.C) && (ni < G.N) && ((unsigned)ih < (unsigned)P.H);
     const int32_t* src = P.x + ((int64_t)ni * P.C + c) * HW + (int64_t)ih * P.W + iws;
-    if (row_ok && iws >= 0 && iws + WN::WS <= P.W) {
+    constexpr int NW = WN::WS + WN::D;  // words staged per slot
+    if constexpr (WN::D == 1) {
+      if (G.pairs) {
+        // 8-byte pieces: iws and the row start are even, so every piece is 8-byte aligned
+        constexpr int NP = (NW + 1) / 2;
+        if (row_ok && iws >= 0 && iws + 2 * NP <= P.W) {
 #pragma unroll
-      for (int i = 0; i < WN::WS; ++i) cp_async4(dst + i, src + i, true);
+          for (int j = 0; j < NP; ++j) cp_async8(dst + 2 * j, src + 2 * j, true);
+        } else {
+#pragma unroll
+          for (int j = 0; j < NP; ++j) {
+            const int col = iws + 2 * j;  // even, so a piece is either inside the row or outside (W even)
+            const bool ok = row_ok && col >= 0 && col < P.W;
+            cp_async8(dst + 2 * j, ok ? (const void*)(src + 2 * j) : (const void*)P.x, ok);
+          }
+        }
+        continue;
+      }
+    }
+    if (row_ok && iws >= 0 && iws + NW <= P.W) {
+#pragma unroll
+      for (int i = 0; i < NW; ++i) cp_async4(dst + i, src + i, true);
     } else {
 #pragma unroll
-      for (int i = 0; i < WN::WS; ++i) {
+      for (int i = 0; i < NW; ++i) {
         const bool ok = row_ok && ((unsigned)(iws + i) < (unsigned)P.W);
         cp_async4(dst + i, ok ? (const void*)(src + i) : (const void*)P.x, ok);
       }
@@ -249,7 +279,7 @@ __device__ __forceinline__ void compute_stage(const DirectGeom G, const int32_t*
         for (int j = 0; j < TN; ++j) {
 #pragma unroll
           for (int i = 0; i < NI; ++i) {
-            const int t = w[(I0 + i) * SIG + s] >> sh[j];  // Eq. 1
+            const int t = w[(I0 + i) * SIG + s + WN::D] >> sh[j];  // Eq. 1
             if constexpr (sizeof(Acc) == 4) {
               acc[i][j] += (uint32_t)sg[j] * (uint32_t)t;  // Eq. 2 + accumulate (mod 2^32)
             } else {
@@ -557,7 +587,7 @@ bool choose_geom(const GemmParams& p, size_t split_capacity, Choice& ch) {
   // variant); with a workspace (the chained forward) the atomic split is
   // used: measured faster there (ResNet18 batch 1: 0.51 vs 0.63 ms per forward).
   const bool allow_cluster = split_capacity == 0 && ch.TM == 7 && (p.S == 3 || p.S == 7);
-  const int WS = (ch.TM - 1) * p.sw + p.S;
+  const int WS = (ch.TM - 1) * p.sw + p.S + (p.sw == 2 ? 1 : 0);  // staged words, with Win<>::D
   const int WSP = (WS + 3) / 4 * 4 + (((WS + 3) / 4) % 2 == 0 ? 4 : 0);  // as Win<>::WSP
   int gw = (p.OW + ch.TM - 1) / ch.TM;
   if (gw > 8) {
@@ -620,6 +650,9 @@ bool choose_geom(const GemmParams& p, size_t split_capacity, Choice& ch) {
   if (run < 1) run = 1;
   if (run > 16 && p.xcodes == nullptr) return false;
   G.run = run;
+  // 8-byte halo pieces: the first staged column iw0 + g TM sig - 1 is even when
+  // the padding is odd, and a row starts on an even word when W is even
+  G.pairs = (p.sw == 2 && (p.W % 2) == 0 && (p.pw % 2) == 1 && (reinterpret_cast<uintptr_t>(p.x) & 7) == 0) ? 1 : 0;
   G.dGW = make_fastdiv((uint32_t)G.GW);
   G.dHR = make_fastdiv((uint32_t)G.HR);
   G.dHP = make_fastdiv((uint32_t)G.HP);
@@ -670,14 +703,25 @@ bool set_attributes() {
   return state == 1;
 }
 
-// Whether the device can co-schedule a cluster of cs CTAs of this kernel
-// (cached per process and size).
+// How many clusters of cs CTAs of this kernel, with smem bytes of shared
+// memory each, the device holds at once (0: none).  Cached per process for
+// up to kCacheEntries (size, shared memory) pairs; past that it is queried
+// each time.
 template <int SIG, int S, int TM>
-bool cluster_ok(int cs, size_t smem) {
-  if (!set_attributes<SIG, S, TM, true>()) return false;
-  static int cache[kMaxCluster + 1] = {0};
-  if (cs < 2 || cs > kMaxCluster) return false;
-  if (cache[cs] == 0) {
+int max_clusters(int cs, size_t smem) {
+  if (!set_attributes<SIG, S, TM, true>()) return 0;
+  if (cs < 2 || cs > kMaxCluster) return 0;
+  constexpr int kCacheEntries = 64;
+  struct Entry {
+    int cs;
+    size_t smem;
+    int n;
+  };
+  static Entry cache[kCacheEntries];
+  static int used = 0;
+  for (int i = 0; i < used; ++i)
+    if (cache[i].cs == cs && cache[i].smem == smem) return cache[i].n;
+  {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(1, 1, cs);
     cfg.blockDim = dim3(kMaxThreads, 1, 1);
@@ -694,9 +738,10 @@ bool cluster_ok(int cs, size_t smem) {
       (void)cudaGetLastError();
       n = 0;
     }
-    cache[cs] = n > 0 ? 1 : -1;
+    n = n > 0 ? n : 0;
+    if (used < kCacheEntries) cache[used++] = Entry{cs, smem, n};
+    return n;
   }
-  return cache[cs] > 0;
 }
 
 // Cluster-split variants exist for the network shapes (TM = 7; 3x3 and 7x7 kernels).
@@ -707,11 +752,25 @@ cudaError_t launch_direct(const GemmParams& p, const DirectGeom& G0, cudaStream_
   if (!set_attributes<SIG, S, TM, false>()) return cudaErrorInvalidValue;
   DirectGeom G = G0;
   if (G.cluster > 1) {
-    // the largest cluster size the device accepts; without one, no split
+    // The cluster size with the least time, counted as waves x stages per
+    // rank, over every size up to 16 with at least one stage per rank: the
+    // device holds max_clusters(cs) clusters at once, which can be fewer
+    // than the SM slots allow (e.g. 110 clusters of 4 for 112 needed: two of
+    // them would run in a second wave), and a larger cluster in two waves
+    // can beat a smaller one in one.  cs = 1: no split.
     int cs = 1;
     if constexpr (has_cluster_variant(S, TM)) {
-      cs = G.cluster;
-      while (cs >= 2 && !cluster_ok<SIG, S, TM>(cs, launch_smem_bytes(G, TM))) --cs;
+      const int64_t tiles = (int64_t)G.tiles_w * G.tiles_h * ((p.cols + NT - 1) / NT);
+      int64_t best = ((tiles + kSlots - 1) / kSlots) * G.n_stages;
+      for (int c = 2; c <= std::min(kMaxCluster, G.n_stages); ++c) {
+        const int n = max_clusters<SIG, S, TM>(c, launch_smem_bytes(G, TM));
+        if (n <= 0) continue;
+        const int64_t cost = ((tiles + n - 1) / n) * ((G.n_stages + c - 1) / c);
+        if (cost < best) {
+          best = cost;
+          cs = c;
+        }
+      }
     }
     if (cs >= 2) {
       G.cluster = cs;

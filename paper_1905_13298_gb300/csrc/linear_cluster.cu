@@ -416,12 +416,23 @@ cudaError_t launch_tmr(const GemmParams& p, cudaStream_t st) {
   constexpr int MR = 8 * TMR;
   const int64_t tiles = ((p.rows + MR - 1) / MR) * ((p.cols + NT - 1) / NT);
   const int64_t stages = (p.kred + KC - 1) / KC;
-  // the cluster size: at most one wave of CTAs, at least one stage per CTA,
-  // and a size the device accepts (trailing slices may still be empty)
-  int64_t cs = std::min<int64_t>(std::min<int64_t>(kSlots / std::max<int64_t>(tiles, 1), kMaxCluster), stages);
-  cs = std::max<int64_t>(cs, 1);
-  while (cs > 1 && active_clusters<TMR, XV>((int)cs) <= 0) --cs;
-  if (active_clusters<TMR, XV>((int)cs) <= 0) return cudaErrorLaunchOutOfResources;
+  // the cluster size: at most one wave of CTAs and at least one stage per
+  // CTA, chosen for the least time counted as waves x stages per CTA, where
+  // a wave is the number of clusters the device holds at once (trailing
+  // slices may still be empty)
+  const int64_t cs_max = std::max<int64_t>(
+      std::min<int64_t>(std::min<int64_t>(kSlots / std::max<int64_t>(tiles, 1), kMaxCluster), stages), 1);
+  int64_t cs = 0, best = 0;
+  for (int64_t c = 1; c <= cs_max; ++c) {
+    const int n = active_clusters<TMR, XV>((int)c);
+    if (n <= 0) continue;
+    const int64_t cost = ((tiles + n - 1) / n) * ((stages + c - 1) / c);
+    if (cs == 0 || cost < best) {
+      best = cost;
+      cs = c;
+    }
+  }
+  if (cs == 0) return cudaErrorLaunchOutOfResources;
   const int64_t stages_per_cta = (stages + cs - 1) / cs;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)((p.rows + MR - 1) / MR), (unsigned)((p.cols + NT - 1) / NT), (unsigned)cs);
