@@ -4,20 +4,25 @@
 //
 // x is bf16, W = s * 2^p is exact in bf16 (sign bit, exponent 127 + p, zero
 // mantissa; s = 0 gives +0), so every product is exact and only the fp32
-// accumulation rounds.  This is a dense contraction, so it runs as a GEMM:
-//   * one CTA per 128 x 256 output tile, 6 warps:
-//       warp 0  one elected thread issues TMA loads (128B-swizzled K-major
-//               tiles of 64 bf16) into a 4-stage shared-memory ring,
-//       warp 1  allocates 256 TMEM columns; one thread issues tcgen05.mma
-//               (kind::f16, M=128, N=256, K=16, fp32 accumulator in TMEM),
-//               and frees each ring slot with tcgen05.commit,
-//       warps 2-5 wait for the last commit, read the accumulator with
-//               tcgen05.ld (one TMEM lane quarter per warp), add the bias,
-//               apply ReLU and store fp32 rows.
-//   * mbarriers: full[s] (TMA bytes landed), empty[s] (MMAs done reading
-//     slot s), accum (all MMAs done).  Every wait is bounded by a clock
-//     deadline; on expiry the kernel records a fault flag, stops issuing
-//     work, waits (bounded) for issued work and frees its TMEM.
+// accumulation rounds.  This is a dense contraction, so it runs as a GEMM.
+// Persistent: one CTA per SM walks the 128 x 256 output tiles t = blockIdx.x,
+// blockIdx.x + gridDim.x, ... (m fastest), 6 warps:
+//   warp 0     one elected thread issues TMA loads (128B-swizzled K-major
+//              tiles of 64 bf16) into a 4-stage shared-memory ring that runs
+//              on across tiles,
+//   warp 1     allocates 512 TMEM columns: two 256-column fp32 accumulators.
+//              One thread issues tcgen05.mma (kind::f16, M=128, N=256, K=16)
+//              for tile i into accumulator i % 2, frees each ring slot with
+//              tcgen05.commit and commits the tile to tfull[i % 2],
+//   warps 2-5  wait for tfull, read the accumulator with tcgen05.ld (one TMEM
+//              lane quarter per warp), release it (tempty) and add the bias,
+//              apply ReLU and store fp32 rows, while the MMAs of the next
+//              tile run into the other accumulator.
+// mbarriers: full[s] (TMA bytes landed), empty[s] (MMAs done reading slot s),
+// tfull[b] (tile's MMAs done), tempty[b] (accumulator b read out), done (all
+// MMAs of the CTA finished, waited for before TMEM is freed).  Every wait is
+// bounded by a clock deadline; on expiry the kernel records a fault flag,
+// stops issuing work, waits (bounded) for issued work and frees its TMEM.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -33,8 +38,10 @@ constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
 constexpr int A_BYTES = BM * BK * 2;  // 16 KB
 constexpr int B_BYTES = BN * BK * 2;  // 32 KB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int TMEM_COLS = 256;
+constexpr int ACC_BUFS = 2;
+constexpr int TMEM_COLS = ACC_BUFS * BN;  // 512: the whole tensor memory of an SM
 constexpr int kThreads = 192;
+constexpr int kEpiWarps = 4;
 constexpr long long kTimeoutCycles = 4000000000LL;  // about 2 s at 2 GHz
 
 struct Bf16Params {
@@ -47,7 +54,9 @@ struct Bf16Params {
 struct __align__(8) Barriers {
   uint64_t full[STAGES];
   uint64_t empty[STAGES];
-  uint64_t accum;
+  uint64_t tfull[ACC_BUFS];
+  uint64_t tempty[ACC_BUFS];
+  uint64_t done;
   uint32_t tmem_base;
   int abort;
 };
@@ -62,6 +71,9 @@ __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
 __device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
                : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
@@ -87,6 +99,12 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
     }
   }
   return true;
+}
+// Bounded wait that ignores the abort flag (draining work already issued).
+__device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity) {
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity) && clock64() - t0 < kTimeoutCycles) {
+  }
 }
 
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x, int y) {
@@ -134,8 +152,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   Barriers* bars = reinterpret_cast<Barriers*>(smem + STAGES * STAGE_BYTES);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t m0 = (int64_t)blockIdx.x * BM;
-  const int64_t n0 = (int64_t)blockIdx.y * BN;
+  const int64_t tiles_m = (P.M + BM - 1) / BM;
+  const int64_t ntiles = tiles_m * ((P.N + BN - 1) / BN);
   const int nk = (int)((P.K + BK - 1) / BK);
   volatile int* abort = &bars->abort;
 
@@ -144,7 +162,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bars->full[s], 1);
       mbar_init(&bars->empty[s], 1);
     }
-    mbar_init(&bars->accum, 1);
+    for (int b = 0; b < ACC_BUFS; ++b) {
+      mbar_init(&bars->tfull[b], 1);
+      mbar_init(&bars->tempty[b], kEpiWarps);
+    }
+    mbar_init(&bars->done, 1);
     bars->abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -158,95 +180,129 @@ __global__ void __launch_bounds__(kThreads, 1)
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-  const uint32_t tmem_d = bars->tmem_base;
+  const uint32_t tmem_base = bars->tmem_base;
 
   if (warp == 0) {
-    if (lane == 0) {  // TMA producer
-      int issued = 0;
-      for (int kt = 0; kt < nk; ++kt) {
-        const int s = kt % STAGES;
-        const uint32_t ph = (uint32_t)(kt / STAGES) & 1u;
-        if (kt >= STAGES && !mbar_wait(&bars->empty[s], ph ^ 1u, abort)) break;
-        unsigned char* a = smem + s * STAGE_BYTES;
-        mbar_expect_tx(&bars->full[s], STAGE_BYTES);
-        tma_load_2d(a, &tmap_x, &bars->full[s], kt * BK, (int)m0);
-        tma_load_2d(a + A_BYTES, &tmap_w, &bars->full[s], kt * BK, (int)n0);
-        issued = kt + 1;
-      }
-      // before leaving, let every issued copy land (bounded): waiting on the
-      // last STAGES full barriers covers all copies still in flight
-      for (int kt = (issued > STAGES ? issued - STAGES : 0); kt < issued; ++kt) {
-        const long long t0 = clock64();
-        while (!mbar_try_wait(&bars->full[kt % STAGES], (uint32_t)(kt / STAGES) & 1u) &&
-               clock64() - t0 < kTimeoutCycles) {
+    if (lane == 0) {  // TMA producer: the ring's slot counter runs on across tiles
+      int64_t it = 0;
+      bool ok = true;
+      for (int64_t t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
+        const int m0 = (int)((t % tiles_m) * BM), n0 = (int)((t / tiles_m) * BN);
+        for (int kt = 0; kt < nk; ++kt, ++it) {
+          const int s = (int)(it % STAGES);
+          const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
+          if (it >= STAGES && !mbar_wait(&bars->empty[s], ph ^ 1u, abort)) {
+            ok = false;
+            break;
+          }
+          unsigned char* a = smem + s * STAGE_BYTES;
+          mbar_expect_tx(&bars->full[s], STAGE_BYTES);
+          tma_load_2d(a, &tmap_x, &bars->full[s], kt * BK, m0);
+          tma_load_2d(a + A_BYTES, &tmap_w, &bars->full[s], kt * BK, n0);
         }
       }
+      // before leaving, let every issued copy land (bounded): the last
+      // STAGES full barriers cover all copies still in flight
+      for (int64_t j = (it > STAGES ? it - STAGES : 0); j < it; ++j)
+        mbar_drain(&bars->full[j % STAGES], (uint32_t)(j / STAGES) & 1u);
     }
   } else if (warp == 1) {
     if (lane == 0) {  // MMA issuer
+      int64_t it = 0;
+      int64_t i = 0;  // tiles of this CTA so far
       bool ok = true;
-      for (int kt = 0; kt < nk && ok; ++kt) {
-        const int s = kt % STAGES;
-        const uint32_t ph = (uint32_t)(kt / STAGES) & 1u;
-        ok = mbar_wait(&bars->full[s], ph, abort);
-        if (!ok) break;
+      for (int64_t t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++i) {
+        const int b = (int)(i & 1);
+        // accumulator b is free once the epilogue has read tile i - 2 out of it
+        if (i >= ACC_BUFS && !mbar_wait(&bars->tempty[b], (uint32_t)((i / ACC_BUFS) - 1) & 1u, abort)) break;
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        const uint32_t a = smem_u32(smem + s * STAGE_BYTES);
-        const uint32_t b = a + A_BYTES;
+        const uint32_t tmem_d = tmem_base + (uint32_t)(b * BN);
+        for (int kt = 0; kt < nk; ++kt, ++it) {
+          const int s = (int)(it % STAGES);
+          const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
+          if (!mbar_wait(&bars->full[s], ph, abort)) {
+            ok = false;
+            break;
+          }
+          asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+          const uint32_t a = smem_u32(smem + s * STAGE_BYTES);
+          const uint32_t bb = a + A_BYTES;
 #pragma unroll
-        for (int k = 0; k < BK / 16; ++k) {
-          umma_bf16(tmem_d, sw128_desc(a + 32 * k), sw128_desc(b + 32 * k), (kt > 0 || k > 0) ? 1u : 0u);
+          for (int k = 0; k < BK / 16; ++k)
+            umma_bf16(tmem_d, sw128_desc(a + 32 * k), sw128_desc(bb + 32 * k), (kt > 0 || k > 0) ? 1u : 0u);
+          umma_commit(&bars->empty[s]);  // slot s is free once these MMAs have read it
         }
-        umma_commit(&bars->empty[s]);  // slot s is free once these MMAs have read it
+        if (ok) umma_commit(&bars->tfull[b]);  // fires when the tile's MMAs have completed
       }
-      umma_commit(&bars->accum);  // fires when every issued MMA has completed
+      // every MMA issued by this CTA has completed before TMEM is freed
+      umma_commit(&bars->done);
+      mbar_drain(&bars->done, 0u);
     }
   } else {
     // epilogue: warps 2..5 own TMEM lane quarters (warp % 4)
     const int q = warp & 3;
-    const bool ok = mbar_wait(&bars->accum, 0u, abort);
-    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    const int64_t row = m0 + 32 * q + lane;
     const bool relu = (P.flags & DS_RELU) != 0;
-    for (int c0 = 0; c0 < BN; c0 += 32) {
-      uint32_t r[32];
-      const uint32_t taddr = tmem_d + ((uint32_t)(32 * q) << 16) + (uint32_t)c0;
-      asm volatile(
-          "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, "
-          "%14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
-          : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-            "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
-            "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]),
-            "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]),
-            "=r"(r[30]), "=r"(r[31])
-          : "r"(taddr)
-          : "memory");
-      asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-      if (!ok || row >= P.M) continue;
-      float* yrow = P.y + row * P.N + n0 + c0;
-      const int64_t nvalid = P.N - (n0 + c0);
-      if (nvalid >= 32 && (P.N & 3) == 0) {
-#pragma unroll
-        for (int j = 0; j < 32; j += 4) {
-          float4 v;
-          v.x = __uint_as_float(r[j]) + (P.bias ? __ldg(P.bias + n0 + c0 + j) : 0.f);
-          v.y = __uint_as_float(r[j + 1]) + (P.bias ? __ldg(P.bias + n0 + c0 + j + 1) : 0.f);
-          v.z = __uint_as_float(r[j + 2]) + (P.bias ? __ldg(P.bias + n0 + c0 + j + 2) : 0.f);
-          v.w = __uint_as_float(r[j + 3]) + (P.bias ? __ldg(P.bias + n0 + c0 + j + 3) : 0.f);
-          if (relu) {
-            v.x = fmaxf(v.x, 0.f);
-            v.y = fmaxf(v.y, 0.f);
-            v.z = fmaxf(v.z, 0.f);
-            v.w = fmaxf(v.w, 0.f);
-          }
-          *reinterpret_cast<float4*>(yrow + j) = v;
+    const bool bias_vec = P.bias != nullptr && (reinterpret_cast<uintptr_t>(P.bias) & 15) == 0;
+    int64_t i = 0;
+    for (int64_t t = blockIdx.x; t < ntiles; t += gridDim.x, ++i) {
+      const int b = (int)(i & 1);
+      if (!mbar_wait(&bars->tfull[b], (uint32_t)(i / ACC_BUFS) & 1u, abort)) break;
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      const int64_t m0 = (t % tiles_m) * BM, n0 = (t / tiles_m) * BN;
+      const int64_t row = m0 + 32 * q + lane;
+      for (int c0 = 0; c0 < BN; c0 += 32) {
+        uint32_t r[32];
+        const uint32_t taddr = tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(b * BN + c0);
+        asm volatile(
+            "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, "
+            "%14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+            : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+              "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
+              "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
+              "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
+              "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+            : "r"(taddr)
+            : "memory");
+        asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+        if (c0 + 32 == BN) {
+          // the whole accumulator is in registers: hand it back to the MMA warp
+          asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&bars->tempty[b]);
         }
-      } else {
+        if (row >= P.M) continue;
+        float* yrow = P.y + row * P.N + n0 + c0;
+        const int64_t nvalid = P.N - (n0 + c0);
+        if (nvalid >= 32 && (P.N & 3) == 0) {
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          if (j < nvalid) {
-            float v = __uint_as_float(r[j]) + (P.bias ? __ldg(P.bias + n0 + c0 + j) : 0.f);
-            yrow[j] = relu ? fmaxf(v, 0.f) : v;
+          for (int j = 0; j < 32; j += 4) {
+            float4 bv = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (bias_vec) {
+              bv = __ldg(reinterpret_cast<const float4*>(P.bias + n0 + c0 + j));
+            } else if (P.bias) {
+              bv = make_float4(__ldg(P.bias + n0 + c0 + j), __ldg(P.bias + n0 + c0 + j + 1),
+                               __ldg(P.bias + n0 + c0 + j + 2), __ldg(P.bias + n0 + c0 + j + 3));
+            }
+            float4 v;
+            v.x = __uint_as_float(r[j]) + bv.x;
+            v.y = __uint_as_float(r[j + 1]) + bv.y;
+            v.z = __uint_as_float(r[j + 2]) + bv.z;
+            v.w = __uint_as_float(r[j + 3]) + bv.w;
+            if (relu) {
+              v.x = fmaxf(v.x, 0.f);
+              v.y = fmaxf(v.y, 0.f);
+              v.z = fmaxf(v.z, 0.f);
+              v.w = fmaxf(v.w, 0.f);
+            }
+            *reinterpret_cast<float4*>(yrow + j) = v;
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            if (j < nvalid) {
+              float v = __uint_as_float(r[j]) + (P.bias ? __ldg(P.bias + n0 + c0 + j) : 0.f);
+              yrow[j] = relu ? fmaxf(v, 0.f) : v;
+            }
           }
         }
       }
@@ -256,7 +312,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   if (warp == 1) {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_d), "r"(TMEM_COLS)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(TMEM_COLS)
                  : "memory");
   }
 }
@@ -336,8 +392,16 @@ cudaError_t launch_linear_bf16(const uint16_t* x, const uint16_t* w16, const flo
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
+  static int sms = 0;
+  if (sms == 0) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+  }
   Bf16Params p{y, bias, M, N, K, flags};
-  dim3 grid((unsigned)((M + BM - 1) / BM), (unsigned)((N + BN - 1) / BN));
+  const int64_t tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
+  const unsigned grid = (unsigned)(tiles < sms ? tiles : sms);  // persistent: one CTA per SM
   linear_bf16_kernel<<<grid, kThreads, smem, st>>>(mx, mw, p);
   return cudaGetLastError();
 }

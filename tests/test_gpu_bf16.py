@@ -63,6 +63,14 @@ def test_bf16_small_shapes(dslib, M, K, N):
     _check(y, bits, s, p, b)
 
 
+@pytest.mark.parametrize("M,K,N", [(2560, 72, 2560), (1000, 40, 5000)])
+def test_bf16_more_tiles_than_sms(dslib, M, K, N):
+    """More 128 x 256 output tiles (200, 160) than SMs, ragged edges: every output checked."""
+    bits, s, p, b = _case(M + 3 * K + N, M, K, N)
+    y, _ = _run(dslib, bits, s, p, b, relu=True)
+    _check(y, bits, s, p, b, relu=True)
+
+
 def test_bf16_relu_and_exact_small_integers(dslib):
     """Small-integer activations with few terms: the fp32 sum is exact, so the result is bit-exact."""
     M, K, N = 130, 64, 257

@@ -36,6 +36,11 @@ GEOMS = [
     (1, 40, 7, 7, 130, 1, 1, 1, 0),
     (2, 48, 8, 8, 72, 1, 1, 1, 0),      # 1x1, OH*OW % 4 == 0: 16-byte epilogue, ragged channel tile
     (1, 20, 16, 16, 36, 1, 1, 2, 0),    # 1x1 / 2, 16-byte epilogue, channels not a multiple of 16
+    # stride 2: halo slots start one column early; 8-byte pieces need an even width and an odd padding
+    (2, 6, 10, 10, 12, 3, 3, 2, 0),     # even padding: 4-byte copies, 8-pixel groups
+    (1, 4, 20, 20, 8, 3, 3, 2, 1),      # 8-byte pieces, 8-pixel groups (OW = 10)
+    (2, 5, 28, 30, 9, 7, 7, 2, 3),      # 7x7/2 with 8-byte pieces, OW = 15
+    (1, 3, 17, 14, 5, 3, 3, 2, 2),      # padding 2: 4-byte copies
 ]
 
 
