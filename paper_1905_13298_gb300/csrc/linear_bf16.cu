@@ -6,7 +6,9 @@
 // mantissa; s = 0 gives +0), so every product is exact and only the fp32
 // accumulation rounds.  This is a dense contraction, so it runs as a GEMM.
 // Persistent: one CTA per SM walks the 128 x 256 output tiles t = blockIdx.x,
-// blockIdx.x + gridDim.x, ... (m fastest), 6 warps:
+// blockIdx.x + gridDim.x, ... in grouped order (tile_of): groups of G row
+// tiles, n fastest inside a group, with G x (column tiles) about one wave, so
+// the tiles in flight share their x rows and W rows in L2.  6 warps:
 //   warp 0     one elected thread issues TMA loads (128B-swizzled K-major
 //              tiles of 64 bf16) into a 4-stage shared-memory ring that runs
 //              on across tiles,
@@ -143,6 +145,16 @@ __device__ __forceinline__ void umma_commit(uint64_t* bar) {
                : "memory");
 }
 
+// Tile t of the grouped order: rows [m0, m0 + BM), columns [n0, n0 + BN).
+__device__ __forceinline__ void tile_of(int64_t t, int64_t tiles_m, int64_t tiles_n, int64_t G, int& m0, int& n0) {
+  const int64_t per_group = G * tiles_n;
+  const int64_t first_m = (t / per_group) * G;
+  const int64_t gsize = tiles_m - first_m < G ? tiles_m - first_m : G;
+  const int64_t r = t - (t / per_group) * per_group;
+  m0 = (int)((first_m + r % gsize) * BM);
+  n0 = (int)((r / gsize) * BN);
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
     linear_bf16_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant__ CUtensorMap tmap_w,
                        const Bf16Params P) {
@@ -153,7 +165,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   Barriers* bars = reinterpret_cast<Barriers*>(smem + STAGES * STAGE_BYTES);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int64_t tiles_m = (P.M + BM - 1) / BM;
-  const int64_t ntiles = tiles_m * ((P.N + BN - 1) / BN);
+  const int64_t tiles_n = (P.N + BN - 1) / BN;
+  const int64_t ntiles = tiles_m * tiles_n;
+  // rows tiles per group: about one wave of CTAs per group
+  int64_t G = (gridDim.x + tiles_n - 1) / tiles_n;
+  G = G < 1 ? 1 : (G > tiles_m ? tiles_m : G);
   const int nk = (int)((P.K + BK - 1) / BK);
   volatile int* abort = &bars->abort;
 
@@ -187,7 +203,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       int64_t it = 0;
       bool ok = true;
       for (int64_t t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
-        const int m0 = (int)((t % tiles_m) * BM), n0 = (int)((t / tiles_m) * BN);
+        int m0, n0;
+        tile_of(t, tiles_m, tiles_n, G, m0, n0);
         for (int kt = 0; kt < nk; ++kt, ++it) {
           const int s = (int)(it % STAGES);
           const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
@@ -248,7 +265,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int b = (int)(i & 1);
       if (!mbar_wait(&bars->tfull[b], (uint32_t)(i / ACC_BUFS) & 1u, abort)) break;
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-      const int64_t m0 = (t % tiles_m) * BM, n0 = (t / tiles_m) * BN;
+      int tm0, tn0;
+      tile_of(t, tiles_m, tiles_n, G, tm0, tn0);
+      const int64_t m0 = tm0, n0 = tn0;
       const int64_t row = m0 + 32 * q + lane;
       for (int c0 = 0; c0 < BN; c0 += 32) {
         uint32_t r[32];
