@@ -24,6 +24,7 @@
 #include <cooperative_groups.h>
 
 #include <algorithm>
+#include <mutex>
 
 #include "ds_common.cuh"
 
@@ -689,18 +690,18 @@ size_t launch_smem_bytes(const DirectGeom& G, int TM) {
 
 template <int SIG, int S, int TM, bool CL>
 bool set_attributes() {
-  // once per process (not a stream operation, so a forward captured in a CUDA
-  // graph after a first eager call issues no attribute call)
-  static int state = 0;  // 0 unset, 1 ok, -1 failed
-  if (state == 0) {
-    const bool ok = cudaFuncSetAttribute(conv_direct_kernel<SIG, S, TM, CL>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget) == cudaSuccess &&
-                    (!CL || cudaFuncSetAttribute(conv_direct_kernel<SIG, S, TM, CL>,
-                                                 cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess);
-    if (!ok) (void)cudaGetLastError();
-    state = ok ? 1 : -1;
-  }
-  return state == 1;
+  // once per process, thread-safe (a function-local static is initialised
+  // once); not a stream operation, so a forward captured in a CUDA graph
+  // after a first eager call issues no attribute call
+  static const bool ok = [] {
+    const bool r = cudaFuncSetAttribute(conv_direct_kernel<SIG, S, TM, CL>,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget) == cudaSuccess &&
+                   (!CL || cudaFuncSetAttribute(conv_direct_kernel<SIG, S, TM, CL>,
+                                                cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess);
+    if (!r) (void)cudaGetLastError();
+    return r;
+  }();
+  return ok;
 }
 
 // How many clusters of cs CTAs of this kernel, with smem bytes of shared
@@ -719,6 +720,8 @@ int max_clusters(int cs, size_t smem) {
   };
   static Entry cache[kCacheEntries];
   static int used = 0;
+  static std::mutex mu;  // the cache is shared by every host thread
+  std::lock_guard<std::mutex> lock(mu);
   for (int i = 0; i < used; ++i)
     if (cache[i].cs == cs && cache[i].smem == smem) return cache[i].n;
   {

@@ -376,13 +376,10 @@ int pw_stages_per_split(const GemmParams& p, size_t split_capacity) {
 template <bool STRIDED>
 cudaError_t launch_pw(const GemmParams& p, cudaStream_t st) {
   const size_t smem = sizeof(PwSmem);
-  static bool attr_set = false;  // once per process (see conv_direct.cu)
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(conv_pointwise_kernel<STRIDED>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  // once per process, thread-safe (see conv_direct.cu)
+  static const cudaError_t attr = cudaFuncSetAttribute(conv_pointwise_kernel<STRIDED>,
+                                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (attr != cudaSuccess) return attr;
   const int n_stages = (p.C + KC - 1) / KC;
   const int sps = pw_stages_per_split(p, p.split_acc ? p.split_capacity : 0);
   const int splits = (n_stages + sps - 1) / sps;

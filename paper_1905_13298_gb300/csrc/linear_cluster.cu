@@ -34,6 +34,7 @@
 #include <cooperative_groups.h>
 
 #include <algorithm>
+#include <mutex>
 
 #include "ds_common.cuh"
 
@@ -68,10 +69,6 @@ struct ClSmem {
 __device__ __forceinline__ void cp_async4(void* smem_dst, const void* gsrc, bool valid) {
   const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
   asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(d), "l"(gsrc), "r"(valid ? 4 : 0));
-}
-__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gsrc, bool valid) {
-  const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(gsrc), "r"(valid ? 16 : 0));
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::); }
@@ -379,6 +376,8 @@ template <int TMR, bool XV>
 int active_clusters(int cs) {
   static int cache[kMaxCluster + 1] = {0};
   static bool attrs_set = false;
+  static std::mutex mu;  // the cache is shared by every host thread
+  std::lock_guard<std::mutex> lock(mu);
   if (cs < 1 || cs > kMaxCluster) return 0;
   if (cache[cs] != 0) return cache[cs] > 0 ? cache[cs] : 0;
   auto kern = linear_cluster_kernel<TMR, XV>;

@@ -386,13 +386,10 @@ __global__ void __launch_bounds__(THREADS, 3) shift_gemm_kernel(const GemmParams
 template <bool CONV, bool VEC>
 cudaError_t launch_impl(const GemmParams& p, cudaStream_t st) {
   const size_t smem = sizeof(Smem);
-  static bool attr_set = false;  // once per process (see conv_direct.cu)
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(shift_gemm_kernel<CONV, VEC>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  // once per process, thread-safe (see conv_direct.cu)
+  static const cudaError_t attr = cudaFuncSetAttribute(shift_gemm_kernel<CONV, VEC>,
+                                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (attr != cudaSuccess) return attr;
   dim3 grid((unsigned)((p.rows + MT - 1) / MT), (unsigned)((p.cols + NT - 1) / NT));
   shift_gemm_kernel<CONV, VEC><<<grid, THREADS, smem, st>>>(p);
   return cudaGetLastError();
