@@ -32,8 +32,9 @@ constexpr int XS = 36;        // words per x-tile row (32 + 4 pad: conflict-free
 
 struct __align__(16) Smem {
   int32_t xs[2][MT * XS];
-  int32_t shs[2][kChunk * NT];  // shift amount -p per (k, col)
-  int32_t sgs[2][kChunk * NT];  // sign s per (k, col)
+  // codes per k: for each 32-column block, 32 shift amounts -p then 32 signs
+  // (the expanded layout's row, so that layout is copied as is)
+  int32_t cs[2][kChunk * 2 * NT];
 };
 
 __device__ __forceinline__ void cp_async4(void* smem_dst, const void* gsrc, bool valid) {
@@ -72,23 +73,43 @@ struct RowCtx {
   bool valid;
 };
 
+// FC x tile, 16-byte pieces: piece t + THREADS i is quad t % 8 of row
+// t / 8 + 16 i, the same for every chunk, so the source address is computed
+// once (row t / 8 at chunk 0) and the rows present kept as a bit mask.
+struct XQuads {
+  const int32_t* src;
+  int64_t row_step;  // words between rows t / 8 + 16 i and t / 8 + 16 (i + 1)
+  uint32_t rows_ok;  // bit i: row t / 8 + 16 i exists
+};
+
+__device__ __forceinline__ XQuads x_quads(const GemmParams& P, int64_t row0) {
+  const int t = threadIdx.x;
+  XQuads q;
+  q.src = P.x + (row0 + (t >> 3)) * P.kred + 4 * (t & 7);
+  q.row_step = 16 * P.kred;
+  q.rows_ok = 0u;
+#pragma unroll
+  for (int i = 0; i < (MT * 8) / THREADS; ++i)
+    if (row0 + (t >> 3) + 16 * i < P.rows) q.rows_ok |= 1u << i;
+  return q;
+}
+
 template <bool CONV, bool VEC>
 __device__ __forceinline__ void stage_x(const GemmParams& P, Smem& sm, int buf, int64_t row0,
-                                        int64_t g, const RowCtx& rc) {
+                                        int64_t g, const RowCtx& rc, const XQuads& xq) {
   const int t = threadIdx.x;
   int32_t* xs = sm.xs[buf];
   if constexpr (!CONV) {
     if constexpr (VEC) {
       // 128 rows x 8 quads of 16 B; consecutive threads take consecutive quads.
+      const bool k_ok = g * kChunk + 4 * (t & 7) < P.kred;
+      const int32_t* src = xq.src + g * kChunk;
+      int32_t* dst = xs + (t >> 3) * XS + 4 * (t & 7);
 #pragma unroll
       for (int i = 0; i < (MT * 8) / THREADS; ++i) {
-        const int piece = t + THREADS * i;
-        const int r = piece >> 3, q = piece & 7;
-        const int64_t row = row0 + r;
-        const int64_t k = g * kChunk + q * 4;
-        const bool ok = (row < P.rows) && (k < P.kred);
-        const int32_t* src = ok ? (P.x + row * P.kred + k) : P.x;
-        cp_async16(xs + r * XS + q * 4, src, ok);
+        const bool ok = k_ok && ((xq.rows_ok >> i) & 1u);
+        cp_async16(dst + 16 * i * XS, ok ? src : P.x, ok);
+        src += xq.row_step;
       }
     } else {
 #pragma unroll 4
@@ -158,8 +179,7 @@ __device__ __forceinline__ void store_codes(Smem& sm, int buf, const CodeRegs& c
   const int t = threadIdx.x;
   const int n = t & (NT - 1);
   const int h = t >> 6;
-  int32_t* shs = sm.shs[buf];
-  int32_t* sgs = sm.sgs[buf];
+  int32_t* cs = sm.cs[buf] + (n >> 5) * 64 + (n & 31);
 #pragma unroll
   for (int i = 0; i < 16; ++i) {
     const int k = 16 * h + i;
@@ -167,8 +187,8 @@ __device__ __forceinline__ void store_codes(Smem& sm, int buf, const CodeRegs& c
     const int sh = (int)((w >> (4 * (i & 7))) & 15u);
     const int neg = (int)((c.bits.x >> k) & 1u);
     const int nz = (int)((c.bits.y >> k) & 1u);
-    shs[k * NT + n] = sh;
-    sgs[k * NT + n] = nz - 2 * neg;
+    cs[k * 2 * NT] = sh;
+    cs[k * 2 * NT + 32] = nz - 2 * neg;
   }
 }
 
@@ -180,8 +200,9 @@ template <int ROW0, int ROWS, typename Acc>
 __device__ __forceinline__ void compute_chunk(const Smem& sm, int buf, int tm, int tn,
                                               Acc (&acc)[ROWS][TN]) {
   const int32_t* xs = sm.xs[buf] + (tm + 16 * ROW0) * XS;
-  const int32_t* shs = sm.shs[buf] + tn * TN;
-  const int32_t* sgs = sm.sgs[buf] + tn * TN;
+  static_assert(32 % TN == 0, "a thread's columns lie in one 32-column block");
+  const int32_t* shs = sm.cs[buf] + ((tn * TN) >> 5) * 64 + ((tn * TN) & 31);
+  const int32_t* sgs = shs + 32;
 #pragma unroll 2
   for (int kq = 0; kq < kChunk / 4; ++kq) {
     int4 xv[ROWS];
@@ -190,10 +211,10 @@ __device__ __forceinline__ void compute_chunk(const Smem& sm, int buf, int tm, i
 #pragma unroll
     for (int kk = 0; kk < 4; ++kk) {
       const int k = 4 * kq + kk;
-      const int4 s0 = *reinterpret_cast<const int4*>(shs + k * NT);
-      const int4 s1 = *reinterpret_cast<const int4*>(shs + k * NT + 4);
-      const int4 g0 = *reinterpret_cast<const int4*>(sgs + k * NT);
-      const int4 g1 = *reinterpret_cast<const int4*>(sgs + k * NT + 4);
+      const int4 s0 = *reinterpret_cast<const int4*>(shs + k * 2 * NT);
+      const int4 s1 = *reinterpret_cast<const int4*>(shs + k * 2 * NT + 4);
+      const int4 g0 = *reinterpret_cast<const int4*>(sgs + k * 2 * NT);
+      const int4 g1 = *reinterpret_cast<const int4*>(sgs + k * 2 * NT + 4);
       const int sh[TN] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
       const int sg[TN] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
       // column-outer order: consecutive SHF / IMAD share their shift / sign operand
@@ -230,10 +251,21 @@ __device__ __forceinline__ void run_tile(const GemmParams& P, Smem& sm, int64_t 
     for (int j = 0; j < TN; ++j) acc[i][j] = 0;
 
   const int64_t nch = P.n_chunks;
+  // codes: the expanded layout is copied with cp.async next to x (two 16-index
+  // halves per chunk); else decoded from the blob through registers, loaded
+  // before the compute and stored after it
+  const bool expanded = P.xcodes != nullptr;
+  static_assert(THREADS == 128 && NT == 64 && kChunk == 32, "ExpandedCodeStager's stage shape, twice per chunk");
+  const ExpandedCodeStager cst(P.xcodes, P.cols, P.kred, col0, 0);
+  const XQuads xq = x_quads(P, row0);
   // prologue: chunk 0 into stage 0
-  stage_x<CONV, VEC>(P, sm, 0, row0, 0, rc);
+  stage_x<CONV, VEC>(P, sm, 0, row0, 0, rc, xq);
+  if (expanded) {
+    cst.stage(P.xcodes, P.kred, sm.cs[0], 0);
+    cst.stage(P.xcodes, P.kred, sm.cs[0] + 16 * 2 * NT, 1);
+  }
   cp_async_commit();
-  {
+  if (!expanded) {
     CodeRegs c0 = load_codes(P, col0, 0);
     store_codes(sm, 0, c0);
   }
@@ -242,16 +274,20 @@ __device__ __forceinline__ void run_tile(const GemmParams& P, Smem& sm, int64_t 
     const bool more = (g + 1 < nch);
     CodeRegs cn;
     if (more) {
-      stage_x<CONV, VEC>(P, sm, buf ^ 1, row0, g + 1, rc);
+      stage_x<CONV, VEC>(P, sm, buf ^ 1, row0, g + 1, rc, xq);
+      if (expanded) {
+        cst.stage(P.xcodes, P.kred, sm.cs[buf ^ 1], (int)(2 * g + 2));
+        cst.stage(P.xcodes, P.kred, sm.cs[buf ^ 1] + 16 * 2 * NT, (int)(2 * g + 3));
+      }
       cp_async_commit();
-      cn = load_codes(P, col0, g + 1);
+      if (!expanded) cn = load_codes(P, col0, g + 1);
       cp_async_wait<1>();
     } else {
       cp_async_wait<0>();
     }
     __syncthreads();
     compute_chunk<ROW0, ROWS, Acc>(sm, buf, tm, tn, acc);
-    if (more) store_codes(sm, buf ^ 1, cn);
+    if (more && !expanded) store_codes(sm, buf ^ 1, cn);
     __syncthreads();
   }
 
