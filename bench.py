@@ -175,7 +175,9 @@ def oracle_conv_sample(wl, n_images: int, seed: int):
     return dt, terms
 
 
-def cpu_baseline(wl, n_images: int = 16):
+def cpu_baseline(wl, n_images: int | None = None):
+    """The oracle on the whole batch (about 10 s on one core), or on n_images of it."""
+    n_images = wl["N"] if n_images is None else n_images
     dt, terms = oracle_conv_sample(wl, n_images, si.SEED_BASE + 2)
     return {"value": terms / dt / 1e9, "unit": METRIC, "cores": 1, "kind": "oracle",
             "sample": f"{n_images} of {wl['N']} images of the same layer (numpy int64 oracle, 1 thread), "
