@@ -33,6 +33,7 @@ ALG_INT_OPS_PER_TERM = 2      # one shift + one add/subtract per term (Fig. 1a: 
 # DRAM bytes (read + write) of one conv_direct_kernel<1,3,7,0> launch on this workload, from one ncu capture
 # of the current kernel (dram__bytes_read.sum + dram__bytes_write.sum); y stays in L2 at kernel end.
 NCU_TRAFFIC_BYTES = 26.13e6
+E2E_CHUNKS = 4  # chunks of the batch in the end-to-end measurement
 
 
 def workload_conv2x(batch: int):
@@ -552,16 +553,32 @@ def run_gpu(args, wl, rank, world, local_rank):
     kern_ms = float(np.mean([a.elapsed_time(b) for a, b in evs]))
     ms_total, kern_ms = reduce_max_over_ranks([ms_total, kern_ms], dev)
 
-    # end to end through the public API with host buffers
+    # End to end through the public API with host buffers: every step copies
+    # the batch in from pinned host memory, runs the layer and copies the
+    # result back.  The images are independent, so the batch goes as E2E_CHUNKS
+    # chunks, each on a stream of its own (its copy in, ds_conv2d_shift with
+    # its own max|x| slot, its copy out, in that order), and one chunk's copies
+    # overlap the others' compute.
     xh = torch.from_numpy(x).pin_memory()
     yh = torch.empty((N, K, H, W), dtype=torch.int32).pin_memory()
     xd, yd = xs[0], ys[0]
-    a = amax_io[0:2]
+    nch = E2E_CHUNKS if N % E2E_CHUNKS == 0 else 1
+    nb = N // nch
+    cstreams = [torch.cuda.Stream(device=dev) for _ in range(nch)]
+    camax = torch.zeros((nch, 2), dtype=torch.int32, device=dev)
 
     def e2e_step():
-        xd.copy_(xh, non_blocking=True)
-        ds.ds_conv2d_shift(xd, w.desc, bd, None, yd, N, C, H, W, K, R, S, 1, 1, 1, 1, 0, a, st)
-        yh.copy_(yd, non_blocking=True)
+        for j, cs in enumerate(cstreams):
+            with torch.cuda.stream(cs):
+                lo, hi = j * nb, (j + 1) * nb
+                xd[lo:hi].copy_(xh[lo:hi], non_blocking=True)
+                ds.ds_conv2d_shift(xd[lo:hi], w.desc, bd, None, yd[lo:hi], nb, C, H, W, K, R, S, 1, 1, 1, 1, 0,
+                                   camax[j], cs.cuda_stream)
+                yh[lo:hi].copy_(yd[lo:hi], non_blocking=True)
+
+    def join():  # the timing stream waits for every chunk stream
+        for cs in cstreams:
+            stream.wait_stream(cs)
 
     for _ in range(max(1, args.warmup)):
         e2e_step()
@@ -571,12 +588,20 @@ def run_gpu(args, wl, rank, world, local_rank):
     if dist:
         dist.barrier()
     e0.record(stream)
+    for cs in cstreams:
+        cs.wait_stream(stream)  # no chunk starts before e0
     for _ in range(args.steps):
         e2e_step()
+    join()
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1)
     e2e_ms = reduce_max_over_ranks([e2e_ms], dev)[0]
+    # the host copy of the last step's result, checked on its first image
+    e2e_parity = None
+    if rank == 0:
+        from oracle import deepshift_oracle as O
+        e2e_parity = bool(np.array_equal(yh[0:1].numpy(), O.conv2d_shift(x[0:1], s, p, b, (1, 1), (1, 1))))
 
     # parity spot check of the timed output (whole-tensor parity lives in tests/)
     if rank == 0:
@@ -613,7 +638,8 @@ def run_gpu(args, wl, rank, world, local_rank):
                          "hbm_gbs": alg_bytes / (kern_ms / 1e3) / 1e9,
                          "hbm_frac": alg_bytes / (kern_ms / 1e3) / 1e9 / float(peaks.get("hbm_gbs", 6800.0))},
             "e2e": {"value": wl["terms"] * args.steps * world / (e2e_ms / 1e3) / 1e9, "unit": METRIC,
-                    "h2d_bytes_per_step": int(x.nbytes), "d2h_bytes_per_step": int(x.nbytes // C * K)},
+                    "h2d_bytes_per_step": int(x.nbytes), "d2h_bytes_per_step": int(x.nbytes // C * K),
+                    "pipeline": f"{nch} chunks of {nb} images, one stream each", "parity_spot_check": e2e_parity},
             "gpu_launches": 2 * args.steps,
             "clocks": clocks,
             "parity_spot_check": parity,
