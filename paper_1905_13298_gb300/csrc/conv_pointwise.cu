@@ -44,23 +44,6 @@ struct __align__(16) PwSmem {
   int32_t cs[2][KC * 2 * NT];  // per input channel: NB blocks of {32 shifts, 32 signs}
 };
 
-__device__ __forceinline__ void cp_async4(void* smem_dst, const void* gsrc, bool valid) {
-  const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
-  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(d), "l"(gsrc), "r"(valid ? 4 : 0));
-}
-__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gsrc, bool valid) {
-  const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(gsrc), "r"(valid ? 16 : 0));
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
-__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::); }
-__device__ __forceinline__ int32_t add_sat(int32_t a, int32_t b) {
-  int32_t r;
-  asm("add.sat.s32 %0, %1, %2;\n" : "=r"(r) : "r"(a), "r"(b));
-  return r;
-}
-__device__ __forceinline__ uint32_t uabs(int32_t v) { return v < 0 ? (uint32_t)0 - (uint32_t)v : (uint32_t)v; }
-
 // This thread's staging assignment: pixel quad q = t % 32 of the tile, input
 // channels t / 32 + 4 j.  Input offsets of the quad's 4 pixels (channel 0).
 struct QuadCtx {

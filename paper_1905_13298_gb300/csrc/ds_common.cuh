@@ -143,6 +143,36 @@ __host__ __device__ inline int64_t expanded_words(int64_t n_out, int64_t k_red) 
 }
 
 #ifdef __CUDACC__
+// Asynchronous global -> shared copies of 4, 8 or 16 bytes; valid = false
+// zero-fills the destination (source size 0).  4 and 8 bytes go through L1,
+// 16 bytes bypass it.
+__device__ __forceinline__ void cp_async4(void* smem_dst, const void* gsrc, bool valid) {
+  const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(d), "l"(gsrc), "r"(valid ? 4 : 0));
+}
+__device__ __forceinline__ void cp_async8(void* smem_dst, const void* gsrc, bool valid) {
+  const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;\n" ::"r"(d), "l"(gsrc), "r"(valid ? 8 : 0));
+}
+__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gsrc, bool valid) {
+  const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(gsrc), "r"(valid ? 16 : 0));
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
+// Wait until at most N of this thread's committed copy groups are in flight.
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;\n" ::"n"(N));
+}
+__device__ __forceinline__ void cp_async_wait_all() { cp_async_wait<0>(); }
+// Saturating int32 addition (the residual join) and |v| as an unsigned value.
+__device__ __forceinline__ int32_t add_sat(int32_t a, int32_t b) {
+  int32_t r;
+  asm("add.sat.s32 %0, %1, %2;\n" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+__device__ __forceinline__ uint32_t uabs(int32_t v) { return v < 0 ? (uint32_t)0 - (uint32_t)v : (uint32_t)v; }
+
 // Staging of the expanded codes of 64 columns (two 32-column blocks) and 16
 // reduction indices per stage, by 128 threads: the stage is 512 16-byte
 // pieces, and thread t copies the pieces at index kl = t / 16 and kl + 8 of

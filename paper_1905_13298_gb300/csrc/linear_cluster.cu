@@ -66,14 +66,6 @@ struct ClSmem {
   };
 };
 
-__device__ __forceinline__ void cp_async4(void* smem_dst, const void* gsrc, bool valid) {
-  const uint32_t d = (uint32_t)__cvta_generic_to_shared(smem_dst);
-  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(d), "l"(gsrc), "r"(valid ? 4 : 0));
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
-__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::); }
-__device__ __forceinline__ uint32_t uabs(int32_t v) { return v < 0 ? (uint32_t)0 - (uint32_t)v : (uint32_t)v; }
-
 // x rows [row0, row0 + MR), reduction indices [k0, k0 + 16) clipped to kend
 // (the end of this CTA's slice); zero elsewhere.  Piece e of a stage (e =
 // threadIdx.x + THREADS u) is 4 consecutive k of one row: row e / 4, k0 +
@@ -131,7 +123,6 @@ struct XStager {
     }
   }
 };
-
 
 // Blob path: the stage starting at k0 (a multiple of 16) is half (k0 / 16) % 2
 // of packed chunk k0 / 32.  Thread t decodes 8 indices of column t % 64

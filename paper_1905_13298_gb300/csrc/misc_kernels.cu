@@ -125,9 +125,6 @@ cudaError_t launch_expand(const uint8_t* blob, int64_t n_out, int64_t k_red, int
 
 // max |x| (as u32, |INT32_MIN| = 2^31).  Grid-stride over 16-byte vectors,
 // warp reduction, one atomicMax per warp.  The target is zeroed first.
-__device__ __forceinline__ uint32_t uabs32(int32_t v) {
-  return v < 0 ? (uint32_t)0 - (uint32_t)v : (uint32_t)v;
-}
 
 __global__ void absmax_kernel(const int32_t* __restrict__ x, int64_t n, uint32_t* out) {
   uint32_t m = 0;
@@ -142,18 +139,18 @@ __global__ void absmax_kernel(const int32_t* __restrict__ x, int64_t n, uint32_t
     for (; i + 3 * stride < nv; i += 4 * stride) {
       const int4 a = __ldg(xv + i), b = __ldg(xv + i + stride);
       const int4 c = __ldg(xv + i + 2 * stride), d = __ldg(xv + i + 3 * stride);
-      m = max(m, max(max(uabs32(a.x), uabs32(a.y)), max(uabs32(a.z), uabs32(a.w))));
-      m = max(m, max(max(uabs32(b.x), uabs32(b.y)), max(uabs32(b.z), uabs32(b.w))));
-      m = max(m, max(max(uabs32(c.x), uabs32(c.y)), max(uabs32(c.z), uabs32(c.w))));
-      m = max(m, max(max(uabs32(d.x), uabs32(d.y)), max(uabs32(d.z), uabs32(d.w))));
+      m = max(m, max(max(uabs(a.x), uabs(a.y)), max(uabs(a.z), uabs(a.w))));
+      m = max(m, max(max(uabs(b.x), uabs(b.y)), max(uabs(b.z), uabs(b.w))));
+      m = max(m, max(max(uabs(c.x), uabs(c.y)), max(uabs(c.z), uabs(c.w))));
+      m = max(m, max(max(uabs(d.x), uabs(d.y)), max(uabs(d.z), uabs(d.w))));
     }
     for (; i < nv; i += stride) {
       const int4 a = __ldg(xv + i);
-      m = max(m, max(max(uabs32(a.x), uabs32(a.y)), max(uabs32(a.z), uabs32(a.w))));
+      m = max(m, max(max(uabs(a.x), uabs(a.y)), max(uabs(a.z), uabs(a.w))));
     }
-    for (int64_t j = (nv << 2) + tid; j < n; j += stride) m = max(m, uabs32(x[j]));
+    for (int64_t j = (nv << 2) + tid; j < n; j += stride) m = max(m, uabs(x[j]));
   } else {
-    for (int64_t i = tid; i < n; i += stride) m = max(m, uabs32(x[i]));
+    for (int64_t i = tid; i < n; i += stride) m = max(m, uabs(x[i]));
   }
   // block reduction, then one atomic per block
   __shared__ uint32_t wmax[32];
@@ -170,9 +167,17 @@ __global__ void absmax_kernel(const int32_t* __restrict__ x, int64_t n, uint32_t
 cudaError_t launch_absmax(const int32_t* x, int64_t n, uint32_t* out, cudaStream_t st) {
   cudaError_t e = cudaMemsetAsync(out, 0, sizeof(uint32_t), st);
   if (e != cudaSuccess) return e;
-  int dev = 0, sms = 152;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  // the SM count, read once per process (thread-safe function-local static)
+  static const int sms = [] {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) !=
+                                                  cudaSuccess) {
+      (void)cudaGetLastError();
+      return 0;
+    }
+    return n;
+  }();
+  if (sms <= 0) return cudaErrorInvalidDevice;
   const int threads = 256;
   int64_t want = (n / 16 + threads - 1) / threads;
   int64_t blocks = want < (int64_t)sms * 4 ? want : (int64_t)sms * 4;
