@@ -1,0 +1,31 @@
+"""Host logic of bench.py that decides whether a timing is kept: the clock
+summary (throttle reasons must be reported) and the workload bookkeeping."""
+import bench
+
+
+def test_clock_summary_reports_throttling():
+    lines = [
+        "0, 2070, 2070, 900.5, 0x0000000000000000, Not Active, Not Active, Not Active, Not Active",
+        "0, 1995, 2070, 1390.0, 0x0000000000000004, Not Active, Not Active, Not Active, Active",
+        "0, 2070, 2070, 1010.2, 0x0000000000000000, Not Active, Active, Not Active, Not Active",
+        "garbage line",
+        "0, [N/A], 2070, 0, 0x0, Not Active, Not Active, Not Active, Not Active",
+    ]
+    s = bench.ClockSampler.summarize(lines)
+    assert s["samples"] == 3
+    assert s["sm_mhz"] == 2070.0 and s["sm_max_mhz"] == 2070.0
+    assert s["reasons"] == ["hw_thermal_slowdown", "sw_power_cap"]
+
+
+def test_clock_summary_clean_and_empty():
+    clean = ["0, 2070, 2070, 800, 0x0, Not Active, Not Active, Not Active, Not Active"] * 4
+    assert bench.ClockSampler.summarize(clean) == {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": [],
+                                                    "samples": 4}
+    assert bench.ClockSampler.summarize([])["sm_mhz"] is None
+
+
+def test_default_workload_is_the_conv2x_layer():
+    wl = bench.workload_by_name("conv2x", None)
+    assert (wl["N"], wl["C"], wl["H"], wl["W"], wl["K"], wl["R"], wl["S"]) == (32, 64, 56, 56, 64, 3, 3)
+    assert wl["terms"] == 32 * 64 * 56 * 56 * 64 * 9 == 3_699_376_128
+    assert 32 % bench.E2E_CHUNKS == 0
