@@ -20,9 +20,13 @@ ResNet: stem; then per block conv1, conv2 (, conv3 for bottleneck) and the
 downsample conv if the block has one; then the FC.  VGG16: the 13 convs,
 then the 3 FCs.
 
-parity unpinned beyond composition: the chain is checked only through its
-pinned parts (conv, FC, pools, residual join) and one library special case
-(tests/test_oracle_pins.py::test_resnet_chain_matches_float64_library_case).
+Pins: the chain is built only from pinned parts (conv, FC, pools, residual
+join), and the whole chain of each network equals a float64 composition of
+library routines (torch conv2d, max_pool2d, avg_pool2d + floor, linear) on a
+special case where every term is exact: one non-zero code per output channel
+with p = 0 (tests/test_oracle_pins.py, *_chain_matches_float64_library_case,
+ResNet18, ResNet50 and VGG16 on 32 x 32 images).  A wrong stride, padding,
+pool, shortcut, ReLU placement or layer order changes that result.
 """
 from __future__ import annotations
 
@@ -77,7 +81,7 @@ def resnet_forward(x, params, arch: str = "resnet18"):
 
 
 def vgg16_forward(x, params):
-    """Forward of an all-shift VGG16; x int32 [N, 3, 224, 224]; returns int32 [N, 1000]."""
+    """Forward of an all-shift VGG16; x int32 [N, 3, H, W] (224 x 224 in the workloads); returns int32 [N, 1000]."""
     it = iter(params)
     for v in VGG16_CFG:
         if v == "M":

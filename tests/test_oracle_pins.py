@@ -492,6 +492,41 @@ def test_resnet_chain_matches_float64_library_case(arch, kind, blocks):
     assert np.array_equal(got.astype(np.float64), want)
 
 
+def _torch_vgg16(x, params):
+    """float64 torch restatement (library conv2d / max_pool2d / linear) of VGG16 (configuration D)."""
+    t = lambda a: torch.from_numpy(np.asarray(a, dtype=np.float64))
+    it = iter(params)
+    v = t(x)
+    for c in (64, 64, "M", 128, 128, "M", 256, 256, 256, "M", 512, 512, 512, "M", 512, 512, 512, "M"):
+        if c == "M":
+            v = F.max_pool2d(v, 2, 2)
+        else:
+            s, p, b = next(it)
+            v = F.relu(F.conv2d(v, t(s * np.ldexp(1.0, p)), t(b), stride=1, padding=1))
+    v = v.reshape(v.shape[0], -1)
+    for i in range(3):
+        s, p, b = next(it)
+        w = s.reshape(s.shape[0], -1) * np.ldexp(1.0, p.reshape(p.shape[0], -1))
+        v = F.linear(v, t(w), t(b))
+        if i < 2:
+            v = F.relu(v)
+    return v
+
+
+def test_vgg16_chain_matches_float64_library_case():
+    """VGG16 (32 x 32 input, so the first FC has 512 inputs): one-hot codes with p = 0 make every
+    term exact, so the oracle's chain equals the float64 library composition exactly."""
+    from oracle import networks as ON
+    from paper_1905_13298_gb300 import networks as PN   # layer shapes only (no library call)
+    _, shapes = PN.vgg16_program(32, 32)
+    params = _one_hot_params(shapes, 4)
+    x = si.image_batch(6, 2, 3, 32, 32)
+    got = ON.vgg16_forward(x, params)
+    want = _torch_vgg16(x, params).numpy()
+    assert np.abs(want).max() < 2 ** 31
+    assert np.array_equal(got.astype(np.float64), want)
+
+
 def test_bf16_weight_bits_decode_to_s_times_power_of_two():
     """bf16 patterns of the float variant's weights decode (via float32 bit casts) to s * 2^p exactly."""
     s = np.array([[1, -1, 0, 1], [-1, 1, 1, 0]])
