@@ -1,0 +1,153 @@
+"""Mistakes planted in the oracle, on the CPU, must fail the pins.
+
+Each case replaces one oracle function by a copy with one plausible mistake
+(a truncating shift, the flip before the shift, a dropped term, no bias, no
+saturation, a left shift, a true convolution instead of cross-correlation, a
+truncating average, a swapped nibble, a wrong column constant, a wrong term
+sign) and runs the pins of tests/test_oracle_pins.py until one fails.  A
+mistake that no pin catches fails this test.  The unmutated oracle passes every
+pin (test_oracle_pins.py itself).
+"""
+import numpy as np
+import pytest
+
+import test_oracle_pins as pins
+from oracle import deepshift_oracle as O
+
+_ORIG = {name: getattr(O, name) for name in ("linear_shift_acc", "conv2d_shift_acc", "sat32", "avgpool_floor",
+                                              "pack_planes6", "column_constants", "term", "shift")}
+
+# the pins to run, cheapest first (parametrized pins with their first case)
+_PINS = [
+    pins.test_term_golden_cases,
+    pins.test_linear_golden_cases,
+    pins.test_conv_golden_cases,
+    pins.test_avgpool_floor_golden_and_library,
+    pins.test_pack_golden_tiny_blob,
+    pins.test_column_constants_closed_forms,
+    pins.test_linear_saturation_boundaries,
+    pins.test_linear_trivial_weights,
+    pins.test_linear_negation_invariance,
+    pins.test_linear_exact_float64_when_x_multiple_of_2_15,
+    pins.test_linear_ternary_p0_is_int_matmul,
+    pins.test_term_exhaustive_codes_vs_rational_floor_and_bit_strings,
+    pins.test_linear_brute_force_tiny,
+    pins.test_conv_identity_and_sampled_elements,
+    pins.test_conv_negation_invariance,
+    lambda: pins.test_conv_exact_float64_when_x_multiple_of_2_15((2, 3, 7, 6, 4, 3, 3, 1, 1, 1, 1)),
+    lambda: pins.test_conv_equals_im2col_plus_linear((2, 3, 6, 5, 4, 3, 3, 1, 1, 1, 1)),
+]
+
+
+def _linear_acc(rule, drop_last=False, use_bias=True):
+    """LinearShift accumulator with the per-term rule rule(x_col, s_col, p_col) -> [M, N] terms."""
+    def acc_fn(x, s, p, b=None):
+        x = np.asarray(x, dtype=np.int64)
+        s = np.asarray(s, dtype=np.int64)
+        p = np.asarray(p, dtype=np.int64)
+        M, K = x.shape
+        acc = np.zeros((M, s.shape[0]), dtype=np.int64)
+        if b is not None and use_bias:
+            acc += np.asarray(b, dtype=np.int64)[None, :]
+        for k in range(K - 1 if drop_last and K > 1 else K):
+            acc += rule(x[:, k][:, None], s[:, k][None, :], p[:, k][None, :])
+        return acc
+    return acc_fn
+
+
+def _floor_rule(x, s, p):
+    return s * np.floor_divide(x, np.left_shift(np.int64(1), -p))
+
+
+def _trunc_rule(x, s, p):  # division rounding toward zero
+    d = np.left_shift(np.int64(1), -p)
+    return s * (np.sign(x) * (np.abs(x) // d))
+
+
+def _flip_first_rule(x, s, p):  # (s * x) >> -p
+    return np.floor_divide(s * x, np.left_shift(np.int64(1), -p))
+
+
+def _left_shift_rule(x, s, p):  # x << -p
+    return s * (x * np.left_shift(np.int64(1), -p))
+
+
+def _true_convolution(x, s, p, b=None, stride=(1, 1), pad=(0, 0)):
+    s = np.asarray(s)[:, :, ::-1, ::-1]
+    p = np.asarray(p)[:, :, ::-1, ::-1]
+    return _ORIG["conv2d_shift_acc"](x, s, p, b, stride, pad)
+
+
+def _conv_without_bias(x, s, p, b=None, stride=(1, 1), pad=(0, 0)):
+    return _ORIG["conv2d_shift_acc"](x, s, p, None, stride, pad)
+
+
+def _trunc_average(x, k, stride):
+    x = np.asarray(x, dtype=np.int64)
+    N, C, H, W = x.shape
+    OH, OW = (H - k) // stride + 1, (W - k) // stride + 1
+    out = np.zeros((N, C, OH, OW), dtype=np.int64)
+    for oh in range(OH):
+        for ow in range(OW):
+            sm = x[:, :, oh * stride:oh * stride + k, ow * stride:ow * stride + k].sum(axis=(2, 3))
+            out[:, :, oh, ow] = np.sign(sm) * (np.abs(sm) // (k * k))
+    return out.astype(np.int32)
+
+
+def _swapped_nibbles(s, p):
+    blob = _ORIG["pack_planes6"](s, p).copy()
+    L = O.blob_layout(*np.shape(s))
+    nib = blob[L["nib"]:L["bits"]]
+    blob[L["nib"]:L["bits"]] = ((nib & 0x0F) << 4) | (nib >> 4)  # the two nibbles of each byte swapped
+    return blob
+
+
+def _wrong_column_a(s, p):
+    A, nnz = _ORIG["column_constants"](s, p)
+    s2 = np.asarray(s, dtype=np.int64).reshape(np.shape(s)[0], -1)
+    p2 = np.asarray(p, dtype=np.int64).reshape(np.shape(p)[0], -1)
+    A = (np.abs(s2) * np.left_shift(np.int64(1), 14 + p2)).sum(axis=1)  # 2^(14 + p) instead of 2^(15 + p)
+    return A.astype(np.int64), nnz
+
+
+MUTANTS = {  # each case patches exactly one oracle function
+    "truncating shift (term)": {"shift": lambda x, p: int(np.sign(x)) * (abs(x) >> (-p))},
+    "truncating shift (LinearShift)": {"linear_shift_acc": _linear_acc(_trunc_rule)},
+    "flip before shift (term)": {"term": lambda x, s, p: (s * x) // (1 << (-p))},
+    "flip before shift (LinearShift)": {"linear_shift_acc": _linear_acc(_flip_first_rule)},
+    "left shift (term)": {"shift": lambda x, p: x << (-p)},
+    "left shift (LinearShift)": {"linear_shift_acc": _linear_acc(_left_shift_rule)},
+    "wrong term sign (term)": {"term": lambda x, s, p: -s * (x // (1 << (-p)))},
+    "wrong term sign (LinearShift)": {"linear_shift_acc": _linear_acc(lambda x, s, p: -_floor_rule(x, s, p))},
+    "dropped term (LinearShift)": {"linear_shift_acc": _linear_acc(_floor_rule, drop_last=True)},
+    "no bias (LinearShift)": {"linear_shift_acc": _linear_acc(_floor_rule, use_bias=False)},
+    "no bias (ConvShift)": {"conv2d_shift_acc": _conv_without_bias},
+    "true convolution (ConvShift)": {"conv2d_shift_acc": _true_convolution},
+    "no saturation": {"sat32": lambda v: np.asarray(v)},
+    "truncating average": {"avgpool_floor": _trunc_average},
+    "swapped nibbles (packing)": {"pack_planes6": _swapped_nibbles},
+    "wrong column constant": {"column_constants": _wrong_column_a},
+}
+
+
+@pytest.mark.parametrize("name", list(MUTANTS))
+def test_planted_mistake_is_caught(name, monkeypatch):
+    for fn_name, fn in MUTANTS[name].items():
+        monkeypatch.setattr(O, fn_name, fn)
+    caught = []
+    for pin in _PINS:
+        try:
+            pin()
+        except (AssertionError, ValueError, IndexError) as e:
+            caught.append((getattr(pin, "__name__", "pin"), type(e).__name__))
+            break
+    assert caught, f"no pin caught the planted mistake: {name}"
+
+
+def test_control_correct_rewrite_passes_every_pin(monkeypatch):
+    """The harness itself: a correct restatement put in through the same plumbing fails no pin."""
+    monkeypatch.setattr(O, "linear_shift_acc", _linear_acc(_floor_rule))
+    monkeypatch.setattr(O, "conv2d_shift_acc", lambda x, s, p, b=None, stride=(1, 1), pad=(0, 0):
+                        _ORIG["conv2d_shift_acc"](x, s, p, b, stride, pad))
+    for pin in _PINS:
+        pin()
