@@ -4,7 +4,8 @@ Each case replaces one oracle function by a copy with one plausible mistake
 (a truncating shift, the flip before the shift, a dropped term, no bias, no
 saturation, a left shift, a true convolution instead of cross-correlation, a
 truncating average, a swapped nibble, a wrong column constant, a wrong term
-sign) and runs the pins of tests/test_oracle_pins.py until one fails.  A
+sign, a quantizer that floors log2|W|, a truncating Q16.16 conversion, an
+input gradient without the rot180 or with the flip first) and runs the pins of tests/test_oracle_pins.py until one fails.  A
 mistake that no pin catches fails this test.  The unmutated oracle passes every
 pin (test_oracle_pins.py itself).
 """
@@ -15,7 +16,9 @@ import test_oracle_pins as pins
 from oracle import deepshift_oracle as O
 
 _ORIG = {name: getattr(O, name) for name in ("linear_shift_acc", "conv2d_shift_acc", "sat32", "avgpool_floor",
-                                              "pack_planes6", "column_constants", "term", "shift")}
+                                              "pack_planes6", "column_constants", "term", "shift",
+                                              "quantize_weights", "quantize_activations",
+                                              "conv2d_shift_backward_x_acc", "linear_shift_backward_x_acc")}
 
 # the pins to run, cheapest first (parametrized pins with their first case)
 _PINS = [
@@ -36,6 +39,15 @@ _PINS = [
     pins.test_conv_negation_invariance,
     lambda: pins.test_conv_exact_float64_when_x_multiple_of_2_15((2, 3, 7, 6, 4, 3, 3, 1, 1, 1, 1)),
     lambda: pins.test_conv_equals_im2col_plus_linear((2, 3, 6, 5, 4, 3, 3, 1, 1, 1, 1)),
+    pins.test_quantize_weights_powers_of_two_are_fixed_points,
+    pins.test_quantize_weights_against_exact_rationals,
+    pins.test_quantize_activations_ties_saturation_and_specials,
+    pins.test_quantize_activations_against_exact_rationals_and_torch_round,
+    pins.test_linear_backward_x_equals_float64_matmul_on_exact_inputs,
+    lambda: pins.test_conv_backward_x_equals_float64_autograd_on_exact_inputs(pins.BWD_GEOMS[0]),
+    lambda: pins.test_conv_backward_x_equals_float64_autograd_on_exact_inputs(pins.BWD_GEOMS[1]),
+    pins.test_linear_backward_x_is_forward_with_transposed_codes,
+    lambda: pins.test_conv_backward_x_brute_force_gather_with_floor(pins.BWD_GEOMS[0]),
 ]
 
 
@@ -110,7 +122,42 @@ def _wrong_column_a(s, p):
     return A.astype(np.int64), nnz
 
 
+def _floor_log2_quantizer(W, p_min=O.P_MIN):  # floor(log2|W|) instead of round
+    s, p = _ORIG["quantize_weights"](W, p_min)
+    w = np.abs(np.asarray(W, dtype=np.float32).astype(np.float64))
+    ok = np.isfinite(w) & (w > 0)
+    _, e = np.frexp(np.where(ok, w, 1.0))
+    p2 = np.where(ok, np.clip(e.astype(np.int64) - 1, p_min, 0), p)
+    return s, p2.astype(np.int8)
+
+
+def _truncating_q16(x):  # x * 2^16 truncated toward zero instead of rounded half to even
+    y = np.asarray(x, dtype=np.float32).astype(np.float64) * 65536.0
+    y = np.where(np.isnan(y), 0.0, np.trunc(y))
+    return np.clip(y, O.INT32_MIN, O.INT32_MAX).astype(np.int64).astype(np.int32)
+
+
+def _backward_without_rot180(dy, s, p, in_hw, stride=(1, 1), pad=(0, 0)):
+    s = np.asarray(s)[:, :, ::-1, ::-1]
+    p = np.asarray(p)[:, :, ::-1, ::-1]
+    return _ORIG["conv2d_shift_backward_x_acc"](dy, s, p, in_hw, stride, pad)
+
+
+def _linear_backward_flip_first(dy, s, p):  # (s * dy) >> -p
+    dy = np.asarray(dy, dtype=np.int64)
+    s = np.asarray(s, dtype=np.int64)
+    p = np.asarray(p, dtype=np.int64)
+    acc = np.zeros((dy.shape[0], s.shape[1]), dtype=np.int64)
+    for n in range(s.shape[0]):
+        acc += np.floor_divide(s[n][None, :] * dy[:, n][:, None], np.left_shift(np.int64(1), -p[n])[None, :])
+    return acc
+
+
 MUTANTS = {  # each case patches exactly one oracle function
+    "quantizer floors log2": {"quantize_weights": _floor_log2_quantizer},
+    "Q16.16 truncates": {"quantize_activations": _truncating_q16},
+    "input gradient without rot180": {"conv2d_shift_backward_x_acc": _backward_without_rot180},
+    "input gradient flips first (FC)": {"linear_shift_backward_x_acc": _linear_backward_flip_first},
     "truncating shift (term)": {"shift": lambda x, p: int(np.sign(x)) * (abs(x) >> (-p))},
     "truncating shift (LinearShift)": {"linear_shift_acc": _linear_acc(_trunc_rule)},
     "flip before shift (term)": {"term": lambda x, s, p: (s * x) // (1 << (-p))},
