@@ -49,6 +49,14 @@ typedef enum {
   DS_ERR_CUDA = 7              /* a CUDA runtime call or launch failed */
 } ds_status;
 
+/* Size limits.  Every size the library forms from caller dimensions is
+ * bounded before it can overflow 64 bits.  A code matrix holds at most 2^48
+ * codes, with n_out <= 2^31 and k_red <= 2^40 (2^36 for the expanded and
+ * bf16 layouts); a tensor holds at most 2^62 bytes; a zero-padded image
+ * extent (H + 2 pad) is at most 2^31 - 1; one convolution image has at most
+ * 2^31 input values (C x H x W) and 2^30 output positions (OH x OW).  Larger
+ * dimensions give DS_ERR_UNSUPPORTED, and 0 from the size queries. */
+
 /* Description of the last error on the calling thread ("" if none). */
 const char* ds_last_error(void);
 

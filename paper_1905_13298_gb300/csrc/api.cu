@@ -3,6 +3,7 @@
 #include <stdarg.h>
 #include <stdio.h>
 
+#include <initializer_list>
 #include <string>
 
 #include "ds_common.cuh"
@@ -39,6 +40,57 @@ ds_status cuda_check(cudaError_t e, const char* what) {
 
 static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
+// Byte size of an int32 tensor with the given positive extents, or -1 when it
+// exceeds 2^62 bytes: no buffer is that large, and the bound keeps every
+// element offset the kernels form inside int64.
+static int64_t int32_tensor_bytes(std::initializer_list<int64_t> dims) {
+  int64_t n = sizeof(int32_t);
+  for (int64_t d : dims)
+    if (d <= 0 || __builtin_mul_overflow(n, d, &n) || n > (int64_t(1) << 62)) return -1;
+  return n;
+}
+
+// A code matrix is accepted when n_out <= 2^31, k_red <= k_max and it holds
+// at most 2^48 codes, which keeps every size derived from it (packed,
+// expanded, bf16) far inside 64 bits.
+static bool code_matrix_in_range(int64_t n_out, int64_t k_red, int64_t k_max) {
+  return n_out > 0 && k_red > 0 && n_out <= (int64_t(1) << 31) && k_red <= k_max &&
+         k_red <= (int64_t(1) << 48) / n_out;
+}
+
+// True when the byte ranges [a, a + na) and [b, b + nb) intersect.  The ends
+// are formed as integers, so no pointer is moved past its buffer.
+static bool ranges_overlap(const void* a, int64_t na, const void* b, int64_t nb) {
+  const uintptr_t ua = reinterpret_cast<uintptr_t>(a), ub = reinterpret_cast<uintptr_t>(b);
+  return ua < ub + static_cast<uintptr_t>(nb) && ub < ua + static_cast<uintptr_t>(na);
+}
+
+// Output size of a window (convolution or pooling) over a zero-padded image,
+// formed in 64 bits: positive extents and strides, non-negative pads, a
+// window no larger than the padded image, and a padded extent within int32.
+ds_status window_output(int H, int W, int R, int S, int stride_h, int stride_w, int pad_h, int pad_w, int* OH,
+                        int* OW) {
+  if (H <= 0 || W <= 0 || R <= 0 || S <= 0) return fail(DS_ERR_SHAPE, "H, W, R and S must be positive");
+  if (stride_h <= 0 || stride_w <= 0 || pad_h < 0 || pad_w < 0)
+    return fail(DS_ERR_SHAPE, "strides must be positive and pads non-negative");
+  const int64_t hp = (int64_t)H + 2 * (int64_t)pad_h, wp = (int64_t)W + 2 * (int64_t)pad_w;
+  if (hp < R || wp < S) return fail(DS_ERR_SHAPE, "kernel larger than padded input");
+  if (hp > INT32_MAX || wp > INT32_MAX) return fail(DS_ERR_UNSUPPORTED, "padded input larger than 2^31 - 1");
+  *OH = (int)((hp - R) / stride_h + 1);
+  *OW = (int)((wp - S) / stride_w + 1);
+  return DS_OK;
+}
+
+// Per-image limits of the convolution and pooling kernels, which index
+// within one image in 32 bits: C x H x W <= 2^31 inputs, OH x OW <= 2^30
+// outputs per plane.
+ds_status check_image(int C, int H, int W, int OH, int OW) {
+  const int64_t xb = int32_tensor_bytes({C, H, W});
+  if (xb < 0 || xb > (int64_t(4) << 31) || (int64_t)OH * OW > (int64_t)1 << 30)
+    return fail(DS_ERR_UNSUPPORTED, "image too large");
+  return DS_OK;
+}
+
 // Checks a descriptor filled by ds_pack_shift_weights against the call's dims.
 ds_status check_weights(const ds_weights* w, int64_t n_out, int64_t k_red) {
   if (w == nullptr) return fail(DS_ERR_INVALID_ARG, "weights descriptor is NULL");
@@ -48,6 +100,9 @@ ds_status check_weights(const ds_weights* w, int64_t n_out, int64_t k_red) {
   if (w->n_out != n_out || w->k_red != k_red)
     return fail(DS_ERR_SHAPE, "weights are %lld x %lld, call needs %lld x %lld", (long long)w->n_out,
                 (long long)w->k_red, (long long)n_out, (long long)k_red);
+  if (ds_packed_weight_bytes(n_out, k_red) == 0)
+    return fail(DS_ERR_UNSUPPORTED, "a %lld x %lld code matrix is outside the supported range", (long long)n_out,
+                (long long)k_red);
   const BlobLayout L = blob_layout(n_out, k_red);
   if (w->n_chunks != L.n_chunks || w->packed_bytes < (size_t)L.total)
     return fail(DS_ERR_INVALID_ARG, "weights descriptor is inconsistent with its dims");
@@ -187,8 +242,7 @@ size_t ds_abi_struct_size(int which) {
 }
 
 size_t ds_packed_weight_bytes(int64_t n_out, int64_t k_red) {
-  if (n_out <= 0 || k_red <= 0) return 0;
-  if (n_out > (int64_t(1) << 31) || k_red > (int64_t(1) << 40)) return 0;
+  if (!code_matrix_in_range(n_out, k_red, int64_t(1) << 40)) return 0;
   return (size_t)blob_layout(n_out, k_red).total;
 }
 
@@ -296,8 +350,7 @@ ds_status ds_pack_shift_weights_backward(const int8_t* s, const int8_t* p, int K
 }
 
 size_t ds_expanded_weight_bytes(int64_t n_out, int64_t k_red) {
-  if (n_out <= 0 || k_red <= 0) return 0;
-  if (n_out > (int64_t(1) << 31) || k_red > (int64_t(1) << 36)) return 0;
+  if (!code_matrix_in_range(n_out, k_red, int64_t(1) << 36)) return 0;
   return (size_t)expanded_words(n_out, k_red) * sizeof(int32_t);
 }
 
@@ -321,8 +374,7 @@ ds_status ds_expand_shift_weights(ds_weights* w, void* expanded, size_t expanded
 }
 
 size_t ds_bf16_weight_bytes(int64_t n_out, int64_t k_red) {
-  if (n_out <= 0 || k_red <= 0) return 0;
-  if (n_out > (int64_t(1) << 31) || k_red > (int64_t(1) << 36)) return 0;
+  if (!code_matrix_in_range(n_out, k_red, int64_t(1) << 36)) return 0;
   return (size_t)(n_out * bf16_kpad(k_red) * 2 + 255) / 256 * 256;
 }
 
@@ -382,13 +434,13 @@ ds_status ds_conv2d_shift_backward_x(const int32_t* dy, const ds_weights* w_bwd,
     return fail(DS_ERR_SHAPE, "N, C, H, W, K, R, S must be positive");
   if (stride_h <= 0 || stride_w <= 0 || stride_h > 16 || stride_w > 16 || pad_h < 0 || pad_w < 0)
     return fail(DS_ERR_SHAPE, "strides must be in [1, 16] and pads non-negative");
-  if (H + 2 * pad_h < R || W + 2 * pad_w < S) return fail(DS_ERR_SHAPE, "kernel larger than padded input");
+  int OH = 0, OW = 0;
+  ds_status rg = window_output(H, W, R, S, stride_h, stride_w, pad_h, pad_w, &OH, &OW);
+  if (rg != DS_OK) return rg;
   if (flags & ~(DS_AMAX_IN | DS_AMAX_OUT | DS_FORCE_INT64 | DS_CONV_IM2COL))
     return fail(DS_ERR_INVALID_ARG, "only DS_AMAX_IN, DS_AMAX_OUT, DS_FORCE_INT64, DS_CONV_IM2COL apply here");
   if ((flags & (DS_AMAX_IN | DS_AMAX_OUT)) && amax_io == nullptr)
     return fail(DS_ERR_INVALID_ARG, "DS_AMAX_IN / DS_AMAX_OUT need amax_io");
-  const int OH = (H + 2 * pad_h - R) / stride_h + 1;
-  const int OW = (W + 2 * pad_w - S) / stride_w + 1;
   // one descriptor per tap phase (a, b), as ds_pack_shift_weights_backward fills them
   bool empty_phase = false;
   for (int a = 0; a < stride_h; ++a)
@@ -409,19 +461,19 @@ ds_status ds_conv2d_shift_backward_x(const int32_t* dy, const ds_weights* w_bwd,
     return ds_conv2d_shift(dy, w_bwd, nullptr, nullptr, dx, N, K, OH, OW, C, R, S, 1, 1, R - 1 - pad_h,
                            S - 1 - pad_w, flags, amax_io, stream);
   if (!aligned16(dy) || !aligned16(dx)) return fail(DS_ERR_ALIGNMENT, "dy and dx must be 16-byte aligned");
-  const int64_t ny = (int64_t)N * K * OH * OW, nx = (int64_t)N * C * H * W;
-  const char* ya = reinterpret_cast<const char*>(dy);
-  const char* xa = reinterpret_cast<const char*>(dx);
-  if (xa < ya + ny * 4 && ya < xa + nx * 4) return fail(DS_ERR_INVALID_ARG, "dx must not overlap dy");
-  if ((int64_t)H * W > (int64_t)1 << 30 || (int64_t)K * OH * OW > (int64_t)1 << 31)
-    return fail(DS_ERR_UNSUPPORTED, "image too large");
+  // dY is this pass's input image (K x OH x OW) and dX its output plane (H x W)
+  ds_status ri = check_image(K, OH, OW, H, W);
+  if (ri != DS_OK) return ri;
+  const int64_t yb = int32_tensor_bytes({N, K, OH, OW}), xb = int32_tensor_bytes({N, C, H, W});
+  if (xb < 0 || yb < 0) return fail(DS_ERR_UNSUPPORTED, "dx or dy larger than 2^62 bytes");
+  if (ranges_overlap(dx, xb, dy, yb)) return fail(DS_ERR_INVALID_ARG, "dx must not overlap dy");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   GemmParams base{};
   base.flags = flags & ~DS_CONV_IM2COL;
-  ds_status r = prepare_amax(dy, ny, flags, amax_io, st, base);
+  ds_status r = prepare_amax(dy, yb / (int64_t)sizeof(int32_t), flags, amax_io, st, base);
   if (r != DS_OK) return r;
   if (empty_phase) {
-    r = cuda_check(cudaMemsetAsync(dx, 0, (size_t)nx * sizeof(int32_t), st), "dx reset");
+    r = cuda_check(cudaMemsetAsync(dx, 0, (size_t)xb, st), "dx reset");
     if (r != DS_OK) return r;
   }
   // output phase (rh, rw): dX rows rh, rh + sh, ...; they receive the taps r = a + sh t with
@@ -504,10 +556,9 @@ ds_status ds_linear_shift(const int32_t* x, const ds_weights* w, const int32_t* 
   if (!aligned16(x) || !aligned16(y)) return fail(DS_ERR_ALIGNMENT, "x and y must be 16-byte aligned");
   ds_status r = check_weights(w, N, K);
   if (r != DS_OK) return r;
-  const int64_t xb = M * K * 4, yb = M * N * 4;
-  const char* xa = reinterpret_cast<const char*>(x);
-  const char* ya = reinterpret_cast<const char*>(y);
-  if (xa < ya + yb && ya < xa + xb) return fail(DS_ERR_INVALID_ARG, "y must not overlap x");
+  const int64_t xb = int32_tensor_bytes({M, K}), yb = int32_tensor_bytes({M, N});
+  if (xb < 0 || yb < 0) return fail(DS_ERR_UNSUPPORTED, "x or y larger than 2^62 bytes");
+  if (ranges_overlap(x, xb, y, yb)) return fail(DS_ERR_INVALID_ARG, "y must not overlap x");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   GemmParams p{};
   p.x = x;
@@ -532,27 +583,23 @@ ds_status ds_conv2d_shift(const int32_t* x, const ds_weights* w, const int32_t* 
   if (!x || !y) return fail(DS_ERR_INVALID_ARG, "NULL x or y");
   if (N <= 0 || C <= 0 || H <= 0 || W <= 0 || K <= 0 || R <= 0 || S <= 0)
     return fail(DS_ERR_SHAPE, "N, C, H, W, K, R, S must be positive");
-  if (stride_h <= 0 || stride_w <= 0 || pad_h < 0 || pad_w < 0)
-    return fail(DS_ERR_SHAPE, "strides must be positive and pads non-negative");
-  if (H + 2 * pad_h < R || W + 2 * pad_w < S) return fail(DS_ERR_SHAPE, "kernel larger than padded input");
+  int OH = 0, OW = 0;
+  ds_status r = window_output(H, W, R, S, stride_h, stride_w, pad_h, pad_w, &OH, &OW);
+  if (r != DS_OK) return r;
   if (flags & ~kKnownFlags) return fail(DS_ERR_INVALID_ARG, "unknown flag bits 0x%x", flags & ~kKnownFlags);
   if ((flags & DS_RESIDUAL) && residual == nullptr)
     return fail(DS_ERR_INVALID_ARG, "DS_RESIDUAL needs a residual tensor");
   if ((flags & (DS_AMAX_IN | DS_AMAX_OUT)) && amax_io == nullptr)
     return fail(DS_ERR_INVALID_ARG, "DS_AMAX_IN / DS_AMAX_OUT need amax_io");
   if (!aligned16(x) || !aligned16(y)) return fail(DS_ERR_ALIGNMENT, "x and y must be 16-byte aligned");
-  const int OH = (H + 2 * pad_h - R) / stride_h + 1;
-  const int OW = (W + 2 * pad_w - S) / stride_w + 1;
   const int64_t kred = (int64_t)C * R * S;
-  ds_status r = check_weights(w, K, kred);
+  r = check_weights(w, K, kred);
   if (r != DS_OK) return r;
-  const int64_t nx = (int64_t)N * C * H * W;
-  const int64_t ny = (int64_t)N * K * OH * OW;
-  const char* xa = reinterpret_cast<const char*>(x);
-  const char* ya = reinterpret_cast<const char*>(y);
-  if (xa < ya + ny * 4 && ya < xa + nx * 4) return fail(DS_ERR_INVALID_ARG, "y must not overlap x");
-  if ((int64_t)OH * OW > (int64_t)1 << 30 || (int64_t)C * H * W > (int64_t)1 << 31)
-    return fail(DS_ERR_UNSUPPORTED, "image too large");
+  r = check_image(C, H, W, OH, OW);
+  if (r != DS_OK) return r;
+  const int64_t xb = int32_tensor_bytes({N, C, H, W}), yb = int32_tensor_bytes({N, K, OH, OW});
+  if (xb < 0 || yb < 0) return fail(DS_ERR_UNSUPPORTED, "x or y larger than 2^62 bytes");
+  if (ranges_overlap(x, xb, y, yb)) return fail(DS_ERR_INVALID_ARG, "y must not overlap x");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   GemmParams p{};
   p.x = x;
@@ -575,7 +622,7 @@ ds_status ds_conv2d_shift(const int32_t* x, const ds_weights* w, const int32_t* 
   p.OH = OH;
   p.OW = OW;
   fill_blob_offsets(p, w);
-  r = prepare_amax(x, nx, flags, amax_io, st, p);
+  r = prepare_amax(x, xb / (int64_t)sizeof(int32_t), flags, amax_io, st, p);
   if (r != DS_OK) return r;
   if (!(flags & DS_CONV_IM2COL)) {
     if (conv_pointwise_supported(p))

@@ -118,6 +118,9 @@ cudaError_t launch_avgpool_floor(const int32_t* x, int32_t* y, int64_t planes, i
                                  int R, int S, int stride, cudaStream_t st);
 // Defined in api.cu: launches after validation, with explicit amax slots.
 ds_status check_weights(const ds_weights* w, int64_t n_out, int64_t k_red);
+ds_status window_output(int H, int W, int R, int S, int stride_h, int stride_w, int pad_h, int pad_w, int* OH,
+                        int* OW);
+ds_status check_image(int C, int H, int W, int OH, int OW);
 ds_status conv_launch(const int32_t* x, const ds_weights* w, const int32_t* bias, const int32_t* residual,
                       int32_t* y, int N, int C, int H, int W, int K, int R, int S, int stride, int pad,
                       uint32_t flags, const uint32_t* amax_in, uint32_t* amax_out, cudaStream_t st,

@@ -9,6 +9,7 @@
 // floor-average never exceed it) and writes max|y| into its own word, so the
 // accumulator-width proof of every layer happens on the device.
 #include <algorithm>
+#include <string>
 #include <vector>
 
 #include "ds_common.cuh"
@@ -31,6 +32,12 @@ struct Plan {
   int n_slots = 0;
 };
 
+// Re-raises a failed check with the layer's index in front of its message.
+ds_status layer_fail(ds_status st, int i) {
+  const std::string what = ds_last_error();
+  return fail(st, "layer %d: %s", i, what.c_str());
+}
+
 ds_status plan_program(const ds_layer* L, int n, int batch, Plan& P) {
   if (L == nullptr || n <= 0) return fail(DS_ERR_INVALID_ARG, "empty layer program");
   if (batch <= 0) return fail(DS_ERR_SHAPE, "batch must be positive");
@@ -46,6 +53,8 @@ ds_status plan_program(const ds_layer* L, int n, int batch, Plan& P) {
   std::vector<bool> defined(P.n_slots, false);
   P.slot_elems.assign(P.n_slots, 0);
   P.out_shape.assign(n, Shape{});
+  if (L[0].C <= 0 || L[0].H <= 0 || L[0].W <= 0) return fail(DS_ERR_SHAPE, "input image must have positive C, H, W");
+  if (check_image(L[0].C, L[0].H, L[0].W, 1, 1) != DS_OK) return fail(DS_ERR_UNSUPPORTED, "input image too large");
   slot[0] = Shape{L[0].C, L[0].H, L[0].W};
   defined[0] = true;
   bool wrote_y = false;
@@ -62,10 +71,13 @@ ds_status plan_program(const ds_layer* L, int n, int batch, Plan& P) {
                       in.H, in.W);
         if (l.K <= 0 || l.R <= 0 || l.S <= 0 || l.stride <= 0 || l.pad < 0)
           return fail(DS_ERR_SHAPE, "layer %d: bad conv geometry", i);
-        if (l.H + 2 * l.pad < l.R || l.W + 2 * l.pad < l.S) return fail(DS_ERR_SHAPE, "layer %d: kernel too big", i);
-        ds_status r = check_weights(l.w, l.K, (int64_t)l.C * l.R * l.S);
+        int oh = 0, ow = 0;
+        ds_status r = window_output(l.H, l.W, l.R, l.S, l.stride, l.stride, l.pad, l.pad, &oh, &ow);
+        if (r == DS_OK) r = check_image(l.C, l.H, l.W, oh, ow);
+        if (r != DS_OK) return layer_fail(r, i);
+        r = check_weights(l.w, l.K, (int64_t)l.C * l.R * l.S);
         if (r != DS_OK) return r;
-        out = Shape{l.K, (l.H + 2 * l.pad - l.R) / l.stride + 1, (l.W + 2 * l.pad - l.S) / l.stride + 1};
+        out = Shape{l.K, oh, ow};
         P.split_bytes = std::max(P.split_bytes,
                                  conv_split_bytes(conv_params(l.w, batch, l.C, l.H, l.W, l.K, l.R, l.S, l.stride, l.pad)));
         break;
@@ -75,6 +87,7 @@ ds_status plan_program(const ds_layer* L, int n, int batch, Plan& P) {
           return fail(DS_ERR_SHAPE, "layer %d: FC input of %lld features, slot holds %lld", i,
                       (long long)((int64_t)l.C * l.H * l.W), (long long)in.elems());
         if (l.K <= 0) return fail(DS_ERR_SHAPE, "layer %d: bad FC width", i);
+        if (l.K > 65535LL * 64) return fail(DS_ERR_UNSUPPORTED, "layer %d: FC wider than 65535 x 64", i);
         if (l.flags & DS_RESIDUAL) return fail(DS_ERR_INVALID_ARG, "layer %d: residual on FC", i);
         ds_status r = check_weights(l.w, l.K, in.elems());
         if (r != DS_OK) return r;
@@ -88,9 +101,12 @@ ds_status plan_program(const ds_layer* L, int n, int batch, Plan& P) {
         if (l.op == DS_OP_AVGPOOL && l.pad != 0) return fail(DS_ERR_UNSUPPORTED, "layer %d: padded avgpool", i);
         if (l.R <= 0 || l.S <= 0 || l.stride <= 0 || pad < 0 || pad >= l.R || pad >= l.S)
           return fail(DS_ERR_SHAPE, "layer %d: bad pool geometry", i);
-        if (l.H + 2 * pad < l.R || l.W + 2 * pad < l.S) return fail(DS_ERR_SHAPE, "layer %d: window too big", i);
+        int oh = 0, ow = 0;
+        ds_status r = window_output(l.H, l.W, l.R, l.S, l.stride, l.stride, pad, pad, &oh, &ow);
+        if (r == DS_OK) r = check_image(1, l.H, l.W, oh, ow);  // the pools index one plane at a time
+        if (r != DS_OK) return layer_fail(r, i);
         if (l.flags != 0) return fail(DS_ERR_INVALID_ARG, "layer %d: flags on a pool", i);
-        out = Shape{l.C, (l.H + 2 * pad - l.R) / l.stride + 1, (l.W + 2 * pad - l.S) / l.stride + 1};
+        out = Shape{l.C, oh, ow};
         break;
       }
       default:
@@ -116,7 +132,12 @@ ds_status plan_program(const ds_layer* L, int n, int batch, Plan& P) {
   size_t off = P.amax_bytes + P.split_bytes;
   for (int s = 2; s < P.n_slots; ++s) {
     P.slot_off[s] = off;
-    off += ((size_t)P.slot_elems[s] * batch * sizeof(int32_t) + 255) / 256 * 256;
+    int64_t bytes = 0;
+    if (__builtin_mul_overflow(P.slot_elems[s], (int64_t)batch * (int64_t)sizeof(int32_t), &bytes) ||
+        bytes > (int64_t(1) << 62))
+      return fail(DS_ERR_UNSUPPORTED, "slot %d larger than 2^62 bytes", s);
+    off += ((size_t)bytes + 255) / 256 * 256;
+    if (off > (size_t(1) << 62)) return fail(DS_ERR_UNSUPPORTED, "workspace larger than 2^62 bytes");
   }
   P.total = off;
   return DS_OK;

@@ -129,6 +129,88 @@ def test_validation_happens_before_cuda(ds):
     assert L.ds_quantize_q16(16, 4, 34, None) == ds.DS_ERR_ALIGNMENT
 
 
+def _descriptor(ds, n_out, k_red):
+    """A descriptor that passes the host checks for an (n_out, k_red) code matrix (its blob is never read)."""
+    return ds.ds_weights(magic=ds.DS_WEIGHTS_MAGIC, format=ds.DS_FORMAT_PLANES6, n_out=n_out, k_red=k_red,
+                         n_chunks=(k_red + 31) // 32, packed=256, packed_bytes=ds.ds_packed_weight_bytes(n_out, k_red))
+
+
+def test_size_arithmetic_never_wraps(ds):
+    """Sizes formed from caller dimensions are bounded before they can overflow 64 bits: absurd dimensions give
+    a status, never a wrapped size or a check done on wrapped numbers."""
+    L = ds.lib()
+    # size queries: each dimension in range but the product too large gives 0, not a wrapped size
+    assert ds.ds_packed_weight_bytes(1 << 20, 1 << 28) > 0            # 2^48 codes: the largest accepted
+    assert ds.ds_packed_weight_bytes(1 << 20, (1 << 28) + 1) == 0
+    assert ds.ds_packed_weight_bytes(1 << 31, 1 << 40) == 0
+    assert ds.ds_expanded_weight_bytes(1 << 31, 1 << 36) == 0
+    assert ds.ds_bf16_weight_bytes(1 << 31, 1 << 36) == 0
+    assert ds.ds_expanded_weight_bytes(64, 1024) == 2 * 1024 * 64 * 4
+    # a forged descriptor outside the range is refused before its layout is computed
+    n_big = 65535 * 64                                                 # the widest FC layer accepted
+    big = ds.ds_weights(magic=ds.DS_WEIGHTS_MAGIC, format=ds.DS_FORMAT_PLANES6, n_out=n_big, k_red=1 << 40,
+                        n_chunks=1 << 35, packed=256, packed_bytes=(1 << 64) - 1)
+    assert L.ds_linear_shift(16, ctypes.byref(big), None, 4096, 1, 1 << 40, n_big, 0, None,
+                             None) == ds.DS_ERR_UNSUPPORTED
+    assert "supported range" in ds.ds_last_error()
+    # FC: M x K x 4 bytes = 2^72 would wrap to 0
+    w = _descriptor(ds, 1, 1 << 30)
+    assert L.ds_linear_shift(16, ctypes.byref(w), None, 1 << 48, 1 << 40, 1 << 30, 1, 0, None,
+                             None) == ds.DS_ERR_UNSUPPORTED
+    assert "2^62" in ds.ds_last_error()
+    # conv: 2 x pad overflows int32; the padded extent is formed in 64 bits
+    w1 = _descriptor(ds, 1, 9)
+    for pad in ((1 << 30) + 5, (1 << 31) - 1):
+        assert L.ds_conv2d_shift(16, ctypes.byref(w1), None, None, 1 << 40, 1, 1, 8, 8, 1, 3, 3, 1, 1, pad, 0, 0,
+                                 None, None) == ds.DS_ERR_UNSUPPORTED
+        assert "padded" in ds.ds_last_error()
+        assert L.ds_conv2d_shift_backward_x(16, ctypes.byref(w1), 1 << 40, 1, 1, 8, 8, 1, 3, 3, 2, 2, pad, 0, 0,
+                                            None, None) == ds.DS_ERR_UNSUPPORTED
+    # conv: an image past the kernels' 32-bit per-image indexing, and a batch past 2^62 bytes
+    wc = _descriptor(ds, 1, (1 << 31) - 1)
+    assert L.ds_conv2d_shift(16, ctypes.byref(wc), None, None, 1 << 40, 1, (1 << 31) - 1, 2, 2, 1, 1, 1, 1, 1, 0,
+                             0, 0, None, None) == ds.DS_ERR_UNSUPPORTED
+    assert "image too large" in ds.ds_last_error()
+    wk = _descriptor(ds, 1 << 16, 16)
+    assert L.ds_conv2d_shift(16, ctypes.byref(wk), None, None, 1 << 40, (1 << 31) - 1, 16, 1 << 7, 1 << 7, 1 << 16,
+                             1, 1, 1, 1, 0, 0, 0, None, None) == ds.DS_ERR_UNSUPPORTED
+    assert "2^62" in ds.ds_last_error()
+
+
+def test_program_size_arithmetic_never_wraps(ds):
+    """The layer-program planner applies the same bounds: the padded extent, the per-image limits and the
+    workspace size are checked without overflow, and the failing layer is named."""
+    L = ds.lib()
+
+    def program(pad=0, K=4, H=32, batch=2):
+        w = _descriptor(ds, K, 1)
+        layers = (ds.ds_layer * 2)()
+        conv, pool = layers[0], layers[1]
+        conv.op, conv.in_, conv.aux, conv.out = ds.DS_OP_CONV, 0, -1, 2
+        conv.C, conv.H, conv.W, conv.K, conv.R, conv.S, conv.stride, conv.pad = 1, H, H, K, 1, 1, 1, pad
+        conv.w = ctypes.pointer(w)
+        OH = H + 2 * pad if pad < (1 << 20) else 1  # the conv is refused before the pool is looked at
+        pool.op, pool.in_, pool.aux, pool.out = ds.DS_OP_MAXPOOL, 2, -1, 1
+        pool.C, pool.H, pool.W, pool.K, pool.R, pool.S, pool.stride, pool.pad = K, OH, OH, 0, 1, 1, 1, 0
+        return layers, batch, w
+
+    layers, batch, _w = program()
+    assert ds.ds_shift_forward_workspace_bytes(layers, 2, batch) > 2 * 4 * 32 * 32 * 4
+    layers, batch, _w = program(pad=(1 << 30) + 5)
+    assert ds.ds_shift_forward_workspace_bytes(layers, 2, batch) == 0
+    assert ds.ds_last_error().startswith("layer 0:") and "padded" in ds.ds_last_error()
+    # 2^16 channels of 2^20 outputs per image is 2^38 bytes; 2^24 images of that pass 2^62
+    layers, batch, _w = program(K=1 << 16, H=1 << 10, batch=1 << 24)
+    assert ds.ds_shift_forward_workspace_bytes(layers, 2, batch) == 0
+    assert "2^62" in ds.ds_last_error()
+    layers, batch, _w = program(K=1 << 16, H=1 << 10, batch=1 << 10)
+    assert ds.ds_shift_forward_workspace_bytes(layers, 2, batch) >= (1 << 48)
+    # the network input itself: non-positive or past the per-image limit
+    layers, batch, _w = program(H=1 << 16)
+    assert ds.ds_shift_forward_workspace_bytes(layers, 2, batch) == 0
+    assert "too large" in ds.ds_last_error()
+
+
 def test_no_cpu_fallback_without_library(tmp_path, monkeypatch, ds):
     """The binding refuses to run when the shared library is missing."""
     monkeypatch.setattr(ds, "_lib", None)
