@@ -2,10 +2,15 @@
 
 Each case replaces one oracle function by a copy with one plausible mistake
 (a truncating shift, the flip before the shift, a dropped term, no bias, no
-saturation, a left shift, a true convolution instead of cross-correlation, a
-truncating average, a swapped nibble, a wrong column constant, a wrong term
-sign, a quantizer that floors log2|W|, a truncating Q16.16 conversion, an
-input gradient without the rot180 or with the flip first) and runs the pins of tests/test_oracle_pins.py until one fails.  A
+saturation or a saturation before the bias, a left shift, a true convolution
+instead of cross-correlation, a truncating average, a max-pool that pads with
+zeros, a residual join with the ReLU first or with wraparound, a swapped
+nibble, a wrong column constant, a wrong term sign, a quantizer that floors
+log2|W| or rounds in the linear domain, a truncating Q16.16 conversion or one
+with ties away from zero, an input gradient without the rot180 or with the
+flip first, sampled-element and layout helpers with one slip each, an int32
+bound that drops a term, a ResNet block joined after its ReLU) and runs the
+pins of tests/test_oracle_pins.py until one fails.  A
 mistake that no pin catches fails this test.  The unmutated oracle passes every
 pin (test_oracle_pins.py itself).
 """
@@ -14,11 +19,15 @@ import pytest
 
 import test_oracle_pins as pins
 from oracle import deepshift_oracle as O
+from oracle import networks as ON
 
 _ORIG = {name: getattr(O, name) for name in ("linear_shift_acc", "conv2d_shift_acc", "sat32", "avgpool_floor",
                                               "pack_planes6", "column_constants", "term", "shift",
                                               "quantize_weights", "quantize_activations",
-                                              "conv2d_shift_backward_x_acc", "linear_shift_backward_x_acc")}
+                                              "conv2d_shift_backward_x_acc", "linear_shift_backward_x_acc",
+                                              "maxpool2d", "conv2d_shift_at", "linear_shift_at",
+                                              "int32_accumulation_is_exact", "expand_codes", "weights_bf16_bits",
+                                              "unpack_planes6", "backward_codes", "backward_phase_codes")}
 
 # the pins to run, cheapest first (parametrized pins with their first case)
 _PINS = [
@@ -48,6 +57,15 @@ _PINS = [
     lambda: pins.test_conv_backward_x_equals_float64_autograd_on_exact_inputs(pins.BWD_GEOMS[1]),
     pins.test_linear_backward_x_is_forward_with_transposed_codes,
     lambda: pins.test_conv_backward_x_brute_force_gather_with_floor(pins.BWD_GEOMS[0]),
+    pins.test_maxpool_golden_and_library,
+    pins.test_add_relu_golden,
+    pins.test_accumulation_bound_is_sound_at_the_int32_edge,
+    pins.test_expand_layout_closed_form,
+    pins.test_bf16_weight_bits_decode_to_s_times_power_of_two,
+    pins.test_pack_round_trip_and_sizes,
+    lambda: pins.test_conv_backward_x_stride1_is_forward_conv_with_rot180_codes(pins.BWD_GEOMS[0]),
+    lambda: pins.test_conv_backward_x_phase_decomposition(pins.BWD_GEOMS[1]),
+    lambda: pins.test_resnet_chain_matches_float64_library_case("resnet18", "basic", [2, 2, 2, 2]),
 ]
 
 
@@ -153,7 +171,101 @@ def _linear_backward_flip_first(dy, s, p):  # (s * dy) >> -p
     return acc
 
 
-MUTANTS = {  # each case patches exactly one oracle function
+def _maxpool_zero_padding(x, k, stride, pad):  # padded taps read as 0 instead of being ignored
+    x = np.pad(np.asarray(x, dtype=np.int64), ((0, 0), (0, 0), (pad, pad), (pad, pad)))
+    return _ORIG["maxpool2d"](x, k, stride, 0)
+
+
+def _relu_before_join(a, b):  # ReLU(a) + b, nothing after the join
+    return O.sat32(np.maximum(np.asarray(a, np.int64), 0) + np.asarray(b, np.int64)).astype(np.int32)
+
+
+def _wrapping_join(a, b):  # int32 wraparound instead of saturation
+    v = (np.asarray(a, np.int64) + np.asarray(b, np.int64) + (1 << 31)) % (1 << 32) - (1 << 31)
+    return np.maximum(v, 0).astype(np.int32)
+
+
+def _saturate_before_bias(x, s, p, b=None, relu=False):  # sat32(sat32(sum) + b) instead of one saturation
+    y = np.asarray(O.sat32(O.linear_shift_acc(x, s, p, None)), np.int64)
+    if b is not None:
+        y = O.sat32(y + np.asarray(b, np.int64)[None, :])
+    y = np.maximum(y, 0) if relu else y
+    return np.asarray(y).astype(np.int32)
+
+
+def _quantizer_rounds_linearly(W, p_min=O.P_MIN):  # nearest power of two by |W - 2^n|, not round(log2|W|)
+    s, p = _ORIG["quantize_weights"](W, p_min)
+    w = np.abs(np.asarray(W, dtype=np.float32).astype(np.float64))
+    ok = np.isfinite(w) & (w > 0)
+    m, e = np.frexp(np.where(ok, w, 1.0))  # w between 2^(e-1) and 2^e; their midpoint is at m = 3/4
+    p2 = np.where(ok, np.clip(e.astype(np.int64) - 1 + (m >= 0.75), p_min, 0), p)
+    return s, p2.astype(np.int8)
+
+
+def _q16_ties_away(x):  # ties rounded away from zero instead of to even
+    y = np.asarray(x, dtype=np.float32).astype(np.float64) * 65536.0
+    y = np.where(np.isnan(y), 0.0, np.sign(y) * np.floor(np.abs(y) + 0.5))
+    return np.clip(y, O.INT32_MIN, O.INT32_MAX).astype(np.int64).astype(np.int32)
+
+
+def _expand_halves_swapped(s, p):  # signs in words 0..31, shifts in 32..63
+    e = _ORIG["expand_codes"](s, p)
+    return np.ascontiguousarray(np.concatenate([e[..., 32:], e[..., :32]], axis=-1))
+
+
+def _bf16_exponent_off_by_one(s, p):  # exponent 128 + p
+    bits = _ORIG["weights_bf16_bits"](s, p).astype(np.int64)
+    return np.where(bits != 0, bits + (1 << 7), 0).astype(np.uint16)
+
+
+def _unpack_without_sign_plane(blob, n_out, k_red):
+    s, p = _ORIG["unpack_planes6"](blob, n_out, k_red)
+    return np.abs(s).astype(np.int8), p
+
+
+def _backward_codes_without_rot180(s, p):  # channels swapped, taps not rotated
+    sb, pb = _ORIG["backward_codes"](s, p)
+    return np.ascontiguousarray(sb[:, :, ::-1, ::-1]), np.ascontiguousarray(pb[:, :, ::-1, ::-1])
+
+
+def _phase_codes_without_rot180(s, p, stride):
+    out = _ORIG["backward_phase_codes"](s, p, stride)
+    return {key: None if v is None else tuple(np.ascontiguousarray(a[:, :, ::-1, ::-1]) for a in v)
+            for key, v in out.items()}
+
+
+def _join_after_relu(x, prm, stride, pad, relu, residual=None):  # ReLU on the branch, then a plain join
+    s, p, b = prm
+    y = O.conv2d_shift(x, s, p, b, (stride, stride), (pad, pad), relu=relu or residual is not None)
+    if residual is not None:
+        return O.sat32(y.astype(np.int64) + np.asarray(residual, np.int64)).astype(np.int32)
+    return y
+
+
+MUTANTS = {  # each case patches exactly one oracle function ("networks." names one in oracle/networks.py)
+    "max-pool pads with zeros": {"maxpool2d": _maxpool_zero_padding},
+    "ReLU before the residual join": {"add_relu": _relu_before_join},
+    "residual join wraps": {"add_relu": _wrapping_join},
+    "saturation before the bias": {"linear_shift": _saturate_before_bias},
+    "sampled conv element shifted by the pad": {
+        "conv2d_shift_at": lambda x, s, p, b, stride, pad, n, k, oh, ow:
+            _ORIG["conv2d_shift_at"](x, s, p, b, stride, (-pad[0], -pad[1]), n, k, oh, ow)},
+    "sampled FC element without bias": {
+        "linear_shift_at": lambda x, s, p, b, m, n: _ORIG["linear_shift_at"](x, s, p, None, m, n)},
+    "int32 bound without nnz": {
+        "int32_accumulation_is_exact": lambda amax, A, nnz, babs:
+            _ORIG["int32_accumulation_is_exact"](amax, A, 0, babs)},
+    "int32 bound without the bias": {
+        "int32_accumulation_is_exact": lambda amax, A, nnz, babs:
+            _ORIG["int32_accumulation_is_exact"](amax, A, nnz, 0)},
+    "quantizer rounds in the linear domain": {"quantize_weights": _quantizer_rounds_linearly},
+    "Q16.16 ties away from zero": {"quantize_activations": _q16_ties_away},
+    "expanded layout halves swapped": {"expand_codes": _expand_halves_swapped},
+    "bf16 exponent off by one": {"weights_bf16_bits": _bf16_exponent_off_by_one},
+    "unpack ignores the sign plane": {"unpack_planes6": _unpack_without_sign_plane},
+    "input-gradient codes without rot180": {"backward_codes": _backward_codes_without_rot180},
+    "phase codes without rot180": {"backward_phase_codes": _phase_codes_without_rot180},
+    "ResNet joins after the ReLU": {"networks._conv": _join_after_relu},
     "quantizer floors log2": {"quantize_weights": _floor_log2_quantizer},
     "Q16.16 truncates": {"quantize_activations": _truncating_q16},
     "input gradient without rot180": {"conv2d_shift_backward_x_acc": _backward_without_rot180},
@@ -180,7 +292,10 @@ MUTANTS = {  # each case patches exactly one oracle function
 @pytest.mark.parametrize("name", list(MUTANTS))
 def test_planted_mistake_is_caught(name, monkeypatch):
     for fn_name, fn in MUTANTS[name].items():
-        monkeypatch.setattr(O, fn_name, fn)
+        if fn_name.startswith("networks."):
+            monkeypatch.setattr(ON, fn_name.split(".", 1)[1], fn)
+        else:
+            monkeypatch.setattr(O, fn_name, fn)
     caught = []
     for pin in _PINS:
         try:

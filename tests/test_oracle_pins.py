@@ -93,7 +93,7 @@ def test_term_rejects_out_of_range_codes():
 # --------------------------------------------------------------------------
 
 def test_linear_golden_cases():
-    for case in ("fc1", "sat1"):
+    for case in ("fc1", "sat1", "sat_bias"):
         g = _golden_layer(case)
         x = np.array([g["x"]], np.int64)
         K = x.shape[1]
@@ -219,6 +219,32 @@ def test_accumulation_bound_holds_and_is_tight():
     # -INT32_MIN with s = -1 does not fit int32: the bound must refuse it
     assert not O.int32_accumulation_is_exact(1 << 31, 1 << 15, 1, 0)
     assert O.int32_accumulation_is_exact((1 << 31) - 2, 1 << 15, 1, 0)
+
+
+def test_accumulation_bound_is_sound_at_the_int32_edge():
+    """Near the int32 edge the bound admits no column whose worst-case sum overflows (reading R-acc).
+
+    The worst case of a column with s = -1 and p = 0, -1, ..., -15 is x = -amax on every term: each term is then
+    ceil(amax / 2^k), and a positive bias adds b.  That sum is written out here with Python ints.  For amax swept
+    across the point where it passes INT32_MAX, the bound may answer True only when the sum fits, and it does
+    answer True a little below the edge, so it is not vacuous.
+    """
+    ks = range(16)
+    s = -np.ones((1, 16), np.int64)
+    p = -np.arange(16)[None, :]
+    A, nnz = O.column_constants(s, p)
+    for babs in (0, 1, 2, 3, 12345, (1 << 20) + 3):   # several positions of the edge
+        def worst(amax):
+            return sum(-(-amax // (1 << k)) for k in ks) + babs
+        lo, hi = 0, 1 << 31             # the largest amax whose worst case fits: worst(lo) <= INT32_MAX < worst(hi)
+        while hi - lo > 1:
+            mid = (lo + hi) // 2
+            lo, hi = (mid, hi) if worst(mid) <= O.INT32_MAX else (lo, mid)
+        answers = {amax: O.int32_accumulation_is_exact(amax, int(A[0]), int(nnz[0]), babs)
+                   for amax in range(lo - 64, lo + 64)}
+        for amax, ok in answers.items():
+            assert not ok or worst(amax) <= O.INT32_MAX, (amax, babs)
+        assert answers[lo - 64]
 
 
 def test_column_constants_closed_forms():
