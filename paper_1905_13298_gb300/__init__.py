@@ -150,6 +150,41 @@ def _ptr(t) -> int | None:
     return t.data_ptr()
 
 
+def _need(t, name: str, dtypes, shape=None, min_numel: int = 0) -> None:
+    """Checks a tensor argument of the tensor-level helpers (None passes).  The C ABI sees only an
+    address, so a tensor of another dtype, a strided view or a wrong shape would be read as something
+    it is not: each is refused here instead."""
+    if t is None:
+        return
+    dtypes = dtypes if isinstance(dtypes, tuple) else (dtypes,)
+    if t.dtype not in dtypes:
+        raise ValueError(f"{name} must be {' or '.join(str(d) for d in dtypes)}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {tuple(shape)}")
+    if t.numel() < min_numel:
+        raise ValueError(f"{name} needs at least {min_numel} elements")
+
+
+def _on_one_gpu(**tensors) -> None:
+    """Every tensor given (None passes) is CUDA memory on the first one's device."""
+    device = None
+    for name, t in tensors.items():
+        if t is None:
+            continue
+        if t.device.type != "cuda":
+            raise ValueError(f"{name} must be a CUDA tensor")
+        device = device or t.device
+        if t.device != device:
+            raise ValueError(f"{name} is on {t.device}, the input on {device}")
+
+
+def _need_amax(amax_io) -> None:
+    import torch
+    _need(amax_io, "amax_io", (torch.int32, torch.uint32), min_numel=2)
+
+
 def _stream(stream) -> int | None:
     if stream is not None:
         return stream if isinstance(stream, int) else stream.cuda_stream
@@ -309,8 +344,14 @@ def expand_shift_weights_bf16(w: PackedShiftWeights, stream=None) -> PackedShift
 def linear_shift_bf16(x, w: PackedShiftWeights, bias=None, relu: bool = False, out=None, stream=None):
     """Float LinearShift: fp32 y = bias + x @ W^T (ReLU) for bf16 x [M, K] on the tensor cores."""
     import torch
+    _need(x, "x", torch.bfloat16)
+    if x.dim() != 2:
+        raise ValueError("x must be [M, K]")
     M, K = x.shape
     N = w.n_out
+    _need(bias, "bias", torch.float32, (N,))
+    _need(out, "out", torch.float32, (M, N))
+    _on_one_gpu(x=x, bias=bias, out=out)
     y = out if out is not None else torch.empty((M, N), dtype=torch.float32, device=x.device)
     ds_linear_shift_bf16(x, w.desc, bias, y, M, K, N, DS_RELU if relu else 0, stream)
     return y
@@ -408,8 +449,15 @@ def linear_shift(x, w: PackedShiftWeights, bias=None, relu: bool = False, amax_i
                  out=None, stream=None):
     """y = sat32(bias + sum s * (x >> -p)) [ReLU] for int32 x [M, K] on the GPU."""
     import torch
+    _need(x, "x", torch.int32)
+    if x.dim() != 2:
+        raise ValueError("x must be [M, K]")
     M, K = x.shape
     N = w.n_out
+    _need(bias, "bias", torch.int32, (N,))
+    _need(out, "out", torch.int32, (M, N))
+    _need_amax(amax_io)
+    _on_one_gpu(x=x, bias=bias, out=out, amax_io=amax_io)
     y = out if out is not None else torch.empty((M, N), dtype=torch.int32, device=x.device)
     ds_linear_shift(x, w.desc, bias, y, M, K, N, flags | (DS_RELU if relu else 0), amax_io, stream)
     return y
@@ -419,11 +467,19 @@ def conv2d_shift(x, w: PackedShiftWeights, kernel_size, bias=None, stride=(1, 1)
                  relu: bool = False, residual=None, amax_io=None, flags: int = 0, out=None, stream=None):
     """ConvShift forward on int32 NCHW x; w packed from OIHW codes."""
     import torch
+    _need(x, "x", torch.int32)
+    if x.dim() != 4:
+        raise ValueError("x must be [N, C, H, W]")
     N, C, H, W = x.shape
     R, S = kernel_size
     K = w.n_out
     OH = (H + 2 * padding[0] - R) // stride[0] + 1
     OW = (W + 2 * padding[1] - S) // stride[1] + 1
+    _need(bias, "bias", torch.int32, (K,))
+    _need(residual, "residual", torch.int32, (N, K, OH, OW))
+    _need(out, "out", torch.int32, (N, K, OH, OW))
+    _need_amax(amax_io)
+    _on_one_gpu(x=x, bias=bias, residual=residual, out=out, amax_io=amax_io)
     y = out if out is not None else torch.empty((N, K, OH, OW), dtype=torch.int32, device=x.device)
     f = flags | (DS_RELU if relu else 0) | (DS_RESIDUAL if residual is not None else 0)
     ds_conv2d_shift(x, w.desc, bias, residual, y, N, C, H, W, K, R, S, stride[0], stride[1], padding[0],

@@ -211,6 +211,39 @@ def test_program_size_arithmetic_never_wraps(ds):
     assert "too large" in ds.ds_last_error()
 
 
+def test_tensor_helpers_refuse_mismatched_tensors(ds):
+    """The tensor-level helpers check dtype, layout, shape and device before the ABI sees an address."""
+    import torch
+    w = ds.PackedShiftWeights(None, _descriptor(ds, 4, 8))
+    x = torch.zeros((3, 8), dtype=torch.int32)
+    i32 = lambda *shape: torch.zeros(shape, dtype=torch.int32)
+    wc = ds.PackedShiftWeights(None, _descriptor(ds, 6, 2 * 3 * 3))
+    xc = i32(1, 2, 5, 5)
+    conv = lambda **kw: ds.conv2d_shift(xc if "x" not in kw else kw.pop("x"), wc, (3, 3), padding=(1, 1), **kw)
+    xb = torch.zeros((3, 8), dtype=torch.bfloat16)
+    cases = [
+        (lambda: ds.linear_shift(x.float(), w), "int32"),
+        (lambda: ds.linear_shift(i32(8, 3).t(), w), "contiguous"),
+        (lambda: ds.linear_shift(x[0], w), "[M, K]"),
+        (lambda: ds.linear_shift(x, w, bias=i32(5)), "shape"),
+        (lambda: ds.linear_shift(x, w, bias=torch.zeros(4, dtype=torch.int64)), "int32"),
+        (lambda: ds.linear_shift(x, w, out=i32(3, 5)), "shape"),
+        (lambda: ds.linear_shift(x, w, amax_io=i32(1)), "at least 2"),
+        (lambda: ds.linear_shift(x, w, bias=i32(4), out=i32(3, 4), amax_io=i32(2)), "CUDA"),
+        (lambda: conv(x=i32(2, 5, 5)), "[N, C, H, W]"),
+        (lambda: conv(bias=i32(5)), "shape"),
+        (lambda: conv(residual=i32(1, 6, 4, 4)), "shape"),
+        (lambda: conv(out=torch.zeros((1, 6, 5, 5), dtype=torch.float32)), "int32"),
+        (lambda: conv(bias=i32(6), residual=i32(1, 6, 5, 5), out=i32(1, 6, 5, 5)), "CUDA"),
+        (lambda: ds.linear_shift_bf16(xb.float(), w), "bfloat16"),
+        (lambda: ds.linear_shift_bf16(xb, w, bias=i32(4)), "float32"),
+        (lambda: ds.linear_shift_bf16(xb, w, bias=torch.zeros(4)), "CUDA"),
+    ]
+    for call, what in cases:
+        with pytest.raises(ValueError, match=re.escape(what)):
+            call()
+
+
 def test_no_cpu_fallback_without_library(tmp_path, monkeypatch, ds):
     """The binding refuses to run when the shared library is missing."""
     monkeypatch.setattr(ds, "_lib", None)
