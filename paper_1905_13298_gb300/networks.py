@@ -11,8 +11,10 @@ import ctypes
 import math
 from dataclasses import dataclass
 
-from . import (DS_OP_AVGPOOL, DS_OP_CONV, DS_OP_FC, DS_OP_MAXPOOL, DS_RELU, DS_RESIDUAL, ds_layer,
-               ds_shift_forward, ds_shift_forward_workspace_bytes, pack_shift_weights)
+import numpy as np
+
+from . import (DS_OP_AVGPOOL, DS_OP_CONV, DS_OP_FC, DS_OP_MAXPOOL, DS_RELU, DS_RESIDUAL, _need, _on_one_gpu,
+               ds_last_error, ds_layer, ds_shift_forward, ds_shift_forward_workspace_bytes, pack_shift_weights)
 
 
 @dataclass
@@ -176,10 +178,15 @@ class ShiftNetwork:
         self.batch = batch
         self.weights = []
         self.biases = []
-        for s, p, bias in params:
+        for i, (s, p, bias) in enumerate(params):
+            b = np.asarray(bias)
+            if b.shape != (np.shape(s)[0],) or not np.issubdtype(b.dtype, np.integer):
+                raise ValueError(f"bias {i} must be {np.shape(s)[0]} integers (one per output channel)")
+            if b.size and (b.min() < -(1 << 31) or b.max() >= (1 << 31)):
+                raise ValueError(f"bias {i} does not fit int32")
             w = pack_shift_weights(torch.from_numpy(s).to(device), torch.from_numpy(p).to(device), expand=expand)
             self.weights.append(w)
-            self.biases.append(torch.from_numpy(bias).to(device))
+            self.biases.append(torch.from_numpy(np.ascontiguousarray(b, dtype=np.int32)).to(device))
         self.layers = (ds_layer * len(specs))()
         for i, sp in enumerate(specs):
             L = self.layers[i]
@@ -190,15 +197,22 @@ class ShiftNetwork:
                 L.w = ctypes.pointer(self.weights[sp.param].desc)
                 L.bias = self.biases[sp.param].data_ptr()
         nbytes = ds_shift_forward_workspace_bytes(self.layers, len(specs), batch)
+        if nbytes == 0:
+            raise ValueError(f"the layer program was refused: {ds_last_error()}")
         self.workspace = torch.empty(nbytes, dtype=torch.uint8, device=device)
+        self.in_shape = (batch, specs[0].C, specs[0].H, specs[0].W)
         self.out_shape = (batch,) + output_shape([sp for sp in specs if sp.out == 1][-1])
 
     def forward(self, x, y=None, stream=None):
+        """Runs the program on int32 x of shape (batch, C, H, W) (the first layer's input) into y (new, or
+        a contiguous int32 tensor of at least out_shape's size) on the workspace's device."""
         import torch
+        _need(x, "x", torch.int32, self.in_shape)
+        if y is not None and (y.dtype != torch.int32 or not y.is_contiguous() or y.numel() < math.prod(self.out_shape)):
+            raise ValueError(f"y must be a contiguous int32 tensor of at least {math.prod(self.out_shape)} elements")
+        _on_one_gpu(workspace=self.workspace, x=x, y=y)
         if y is None:
             y = torch.empty(self.out_shape, dtype=torch.int32, device=x.device)
-        elif y.dtype != torch.int32 or not y.is_contiguous() or y.numel() < math.prod(self.out_shape):
-            raise ValueError(f"y must be a contiguous int32 tensor of at least {math.prod(self.out_shape)} elements")
         ds_shift_forward(self.layers, len(self.specs), x, y, self.workspace, self.workspace.numel(), self.batch,
                          stream)
         return y

@@ -286,6 +286,35 @@ def test_forward_program_validation_without_gpu(ds):
     assert L.ds_shift_forward(layers, n, 16, 16, 256, good - 1, 32, None) == ds.DS_ERR_BUFFER_TOO_SMALL
 
 
+def test_network_refuses_mismatched_inputs_and_biases(ds):
+    """ShiftNetwork checks its biases before packing and its input against the program before a launch:
+    an input with fewer images than the program was built for would otherwise be read past its end."""
+    import torch
+    from paper_1905_13298_gb300 import networks as PN
+    specs, shapes = PN.resnet_program("resnet18", 32, 32)
+    s = np.zeros(shapes[0], np.int8)
+    for bias, what in ((np.zeros(63, np.int32), "bias 0"), (np.zeros(64, np.float32), "bias 0"),
+                       (np.full(64, 1 << 31, np.int64), "int32")):
+        with pytest.raises(ValueError, match=what):
+            PN.ShiftNetwork(specs, [(s, s, bias)], batch=2, device="cpu")
+    with pytest.raises(ValueError, match="CUDA"):   # an in-range int64 bias passes; packing wants the GPU
+        PN.ShiftNetwork(specs, [(s, s, np.zeros(64, np.int64))], batch=2, device="cpu")
+    net = object.__new__(PN.ShiftNetwork)
+    net.specs, net.batch = specs, 2
+    net.in_shape, net.out_shape = (2, 3, 32, 32), (2, 1000, 1, 1)
+    net.workspace = torch.empty(256, dtype=torch.uint8)
+    x = torch.zeros(net.in_shape, dtype=torch.int32)
+    cases = [(lambda: net.forward(torch.zeros((1, 3, 32, 32), dtype=torch.int32)), "shape"),
+             (lambda: net.forward(x.float()), "int32"),
+             (lambda: net.forward(torch.zeros((2, 3, 32, 32), dtype=torch.int32).transpose(2, 3)), "contiguous"),
+             (lambda: net.forward(x, torch.zeros(net.out_shape)), "y must be"),
+             (lambda: net.forward(x, torch.zeros((2, 999), dtype=torch.int32)), "y must be"),
+             (lambda: net.forward(x, torch.zeros(net.out_shape, dtype=torch.int32)), "CUDA")]
+    for call, what in cases:
+        with pytest.raises(ValueError, match=what):
+            call()
+
+
 def test_network_output_shapes(ds):
     """ShiftNetwork sizes its output from the last layer writing the output slot (conv, pool or FC)."""
     from paper_1905_13298_gb300 import networks as PN
