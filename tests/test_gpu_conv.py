@@ -78,6 +78,31 @@ def test_conv_saturating_inputs(dslib, flags):
     assert np.array_equal(got, want)
 
 
+@pytest.mark.parametrize("geom", [GEOMS[0], GEOMS[1], GEOMS[2]])
+@pytest.mark.parametrize("flags", [0, 32])
+@pytest.mark.parametrize("expand", [False, True])
+def test_conv_degenerate_codes(dslib, geom, flags, expand):
+    """The degenerate cases of the method on the conv kernels: every sign zero gives y = sat32(b) at every
+    position (padding included); s = -1, p = 0 on x = INT32_MIN makes every in-image term 2^31, outside
+    int32, so the 64-bit path is taken (every window here holds at least four such terms: all outputs
+    saturate)."""
+    N, C, H, W, K, R, S, st, pd = geom
+    x, s, p, b = si.conv_layer(sum(geom) * 13 + flags, N, C, H, W, K, R, S, -(1 << 31), 1 << 31)
+    OH = (H + 2 * pd - R) // st + 1
+    OW = (W + 2 * pd - S) // st + 1
+    got, amax = _run(dslib, x, np.zeros_like(s), p, b, (st, st), (pd, pd), flags=flags, expand=expand)
+    assert np.array_equal(got, np.broadcast_to(b[None, :, None, None], (N, K, OH, OW)))
+    assert amax[1] == O.absmax(b)
+    xm = np.full(x.shape, -(1 << 31), np.int32)
+    sm = -np.ones(s.shape, np.int8)
+    pm = np.zeros(s.shape, np.int8)
+    want = O.conv2d_shift(xm, sm, pm, b, (st, st), (pd, pd))
+    assert (want == O.INT32_MAX).all()
+    got, amax = _run(dslib, xm, sm, pm, b, (st, st), (pd, pd), flags=flags, expand=expand)
+    assert np.array_equal(got, want)
+    assert amax[1] == O.absmax(want)
+
+
 # ResNet18 / ResNet50 / VGG16 layer shapes at a small batch, both kernels
 NET_GEOMS = [
     (1, 3, 224, 224, 64, 7, 7, 2, 3),    # stem 7x7/2

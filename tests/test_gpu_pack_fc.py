@@ -92,6 +92,27 @@ def test_linear_shift_bitexact(dslib, M, K, N, flags, expand):
     assert amax[1] == O.absmax(want)
 
 
+# one shape per FC kernel: cluster (small M) and shift GEMM (M = 1024, N = 3712)
+@pytest.mark.parametrize("M,K,N", [(1, 1, 1), (9, 700, 130), (1024, 40, 3712)])
+@pytest.mark.parametrize("expand", [False, True])
+def test_linear_shift_degenerate_codes(dslib, M, K, N, expand):
+    """The degenerate cases of the method: every sign zero gives y = sat32(b) (nnz = 0 and A = 0 in every
+    column); s = -1, p = 0 on x = INT32_MIN makes every term 2^31, the one term value outside int32, so the
+    accumulator bound must refuse the 32-bit path wherever the exact sums leave int32."""
+    x, s, p, b = si.fc_layer(M + 7 * K + N, M, K, N, -(1 << 31), 1 << 31)
+    got, amax = _run_fc(dslib, x, np.zeros_like(s), p, b, dslib.DS_AMAX_OUT, expand=expand)
+    assert np.array_equal(got, np.broadcast_to(b, (M, N)))
+    assert amax[1] == O.absmax(b)
+    xm = np.full((M, K), -(1 << 31), np.int32)
+    sm = -np.ones((N, K), np.int8)
+    pm = np.zeros((N, K), np.int8)
+    want = O.linear_shift(xm, sm, pm, b)
+    assert K == 1 or (O.linear_shift_acc(xm, sm, pm, b) > O.INT32_MAX).all()
+    got, amax = _run_fc(dslib, xm, sm, pm, b, dslib.DS_AMAX_OUT, expand=expand)
+    assert np.array_equal(got, want)
+    assert amax[0] == 1 << 31 and amax[1] == O.absmax(want)
+
+
 def test_linear_shift_config1_bitexact(dslib):
     x, s, p, b = si.config1()
     want = O.linear_shift(x, s, p, b)
