@@ -84,6 +84,17 @@ def test_bf16_relu_and_exact_small_integers(dslib):
     assert np.array_equal(y, want)
 
 
+@pytest.mark.parametrize("M,K,N", [(1, 8, 1), (300, 520, 260)])
+def test_bf16_zero_codes_give_the_bias(dslib, M, K, N):
+    """Every sign zero decodes to W = +0, so every product and the fp32 sum are exact zeros: y equals the
+    bias exactly (and ReLU of it)."""
+    bits, s, p, b = _case(M * 5 + K + N, M, K, N)
+    for relu in (False, True):
+        y, _ = _run(dslib, bits, np.zeros_like(s), p, b, relu=relu)
+        want = np.broadcast_to(b.astype(np.float64), (M, N))
+        assert np.array_equal(y, np.maximum(want, 0) if relu else want)
+
+
 def test_bf16_config4_float_sampled(dslib):
     """The float variant of the large FC shape, 8192 x 4096 x 4096, on sampled rows."""
     M, K, N = 8192, 4096, 4096
