@@ -69,6 +69,31 @@ def test_linear_backward_x_saturates(dslib):
     assert np.array_equal(dx.cpu().numpy(), want)
 
 
+def _degenerate_cases(seed, code_shape, dy_shape, bwd):
+    """(s, p, dy, want) for the degenerate codes: every sign zero (dX = 0), and s = -1, p = 0 on dY = INT32_MIN,
+    where every term is 2^31 (outside int32): dX saturates wherever a term reaches it."""
+    zero = (np.zeros(code_shape, np.int8), si.shift_codes_uniform(seed, code_shape),
+            si.activations(seed + 1, dy_shape, -(1 << 31), 1 << 31))
+    edge = (-np.ones(code_shape, np.int8), np.zeros(code_shape, np.int8), np.full(dy_shape, -(1 << 31), np.int32))
+    out = []
+    for s, p, dy in (zero, edge):
+        out.append((s, p, dy, bwd(dy, s, p)))
+    assert not out[0][3].any()
+    assert out[1][3].max() == O.INT32_MAX and out[1][3].min() >= 0
+    return out
+
+
+@pytest.mark.parametrize("M,K,N", [(1, 1, 1), (33, 130, 65), (200, 64, 1000)])
+def test_linear_backward_x_degenerate_codes(dslib, M, K, N):
+    for s, p, dy, want in _degenerate_cases(M + K + N, (N, K), (M, N), O.linear_shift_backward_x):
+        w = dslib.pack_shift_weights_backward(_dev(s), _dev(p))
+        dx = torch.empty((M, K), dtype=torch.int32, device="cuda")
+        amax = torch.zeros(2, dtype=torch.int32, device="cuda")
+        dslib.ds_linear_shift_backward_x(_dev(dy), w.desc[0], dx, M, K, N, dslib.DS_AMAX_OUT, amax)
+        assert np.array_equal(dx.cpu().numpy(), want)
+        assert amax.cpu().numpy().view(np.uint32)[1] == O.absmax(want)
+
+
 # N, C, H, W, K, R, S, stride, pad
 CONV_GEOMS = [
     (2, 3, 7, 6, 4, 3, 3, 1, 1),
@@ -81,7 +106,8 @@ CONV_GEOMS = [
     (1, 5, 6, 6, 3, 1, 1, 1, 1),        # pad > R - 1: the gather path even at stride 1
     (2, 4, 10, 9, 6, 5, 3, 2, 2),       # non-square kernel
     (1, 6, 11, 10, 5, 5, 5, 3, 2),      # stride 3
-    (2, 7, 9, 9, 4, 3, 3, 2, 0),        # stride 2, no padding: the last input row / column get no gradient
+    (2, 7, 9, 9, 4, 3, 3, 2, 0),        # stride 2, no padding: (9 - 3) / 2 whole steps, every row is reached
+    (2, 7, 10, 10, 4, 3, 3, 2, 0),      # stride 2, no padding: the last input row and column get no gradient
 ]
 
 
@@ -102,6 +128,24 @@ def test_conv_backward_x_bitexact(dslib, geom, flags, expand):
     want = O.conv2d_shift_backward_x(dy, s, p, (H, W), (st, st), (pd, pd))
     assert np.array_equal(dx.cpu().numpy(), want)
     assert amax.cpu().numpy().view(np.uint32)[1] == O.absmax(want)
+
+
+@pytest.mark.parametrize("geom", [CONV_GEOMS[0], CONV_GEOMS[1], CONV_GEOMS[2], CONV_GEOMS[-2], CONV_GEOMS[-1]])
+@pytest.mark.parametrize("flags", [0, 32])  # default / forced gather path
+def test_conv_backward_x_degenerate_codes(dslib, geom, flags):
+    """Zero codes give dX = 0 everywhere; s = -1, p = 0 on dY = INT32_MIN saturates every position a tap
+    reaches and leaves 0 where none does (stride 2 without padding: the last row and column)."""
+    N, C, H, W, K, R, S, st, pd = geom
+    OH, OW = O.conv_out_size(H, R, st, pd), O.conv_out_size(W, S, st, pd)
+    bwd = lambda dy, s, p: O.conv2d_shift_backward_x(dy, s, p, (H, W), (st, st), (pd, pd))
+    for s, p, dy, want in _degenerate_cases(sum(geom) + flags, (K, C, R, S), (N, K, OH, OW), bwd):
+        w = dslib.pack_shift_weights_backward(_dev(s), _dev(p), (st, st))
+        dx = torch.empty((N, C, H, W), dtype=torch.int32, device="cuda")
+        amax = torch.zeros(2, dtype=torch.int32, device="cuda")
+        dslib.ds_conv2d_shift_backward_x(_dev(dy), w.desc, dx, N, C, H, W, K, R, S, st, st, pd, pd,
+                                         flags | dslib.DS_AMAX_OUT, amax)
+        assert np.array_equal(dx.cpu().numpy(), want)
+        assert amax.cpu().numpy().view(np.uint32)[1] == O.absmax(want)
 
 
 @pytest.mark.parametrize("geom", [(2, 64, 56, 56, 64, 3, 3, 1, 1), (2, 64, 56, 56, 128, 1, 1, 2, 0),
