@@ -110,6 +110,13 @@ def measured_peaks():
     return {"hbm_gbs": 6800.0, "sm_max_mhz": 2070.0, "bf16_tflops": 1900.0}, "fallback"
 
 
+def smi_gpu_id(index: int, visible: str | None) -> str:
+    """nvidia-smi's --id of this process's CUDA device `index`: CUDA numbers only the devices listed in
+    CUDA_VISIBLE_DEVICES (indices or UUIDs, both accepted by --id), nvidia-smi every GPU of the machine."""
+    ids = [v.strip() for v in (visible or "").split(",") if v.strip()]
+    return ids[index] if index < len(ids) else str(index)
+
+
 class ClockSampler:
     """Samples nvidia-smi SM clocks and throttle reasons while the timed region runs."""
 
@@ -118,7 +125,7 @@ class ClockSampler:
              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
     def __init__(self, gpu_index: int):
-        self.gpu = gpu_index
+        self.gpu = smi_gpu_id(gpu_index, os.environ.get("CUDA_VISIBLE_DEVICES"))
         self.proc = None
         self.lines = []
         self.thread = None

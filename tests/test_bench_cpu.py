@@ -24,6 +24,14 @@ def test_clock_summary_clean_and_empty():
     assert bench.ClockSampler.summarize([])["sm_mhz"] is None
 
 
+def test_clock_sampler_queries_the_gpu_in_use():
+    """nvidia-smi numbers every GPU of the machine; CUDA only the visible ones."""
+    assert bench.smi_gpu_id(0, None) == "0" and bench.smi_gpu_id(3, "") == "3"
+    assert bench.smi_gpu_id(0, "5") == "5"
+    assert bench.smi_gpu_id(1, "4, 6,7") == "6"
+    assert bench.smi_gpu_id(0, "GPU-1a2b") == "GPU-1a2b"
+
+
 def test_default_workload_is_the_conv2x_layer():
     wl = bench.workload_by_name("conv2x", None)
     assert (wl["N"], wl["C"], wl["H"], wl["W"], wl["K"], wl["R"], wl["S"]) == (32, 64, 56, 56, 64, 3, 3)
