@@ -86,6 +86,7 @@ def sat32(v):
 
 
 def _check_codes(s: np.ndarray, p: np.ndarray) -> None:
+    """Rejects codes outside s in {-1, 0, +1} (Eq. 2) and p in [-15, 0] (Sec. 4 clipping; reading R-p+)."""
     if s.shape != p.shape:
         raise ValueError("s and p must have the same shape")
     if not np.isin(s, (-1, 0, 1)).all():
@@ -104,6 +105,7 @@ def linear_shift_acc(x: np.ndarray, s: np.ndarray, p: np.ndarray, b=None) -> np.
     acc[m, n] = b[n] + sum_k s[n, k] * floor(x[m, k] / 2^-p[n, k]).
     x: [M, K] integer; s, p: [N, K]; b: [N] or None.  Returns int64 [M, N].
     The loop runs over k; each step adds one term to every (m, n).
+    Follows Eq. 3 (fully-connected form) with the terms of Eq. 1-2, reading R-order, summed exactly (reading R-acc).
     """
     x = np.asarray(x, dtype=np.int64)
     s = np.asarray(s, dtype=np.int64)
@@ -124,7 +126,9 @@ def linear_shift_acc(x: np.ndarray, s: np.ndarray, p: np.ndarray, b=None) -> np.
 
 
 def linear_shift(x, s, p, b=None, relu: bool = False) -> np.ndarray:
-    """LinearShift forward on Q16.16 int32: sat32(acc), then optional ReLU.  Returns int32."""
+    """LinearShift forward on Q16.16 int32: sat32(acc), then optional ReLU.  Returns int32.
+
+    Follows Eq. 3 (fully-connected form) and reading R-acc (one saturation, after the bias)."""
     y = sat32(linear_shift_acc(x, s, p, b))
     if relu:
         y = np.maximum(y, 0)
@@ -136,6 +140,7 @@ def linear_shift(x, s, p, b=None, relu: bool = False) -> np.ndarray:
 # --------------------------------------------------------------------------
 
 def conv_out_size(h: int, r: int, stride: int, pad: int) -> int:
+    """Output extent of the convolutional form of Eq. 3 (reading R-conv: zero padding, stride)."""
     return (h + 2 * pad - r) // stride + 1
 
 
@@ -176,7 +181,9 @@ def conv2d_shift_acc(x, s, p, b=None, stride=(1, 1), pad=(0, 0)) -> np.ndarray:
 
 
 def conv2d_shift(x, s, p, b=None, stride=(1, 1), pad=(0, 0), relu: bool = False) -> np.ndarray:
-    """ConvShift forward on Q16.16 int32 NCHW: sat32(acc), then optional ReLU.  Returns int32."""
+    """ConvShift forward on Q16.16 int32 NCHW: sat32(acc), then optional ReLU.  Returns int32.
+
+    Follows Eq. 3 (convolutional form), readings R-conv and R-acc."""
     y = sat32(conv2d_shift_acc(x, s, p, b, stride, pad))
     if relu:
         y = np.maximum(y, 0)
@@ -187,6 +194,7 @@ def conv2d_shift_at(x, s, p, b, stride, pad, n: int, k: int, oh: int, ow: int) -
     """One output element of ConvShift (before saturation), as a Python int.
 
     Used to check sampled outputs of full-size launches one by one.
+    Follows Eq. 3 (convolutional form) and reading R-conv, term by term with Eq. 1-2.
     """
     N, C, H, W = x.shape
     _, _, R, S = s.shape
@@ -202,7 +210,9 @@ def conv2d_shift_at(x, s, p, b, stride, pad, n: int, k: int, oh: int, ow: int) -
 
 
 def linear_shift_at(x, s, p, b, m: int, n: int) -> int:
-    """One output element of LinearShift (before saturation), as a Python int."""
+    """One output element of LinearShift (before saturation), as a Python int.
+
+    Follows Eq. 3 (fully-connected form), term by term with Eq. 1-2."""
     acc = int(b[n]) if b is not None else 0
     for k in range(x.shape[1]):
         acc += term(int(x[m, k]), int(s[n, k]), int(p[n, k]))
@@ -214,7 +224,9 @@ def linear_shift_at(x, s, p, b, m: int, n: int) -> int:
 # --------------------------------------------------------------------------
 
 def absmax(x) -> int:
-    """max |x| over an int32 tensor, as a non-negative Python int (|INT32_MIN| = 2^31)."""
+    """max |x| over an int32 tensor, as a non-negative Python int (|INT32_MIN| = 2^31).
+
+    The input bound of reading R-acc's int32 proof."""
     x = np.asarray(x, dtype=np.int64)
     return int(np.abs(x).max()) if x.size else 0
 
@@ -224,6 +236,7 @@ def column_constants(s, p):
 
     A[n]   = sum_k |s[n,k]| * 2^(15 + p[n,k])   (sum of |weights| in units of 2^-15)
     nnz[n] = #{k : s[n,k] != 0}
+    Column constants of reading R-acc's int32 proof (|s| 2^p is the magnitude of flip(2^P, S), Eq. 3).
     """
     s = np.asarray(s, dtype=np.int64).reshape(np.shape(s)[0], -1)
     p = np.asarray(p, dtype=np.int64).reshape(np.shape(p)[0], -1)
@@ -237,6 +250,7 @@ def int32_accumulation_is_exact(amax: int, A: int, nnz: int, babs: int) -> bool:
 
     |floor(x / 2^k)| <= ceil(|x| / 2^k) <= |x| / 2^k + 1 - 2^-k, so the sum is at
     most ceil(amax * A / 2^15) + nnz + |b|.
+    Reading R-acc: when the exact sum provably fits int32, 32-bit accumulation is exact.
     """
     return ((amax * A + (1 << 15) - 1) >> 15) + nnz + babs <= INT32_MAX
 
@@ -280,7 +294,9 @@ def avgpool_floor(x, k: int, stride: int) -> np.ndarray:
 
 
 def add_relu(a, b) -> np.ndarray:
-    """Residual join: ReLU(sat32(a + b)) on int32 tensors."""
+    """Residual join: ReLU(sat32(a + b)) on int32 tensors.
+
+    Residual join of the ResNet chain (reading R-acc: one saturation, then ReLU; reading R-bn: no BatchNorm)."""
     v = sat32(np.asarray(a, dtype=np.int64) + np.asarray(b, dtype=np.int64))
     return np.maximum(v, 0).astype(np.int32)
 
@@ -311,7 +327,9 @@ def linear_shift_float(x_f64, s, p, b=None) -> np.ndarray:
 
 
 def linear_shift_float_absterms(x_f64, s, p) -> np.ndarray:
-    """sum_k |s * 2^p * x| per output, the scale of the float variant's tolerance."""
+    """sum_k |s * 2^p * x| per output, the scale of the float variant's tolerance.
+
+    Scale of reading R-float's tolerance for Eq. 3 with W = flip(2^P, S)."""
     x = np.abs(np.asarray(x_f64, dtype=np.float64))
     w = np.abs(np.asarray(s, dtype=np.float64)) * np.ldexp(1.0, np.asarray(p, dtype=np.int64))
     return x @ w.T
@@ -328,7 +346,9 @@ FORMAT_PLANES6 = 1
 
 
 def blob_layout(n_out: int, k_red: int) -> dict:
-    """Byte offsets of the regions of a planes6 blob."""
+    """Byte offsets of the regions of a planes6 blob.
+
+    Storage of the codes of Eq. 3 (reading R-code: 4 shift bits, a sign plane and a non-zero plane)."""
     n_chunks = (k_red + 31) // 32
     nib = BLOB_HEADER
     bits = nib + n_chunks * n_out * 16
@@ -344,6 +364,7 @@ def pack_planes6(s, p) -> np.ndarray:
 
     Returns the blob as uint8 [total].  The header carries magic, format, dims,
     invalid_count = 0, nnz_max and a_max.
+    Storage format of reading R-code (6 bits per weight for the 33 code states of Eq. 2 and Sec. 4).
     """
     s = np.asarray(s, dtype=np.int64)
     p = np.asarray(p, dtype=np.int64)
@@ -380,7 +401,9 @@ def pack_planes6(s, p) -> np.ndarray:
 
 
 def unpack_planes6(blob, n_out: int, k_red: int):
-    """Inverse of pack_planes6 for the code regions: returns (s, p) int8 [n_out, k_red]."""
+    """Inverse of pack_planes6 for the code regions: returns (s, p) int8 [n_out, k_red].
+
+    Reading R-code, read back."""
     blob = np.asarray(blob, dtype=np.uint8)
     L = blob_layout(n_out, k_red)
     nch = L["n_chunks"]
@@ -401,7 +424,8 @@ def unpack_planes6(blob, n_out: int, k_red: int):
 
 def expand_codes(s, p) -> np.ndarray:
     """Expanded execution layout of [n_out, k_red] codes (documented in include/deepshift.h):
-    int32 [ceil(n_out/32)][k_red][64], words 0..31 = -p and 32..63 = s of columns 32*cb + c."""
+    int32 [ceil(n_out/32)][k_red][64], words 0..31 = -p and 32..63 = s of columns 32*cb + c.
+    Execution layout of the codes of Eq. 3 (-p and s per weight as 32-bit words)."""
     s = np.asarray(s, dtype=np.int64)
     p = np.asarray(p, dtype=np.int64)
     _check_codes(s, p)
@@ -465,7 +489,8 @@ def quantize_activations(x) -> np.ndarray:
 # ---------------------------------------------------------------------------
 def linear_shift_backward_x_acc(dy, s, p) -> np.ndarray:
     """Exact int64 dC/dX of LinearShift: dx[m, k] = sum_n s[n, k] * floor(dy[m, n] / 2^-p[n, k]),
-    i.e. dC/dY W_q^T with every product a shift and a flip.  dy: [M, N]; s, p: [N, K]."""
+    i.e. dC/dY W_q^T with every product a shift and a flip.  dy: [M, N]; s, p: [N, K].
+    Follows Eq. 7 (fully-connected form) with reading R-bwd."""
     dy = np.asarray(dy, dtype=np.int64)
     s = np.asarray(s, dtype=np.int64)
     p = np.asarray(p, dtype=np.int64)
@@ -482,6 +507,7 @@ def linear_shift_backward_x_acc(dy, s, p) -> np.ndarray:
 
 
 def linear_shift_backward_x(dy, s, p) -> np.ndarray:
+    """Eq. 7 (fully-connected form) with reading R-bwd: sat32 of the exact sum."""
     return sat32(linear_shift_backward_x_acc(dy, s, p)).astype(np.int32)
 
 
@@ -490,7 +516,8 @@ def conv2d_shift_backward_x_acc(dy, s, p, in_hw, stride=(1, 1), pad=(0, 0)) -> n
     implies: output (n, k, oh, ow) read input (c, oh*sh + r - ph, ow*sw + q - pw)
     through code (k, c, r, q), so its gradient term s * floor(dy / 2^-p) is added
     there (positions in the padding are dropped).  dy: [N, K, OH, OW];
-    s, p: [K, C, R, S]; in_hw = (H, W); returns int64 [N, C, H, W]."""
+    s, p: [K, C, R, S]; in_hw = (H, W); returns int64 [N, C, H, W].
+    Follows Eq. 7 and its footnote (convolutional form) with reading R-bwd."""
     dy = np.asarray(dy, dtype=np.int64)
     s = np.asarray(s, dtype=np.int64)
     p = np.asarray(p, dtype=np.int64)
@@ -514,6 +541,7 @@ def conv2d_shift_backward_x_acc(dy, s, p, in_hw, stride=(1, 1), pad=(0, 0)) -> n
 
 
 def conv2d_shift_backward_x(dy, s, p, in_hw, stride=(1, 1), pad=(0, 0)) -> np.ndarray:
+    """Eq. 7 and its footnote (convolutional form) with reading R-bwd: sat32 of the exact sum."""
     return sat32(conv2d_shift_backward_x_acc(dy, s, p, in_hw, stride, pad)).astype(np.int32)
 
 
@@ -532,7 +560,9 @@ def backward_codes(s, p):
 
 
 def phase_taps(R: int, stride: int, a: int) -> int:
-    """Number of taps r = a, a + stride, ... below R."""
+    """Number of taps r = a, a + stride, ... below R.
+
+    Tap count of one phase of a strided input gradient (Eq. 7 footnote, split by stride phase)."""
     return (R - 1 - a) // stride + 1 if a < R else 0
 
 

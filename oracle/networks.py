@@ -39,6 +39,8 @@ VGG16_CFG = [64, 64, "M", 128, 128, "M", 256, 256, 256, "M", 512, 512, 512, "M",
 
 
 def _conv(x, prm, stride, pad, relu, residual=None):
+    """One ConvShift layer of a chain (Eq. 3, convolutional form; readings R-conv, R-acc), then either the
+    residual join ReLU(sat32(y + residual)) or the optional ReLU."""
     s, p, b = prm
     y = O.conv2d_shift(x, s, p, b, (stride, stride), (pad, pad), relu=False)
     if residual is not None:
@@ -47,7 +49,10 @@ def _conv(x, prm, stride, pad, relu, residual=None):
 
 
 def resnet_forward(x, params, arch: str = "resnet18"):
-    """Forward of an all-shift ResNet; x int32 [N, 3, 224, 224]; returns int32 [N, 1000]."""
+    """Forward of an all-shift ResNet; x int32 [N, 3, 224, 224]; returns int32 [N, 1000].
+
+    Every conv and FC is a shift layer (Eq. 3 with Sec. 4's fixed point); pools follow reading R-pool, and
+    BatchNorm is omitted (reading R-bn)."""
     kind, blocks = RESNET_STAGES[arch]
     it = iter(params)
     x = _conv(x, next(it), 2, 3, relu=True)
@@ -81,7 +86,9 @@ def resnet_forward(x, params, arch: str = "resnet18"):
 
 
 def vgg16_forward(x, params):
-    """Forward of an all-shift VGG16; x int32 [N, 3, H, W] (224 x 224 in the workloads); returns int32 [N, 1000]."""
+    """Forward of an all-shift VGG16; x int32 [N, 3, H, W] (224 x 224 in the workloads); returns int32 [N, 1000].
+
+    Every conv and FC is a shift layer (Eq. 3 with Sec. 4's fixed point); max-pools follow reading R-pool."""
     it = iter(params)
     for v in VGG16_CFG:
         if v == "M":
