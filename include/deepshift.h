@@ -60,11 +60,11 @@ typedef enum {
 /* Description of the last error on the calling thread ("" if none). */
 const char* ds_last_error(void);
 
-/* Library version: major * 10000 + minor * 100 + patch. */
+/* Library version: major * 10000 + minor * 100 + patch (a library utility: no counterpart in the paper). */
 int ds_version(void);
 
 /* sizeof of the ABI structs as compiled into the library (0: ds_weights, 1: ds_layer), so that
- * bindings can check their layout; 0 for any other argument. */
+ * bindings can check their layout; 0 for any other argument (a library utility: no counterpart in the paper). */
 size_t ds_abi_struct_size(int which);
 
 /* ---------------------------------------------------------------------------
@@ -162,7 +162,7 @@ ds_status ds_pack_shift_weights(const int8_t* s, const int8_t* p, int64_t n_out,
 size_t ds_expanded_weight_bytes(int64_t n_out, int64_t k_red);
 
 /*
- * Expand packed weights into `expanded` (device, 16-byte aligned, at least
+ * Expand packed weights (the codes of Eq. 3's flip(2^P, S)) into `expanded` (device, 16-byte aligned, at least
  * ds_expanded_weight_bytes bytes, caller-owned and outliving every use) and
  * record it in *w (w->expanded, w->expanded_bytes).  Stream-ordered and
  * asynchronous; the blob must stay valid.  Errors: DS_ERR_INVALID_ARG for an
@@ -185,14 +185,15 @@ ds_status ds_expand_shift_weights(ds_weights* w, void* expanded, size_t expanded
 size_t ds_bf16_weight_bytes(int64_t n_out, int64_t k_red);
 
 /*
- * Decode packed weights into bf16 W[n][k] = s * 2^p (sign bit, exponent 127 + p,
+ * Decode packed weights into bf16 W[n][k] = s * 2^p = flip(2^P, S) of Eq. 3 (sign bit, exponent 127 + p,
  * zero mantissa; +0 for s = 0) in `buf` (device, 16-byte aligned, caller-owned)
  * and record it in w->weights_bf16.  Stream-ordered, asynchronous.
  */
 ds_status ds_expand_shift_weights_bf16(ds_weights* w, void* buf, size_t bytes, void* stream);
 
 /*
- * Float LinearShift on tcgen05 tensor cores (TMA-fed, TMEM accumulator).
+ * Float LinearShift (Eq. 3, fully-connected form, in the float form the paper trains with, Sec. 4) on tcgen05
+ * tensor cores (TMA-fed, TMEM accumulator).
  *   x     device bf16 bit patterns (uint16) [M][K], row-major, K % 8 == 0
  *   w     weights with w->weights_bf16 set, n_out == N, k_red == K
  *   bias  device fp32 [N] or NULL
@@ -203,7 +204,8 @@ ds_status ds_expand_shift_weights_bf16(ds_weights* w, void* buf, size_t bytes, v
 ds_status ds_linear_shift_bf16(const uint16_t* x, const ds_weights* w, const float* bias, float* y, int64_t M,
                                int64_t K, int64_t N, uint32_t flags, void* stream);
 
-/* 1 if a bounded wait of the float kernel gave up (a fault record; 0 normally, -1 if unreadable). */
+/* 1 if a bounded wait of the float kernel gave up (a fault record; 0 normally, -1 if unreadable; a library
+ * utility: no counterpart in the paper). */
 int ds_bf16_fault_flag(void);
 
 /* ---------------------------------------------------------------------------
@@ -317,7 +319,8 @@ typedef struct ds_layer {
 size_t ds_shift_forward_workspace_bytes(const ds_layer* layers, int n, int batch);
 
 /*
- * Runs the program: x = slot 0 (device, [batch][C0][H0][W0] of layer 0),
+ * Runs the program (shift layers of Eq. 3 with the Sec. 4 fixed point, pools as described above):
+ * x = slot 0 (device, [batch][C0][H0][W0] of layer 0),
  * y = slot 1 (device, the tensor of the last layer that writes slot 1),
  * ws = workspace (device, 256-byte aligned, >= the bytes above).
  * Validation errors (DS_ERR_SHAPE, DS_ERR_INVALID_ARG, ...) are reported
@@ -401,7 +404,8 @@ ds_status ds_quantize_shift_weights(const float* w, int64_t n, int p_min, int8_t
 ds_status ds_quantize_q16(const float* x, int64_t n, int32_t* q, void* stream);
 
 /*
- * max |x| over n int32 values, written to *amax (device u32; |INT32_MIN| = 2^31).
+ * max |x| over n int32 values, written to *amax (device u32; |INT32_MIN| = 2^31): the input of the
+ * accumulator-width proof above (the paper is silent on overflow; Sec. 4 fixes only the 32-bit format).
  */
 ds_status ds_absmax(const int32_t* x, int64_t n, uint32_t* amax, void* stream);
 
