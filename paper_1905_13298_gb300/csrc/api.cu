@@ -1,4 +1,6 @@
-// C ABI entry points: argument validation, then stream-ordered launches.
+// C ABI entry points of the shift operators (Eq. 3), the code conversion
+// (Eq. 4-6) and the input gradient (Eq. 7): argument validation, then
+// stream-ordered launches.
 // Nothing is launched and no output is written when validation fails.
 #include <stdarg.h>
 #include <stdio.h>

@@ -1,6 +1,8 @@
-// Integer pooling for the chained forward of ResNet / VGG shaped networks.
-// Max-pool ignores padded taps; average pool is floor(sum / (R*S)) over a
-// window without padding (floor division, also for negative sums).
+// Integer pooling for the chained forward of ResNet / VGG shaped networks
+// (the pools around the shift layers of Eq. 3; the paper does not define
+// them on fixed point).  Max-pool ignores padded taps; average pool is
+// floor(sum / (R*S)) over a window without padding (floor division, also for
+// negative sums).
 #include "ds_common.cuh"
 
 namespace ds {

@@ -1,4 +1,7 @@
-// Shared definitions of the DeepShift CUDA library (sm_103a).
+// Shared definitions of the DeepShift CUDA library (sm_103a): the packed code
+// layout of Eq. 3's flip(2^P, S) (4 shift bits, a sign plane and a non-zero
+// plane per 32-weight chunk), the launch parameters of the shift kernels
+// (Eq. 1-3 on Sec. 4's fixed point) and their asynchronous-copy helpers.
 #pragma once
 
 #include <cuda_runtime.h>

@@ -1,4 +1,4 @@
-// LinearShift for callers that cannot allocate device memory.
+// LinearShift (Eq. 3) for callers that cannot allocate device memory.
 //
 // ds_linear_shift needs two 32-bit words of device scratch (amax_io): the
 // max|x| written by its pre-pass and read by the kernel to prove that 32-bit

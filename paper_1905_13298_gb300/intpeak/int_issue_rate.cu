@@ -1,5 +1,8 @@
 // Integer issue-rate microbenchmark for the roofline denominator of the
 // shift kernels (built as its own small library, not part of the C ABI).
+// A DeepShift term (Eq. 1-2: a shift and a sign flip, the multiply of Fig. 1a
+// replaced) is SHF + IMAD here, so kind 2 measures the rate a term loop can
+// reach.
 //
 // Each kernel runs a register-resident loop of one instruction mix with
 // enough independent chains to hide latency over a grid of CTAs, and records
