@@ -324,7 +324,11 @@ size_t ds_shift_forward_workspace_bytes(const ds_layer* layers, int n, int batch
  * y = slot 1 (device, the tensor of the last layer that writes slot 1),
  * ws = workspace (device, 256-byte aligned, >= the bytes above).
  * Validation errors (DS_ERR_SHAPE, DS_ERR_INVALID_ARG, ...) are reported
- * before anything is launched.  Asynchronous, stream-ordered, no allocation.
+ * before anything is launched.  Asynchronous, stream-ordered, no device
+ * allocation; the planner's small host arrays are allocated before the first
+ * launch, and a failed host allocation returns DS_ERR_UNSUPPORTED ("host
+ * memory allocation failed") with nothing launched.  No C++ exception leaves
+ * any entry point.
  */
 ds_status ds_shift_forward(const ds_layer* layers, int n, const int32_t* x, int32_t* y, void* ws,
                            size_t ws_bytes, int batch, void* stream);

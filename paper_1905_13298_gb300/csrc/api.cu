@@ -4,15 +4,17 @@
 // Nothing is launched and no output is written when validation fails.
 #include <stdarg.h>
 #include <stdio.h>
+#include <string.h>
 
 #include <initializer_list>
-#include <string>
 
 #include "ds_common.cuh"
 
 namespace ds {
 
-static thread_local std::string g_last_error;
+// The last error of the calling thread, in a fixed buffer: recording an error
+// never allocates, so no entry point can fail (or throw) while reporting one.
+static thread_local char g_last_error[512];
 
 void set_error(const char* fmt, ...) {
   char buf[512];
@@ -20,10 +22,10 @@ void set_error(const char* fmt, ...) {
   va_start(ap, fmt);
   vsnprintf(buf, sizeof(buf), fmt, ap);
   va_end(ap);
-  g_last_error = buf;
+  memcpy(g_last_error, buf, sizeof(buf));
 }
 
-void clear_error() { g_last_error.clear(); }
+void clear_error() { g_last_error[0] = '\0'; }
 
 ds_status fail(ds_status st, const char* fmt, ...) {
   char buf[512];
@@ -31,7 +33,7 @@ ds_status fail(ds_status st, const char* fmt, ...) {
   va_start(ap, fmt);
   vsnprintf(buf, sizeof(buf), fmt, ap);
   va_end(ap);
-  g_last_error = buf;
+  memcpy(g_last_error, buf, sizeof(buf));
   return st;
 }
 
@@ -235,7 +237,7 @@ using namespace ds;
 
 extern "C" {
 
-const char* ds_last_error(void) { return g_last_error.c_str(); }
+const char* ds_last_error(void) { return g_last_error; }
 
 int ds_version(void) { return 100; }
 

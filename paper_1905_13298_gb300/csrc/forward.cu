@@ -8,8 +8,10 @@
 // its producer (pools pass their input's bound through, since max-pool and
 // floor-average never exceed it) and writes max|y| into its own word, so the
 // accumulator-width proof of every layer happens on the device.
+#include <stdio.h>
+
 #include <algorithm>
-#include <string>
+#include <exception>
 #include <vector>
 
 #include "ds_common.cuh"
@@ -34,8 +36,9 @@ struct Plan {
 
 // Re-raises a failed check with the layer's index in front of its message.
 ds_status layer_fail(ds_status st, int i) {
-  const std::string what = ds_last_error();
-  return fail(st, "layer %d: %s", i, what.c_str());
+  char what[512];
+  snprintf(what, sizeof(what), "%s", ds_last_error());
+  return fail(st, "layer %d: %s", i, what);
 }
 
 ds_status plan_program(const ds_layer* L, int n, int batch, Plan& P) {
@@ -150,16 +153,24 @@ using namespace ds;
 
 extern "C" {
 
+// The planner and the executor keep small host arrays (per slot and per
+// layer).  No exception may leave a C entry point: a failed host allocation
+// becomes a status, reported before anything is launched (every array exists
+// before the first launch).
 size_t ds_shift_forward_workspace_bytes(const ds_layer* layers, int n, int batch) {
   clear_error();
-  Plan P;
-  if (plan_program(layers, n, batch, P) != DS_OK) return 0;
-  return P.total;
+  try {
+    Plan P;
+    if (plan_program(layers, n, batch, P) != DS_OK) return 0;
+    return P.total;
+  } catch (const std::exception&) {
+    fail(DS_ERR_UNSUPPORTED, "host memory allocation failed");
+    return 0;
+  }
 }
 
-ds_status ds_shift_forward(const ds_layer* L, int n, const int32_t* x, int32_t* y, void* ws, size_t ws_bytes,
-                           int batch, void* stream) {
-  clear_error();
+static ds_status shift_forward(const ds_layer* L, int n, const int32_t* x, int32_t* y, void* ws, size_t ws_bytes,
+                               int batch, void* stream) {
   if (!x || !y || !ws) return fail(DS_ERR_INVALID_ARG, "NULL x, y or workspace");
   Plan P;
   ds_status r = plan_program(L, n, batch, P);
@@ -220,6 +231,16 @@ ds_status ds_shift_forward(const ds_layer* L, int n, const int32_t* x, int32_t* 
     if (r != DS_OK) return r;
   }
   return DS_OK;
+}
+
+ds_status ds_shift_forward(const ds_layer* L, int n, const int32_t* x, int32_t* y, void* ws, size_t ws_bytes,
+                           int batch, void* stream) {
+  clear_error();
+  try {
+    return shift_forward(L, n, x, y, ws, ws_bytes, batch, stream);
+  } catch (const std::exception&) {
+    return fail(DS_ERR_UNSUPPORTED, "host memory allocation failed");
+  }
 }
 
 }  // extern "C"
