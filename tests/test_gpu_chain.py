@@ -56,6 +56,18 @@ def test_resnet18_stress_codes_saturate_exactly(dslib):
     assert np.array_equal(_run(prog, params, x), want)
 
 
+def test_resnet18_zero_codes(dslib):
+    """Every sign zero (nnz = 0 and A = 0 in every column of every layer): each layer's output is its bias after
+    the epilogue, carried through pools, residual joins and the max|x| hand-off between layers."""
+    from paper_1905_13298_gb300 import networks as PN
+    prog = PN.resnet_program("resnet18", 32, 32)
+    params = [(np.zeros_like(s), p, b) for s, p, b in si.network_params(prog[1], 500)]
+    x = si.image_batch(11, 2, 3, 32, 32)
+    want = ON.resnet_forward(x, params, "resnet18")
+    assert np.array_equal(want, np.broadcast_to(params[-1][2], want.shape))   # the FC sees only its bias
+    assert np.array_equal(_run(prog, params, x), want)
+
+
 def test_resnet18_full_size_batch1(dslib):
     """The ResNet18-architecture forward at 224 x 224, batch 1: every output."""
     from paper_1905_13298_gb300 import networks as PN
