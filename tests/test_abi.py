@@ -244,6 +244,28 @@ def test_tensor_helpers_refuse_mismatched_tensors(ds):
             call()
 
 
+def test_plain_c_client_builds_and_runs(tmp_path, ds):
+    """The header is C99 and the library links into a plain C program (no Python, no torch): size queries and
+    argument validation answer as documented without a GPU (tests/c_abi_client.c)."""
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    lib_dir = os.path.dirname(ds.LIB_PATH)
+    exe = str(tmp_path / "c_abi_client")
+    cmd = [cc, "-std=c99", "-Wall", "-Wextra", "-Werror", "-pedantic", "-I", os.path.join(ROOT, "include"),
+           os.path.join(ROOT, "tests", "c_abi_client.c"), "-o", exe, "-L", lib_dir, "-ldeepshift",
+           f"-Wl,-rpath,{lib_dir}"]
+    r = subprocess.run(cmd, capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    env = dict(os.environ)
+    env["LD_LIBRARY_PATH"] = os.pathsep.join(p for p in ("/usr/local/cuda/lib64", env.get("LD_LIBRARY_PATH")) if p)
+    r = subprocess.run([exe], capture_output=True, text=True, env=env, timeout=60)
+    assert r.returncode == 0, f"check {r.returncode} failed: {r.stdout}{r.stderr}"
+    assert "c abi client ok" in r.stdout
+
+
 def test_no_cpu_fallback_without_library(tmp_path, monkeypatch, ds):
     """The binding refuses to run when the shared library is missing."""
     monkeypatch.setattr(ds, "_lib", None)
