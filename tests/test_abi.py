@@ -244,6 +244,34 @@ def test_tensor_helpers_refuse_mismatched_tensors(ds):
             call()
 
 
+def test_last_error_is_per_thread(ds):
+    """ds_last_error is thread-local: threads that fail different checks each read their own message."""
+    import threading
+    L = ds.lib()
+    w = ds.ds_weights()
+    calls = {
+        "NULL": lambda: L.ds_linear_shift(None, ctypes.byref(w), None, None, 1, 1, 1, 0, None, None),
+        "n must be positive": lambda: L.ds_absmax(16, 0, 16, None),
+        "p_min": lambda: L.ds_quantize_shift_weights(16, 4, -16, 16, 32, None),
+    }
+    wrong = []
+
+    def worker(expect, call):
+        for _ in range(2000):
+            call()
+            msg = ds.ds_last_error()
+            if expect not in msg:
+                wrong.append((expect, msg))
+                return
+
+    threads = [threading.Thread(target=worker, args=kv) for kv in calls.items()]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    assert not wrong, wrong[:3]
+
+
 def test_plain_c_client_builds_and_runs(tmp_path, ds):
     """The header is C99 and the library links into a plain C program (no Python, no torch): size queries and
     argument validation answer as documented without a GPU (tests/c_abi_client.c)."""
