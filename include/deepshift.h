@@ -49,6 +49,13 @@ typedef enum {
   DS_ERR_CUDA = 7              /* a CUDA runtime call or launch failed */
 } ds_status;
 
+/* Devices.  Kernel attributes (the opt-in shared-memory size, non-portable
+ * cluster sizes) are set once per process, on the device that is current at a
+ * kernel's first launch: drive one GPU per process (one process per GPU, as
+ * the multi-GPU replicas do).  A launch on a second device from the same
+ * process is not supported; it fails with DS_ERR_CUDA rather than computing
+ * anything wrong. */
+
 /* Size limits.  Every size the library forms from caller dimensions is
  * bounded before it can overflow 64 bits.  A code matrix holds at most 2^48
  * codes, with n_out <= 2^31 and k_red <= 2^40 (2^36 for the expanded and
