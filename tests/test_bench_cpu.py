@@ -37,3 +37,40 @@ def test_default_workload_is_the_conv2x_layer():
     assert (wl["N"], wl["C"], wl["H"], wl["W"], wl["K"], wl["R"], wl["S"]) == (32, 64, 56, 56, 64, 3, 3)
     assert wl["terms"] == 32 * 64 * 56 * 56 * 64 * 9 == 3_699_376_128
     assert 32 % bench.E2E_CHUNKS == 0
+
+
+def _run_bench(args, env_extra=None):
+    import json
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    env = dict(os.environ, **(env_extra or {}))
+    r = subprocess.run([sys.executable, os.path.join(root, "bench.py"), *args], capture_output=True, text=True,
+                       env=env, cwd=root, timeout=300)
+    lines = [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
+    return r.returncode, [json.loads(ln) for ln in lines], r.stderr
+
+
+def test_reference_arm_prints_the_contract_line():
+    """--impl reference times the oracle on the host (no GPU) and prints one JSON line with the base keys."""
+    rc, lines, err = _run_bench(["--impl", "reference", "--steps", "1", "--warmup", "1"])
+    assert rc == 0, err
+    assert len(lines) == 1
+    d = lines[0]
+    assert d["impl"] == "reference" and d["value"] > 0 and d["unit"] == d["metric"]
+    for key in ("n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better", "scaling", "vs_baseline", "dtype",
+                "data", "config"):
+        assert key in d, key
+    assert d["steps"] == 1 and d["warmup"] == 1 and d["higher_is_better"] is True
+    assert d["config"]["workload"] == "resnet18_conv2x_convshift_3x3"
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
+    assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+
+
+def test_reference_arm_runs_on_rank_zero_only():
+    rc, lines, err = _run_bench(["--impl", "reference", "--steps", "1", "--warmup", "1"],
+                                {"RANK": "1", "WORLD_SIZE": "2", "LOCAL_RANK": "1"})
+    assert rc == 0, err
+    assert lines == []
