@@ -27,7 +27,6 @@ import synth_inputs as si  # noqa: E402
 
 METRIC = "Gshift-ops/s"
 L2_BYTES = 129 * 1024 * 1024
-SMS = 152
 INT_OPS_PER_CLK_PER_SM = 128  # 4 SMSPs x 32 lanes: 16-lane ALU pipe + 16-lane FMA pipe (IMAD)
 ALG_INT_OPS_PER_TERM = 2      # one shift + one add/subtract per term (Fig. 1a: MAC -> shift + add)
 # DRAM bytes (read + write) of one conv_direct_kernel<1,3,7,0> launch on this workload, from one ncu capture
@@ -108,6 +107,16 @@ def measured_peaks():
         with open(path) as f:
             return json.load(f), "measured"
     return {"hbm_gbs": 6800.0, "sm_max_mhz": 2070.0, "bf16_tflops": 1900.0}, "fallback"
+
+
+def alu_peak(dev=None):
+    """INT32 issue roofline of the device: (T int-ops/s, SMs, SM MHz, peak source).  SMs are read from the
+    device; the clock is MEASURED_PEAKS.json's maximum SM clock (else the recipe's fallback)."""
+    import torch
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    peaks, kind = measured_peaks()
+    sm_max = float(peaks.get("sm_max_mhz", 2070.0))
+    return sms * INT_OPS_PER_CLK_PER_SM * sm_max * 1e6 / 1e12, sms, sm_max, kind
 
 
 def smi_gpu_id(index: int, visible: str | None) -> str:
@@ -305,8 +314,7 @@ def run_gpu_other(args, wl, rank, world, local_rank):
     clocks = sampler.stop()
     ms = e0.elapsed_time(e1)
     peaks, _ = measured_peaks()
-    sm_max = float(peaks.get("sm_max_mhz", 2070.0))
-    alu_peak = SMS * INT_OPS_PER_CLK_PER_SM * sm_max * 1e6 / 1e12
+    alu_tops = alu_peak(dev)[0]
     value = terms * args.steps / (ms / 1e3) / 1e9
     if wl["kind"] == "fc16":
         tflops = 2 * terms / (ms / args.steps / 1e3) / 1e12
@@ -314,8 +322,8 @@ def run_gpu_other(args, wl, rank, world, local_rank):
         roof = {"bound": "tensor", "achieved": tflops, "peak": peak, "unit": "TFLOP/s", "frac": tflops / peak,
                 "traffic": None, "kernel": "linear_bf16_kernel", "peak_basis": "bf16_tflops (burst), measured"}
     else:
-        roof = {"bound": "alu", "achieved": 2 * terms / (ms / args.steps / 1e3) / 1e12, "peak": alu_peak,
-                "unit": "Tintop/s", "frac": 2 * terms / (ms / args.steps / 1e3) / 1e12 / alu_peak,
+        roof = {"bound": "alu", "achieved": 2 * terms / (ms / args.steps / 1e3) / 1e12, "peak": alu_tops,
+                "unit": "Tintop/s", "frac": 2 * terms / (ms / args.steps / 1e3) / 1e12 / alu_tops,
                 "traffic": None, "kernel": "whole step"}
     out = {"metric": METRIC, "value": value, "unit": METRIC, "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
            "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
@@ -416,7 +424,7 @@ def time_fc_layer(args, ds, dev, seed, M, K, N, backward=False):
     ms = e0.elapsed_time(e1) / reps
     terms = M * K * N
     return dict(shape=f"FC {K}->{N}", terms=terms, ms=ms, gsops=terms / ms / 1e6,
-                frac=2 * terms / (ms / 1e3) / (SMS * INT_OPS_PER_CLK_PER_SM * 2070e6))
+                frac=2 * terms / (ms / 1e3) / (alu_peak(dev)[0] * 1e12))
 
 
 def run_layer_sweep(args, wl, local_rank):
@@ -490,7 +498,7 @@ def run_layer_sweep(args, wl, local_rank):
         ms = e0.elapsed_time(e1) / reps
         terms = B * sp.K * OH * OW * sp.C * sp.R * sp.S
         r = dict(layer=i, shape=f"{sp.C}x{sp.H}x{sp.W}->{sp.K} {sp.R}x{sp.S}/{sp.stride}", terms=terms, ms=ms,
-                 gsops=terms / ms / 1e6, frac=2 * terms / (ms / 1e3) / (SMS * INT_OPS_PER_CLK_PER_SM * 2070e6))
+                 gsops=terms / ms / 1e6, frac=2 * terms / (ms / 1e3) / (alu_peak(dev)[0] * 1e12))
         seen[key] = r
         rows.append(r)
         tot_terms += terms
@@ -629,8 +637,7 @@ def run_gpu(args, wl, rank, world, local_rank):
         peaks, peak_kind = measured_peaks()
         terms_total = wl["terms"] * args.steps * world
         value = terms_total / (ms_total / 1e3) / 1e9
-        sm_max = float(peaks.get("sm_max_mhz", 2070.0))
-        alu_peak = SMS * INT_OPS_PER_CLK_PER_SM * sm_max * 1e6 / 1e12  # T int-ops/s
+        alu_tops, sms, sm_max, _ = alu_peak(dev)  # T int-ops/s
         achieved = ALG_INT_OPS_PER_TERM * wl["terms"] / (kern_ms / 1e3) / 1e12
         alg_bytes = 4 * (N * C * H * W + N * K * H * W) + ds.ds_packed_weight_bytes(K, C * R * S) + 4 * K
         out = {
@@ -642,10 +649,10 @@ def run_gpu(args, wl, rank, world, local_rank):
                        "activations": "uniform [0, 2^20) int32 Q16.16",
                        "l2": f"rotating {n_rot} input/output sets ({n_rot * per_step_bytes / 2**20:.0f} MiB > L2)",
                        "step": "absmax pre-pass + ConvShift (fused bias/saturate epilogue)"},
-            "roofline": {"bound": "alu", "achieved": achieved, "peak": alu_peak, "unit": "Tintop/s",
-                         "frac": achieved / alu_peak, "traffic": NCU_TRAFFIC_BYTES,
+            "roofline": {"bound": "alu", "achieved": achieved, "peak": alu_tops, "unit": "Tintop/s",
+                         "frac": achieved / alu_tops, "traffic": NCU_TRAFFIC_BYTES,
                          "kernel": "conv_direct_kernel<1,3,7,0>", "kernel_ms": kern_ms,
-                         "peak_basis": f"{SMS} SMs x {INT_OPS_PER_CLK_PER_SM} int32 ops/clk x {sm_max:.0f} MHz "
+                         "peak_basis": f"{sms} SMs x {INT_OPS_PER_CLK_PER_SM} int32 ops/clk x {sm_max:.0f} MHz "
                                        f"(sm_max_mhz, {peak_kind})",
                          "alg_int_ops_per_launch": ALG_INT_OPS_PER_TERM * wl["terms"],
                          "hbm_gbs": alg_bytes / (kern_ms / 1e3) / 1e9,

@@ -54,7 +54,8 @@ typedef enum {
  * kernel's first launch: drive one GPU per process (one process per GPU, as
  * the multi-GPU replicas do).  A launch on a second device from the same
  * process is not supported; it fails with DS_ERR_CUDA rather than computing
- * anything wrong. */
+ * anything wrong.  The device's SM count, which sizes grids, split
+ * reductions and cluster choices, is likewise read once per process. */
 
 /* Size limits.  Every size the library forms from caller dimensions is
  * bounded before it can overflow 64 bits.  A code matrix holds at most 2^48
@@ -211,8 +212,11 @@ ds_status ds_expand_shift_weights_bf16(ds_weights* w, void* buf, size_t bytes, v
 ds_status ds_linear_shift_bf16(const uint16_t* x, const ds_weights* w, const float* bias, float* y, int64_t M,
                                int64_t K, int64_t N, uint32_t flags, void* stream);
 
-/* 1 if a bounded wait of the float kernel gave up (a fault record; 0 normally, -1 if unreadable; a library
- * utility: no counterpart in the paper). */
+/* 1 if a bounded wait of the float kernel gave up in any ds_linear_shift_bf16 launch since the previous call of
+ * this function (or since the library loaded), 0 if none did, -1 if the flag could not be read.  Reading clears
+ * the flag.  The flag is device-wide and not per call: synchronise the streams of the calls it should cover
+ * first (the read itself is a synchronous copy).  A launch whose wait gave up stops early, so its y is
+ * incomplete.  A library utility: no counterpart in the paper. */
 int ds_bf16_fault_flag(void);
 
 /* ---------------------------------------------------------------------------

@@ -53,7 +53,8 @@ __global__ void avgpool_floor_kernel(const int32_t* __restrict__ x, int32_t* __r
 
 static int64_t pool_blocks(int64_t total, int threads) {
   int64_t b = (total + threads - 1) / threads;
-  return b > 152 * 32 ? 152 * 32 : (b < 1 ? 1 : b);
+  const int64_t cap = (int64_t)(sm_count() > 0 ? sm_count() : 1) * 32;  // grid-stride beyond 32 CTAs per SM
+  return b > cap ? cap : (b < 1 ? 1 : b);
 }
 
 cudaError_t launch_maxpool(const int32_t* x, int32_t* y, int64_t planes, int H, int W, int OH, int OW, int R,

@@ -38,7 +38,8 @@ constexpr int NT = 32;                  // output channels per CTA
 constexpr int CG = NT / TN;             // channel groups per CTA
 constexpr int kMaxThreads = 256;        // 8 warps: every SM sub-partition gets the same share
 constexpr int kSmemBudget = 74 * 1024;  // 3 CTAs per SM
-constexpr int kSlots = 152 * 3;         // resident CTAs on a GB300
+// resident CTAs of the device (3 per SM)
+inline int64_t slots() { return (int64_t)sm_count() * 3; }
 constexpr int kMaxCluster = 16;         // CTAs per thread-block cluster (non-portable maximum)
 
 // The CTA tiles run over the stacked output rows gr = n * OH + oh of all
@@ -608,7 +609,7 @@ bool choose_geom(const GemmParams& p, size_t split_capacity, Choice& ch) {
   const int64_t ctas = (int64_t)((p.OW + ch.TM * G.GW - 1) / (ch.TM * G.GW)) * tiles_h * ((p.cols + NT - 1) / NT);
   // A grid that does not fill every SM slot once splits its stages over the
   // CTAs of a cluster: then use stages small enough that every rank gets one.
-  const int target = (int)std::min<int64_t>(kMaxCluster, ctas < kSlots ? kSlots / std::max<int64_t>(ctas, 1) : 1);
+  const int target = (int)std::min<int64_t>(kMaxCluster, ctas < slots() ? slots() / std::max<int64_t>(ctas, 1) : 1);
   if (allow_cluster && target >= 2 && (p.C + cc - 1) / cc < target) {
     int want = std::max(1, p.C / target);
     for (int d = want; d >= 1; --d)
@@ -647,8 +648,8 @@ bool choose_geom(const GemmParams& p, size_t split_capacity, Choice& ch) {
     G.splits = G.cluster;
   } else {
     const size_t need = (size_t)p.rows * p.cols * sizeof(int64_t);
-    if (split_capacity >= need && ctas < kSlots && G.n_stages > 1) {
-      int want = (int)std::min<int64_t>(G.n_stages, (2 * kSlots + ctas - 1) / ctas);
+    if (split_capacity >= need && ctas < slots() && G.n_stages > 1) {
+      int want = (int)std::min<int64_t>(G.n_stages, (2 * slots() + ctas - 1) / ctas);
       G.stages_per_split = (G.n_stages + want - 1) / want;
       G.splits = (G.n_stages + G.stages_per_split - 1) / G.stages_per_split;
     }
@@ -740,7 +741,7 @@ cudaError_t launch_direct(const GemmParams& p, const DirectGeom& G0, cudaStream_
     int cs = 1;
     if constexpr (has_cluster_variant(S, TM)) {
       const int64_t tiles = (int64_t)G.tiles_w * G.tiles_h * ((p.cols + NT - 1) / NT);
-      int64_t best = ((tiles + kSlots - 1) / kSlots) * G.n_stages;
+      int64_t best = ((tiles + slots() - 1) / std::max<int64_t>(slots(), 1)) * G.n_stages;
       for (int c = 2; c <= std::min(kMaxCluster, G.n_stages); ++c) {
         const int n = max_clusters<SIG, S, TM>(c, launch_smem_bytes(G, TM));
         if (n <= 0) continue;
@@ -825,7 +826,7 @@ cudaError_t prepare_split_scratch(const GemmParams& p, cudaStream_t st) {
 cudaError_t launch_split_finalize(const GemmParams& p, cudaStream_t st) {
   const int64_t total = p.rows * p.cols;
   int64_t blocks = (total + 255) / 256;
-  if (blocks > kSlots * 8) blocks = kSlots * 8;
+  if (blocks > std::max<int64_t>(slots(), 1) * 8) blocks = std::max<int64_t>(slots(), 1) * 8;
   conv_split_finalize_kernel<<<(unsigned)blocks, 256, 0, st>>>(p, total);
   return cudaGetLastError();
 }

@@ -36,7 +36,8 @@ constexpr int THREADS = 128;  // PG x (NT / TN)
 constexpr int KC = 16;        // input channels per stage (half of a packed 32-index chunk)
 constexpr int NB = NT / 32;   // 32-channel blocks of the expanded layout per CTA
 constexpr int QUADS = MT / 4;
-constexpr int kSlots = 152 * 4;  // resident CTAs on a GB300
+// resident CTAs of the device (4 per SM)
+inline int64_t slots() { return (int64_t)sm_count() * 4; }
 static_assert(PG * (NT / TN) == THREADS && THREADS % QUADS == 0, "tile shape");
 
 struct __align__(16) PwSmem {
@@ -351,8 +352,8 @@ int pw_stages_per_split(const GemmParams& p, size_t split_capacity) {
   const int n_stages = (p.C + KC - 1) / KC;
   const int64_t ctas = ((p.rows + MT - 1) / MT) * ((p.cols + NT - 1) / NT);
   const size_t need = (size_t)p.rows * p.cols * sizeof(int64_t);
-  if (split_capacity < need || ctas >= kSlots || n_stages < 2) return n_stages;
-  const int want = (int)std::min<int64_t>(n_stages, (2 * kSlots + ctas - 1) / ctas);
+  if (split_capacity < need || ctas >= slots() || n_stages < 2) return n_stages;
+  const int want = (int)std::min<int64_t>(n_stages, (2 * slots() + ctas - 1) / ctas);
   return (n_stages + want - 1) / want;
 }
 

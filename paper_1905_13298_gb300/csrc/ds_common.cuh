@@ -136,6 +136,10 @@ ds_status fc_launch(const int32_t* x, const ds_weights* w, const int32_t* bias, 
 cudaError_t launch_quantize_weights(const float* w, int64_t n, int p_min, int8_t* s, int8_t* p, cudaStream_t st);
 cudaError_t launch_quantize_q16(const float* x, int64_t n, int32_t* q, cudaStream_t st);
 // Defined in misc_kernels.cu.
+// Streaming multiprocessors of the device this process uses, read once per
+// process (one device per process); 0 when no device can be queried, in which
+// case the grid heuristics plan no split reduction and no launch succeeds.
+int sm_count();
 cudaError_t launch_absmax(const int32_t* x, int64_t n, uint32_t* out, cudaStream_t st);
 // bwd != nullptr: pack one phase of the input-gradient codes of forward codes
 // [K][C][R][S]: bwd = {K, C, R, S, sh, sw, a, b, Th, Tw}; column c, index

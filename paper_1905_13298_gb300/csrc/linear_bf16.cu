@@ -428,8 +428,11 @@ cudaError_t launch_linear_bf16(const uint16_t* x, const uint16_t* w16, const flo
 }
 
 int read_bf16_fault_flag() {
+  // read, then clear: the flag covers the float calls since the previous read
   int v = 0;
   if (cudaMemcpyFromSymbol(&v, g_bf16_fault, sizeof(int)) != cudaSuccess) return -1;
+  const int zero = 0;
+  if (v != 0 && cudaMemcpyToSymbol(g_bf16_fault, &zero, sizeof(int)) != cudaSuccess) return -1;
   return v;
 }
 

@@ -49,7 +49,8 @@ constexpr int THREADS = 128;  // 8 row groups x 16 column groups
 constexpr int KC = 16;        // reduction indices per stage (half of a packed 32-index chunk)
 constexpr int CW = 2 * 64;    // code words per k: 2 blocks of {32 shifts, 32 signs}
 constexpr int kMinBlocks = 5;
-constexpr int kSlots = 152 * kMinBlocks;  // resident CTAs on a GB300
+// resident CTAs of the device (kMinBlocks per SM)
+inline int64_t slots() { return (int64_t)sm_count() * kMinBlocks; }
 constexpr int kMaxCluster = 16;
 
 template <int TMR>
@@ -411,7 +412,7 @@ cudaError_t launch_tmr(const GemmParams& p, cudaStream_t st) {
   // a wave is the number of clusters the device holds at once (trailing
   // slices may still be empty)
   const int64_t cs_max = std::max<int64_t>(
-      std::min<int64_t>(std::min<int64_t>(kSlots / std::max<int64_t>(tiles, 1), kMaxCluster), stages), 1);
+      std::min<int64_t>(std::min<int64_t>(slots() / std::max<int64_t>(tiles, 1), kMaxCluster), stages), 1);
   int64_t cs = 0, best = 0;
   for (int64_t c = 1; c <= cs_max; ++c) {
     const int n = active_clusters<TMR, XV>((int)c);
@@ -451,7 +452,7 @@ cudaError_t launch_xv(const GemmParams& p, cudaStream_t st) {
 bool linear_cluster_preferred(const GemmParams& p) {
   // the 128 x 64 tiles of shift_gemm.cu would not fill the SMs three times over
   const int64_t gemm_ctas = ((p.rows + 127) / 128) * ((p.cols + NT - 1) / NT);
-  return gemm_ctas < 3 * 152 && (p.cols + NT - 1) / NT <= 65535 && (p.rows + 7) / 8 <= (int64_t)INT32_MAX;
+  return gemm_ctas < 3 * (int64_t)sm_count() && (p.cols + NT - 1) / NT <= 65535 && (p.rows + 7) / 8 <= (int64_t)INT32_MAX;
 }
 
 cudaError_t launch_linear_cluster(const GemmParams& p, cudaStream_t st) {

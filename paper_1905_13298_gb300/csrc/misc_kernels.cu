@@ -164,10 +164,9 @@ __global__ void absmax_kernel(const int32_t* __restrict__ x, int64_t n, uint32_t
   }
 }
 
-cudaError_t launch_absmax(const int32_t* x, int64_t n, uint32_t* out, cudaStream_t st) {
-  cudaError_t e = cudaMemsetAsync(out, 0, sizeof(uint32_t), st);
-  if (e != cudaSuccess) return e;
-  // the SM count, read once per process (thread-safe function-local static)
+int sm_count() {
+  // read once per process (thread-safe function-local static); the library
+  // serves one device per process
   static const int sms = [] {
     int dev = 0, n = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) !=
@@ -177,7 +176,14 @@ cudaError_t launch_absmax(const int32_t* x, int64_t n, uint32_t* out, cudaStream
     }
     return n;
   }();
-  if (sms <= 0) return cudaErrorInvalidDevice;
+  return sms;
+}
+
+cudaError_t launch_absmax(const int32_t* x, int64_t n, uint32_t* out, cudaStream_t st) {
+  const int sms = sm_count();
+  if (sms <= 0) return cudaErrorNoDevice;
+  cudaError_t e = cudaMemsetAsync(out, 0, sizeof(uint32_t), st);
+  if (e != cudaSuccess) return e;
   const int threads = 256;
   int64_t want = (n / 16 + threads - 1) / threads;
   int64_t blocks = want < (int64_t)sms * 4 ? want : (int64_t)sms * 4;

@@ -19,6 +19,10 @@ constexpr int kStaticScratchWords = 64;
 constexpr int kWordsPerCall = 2;
 static __device__ __align__(256) uint32_t g_static_scratch[kStaticScratchWords];
 
+// The address is cached per device ordinal so that it is right for whichever
+// device is current.  The rest of the library still serves one device per
+// process (deepshift.h, "Devices"): the grid heuristics read the SM count of
+// the first device once, so use this entry point on one device per process.
 constexpr int kMaxDevices = 64;
 std::mutex g_mutex;
 uint32_t* g_scratch_addr[kMaxDevices] = {nullptr};

@@ -21,7 +21,6 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kBlocksPerSm = 8;
-constexpr int kSms = 152;
 constexpr int kUnroll = 4;  // independent 16-byte loads in flight per thread
 
 struct Code {
@@ -117,7 +116,7 @@ __global__ void __launch_bounds__(kThreads) quantize_q16_kernel(const float* __r
 
 unsigned grid_for(int64_t n) {
   const int64_t want = (n / 4 + (int64_t)kThreads * kUnroll - 1) / ((int64_t)kThreads * kUnroll);
-  const int64_t cap = (int64_t)kSms * kBlocksPerSm;
+  const int64_t cap = (int64_t)(sm_count() > 0 ? sm_count() : 1) * kBlocksPerSm;
   return (unsigned)(want < 1 ? 1 : (want > cap ? cap : want));
 }
 

@@ -3,11 +3,20 @@
 ds_linear_shift_static_scratch serves callers that cannot allocate device
 memory (a plugin handed only its buffers, a host callback, a real-time path):
 its two scratch words live in a static device array of the library.  These
-checks call it through the C ABI and compare it with ds_linear_shift, which
-takes caller-allocated scratch, on two calls in a row.  The second call uses
-inputs with a different max|x| so that a stale value left in the shared array
-by the first call would show up.  This file is collected last so that a run
-that stops at the first failure has already run every other test.
+checks call it through the C ABI on three calls in a row and compare every
+output with ds_linear_shift (caller-allocated scratch) and with the CPU
+oracle.
+
+The calls alternate small and full-range activations (small, full range,
+small), so each call runs after one whose max|x| differs from its own.  What
+they check is output parity after any history of the shared array.  They do
+not observe the array itself: the pre-pass folds max|x| in with a max, so a
+leftover value can only be larger than the true one, which selects the 64-bit
+path, and that path is exact too.  A leftover value therefore cannot change
+an output.
+
+This file is collected last so that a run that stops at the first failure
+has already run every other test.
 """
 import ctypes
 
@@ -16,6 +25,7 @@ import pytest
 import torch
 
 import synth_inputs as si
+from oracle import deepshift_oracle as O
 
 pytestmark = pytest.mark.gpu
 
@@ -36,9 +46,11 @@ def test_static_scratch_matches_allocating_entry_point(dslib):
     L = ds.lib()
     stream = torch.cuda.current_stream().cuda_stream
     M, K, N = 150, 300, 70
-    # call 1: full-range activations (64-bit path); call 2: small activations (32-bit path)
-    cases = [si.fc_layer(41, M, K, N, -(1 << 31), 1 << 31), si.fc_layer(42, M, K, N, -(1 << 20), 1 << 20)]
-    for flags, (x, s, p, b) in zip((ds.DS_RELU, 0), cases):
+    # small activations (32-bit path), full-range ones (64-bit path), small again
+    cases = [(0, si.fc_layer(42, M, K, N, -(1 << 20), 1 << 20)),
+             (ds.DS_RELU, si.fc_layer(41, M, K, N, -(1 << 31), 1 << 31)),
+             (ds.DS_RELU, si.fc_layer(43, M, K, N, -(1 << 18), 1 << 18))]
+    for flags, (x, s, p, b) in cases:
         w = ds.pack_shift_weights(_dev(s), _dev(p))
         xd, bd = _dev(x), _dev(b)
         want = _reference(ds, xd, w, bd, M, K, N, flags)
@@ -49,6 +61,7 @@ def test_static_scratch_matches_allocating_entry_point(dslib):
         torch.cuda.synchronize()
         # integer path: the tolerance of every parity test here is bit-exact
         assert torch.equal(y, want)
+        assert np.array_equal(y.cpu().numpy(), O.linear_shift(x, s, p, b, relu=bool(flags & ds.DS_RELU)))
 
 
 def test_static_scratch_rejects_amax_flags(dslib):
