@@ -207,6 +207,34 @@ def cpu_baseline(wl, n_images: int | None = None):
                       f"{dt:.1f} s"}
 
 
+def _oracle_images(job):
+    """Worker of the all-cores oracle timing: the oracle on a slice of the batch (one process per core)."""
+    x, s, p, b, stride, pad = job
+    from oracle import deepshift_oracle as O
+    return O.conv2d_shift(x, s, p, b, (stride, stride), (pad, pad)).shape[0]
+
+
+def cpu_baseline_all_cores(wl, cores: int | None = None):
+    """The same oracle on the whole batch, one process per host core, each on its share of the images (the
+    oracle itself is single-threaded numpy).  Spawned processes (never forked after CUDA is initialised); the
+    pool is started and warmed up before the timed region."""
+    import multiprocessing as mp
+    cores = cores or os.cpu_count() or 1
+    x, s, p, b = si.conv_layer(si.SEED_BASE + 2, wl["N"], wl["C"], wl["H"], wl["W"], wl["K"], wl["R"], wl["S"])
+    n_proc = min(cores, wl["N"])
+    bounds = np.linspace(0, wl["N"], n_proc + 1).astype(int)
+    jobs = [(x[lo:hi], s, p, b, wl["stride"], wl["pad"]) for lo, hi in zip(bounds[:-1], bounds[1:]) if hi > lo]
+    with mp.get_context("spawn").Pool(n_proc) as pool:
+        pool.map(_oracle_images, [(x[:1, :, :4, :4], s, p, b, wl["stride"], wl["pad"])] * n_proc)  # warm-up
+        t0 = time.perf_counter()
+        done = sum(pool.map(_oracle_images, jobs))
+        dt = time.perf_counter() - t0
+    assert done == wl["N"]
+    return {"value": wl["terms"] / dt / 1e9, "unit": METRIC, "cores": n_proc, "kind": "oracle",
+            "sample": f"all {wl['N']} images, one spawned process per core ({n_proc} of nproc {os.cpu_count()}), "
+                      f"{dt:.1f} s"}
+
+
 def run_reference(args, wl, rank, world):
     if rank != 0:
         return
@@ -443,7 +471,10 @@ def run_layer_sweep(args, wl, local_rank):
     rows = []
     tot_terms = tot_ms = 0.0
     bwd = bool(wl.get("backward"))
+    only = {int(v) for v in args.layers.split(",")} if args.layers else None
     for i, sp in enumerate(specs):
+        if only is not None and i not in only:
+            continue
         if sp.op == ds.DS_OP_FC:
             r = time_fc_layer(args, ds, dev, si.SEED_BASE + 5 + i, B, sp.C * sp.H * sp.W, sp.K, backward=bwd)
             r["layer"] = i
@@ -510,6 +541,82 @@ def run_layer_sweep(args, wl, local_rank):
            "config": {"workload": wl["name"], "layers": [{k: (round(v, 4) if isinstance(v, float) else v)
                                                           for k, v in r.items()} for r in rows]}}
     print(json.dumps(out), flush=True)
+
+
+def resnet18_forward_record(args, dev):
+    """ms / forward and Gshift-ops/s of the ResNet18-architecture forward at 224 x 224 (every conv and FC a
+    shift layer, per-layer centred codes), batch 32 and batch 1, on device-resident inputs."""
+    import torch
+    from paper_1905_13298_gb300 import networks as PN
+    specs, shapes = PN.resnet_program("resnet18")
+    params = si.network_params(shapes, si.SEED_BASE + 3)
+    rec = {"workload": "resnet18_shift_forward_224", "unit": "ms/forward"}
+    for batch, graph in ((32, False), (1, True)):
+        net = PN.ShiftNetwork(specs, params, batch=batch, device=dev, expand=True)
+        xd = torch.from_numpy(si.image_batch(si.SEED_BASE + 3, batch)).to(dev)
+        y = torch.empty(net.out_shape, dtype=torch.int32, device=dev)
+
+        def fwd():
+            net.forward(xd, y, torch.cuda.current_stream().cuda_stream)
+        for _ in range(max(3, args.warmup)):
+            fwd()
+        torch.cuda.synchronize()
+        run = fwd
+        if graph:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, capture_error_mode="relaxed"):
+                fwd()
+            torch.cuda.synchronize()
+            run = g.replay
+        reps = 20 if batch > 1 else 200
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            run()
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / reps
+        terms = PN.shift_terms(specs, batch)
+        alu_tops = alu_peak(dev)[0]
+        rec[f"batch{batch}"] = {"ms_per_forward": ms, "gshift_ops_per_s": terms / ms / 1e6,
+                                "frac": 2 * terms / (ms / 1e3) / (alu_tops * 1e12), "terms": terms,
+                                "kernel_launches": 1 + len(specs), "cuda_graph": graph}
+        del net, xd, y
+    return rec
+
+
+def sustained_record(step, n_rot, wl, dev, local_rank, seconds: float = 2.5):
+    """The default step back to back for a few seconds, clocks sampled meanwhile: Gshift-ops/s, the median SM
+    clock under load, and the roofline fraction both at the maximum clock and at the median one."""
+    import torch
+    for i in range(10):
+        step(i)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for i in range(50):
+        step(i)
+    e1.record()
+    torch.cuda.synchronize()
+    n = max(100, int(seconds * 1e3 / (e0.elapsed_time(e1) / 50)))
+    sampler = ClockSampler(local_rank)
+    sampler.start()
+    time.sleep(0.3)
+    e0.record()
+    for i in range(n):
+        step(i)
+    e1.record()
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    ms = e0.elapsed_time(e1)
+    alu_tops, sms, sm_max, _ = alu_peak(dev)
+    rate = wl["terms"] * n / (ms / 1e3)
+    rec = {"steps": n, "seconds": ms / 1e3, "gshift_ops_per_s": rate / 1e9, "clocks": clocks,
+           "frac": 2 * rate / (alu_tops * 1e12), "l2": f"rotating {n_rot} input/output sets, as the timed steps"}
+    if clocks.get("sm_mhz"):
+        rec["frac_at_median_clock"] = 2 * rate / (sms * INT_OPS_PER_CLK_PER_SM * clocks["sm_mhz"] * 1e6)
+        rec["shift_ops_per_sm_clock"] = rate / (sms * clocks["sm_mhz"] * 1e6)
+    return rec
 
 
 def run_gpu(args, wl, rank, world, local_rank):
@@ -633,6 +740,12 @@ def run_gpu(args, wl, rank, world, local_rank):
     else:
         parity = None
 
+    # The metric's whole-network figure: ResNet18 (224 x 224) chained forward through ds_shift_forward,
+    # batch 32 and batch 1 (CUDA graph replay: at batch 1 a forward is launch bound).
+    resnet18 = resnet18_forward_record(args, dev) if rank == 0 and not args.no_extras else None
+    # A seconds-long back-to-back run of the same step with the clocks sampled under load.
+    sustained = sustained_record(step, n_rot, wl, dev, local_rank) if rank == 0 and not args.no_extras else None
+
     if rank == 0:
         peaks, peak_kind = measured_peaks()
         terms_total = wl["terms"] * args.steps * world
@@ -664,8 +777,13 @@ def run_gpu(args, wl, rank, world, local_rank):
             "clocks": clocks,
             "parity_spot_check": parity,
         }
+        if resnet18 is not None:
+            out["resnet18_forward"] = resnet18
+        if sustained is not None:
+            out["sustained"] = sustained
         if not args.no_cpu_baseline:
             out["cpu_baseline"] = cpu_baseline(wl)
+            out["cpu_baseline"]["all_cores"] = cpu_baseline_all_cores(wl)
         print(json.dumps(out), flush=True)
     if dist:
         dist.destroy_process_group()
@@ -679,9 +797,13 @@ def main():
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--batch", type=int, default=None)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="default workload: skip the ResNet18 forward and sustained-clock sub-records")
     ap.add_argument("--workload", default="conv2x", choices=["conv2x", "fc_large", "fc_vgg16_fc1", "fc_large_bf16", "quantize_vgg16_fc1", "q16_input", "resnet18", "resnet50", "vgg16",
                                                          "sweep_resnet18", "sweep_resnet50", "sweep_vgg16",
                                                          "sweep_resnet18_backward", "sweep_resnet50_backward"])
+    ap.add_argument("--layers", default=None,
+                    help="layer sweeps: comma-separated layer indices of the program to run (default: all)")
     ap.add_argument("--graph", action="store_true", help="replay each step from a CUDA graph (other workloads)")
     args = ap.parse_args()
     rank = int(os.environ.get("RANK", "0"))

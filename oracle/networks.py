@@ -38,6 +38,40 @@ RESNET_STAGES = {"resnet18": ("basic", [2, 2, 2, 2]), "resnet50": ("bottleneck",
 VGG16_CFG = [64, 64, "M", 128, 128, "M", 256, 256, 256, "M", 512, 512, 512, "M", 512, 512, 512, "M"]
 
 
+def layer_shapes(arch: str, H: int = 224, W: int = 224):
+    """Shapes of the shift layers of an architecture, in parameter order: (K, C, R, S) per conv and
+    (n_out, k_in) per FC, as the forwards below consume them."""
+    if arch == "vgg16":
+        shapes, c, h, w = [], 3, H, W
+        for v in VGG16_CFG:
+            if v == "M":
+                h, w = h // 2, w // 2
+            else:
+                shapes.append((v, c, 3, 3))
+                c = v
+        k = c * h * w
+        for n in (4096, 4096, 1000):
+            shapes.append((n, k))
+            k = n
+        return shapes
+    kind, blocks = RESNET_STAGES[arch]
+    shapes, c = [(64, 3, 7, 7)], 64
+    for stage, nb in enumerate(blocks):
+        for bi in range(nb):
+            stride = 2 if (stage > 0 and bi == 0) else 1
+            planes = 64 * (2 ** stage)
+            out_c = planes if kind == "basic" else planes * 4
+            if kind == "basic":
+                shapes += [(planes, c, 3, 3), (planes, planes, 3, 3)]
+            else:
+                shapes += [(planes, c, 1, 1), (planes, planes, 3, 3), (out_c, planes, 1, 1)]
+            if stride != 1 or c != out_c:
+                shapes.append((out_c, c, 1, 1))
+            c = out_c
+    shapes.append((1000, c))
+    return shapes
+
+
 def _conv(x, prm, stride, pad, relu, residual=None):
     """One ConvShift layer of a chain (Eq. 3, convolutional form; readings R-conv, R-acc), then either the
     residual join ReLU(sat32(y + residual)) or the optional ReLU."""

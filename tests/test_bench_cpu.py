@@ -74,3 +74,11 @@ def test_reference_arm_runs_on_rank_zero_only():
                                 {"RANK": "1", "WORLD_SIZE": "2", "LOCAL_RANK": "1"})
     assert rc == 0, err
     assert lines == []
+
+
+def test_all_cores_oracle_timing_covers_the_batch():
+    """The all-cores CPU baseline splits the batch over spawned processes and times the whole of it."""
+    wl = dict(name="tiny", N=5, C=3, H=6, W=5, K=4, R=3, S=3, stride=1, pad=1, terms=5 * 4 * 6 * 5 * 3 * 9)
+    r = bench.cpu_baseline_all_cores(wl, cores=2)
+    assert r["kind"] == "oracle" and r["cores"] == 2 and r["value"] > 0 and r["unit"] == bench.METRIC
+    assert "all 5 images" in r["sample"]

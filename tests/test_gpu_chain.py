@@ -157,3 +157,45 @@ def test_split_scratch_large_then_small_layers(dslib):
         y = net.forward(xd)
         torch.cuda.synchronize()
         assert np.array_equal(y.cpu().numpy().reshape(4, -1), want)
+
+
+def _stored_logits():
+    """Oracle logits of the full-size forwards (tests/golden/network_outputs_224.txt, written by
+    tests/golden/make_network_outputs.py with oracle/networks.py): (arch, batch, image) -> (digests, logits)."""
+    import os
+    path = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "network_outputs_224.txt")
+    out = {}
+    with open(path) as f:
+        for line in f:
+            if line.startswith("#") or not line.strip():
+                continue
+            v = line.split()
+            out[(v[0], int(v[1]), int(v[2]))] = ((v[3], v[4]), np.array([int(t) for t in v[5:]], dtype=np.int64))
+    return out
+
+
+def _digests(x, params):
+    import hashlib
+    hx = hashlib.sha256(np.ascontiguousarray(x).tobytes()).hexdigest()[:16]
+    h = hashlib.sha256()
+    for s, p, b in params:
+        for a in (s, p, b):
+            h.update(np.ascontiguousarray(a).tobytes())
+    return hx, h.hexdigest()[:16]
+
+
+@pytest.mark.parametrize("arch,batch", [("resnet18", 32), ("resnet50", 64), ("vgg16", 64)])
+def test_full_size_chain_first_and_last_image(dslib, arch, batch):
+    """The benchmarked chained forwards at full size (224 x 224; ResNet18 at batch 32, ResNet50 and VGG16 at
+    batch 64), run as the benchmark runs them (one ds_shift_forward over the whole batch, expanded codes): the
+    first and the last image's 1000 logits equal the oracle's, element by element."""
+    from paper_1905_13298_gb300 import networks as PN
+    prog = PN.resnet_program(arch) if arch != "vgg16" else PN.vgg16_program()
+    params = si.network_params(prog[1], si.SEED_BASE + 3)
+    x = si.image_batch(si.SEED_BASE + 3, batch)
+    stored = _stored_logits()
+    y = _run(prog, params, x)
+    for image in (0, batch - 1):
+        digests, want = stored[(arch, batch, image)]
+        assert _digests(x[image:image + 1], params) == digests, "stale fixture: regenerate the stored logits"
+        assert np.array_equal(y[image], want), image

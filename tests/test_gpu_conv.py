@@ -136,15 +136,20 @@ def test_conv_config2_two_images_full(dslib, expand):
     assert np.array_equal(got, want)
 
 
+_CONFIG2_ORACLE = {}
+
+
+def _config2_oracle(x, s, p, b):
+    """The oracle on the whole N = 32 batch (about 15 s), computed once per session."""
+    if "y" not in _CONFIG2_ORACLE:
+        _CONFIG2_ORACLE["y"] = O.conv2d_shift(x, s, p, b, (1, 1), (1, 1))
+    return _CONFIG2_ORACLE["y"]
+
+
 @pytest.mark.parametrize("expand", [False, True])
-def test_conv_config2_full_batch_sampled(dslib, expand):
-    """The full N = 32 launch (as timed by the benchmark); sampled outputs checked one by one."""
+def test_conv_config2_full_batch_every_output(dslib, expand):
+    """The full N = 32 launch as the benchmark times it (the expanded layout; the packed blob too): every one
+    of the 6.4 M outputs against the oracle."""
     x, s, p, b = si.config2()
     got, _ = _run(dslib, x, s, p, b, (1, 1), (1, 1), expand=expand)
-    rng = np.random.default_rng(1)
-    pts = [(0, 0, 0, 0), (31, 63, 55, 55), (5, 7, 0, 55), (17, 40, 55, 0)]
-    pts += [tuple(int(v) for v in (rng.integers(32), rng.integers(64), rng.integers(56), rng.integers(56)))
-            for _ in range(40)]
-    for (n, k, oh, ow) in pts:
-        want = O.conv2d_shift_at(x, s, p, b, (1, 1), (1, 1), n, k, oh, ow)
-        assert got[n, k, oh, ow] == max(min(want, O.INT32_MAX), O.INT32_MIN), (n, k, oh, ow)
+    assert np.array_equal(got, _config2_oracle(x, s, p, b))

@@ -146,10 +146,13 @@ def test_linear_shift_amax_in_is_used(dslib):
     assert np.array_equal(y.cpu().numpy(), O.linear_shift(x, s, p, b))
 
 
-def test_linear_shift_config4_sampled(dslib):
-    """Full-size 8192 x 4096 x 4096 launch; sampled outputs checked one by one."""
+@pytest.mark.parametrize("expand", [False, True])
+def test_linear_shift_config4_sampled(dslib, expand):
+    """Full-size 8192 x 4096 x 4096 launch (the expanded layout is the one the benchmark times); sampled
+    outputs checked one by one, and 24 whole rows (tile edges, the last row, random rows) against the
+    vectorised oracle."""
     x, s, p, b = si.config4_int()
-    w = _pack(dslib, s, p)
+    w = _pack(dslib, s, p, expand=expand)
     amax_io = torch.zeros(2, dtype=torch.int32, device="cuda")
     y = dslib.linear_shift(_dev(x), w, _dev(b), amax_io=amax_io).cpu().numpy()
     rng = np.random.default_rng(0)
@@ -158,6 +161,6 @@ def test_linear_shift_config4_sampled(dslib):
     for m, n in zip(rows, cols):
         want = O.linear_shift_at(x, s, p, b, int(m), int(n))
         assert y[m, n] == max(min(want, O.INT32_MAX), O.INT32_MIN)
-    # whole rows against the vectorised oracle
-    for m in (0, 4097):
-        assert np.array_equal(y[m:m + 1], O.linear_shift(x[m:m + 1], s, p, b))
+    whole = [0, 127, 128, 4095, 4096, 4097, 8064, 8191] + [int(v) for v in rng.integers(0, 8192, 16)]
+    for m in whole:
+        assert np.array_equal(y[m:m + 1], O.linear_shift(x[m:m + 1], s, p, b)), m

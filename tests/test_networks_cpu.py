@@ -72,3 +72,14 @@ def test_vgg16_terms_and_layers():
     assert _vgg16_per_image() == 15_470_264_320
     assert PN.shift_terms(specs, 64) == 64 * _vgg16_per_image()
     assert _counts(specs) == (13, 3)
+
+
+def test_programs_and_oracle_agree_on_layer_shapes():
+    """The layer programs the library runs and the oracle's architectures (which write the stored full-size
+    logits) list the same shift layers, in the same parameter order, at every image size the tests use."""
+    from oracle import networks as ON
+    for arch in ("resnet18", "resnet50"):
+        for hw in ((224, 224), (64, 64), (32, 32)):
+            assert [tuple(s) for s in PN.resnet_program(arch, *hw)[1]] == ON.layer_shapes(arch, *hw)
+    for hw in ((224, 224), (32, 32)):
+        assert [tuple(s) for s in PN.vgg16_program(*hw)[1]] == ON.layer_shapes("vgg16", *hw)
