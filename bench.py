@@ -57,6 +57,12 @@ def workload_by_name(name: str, batch):
         M, K, N = batch or 64, 25088, 4096
         return dict(name=f"fc_shift_vgg16_fc1_b{M}_int32", kind="fc", M=M, K=K, Nout=N, terms=M * K * N,
                     centred=True)
+    if name == "pack_vgg16_fc1":
+        # int8 sign and shift codes of VGG16's first FC layer -> the 6-bit packed blob (weight packing)
+        n_out, k_red = 4096, 25088
+        n = n_out * k_red
+        return dict(name="pack_weights_vgg16_fc1_4096x25088", kind="pack", n=n, n_out=n_out, k_red=k_red,
+                    bytes=2 * n + n * 3 // 4 + 12 * n_out)
     if name == "quantize_vgg16_fc1":
         # float32 weights of VGG16's first FC layer -> int8 sign and shift codes (DeepShift-Q)
         n = 4096 * 25088
@@ -372,7 +378,20 @@ def run_conversion(args, wl, local_rank):
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
     n = wl["n"]
-    if wl["kind"] == "quant":
+    sync_call = False
+    if wl["kind"] == "pack":
+        shp = (wl["n_out"], wl["k_red"])
+        sd = torch.from_numpy(si.sign_codes(si.SEED_BASE + 48, shp)).to(dev)
+        pd = torch.from_numpy(si.shift_codes_uniform(si.SEED_BASE + 48, shp)).to(dev)
+        nb = ds.ds_packed_weight_bytes(*shp)
+        blob = torch.empty(nb, dtype=torch.uint8, device=dev)
+
+        def step():  # synchronous: the call waits for the pack to read the code-range verdict
+            ds.ds_pack_shift_weights(sd, pd, wl["n_out"], wl["k_red"], blob, nb,
+                                     torch.cuda.current_stream().cuda_stream)
+        kernel = "pack_kernel + pack_maxima_kernel (+ blob memset)"
+        sync_call = True
+    elif wl["kind"] == "quant":
         src = torch.from_numpy(si.float_weights(si.SEED_BASE + 46, (n,), -18, 1)).to(dev)
         s = torch.empty(n, dtype=torch.int8, device=dev)
         p = torch.empty(n, dtype=torch.int8, device=dev)
@@ -395,24 +414,29 @@ def run_conversion(args, wl, local_rank):
     sampler.start()
     time.sleep(0.3)
     torch.cuda.synchronize()
+    t0 = time.perf_counter()
     e0.record()
     for _ in range(args.steps):
         step()
     e1.record()
     torch.cuda.synchronize()
+    t1 = time.perf_counter()
     clocks = sampler.stop()
-    ms = e0.elapsed_time(e1) / args.steps
+    # a synchronous call is timed as its caller sees it (host clock, its wait included)
+    ms = (t1 - t0) * 1e3 / args.steps if sync_call else e0.elapsed_time(e1) / args.steps
     gbs = wl["bytes"] / (ms / 1e3) / 1e9
     peaks, src_name = measured_peaks()
     peak = float(peaks.get("hbm_gbs", 6800.0))
     out = {"metric": "GB/s", "value": gbs, "unit": "GB/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
            "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-           "dtype": "f32->int8" if wl["kind"] == "quant" else "f32->int32", "data": "synthetic",
+           "dtype": {"quant": "f32->int8", "q16": "f32->int32", "pack": "int8->u8"}[wl["kind"]], "data": "synthetic",
            "config": {"workload": wl["name"], "elements": n, "bytes_per_step": wl["bytes"],
                       "l2": "inputs and outputs larger than L2"},
            "roofline": {"bound": "hbm", "achieved": gbs, "peak": peak, "unit": "GB/s", "frac": gbs / peak,
                         "traffic": None, "kernel": kernel, "peak_basis": f"hbm_gbs, {src_name}"},
-           "gpu_launches": args.steps, "clocks": clocks}
+           "gpu_launches": args.steps * (2 if wl["kind"] == "pack" else 1), "clocks": clocks}
+    if sync_call:
+        out["config"]["timing"] = "host clock around each synchronous call (memset, two kernels, header read)"
     print(json.dumps(out), flush=True)
 
 
@@ -799,7 +823,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extras", action="store_true",
                     help="default workload: skip the ResNet18 forward and sustained-clock sub-records")
-    ap.add_argument("--workload", default="conv2x", choices=["conv2x", "fc_large", "fc_vgg16_fc1", "fc_large_bf16", "quantize_vgg16_fc1", "q16_input", "resnet18", "resnet50", "vgg16",
+    ap.add_argument("--workload", default="conv2x", choices=["conv2x", "fc_large", "fc_vgg16_fc1", "fc_large_bf16", "pack_vgg16_fc1", "quantize_vgg16_fc1", "q16_input", "resnet18", "resnet50", "vgg16",
                                                          "sweep_resnet18", "sweep_resnet50", "sweep_vgg16",
                                                          "sweep_resnet18_backward", "sweep_resnet50_backward"])
     ap.add_argument("--layers", default=None,
@@ -818,7 +842,7 @@ def main():
         run_gpu(args, wl, rank, world, local_rank)
     elif wl["kind"] == "sweep":
         run_layer_sweep(args, wl, local_rank)
-    elif wl["kind"] in ("quant", "q16"):
+    elif wl["kind"] in ("quant", "q16", "pack"):
         run_conversion(args, wl, local_rank)
     else:
         run_gpu_other(args, wl, rank, world, local_rank)

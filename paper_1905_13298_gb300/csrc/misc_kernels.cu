@@ -7,15 +7,21 @@
 
 namespace ds {
 
-// One thread per output column: walks the column's reduction range chunk by
-// chunk, validates the codes, writes the nibble and bit-plane records and the
-// column constants A[n] and nnz[n], and folds them into the header maxima.
 struct BwdMap {
   int K, C, R, S, sh, sw, a, b, Th, Tw;  // K == 0: forward layout
 };
 
-__global__ void pack_kernel(const int8_t* __restrict__ s, const int8_t* __restrict__ p,
-                            int64_t n_out, int64_t k_red, uint8_t* __restrict__ blob, const BwdMap m) {
+// One warp per (column n, range of 32-index chunks).  Lane j holds code j of
+// a chunk: with the forward layout the warp's two loads are 32 consecutive
+// bytes of row n (coalesced).  The chunk's records come from warp votes (sign
+// and non-zero planes) and an OR over each group of 8 lanes (the four shift
+// words); lane 0 writes them.  Records of consecutive columns are adjacent,
+// and consecutive warps take consecutive columns, so the writes of a block
+// merge.  Per-column constants A[n], nnz[n] and the invalid count are added
+// atomically (the blob starts zeroed); pack_maxima_kernel then folds the
+// columns into the header maxima.
+__global__ void pack_kernel(const int8_t* __restrict__ s, const int8_t* __restrict__ p, int64_t n_out,
+                            int64_t k_red, uint8_t* __restrict__ blob, const BwdMap m, int64_t parts) {
   const BlobLayout L = blob_layout(n_out, k_red);
   BlobHeader* hdr = reinterpret_cast<BlobHeader*>(blob);
   if (blockIdx.x == 0 && threadIdx.x == 0) {
@@ -25,64 +31,116 @@ __global__ void pack_kernel(const int8_t* __restrict__ s, const int8_t* __restri
     hdr->k_red = k_red;
     hdr->n_chunks = L.n_chunks;
   }
-  const int64_t n = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  if (n >= n_out) return;
-  // forward: column n's codes are row n.  Input-gradient phase (m.K > 0):
-  // column n is input channel n, index k = (k_out, t, u) reads the code of tap
-  // (m.a + m.sh (Th-1-t), m.b + m.sw (Tw-1-u)) of (k_out, n)
+  const unsigned full = 0xffffffffu;
+  const int lane = threadIdx.x & 31;
+  const int64_t per = (L.n_chunks + parts - 1) / parts;  // chunks per warp
+  const int64_t units = n_out * parts;
   const int64_t tt = (int64_t)m.Th * m.Tw;
-  auto offset = [&](int64_t k) -> int64_t {
-    if (m.K == 0) return n * k_red + k;
-    const int64_t ko = k / tt, rem = k - ko * tt;
-    const int64_t t = rem / m.Tw, u = rem - t * m.Tw;
-    const int64_t r = m.a + (int64_t)m.sh * (m.Th - 1 - t), q = m.b + (int64_t)m.sw * (m.Tw - 1 - u);
-    return ((ko * m.C + n) * m.R + r) * m.S + q;
-  };
   uint4* nib = reinterpret_cast<uint4*>(blob + L.nib);
   uint2* bits = reinterpret_cast<uint2*>(blob + L.bits);
-  unsigned long long a_sum = 0;
-  uint32_t nnz = 0, invalid = 0;
-  for (int64_t g = 0; g < L.n_chunks; ++g) {
-    uint32_t w[4] = {0u, 0u, 0u, 0u};
-    uint32_t neg = 0u, nz = 0u;
-    for (int j = 0; j < kChunk; ++j) {
-      const int64_t k = g * kChunk + j;
-      if (k >= k_red) break;
-      const int64_t o = offset(k);
-      const int sv = s[o];
-      const int pv = p[o];
-      if (sv < -1 || sv > 1 || pv < -15 || pv > 0) {
-        ++invalid;
-        continue;
+  for (int64_t u = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; u < units;
+       u += ((int64_t)gridDim.x * blockDim.x) >> 5) {
+    const int64_t n = u % n_out;
+    const int64_t g0 = (u / n_out) * per;
+    const int64_t g1 = g0 + per < L.n_chunks ? g0 + per : L.n_chunks;
+    // forward: column n's codes are row n.  Input-gradient phase (m.K > 0):
+    // column n is input channel n, index k = (k_out, t, u) reads the code of
+    // tap (m.a + m.sh (Th-1-t), m.b + m.sw (Tw-1-u)) of (k_out, n)
+    auto offset = [&](int64_t k) -> int64_t {
+      if (m.K == 0) return n * k_red + k;
+      const int64_t ko = k / tt, rem = k - ko * tt;
+      const int64_t t = rem / m.Tw, v = rem - t * m.Tw;
+      const int64_t r = m.a + (int64_t)m.sh * (m.Th - 1 - t), q = m.b + (int64_t)m.sw * (m.Tw - 1 - v);
+      return ((ko * m.C + n) * m.R + r) * m.S + q;
+    };
+    unsigned long long a_sum = 0;
+    uint32_t nnz = 0, invalid = 0;
+#pragma unroll 4
+    for (int64_t g = g0; g < g1; ++g) {
+      const int64_t k = g * kChunk + lane;
+      int sv = 0, pv = 0;
+      const bool in = k < k_red;
+      if (in) {
+        const int64_t o = offset(k);
+        sv = s[o];
+        pv = p[o];
       }
-      w[j >> 3] |= (uint32_t)(-pv) << (4 * (j & 7));
-      if (sv == -1) neg |= 1u << j;
-      if (sv != 0) {
-        nz |= 1u << j;
-        ++nnz;
-        a_sum += 1ull << (15 + pv);
+      const bool bad = in && (sv < -1 || sv > 1 || pv < -15 || pv > 0);
+      const bool ok = in && !bad;
+      const uint32_t neg = __ballot_sync(full, ok && sv == -1);
+      const uint32_t nz = __ballot_sync(full, ok && sv != 0);
+      const uint32_t badm = __ballot_sync(full, bad);
+      uint32_t w = ok ? (uint32_t)(-pv) << (4 * (lane & 7)) : 0u;
+      w |= __shfl_xor_sync(full, w, 1);
+      w |= __shfl_xor_sync(full, w, 2);
+      w |= __shfl_xor_sync(full, w, 4);
+      const uint32_t w1 = __shfl_sync(full, w, 8), w2 = __shfl_sync(full, w, 16), w3 = __shfl_sync(full, w, 24);
+      const uint32_t a = __reduce_add_sync(full, (ok && sv != 0) ? (1u << (15 + pv)) : 0u);  // <= 2^20
+      if (lane == 0) {
+        nib[g * n_out + n] = make_uint4(w, w1, w2, w3);
+        bits[g * n_out + n] = make_uint2(neg, nz);
       }
+      a_sum += a;
+      nnz += (uint32_t)__popc(nz);
+      invalid += (uint32_t)__popc(badm);
     }
-    nib[g * n_out + n] = make_uint4(w[0], w[1], w[2], w[3]);
-    bits[g * n_out + n] = make_uint2(neg, nz);
+    if (lane == 0) {
+      atomicAdd(reinterpret_cast<unsigned long long*>(blob + L.col_a) + n, a_sum);
+      atomicAdd(reinterpret_cast<uint32_t*>(blob + L.nnz) + n, nnz);
+      if (invalid) atomicAdd(&hdr->invalid_count, invalid);
+    }
   }
-  reinterpret_cast<unsigned long long*>(blob + L.col_a)[n] = a_sum;
-  reinterpret_cast<uint32_t*>(blob + L.nnz)[n] = nnz;
-  if (invalid) atomicAdd(&hdr->invalid_count, invalid);
-  atomicMax(&hdr->nnz_max, nnz);
-  atomicMax(&hdr->a_max, a_sum);
+}
+
+// Header maxima over the columns' A[n] and nnz[n].
+__global__ void pack_maxima_kernel(uint8_t* __restrict__ blob, int64_t n_out, int64_t k_red) {
+  const BlobLayout L = blob_layout(n_out, k_red);
+  BlobHeader* hdr = reinterpret_cast<BlobHeader*>(blob);
+  const unsigned long long* A = reinterpret_cast<const unsigned long long*>(blob + L.col_a);
+  const uint32_t* nz = reinterpret_cast<const uint32_t*>(blob + L.nnz);
+  unsigned long long am = 0;
+  uint32_t nm = 0;
+  for (int64_t n = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; n < n_out; n += (int64_t)gridDim.x * blockDim.x) {
+    am = A[n] > am ? A[n] : am;
+    nm = nz[n] > nm ? nz[n] : nm;
+  }
+  nm = __reduce_max_sync(0xffffffffu, nm);
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) {
+    const unsigned long long v = __shfl_xor_sync(0xffffffffu, am, o);
+    am = v > am ? v : am;
+  }
+  if ((threadIdx.x & 31) == 0) {
+    if (nm) atomicMax(&hdr->nnz_max, nm);
+    if (am) atomicMax(&hdr->a_max, am);
+  }
 }
 
 cudaError_t launch_pack(const int8_t* s, const int8_t* p, int64_t n_out, int64_t k_red,
                         uint8_t* blob, cudaStream_t st, const int* bwd) {
-  // zero the whole blob: header counters, and the tail padding stays defined
+  // zero the whole blob: header counters, column constants (added atomically), tail padding
   cudaError_t e = cudaMemsetAsync(blob, 0, (size_t)blob_layout(n_out, k_red).total, st);
   if (e != cudaSuccess) return e;
-  const int threads = 128;
-  const int64_t blocks = (n_out + threads - 1) / threads;
+  const int sms = sm_count();
+  if (sms <= 0) return cudaErrorNoDevice;
   BwdMap m{0, 0, 1, 1, 1, 1, 0, 0, 1, 1};
   if (bwd != nullptr) m = BwdMap{bwd[0], bwd[1], bwd[2], bwd[3], bwd[4], bwd[5], bwd[6], bwd[7], bwd[8], bwd[9]};
-  pack_kernel<<<(unsigned)blocks, threads, 0, st>>>(s, p, n_out, k_red, blob, m);
+  // enough warps for 64 per SM: split each column's chunks into parts when there are few columns
+  const int threads = 256;
+  const int64_t n_chunks = blob_layout(n_out, k_red).n_chunks;
+  const int64_t want = (int64_t)sms * 64;
+  int64_t parts = (want + n_out - 1) / n_out;
+  if (parts > n_chunks) parts = n_chunks;
+  if (parts < 1) parts = 1;
+  const int64_t units = n_out * parts;
+  int64_t blocks = (units + threads / 32 - 1) / (threads / 32);
+  if (blocks > (int64_t)sms * 32) blocks = (int64_t)sms * 32;  // grid-stride beyond
+  pack_kernel<<<(unsigned)blocks, threads, 0, st>>>(s, p, n_out, k_red, blob, m, parts);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  int64_t mb = (n_out + threads - 1) / threads;
+  if (mb > (int64_t)sms * 8) mb = (int64_t)sms * 8;
+  pack_maxima_kernel<<<(unsigned)mb, threads, 0, st>>>(blob, n_out, k_red);
   return cudaGetLastError();
 }
 

@@ -17,7 +17,8 @@ def _pack(ds, s, p, expand=False):
     return ds.pack_shift_weights(_dev(s.astype(np.int8)), _dev(p.astype(np.int8)), expand=expand)
 
 
-@pytest.mark.parametrize("n_out,k_red", [(1, 1), (3, 31), (64, 576), (65, 33), (512, 784), (130, 100)])
+@pytest.mark.parametrize("n_out,k_red", [(1, 1), (3, 31), (64, 576), (65, 33), (512, 784), (130, 100),
+                                         (3, 100000), (1024, 1152), (9, 4129)])
 def test_pack_blob_bitexact(dslib, n_out, k_red):
     seed = n_out * 7919 + k_red
     s = si.sign_codes(seed, (n_out, k_red))
