@@ -17,13 +17,22 @@
 // as one 16-byte store when OH*OW is a multiple of 4.  Accumulator width as
 // in shift_gemm.cu.
 //
-// Split reduction (chained forward, layers whose grid would not fill the
-// SMs, e.g. 2048 input channels on 7x7 maps): grid.z CTAs share a tile's
-// stages and add their exact partial sums into an int64 workspace with
-// 64-bit atomics; the finalize kernel of conv_direct.cu applies the epilogue.
+// Split reduction (layers whose grid would not fill the SMs, e.g. 2048
+// input channels on 7x7 maps, or a 1x1/2 downsample at batch 32): grid.z
+// CTAs share a tile's stages.  With a workspace (the chained forward) they
+// add their exact partial sums into it with 64-bit atomics and the finalize
+// kernel of conv_direct.cu applies the epilogue; without one (a standalone
+// call) the CTAs form a thread-block cluster, and each rank reduces a share
+// of the tile's partial sums over all ranks through distributed shared
+// memory and applies the epilogue itself.
+#include <cooperative_groups.h>
+
 #include <algorithm>
+#include <mutex>
 
 #include "ds_common.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace ds {
 namespace {
@@ -36,6 +45,7 @@ constexpr int THREADS = 128;  // PG x (NT / TN)
 constexpr int KC = 16;        // input channels per stage (half of a packed 32-index chunk)
 constexpr int NB = NT / 32;   // 32-channel blocks of the expanded layout per CTA
 constexpr int QUADS = MT / 4;
+constexpr int kMaxCluster = 16;  // CTAs per thread-block cluster (non-portable maximum)
 // resident CTAs of the device (4 per SM)
 inline int64_t slots() { return (int64_t)sm_count() * 4; }
 static_assert(PG * (NT / TN) == THREADS && THREADS % QUADS == 0, "tile shape");
@@ -167,7 +177,92 @@ __device__ __forceinline__ void compute_stage(const int32_t* xs, const int32_t* 
   }
 }
 
-template <bool STRIDED, int I0, int NI, typename Acc>
+// Output value of an exact (64-bit) or proven-exact (32-bit) sum plus bias:
+// saturated to int32 (the 64-bit path; the 32-bit path cannot leave it).
+template <typename Acc>
+__device__ __forceinline__ int32_t finish_sum(Acc a, int32_t b) {
+  if constexpr (sizeof(Acc) == 4) {
+    return (int32_t)(a + (uint32_t)b);
+  } else {
+    int64_t v = a + (int64_t)b;
+    v = v > (int64_t)INT32_MAX ? (int64_t)INT32_MAX : v;
+    v = v < (int64_t)INT32_MIN ? (int64_t)INT32_MIN : v;
+    return (int32_t)v;
+  }
+}
+
+// Cluster split: this CTA's partial sums go to its shared memory as
+// red[(thread * NI + i) * TN + j]; every rank has the same tile mapping, so
+// entry f of every rank belongs to the same output (pixel slot i of thread
+// f / NI, its channels j).  Rank r sums the entries f = r * THREADS + t
+// (mod cs * THREADS) over all ranks through distributed shared memory (the
+// 32-bit partials are exact whenever the bound holds: each is a subset of the
+// terms) and applies the epilogue.  The second cluster barrier keeps every
+// rank's shared memory alive until the remote reads end.
+template <int I0, int NI, typename Acc>
+__device__ __forceinline__ void cluster_epilogue(const GemmParams& P, PwSmem& sm, int64_t m0, int64_t col0,
+                                                 const Acc (&acc)[NI][TN], uint32_t& amax_local) {
+  static_assert(THREADS * NI * TN * sizeof(Acc) <= sizeof(PwSmem), "partials fit the staging buffers");
+  const int t = threadIdx.x;
+  Acc* red = reinterpret_cast<Acc*>(&sm);
+#pragma unroll
+  for (int i = 0; i < NI; ++i)
+#pragma unroll
+    for (int j = 0; j < TN; ++j) red[(t * NI + i) * TN + j] = acc[i][j];
+  cg::cluster_group cl = cg::this_cluster();
+  cl.sync();  // all partials written
+  const int rank = (int)cl.block_rank();
+  const int cs = (int)cl.num_blocks();
+  const int64_t OHW = (int64_t)P.OH * P.OW;
+  const bool relu = (P.flags & DS_RELU) != 0;
+  const int32_t* resid = (P.flags & DS_RESIDUAL) ? P.residual : nullptr;
+  for (int f = rank * THREADS + t; f < THREADS * NI; f += cs * THREADS) {
+    const int ft = f / NI, i = f - ft * NI;
+    const int li = I0 + i;
+    const int64_t m = m0 + 4 * (ft % PG) + (li & 3) + (MT / 2) * (li >> 2);
+    Acc sum[TN];
+#pragma unroll
+    for (int j = 0; j < TN; ++j) sum[j] = 0;
+    for (int q = 0; q < cs; ++q) {
+      const Acc* src = cl.map_shared_rank(red, q) + f * TN;
+      if constexpr (sizeof(Acc) == 4) {
+#pragma unroll
+        for (int v = 0; v < TN / 4; ++v) {
+          const uint4 w = *reinterpret_cast<const uint4*>(src + 4 * v);
+          sum[4 * v] += w.x;
+          sum[4 * v + 1] += w.y;
+          sum[4 * v + 2] += w.z;
+          sum[4 * v + 3] += w.w;
+        }
+      } else {
+#pragma unroll
+        for (int v = 0; v < TN / 2; ++v) {
+          const longlong2 w = *reinterpret_cast<const longlong2*>(src + 2 * v);
+          sum[2 * v] += w.x;
+          sum[2 * v + 1] += w.y;
+        }
+      }
+    }
+    if (m >= P.rows) continue;
+    const int64_t n = m / OHW;
+    const int64_t base = n * P.cols * OHW + (m - n * OHW);
+    const int64_t c0 = col0 + (ft / PG) * TN;
+#pragma unroll
+    for (int j = 0; j < TN; ++j) {
+      const int64_t col = c0 + j;
+      if (col >= P.cols) break;
+      const int64_t idx = base + col * OHW;
+      int32_t o = finish_sum<Acc>(sum[j], P.bias != nullptr ? __ldg(P.bias + col) : 0);
+      if (resid != nullptr) o = add_sat(o, __ldg(resid + idx));
+      if (relu) o = max(o, 0);
+      amax_local = max(amax_local, uabs(o));
+      P.y[idx] = o;
+    }
+  }
+  cl.sync();  // no rank reuses its shared memory (next pass) or exits while another reads it
+}
+
+template <bool STRIDED, bool CL, int I0, int NI, typename Acc>
 __device__ __forceinline__ void run_tile(const GemmParams& P, PwSmem& sm, int64_t m0, int64_t col0,
                                          const QuadCtx& q, int st_begin, int st_end, uint32_t& amax_local) {
   const int t = threadIdx.x;
@@ -181,11 +276,13 @@ __device__ __forceinline__ void run_tile(const GemmParams& P, PwSmem& sm, int64_
 
   static_assert(KC == 16 && NB == 2 && THREADS == 128, "ExpandedCodeStager's stage shape");
   const ExpandedCodeStager cst(P.xcodes, P.cols, P.kred, col0, (int64_t)st_begin * KC);
-  stage_x<STRIDED>(P, sm.xs[0], q, st_begin * KC);
-  if (expanded) cst.stage(P.xcodes, P.kred, sm.cs[0], 0);
-  cp_async_commit();
-  if (!expanded) decode_codes(P, sm.cs[0], col0, st_begin);
-  cp_async_wait_all();
+  if (st_begin < st_end) {  // a trailing rank of a cluster may have no stage: zero partial sums
+    stage_x<STRIDED>(P, sm.xs[0], q, st_begin * KC);
+    if (expanded) cst.stage(P.xcodes, P.kred, sm.cs[0], 0);
+    cp_async_commit();
+    if (!expanded) decode_codes(P, sm.cs[0], col0, st_begin);
+    cp_async_wait_all();
+  }
   for (int st = st_begin; st < st_end; ++st) {
     const int b = (st - st_begin) & 1;
     const bool more = st + 1 < st_end;
@@ -201,8 +298,12 @@ __device__ __forceinline__ void run_tile(const GemmParams& P, PwSmem& sm, int64_
       cp_async_wait_all();
     }
   }
-  __syncthreads();  // a second pass (64-bit path) reuses the buffers
+  __syncthreads();  // a second pass (64-bit path) or the cluster partials reuse the buffers
 
+  if constexpr (CL) {
+    cluster_epilogue<I0, NI, Acc>(P, sm, m0, col0, acc, amax_local);
+    return;
+  }
   const int64_t OHW = (int64_t)P.OH * P.OW;
   if (P.split_acc != nullptr) {
     // split reduction: exact partial sums (a subset of the terms, so 32-bit
@@ -238,16 +339,7 @@ __device__ __forceinline__ void run_tile(const GemmParams& P, PwSmem& sm, int64_
     const int64_t col = col0 + tn * TN + j;
     bcol[j] = (P.bias != nullptr && col < P.cols) ? __ldg(P.bias + col) : 0;
   }
-  auto finish = [](Acc a, int32_t b) -> int32_t {
-    if constexpr (sizeof(Acc) == 4) {
-      return (int32_t)(a + (uint32_t)b);
-    } else {
-      int64_t v = a + (int64_t)b;
-      v = v > (int64_t)INT32_MAX ? (int64_t)INT32_MAX : v;
-      v = v < (int64_t)INT32_MIN ? (int64_t)INT32_MIN : v;
-      return (int32_t)v;
-    }
-  };
+  auto finish = [](Acc a, int32_t b) -> int32_t { return finish_sum<Acc>(a, b); };
   if (vec) {
 #pragma unroll
     for (int qd = 0; qd < NI / 4; ++qd) {
@@ -322,8 +414,11 @@ __device__ __forceinline__ bool tile_int32_exact(const GemmParams& P, int64_t co
   return !__syncthreads_or(unsafe);
 }
 
-template <bool STRIDED>
-__global__ void __launch_bounds__(THREADS, 4) conv_pointwise_kernel(const GemmParams P, int stages_per_split) {
+// The cluster variant allows 3 CTAs per SM (168 registers): at 4 its reduction
+// epilogue spilled into the hot loop, and it runs only on grids that do not
+// fill the SMs anyway.
+template <bool STRIDED, bool CL>
+__global__ void __launch_bounds__(THREADS, CL ? 3 : 4) conv_pointwise_kernel(const GemmParams P, int stages_per_split) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   PwSmem& sm = *reinterpret_cast<PwSmem*>(smem_raw);
   const int64_t m0 = (int64_t)blockIdx.x * MT;
@@ -334,10 +429,10 @@ __global__ void __launch_bounds__(THREADS, 4) conv_pointwise_kernel(const GemmPa
   const QuadCtx q = quad_ctx<STRIDED>(P, m0);
   uint32_t amax_local = 0;
   if (tile_int32_exact(P, col0)) {
-    run_tile<STRIDED, 0, 8, uint32_t>(P, sm, m0, col0, q, st_begin, st_end, amax_local);
+    run_tile<STRIDED, CL, 0, 8, uint32_t>(P, sm, m0, col0, q, st_begin, st_end, amax_local);
   } else {
-    run_tile<STRIDED, 0, 4, int64_t>(P, sm, m0, col0, q, st_begin, st_end, amax_local);
-    run_tile<STRIDED, 4, 4, int64_t>(P, sm, m0, col0, q, st_begin, st_end, amax_local);
+    run_tile<STRIDED, CL, 0, 4, int64_t>(P, sm, m0, col0, q, st_begin, st_end, amax_local);
+    run_tile<STRIDED, CL, 4, 4, int64_t>(P, sm, m0, col0, q, st_begin, st_end, amax_local);
   }
   if (P.amax_out != nullptr && P.split_acc == nullptr) {
     amax_local = __reduce_max_sync(0xffffffffu, amax_local);
@@ -357,25 +452,106 @@ int pw_stages_per_split(const GemmParams& p, size_t split_capacity) {
   return (n_stages + want - 1) / want;
 }
 
+template <bool STRIDED, bool CL>
+bool set_pw_attributes() {
+  // once per process, thread-safe (see conv_direct.cu)
+  static const bool ok = [] {
+    const bool r = cudaFuncSetAttribute(conv_pointwise_kernel<STRIDED, CL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        (int)sizeof(PwSmem)) == cudaSuccess &&
+                   (!CL || cudaFuncSetAttribute(conv_pointwise_kernel<STRIDED, CL>,
+                                                cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess);
+    if (!r) (void)cudaGetLastError();
+    return r;
+  }();
+  return ok;
+}
+
+// How many clusters of cs CTAs the device holds at once (0: none); queried
+// once per process and size.
+template <bool STRIDED>
+int pw_max_clusters(int cs) {
+  if (cs < 2 || cs > kMaxCluster || !set_pw_attributes<STRIDED, true>()) return 0;
+  static int cache[kMaxCluster + 1] = {0};
+  static std::mutex mu;  // shared by every host thread
+  std::lock_guard<std::mutex> lock(mu);
+  if (cache[cs] != 0) return cache[cs] > 0 ? cache[cs] : 0;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(1, 1, cs);
+  cfg.blockDim = dim3(THREADS, 1, 1);
+  cfg.dynamicSmemBytes = sizeof(PwSmem);
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeClusterDimension;
+  attr.val.clusterDim.x = 1;
+  attr.val.clusterDim.y = 1;
+  attr.val.clusterDim.z = cs;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, conv_pointwise_kernel<STRIDED, true>, &cfg) != cudaSuccess) {
+    (void)cudaGetLastError();
+    n = 0;
+  }
+  cache[cs] = n > 0 ? n : -1;
+  return n > 0 ? n : 0;
+}
+
+// Cluster size of a standalone call whose grid does not fill every SM slot
+// once: the size with the least time, counted as waves x stages per rank
+// (as the direct kernel chooses it); 1: no split.
+template <bool STRIDED>
+int pw_cluster_size(const GemmParams& p) {
+  const int n_stages = (p.C + KC - 1) / KC;
+  const int64_t tiles = ((p.rows + MT - 1) / MT) * ((p.cols + NT - 1) / NT);
+  if (tiles >= slots() || n_stages < 2) return 1;
+  int cs = 1;
+  int64_t best = ((tiles + slots() - 1) / std::max<int64_t>(slots(), 1)) * n_stages;
+  for (int c = 2; c <= std::min(kMaxCluster, n_stages); ++c) {
+    const int n = pw_max_clusters<STRIDED>(c);
+    if (n <= 0) continue;
+    const int64_t cost = ((tiles + n - 1) / n) * ((n_stages + c - 1) / c);
+    if (cost < best) {
+      best = cost;
+      cs = c;
+    }
+  }
+  return cs;
+}
+
 template <bool STRIDED>
 cudaError_t launch_pw(const GemmParams& p, cudaStream_t st) {
   const size_t smem = sizeof(PwSmem);
-  // once per process, thread-safe (see conv_direct.cu)
-  static const cudaError_t attr = cudaFuncSetAttribute(conv_pointwise_kernel<STRIDED>,
-                                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (attr != cudaSuccess) return attr;
+  if (!set_pw_attributes<STRIDED, false>()) return cudaErrorInvalidValue;
   const int n_stages = (p.C + KC - 1) / KC;
   const int sps = pw_stages_per_split(p, p.split_acc ? p.split_capacity : 0);
   const int splits = (n_stages + sps - 1) / sps;
   GemmParams q = p;
+  const dim3 grid1((unsigned)((p.rows + MT - 1) / MT), (unsigned)((p.cols + NT - 1) / NT), 1u);
   if (splits == 1) {
     q.split_acc = nullptr;
+    int cs = pw_cluster_size<STRIDED>(p);
+    const int sps_cl = (n_stages + cs - 1) / cs;
+    cs = (n_stages + sps_cl - 1) / sps_cl;  // every rank gets at least one stage
+    if (cs >= 2) {
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3(grid1.x, grid1.y, (unsigned)cs);
+      cfg.blockDim = dim3(THREADS, 1, 1);
+      cfg.dynamicSmemBytes = smem;
+      cfg.stream = st;
+      cudaLaunchAttribute attr;
+      attr.id = cudaLaunchAttributeClusterDimension;
+      attr.val.clusterDim.x = 1;
+      attr.val.clusterDim.y = 1;
+      attr.val.clusterDim.z = (unsigned)cs;
+      cfg.attrs = &attr;
+      cfg.numAttrs = 1;
+      return cudaLaunchKernelEx(&cfg, conv_pointwise_kernel<STRIDED, true>, q, sps_cl);
+    }
   } else {
     cudaError_t e = prepare_split_scratch(q, st);
     if (e != cudaSuccess) return e;
   }
-  dim3 grid((unsigned)((p.rows + MT - 1) / MT), (unsigned)((p.cols + NT - 1) / NT), (unsigned)splits);
-  conv_pointwise_kernel<STRIDED><<<grid, THREADS, smem, st>>>(q, sps);
+  const dim3 grid(grid1.x, grid1.y, (unsigned)splits);
+  conv_pointwise_kernel<STRIDED, false><<<grid, THREADS, smem, st>>>(q, sps);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || splits == 1) return e;
   return launch_split_finalize(q, st);

@@ -16,9 +16,12 @@ import subprocess
 HERE = os.path.dirname(os.path.abspath(__file__))
 SRC = os.path.join(HERE, "int_issue_rate.cu")
 LIB = os.path.join(HERE, "libds_intpeak.so")
-KINDS = {0: "SHF", 1: "IMAD", 2: "SHF+IMAD", 3: "IADD", 4: "LOP", 5: "IMAD.HI", 6: "ADD+ADD"}
-# instructions per inner iteration: 64 of the mix (128 for SHF+IMAD) + 8 x-updates
-INSTR_PER_ITER = {0: 72, 1: 72, 2: 136, 3: 72, 4: 72, 5: 72, 6: 136}
+KINDS = {0: "SHF", 1: "IMAD", 2: "SHF+IMAD", 3: "IADD", 4: "LOP", 5: "IMAD.HI", 6: "ADD+ADD", 7: "SWAR16"}
+# instructions per inner iteration: 64 of the mix (128 for the pairs, 192 for the SWAR triple) + 8 x-updates
+INSTR_PER_ITER = {0: 72, 1: 72, 2: 136, 3: 72, 4: 72, 5: 72, 6: 136, 7: 200}
+# DeepShift terms (shift + sign flip + accumulate) per inner iteration, for the mixes that form a term:
+# SHF+IMAD one term per pair, IMAD.HI one per instruction, SWAR16 two (one per 16-bit lane) per triple
+TERMS_PER_ITER = {2: 64, 5: 64, 7: 128}
 
 
 def build() -> str:
@@ -54,7 +57,10 @@ def measure(iters: int = 4096, threads: int = 256, blocks_per_sm: int = 2):
             sel = sm == s
             span = float(c[sel, 1].max() - c[sel, 0].min())
             rates.append(int(sel.sum()) * threads * iters * INSTR_PER_ITER[kind] / span)
-        res[name] = {"thread_instr_per_clk_per_sm": sum(rates) / len(rates),
+        rate = sum(rates) / len(rates)
+        if kind in TERMS_PER_ITER:
+            res.setdefault("terms_per_clk_per_sm", {})[name] = rate * TERMS_PER_ITER[kind] / INSTR_PER_ITER[kind]
+        res[name] = {"thread_instr_per_clk_per_sm": rate,
                      "wall_tinstr_per_s": blocks * threads * iters * INSTR_PER_ITER[kind] / (ms.value / 1e3) / 1e12,
                      "ms": ms.value}
     return res

@@ -17,6 +17,11 @@
 //   kind 4: LOP3 only       (xor/and chains)
 //   kind 5: IMAD.HI only    (mad.hi.s32: high word of x * m plus acc)
 //   kind 6: IADD3 pairs     (acc = acc + a + b, three-input adds)
+//   kind 7: SWAR pair       (two 16-bit activations per register, Sec. 5.2.1's narrow format: one shift
+//                            of both lanes, one LOP3 (t & m) ^ c that clears the high lane's bits shifted
+//                            into the low lane and flips the lanes' sign bits for the sign extension,
+//                            whose constant is folded into a per-column correction, and one IMAD by the
+//                            sign: 3 instructions per 2 terms)
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -25,12 +30,14 @@ namespace {
 template <int KIND>
 __global__ void __launch_bounds__(256) mix_kernel(const int* __restrict__ seed, int iters, int* out,
                                                   long long* cycles, int* smid) {
-  int x[8], s[8], g[8], acc[8][8];
+  int x[8], s[8], g[8], m[8], c[8], acc[8][8];
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     x[i] = seed[(threadIdx.x + i) & 63];
     s[i] = seed[64 + i] & 15;
     g[i] = seed[72 + i];
+    m[i] = seed[(64 + 3 * i) & 79] | 0x0000ffff;
+    c[i] = seed[(72 + 5 * i) & 79] & 0x80008000;
 #pragma unroll
     for (int j = 0; j < 8; ++j) acc[i][j] = i ^ j;
   }
@@ -53,6 +60,11 @@ __global__ void __launch_bounds__(256) mix_kernel(const int* __restrict__ seed, 
           asm volatile("add.s32 %0, %0, %1;" : "+r"(acc[i][j]) : "r"(x[i]));
         } else if (KIND == 5) {
           asm volatile("mad.hi.s32 %0, %1, %2, %0;" : "+r"(acc[i][j]) : "r"(x[i]), "r"(g[j]));
+        } else if (KIND == 7) {
+          int t;
+          asm volatile("shr.s32 %0, %1, %2;" : "=r"(t) : "r"(x[i]), "r"(s[j]));
+          asm volatile("lop3.b32 %0, %0, %1, %2, 0x6A;" : "+r"(t) : "r"(m[j]), "r"(c[j]));
+          asm volatile("mad.lo.s32 %0, %1, %2, %0;" : "+r"(acc[i][j]) : "r"(g[j]), "r"(t));
         } else if (KIND == 6) {
           asm volatile("{\n\t.reg .s32 t;\n\tadd.s32 t, %1, %2;\n\tadd.s32 %0, %0, t;\n\t}" : "+r"(acc[i][j]) : "r"(x[i]), "r"(g[j]));
         } else {
@@ -97,6 +109,7 @@ extern "C" int ds_probe_int_mix(int kind, int blocks, int threads, int iters, co
     case 3: mix_kernel<3><<<blocks, threads>>>(seed, iters, out, cycles, smid); break;
     case 5: mix_kernel<5><<<blocks, threads>>>(seed, iters, out, cycles, smid); break;
     case 6: mix_kernel<6><<<blocks, threads>>>(seed, iters, out, cycles, smid); break;
+    case 7: mix_kernel<7><<<blocks, threads>>>(seed, iters, out, cycles, smid); break;
     default: mix_kernel<4><<<blocks, threads>>>(seed, iters, out, cycles, smid); break;
   }
   cudaEventRecord(b);

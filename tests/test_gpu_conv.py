@@ -103,6 +103,33 @@ def test_conv_degenerate_codes(dslib, geom, flags, expand):
     assert amax[1] == O.absmax(want)
 
 
+# Standalone calls whose grid does not fill the SMs at the batch the layer sweeps time them: the reduction is
+# split over the CTAs of a thread-block cluster (1x1: pointwise kernel; 3x3/2: direct kernel)
+SPLIT_GEOMS = [
+    (32, 256, 14, 14, 512, 1, 1, 2, 0),   # ResNet18 downsample 1x1/2, batch 32
+    (32, 128, 28, 28, 256, 1, 1, 2, 0),   # ResNet18 downsample 1x1/2, batch 32
+    (8, 2048, 7, 7, 512, 1, 1, 1, 0),     # ResNet50 bottleneck reduce on 7 x 7
+    (32, 256, 14, 14, 512, 3, 3, 2, 1),   # ResNet18 conv5_1 3x3/2, batch 32
+]
+
+
+@pytest.mark.parametrize("geom", SPLIT_GEOMS)
+@pytest.mark.parametrize("flags,residual", [(0, False), (16, False), (0, True)])
+def test_conv_standalone_cluster_split(dslib, geom, flags, residual):
+    """Every output of the under-filled layers, with the expanded codes the sweeps use: the 32-bit path, the
+    forced 64-bit path, and the residual join with ReLU."""
+    N, C, H, W, K, R, S, st, pd = geom
+    x, s, p, b = si.conv_layer(sum(geom) * 17 + flags, N, C, H, W, K, R, S, 0, 1 << 20, si.layer_centre(C, R, S))
+    OH = (H + 2 * pd - R) // st + 1
+    OW = (W + 2 * pd - S) // st + 1
+    res = si.activations(77, (N, K, OH, OW), -(1 << 31), 1 << 31) if residual else None
+    acc = O.conv2d_shift(x, s, p, b, (st, st), (pd, pd))
+    want = O.add_relu(acc, res) if residual else np.maximum(acc, 0)
+    got, amax = _run(dslib, x, s, p, b, (st, st), (pd, pd), relu=True, residual=res, flags=flags, expand=True)
+    assert np.array_equal(got, want)
+    assert amax[1] == O.absmax(want)
+
+
 # ResNet18 / ResNet50 / VGG16 layer shapes at a small batch, both kernels
 NET_GEOMS = [
     (1, 3, 224, 224, 64, 7, 7, 2, 3),    # stem 7x7/2
