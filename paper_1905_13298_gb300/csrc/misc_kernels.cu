@@ -92,6 +92,95 @@ __global__ void pack_kernel(const int8_t* __restrict__ s, const int8_t* __restri
   }
 }
 
+// Forward layout with 4-byte aligned rows (k_red % 4 == 0, s and p 4-byte
+// aligned): the same records, 128 reduction indices (4 chunks) per warp step.
+// Lane j loads codes 4j .. 4j + 3 of the step with one 32-bit load of s and
+// one of p, so lanes 8q .. 8q + 7 hold chunk q.  Each lane forms its 4 codes'
+// plane bits and nibbles; ORs over each group of 8 lanes (planes) and over
+// lane pairs (the shift word of 8 codes) assemble the records; lanes 8q + 2w
+// write shift word w of chunk q and lane 8q writes its bit planes.
+__global__ void pack_kernel_vec4(const int8_t* __restrict__ s, const int8_t* __restrict__ p, int64_t n_out,
+                                 int64_t k_red, uint8_t* __restrict__ blob, int64_t parts) {
+  const BlobLayout L = blob_layout(n_out, k_red);
+  BlobHeader* hdr = reinterpret_cast<BlobHeader*>(blob);
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    hdr->magic = DS_WEIGHTS_MAGIC;
+    hdr->format = DS_FORMAT_PLANES6;
+    hdr->n_out = n_out;
+    hdr->k_red = k_red;
+    hdr->n_chunks = L.n_chunks;
+  }
+  const unsigned full = 0xffffffffu;
+  const int lane = threadIdx.x & 31;
+  const int jj = lane & 7;  // lane within its chunk's group
+  const int64_t steps = (k_red + 127) / 128;
+  const int64_t per = (steps + parts - 1) / parts;
+  const int64_t units = n_out * parts;
+  uint32_t* nibw = reinterpret_cast<uint32_t*>(blob + L.nib);
+  uint2* bits = reinterpret_cast<uint2*>(blob + L.bits);
+  for (int64_t u = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; u < units;
+       u += ((int64_t)gridDim.x * blockDim.x) >> 5) {
+    const int64_t n = u % n_out;
+    const int64_t b0 = (u / n_out) * per;
+    const int64_t b1 = b0 + per < steps ? b0 + per : steps;
+    const uint32_t* srow = reinterpret_cast<const uint32_t*>(s + n * k_red);
+    const uint32_t* prow = reinterpret_cast<const uint32_t*>(p + n * k_red);
+    uint32_t a_sum = 0, nnz = 0, invalid = 0;  // per lane; a lane adds at most 2^15 per code
+    unsigned long long a_col = 0;
+#pragma unroll 2
+    for (int64_t b = b0; b < b1; ++b) {
+      const int64_t k0 = b * 128 + 4 * lane;
+      const bool in = k0 < k_red;  // k_red % 4 == 0: all 4 codes or none
+      const uint32_t sw = in ? __ldg(srow + (k0 >> 2)) : 0u;
+      const uint32_t pw = in ? __ldg(prow + (k0 >> 2)) : 0u;
+      uint32_t nb = 0u, zb = 0u, nib = 0u;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int sv = (int)(int8_t)(sw >> (8 * i));
+        const int pv = (int)(int8_t)(pw >> (8 * i));
+        const bool bad = in && ((unsigned)(sv + 1) > 2u || (unsigned)(pv + 15) > 15u);
+        const bool ok = in && !bad;
+        invalid += bad ? 1u : 0u;
+        if (ok) {
+          nib |= (uint32_t)(-pv) << (4 * i);
+          if (sv != 0) {
+            zb |= 1u << i;
+            a_sum += 1u << (15 + pv);
+          }
+          if (sv == -1) nb |= 1u << i;
+        }
+      }
+      nnz += (uint32_t)__popc(zb);
+      // planes of chunk q: lane 8q + jj holds bits 4 jj .. 4 jj + 3
+      uint32_t np = nb << (4 * jj), zp = zb << (4 * jj);
+      np |= __shfl_xor_sync(full, np, 1);
+      zp |= __shfl_xor_sync(full, zp, 1);
+      np |= __shfl_xor_sync(full, np, 2);
+      zp |= __shfl_xor_sync(full, zp, 2);
+      np |= __shfl_xor_sync(full, np, 4);
+      zp |= __shfl_xor_sync(full, zp, 4);
+      // shift word w (codes 8w .. 8w + 7) of chunk q: lanes 8q + 2w, 8q + 2w + 1
+      uint32_t w = nib << (16 * (jj & 1));
+      w |= __shfl_xor_sync(full, w, 1);
+      const int64_t g = b * 4 + (lane >> 3);  // this lane's chunk
+      if (g < L.n_chunks) {
+        if ((jj & 1) == 0) nibw[(g * n_out + n) * 4 + (jj >> 1)] = w;
+        if (jj == 0) bits[g * n_out + n] = make_uint2(np, zp);
+      }
+      // fold the lanes' column-constant partials every step (a warp step adds at most 2^22)
+      a_col += __reduce_add_sync(full, a_sum);
+      a_sum = 0;
+    }
+    nnz = __reduce_add_sync(full, nnz);
+    invalid = __reduce_add_sync(full, invalid);
+    if (lane == 0) {
+      atomicAdd(reinterpret_cast<unsigned long long*>(blob + L.col_a) + n, a_col);
+      atomicAdd(reinterpret_cast<uint32_t*>(blob + L.nnz) + n, nnz);
+      if (invalid) atomicAdd(&hdr->invalid_count, invalid);
+    }
+  }
+}
+
 // Header maxima over the columns' A[n] and nnz[n].
 __global__ void pack_maxima_kernel(uint8_t* __restrict__ blob, int64_t n_out, int64_t k_red) {
   const BlobLayout L = blob_layout(n_out, k_red);
@@ -132,10 +221,20 @@ cudaError_t launch_pack(const int8_t* s, const int8_t* p, int64_t n_out, int64_t
   int64_t parts = (want + n_out - 1) / n_out;
   if (parts > n_chunks) parts = n_chunks;
   if (parts < 1) parts = 1;
+  const bool vec4 = bwd == nullptr && (k_red % 4) == 0 && (reinterpret_cast<uintptr_t>(s) & 3) == 0 &&
+                    (reinterpret_cast<uintptr_t>(p) & 3) == 0;
+  if (vec4) {  // 128-index steps: split a column's steps into parts the same way
+    const int64_t steps = (k_red + 127) / 128;
+    if (parts > steps) parts = steps;
+  }
   const int64_t units = n_out * parts;
   int64_t blocks = (units + threads / 32 - 1) / (threads / 32);
   if (blocks > (int64_t)sms * 32) blocks = (int64_t)sms * 32;  // grid-stride beyond
-  pack_kernel<<<(unsigned)blocks, threads, 0, st>>>(s, p, n_out, k_red, blob, m, parts);
+  if (vec4) {
+    pack_kernel_vec4<<<(unsigned)blocks, threads, 0, st>>>(s, p, n_out, k_red, blob, parts);
+  } else {
+    pack_kernel<<<(unsigned)blocks, threads, 0, st>>>(s, p, n_out, k_red, blob, m, parts);
+  }
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   int64_t mb = (n_out + threads - 1) / threads;
