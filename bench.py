@@ -299,7 +299,8 @@ def run_gpu_other(args, wl, rank, world, local_rank):
                                      si.layer_centre(wl["K"], 1, 1))
         else:
             x, s, p, b = si.config4_int()
-        w = ds.pack_shift_weights(torch.from_numpy(s).to(dev), torch.from_numpy(p).to(dev), expand=True)
+        w = ds.pack_shift_weights(torch.from_numpy(s).to(dev), torch.from_numpy(p).to(dev),
+                                  expand=args.codes == "expanded")
         xd, bd = torch.from_numpy(x).to(dev), torch.from_numpy(b).to(dev)
         y = torch.empty((wl["M"], wl["Nout"]), dtype=torch.int32, device=dev)
         a = torch.zeros(2, dtype=torch.int32, device=dev)
@@ -362,7 +363,8 @@ def run_gpu_other(args, wl, rank, world, local_rank):
     out = {"metric": METRIC, "value": value, "unit": METRIC, "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
            "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
            "dtype": "bf16" if wl["kind"] == "fc16" else "int32", "data": "synthetic",
-           "config": {"workload": wl["name"], "cuda_graph": bool(args.graph), "terms_per_step": terms},
+           "config": {"workload": wl["name"], "cuda_graph": bool(args.graph), "terms_per_step": terms,
+                      "codes": args.codes},
            "roofline": roof,
            "gpu_launches": launches * args.steps, "clocks": clocks, "h2d_bytes_per_step_e2e": h2d}
     print(json.dumps(out), flush=True)
@@ -828,6 +830,9 @@ def main():
                                                          "sweep_resnet18_backward", "sweep_resnet50_backward"])
     ap.add_argument("--layers", default=None,
                     help="layer sweeps: comma-separated layer indices of the program to run (default: all)")
+    ap.add_argument("--codes", default="expanded", choices=["expanded", "packed"],
+                    help="FC workloads: run on the expanded execution layout (8 bytes per weight) or decode the "
+                         "6-bit packed blob in the kernel")
     ap.add_argument("--graph", action="store_true", help="replay each step from a CUDA graph (other workloads)")
     args = ap.parse_args()
     rank = int(os.environ.get("RANK", "0"))

@@ -15,18 +15,19 @@
 // reads are done.  No global scratch memory is used.
 //
 // 128 threads: thread (tm, tn) = (t % 8, t / 8) owns columns 4 tn .. 4 tn + 3
-// and TMR rows: row tm (TMR = 1), rows 4 tm .. 4 tm + 3 (TMR = 4), or two such
-// quads 32 rows apart (TMR = 8), so that the 8 row groups of a warp read
-// distinct banks.  Per stage of 16 k the CTA stages x transposed ([k][row], so
-// a thread's rows at one k are one or two 16-byte loads) and the stage's
-// codes (expanded layout: 16-byte cp.async; else decoded from the packed
-// blob; the expanded copy is ExpandedCodeStager).  x arrives in 16-byte pieces of 4 k of one row (4-byte copies when K
-// is not a multiple of 4, as rows are then not 16-byte aligned) in a row-major
-// scratch tile; once a thread's own copies have landed it writes its pieces
-// transposed, so no barrier is added.  Every thread copies the same pieces at
-// every stage: its source pointers only advance by 16 k.  Per term the hot
-// loop is one SHF and one IMAD, as in shift_gemm.cu; at most 96 registers,
-// 5 CTAs per SM.
+// and the TMR rows tm + 8 i, so that the 8 row groups of a warp read 8
+// consecutive rows.  Per stage of 16 k the CTA stages x row-major ([row][16
+// k], rows padded to 20 words: the 16-byte loads of 8 consecutive rows hit
+// distinct banks), copied in 16-byte pieces of 4 k of one row (4-byte copies
+// when K is not a multiple of 4, as rows are then not 16-byte aligned), and
+// the stage's codes (expanded layout: 16-byte cp.async through
+// ExpandedCodeStager; else decoded from the packed blob).  Every thread
+// copies the same pieces at every stage: its source pointers only advance by
+// 16 k.  Per 4 k the hot loop loads each of its rows' x with one 16-byte
+// load, then per k the codes of its 4 columns and runs one SHF and one IMAD
+// per term, as in shift_gemm.cu; at most 96 registers, 5 CTAs per SM.  The
+// 64-bit path of TMR = 8 runs as two passes of 4 rows each, so that its
+// accumulators fit the register budget.
 // Accumulator width as in shift_gemm.cu: the bound proven for the whole sum
 // also covers every partial sum (a subset of its terms), so 32-bit partials
 // are exact whenever the 32-bit path is taken, and their wrap-around sum is
@@ -56,12 +57,13 @@ constexpr int kMaxCluster = 16;
 template <int TMR>
 struct ClSmem {
   static constexpr int MR = 8 * TMR;
-  static constexpr int XR = MR + 4;  // words per staged k (16-byte aligned rows of the transposed tile)
+  // words per staged row: 16 k plus 4 of padding, so that the 16-byte loads
+  // of 8 consecutive rows by one warp fall on 8 distinct bank quads
+  static constexpr int XRW = KC + 4;
   union {
     struct {
-      int32_t xs[2][KC * XR];
+      int32_t xs[2][MR * XRW];  // x of a stage, row-major [row][16 k]
       int32_t cs[2][KC * CW];
-      int32_t xt[MR * KC];  // x of the stage in flight, row-major [row][16 k]
     } st;
     int64_t red[MR * NT];  // the partial sums (int64 or int32) after the reduction loop
   };
@@ -71,9 +73,9 @@ struct ClSmem {
 // (the end of this CTA's slice); zero elsewhere.  Piece e of a stage (e =
 // threadIdx.x + THREADS u) is 4 consecutive k of one row: row e / 4, k0 +
 // 4 (e % 4); consecutive threads read consecutive pieces of a row.  copy()
-// puts it at xt[4 e] (XV: one 16-byte copy whose source size zero-fills a
-// ragged end; else four 4-byte copies), transpose() moves the thread's own
-// landed pieces to xs[k][row].  src[u]: the piece's address at stage 0.
+// puts it at xs[row][4 (e % 4)] (XV: one 16-byte copy whose source size
+// zero-fills a ragged end; else four 4-byte copies).  src[u]: the piece's
+// address at stage 0.
 template <int TMR, bool XV>
 struct XStager {
   static constexpr int MR = 8 * TMR;
@@ -91,36 +93,24 @@ struct XStager {
       src[u] = ok ? P.x + row * P.kred + kbeg + 4 * (e % 4) : P.x;
     }
   }
-  __device__ __forceinline__ void copy(const GemmParams& P, int32_t* xt, int64_t kend, int st) const {
+  __device__ __forceinline__ void copy(const GemmParams& P, int32_t* xs, int64_t kend, int st) const {
+    constexpr int XRW = ClSmem<TMR>::XRW;
 #pragma unroll
     for (int u = 0; u < PIECES; ++u) {
       const int e = threadIdx.x + THREADS * u;
       if (e >= NP) continue;
       const int64_t left = kend - (kp[u] + (int64_t)st * KC);  // valid k of the piece, if positive
       const int32_t* s = src[u] + (int64_t)st * KC;
+      int32_t* dst = xs + (e / 4) * XRW + 4 * (e % 4);
       if constexpr (XV) {
         const int n = left >= 4 ? 16 : (left > 0 ? 4 * (int)left : 0);
-        const uint32_t d = (uint32_t)__cvta_generic_to_shared(xt + 4 * e);
+        const uint32_t d = (uint32_t)__cvta_generic_to_shared(dst);
         asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(n ? s : P.x), "r"(n));
       } else {
 #pragma unroll
         for (int i = 0; i < 4; ++i)
-          cp_async4(xt + 4 * e + i, i < left ? (const void*)(s + i) : (const void*)P.x, i < left);
+          cp_async4(dst + i, i < left ? (const void*)(s + i) : (const void*)P.x, i < left);
       }
-    }
-  }
-  __device__ __forceinline__ void transpose(const int32_t* xt, int32_t* xs) const {
-    constexpr int XR = ClSmem<TMR>::XR;
-#pragma unroll
-    for (int u = 0; u < PIECES; ++u) {
-      const int e = threadIdx.x + THREADS * u;
-      if (e >= NP) continue;
-      const int4 v = *reinterpret_cast<const int4*>(xt + 4 * e);
-      int32_t* d = xs + (4 * (e % 4)) * XR + e / 4;
-      d[0] = v.x;
-      d[XR] = v.y;
-      d[2 * XR] = v.z;
-      d[3 * XR] = v.w;
     }
   }
 };
@@ -151,51 +141,45 @@ __device__ __forceinline__ void decode_codes(const GemmParams& P, int32_t* cs, i
   }
 }
 
-// Tile row of this thread's i-th row.
+// Tile row of this thread's i-th row: tm + 8 i, so that the 8 row groups of a
+// warp read 8 consecutive rows (distinct banks at the padded row stride).
 template <int TMR>
 __device__ __forceinline__ int thread_row(int tm, int i) {
-  if constexpr (TMR == 1) {
-    return tm;
-  } else {
-    return (i >> 2) * 32 + 4 * tm + (i & 3);
-  }
+  return tm + 8 * i;
 }
 
-template <int TMR, typename Acc>
+// The hot loop over one stage for this thread's rows I0 .. I0 + NI - 1: per 4
+// k one 16-byte load of x per row, then per k the 4 columns' shifts and signs
+// (two 16-byte loads) and NI x 4 terms of one SHF and one IMAD each.
+template <int TMR, int I0, int NI, typename Acc>
 __device__ __forceinline__ void compute_stage(const int32_t* xs, const int32_t* cs, int tm, int tn,
-                                              Acc (&acc)[TMR][TN]) {
-  constexpr int XR = ClSmem<TMR>::XR;
+                                              Acc (&acc)[NI][TN]) {
+  constexpr int XRW = ClSmem<TMR>::XRW;
   const int32_t* cb = cs + ((tn * TN) >> 5) * 64 + ((tn * TN) & 31);
-  const int32_t* xb = xs + (TMR == 1 ? tm : 4 * tm);
 #pragma unroll
-  for (int k = 0; k < KC; ++k) {
-    int x[TMR];
-    if constexpr (TMR % 4 == 0) {
+  for (int k4 = 0; k4 < KC; k4 += 4) {
+    int4 xv[NI];
 #pragma unroll
-      for (int v = 0; v < TMR / 4; ++v) {
-        const int4 a = *reinterpret_cast<const int4*>(xb + k * XR + 32 * v);
-        x[4 * v] = a.x;
-        x[4 * v + 1] = a.y;
-        x[4 * v + 2] = a.z;
-        x[4 * v + 3] = a.w;
-      }
-    } else {
-      static_assert(TMR == 1, "row mapping");
-      x[0] = xb[k * XR];
-    }
-    const int4 s4 = *reinterpret_cast<const int4*>(cb + k * CW);
-    const int4 g4 = *reinterpret_cast<const int4*>(cb + k * CW + 32);
-    const int sh[TN] = {s4.x, s4.y, s4.z, s4.w};
-    const int sg[TN] = {g4.x, g4.y, g4.z, g4.w};
+    for (int i = 0; i < NI; ++i)
+      xv[i] = *reinterpret_cast<const int4*>(xs + thread_row<TMR>(tm, I0 + i) * XRW + k4);
 #pragma unroll
-    for (int i = 0; i < TMR; ++i) {
+    for (int kk = 0; kk < 4; ++kk) {
+      const int k = k4 + kk;
+      const int4 s4 = *reinterpret_cast<const int4*>(cb + k * CW);
+      const int4 g4 = *reinterpret_cast<const int4*>(cb + k * CW + 32);
+      const int sh[TN] = {s4.x, s4.y, s4.z, s4.w};
+      const int sg[TN] = {g4.x, g4.y, g4.z, g4.w};
 #pragma unroll
-      for (int j = 0; j < TN; ++j) {
-        const int t = x[i] >> sh[j];  // Eq. 1
-        if constexpr (sizeof(Acc) == 4) {
-          acc[i][j] += (uint32_t)sg[j] * (uint32_t)t;  // Eq. 2 + accumulate (mod 2^32)
-        } else {
-          acc[i][j] += (int64_t)sg[j] * (int64_t)t;
+      for (int i = 0; i < NI; ++i) {
+        const int x = kk == 0 ? xv[i].x : kk == 1 ? xv[i].y : kk == 2 ? xv[i].z : xv[i].w;
+#pragma unroll
+        for (int j = 0; j < TN; ++j) {
+          const int t = x >> sh[j];  // Eq. 1
+          if constexpr (sizeof(Acc) == 4) {
+            acc[i][j] += (uint32_t)sg[j] * (uint32_t)t;  // Eq. 2 + accumulate (mod 2^32)
+          } else {
+            acc[i][j] += (int64_t)sg[j] * (int64_t)t;
+          }
         }
       }
     }
@@ -225,17 +209,20 @@ __device__ __forceinline__ bool tile_int32_exact(const GemmParams& P, int64_t co
   return !__syncthreads_or(unsafe);
 }
 
-template <int TMR, bool XV, typename Acc>
+// One pass over the CTA's slice for this thread's rows I0 .. I0 + NI - 1 (the
+// 32-bit path: all TMR rows at once; the 64-bit path of TMR = 8: two passes
+// of one row quad each, so that its 64-bit accumulators fit the registers),
+// then the cluster reduction of the tile rows those thread rows cover.
+template <int TMR, bool XV, typename Acc, int I0, int NI>
 __device__ __forceinline__ void run_cluster_tile(const GemmParams& P, ClSmem<TMR>& sm, cg::cluster_group& cl,
                                                  int64_t row0, int64_t col0, int64_t kbeg, int64_t kend,
                                                  uint32_t& amax_local) {
-  constexpr int MR = 8 * TMR;
   const int t = threadIdx.x;
   const int tm = t % 8, tn = t / 8;
   const bool expanded = P.xcodes != nullptr;
-  Acc acc[TMR][TN];
+  Acc acc[NI][TN];
 #pragma unroll
-  for (int i = 0; i < TMR; ++i)
+  for (int i = 0; i < NI; ++i)
 #pragma unroll
     for (int j = 0; j < TN; ++j) acc[i][j] = 0;
 
@@ -245,12 +232,11 @@ __device__ __forceinline__ void run_cluster_tile(const GemmParams& P, ClSmem<TMR
   const XStager<TMR, XV> xst(P, row0, kbeg, kend);
   const ExpandedCodeStager cst(P.xcodes, P.cols, P.kred, col0, kbeg);
   if (nst > 0) {
-    xst.copy(P, sm.st.xt, kend, 0);
+    xst.copy(P, sm.st.xs[0], kend, 0);
     if (expanded) cst.stage(P.xcodes, P.kred, sm.st.cs[0], 0);
     cp_async_commit();
     if (!expanded) decode_codes(P, sm.st.cs[0], col0, kbeg);
     cp_async_wait_all();
-    xst.transpose(sm.st.xt, sm.st.xs[0]);
   }
   for (int st = 0; st < nst; ++st) {
     const int b = st & 1;
@@ -258,15 +244,14 @@ __device__ __forceinline__ void run_cluster_tile(const GemmParams& P, ClSmem<TMR
     const int64_t k1 = kbeg + (int64_t)(st + 1) * KC;
     __syncthreads();
     if (more) {
-      xst.copy(P, sm.st.xt, kend, st + 1);
+      xst.copy(P, sm.st.xs[b ^ 1], kend, st + 1);
       if (expanded) cst.stage(P.xcodes, P.kred, sm.st.cs[b ^ 1], st + 1);
       cp_async_commit();
     }
-    compute_stage<TMR, Acc>(sm.st.xs[b], sm.st.cs[b], tm, tn, acc);
+    compute_stage<TMR, I0, NI, Acc>(sm.st.xs[b], sm.st.cs[b], tm, tn, acc);
     if (more) {
       if (!expanded) decode_codes(P, sm.st.cs[b ^ 1], col0, k1);
       cp_async_wait_all();
-      xst.transpose(sm.st.xt, sm.st.xs[b ^ 1]);
     }
   }
   __syncthreads();  // every thread is done with the staging buffers: they hold the partials next
@@ -274,8 +259,8 @@ __device__ __forceinline__ void run_cluster_tile(const GemmParams& P, ClSmem<TMR
   // this CTA's partial sums, [MR][64] row-major, 16 bytes per (row, 4 columns) for 32-bit
   Acc* red = reinterpret_cast<Acc*>(sm.red);
 #pragma unroll
-  for (int i = 0; i < TMR; ++i) {
-    Acc* dst = red + thread_row<TMR>(tm, i) * NT + tn * TN;
+  for (int i = 0; i < NI; ++i) {
+    Acc* dst = red + thread_row<TMR>(tm, I0 + i) * NT + tn * TN;
 #pragma unroll
     for (int j = 0; j < TN; ++j) dst[j] = acc[i][j];
   }
@@ -285,9 +270,12 @@ __device__ __forceinline__ void run_cluster_tile(const GemmParams& P, ClSmem<TMR
   const int cs_n = (int)cl.num_blocks();
   const bool relu = (P.flags & DS_RELU) != 0;
   const bool vec_out = (P.cols % 4) == 0;
-  constexpr int GROUPS = MR * (NT / TN);  // (row, 4 columns) groups of the tile
+  // tile rows of this pass: all 8 TMR rows, or the 32 rows of one row quad
+  constexpr int ROWS = TMR == 1 ? 8 : 8 * NI;
+  constexpr int ROW0 = TMR == 1 ? 0 : (I0 / 4) * 32;
+  constexpr int GROUPS = ROWS * (NT / TN);  // (row, 4 columns) groups of the pass
   for (int gi = rank * THREADS + t; gi < GROUPS; gi += cs_n * THREADS) {
-    const int r = gi / (NT / TN), c4 = gi % (NT / TN);
+    const int r = ROW0 + gi / (NT / TN), c4 = gi % (NT / TN);
     Acc sum[TN] = {0, 0, 0, 0};
     for (int q = 0; q < cs_n; ++q) {
       const Acc* src = cl.map_shared_rank(red, q) + r * NT + c4 * TN;
@@ -352,9 +340,12 @@ __global__ void __launch_bounds__(THREADS, kMinBlocks) linear_cluster_kernel(con
   const int64_t kend = min(P.kred, kbeg + k_per_cta);
   uint32_t amax_local = 0;
   if (tile_int32_exact(P, col0)) {
-    run_cluster_tile<TMR, XV, uint32_t>(P, sm, cl, row0, col0, kbeg, kend, amax_local);
+    run_cluster_tile<TMR, XV, uint32_t, 0, TMR>(P, sm, cl, row0, col0, kbeg, kend, amax_local);
+  } else if constexpr (TMR == 8) {
+    run_cluster_tile<TMR, XV, int64_t, 0, 4>(P, sm, cl, row0, col0, kbeg, kend, amax_local);
+    run_cluster_tile<TMR, XV, int64_t, 4, 4>(P, sm, cl, row0, col0, kbeg, kend, amax_local);
   } else {
-    run_cluster_tile<TMR, XV, int64_t>(P, sm, cl, row0, col0, kbeg, kend, amax_local);
+    run_cluster_tile<TMR, XV, int64_t, 0, TMR>(P, sm, cl, row0, col0, kbeg, kend, amax_local);
   }
   if (P.amax_out != nullptr) {
     amax_local = __reduce_max_sync(0xffffffffu, amax_local);
