@@ -192,6 +192,7 @@ __device__ __forceinline__ uint32_t uabs(int32_t v) { return v < 0 ? (uint32_t)0
 struct ExpandedCodeStager {
   const int32_t* src;  // (block 0, kl) at stage 0
   int64_t kp;          // kl's reduction index at stage 0
+  int64_t kred_words;  // words between the two blocks' rows of one index: kred * 64
   bool b1;             // block 1 exists
   __device__ __forceinline__ ExpandedCodeStager(const int32_t* xcodes, int64_t cols, int64_t kred, int64_t col0,
                                                 int64_t kbeg) {
@@ -199,7 +200,20 @@ struct ExpandedCodeStager {
     const int64_t cb = col0 / 32;
     b1 = cb + 1 < (cols + 31) / 32;
     kp = kbeg + (t >> 4);
+    kred_words = kred * 64;
     src = xcodes != nullptr ? xcodes + (cb * kred + kp) * 64 + (t & 15) * 4 : xcodes;
+  }
+  // stage st with both blocks present and all 16 indices inside the reduction: no checks
+  __device__ __forceinline__ void stage_full(int32_t* cs, int st) const {
+    const int t = threadIdx.x;
+    const int32_t* s = src + (int64_t)st * 16 * 64;
+    const uint32_t d = (uint32_t)__cvta_generic_to_shared(cs + (t >> 4) * 128 + (t & 15) * 4);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int kl8 = (u & 1) * 8, b = u >> 1;
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(d + (uint32_t)(kl8 * 128 + b * 64) * 4),
+                   "l"(s + kl8 * 64 + b * kred_words));
+    }
   }
   // stage st (indices kbeg + 16 st ..) into cs; zero fill past kred and for an absent block
   __device__ __forceinline__ void stage(const int32_t* xcodes, int64_t kred, int32_t* cs, int st) const {

@@ -15,19 +15,18 @@
 // reads are done.  No global scratch memory is used.
 //
 // 128 threads: thread (tm, tn) = (t % 8, t / 8) owns columns 4 tn .. 4 tn + 3
-// and the TMR rows tm + 8 i, so that the 8 row groups of a warp read 8
-// consecutive rows.  Per stage of 16 k the CTA stages x row-major ([row][16
-// k], rows padded to 20 words: the 16-byte loads of 8 consecutive rows hit
-// distinct banks), copied in 16-byte pieces of 4 k of one row (4-byte copies
-// when K is not a multiple of 4, as rows are then not 16-byte aligned), and
-// the stage's codes (expanded layout: 16-byte cp.async through
-// ExpandedCodeStager; else decoded from the packed blob).  Every thread
-// copies the same pieces at every stage: its source pointers only advance by
-// 16 k.  Per 4 k the hot loop loads each of its rows' x with one 16-byte
-// load, then per k the codes of its 4 columns and runs one SHF and one IMAD
-// per term, as in shift_gemm.cu; at most 96 registers, 5 CTAs per SM.  The
-// 64-bit path of TMR = 8 runs as two passes of 4 rows each, so that its
-// accumulators fit the register budget.
+// and TMR rows: row tm (TMR = 1), rows 4 tm .. 4 tm + 3 (TMR = 4), or two such
+// quads 32 rows apart (TMR = 8), so that the 8 row groups of a warp read
+// distinct banks.  Per stage of 16 k the CTA stages x transposed ([k][row], so
+// a thread's rows at one k are one or two 16-byte loads) and the stage's
+// codes (expanded layout: 16-byte cp.async; else decoded from the packed
+// blob; the expanded copy is ExpandedCodeStager).  x arrives in 16-byte pieces of 4 k of one row (4-byte copies when K
+// is not a multiple of 4, as rows are then not 16-byte aligned) in a row-major
+// scratch tile; once a thread's own copies have landed it writes its pieces
+// transposed, so no barrier is added.  Every thread copies the same pieces at
+// every stage: its source pointers only advance by 16 k.  Per term the hot
+// loop is one SHF and one IMAD, as in shift_gemm.cu; at most 96 registers,
+// 5 CTAs per SM.
 // Accumulator width as in shift_gemm.cu: the bound proven for the whole sum
 // also covers every partial sum (a subset of its terms), so 32-bit partials
 // are exact whenever the 32-bit path is taken, and their wrap-around sum is
@@ -57,13 +56,12 @@ constexpr int kMaxCluster = 16;
 template <int TMR>
 struct ClSmem {
   static constexpr int MR = 8 * TMR;
-  // words per staged row: 16 k plus 4 of padding, so that the 16-byte loads
-  // of 8 consecutive rows by one warp fall on 8 distinct bank quads
-  static constexpr int XRW = KC + 4;
+  static constexpr int XR = MR + 4;  // words per staged k (16-byte aligned rows of the transposed tile)
   union {
     struct {
-      int32_t xs[2][MR * XRW];  // x of a stage, row-major [row][16 k]
+      int32_t xs[2][KC * XR];
       int32_t cs[2][KC * CW];
+      int32_t xt[MR * KC];  // x of the stage in flight, row-major [row][16 k]
     } st;
     int64_t red[MR * NT];  // the partial sums (int64 or int32) after the reduction loop
   };
@@ -71,11 +69,13 @@ struct ClSmem {
 
 // x rows [row0, row0 + MR), reduction indices [k0, k0 + 16) clipped to kend
 // (the end of this CTA's slice); zero elsewhere.  Piece e of a stage (e =
-// threadIdx.x + THREADS u) is 4 consecutive k of one row: row e / 4, k0 +
-// 4 (e % 4); consecutive threads read consecutive pieces of a row.  copy()
-// puts it at xs[row][4 (e % 4)] (XV: one 16-byte copy whose source size
-// zero-fills a ragged end; else four 4-byte copies).  src[u]: the piece's
-// address at stage 0.
+// threadIdx.x + THREADS u) is 4 consecutive k of one row: row e % MR, k0 +
+// 4 (e / MR), so that the pieces of a warp are consecutive rows at one k and
+// its transposing 4-byte stores hit consecutive words.  copy() puts a piece
+// at xt[4 e] (XV: one 16-byte copy whose source size zero-fills a ragged end;
+// else four 4-byte copies; through L1, where the piece beside it in its row
+// arrives with it), transpose() moves the thread's own landed pieces to
+// xs[k][row].  src[u]: the piece's address at stage 0.
 template <int TMR, bool XV>
 struct XStager {
   static constexpr int MR = 8 * TMR;
@@ -87,30 +87,59 @@ struct XStager {
 #pragma unroll
     for (int u = 0; u < PIECES; ++u) {
       const int e = threadIdx.x + THREADS * u;
-      const int64_t row = row0 + e / 4;
+      const int64_t row = row0 + e % MR;
       const bool ok = e < NP && row < P.rows;
-      kp[u] = ok ? kbeg + 4 * (e % 4) : kend;
-      src[u] = ok ? P.x + row * P.kred + kbeg + 4 * (e % 4) : P.x;
+      kp[u] = ok ? kbeg + 4 * (e / MR) : kend;
+      src[u] = ok ? P.x + row * P.kred + kbeg + 4 * (e / MR) : P.x;
     }
   }
-  __device__ __forceinline__ void copy(const GemmParams& P, int32_t* xs, int64_t kend, int st) const {
-    constexpr int XRW = ClSmem<TMR>::XRW;
+  // A stage whose pieces may be ragged or absent (the slice's last stage, rows past M).
+  __device__ __forceinline__ void copy(const GemmParams& P, int32_t* xt, int64_t kend, int st) const {
 #pragma unroll
     for (int u = 0; u < PIECES; ++u) {
       const int e = threadIdx.x + THREADS * u;
       if (e >= NP) continue;
       const int64_t left = kend - (kp[u] + (int64_t)st * KC);  // valid k of the piece, if positive
       const int32_t* s = src[u] + (int64_t)st * KC;
-      int32_t* dst = xs + (e / 4) * XRW + 4 * (e % 4);
       if constexpr (XV) {
         const int n = left >= 4 ? 16 : (left > 0 ? 4 * (int)left : 0);
-        const uint32_t d = (uint32_t)__cvta_generic_to_shared(dst);
-        asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(n ? s : P.x), "r"(n));
+        const uint32_t d = (uint32_t)__cvta_generic_to_shared(xt + 4 * e);
+        asm volatile("cp.async.ca.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(n ? s : P.x), "r"(n));
       } else {
 #pragma unroll
         for (int i = 0; i < 4; ++i)
-          cp_async4(dst + i, i < left ? (const void*)(s + i) : (const void*)P.x, i < left);
+          cp_async4(xt + 4 * e + i, i < left ? (const void*)(s + i) : (const void*)P.x, i < left);
       }
+    }
+  }
+  // A stage whose pieces are all whole (every row present, all 16 k inside the slice): no checks.
+  __device__ __forceinline__ void copy_full(int32_t* xt, int st) const {
+#pragma unroll
+    for (int u = 0; u < PIECES; ++u) {
+      const int e = threadIdx.x + THREADS * u;
+      if (e >= NP) continue;
+      const int32_t* s = src[u] + (int64_t)st * KC;
+      if constexpr (XV) {
+        const uint32_t d = (uint32_t)__cvta_generic_to_shared(xt + 4 * e);
+        asm volatile("cp.async.ca.shared.global [%0], [%1], 16;\n" ::"r"(d), "l"(s));
+      } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) cp_async4(xt + 4 * e + i, s + i, true);
+      }
+    }
+  }
+  __device__ __forceinline__ void transpose(const int32_t* xt, int32_t* xs) const {
+    constexpr int XR = ClSmem<TMR>::XR;
+#pragma unroll
+    for (int u = 0; u < PIECES; ++u) {
+      const int e = threadIdx.x + THREADS * u;
+      if (e >= NP) continue;
+      const int4 v = *reinterpret_cast<const int4*>(xt + 4 * e);
+      int32_t* d = xs + (4 * (e / MR)) * XR + e % MR;
+      d[0] = v.x;
+      d[XR] = v.y;
+      d[2 * XR] = v.z;
+      d[3 * XR] = v.w;
     }
   }
 };
@@ -141,45 +170,54 @@ __device__ __forceinline__ void decode_codes(const GemmParams& P, int32_t* cs, i
   }
 }
 
-// Tile row of this thread's i-th row: tm + 8 i, so that the 8 row groups of a
-// warp read 8 consecutive rows (distinct banks at the padded row stride).
+// Tile row of this thread's i-th row.
 template <int TMR>
 __device__ __forceinline__ int thread_row(int tm, int i) {
-  return tm + 8 * i;
+  if constexpr (TMR == 1) {
+    return tm;
+  } else {
+    return (i >> 2) * 32 + 4 * tm + (i & 3);
+  }
 }
 
-// The hot loop over one stage for this thread's rows I0 .. I0 + NI - 1: per 4
-// k one 16-byte load of x per row, then per k the 4 columns' shifts and signs
-// (two 16-byte loads) and NI x 4 terms of one SHF and one IMAD each.
+// The hot loop over one stage for this thread's rows I0 .. I0 + NI - 1 (whole
+// row quads unless TMR = 1).
 template <int TMR, int I0, int NI, typename Acc>
 __device__ __forceinline__ void compute_stage(const int32_t* xs, const int32_t* cs, int tm, int tn,
                                               Acc (&acc)[NI][TN]) {
-  constexpr int XRW = ClSmem<TMR>::XRW;
+  constexpr int XR = ClSmem<TMR>::XR;
   const int32_t* cb = cs + ((tn * TN) >> 5) * 64 + ((tn * TN) & 31);
+  const int32_t* xb = xs + (TMR == 1 ? tm : 4 * tm);
 #pragma unroll
-  for (int k4 = 0; k4 < KC; k4 += 4) {
-    int4 xv[NI];
+  for (int k = 0; k < KC; ++k) {
+    int x[NI];
+    if constexpr (TMR % 4 == 0) {
+      static_assert(NI % 4 == 0 && I0 % 4 == 0, "whole row quads");
 #pragma unroll
-    for (int i = 0; i < NI; ++i)
-      xv[i] = *reinterpret_cast<const int4*>(xs + thread_row<TMR>(tm, I0 + i) * XRW + k4);
+      for (int v = 0; v < NI / 4; ++v) {
+        const int4 a = *reinterpret_cast<const int4*>(xb + k * XR + 32 * (I0 / 4 + v));
+        x[4 * v] = a.x;
+        x[4 * v + 1] = a.y;
+        x[4 * v + 2] = a.z;
+        x[4 * v + 3] = a.w;
+      }
+    } else {
+      static_assert(TMR == 1 && NI == 1 && I0 == 0, "row mapping");
+      x[0] = xb[k * XR];
+    }
+    const int4 s4 = *reinterpret_cast<const int4*>(cb + k * CW);
+    const int4 g4 = *reinterpret_cast<const int4*>(cb + k * CW + 32);
+    const int sh[TN] = {s4.x, s4.y, s4.z, s4.w};
+    const int sg[TN] = {g4.x, g4.y, g4.z, g4.w};
 #pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-      const int k = k4 + kk;
-      const int4 s4 = *reinterpret_cast<const int4*>(cb + k * CW);
-      const int4 g4 = *reinterpret_cast<const int4*>(cb + k * CW + 32);
-      const int sh[TN] = {s4.x, s4.y, s4.z, s4.w};
-      const int sg[TN] = {g4.x, g4.y, g4.z, g4.w};
+    for (int i = 0; i < NI; ++i) {
 #pragma unroll
-      for (int i = 0; i < NI; ++i) {
-        const int x = kk == 0 ? xv[i].x : kk == 1 ? xv[i].y : kk == 2 ? xv[i].z : xv[i].w;
-#pragma unroll
-        for (int j = 0; j < TN; ++j) {
-          const int t = x >> sh[j];  // Eq. 1
-          if constexpr (sizeof(Acc) == 4) {
-            acc[i][j] += (uint32_t)sg[j] * (uint32_t)t;  // Eq. 2 + accumulate (mod 2^32)
-          } else {
-            acc[i][j] += (int64_t)sg[j] * (int64_t)t;
-          }
+      for (int j = 0; j < TN; ++j) {
+        const int t = x[i] >> sh[j];  // Eq. 1
+        if constexpr (sizeof(Acc) == 4) {
+          acc[i][j] += (uint32_t)sg[j] * (uint32_t)t;  // Eq. 2 + accumulate (mod 2^32)
+        } else {
+          acc[i][j] += (int64_t)sg[j] * (int64_t)t;
         }
       }
     }
@@ -217,6 +255,7 @@ template <int TMR, bool XV, typename Acc, int I0, int NI>
 __device__ __forceinline__ void run_cluster_tile(const GemmParams& P, ClSmem<TMR>& sm, cg::cluster_group& cl,
                                                  int64_t row0, int64_t col0, int64_t kbeg, int64_t kend,
                                                  uint32_t& amax_local) {
+  constexpr int MR = 8 * TMR;
   const int t = threadIdx.x;
   const int tm = t % 8, tn = t / 8;
   const bool expanded = P.xcodes != nullptr;
@@ -231,12 +270,15 @@ __device__ __forceinline__ void run_cluster_tile(const GemmParams& P, ClSmem<TMR
   const int nst = kend > kbeg ? (int)((kend - kbeg + KC - 1) / KC) : 0;
   const XStager<TMR, XV> xst(P, row0, kbeg, kend);
   const ExpandedCodeStager cst(P.xcodes, P.cols, P.kred, col0, kbeg);
+  // stages whose x pieces and codes are all whole take the unchecked copies
+  const bool whole_rows = row0 + MR <= P.rows && cst.b1;
   if (nst > 0) {
-    xst.copy(P, sm.st.xs[0], kend, 0);
+    xst.copy(P, sm.st.xt, kend, 0);
     if (expanded) cst.stage(P.xcodes, P.kred, sm.st.cs[0], 0);
     cp_async_commit();
     if (!expanded) decode_codes(P, sm.st.cs[0], col0, kbeg);
     cp_async_wait_all();
+    xst.transpose(sm.st.xt, sm.st.xs[0]);
   }
   for (int st = 0; st < nst; ++st) {
     const int b = st & 1;
@@ -244,14 +286,20 @@ __device__ __forceinline__ void run_cluster_tile(const GemmParams& P, ClSmem<TMR
     const int64_t k1 = kbeg + (int64_t)(st + 1) * KC;
     __syncthreads();
     if (more) {
-      xst.copy(P, sm.st.xs[b ^ 1], kend, st + 1);
-      if (expanded) cst.stage(P.xcodes, P.kred, sm.st.cs[b ^ 1], st + 1);
+      if (whole_rows && k1 + KC <= kend) {
+        xst.copy_full(sm.st.xt, st + 1);
+        if (expanded) cst.stage_full(sm.st.cs[b ^ 1], st + 1);
+      } else {
+        xst.copy(P, sm.st.xt, kend, st + 1);
+        if (expanded) cst.stage(P.xcodes, P.kred, sm.st.cs[b ^ 1], st + 1);
+      }
       cp_async_commit();
     }
     compute_stage<TMR, I0, NI, Acc>(sm.st.xs[b], sm.st.cs[b], tm, tn, acc);
     if (more) {
       if (!expanded) decode_codes(P, sm.st.cs[b ^ 1], col0, k1);
       cp_async_wait_all();
+      xst.transpose(sm.st.xt, sm.st.xs[b ^ 1]);
     }
   }
   __syncthreads();  // every thread is done with the staging buffers: they hold the partials next
@@ -270,8 +318,8 @@ __device__ __forceinline__ void run_cluster_tile(const GemmParams& P, ClSmem<TMR
   const int cs_n = (int)cl.num_blocks();
   const bool relu = (P.flags & DS_RELU) != 0;
   const bool vec_out = (P.cols % 4) == 0;
-  // tile rows of this pass: all 8 TMR rows, or the 32 rows of one row quad
-  constexpr int ROWS = TMR == 1 ? 8 : 8 * NI;
+  // tile rows of this pass: all MR rows, or the 32 rows of one row quad
+  constexpr int ROWS = TMR == 1 ? MR : 8 * NI;
   constexpr int ROW0 = TMR == 1 ? 0 : (I0 / 4) * 32;
   constexpr int GROUPS = ROWS * (NT / TN);  // (row, 4 columns) groups of the pass
   for (int gi = rank * THREADS + t; gi < GROUPS; gi += cs_n * THREADS) {

@@ -125,15 +125,13 @@ __global__ void pack_kernel_vec4(const int8_t* __restrict__ s, const int8_t* __r
     const int64_t b1 = b0 + per < steps ? b0 + per : steps;
     const uint32_t* srow = reinterpret_cast<const uint32_t*>(s + n * k_red);
     const uint32_t* prow = reinterpret_cast<const uint32_t*>(p + n * k_red);
-    uint32_t a_sum = 0, nnz = 0, invalid = 0;  // per lane; a lane adds at most 2^15 per code
+    uint32_t nnz = 0, invalid = 0;  // per lane
     unsigned long long a_col = 0;
-#pragma unroll 2
-    for (int64_t b = b0; b < b1; ++b) {
+    // one warp step: 128 indices of the column from the lane's words sw, pw
+    auto step = [&](int64_t b, uint32_t sw, uint32_t pw) {
       const int64_t k0 = b * 128 + 4 * lane;
       const bool in = k0 < k_red;  // k_red % 4 == 0: all 4 codes or none
-      const uint32_t sw = in ? __ldg(srow + (k0 >> 2)) : 0u;
-      const uint32_t pw = in ? __ldg(prow + (k0 >> 2)) : 0u;
-      uint32_t nb = 0u, zb = 0u, nib = 0u;
+      uint32_t nb = 0u, zb = 0u, nib = 0u, a_sum = 0u;  // a lane adds at most 2^15 per code
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
         const int sv = (int)(int8_t)(sw >> (8 * i));
@@ -167,9 +165,20 @@ __global__ void pack_kernel_vec4(const int8_t* __restrict__ s, const int8_t* __r
         if ((jj & 1) == 0) nibw[(g * n_out + n) * 4 + (jj >> 1)] = w;
         if (jj == 0) bits[g * n_out + n] = make_uint2(np, zp);
       }
-      // fold the lanes' column-constant partials every step (a warp step adds at most 2^22)
-      a_col += __reduce_add_sync(full, a_sum);
-      a_sum = 0;
+      a_col += __reduce_add_sync(full, a_sum);  // a warp step adds at most 2^22
+    };
+    // four steps per iteration, their loads issued before any is decoded
+    for (int64_t b = b0; b < b1; b += 4) {
+      uint32_t sw[4], pw[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const bool in = b + q < b1 && (b + q) * 128 + 4 * lane < k_red;
+        sw[q] = in ? __ldg(srow + (((b + q) * 128) >> 2) + lane) : 0u;
+        pw[q] = in ? __ldg(prow + (((b + q) * 128) >> 2) + lane) : 0u;
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        if (b + q < b1) step(b + q, sw[q], pw[q]);
     }
     nnz = __reduce_add_sync(full, nnz);
     invalid = __reduce_add_sync(full, invalid);
