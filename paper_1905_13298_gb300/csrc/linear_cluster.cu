@@ -69,13 +69,14 @@ struct ClSmem {
 
 // x rows [row0, row0 + MR), reduction indices [k0, k0 + 16) clipped to kend
 // (the end of this CTA's slice); zero elsewhere.  Piece e of a stage (e =
-// threadIdx.x + THREADS u) is 4 consecutive k of one row: row e % MR, k0 +
-// 4 (e / MR), so that the pieces of a warp are consecutive rows at one k and
-// its transposing 4-byte stores hit consecutive words.  copy() puts a piece
-// at xt[4 e] (XV: one 16-byte copy whose source size zero-fills a ragged end;
-// else four 4-byte copies; through L1, where the piece beside it in its row
-// arrives with it), transpose() moves the thread's own landed pieces to
-// xs[k][row].  src[u]: the piece's address at stage 0.
+// threadIdx.x + THREADS u) is 4 consecutive k of one row: with 32 rows or
+// more, a warp's pieces are 16 consecutive rows x 2 adjacent pieces (each
+// row's 32 bytes read together, and the transposing 4-byte stores of the two
+// halves of the warp fall on the two halves of the banks); with 8 rows, row
+// e / 4, piece e % 4.  copy() puts a piece at xt[4 e] (XV: one 16-byte copy
+// whose source size zero-fills a ragged end; else four 4-byte copies),
+// transpose() moves the thread's own landed pieces to xs[k][row].  src[u]:
+// the piece's address at stage 0.
 template <int TMR, bool XV>
 struct XStager {
   static constexpr int MR = 8 * TMR;
@@ -83,14 +84,28 @@ struct XStager {
   static constexpr int PIECES = (NP + THREADS - 1) / THREADS;  // per thread: 1, 1, 2
   const int32_t* src[PIECES];
   int64_t kp[PIECES];  // the piece's first k at stage 0, or the slice end if its row is absent
+  __device__ __forceinline__ static int piece_row(int e) {
+    if constexpr (MR >= 32) {
+      return ((e >> 5) % (MR / 16)) * 16 + (e & 15);
+    } else {
+      return e >> 2;
+    }
+  }
+  __device__ __forceinline__ static int piece_k4(int e) {  // which 4 k of the stage
+    if constexpr (MR >= 32) {
+      return ((e >> 5) / (MR / 16)) * 2 + ((e >> 4) & 1);
+    } else {
+      return e & 3;
+    }
+  }
   __device__ __forceinline__ XStager(const GemmParams& P, int64_t row0, int64_t kbeg, int64_t kend) {
 #pragma unroll
     for (int u = 0; u < PIECES; ++u) {
       const int e = threadIdx.x + THREADS * u;
-      const int64_t row = row0 + e % MR;
+      const int64_t row = row0 + piece_row(e);
       const bool ok = e < NP && row < P.rows;
-      kp[u] = ok ? kbeg + 4 * (e / MR) : kend;
-      src[u] = ok ? P.x + row * P.kred + kbeg + 4 * (e / MR) : P.x;
+      kp[u] = ok ? kbeg + 4 * piece_k4(e) : kend;
+      src[u] = ok ? P.x + row * P.kred + kbeg + 4 * piece_k4(e) : P.x;
     }
   }
   // A stage whose pieces may be ragged or absent (the slice's last stage, rows past M).
@@ -104,7 +119,7 @@ struct XStager {
       if constexpr (XV) {
         const int n = left >= 4 ? 16 : (left > 0 ? 4 * (int)left : 0);
         const uint32_t d = (uint32_t)__cvta_generic_to_shared(xt + 4 * e);
-        asm volatile("cp.async.ca.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(n ? s : P.x), "r"(n));
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(n ? s : P.x), "r"(n));
       } else {
 #pragma unroll
         for (int i = 0; i < 4; ++i)
@@ -121,7 +136,7 @@ struct XStager {
       const int32_t* s = src[u] + (int64_t)st * KC;
       if constexpr (XV) {
         const uint32_t d = (uint32_t)__cvta_generic_to_shared(xt + 4 * e);
-        asm volatile("cp.async.ca.shared.global [%0], [%1], 16;\n" ::"r"(d), "l"(s));
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(d), "l"(s));
       } else {
 #pragma unroll
         for (int i = 0; i < 4; ++i) cp_async4(xt + 4 * e + i, s + i, true);
@@ -135,7 +150,7 @@ struct XStager {
       const int e = threadIdx.x + THREADS * u;
       if (e >= NP) continue;
       const int4 v = *reinterpret_cast<const int4*>(xt + 4 * e);
-      int32_t* d = xs + (4 * (e / MR)) * XR + e % MR;
+      int32_t* d = xs + (4 * piece_k4(e)) * XR + piece_row(e);
       d[0] = v.x;
       d[XR] = v.y;
       d[2 * XR] = v.z;
