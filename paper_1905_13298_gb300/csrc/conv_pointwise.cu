@@ -276,7 +276,7 @@ __device__ __forceinline__ void run_tile(const GemmParams& P, PwSmem& sm, int64_
 
   static_assert(KC == 16 && NB == 2 && THREADS == 128, "ExpandedCodeStager's stage shape");
   const ExpandedCodeStager cst(P.xcodes, P.cols, P.kred, col0, (int64_t)st_begin * KC);
-  if (st_begin < st_end) {  // a trailing rank of a cluster may have no stage: zero partial sums
+  if (!CL || st_begin < st_end) {  // a trailing rank of a cluster may have no stage: zero partial sums
     stage_x<STRIDED>(P, sm.xs[0], q, st_begin * KC);
     if (expanded) cst.stage(P.xcodes, P.kred, sm.cs[0], 0);
     cp_async_commit();
@@ -339,7 +339,16 @@ __device__ __forceinline__ void run_tile(const GemmParams& P, PwSmem& sm, int64_
     const int64_t col = col0 + tn * TN + j;
     bcol[j] = (P.bias != nullptr && col < P.cols) ? __ldg(P.bias + col) : 0;
   }
-  auto finish = [](Acc a, int32_t b) -> int32_t { return finish_sum<Acc>(a, b); };
+  auto finish = [](Acc a, int32_t b) -> int32_t {
+    if constexpr (sizeof(Acc) == 4) {
+      return (int32_t)(a + (uint32_t)b);
+    } else {
+      int64_t v = a + (int64_t)b;
+      v = v > (int64_t)INT32_MAX ? (int64_t)INT32_MAX : v;
+      v = v < (int64_t)INT32_MIN ? (int64_t)INT32_MIN : v;
+      return (int32_t)v;
+    }
+  };
   if (vec) {
 #pragma unroll
     for (int qd = 0; qd < NI / 4; ++qd) {
