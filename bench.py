@@ -31,7 +31,7 @@ INT_OPS_PER_CLK_PER_SM = 128  # 4 SMSPs x 32 lanes: 16-lane ALU pipe + 16-lane F
 ALG_INT_OPS_PER_TERM = 2      # one shift + one add/subtract per term (Fig. 1a: MAC -> shift + add)
 # DRAM bytes (read + write) of one conv_direct_kernel<1,3,7,0> launch on this workload, from one ncu capture
 # of the current kernel (dram__bytes_read.sum + dram__bytes_write.sum); y stays in L2 at kernel end.
-NCU_TRAFFIC_BYTES = 26.15e6
+NCU_TRAFFIC_BYTES = 26.08e6
 E2E_CHUNKS = 4  # chunks of the batch in the end-to-end measurement
 
 
