@@ -219,6 +219,13 @@ ds_status ds_linear_shift_bf16(const uint16_t* x, const ds_weights* w, const flo
  * incomplete.  A library utility: no counterpart in the paper. */
 int ds_bf16_fault_flag(void);
 
+/* Diagnostic: the limit, in SM clock cycles, of each bounded wait of the float kernel's later launches; cycles <= 0
+ * restores the default (4e9 cycles, about 2 s).  A launch whose wait runs out stops issuing work, lets the copies and
+ * tensor-core operations it already issued finish, frees its tensor memory and sets the fault flag above, so a test
+ * can make the waits run out on purpose and the context stays usable.  Process-wide (not per stream or thread).
+ * A library utility: no counterpart in the paper. */
+void ds_bf16_set_wait_limit(long long cycles);
+
 /* ---------------------------------------------------------------------------
  * Accumulator width.  Each compute call proves, on the device and with no
  * host round trip, whether 32-bit accumulation is exact:

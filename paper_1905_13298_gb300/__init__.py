@@ -99,6 +99,7 @@ _SIGNATURES = {
                                             ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
                                             ctypes.c_uint32, ctypes.c_void_p]),
     "ds_bf16_fault_flag": (ctypes.c_int, []),
+    "ds_bf16_set_wait_limit": (None, [ctypes.c_longlong]),
     "ds_absmax": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]),
     "ds_quantize_shift_weights": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_void_p,
                                                  ctypes.c_void_p, ctypes.c_void_p]),
@@ -257,6 +258,10 @@ def ds_linear_shift_bf16(x, w: ds_weights, bias, y, M: int, K: int, N: int, flag
 
 def ds_bf16_fault_flag() -> int:
     return int(lib().ds_bf16_fault_flag())
+
+
+def ds_bf16_set_wait_limit(cycles: int) -> None:
+    lib().ds_bf16_set_wait_limit(cycles)
 
 
 def ds_absmax(x, n: int, amax, stream=None) -> None:

@@ -420,6 +420,8 @@ ds_status ds_linear_shift_bf16(const uint16_t* x, const ds_weights* w, const flo
 
 int ds_bf16_fault_flag(void) { return read_bf16_fault_flag(); }
 
+void ds_bf16_set_wait_limit(long long cycles) { set_bf16_wait_cycles(cycles); }
+
 ds_status ds_linear_shift_backward_x(const int32_t* dy, const ds_weights* w_bwd, int32_t* dx, int64_t M, int64_t K,
                                      int64_t N, uint32_t flags, uint32_t* amax_io, void* stream) {
   clear_error();

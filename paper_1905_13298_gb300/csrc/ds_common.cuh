@@ -114,6 +114,7 @@ cudaError_t launch_expand_bf16(const uint8_t* blob, int64_t n_out, int64_t k_red
 cudaError_t launch_linear_bf16(const uint16_t* x, const uint16_t* w16, const float* bias, float* y, int64_t M,
                                int64_t K, int64_t N, uint32_t flags, cudaStream_t st);
 int read_bf16_fault_flag();
+void set_bf16_wait_cycles(long long cycles);
 // Defined in chain_ops.cu.
 cudaError_t launch_maxpool(const int32_t* x, int32_t* y, int64_t planes, int H, int W, int OH, int OW, int R,
                            int S, int stride, int pad, cudaStream_t st);

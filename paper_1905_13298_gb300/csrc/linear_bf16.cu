@@ -26,6 +26,8 @@
 // bounded by a clock deadline; on expiry the kernel records a fault flag,
 // stops issuing work, waits (bounded) for issued work and frees its TMEM.
 #include <cuda.h>
+
+#include <atomic>
 #include <cudaTypedefs.h>
 
 #include "ds_common.cuh"
@@ -45,12 +47,15 @@ constexpr int TMEM_COLS = ACC_BUFS * BN;  // 512: the whole tensor memory of an 
 constexpr int kThreads = 192;
 constexpr int kEpiWarps = 4;
 constexpr long long kTimeoutCycles = 4000000000LL;  // about 2 s at 2 GHz
+// the wait limit of the next launches (a diagnostic can shorten it to make the waits run out)
+std::atomic<long long> g_wait_cycles{kTimeoutCycles};
 
 struct Bf16Params {
   float* y;
   const float* bias;
   int64_t M, N, K;
   uint32_t flags;
+  long long wait_cycles;  // limit of a bounded wait before the launch gives up (the fault flag)
 };
 
 struct __align__(8) Barriers {
@@ -90,11 +95,11 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 // Bounded wait for the phase with the given parity; false when the CTA
 // aborted or the deadline passed (then the fault flag and abort are set).
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort, long long limit) {
   const long long t0 = clock64();
   while (!mbar_try_wait(bar, parity)) {
     if (*abort) return false;
-    if (clock64() - t0 > kTimeoutCycles) {
+    if (clock64() - t0 > limit) {
       *abort = 1;
       atomicExch(&g_bf16_fault, 1);
       return false;
@@ -102,7 +107,9 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
   }
   return true;
 }
-// Bounded wait that ignores the abort flag (draining work already issued).
+// Bounded wait that ignores the abort flag (draining work already issued);
+// always the full limit, so that issued copies and MMAs land before the CTA
+// frees its tensor memory or exits.
 __device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity) {
   const long long t0 = clock64();
   while (!mbar_try_wait(bar, parity) && clock64() - t0 < kTimeoutCycles) {
@@ -208,7 +215,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int kt = 0; kt < nk; ++kt, ++it) {
           const int s = (int)(it % STAGES);
           const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
-          if (it >= STAGES && !mbar_wait(&bars->empty[s], ph ^ 1u, abort)) {
+          if (it >= STAGES && !mbar_wait(&bars->empty[s], ph ^ 1u, abort, P.wait_cycles)) {
             ok = false;
             break;
           }
@@ -231,13 +238,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int64_t t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++i) {
         const int b = (int)(i & 1);
         // accumulator b is free once the epilogue has read tile i - 2 out of it
-        if (i >= ACC_BUFS && !mbar_wait(&bars->tempty[b], (uint32_t)((i / ACC_BUFS) - 1) & 1u, abort)) break;
+        if (i >= ACC_BUFS && !mbar_wait(&bars->tempty[b], (uint32_t)((i / ACC_BUFS) - 1) & 1u, abort, P.wait_cycles)) break;
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         const uint32_t tmem_d = tmem_base + (uint32_t)(b * BN);
         for (int kt = 0; kt < nk; ++kt, ++it) {
           const int s = (int)(it % STAGES);
           const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
-          if (!mbar_wait(&bars->full[s], ph, abort)) {
+          if (!mbar_wait(&bars->full[s], ph, abort, P.wait_cycles)) {
             ok = false;
             break;
           }
@@ -263,7 +270,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     int64_t i = 0;
     for (int64_t t = blockIdx.x; t < ntiles; t += gridDim.x, ++i) {
       const int b = (int)(i & 1);
-      if (!mbar_wait(&bars->tfull[b], (uint32_t)(i / ACC_BUFS) & 1u, abort)) break;
+      if (!mbar_wait(&bars->tfull[b], (uint32_t)(i / ACC_BUFS) & 1u, abort, P.wait_cycles)) break;
       asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
       int tm0, tn0;
       tile_of(t, tiles_m, tiles_n, G, tm0, tn0);
@@ -420,11 +427,15 @@ cudaError_t launch_linear_bf16(const uint16_t* x, const uint16_t* w16, const flo
     return n;
   }();
   if (sms <= 0) return cudaErrorInvalidDevice;
-  Bf16Params p{y, bias, M, N, K, flags};
+  Bf16Params p{y, bias, M, N, K, flags, g_wait_cycles.load(std::memory_order_relaxed)};
   const int64_t tiles = ((M + BM - 1) / BM) * ((N + BN - 1) / BN);
   const unsigned grid = (unsigned)(tiles < sms ? tiles : sms);  // persistent: one CTA per SM
   linear_bf16_kernel<<<grid, kThreads, smem, st>>>(mx, mw, p);
   return cudaGetLastError();
+}
+
+void set_bf16_wait_cycles(long long cycles) {
+  g_wait_cycles.store(cycles > 0 ? cycles : kTimeoutCycles, std::memory_order_relaxed);
 }
 
 int read_bf16_fault_flag() {

@@ -102,3 +102,29 @@ def test_bf16_config4_float_sampled(dslib):
     y, _ = _run(dslib, bits, s, p, b)
     rows = np.array([0, 1, 127, 128, 4095, 8191])
     _check(y, bits, s, p, b, rows=rows)
+
+
+def test_bounded_wait_expiry_is_reported_and_recovered(dslib):
+    """Failure detection without a fault: with the wait limit cut to one cycle every launch's first bounded wait
+    runs out, so the launch stops issuing, lets its issued copies and MMAs finish, frees its tensor memory and sets
+    the fault flag.  The flag reads 1 (and reading clears it); with the default limit restored the next call is
+    correct and reads 0."""
+    ds = dslib
+    bits, s, p, b = _case(77, 256, 512, 512)
+    x = torch.from_numpy(bits.view(np.int16)).cuda().view(torch.bfloat16)
+    w = ds.pack_shift_weights(torch.from_numpy(s).cuda(), torch.from_numpy(p).cuda())
+    ds.expand_shift_weights_bf16(w)
+    bd = torch.from_numpy(b).cuda()
+    assert ds.ds_bf16_fault_flag() == 0
+    try:
+        ds.ds_bf16_set_wait_limit(1)
+        ds.linear_shift_bf16(x, w, bd)
+        torch.cuda.synchronize()
+    finally:
+        ds.ds_bf16_set_wait_limit(0)
+    assert ds.ds_bf16_fault_flag() == 1
+    assert ds.ds_bf16_fault_flag() == 0  # read and cleared
+    y = ds.linear_shift_bf16(x, w, bd)
+    torch.cuda.synchronize()
+    assert ds.ds_bf16_fault_flag() == 0
+    _check(y.cpu().numpy().astype(np.float64), bits, s, p, b)
