@@ -7,15 +7,36 @@
 
 namespace ds {
 
+// Output e = (plane, oh, ow) of a pool: below 2^31 outputs the coordinates
+// come from two multiply-shift divisions, else from 64-bit ones.
+struct PoolIndex {
+  FastDiv d_ow, d_oh;
+  bool fast;
+};
+__device__ __forceinline__ void pool_coords(int64_t e, int OH, int OW, const PoolIndex& ix, int64_t& pl, int& oh,
+                                            int& ow) {
+  if (ix.fast) {
+    const int t = fdiv((int)e, ix.d_ow);
+    ow = (int)e - t * OW;
+    const int p = fdiv(t, ix.d_oh);
+    oh = t - p * OH;
+    pl = p;
+  } else {
+    ow = (int)(e % OW);
+    const int64_t t = e / OW;
+    oh = (int)(t % OH);
+    pl = t / OH;
+  }
+}
+
 __global__ void maxpool_kernel(const int32_t* __restrict__ x, int32_t* __restrict__ y, int64_t planes,
-                               int H, int W, int OH, int OW, int R, int S, int stride, int pad) {
+                               int H, int W, int OH, int OW, int R, int S, int stride, int pad, PoolIndex ix) {
   const int64_t total = planes * OH * OW;
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
        e += (int64_t)gridDim.x * blockDim.x) {
-    const int ow = (int)(e % OW);
-    const int64_t t = e / OW;
-    const int oh = (int)(t % OH);
-    const int64_t pl = t / OH;
+    int64_t pl;
+    int oh, ow;
+    pool_coords(e, OH, OW, ix, pl, oh, ow);
     const int32_t* xp = x + pl * H * W;
     int32_t m = INT32_MIN;
     for (int r = 0; r < R; ++r) {
@@ -32,15 +53,14 @@ __global__ void maxpool_kernel(const int32_t* __restrict__ x, int32_t* __restric
 }
 
 __global__ void avgpool_floor_kernel(const int32_t* __restrict__ x, int32_t* __restrict__ y, int64_t planes,
-                                     int H, int W, int OH, int OW, int R, int S, int stride) {
+                                     int H, int W, int OH, int OW, int R, int S, int stride, PoolIndex ix) {
   const int64_t total = planes * OH * OW;
   const int64_t d = (int64_t)R * S;
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
        e += (int64_t)gridDim.x * blockDim.x) {
-    const int ow = (int)(e % OW);
-    const int64_t t = e / OW;
-    const int oh = (int)(t % OH);
-    const int64_t pl = t / OH;
+    int64_t pl;
+    int oh, ow;
+    pool_coords(e, OH, OW, ix, pl, oh, ow);
     const int32_t* xp = x + pl * H * W + (int64_t)oh * stride * W + (int64_t)ow * stride;
     int64_t sum = 0;
     for (int r = 0; r < R; ++r)
@@ -49,6 +69,11 @@ __global__ void avgpool_floor_kernel(const int32_t* __restrict__ x, int32_t* __r
     if (sum % d != 0 && sum < 0) --q;  // floor
     y[e] = (int32_t)q;
   }
+}
+
+static PoolIndex pool_index(int64_t planes, int OH, int OW) {
+  const int64_t total = planes * OH * OW;
+  return PoolIndex{make_fastdiv((uint32_t)OW), make_fastdiv((uint32_t)OH), total <= (int64_t)INT32_MAX};
 }
 
 static int64_t pool_blocks(int64_t total, int threads) {
@@ -60,8 +85,8 @@ static int64_t pool_blocks(int64_t total, int threads) {
 cudaError_t launch_maxpool(const int32_t* x, int32_t* y, int64_t planes, int H, int W, int OH, int OW, int R,
                            int S, int stride, int pad, cudaStream_t st) {
   const int threads = 256;
-  maxpool_kernel<<<(unsigned)pool_blocks(planes * OH * OW, threads), threads, 0, st>>>(x, y, planes, H, W, OH, OW,
-                                                                                       R, S, stride, pad);
+  maxpool_kernel<<<(unsigned)pool_blocks(planes * OH * OW, threads), threads, 0, st>>>(
+      x, y, planes, H, W, OH, OW, R, S, stride, pad, pool_index(planes, OH, OW));
   return cudaGetLastError();
 }
 
@@ -69,7 +94,7 @@ cudaError_t launch_avgpool_floor(const int32_t* x, int32_t* y, int64_t planes, i
                                  int R, int S, int stride, cudaStream_t st) {
   const int threads = 256;
   avgpool_floor_kernel<<<(unsigned)pool_blocks(planes * OH * OW, threads), threads, 0, st>>>(
-      x, y, planes, H, W, OH, OW, R, S, stride);
+      x, y, planes, H, W, OH, OW, R, S, stride, pool_index(planes, OH, OW));
   return cudaGetLastError();
 }
 

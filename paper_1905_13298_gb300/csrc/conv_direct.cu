@@ -48,24 +48,6 @@ constexpr int kMaxCluster = 16;         // CTAs per thread-block cluster (non-po
 // n * HP + ihp (HP = H + 2 * pad); output row (n, oh) reads stacked rows
 // n * HP + oh * sig + r.  A tile's halo is the contiguous stacked range its
 // rows read, HR rows at most.
-// Division by a runtime constant d >= 1 of numerators 0 <= n < 2^31 as one
-// widening multiply and a shift (Granlund and Montgomery, "Division by
-// invariant integers using multiplication", PLDI 1994, Thm. 4.2): with
-// l = ceil(log2 d) and m = floor(2^(31+l) / d) + 1, m*d - 2^(31+l) <= d <= 2^l,
-// hence floor(n / d) = floor(n * m / 2^(31+l)) for every such n, and m < 2^32.
-struct FastDiv {
-  uint32_t m;
-  int sh;
-};
-inline FastDiv make_fastdiv(uint32_t d) {
-  int l = 0;
-  while ((1ull << l) < d) ++l;
-  return FastDiv{(uint32_t)((1ull << (31 + l)) / d + 1), 31 + l};
-}
-__device__ __forceinline__ int fdiv(int n, FastDiv f) {
-  return (int)(((uint64_t)(uint32_t)n * f.m) >> f.sh);
-}
-
 struct DirectGeom {
   int TH, GW;        // output rows and pixel groups per row per CTA
   int threads;       // TH * GW * CG
@@ -513,23 +495,68 @@ __global__ void __launch_bounds__(kMaxThreads, 3) conv_direct_kernel(const GemmP
 }
 
 // Epilogue of a split reduction: y = ReLU?(sat32(sat32(acc + bias) + residual)), amax.
-__global__ void conv_split_finalize_kernel(const GemmParams P, int64_t total) {
-  const int64_t OHW = (int64_t)P.OH * P.OW;
+// Quad path (total a multiple of 4 below 2^31, 16-byte aligned y and
+// residual): a thread takes 4 consecutive outputs with 16-byte loads of the
+// int64 partial sums and of the residual and one 16-byte store; the first
+// output's channel comes from two multiply-shift divisions, the others step
+// along (a quad may cross a channel plane).  Otherwise one output per thread
+// with 64-bit divisions.
+__global__ void conv_split_finalize_kernel(const GemmParams P, int64_t total, FastDiv d_ohw, FastDiv d_cols,
+                                           bool quad) {
   const bool relu = (P.flags & DS_RELU) != 0;
   const bool resid = (P.flags & DS_RESIDUAL) != 0;
+  const int64_t prefix = (int64_t)(kSmallScratchBytes / sizeof(int64_t));  // the zero prefix
   uint32_t amax_local = 0;
-  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
-       e += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t col = (e / OHW) % P.cols;
-    int64_t a = P.split_acc[e] + (P.bias ? (int64_t)__ldg(P.bias + col) : 0);
-    if (e < (int64_t)(kSmallScratchBytes / sizeof(int64_t))) P.split_acc[e] = 0;  // the zero prefix
-    a = a > (int64_t)INT32_MAX ? (int64_t)INT32_MAX : a;
-    a = a < (int64_t)INT32_MIN ? (int64_t)INT32_MIN : a;
-    int32_t o = (int32_t)a;
-    if (resid) o = add_sat(o, __ldg(P.residual + e));
-    if (relu) o = max(o, 0);
-    amax_local = max(amax_local, uabs(o));
-    P.y[e] = o;
+  if (quad) {
+    const int OHW = P.OH * P.OW;
+    const int cols = (int)P.cols;
+    const longlong2* acc2 = reinterpret_cast<const longlong2*>(P.split_acc);
+    for (int64_t q = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; q < total / 4;
+         q += (int64_t)gridDim.x * blockDim.x) {
+      const int e = (int)(q * 4);
+      const int plane = fdiv(e, d_ohw);
+      int pix = e - plane * OHW;
+      int col = plane - fdiv(plane, d_cols) * cols;
+      const longlong2 a01 = acc2[2 * q], a23 = acc2[2 * q + 1];
+      if (e < prefix) {
+        reinterpret_cast<longlong2*>(P.split_acc)[2 * q] = make_longlong2(0, 0);
+        reinterpret_cast<longlong2*>(P.split_acc)[2 * q + 1] = make_longlong2(0, 0);
+      }
+      const int4 r4 = resid ? __ldg(reinterpret_cast<const int4*>(P.residual) + q) : make_int4(0, 0, 0, 0);
+      const int64_t a[4] = {a01.x, a01.y, a23.x, a23.y};
+      const int32_t rv[4] = {r4.x, r4.y, r4.z, r4.w};
+      int32_t o[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        int64_t v = a[i] + (P.bias ? (int64_t)__ldg(P.bias + col) : 0);
+        v = v > (int64_t)INT32_MAX ? (int64_t)INT32_MAX : v;
+        v = v < (int64_t)INT32_MIN ? (int64_t)INT32_MIN : v;
+        o[i] = (int32_t)v;
+        if (resid) o[i] = add_sat(o[i], rv[i]);
+        if (relu) o[i] = max(o[i], 0);
+        amax_local = max(amax_local, uabs(o[i]));
+        if (++pix == OHW) {
+          pix = 0;
+          col = col + 1 == cols ? 0 : col + 1;
+        }
+      }
+      reinterpret_cast<int4*>(P.y)[q] = make_int4(o[0], o[1], o[2], o[3]);
+    }
+  } else {
+    const int64_t OHW = (int64_t)P.OH * P.OW;
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
+         e += (int64_t)gridDim.x * blockDim.x) {
+      const int64_t col = (e / OHW) % P.cols;
+      int64_t a = P.split_acc[e] + (P.bias ? (int64_t)__ldg(P.bias + col) : 0);
+      if (e < prefix) P.split_acc[e] = 0;
+      a = a > (int64_t)INT32_MAX ? (int64_t)INT32_MAX : a;
+      a = a < (int64_t)INT32_MIN ? (int64_t)INT32_MIN : a;
+      int32_t o = (int32_t)a;
+      if (resid) o = add_sat(o, __ldg(P.residual + e));
+      if (relu) o = max(o, 0);
+      amax_local = max(amax_local, uabs(o));
+      P.y[e] = o;
+    }
   }
   if (P.amax_out != nullptr) {
     amax_local = __reduce_max_sync(0xffffffffu, amax_local);
@@ -819,9 +846,16 @@ cudaError_t prepare_split_scratch(const GemmParams& p, cudaStream_t st) {
 
 cudaError_t launch_split_finalize(const GemmParams& p, cudaStream_t st) {
   const int64_t total = p.rows * p.cols;
-  int64_t blocks = (total + 255) / 256;
+  const bool quad = total % 4 == 0 && total <= (int64_t)INT32_MAX && (reinterpret_cast<uintptr_t>(p.y) & 15) == 0 &&
+                    (reinterpret_cast<uintptr_t>(p.split_acc) & 15) == 0 &&
+                    (!(p.flags & DS_RESIDUAL) || (reinterpret_cast<uintptr_t>(p.residual) & 15) == 0);
+  const int64_t items = quad ? total / 4 : total;
+  int64_t blocks = (items + 255) / 256;
   if (blocks > std::max<int64_t>(slots(), 1) * 8) blocks = std::max<int64_t>(slots(), 1) * 8;
-  conv_split_finalize_kernel<<<(unsigned)blocks, 256, 0, st>>>(p, total);
+  if (blocks < 1) blocks = 1;
+  const FastDiv d_ohw = make_fastdiv((uint32_t)((int64_t)p.OH * p.OW));
+  const FastDiv d_cols = make_fastdiv((uint32_t)(p.cols < 1 ? 1 : (p.cols > INT32_MAX ? INT32_MAX : p.cols)));
+  conv_split_finalize_kernel<<<(unsigned)blocks, 256, 0, st>>>(p, total, d_ohw, d_cols, quad);
   return cudaGetLastError();
 }
 

@@ -54,6 +54,26 @@ struct BlobHeader {
 };
 static_assert(sizeof(BlobHeader) == 48, "header layout");
 
+// Division by a runtime constant d >= 1 of numerators 0 <= n < 2^31 as one
+// widening multiply and a shift (Granlund and Montgomery, "Division by
+// invariant integers using multiplication", PLDI 1994, Thm. 4.2): with
+// l = ceil(log2 d) and m = floor(2^(31+l) / d) + 1, m*d - 2^(31+l) <= d <= 2^l,
+// hence floor(n / d) = floor(n * m / 2^(31+l)) for every such n, and m < 2^32.
+struct FastDiv {
+  uint32_t m;
+  int sh;
+};
+inline FastDiv make_fastdiv(uint32_t d) {
+  int l = 0;
+  while ((1ull << l) < d) ++l;
+  return FastDiv{(uint32_t)((1ull << (31 + l)) / d + 1), 31 + l};
+}
+#ifdef __CUDACC__
+__device__ __forceinline__ int fdiv(int n, FastDiv f) {
+  return (int)(((uint64_t)(uint32_t)n * f.m) >> f.sh);
+}
+#endif
+
 // ---------------------------------------------------------------------------
 // Parameters of the shift-GEMM kernels (FC and conv implicit GEMM).
 // The GEMM view: rows = FC rows m or conv output pixels (n, oh, ow);
