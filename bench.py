@@ -63,6 +63,11 @@ def workload_by_name(name: str, batch):
         n = n_out * k_red
         return dict(name="pack_weights_vgg16_fc1_4096x25088", kind="pack", n=n, n_out=n_out, k_red=k_red,
                     bytes=2 * n + n * 3 // 4 + 12 * n_out)
+    if name == "specialized_vgg16_conv1":
+        # VGG16's first conv (3 -> 64, 3x3/1/1, 1728 weights) with its codes compiled into the kernel
+        b = batch or 64
+        return dict(name=f"specialized_convshift_vgg16_conv1_b{b}_224", kind="spec", N=b, C=3, H=224, W=224, K=64,
+                    R=3, S=3, stride=1, pad=1, terms=b * 64 * 224 * 224 * 27)
     if name == "quantize_vgg16_fc1":
         # float32 weights of VGG16's first FC layer -> int8 sign and shift codes (DeepShift-Q)
         n = 4096 * 25088
@@ -481,6 +486,71 @@ def time_fc_layer(args, ds, dev, seed, M, K, N, backward=False):
                 frac=2 * terms / (ms / 1e3) / (alu_peak(dev)[0] * 1e12))
 
 
+def run_specialized(args, wl, local_rank):
+    """One small layer through the weight-specialised ConvShift (codes compiled into the kernel) and, on the same
+    inputs, through the generic kernels: value = Gshift-ops/s of the specialised call."""
+    import torch
+    import paper_1905_13298_gb300 as ds
+    from paper_1905_13298_gb300 import build as dsb
+
+    dsb.build_library()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    N, C, H, W, K, R, S, stv, pd = (wl[k] for k in ("N", "C", "H", "W", "K", "R", "S", "stride", "pad"))
+    x, s, p, b = si.conv_layer(si.SEED_BASE + 49, N, C, H, W, K, R, S, -(1 << 17), 1 << 17, si.layer_centre(C, R, S))
+    OH, OW = (H + 2 * pd - R) // stv + 1, (W + 2 * pd - S) // stv + 1
+    t0 = time.perf_counter()
+    h = ds.ds_specialize_conv2d_shift(s, p, K, C, R, S, stv, pd)
+    compile_s = time.perf_counter() - t0
+    xd, bd = torch.from_numpy(x).to(dev), torch.from_numpy(b).to(dev)
+    y = torch.empty((N, K, OH, OW), dtype=torch.int32, device=dev)
+    a = torch.zeros(2, dtype=torch.int32, device=dev)
+    st = torch.cuda.current_stream().cuda_stream
+    ds.ds_absmax(xd, xd.numel(), a, st)
+    w = ds.pack_shift_weights(torch.from_numpy(s).to(dev), torch.from_numpy(p).to(dev), expand=True)
+
+    def spec():
+        ds.ds_conv2d_shift_specialized(h, xd, bd, None, y, N, H, W, ds.DS_RELU | ds.DS_AMAX_IN, a, st)
+
+    def generic():
+        ds.ds_conv2d_shift(xd, w.desc, bd, None, y, N, C, H, W, K, R, S, stv, stv, pd, pd,
+                           ds.DS_RELU | ds.DS_AMAX_IN, a, st)
+
+    def timed(fn, clocks=False):
+        for _ in range(max(3, args.warmup)):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        sampler = ClockSampler(local_rank) if clocks else None
+        if sampler:
+            sampler.start()
+            time.sleep(0.3)
+        e0.record()
+        for _ in range(args.steps):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / args.steps, (sampler.stop() if sampler else None)
+
+    ms_gen, _ = timed(generic)
+    ms, clocks = timed(spec, clocks=True)
+    ds.ds_specialized_destroy(h)
+    alu_tops = alu_peak(dev)[0]
+    terms = wl["terms"]
+    frac = 2 * terms / (ms / 1e3) / (alu_tops * 1e12)
+    out = {"metric": METRIC, "value": terms / ms / 1e6, "unit": METRIC, "n_gpus": 1, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+           "dtype": "int32", "data": "synthetic",
+           "config": {"workload": wl["name"], "compile_seconds": round(compile_s, 2), "generic_ms": ms_gen,
+                      "generic_frac": 2 * terms / (ms_gen / 1e3) / (alu_tops * 1e12),
+                      "zero_weights_elided": int((s == 0).sum()), "weights": int(s.size)},
+           "roofline": {"bound": "alu", "achieved": 2 * terms / (ms / 1e3) / 1e12, "peak": alu_tops,
+                        "unit": "Tintop/s", "frac": frac, "traffic": None,
+                        "kernel": "ds_shift_conv_specialized (NVRTC)"},
+           "gpu_launches": args.steps, "clocks": clocks}
+    print(json.dumps(out), flush=True)
+
+
 def run_layer_sweep(args, wl, local_rank):
     """Every conv and FC layer of the network standalone (own inputs, same shapes as in the chain)."""
     import torch
@@ -825,7 +895,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extras", action="store_true",
                     help="default workload: skip the ResNet18 forward and sustained-clock sub-records")
-    ap.add_argument("--workload", default="conv2x", choices=["conv2x", "fc_large", "fc_vgg16_fc1", "fc_large_bf16", "pack_vgg16_fc1", "quantize_vgg16_fc1", "q16_input", "resnet18", "resnet50", "vgg16",
+    ap.add_argument("--workload", default="conv2x", choices=["conv2x", "fc_large", "fc_vgg16_fc1", "fc_large_bf16", "pack_vgg16_fc1", "specialized_vgg16_conv1", "quantize_vgg16_fc1", "q16_input", "resnet18", "resnet50", "vgg16",
                                                          "sweep_resnet18", "sweep_resnet50", "sweep_vgg16",
                                                          "sweep_resnet18_backward", "sweep_resnet50_backward"])
     ap.add_argument("--layers", default=None,
@@ -847,6 +917,8 @@ def main():
         run_gpu(args, wl, rank, world, local_rank)
     elif wl["kind"] == "sweep":
         run_layer_sweep(args, wl, local_rank)
+    elif wl["kind"] == "spec":
+        run_specialized(args, wl, local_rank)
     elif wl["kind"] in ("quant", "q16", "pack"):
         run_conversion(args, wl, local_rank)
     else:

@@ -431,6 +431,36 @@ ds_status ds_quantize_q16(const float* x, int64_t n, int32_t* q, void* stream);
  */
 ds_status ds_absmax(const int32_t* x, int64_t n, uint32_t* amax, void* stream);
 
+/* ---------------------------------------------------------------------------
+ * Weight-specialised ConvShift (Eq. 3, as ds_conv2d_shift; specialising the kernels to the weights at run time is
+ * the future work of Sec. 6.1).  For a small layer the library writes a kernel in which every weight's shift and
+ * sign are immediates and the zero weights are left out, so a term is one shift by an immediate and one add or
+ * subtract (no shift for p = 0), with no code loads; it compiles the kernel at run time with NVRTC (libnvrtc,
+ * opened on first use) for the current device and keeps it in the returned handle.  Meant for the few-thousand-
+ * weight layers at the input of a network (VGG16's first conv: 1728 weights), where the whole layer fits the
+ * instruction stream.
+ *
+ * ds_specialize_conv2d_shift: s, p HOST int8 codes [K][C][R][S] (s in {-1, 0, +1}, p in [-15, 0]); square
+ * stride (1 or 2) and padding (below R and S); K*C*R*S <= DS_SPECIALIZE_MAX_WEIGHTS, R, S <= 11.  Compiles and
+ * loads (seconds for the largest layers; not stream-ordered, not for a capture).  On success *out owns the kernel
+ * until ds_specialized_destroy.  Errors: DS_ERR_INVALID_ARG (NULL), DS_ERR_SHAPE, DS_ERR_CODE_RANGE,
+ * DS_ERR_UNSUPPORTED (too many weights or channels for the shared-memory tile, NVRTC missing or failing),
+ * DS_ERR_CUDA.
+ *
+ * ds_conv2d_shift_specialized: the layer on x [N][C][H][W] -> y [N][K][OH][OW] (NCHW int32, 16-byte aligned,
+ * not overlapping), bias, residual, flags (DS_RELU, DS_RESIDUAL, DS_AMAX_IN, DS_AMAX_OUT, DS_FORCE_INT64) and
+ * amax_io exactly as ds_conv2d_shift; the same accumulator-width proof picks 32- or 64-bit sums per CTA.  Use it
+ * on the device it was specialised on.  Stream-ordered, allocates nothing.
+ * ------------------------------------------------------------------------- */
+#define DS_SPECIALIZE_MAX_WEIGHTS 4096
+typedef struct ds_specialized ds_specialized;
+ds_status ds_specialize_conv2d_shift(const int8_t* s, const int8_t* p, int K, int C, int R, int S, int stride,
+                                     int pad, ds_specialized** out);
+ds_status ds_conv2d_shift_specialized(const ds_specialized* h, const int32_t* x, const int32_t* bias,
+                                      const int32_t* residual, int32_t* y, int N, int H, int W, uint32_t flags,
+                                      uint32_t* amax_io, void* stream);
+void ds_specialized_destroy(ds_specialized* h);
+
 #ifdef __cplusplus
 }
 #endif

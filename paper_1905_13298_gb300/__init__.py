@@ -100,6 +100,11 @@ _SIGNATURES = {
                                             ctypes.c_uint32, ctypes.c_void_p]),
     "ds_bf16_fault_flag": (ctypes.c_int, []),
     "ds_bf16_set_wait_limit": (None, [ctypes.c_longlong]),
+    "ds_specialize_conv2d_shift": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p] + [ctypes.c_int] * 6 +
+                                   [ctypes.POINTER(ctypes.c_void_p)]),
+    "ds_conv2d_shift_specialized": (ctypes.c_int, [ctypes.c_void_p] * 5 + [ctypes.c_int] * 3 +
+                                    [ctypes.c_uint32, ctypes.c_void_p, ctypes.c_void_p]),
+    "ds_specialized_destroy": (None, [ctypes.c_void_p]),
     "ds_absmax": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p]),
     "ds_quantize_shift_weights": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_void_p,
                                                  ctypes.c_void_p, ctypes.c_void_p]),
@@ -262,6 +267,29 @@ def ds_bf16_fault_flag() -> int:
 
 def ds_bf16_set_wait_limit(cycles: int) -> None:
     lib().ds_bf16_set_wait_limit(cycles)
+
+
+def ds_specialize_conv2d_shift(s, p, K: int, C: int, R: int, S: int, stride: int, pad: int) -> int:
+    """s, p: HOST int8 arrays [K][C][R][S] (numpy, C-contiguous).  Returns the handle (an address)."""
+    import numpy as np
+    s = np.ascontiguousarray(s, dtype=np.int8)
+    p = np.ascontiguousarray(p, dtype=np.int8)
+    if s.size != K * C * R * S or p.size != K * C * R * S:
+        raise DsError(DS_ERR_SHAPE, "codes must hold K*C*R*S values")
+    out = ctypes.c_void_p()
+    _check(lib().ds_specialize_conv2d_shift(s.ctypes.data, p.ctypes.data, K, C, R, S, stride, pad,
+                                            ctypes.byref(out)))
+    return int(out.value)
+
+
+def ds_conv2d_shift_specialized(h: int, x, bias, residual, y, N: int, H: int, W: int, flags: int = 0,
+                                amax_io=None, stream=None) -> None:
+    _check(lib().ds_conv2d_shift_specialized(h, _ptr(x), _ptr(bias), _ptr(residual), _ptr(y), N, H, W, flags,
+                                             _ptr(amax_io), _stream(stream)))
+
+
+def ds_specialized_destroy(h: int) -> None:
+    lib().ds_specialized_destroy(h)
 
 
 def ds_absmax(x, n: int, amax, stream=None) -> None:

@@ -639,3 +639,62 @@ ds_status ds_conv2d_shift(const int32_t* x, const ds_weights* w, const int32_t* 
 }
 
 }  // extern "C"
+
+extern "C" {
+
+ds_status ds_specialize_conv2d_shift(const int8_t* s, const int8_t* p, int K, int C, int R, int S, int stride,
+                                     int pad, ds_specialized** out) {
+  clear_error();
+  if (!s || !p || !out) return fail(DS_ERR_INVALID_ARG, "NULL pointer argument");
+  *out = nullptr;
+  if (K <= 0 || C <= 0 || R <= 0 || S <= 0) return fail(DS_ERR_SHAPE, "K, C, R and S must be positive");
+  if (stride < 1 || stride > 2 || pad < 0 || pad >= R || pad >= S || R > 11 || S > 11)
+    return fail(DS_ERR_UNSUPPORTED, "specialisation supports strides 1 and 2, kernels up to 11, pads below the kernel");
+  const int64_t n = (int64_t)K * C * R * S;
+  if (n > DS_SPECIALIZE_MAX_WEIGHTS)
+    return fail(DS_ERR_UNSUPPORTED, "%lld weights: specialisation holds at most %d", (long long)n,
+                DS_SPECIALIZE_MAX_WEIGHTS);
+  for (int64_t i = 0; i < n; ++i)
+    if (s[i] < -1 || s[i] > 1 || p[i] < -15 || p[i] > 0)
+      return fail(DS_ERR_CODE_RANGE, "code %lld out of range (s = %d, p = %d)", (long long)i, s[i], p[i]);
+  return specialize_conv(s, p, K, C, R, S, stride, pad, out);
+}
+
+ds_status ds_conv2d_shift_specialized(const ds_specialized* h, const int32_t* x, const int32_t* bias,
+                                      const int32_t* residual, int32_t* y, int N, int H, int W, uint32_t flags,
+                                      uint32_t* amax_io, void* stream) {
+  clear_error();
+  if (!h) return fail(DS_ERR_INVALID_ARG, "NULL specialised layer");
+  if (!x || !y) return fail(DS_ERR_INVALID_ARG, "NULL x or y");
+  if (N <= 0) return fail(DS_ERR_SHAPE, "N must be positive");
+  int K = 0, C = 0, R = 0, S = 0, stride = 0, pad = 0;
+  specialized_dims(h, &K, &C, &R, &S, &stride, &pad);
+  int OH = 0, OW = 0;
+  ds_status r = window_output(H, W, R, S, stride, stride, pad, pad, &OH, &OW);
+  if (r != DS_OK) return r;
+  const uint32_t known = DS_RELU | DS_AMAX_IN | DS_AMAX_OUT | DS_RESIDUAL | DS_FORCE_INT64;
+  if (flags & ~known) return fail(DS_ERR_INVALID_ARG, "unknown flag bits 0x%x", flags & ~known);
+  if ((flags & DS_RESIDUAL) && residual == nullptr)
+    return fail(DS_ERR_INVALID_ARG, "DS_RESIDUAL needs a residual tensor");
+  if ((flags & (DS_AMAX_IN | DS_AMAX_OUT)) && amax_io == nullptr)
+    return fail(DS_ERR_INVALID_ARG, "DS_AMAX_IN / DS_AMAX_OUT need amax_io");
+  if (!aligned16(x) || !aligned16(y)) return fail(DS_ERR_ALIGNMENT, "x and y must be 16-byte aligned");
+  r = check_image(C, H, W, OH, OW);
+  if (r != DS_OK) return r;
+  const int64_t xb = int32_tensor_bytes({N, C, H, W}), yb = int32_tensor_bytes({N, K, OH, OW});
+  if (xb < 0 || yb < 0) return fail(DS_ERR_UNSUPPORTED, "x or y larger than 2^62 bytes");
+  if (ranges_overlap(x, xb, y, yb)) return fail(DS_ERR_INVALID_ARG, "y must not overlap x");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  GemmParams p{};
+  p.flags = flags;
+  r = prepare_amax(x, xb / (int64_t)sizeof(int32_t), flags, amax_io, st, p);
+  if (r != DS_OK) return r;
+  return cuda_check(launch_specialized(h, x, bias, (flags & DS_RESIDUAL) ? residual : nullptr, y, N, H, W, OH, OW,
+                                       flags, (flags & DS_FORCE_INT64) ? nullptr : p.amax_in, p.amax_out, st),
+                    "specialised conv2d_shift launch");
+}
+
+void ds_specialized_destroy(ds_specialized* h) { destroy_specialized(h); }
+
+}  // extern "C"
+

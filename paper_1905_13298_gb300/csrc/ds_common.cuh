@@ -156,6 +156,14 @@ ds_status fc_launch(const int32_t* x, const ds_weights* w, const int32_t* bias, 
 // Defined in quantize.cu (DeepShift-Q codes from float weights, Q16.16 from float activations).
 cudaError_t launch_quantize_weights(const float* w, int64_t n, int p_min, int8_t* s, int8_t* p, cudaStream_t st);
 cudaError_t launch_quantize_q16(const float* x, int64_t n, int32_t* q, cudaStream_t st);
+// Defined in specialize.cu (weight-specialised ConvShift compiled at run time).
+ds_status specialize_conv(const int8_t* s, const int8_t* p, int K, int C, int R, int S, int stride, int pad,
+                          ds_specialized** out);
+void specialized_dims(const ds_specialized* h, int* K, int* C, int* R, int* S, int* stride, int* pad);
+cudaError_t launch_specialized(const ds_specialized* h, const int32_t* x, const int32_t* bias,
+                               const int32_t* residual, int32_t* y, int N, int H, int W, int OH, int OW,
+                               uint32_t flags, const uint32_t* amax_in, uint32_t* amax_out, cudaStream_t st);
+void destroy_specialized(ds_specialized* h);
 // Defined in misc_kernels.cu.
 // Streaming multiprocessors of the device this process uses, read once per
 // process (one device per process); 0 when no device can be queried, in which

@@ -379,3 +379,25 @@ def test_network_output_shapes(ds):
     b = PN._Builder(64, 56, 56)
     b.pool(ds.DS_OP_MAXPOOL, 0, 3, 2, 1)
     assert PN.output_shape(b.specs[-1]) == (64, 28, 28)
+
+
+def test_specialisation_validates_before_compiling(ds):
+    """The weight-specialised ConvShift refuses bad requests on the host, before NVRTC or any CUDA call."""
+    import numpy as np
+    L = ds.lib()
+    out = ctypes.c_void_p()
+    s = np.ones((4, 3, 3, 3), np.int8)
+    p = np.zeros((4, 3, 3, 3), np.int8)
+    assert L.ds_specialize_conv2d_shift(None, p.ctypes.data, 4, 3, 3, 3, 1, 1, ctypes.byref(out)) == ds.DS_ERR_INVALID_ARG
+    assert L.ds_specialize_conv2d_shift(s.ctypes.data, p.ctypes.data, 0, 3, 3, 3, 1, 1, ctypes.byref(out)) == ds.DS_ERR_SHAPE
+    assert L.ds_specialize_conv2d_shift(s.ctypes.data, p.ctypes.data, 4, 3, 3, 3, 3, 1, ctypes.byref(out)) == ds.DS_ERR_UNSUPPORTED
+    assert L.ds_specialize_conv2d_shift(s.ctypes.data, p.ctypes.data, 4, 3, 3, 3, 1, 3, ctypes.byref(out)) == ds.DS_ERR_UNSUPPORTED
+    big = np.ones((64, 3, 7, 7), np.int8)  # 9408 weights: more than the instruction stream should hold
+    assert L.ds_specialize_conv2d_shift(big.ctypes.data, np.zeros_like(big).ctypes.data, 64, 3, 7, 7, 2, 3,
+                                        ctypes.byref(out)) == ds.DS_ERR_UNSUPPORTED
+    bad = p.copy()
+    bad[1, 2, 0, 1] = 1  # a positive shift
+    assert L.ds_specialize_conv2d_shift(s.ctypes.data, bad.ctypes.data, 4, 3, 3, 3, 1, 1, ctypes.byref(out)) == ds.DS_ERR_CODE_RANGE
+    assert out.value is None
+    assert L.ds_conv2d_shift_specialized(None, 16, None, None, 4096, 1, 8, 8, 0, None, None) == ds.DS_ERR_INVALID_ARG
+    L.ds_specialized_destroy(None)  # a no-op
