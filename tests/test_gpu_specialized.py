@@ -1,6 +1,6 @@
 """GPU parity of the weight-specialised ConvShift (codes compiled into the kernel at run time) against the CPU
 oracle and the generic ConvShift kernels, bit-exact.  Each specialisation compiles a kernel with NVRTC (seconds),
-so the cases are few and small, plus VGG16's first layer (C = 3, 64 channels, 3x3) at one image."""
+so the cases are few and small, plus VGG16's first layer (C = 3, 64 channels, 3x3) at four images."""
 import numpy as np
 import pytest
 import torch
@@ -94,12 +94,30 @@ def test_specialized_zero_codes_give_the_bias(dslib):
 
 def test_specialized_vgg16_first_layer(dslib):
     """VGG16's first conv (3 -> 64, 3x3/1/1) at 224 x 224, the layer specialisation is meant for: every output of
-    one image against the oracle."""
+    four images against the oracle."""
     ds = dslib
-    x, s, p, b = si.conv_layer(904, 1, 3, 224, 224, 64, 3, 3, -(1 << 17), 1 << 17, si.layer_centre(3, 3, 3))
+    x, s, p, b = si.conv_layer(904, 4, 3, 224, 224, 64, 3, 3, -(1 << 17), 1 << 17, si.layer_centre(3, 3, 3))
     h = ds.ds_specialize_conv2d_shift(s, p, 64, 3, 3, 3, 1, 1)
     try:
-        got, _ = _run(ds, h, x, b, None, 1, 3, 224, 224, 64, 224, 224, ds.DS_RELU)
+        got, _ = _run(ds, h, x, b, None, 4, 3, 224, 224, 64, 224, 224, ds.DS_RELU)
         assert np.array_equal(got, O.conv2d_shift(x, s, p, b, (1, 1), (1, 1), relu=True))
+    finally:
+        ds.ds_specialized_destroy(h)
+
+
+def test_specialized_many_images_walk_tiles(dslib):
+    """Many small images (three row tiles each, the last one ragged) with a residual and no ReLU: a grid of
+    thousands of CTAs, the residual join saturating, max|y| over the joined outputs."""
+    ds = dslib
+    N, C, H, W, K, R = 640, 2, 40, 22, 8, 3
+    x, s, p, b = si.conv_layer(905, N, C, H, W, K, R, R, -(1 << 20), 1 << 20, -3)
+    res = si.activations(906, (N, K, H, W), -(1 << 30), 1 << 30)
+    h = ds.ds_specialize_conv2d_shift(s, p, K, C, R, R, 1, 1)
+    try:
+        got, amax = _run(ds, h, x, b, res, N, C, H, W, K, H, W, ds.DS_RESIDUAL)
+        # the residual join without ReLU: one saturation of the layer's output plus the residual
+        want = O.sat32(O.conv2d_shift(x, s, p, b, (1, 1), (1, 1)).astype(np.int64) + res.astype(np.int64))
+        assert amax[1] == O.absmax(want)
+        assert np.array_equal(got, want)
     finally:
         ds.ds_specialized_destroy(h)
