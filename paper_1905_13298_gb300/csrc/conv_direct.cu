@@ -41,6 +41,7 @@ constexpr int kSmemBudget = 74 * 1024;  // 3 CTAs per SM
 // resident CTAs of the device (3 per SM)
 inline int64_t slots() { return (int64_t)sm_count() * 3; }
 constexpr int kMaxCluster = 16;         // CTAs per thread-block cluster (non-portable maximum)
+constexpr int kChainClusterMaxTarget = 2;  // see choose_geom
 
 // The CTA tiles run over the stacked output rows gr = n * OH + oh of all
 // images, so a tile may span image boundaries (small feature maps, batch 1).
@@ -582,10 +583,7 @@ size_t direct_smem_bytes(const DirectGeom& G) {
 bool choose_geom(const GemmParams& p, size_t split_capacity, Choice& ch) {
   DirectGeom& G = ch.G;
   ch.TM = (p.OW % 7 == 0) ? 7 : 8;
-  // Cluster split for calls without a workspace (the kernels with a cluster
-  // variant); with a workspace (the chained forward) the atomic split is
-  // used: measured faster there (ResNet18 batch 1: 0.51 vs 0.63 ms per forward).
-  const bool allow_cluster = split_capacity == 0 && ch.TM == 7 && (p.S == 3 || p.S == 7);
+  const bool has_cluster = ch.TM == 7 && (p.S == 3 || p.S == 7);  // the kernels with a cluster variant
   const int WS = (ch.TM - 1) * p.sw + p.S + (p.sw == 2 ? 1 : 0);  // staged words, with Win<>::D
   const int WSP = (WS + 3) / 4 * 4 + (((WS + 3) / 4) % 2 == 0 ? 4 : 0);  // as Win<>::WSP
   int gw = (p.OW + ch.TM - 1) / ch.TM;
@@ -631,6 +629,14 @@ bool choose_geom(const GemmParams& p, size_t split_capacity, Choice& ch) {
   // A grid that does not fill every SM slot once splits its stages over the
   // CTAs of a cluster: then use stages small enough that every rank gets one.
   const int target = (int)std::min<int64_t>(kMaxCluster, ctas < slots() ? slots() / std::max<int64_t>(ctas, 1) : 1);
+  // Calls without a workspace split an under-filled grid over a cluster.  With a
+  // workspace (the chained forward) a grid of at least a third of the slots
+  // splits over a cluster too, a smaller one over CTAs adding int64 partial
+  // sums atomically: measured faster for the small grids (ResNet18 batch 1:
+  // 0.51 vs 0.63 ms per forward with clusters throughout), slower for the
+  // others (the atomics, the memset and the finalize cost more than the
+  // cluster barriers).
+  const bool allow_cluster = has_cluster && (split_capacity == 0 || target <= kChainClusterMaxTarget);
   if (allow_cluster && target >= 2 && (p.C + cc - 1) / cc < target) {
     int want = std::max(1, p.C / target);
     for (int d = want; d >= 1; --d)
@@ -669,7 +675,8 @@ bool choose_geom(const GemmParams& p, size_t split_capacity, Choice& ch) {
     G.splits = G.cluster;
   } else {
     const size_t need = (size_t)p.rows * p.cols * sizeof(int64_t);
-    if (split_capacity >= need && ctas < slots() && G.n_stages > 1) {
+    // a grid within an eighth of one full wave runs unsplit
+    if (split_capacity >= need && ctas * 8 < slots() * 7 && G.n_stages > 1) {
       int want = (int)std::min<int64_t>(G.n_stages, (2 * slots() + ctas - 1) / ctas);
       G.stages_per_split = (G.n_stages + want - 1) / want;
       G.splits = (G.n_stages + G.stages_per_split - 1) / G.stages_per_split;
