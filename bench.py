@@ -676,7 +676,9 @@ def resnet18_forward_record(args, dev):
         alu_tops = alu_peak(dev)[0]
         rec[f"batch{batch}"] = {"ms_per_forward": ms, "gshift_ops_per_s": terms / ms / 1e6,
                                 "frac": 2 * terms / (ms / 1e3) / (alu_tops * 1e12), "terms": terms,
-                                "kernel_launches": 1 + len(specs), "cuda_graph": graph}
+                                # the program's ops and the max|x| pre-pass; a split layer adds a finalize
+                                # launch (the ncu launch lists name every kernel of a forward)
+                                "program_ops": 1 + len(specs), "cuda_graph": graph}
         del net, xd, y
     return rec
 
