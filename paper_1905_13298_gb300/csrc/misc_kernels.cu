@@ -301,14 +301,13 @@ __global__ void absmax_kernel(const int32_t* __restrict__ x, int64_t n, uint32_t
     const int64_t nv = n >> 2;
     const int4* xv = reinterpret_cast<const int4*>(x);
     int64_t i = tid;
-    // four independent 16-byte loads in flight per thread
-    for (; i + 3 * stride < nv; i += 4 * stride) {
-      const int4 a = __ldg(xv + i), b = __ldg(xv + i + stride);
-      const int4 c = __ldg(xv + i + 2 * stride), d = __ldg(xv + i + 3 * stride);
-      m = max(m, max(max(uabs(a.x), uabs(a.y)), max(uabs(a.z), uabs(a.w))));
-      m = max(m, max(max(uabs(b.x), uabs(b.y)), max(uabs(b.z), uabs(b.w))));
-      m = max(m, max(max(uabs(c.x), uabs(c.y)), max(uabs(c.z), uabs(c.w))));
-      m = max(m, max(max(uabs(d.x), uabs(d.y)), max(uabs(d.z), uabs(d.w))));
+    // eight independent 16-byte loads in flight per thread
+    for (; i + 7 * stride < nv; i += 8 * stride) {
+      int4 v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) v[u] = __ldg(xv + i + u * stride);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) m = max(m, max(max(uabs(v[u].x), uabs(v[u].y)), max(uabs(v[u].z), uabs(v[u].w))));
     }
     for (; i < nv; i += stride) {
       const int4 a = __ldg(xv + i);
