@@ -252,6 +252,7 @@ size_t ds_packed_weight_bytes(int64_t n_out, int64_t k_red) {
 
 ds_status ds_pack_shift_weights(const int8_t* s, const int8_t* p, int64_t n_out, int64_t k_red,
                                 void* packed, size_t packed_bytes, ds_weights* desc, void* stream) {
+  NvtxRange nvtx_range("ds_pack_shift_weights");
   clear_error();
   if (!s || !p || !packed || !desc) return fail(DS_ERR_INVALID_ARG, "NULL pointer argument");
   if (n_out <= 0 || k_red <= 0) return fail(DS_ERR_SHAPE, "n_out and k_red must be positive");
@@ -318,6 +319,7 @@ size_t ds_packed_weight_bytes_backward(int K, int C, int R, int S, int stride_h,
 ds_status ds_pack_shift_weights_backward(const int8_t* s, const int8_t* p, int K, int C, int R, int S, int stride_h,
                                          int stride_w, void* packed, size_t packed_bytes, ds_weights* desc,
                                          void* stream) {
+  NvtxRange nvtx_range("ds_pack_shift_weights_backward");
   clear_error();
   if (!s || !p || !packed || !desc) return fail(DS_ERR_INVALID_ARG, "NULL pointer argument");
   if (K <= 0 || C <= 0 || R <= 0 || S <= 0) return fail(DS_ERR_SHAPE, "K, C, R and S must be positive");
@@ -359,6 +361,7 @@ size_t ds_expanded_weight_bytes(int64_t n_out, int64_t k_red) {
 }
 
 ds_status ds_expand_shift_weights(ds_weights* w, void* expanded, size_t expanded_bytes, void* stream) {
+  NvtxRange nvtx_range("ds_expand_shift_weights");
   clear_error();
   if (w == nullptr || expanded == nullptr) return fail(DS_ERR_INVALID_ARG, "NULL pointer argument");
   ds_status r = check_weights(w, w->n_out, w->k_red);
@@ -383,6 +386,7 @@ size_t ds_bf16_weight_bytes(int64_t n_out, int64_t k_red) {
 }
 
 ds_status ds_expand_shift_weights_bf16(ds_weights* w, void* buf, size_t bytes, void* stream) {
+  NvtxRange nvtx_range("ds_expand_shift_weights_bf16");
   clear_error();
   if (w == nullptr || buf == nullptr) return fail(DS_ERR_INVALID_ARG, "NULL pointer argument");
   ds_status r = check_weights(w, w->n_out, w->k_red);
@@ -402,6 +406,7 @@ ds_status ds_expand_shift_weights_bf16(ds_weights* w, void* buf, size_t bytes, v
 
 ds_status ds_linear_shift_bf16(const uint16_t* x, const ds_weights* w, const float* bias, float* y, int64_t M,
                                int64_t K, int64_t N, uint32_t flags, void* stream) {
+  NvtxRange nvtx_range("ds_linear_shift_bf16");
   clear_error();
   if (!x || !y) return fail(DS_ERR_INVALID_ARG, "NULL x or y");
   if (M <= 0 || K <= 0 || N <= 0) return fail(DS_ERR_SHAPE, "M, K and N must be positive");
@@ -424,6 +429,7 @@ void ds_bf16_set_wait_limit(long long cycles) { set_bf16_wait_cycles(cycles); }
 
 ds_status ds_linear_shift_backward_x(const int32_t* dy, const ds_weights* w_bwd, int32_t* dx, int64_t M, int64_t K,
                                      int64_t N, uint32_t flags, uint32_t* amax_io, void* stream) {
+  NvtxRange nvtx_range("ds_linear_shift_backward_x");
   clear_error();
   if (flags & ~(DS_AMAX_IN | DS_AMAX_OUT | DS_FORCE_INT64))
     return fail(DS_ERR_INVALID_ARG, "only DS_AMAX_IN, DS_AMAX_OUT and DS_FORCE_INT64 apply to a gradient");
@@ -434,6 +440,7 @@ ds_status ds_linear_shift_backward_x(const int32_t* dy, const ds_weights* w_bwd,
 ds_status ds_conv2d_shift_backward_x(const int32_t* dy, const ds_weights* w_bwd, int32_t* dx, int N, int C, int H,
                                      int W, int K, int R, int S, int stride_h, int stride_w, int pad_h, int pad_w,
                                      uint32_t flags, uint32_t* amax_io, void* stream) {
+  NvtxRange nvtx_range("ds_conv2d_shift_backward_x");
   clear_error();
   if (!dy || !dx || !w_bwd) return fail(DS_ERR_INVALID_ARG, "NULL dy, dx or weights");
   if (N <= 0 || C <= 0 || H <= 0 || W <= 0 || K <= 0 || R <= 0 || S <= 0)
@@ -522,6 +529,7 @@ ds_status ds_conv2d_shift_backward_x(const int32_t* dy, const ds_weights* w_bwd,
 }
 
 ds_status ds_quantize_shift_weights(const float* w, int64_t n, int p_min, int8_t* s, int8_t* p, void* stream) {
+  NvtxRange nvtx_range("ds_quantize_shift_weights");
   clear_error();
   if (!w || !s || !p) return fail(DS_ERR_INVALID_ARG, "NULL pointer argument");
   if (n <= 0) return fail(DS_ERR_SHAPE, "n must be positive");
@@ -532,6 +540,7 @@ ds_status ds_quantize_shift_weights(const float* w, int64_t n, int p_min, int8_t
 }
 
 ds_status ds_quantize_q16(const float* x, int64_t n, int32_t* q, void* stream) {
+  NvtxRange nvtx_range("ds_quantize_q16");
   clear_error();
   if (!x || !q) return fail(DS_ERR_INVALID_ARG, "NULL pointer argument");
   if (n <= 0) return fail(DS_ERR_SHAPE, "n must be positive");
@@ -541,6 +550,7 @@ ds_status ds_quantize_q16(const float* x, int64_t n, int32_t* q, void* stream) {
 }
 
 ds_status ds_absmax(const int32_t* x, int64_t n, uint32_t* amax, void* stream) {
+  NvtxRange nvtx_range("ds_absmax");
   clear_error();
   if (!x || !amax) return fail(DS_ERR_INVALID_ARG, "NULL pointer argument");
   if (n <= 0) return fail(DS_ERR_SHAPE, "n must be positive");
@@ -550,6 +560,7 @@ ds_status ds_absmax(const int32_t* x, int64_t n, uint32_t* amax, void* stream) {
 ds_status ds_linear_shift(const int32_t* x, const ds_weights* w, const int32_t* bias, int32_t* y,
                           int64_t M, int64_t K, int64_t N, uint32_t flags, uint32_t* amax_io,
                           void* stream) {
+  NvtxRange nvtx_range("ds_linear_shift");
   clear_error();
   if (!x || !y) return fail(DS_ERR_INVALID_ARG, "NULL x or y");
   if (M <= 0 || K <= 0 || N <= 0) return fail(DS_ERR_SHAPE, "M, K and N must be positive");
@@ -585,6 +596,7 @@ ds_status ds_conv2d_shift(const int32_t* x, const ds_weights* w, const int32_t* 
                           const int32_t* residual, int32_t* y, int N, int C, int H, int W, int K,
                           int R, int S, int stride_h, int stride_w, int pad_h, int pad_w,
                           uint32_t flags, uint32_t* amax_io, void* stream) {
+  NvtxRange nvtx_range("ds_conv2d_shift");
   clear_error();
   if (!x || !y) return fail(DS_ERR_INVALID_ARG, "NULL x or y");
   if (N <= 0 || C <= 0 || H <= 0 || W <= 0 || K <= 0 || R <= 0 || S <= 0)
@@ -644,6 +656,7 @@ extern "C" {
 
 ds_status ds_specialize_conv2d_shift(const int8_t* s, const int8_t* p, int K, int C, int R, int S, int stride,
                                      int pad, ds_specialized** out) {
+  NvtxRange nvtx_range("ds_specialize_conv2d_shift");
   clear_error();
   if (!s || !p || !out) return fail(DS_ERR_INVALID_ARG, "NULL pointer argument");
   *out = nullptr;
@@ -663,6 +676,7 @@ ds_status ds_specialize_conv2d_shift(const int8_t* s, const int8_t* p, int K, in
 ds_status ds_conv2d_shift_specialized(const ds_specialized* h, const int32_t* x, const int32_t* bias,
                                       const int32_t* residual, int32_t* y, int N, int H, int W, uint32_t flags,
                                       uint32_t* amax_io, void* stream) {
+  NvtxRange nvtx_range("ds_conv2d_shift_specialized");
   clear_error();
   if (!h) return fail(DS_ERR_INVALID_ARG, "NULL specialised layer");
   if (!x || !y) return fail(DS_ERR_INVALID_ARG, "NULL x or y");

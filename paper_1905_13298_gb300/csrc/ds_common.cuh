@@ -8,8 +8,29 @@
 #include <stdint.h>
 
 #include "deepshift.h"
+#include <nvtx3/nvToolsExt.h>  // header-only: a range costs a pointer test unless a profiler is attached
 
 namespace ds {
+
+// An NVTX range for the time of a scope: the entry points and each layer of a
+// chained forward appear by name (and layer index) on a profiler's timeline.
+struct NvtxRange {
+  explicit NvtxRange(const char* name, int index = -1) {
+    nvtxEventAttributes_t a = {};
+    a.version = NVTX_VERSION;
+    a.size = NVTX_EVENT_ATTRIB_STRUCT_SIZE;
+    a.messageType = NVTX_MESSAGE_TYPE_ASCII;
+    a.message.ascii = name;
+    if (index >= 0) {
+      a.payloadType = NVTX_PAYLOAD_TYPE_INT32;
+      a.payload.iValue = index;
+    }
+    nvtxRangePushEx(&a);
+  }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
 
 // ---------------------------------------------------------------------------
 // Error reporting (thread-local last error, see ds_last_error()).

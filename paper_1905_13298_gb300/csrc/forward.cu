@@ -199,10 +199,12 @@ static ds_status shift_forward(const ds_layer* L, int n, const int32_t* x, int32
   if (r != DS_OK) return r;
   slot_amax[0] = amax + n;
 
+  static const char* const kOpName[] = {"layer", "conv", "fc", "maxpool", "avgpool"};
   for (int i = 0; i < n; ++i) {
     const ds_layer& l = L[i];
     const int32_t* xin = slot_ptr[l.in];
     int32_t* yout = slot_ptr[l.out];
+    NvtxRange nvtx_layer(kOpName[(l.op >= DS_OP_CONV && l.op <= DS_OP_AVGPOOL) ? l.op : 0], i);
     switch (l.op) {
       case DS_OP_CONV:
         r = conv_launch(xin, l.w, l.bias, l.aux >= 0 ? slot_ptr[l.aux] : nullptr, yout, batch, l.C, l.H, l.W,
@@ -235,6 +237,7 @@ static ds_status shift_forward(const ds_layer* L, int n, const int32_t* x, int32
 
 ds_status ds_shift_forward(const ds_layer* L, int n, const int32_t* x, int32_t* y, void* ws, size_t ws_bytes,
                            int batch, void* stream) {
+  NvtxRange nvtx_range("ds_shift_forward");
   clear_error();
   try {
     return shift_forward(L, n, x, y, ws, ws_bytes, batch, stream);
