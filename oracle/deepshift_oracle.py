@@ -34,6 +34,9 @@ Readings taken where the paper is silent:
   saturated to the int32 range; NaN becomes 0.
 * Eq. 7 (with its footnote) -- the input gradient of LinearShift is
   dC/dY W_q^T, of ConvShift W_q^rot180 (*) dC/dY.
+* R-code5: the strict 5-bit storage of Sec. 4 (shifts in [-14, 0]) numbers the
+  31 states 0 (zero weight), 1 + (-p) (s = +1) and 16 + (-p) (s = -1); the
+  p of a zero weight is not stored and reads back as 0.
 * R-bwd: the backward terms use the forward's fixed-point semantics: the
   Q16.16 gradient dy is shifted (floor) and flipped, s * (dy >> -p), the sum
   is exact, then saturated to int32.
@@ -419,6 +422,92 @@ def unpack_planes6(blob, n_out: int, k_red: int):
             neg = (int(bits[g, n, 0]) >> j) & 1
             nz = (int(bits[g, n, 1]) >> j) & 1
             s[n, k] = 0 if not nz else (-1 if neg else 1)
+    return s, p
+
+
+# --------------------------------------------------------------------------
+# Strict 5-bit storage (the paper's 5-bit count, Sec. 4, for shifts in
+# [-14, 0]); layout documented in include/deepshift.h, format "codes5"
+# --------------------------------------------------------------------------
+
+FORMAT_CODES5 = 2
+P_MIN_STRICT5 = -14
+
+
+def code5(s: int, p: int) -> int:
+    """The 5-bit code of one weight (reading R-code5): 0 for s = 0, 1 + (-p) for s = +1, 16 + (-p) for s = -1.
+
+    With p in [-14, 0] a ternary sign times 15 shifts plus zero is 31 states, which fit 5 bits (Sec. 4: 4 shift
+    bits and a sign bit; the zero weight takes the code a shift of -15 would need)."""
+    s, p = int(s), int(p)
+    if s == 0 and P_MIN <= p <= P_MAX:
+        return 0
+    if s not in (-1, 1) or not (P_MIN_STRICT5 <= p <= P_MAX):
+        raise ValueError(f"(s, p) = ({s}, {p}) has no 5-bit code")
+    return (1 if s == 1 else 16) + (-p)
+
+
+def decode5(c: int):
+    """Inverse of code5: (s, p), with p = 0 for the zero weight; code 31 is never written and decodes as None."""
+    c = int(c)
+    if c == 0:
+        return 0, 0
+    if 1 <= c <= 15:
+        return 1, -(c - 1)
+    if 16 <= c <= 30:
+        return -1, -(c - 16)
+    return None
+
+
+def codes5_layout(n_out: int, k_red: int) -> dict:
+    """Byte offsets of a codes5 blob: a 256-byte header, then n_out x n_chunks records of 5 u32 bit planes."""
+    n_chunks = (k_red + 31) // 32
+    planes = BLOB_HEADER
+    end = planes + n_out * n_chunks * 20
+    return dict(n_chunks=n_chunks, planes=planes, total=(end + 255) // 256 * 256)
+
+
+def pack_codes5(s, p) -> np.ndarray:
+    """Pack [n_out, k_red] codes into the codes5 blob, one weight at a time: record (n, g) holds, in word b, bit b
+    of code5 of k = 32 g + j at bit j (zero beyond k_red).  Header: magic, format 2, n_out, k_red, n_chunks,
+    invalid_count = 0.  Storage of reading R-code5."""
+    s = np.asarray(s, dtype=np.int64)
+    p = np.asarray(p, dtype=np.int64)
+    n_out, k_red = s.shape
+    L = codes5_layout(n_out, k_red)
+    nch = L["n_chunks"]
+    rec = np.zeros((n_out, nch, 5), dtype=np.uint32)
+    for n in range(n_out):
+        for k in range(k_red):
+            c = code5(s[n, k], p[n, k])
+            g, j = divmod(k, 32)
+            for b in range(5):
+                if (c >> b) & 1:
+                    rec[n, g, b] |= np.uint32(1 << j)
+    blob = np.zeros(L["total"], dtype=np.uint8)
+    blob[0:4] = np.frombuffer(np.uint32(BLOB_MAGIC).tobytes(), np.uint8)
+    blob[4:8] = np.frombuffer(np.uint32(FORMAT_CODES5).tobytes(), np.uint8)
+    blob[8:32] = np.frombuffer(np.array([n_out, k_red, nch], dtype=np.int64).tobytes(), np.uint8)
+    blob[L["planes"]:L["planes"] + rec.nbytes] = np.frombuffer(rec.tobytes(), np.uint8)
+    return blob
+
+
+def unpack_codes5(blob, n_out: int, k_red: int):
+    """Inverse of pack_codes5: (s, p) int8 [n_out, k_red], p = 0 where s = 0.  Reading R-code5, read back."""
+    blob = np.asarray(blob, dtype=np.uint8)
+    L = codes5_layout(n_out, k_red)
+    nch = L["n_chunks"]
+    rec = np.frombuffer(blob[L["planes"]:L["planes"] + n_out * nch * 20].tobytes(), np.uint32).reshape(n_out, nch, 5)
+    s = np.zeros((n_out, k_red), dtype=np.int8)
+    p = np.zeros((n_out, k_red), dtype=np.int8)
+    for n in range(n_out):
+        for k in range(k_red):
+            g, j = divmod(k, 32)
+            c = sum(((int(rec[n, g, b]) >> j) & 1) << b for b in range(5))
+            d = decode5(c)
+            if d is None:
+                raise ValueError(f"code 31 at ({n}, {k})")
+            s[n, k], p[n, k] = d
     return s, p
 
 

@@ -9,7 +9,9 @@ nibble, a wrong column constant, a wrong term sign, a quantizer that floors
 log2|W| or rounds in the linear domain, a truncating Q16.16 conversion or one
 with ties away from zero, an input gradient without the rot180 or with the
 flip first, sampled-element and layout helpers with one slip each, an int32
-bound that drops a term, a ResNet block joined after its ReLU) and runs the
+bound that drops a term, a ResNet block joined after its ReLU, a 5-bit code
+with the signs swapped or its shift off by one, 5-bit planes in reverse
+order) and runs the
 pins of tests/test_oracle_pins.py until one fails.  A
 mistake that no pin catches fails this test.  The unmutated oracle passes every
 pin (test_oracle_pins.py itself).
@@ -17,6 +19,7 @@ pin (test_oracle_pins.py itself).
 import numpy as np
 import pytest
 
+import test_codes5_cpu as pins5
 import test_oracle_pins as pins
 from oracle import deepshift_oracle as O
 from oracle import networks as ON
@@ -27,7 +30,8 @@ _ORIG = {name: getattr(O, name) for name in ("linear_shift_acc", "conv2d_shift_a
                                               "conv2d_shift_backward_x_acc", "linear_shift_backward_x_acc",
                                               "maxpool2d", "conv2d_shift_at", "linear_shift_at",
                                               "int32_accumulation_is_exact", "expand_codes", "weights_bf16_bits",
-                                              "unpack_planes6", "backward_codes", "backward_phase_codes")}
+                                              "unpack_planes6", "backward_codes", "backward_phase_codes",
+                                              "code5", "pack_codes5")}
 
 # the pins to run, cheapest first (parametrized pins with their first case)
 _PINS = [
@@ -66,6 +70,9 @@ _PINS = [
     lambda: pins.test_conv_backward_x_stride1_is_forward_conv_with_rot180_codes(pins.BWD_GEOMS[0]),
     lambda: pins.test_conv_backward_x_phase_decomposition(pins.BWD_GEOMS[1]),
     lambda: pins.test_resnet_chain_matches_float64_library_case("resnet18", "basic", [2, 2, 2, 2]),
+    pins5.test_every_state_has_a_distinct_code_and_reads_back,
+    pins5.test_hand_written_blob,
+    pins5.test_round_trip_of_random_codes,
 ]
 
 
@@ -242,6 +249,21 @@ def _join_after_relu(x, prm, stride, pad, relu, residual=None):  # ReLU on the b
     return y
 
 
+def _code5_signs_swapped(s, p):  # +1 weights numbered from 16, -1 weights from 1
+    c = _ORIG["code5"](s, p)
+    return c if c == 0 else (c + 15 if c <= 15 else c - 15)
+
+
+def _pack5_planes_reversed(s, p):  # bit b of a code stored in plane 4 - b
+    blob = _ORIG["pack_codes5"](s, p).copy()
+    n_out, k_red = np.shape(s)
+    L = O.codes5_layout(n_out, k_red)
+    end = L["planes"] + n_out * L["n_chunks"] * 20
+    rec = blob[L["planes"]:end].view(np.uint32).reshape(-1, 5)
+    blob[L["planes"]:end] = np.ascontiguousarray(rec[:, ::-1]).view(np.uint8).reshape(-1)
+    return blob
+
+
 MUTANTS = {  # each case patches exactly one oracle function ("networks." names one in oracle/networks.py)
     "max-pool pads with zeros": {"maxpool2d": _maxpool_zero_padding},
     "ReLU before the residual join": {"add_relu": _relu_before_join},
@@ -286,6 +308,9 @@ MUTANTS = {  # each case patches exactly one oracle function ("networks." names 
     "truncating average": {"avgpool_floor": _trunc_average},
     "swapped nibbles (packing)": {"pack_planes6": _swapped_nibbles},
     "wrong column constant": {"column_constants": _wrong_column_a},
+    "5-bit codes with the signs swapped": {"code5": _code5_signs_swapped},
+    "5-bit code off by one in the shift": {"code5": lambda s, p: _ORIG["code5"](s, p) + (1 if s != 0 else 0)},
+    "5-bit planes in reverse order": {"pack_codes5": _pack5_planes_reversed},
 }
 
 
