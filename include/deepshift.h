@@ -114,7 +114,8 @@ size_t ds_abi_struct_size(int which);
  * Entries with k >= k_red are zero codes.  n_chunks = ceil(k_red / 32).
  * Storage is 6 bits per weight: 4 shift bits + sign + non-zero.  The paper's
  * 5-bit count (Sec. 4) has 32 states, one short of the 33 states of a ternary
- * sign times 16 shifts, so the non-zero plane is the sixth bit.
+ * sign times 16 shifts, so the non-zero plane is the sixth bit (layers whose
+ * shifts stay in [-14, 0] can be stored in 5 bits: DS_FORMAT_CODES5 below).
  * ------------------------------------------------------------------------- */
 #define DS_FORMAT_PLANES6 1u
 #define DS_WEIGHTS_MAGIC 0x31575344u
@@ -151,6 +152,50 @@ size_t ds_packed_weight_bytes(int64_t n_out, int64_t k_red);
  */
 ds_status ds_pack_shift_weights(const int8_t* s, const int8_t* p, int64_t n_out, int64_t k_red,
                                 void* packed, size_t packed_bytes, ds_weights* desc, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * Strict 5-bit code storage (Sec. 4: 4 shift bits and a sign bit per weight).
+ *
+ * With every shift of a nonzero weight in [-14, 0], a ternary sign times 15
+ * shifts plus the zero weight is 31 states, which fit 5 bits: code 0 is the
+ * zero weight, 1 + (-p) a weight with s = +1, 16 + (-p) one with s = -1 (31
+ * is never written).  This is a storage format for such layers: compute calls
+ * take the 6-bit blob above, made from the codes that ds_unpack_shift_weights5
+ * returns.  The p of a zero weight is not stored and reads back as 0 (no term
+ * depends on it).
+ *
+ * Blob layout (format DS_FORMAT_CODES5, little endian):
+ *   [0, 256)     header: u32 magic (0x31575344), u32 format (2), i64 n_out,
+ *                i64 k_red, i64 n_chunks = ceil(k_red / 32), u32 invalid_count
+ *   @ 256        n_out x n_chunks records of 5 u32, record (n, g) at
+ *                256 + 20 (n n_chunks + g): bit j of word b is bit b of the
+ *                code of k = 32 g + j (zero beyond k_red)
+ * 5 bits per weight, the total rounded up to 256 bytes.
+ * ------------------------------------------------------------------------- */
+#define DS_FORMAT_CODES5 2u
+
+/* Bytes of the 5-bit blob of an n_out x k_red code matrix (0 if invalid). */
+size_t ds_packed5_weight_bytes(int64_t n_out, int64_t k_red);
+
+/*
+ * Store codes (s, p: device int8 [n_out][k_red], row-major) in the 5-bit blob
+ * `packed5` (device, 256-byte aligned, at least ds_packed5_weight_bytes bytes,
+ * caller-owned).  Synchronises `stream` (an offline call) so that it can
+ * report DS_ERR_CODE_RANGE when a code has no 5-bit state (s outside
+ * {-1, 0, 1}, or p outside [-14, 0] for s != 0, or outside [-15, 0] for s = 0);
+ * the blob is then unusable.
+ */
+ds_status ds_pack_shift_weights5(const int8_t* s, const int8_t* p, int64_t n_out, int64_t k_red, void* packed5,
+                                 size_t packed5_bytes, void* stream);
+
+/*
+ * Read a 5-bit blob back into s, p (device int8 [n_out][k_red], caller-owned;
+ * p = 0 where s = 0).  Synchronises `stream`: the header is checked on the
+ * host first (DS_ERR_INVALID_ARG: not a 5-bit blob; DS_ERR_SHAPE: other
+ * dims), and DS_ERR_CODE_RANGE reports codes 31 (written as zero weights).
+ */
+ds_status ds_unpack_shift_weights5(const void* packed5, size_t packed5_bytes, int64_t n_out, int64_t k_red,
+                                   int8_t* s, int8_t* p, void* stream);
 
 /* ---------------------------------------------------------------------------
  * Expanded execution layout (optional).  The packed blob is the storage

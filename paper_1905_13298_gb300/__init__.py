@@ -42,6 +42,7 @@ DS_OP_AVGPOOL = 4
 
 DS_WEIGHTS_MAGIC = 0x31575344
 DS_FORMAT_PLANES6 = 1
+DS_FORMAT_CODES5 = 2
 
 
 class DsError(RuntimeError):
@@ -86,6 +87,11 @@ _SIGNATURES = {
                                                       ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64,
                                                       ctypes.c_int64, ctypes.c_int64, ctypes.c_uint32,
                                                       ctypes.c_void_p]),
+    "ds_packed5_weight_bytes": (ctypes.c_size_t, [ctypes.c_int64, ctypes.c_int64]),
+    "ds_pack_shift_weights5": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64,
+                                              ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]),
+    "ds_unpack_shift_weights5": (ctypes.c_int, [ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int64, ctypes.c_int64,
+                                                ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]),
     "ds_expanded_weight_bytes": (ctypes.c_size_t, [ctypes.c_int64, ctypes.c_int64]),
     "ds_expand_shift_weights": (ctypes.c_int, [ctypes.POINTER(ds_weights), ctypes.c_void_p, ctypes.c_size_t,
                                                ctypes.c_void_p]),
@@ -211,6 +217,20 @@ def ds_pack_shift_weights(s, p, n_out: int, k_red: int, packed, packed_bytes: in
     _check(lib().ds_pack_shift_weights(_ptr(s), _ptr(p), n_out, k_red, _ptr(packed), packed_bytes,
                                        ctypes.byref(desc), _stream(stream)))
     return desc
+
+
+def ds_packed5_weight_bytes(n_out: int, k_red: int) -> int:
+    return int(lib().ds_packed5_weight_bytes(n_out, k_red))
+
+
+def ds_pack_shift_weights5(s, p, n_out: int, k_red: int, packed5, packed5_bytes: int, stream=None) -> None:
+    _check(lib().ds_pack_shift_weights5(_ptr(s), _ptr(p), n_out, k_red, _ptr(packed5), packed5_bytes,
+                                        _stream(stream)))
+
+
+def ds_unpack_shift_weights5(packed5, packed5_bytes: int, n_out: int, k_red: int, s, p, stream=None) -> None:
+    _check(lib().ds_unpack_shift_weights5(_ptr(packed5), packed5_bytes, n_out, k_red, _ptr(s), _ptr(p),
+                                          _stream(stream)))
 
 
 def ds_expanded_weight_bytes(n_out: int, k_red: int) -> int:
@@ -455,6 +475,30 @@ def quantize_q16(x, out=None, stream=None):
     q = out if out is not None else torch.empty(x.shape, dtype=torch.int32, device=x.device)
     ds_quantize_q16(x, x.numel(), q, stream)
     return q
+
+
+def pack_shift_weights5(s, p, stream=None):
+    """Stores int8 codes [n_out, ...] (every shift of a nonzero weight in [-14, 0]) in a new 5-bit blob (device
+    uint8 tensor)."""
+    import torch
+    _need(s, "s", torch.int8)
+    _need(p, "p", torch.int8, tuple(s.shape))
+    _on_one_gpu(s=s, p=p)
+    n_out, k_red = s.shape[0], s[0].numel()
+    nbytes = ds_packed5_weight_bytes(n_out, k_red)
+    blob = torch.empty(nbytes, dtype=torch.uint8, device=s.device)
+    ds_pack_shift_weights5(s, p, n_out, k_red, blob, nbytes, stream)
+    return blob
+
+
+def unpack_shift_weights5(blob, n_out: int, k_red: int, stream=None):
+    """Reads a 5-bit blob back into int8 codes (s, p) of shape [n_out, k_red] (p = 0 where s = 0)."""
+    import torch
+    _need(blob, "blob", torch.uint8)
+    s = torch.empty((n_out, k_red), dtype=torch.int8, device=blob.device)
+    p = torch.empty((n_out, k_red), dtype=torch.int8, device=blob.device)
+    ds_unpack_shift_weights5(blob, blob.numel(), n_out, k_red, s, p, stream)
+    return s, p
 
 
 def pack_shift_weights(s, p, stream=None, expand: bool = False) -> PackedShiftWeights:

@@ -401,3 +401,21 @@ def test_specialisation_validates_before_compiling(ds):
     assert out.value is None
     assert L.ds_conv2d_shift_specialized(None, 16, None, None, 4096, 1, 8, 8, 0, None, None) == ds.DS_ERR_INVALID_ARG
     L.ds_specialized_destroy(None)  # a no-op
+
+
+def test_codes5_sizes_and_validation_without_gpu(ds):
+    """The 5-bit storage: its size query matches the oracle's layout, and every argument check comes before
+    any CUDA call."""
+    for n_out, k_red in [(1, 1), (1, 3), (7, 64), (33, 32), (512, 784)]:
+        assert ds.ds_packed5_weight_bytes(n_out, k_red) == O.codes5_layout(n_out, k_red)["total"]
+    assert ds.ds_packed5_weight_bytes(0, 3) == 0 and ds.ds_packed5_weight_bytes(3, 0) == 0
+    L = ds.lib()
+    v = ctypes.c_void_p
+    assert L.ds_pack_shift_weights5(None, v(16), 1, 1, v(256), 256, None) == ds.DS_ERR_INVALID_ARG
+    assert L.ds_pack_shift_weights5(v(16), v(16), 0, 1, v(256), 256, None) == ds.DS_ERR_SHAPE
+    assert L.ds_pack_shift_weights5(v(16), v(16), 1, 3, v(256), 511, None) == ds.DS_ERR_BUFFER_TOO_SMALL
+    assert L.ds_pack_shift_weights5(v(16), v(16), 1, 3, v(260), 512, None) == ds.DS_ERR_ALIGNMENT
+    assert L.ds_unpack_shift_weights5(None, 512, 1, 3, v(16), v(16), None) == ds.DS_ERR_INVALID_ARG
+    assert L.ds_unpack_shift_weights5(v(256), 512, 1, -3, v(16), v(16), None) == ds.DS_ERR_SHAPE
+    assert L.ds_unpack_shift_weights5(v(256), 100, 1, 3, v(16), v(16), None) == ds.DS_ERR_BUFFER_TOO_SMALL
+    assert L.ds_unpack_shift_weights5(v(264), 512, 1, 3, v(16), v(16), None) == ds.DS_ERR_ALIGNMENT
