@@ -19,12 +19,12 @@
 //
 // Split reduction (layers whose grid would not fill the SMs, e.g. 2048
 // input channels on 7x7 maps, or a 1x1/2 downsample at batch 32): grid.z
-// CTAs share a tile's stages.  With a workspace (the chained forward) they
-// add their exact partial sums into it with 64-bit atomics and the finalize
-// kernel of conv_direct.cu applies the epilogue; without one (a standalone
-// call) the CTAs form a thread-block cluster, and each rank reduces a share
-// of the tile's partial sums over all ranks through distributed shared
-// memory and applies the epilogue itself.
+// CTAs share a tile's stages.  Normally the CTAs form a thread-block
+// cluster, and each rank reduces a share of the tile's partial sums over all
+// ranks through distributed shared memory and applies the epilogue itself.
+// With a workspace (the chained forward) a grid below a sixteenth of the SM
+// slots instead adds its exact partial sums into the workspace with 64-bit
+// atomics, and the finalize kernel of conv_direct.cu applies the epilogue.
 #include <cooperative_groups.h>
 
 #include <algorithm>
