@@ -492,6 +492,9 @@ ds_status ds_conv2d_shift_backward_x(const int32_t* dy, const ds_weights* w_bwd,
   // output phase (rh, rw): dX rows rh, rh + sh, ...; they receive the taps r = a + sh t with
   // a = (rh + pad_h) mod sh, reading gradient row i' + c_h - t (i = sh i' + rh, c_h = (rh + pad_h - a) / sh):
   // a stride-1 correlation of dY with the phase's Th x Tw sub-kernel and padding Th - 1 - c_h
+  // the implicit-GEMM phases go out kMaxGemmPhases per launch (each alone fills few SMs)
+  GemmParams gemm_phases[kMaxGemmPhases];
+  int n_gemm = 0;
   for (int rh = 0; rh < stride_h && rh < H; ++rh)
     for (int rw = 0; rw < stride_w && rw < W; ++rw) {
       const int a = (rh + pad_h) % stride_h, b = (rw + pad_w) % stride_w;
@@ -522,9 +525,26 @@ ds_status ds_conv2d_shift_backward_x(const int32_t* dy, const ds_weights* w_bwd,
       p.yH = H;
       p.yW = W;
       fill_blob_offsets(p, &w_bwd[a * stride_w + b]);
-      r = cuda_check(launch_conv2d_shift(p, st), "conv2d_shift_backward_x (implicit GEMM) launch");
-      if (r != DS_OK) return r;
+      // few columns (the gradient of a layer with few input channels): a thread per 4 pixels and all columns;
+      // DS_CONV_IM2COL keeps the implicit GEMM (testing / comparison)
+      if (conv_narrow_supported(p) && !(flags & DS_CONV_IM2COL)) {
+        r = cuda_check(launch_conv_narrow(p, st), "conv2d_shift_backward_x (narrow) launch");
+        if (r != DS_OK) return r;
+      } else {
+        gemm_phases[n_gemm++] = p;
+        if (n_gemm == kMaxGemmPhases) {
+          r = cuda_check(launch_conv2d_shift_phases(gemm_phases, n_gemm, st),
+                         "conv2d_shift_backward_x (implicit GEMM) launch");
+          if (r != DS_OK) return r;
+          n_gemm = 0;
+        }
+      }
     }
+  if (n_gemm > 0) {
+    r = cuda_check(launch_conv2d_shift_phases(gemm_phases, n_gemm, st),
+                   "conv2d_shift_backward_x (implicit GEMM) launch");
+    if (r != DS_OK) return r;
+  }
   return DS_OK;
 }
 

@@ -127,6 +127,12 @@ struct GemmParams {
   size_t split_capacity;    // bytes available at split_acc
 };
 
+// Defined in shift_gemm.cu: up to kMaxGemmPhases implicit GEMMs (conv, no split) per launch.
+constexpr int kMaxGemmPhases = 4;
+cudaError_t launch_conv2d_shift_phases(const GemmParams* ps, int n, cudaStream_t st);
+// Defined in conv_narrow.cu: stride-1 ConvShift with at most 8 output columns and at most 4 taps per row.
+bool conv_narrow_supported(const GemmParams& p);
+cudaError_t launch_conv_narrow(const GemmParams& p, cudaStream_t st);
 // Launchers (defined in shift_gemm.cu).
 cudaError_t launch_linear_shift(const GemmParams& p, cudaStream_t st);
 // Defined in linear_cluster.cu (small batches: the reduction split over a thread-block cluster).

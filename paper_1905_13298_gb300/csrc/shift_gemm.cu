@@ -18,6 +18,8 @@
 // the previous layer).  Then no wrap-around or saturation can occur and the
 // 32-bit result is exact.  Otherwise the CTA runs the same loop with 64-bit
 // accumulators and saturates the exact sum.
+#include <algorithm>
+
 #include "ds_common.cuh"
 
 namespace ds {
@@ -358,13 +360,9 @@ __device__ __forceinline__ bool tile_int32_exact(const GemmParams& P, int64_t co
   return !__syncthreads_or(unsafe);
 }
 
+// One CTA tile (rows row0.., columns col0..) of the shift GEMM.
 template <bool CONV, bool VEC>
-__global__ void __launch_bounds__(THREADS, 3) shift_gemm_kernel(const GemmParams P) {
-  extern __shared__ __align__(16) unsigned char smem_raw[];
-  Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
-  const int64_t row0 = (int64_t)blockIdx.x * MT;
-  const int64_t col0 = (int64_t)blockIdx.y * NT;
-
+__device__ __forceinline__ void gemm_cta(const GemmParams& P, Smem& sm, int64_t row0, int64_t col0) {
   RowCtx rc{0, 0, 0, false};
   if constexpr (CONV) {
     const int64_t pixel = row0 + threadIdx.x;
@@ -394,6 +392,37 @@ __global__ void __launch_bounds__(THREADS, 3) shift_gemm_kernel(const GemmParams
 }
 
 template <bool CONV, bool VEC>
+__global__ void __launch_bounds__(THREADS, 3) shift_gemm_kernel(const GemmParams P) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  gemm_cta<CONV, VEC>(P, *reinterpret_cast<Smem*>(smem_raw), (int64_t)blockIdx.x * MT, (int64_t)blockIdx.y * NT);
+}
+
+// Several implicit GEMMs in one launch (the tap phases of a strided layer's
+// input gradient, each too small to fill the SMs alone): blockIdx.z picks the
+// phase; a CTA beyond its phase's tiles returns at once.  The phases are
+// selected by constant indices, so each reads its parameters at fixed offsets.
+struct PhaseSet {
+  GemmParams p[kMaxGemmPhases];
+};
+
+__device__ __forceinline__ void phase_cta(const GemmParams& P, Smem& sm) {
+  const int64_t row0 = (int64_t)blockIdx.x * MT, col0 = (int64_t)blockIdx.y * NT;
+  if (row0 >= P.rows || col0 >= P.cols) return;
+  gemm_cta<true, false>(P, sm, row0, col0);
+}
+
+__global__ void __launch_bounds__(THREADS, 3) shift_gemm_phases_kernel(const PhaseSet S) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
+  switch (blockIdx.z) {
+    case 0: phase_cta(S.p[0], sm); break;
+    case 1: phase_cta(S.p[1], sm); break;
+    case 2: phase_cta(S.p[2], sm); break;
+    default: phase_cta(S.p[3], sm); break;
+  }
+}
+
+template <bool CONV, bool VEC>
 cudaError_t launch_impl(const GemmParams& p, cudaStream_t st) {
   const size_t smem = sizeof(Smem);
   // once per process, thread-safe (see conv_direct.cu)
@@ -414,6 +443,32 @@ cudaError_t launch_linear_shift(const GemmParams& p, cudaStream_t st) {
 
 cudaError_t launch_conv2d_shift(const GemmParams& p, cudaStream_t st) {
   return launch_impl<true, false>(p, st);
+}
+
+cudaError_t launch_conv2d_shift_phases(const GemmParams* ps, int n, cudaStream_t st) {
+  static const cudaError_t attr = cudaFuncSetAttribute(shift_gemm_phases_kernel,
+                                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                       (int)sizeof(Smem));
+  if (attr != cudaSuccess) return attr;
+  for (int i0 = 0; i0 < n; i0 += kMaxGemmPhases) {
+    const int m = std::min(kMaxGemmPhases, n - i0);
+    if (m == 1) {
+      cudaError_t e = launch_conv2d_shift(ps[i0], st);
+      if (e != cudaSuccess) return e;
+      continue;
+    }
+    PhaseSet S{};
+    int64_t rt = 0, ct = 0;
+    for (int j = 0; j < m; ++j) {
+      S.p[j] = ps[i0 + j];
+      rt = std::max<int64_t>(rt, (ps[i0 + j].rows + MT - 1) / MT);
+      ct = std::max<int64_t>(ct, (ps[i0 + j].cols + NT - 1) / NT);
+    }
+    shift_gemm_phases_kernel<<<dim3((unsigned)rt, (unsigned)ct, (unsigned)m), THREADS, sizeof(Smem), st>>>(S);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 }  // namespace ds

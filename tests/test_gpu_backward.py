@@ -149,9 +149,10 @@ def test_conv_backward_x_degenerate_codes(dslib, geom, flags):
 
 
 @pytest.mark.parametrize("geom", [(2, 64, 56, 56, 64, 3, 3, 1, 1), (2, 64, 56, 56, 128, 1, 1, 2, 0),
-                                  (2, 64, 56, 56, 128, 3, 3, 2, 1)])
+                                  (2, 64, 56, 56, 128, 3, 3, 2, 1), (2, 3, 224, 224, 64, 7, 7, 2, 3)])
 def test_conv_backward_x_resnet_layers(dslib, geom):
-    """ResNet18 layer shapes (conv2_x, the 1x1/2 and 3x3/2 transitions), 2 images, every output."""
+    """ResNet18 layer shapes (conv2_x, the 1x1/2 and 3x3/2 transitions, the 7x7/2 stem whose 3-column gradient
+    runs the narrow kernel), 2 images, every output."""
     N, C, H, W, K, R, S, st, pd = geom
     s = si.sign_codes(sum(geom), (K, C, R, S))
     p = si.shift_codes_geometric(sum(geom), (K, C, R, S), -6)
