@@ -124,10 +124,12 @@ def test_linear_stays_inside_its_buffers(dslib, shape, expand):
     assert np.array_equal(yg.numpy(want.shape), want)
 
 
-def test_conv_input_gradient_stays_inside_its_buffers(dslib):
-    """Stride 2: one implicit GEMM per tap phase, each with its own descriptor into one guarded blob."""
+@pytest.mark.parametrize("geom", [(2, 6, 11, 12, 8, 3, 2, 1), (2, 20, 11, 12, 8, 3, 2, 1), (1, 3, 23, 21, 16, 7, 2, 3)])
+def test_conv_input_gradient_stays_inside_its_buffers(dslib, geom):
+    """Stride 2: the tap phases with their own descriptors into one guarded blob; 6 and 3 gradient columns run
+    the narrow kernel, 20 the implicit GEMMs of all phases in one launch."""
     ds = dslib
-    N, C, H, W, K, R, st, pd = 2, 6, 11, 12, 8, 3, 2, 1
+    N, C, H, W, K, R, st, pd = geom
     _, s, p, _ = si.conv_layer(77, N, C, H, W, K, R, R)
     OH, OW = (H + 2 * pd - R) // st + 1, (W + 2 * pd - R) // st + 1
     dy = si.activations(78, (N, K, OH, OW), -(1 << 20), 1 << 20)
