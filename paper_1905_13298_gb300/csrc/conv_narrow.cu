@@ -29,23 +29,33 @@ constexpr int kCodeWords = 8192;  // shared-memory words for staged codes (32 KB
 template <int NC>
 __device__ __forceinline__ void stage_codes(const GemmParams& P, int32_t* cs, int64_t k0, int nk) {
   // cs[k][0..NC) = -p, cs[k][NC..2NC) = s of the columns (zero beyond cols)
+  if (P.xcodes != nullptr) {
+    // the expanded layout's row of k holds the NC columns' shifts and signs contiguously (zero beyond
+    // n_out): 16-byte loads, several in flight per thread
+#pragma unroll 4
+    for (int kk = threadIdx.x; kk < nk; kk += THREADS) {
+      const int4* src = reinterpret_cast<const int4*>(P.xcodes + (k0 + kk) * 64);
+      int4* dst = reinterpret_cast<int4*>(cs + kk * 2 * NC);
+#pragma unroll
+      for (int v = 0; v < NC / 4; ++v) {
+        dst[v] = __ldg(src + v);
+        dst[NC / 4 + v] = __ldg(src + 8 + v);
+      }
+    }
+    return;
+  }
   for (int i = threadIdx.x; i < nk * NC; i += THREADS) {
     const int kk = i / NC, col = i - kk * NC;
     const int64_t k = k0 + kk;
     int sh = 0, sg = 0;
     if (col < P.cols) {
-      if (P.xcodes != nullptr) {
-        sh = __ldg(P.xcodes + k * 64 + col);
-        sg = __ldg(P.xcodes + k * 64 + 32 + col);
-      } else {
-        const int64_t g = k >> 5;
-        const int j = (int)(k & 31);
-        const uint32_t nib =
-            __ldg(reinterpret_cast<const uint32_t*>(P.blob + P.off_nib) + (g * P.cols + col) * 4 + (j >> 3));
-        const uint2 bits = __ldg(reinterpret_cast<const uint2*>(P.blob + P.off_bits) + g * P.cols + col);
-        sh = (int)((nib >> (4 * (j & 7))) & 15u);
-        sg = ((bits.y >> j) & 1u) ? (((bits.x >> j) & 1u) ? -1 : 1) : 0;
-      }
+      const int64_t g = k >> 5;
+      const int j = (int)(k & 31);
+      const uint32_t nib =
+          __ldg(reinterpret_cast<const uint32_t*>(P.blob + P.off_nib) + (g * P.cols + col) * 4 + (j >> 3));
+      const uint2 bits = __ldg(reinterpret_cast<const uint2*>(P.blob + P.off_bits) + g * P.cols + col);
+      sh = (int)((nib >> (4 * (j & 7))) & 15u);
+      sg = ((bits.y >> j) & 1u) ? (((bits.x >> j) & 1u) ? -1 : 1) : 0;
     }
     cs[kk * 2 * NC + col] = sh;
     cs[kk * 2 * NC + NC + col] = sg;
@@ -71,6 +81,38 @@ __device__ __forceinline__ bool narrow_int32_exact(const GemmParams& P) {
       unsafe = (((lo + 32767ull) >> 15) + nnz + b) > (unsigned long long)INT32_MAX;
   }
   return !__syncthreads_or(unsafe);
+}
+
+// The TP + S - 1 input values of one row segment (zero outside the image).
+template <int S>
+__device__ __forceinline__ void load_row(const GemmParams& P, const int32_t* xc, int ih, int iw0, int* w) {
+  const bool row_ok = (unsigned)ih < (unsigned)P.H;
+  const int32_t* xr = xc + (int64_t)(row_ok ? ih : 0) * P.W;
+#pragma unroll
+  for (int i = 0; i < TP + S - 1; ++i) {
+    const int iw = iw0 + i;
+    w[i] = (row_ok && (unsigned)iw < (unsigned)P.W) ? __ldg(xr + iw) : 0;
+  }
+}
+
+// The S taps of one (c, r) row: codes ck[s][0..NC) = -p, ck[s][NC..2NC) = s.
+template <int NC, int S, typename Acc>
+__device__ __forceinline__ void row_terms(const int32_t* ck, const int* w, Acc (&acc)[TP][NC]) {
+#pragma unroll
+  for (int s = 0; s < S; ++s) {
+    int sh[NC], sg[NC];
+#pragma unroll
+    for (int v = 0; v < NC / 4; ++v) {
+      const int4 a = reinterpret_cast<const int4*>(ck + s * 2 * NC)[v];
+      const int4 b = reinterpret_cast<const int4*>(ck + s * 2 * NC + NC)[v];
+      sh[4 * v] = a.x, sh[4 * v + 1] = a.y, sh[4 * v + 2] = a.z, sh[4 * v + 3] = a.w;
+      sg[4 * v] = b.x, sg[4 * v + 1] = b.y, sg[4 * v + 2] = b.z, sg[4 * v + 3] = b.w;
+    }
+#pragma unroll
+    for (int j = 0; j < NC; ++j)
+#pragma unroll
+      for (int t = 0; t < TP; ++t) acc[t][j] += (Acc)sg[j] * (Acc)(w[t + s] >> sh[j]);
+  }
 }
 
 template <int NC, int S, typename Acc>
@@ -99,34 +141,22 @@ __device__ __forceinline__ void run_narrow(const GemmParams& P, int32_t* cs, int
     __syncthreads();  // the previous run's codes are no longer read
     stage_codes<NC>(P, cs, (int64_t)c0 * P.R * S, nc * P.R * S);
     __syncthreads();
+    const int32_t* xc0 = P.x + (n * P.C + c0) * HW;
     if (!active) continue;
-    for (int cc = 0; cc < nc; ++cc) {
-      const int32_t* xc = P.x + (n * P.C + c0 + cc) * HW;
-      for (int r = 0; r < P.R; ++r) {
-        const int ih = oh + r - P.ph;
-        int w[TP + S - 1];
-        const bool row_ok = (unsigned)ih < (unsigned)P.H;
-#pragma unroll
-        for (int i = 0; i < TP + S - 1; ++i) {
-          const int iw = iw0 + i;
-          w[i] = (row_ok && (unsigned)iw < (unsigned)P.W) ? __ldg(xc + (int64_t)ih * P.W + iw) : 0;
+    // the (c, r) rows of the run in order, the next row's input values loaded while the current row's terms run
+    const int rows = nc * P.R;
+    int w0[TP + S - 1], w1[TP + S - 1];
+    load_row<S>(P, xc0 + 0, oh - P.ph, iw0, w0);
+    for (int it = 0; it < rows; it += 2) {
+      const int c1 = (it + 1) / P.R, r1 = it + 1 - c1 * P.R;
+      if (it + 1 < rows) load_row<S>(P, xc0 + c1 * HW, oh + r1 - P.ph, iw0, w1);
+      row_terms<NC, S>(cs + it * S * 2 * NC, w0, acc);
+      if (it + 1 < rows) {
+        if (it + 2 < rows) {
+          const int c2 = (it + 2) / P.R, r2 = it + 2 - c2 * P.R;
+          load_row<S>(P, xc0 + c2 * HW, oh + r2 - P.ph, iw0, w0);
         }
-        const int32_t* ck = cs + ((cc * P.R + r) * S) * 2 * NC;
-#pragma unroll
-        for (int s = 0; s < S; ++s) {
-          int sh[NC], sg[NC];
-#pragma unroll
-          for (int v = 0; v < NC / 4; ++v) {
-            const int4 a = reinterpret_cast<const int4*>(ck + s * 2 * NC)[v];
-            const int4 b = reinterpret_cast<const int4*>(ck + s * 2 * NC + NC)[v];
-            sh[4 * v] = a.x, sh[4 * v + 1] = a.y, sh[4 * v + 2] = a.z, sh[4 * v + 3] = a.w;
-            sg[4 * v] = b.x, sg[4 * v + 1] = b.y, sg[4 * v + 2] = b.z, sg[4 * v + 3] = b.w;
-          }
-#pragma unroll
-          for (int j = 0; j < NC; ++j)
-#pragma unroll
-            for (int t = 0; t < TP; ++t) acc[t][j] += (Acc)sg[j] * (Acc)(w[t + s] >> sh[j]);
-        }
+        row_terms<NC, S>(cs + (it + 1) * S * 2 * NC, w1, acc);
       }
     }
   }
