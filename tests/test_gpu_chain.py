@@ -199,3 +199,29 @@ def test_full_size_chain_first_and_last_image(dslib, arch, batch):
         digests, want = stored[(arch, batch, image)]
         assert _digests(x[image:image + 1], params) == digests, "stale fixture: regenerate the stored logits"
         assert np.array_equal(y[image], want), image
+
+
+def test_forward_replays_from_a_cuda_graph(dslib):
+    """The chained forward captured in a CUDA graph (after one eager call) and replayed on new inputs copied into
+    the captured input buffer: every replay equals the oracle, as the eager call does."""
+    from paper_1905_13298_gb300 import networks as PN
+    from oracle import networks as ON
+    prog = PN.resnet_program("resnet18", 64, 64)
+    params = si.network_params(prog[1], 102)
+    net = PN.ShiftNetwork(prog[0], params, batch=2)
+    xs = [si.image_batch(20 + i, 2, 3, 64, 64) for i in range(3)]
+    xd = torch.from_numpy(xs[0]).cuda()
+    y = torch.empty(net.out_shape, dtype=torch.int32, device="cuda")
+    stream = torch.cuda.Stream()
+    with torch.cuda.stream(stream):
+        net.forward(xd, y, stream.cuda_stream)  # eager first: one-time attribute and occupancy queries
+        stream.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream, capture_error_mode="relaxed"):
+            net.forward(xd, y, stream.cuda_stream)
+    torch.cuda.synchronize()
+    for x in xs:
+        xd.copy_(torch.from_numpy(x))
+        g.replay()
+        torch.cuda.synchronize()
+        assert np.array_equal(y.cpu().numpy().reshape(2, -1), ON.resnet_forward(x, params, "resnet18"))
