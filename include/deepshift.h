@@ -353,7 +353,10 @@ ds_status ds_linear_shift_static_scratch(const int32_t* x, const ds_weights* w, 
  * ignored; DS_OP_AVGPOOL: floor(sum / (R*S)), no padding).  Each shift layer
  * proves its accumulator width on the device from the max|x| that its
  * producer wrote (the network input gets one pre-pass), so the whole forward
- * runs without a host round trip and can be captured in a CUDA graph.
+ * runs without a host round trip and can be captured in a CUDA graph.  Make one
+ * eager call with the same program and batch first: the first launch of each
+ * kernel shape sets kernel attributes and queries cluster occupancy, host calls
+ * that a capture in the default (global) mode may refuse.
  * ------------------------------------------------------------------------- */
 #define DS_OP_CONV 1
 #define DS_OP_FC 2
