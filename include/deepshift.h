@@ -343,7 +343,7 @@ ds_status ds_linear_shift_static_scratch(const int32_t* x, const ds_weights* w, 
 /* ---------------------------------------------------------------------------
  * Chained forward (ResNet / VGG shaped networks of shift layers).
  *
- * A network is an array of ds_layer run in order on one stream.  Tensors
+ * A network is an array of ds_layer run in program order.  Tensors
  * live in numbered slots: slot 0 is the network input x, slot 1 the network
  * output y, slots >= 2 are carved from the caller's workspace.  Activations
  * are NCHW int32 Q16.16; an FC layer reads its input slot as [batch][C*H*W].
@@ -395,6 +395,14 @@ size_t ds_shift_forward_workspace_bytes(const ds_layer* layers, int n, int batch
  * launch, and a failed host allocation returns DS_ERR_UNSUPPORTED ("host
  * memory allocation failed") with nothing launched.  No C++ exception leaves
  * any entry point.
+ * A layer that depends on neither its predecessor's output nor a slot that
+ * its predecessor reads or writes (a ResNet block's shortcut beside the main
+ * branch) runs on a side stream of the calling thread, ordered by events on
+ * the slots it reads and writes; the caller's stream waits for the side
+ * stream before the call returns, so `stream` orders everything as before.
+ * The side stream and its events are created on a thread's first call (one
+ * set per host thread, kept until the thread ends); if they cannot be
+ * created, every layer runs on `stream`.
  */
 ds_status ds_shift_forward(const ds_layer* layers, int n, const int32_t* x, int32_t* y, void* ws,
                            size_t ws_bytes, int batch, void* stream);

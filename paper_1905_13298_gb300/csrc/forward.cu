@@ -26,6 +26,13 @@ struct Shape {
 
 struct Plan {
   std::vector<Shape> out_shape;   // per layer
+  // two-stream schedule: a layer that does not depend on its predecessor runs on a side stream
+  // (a ResNet block's shortcut beside its main branch); deps are the earlier layers (-1: the
+  // workspace reset and the input pre-pass) whose results or inputs it must wait for
+  std::vector<char> side;
+  std::vector<std::vector<int>> deps;
+  std::vector<char> signals;      // another stream waits for this layer (index n: the reset)
+  bool any_side = false;
   std::vector<int64_t> slot_elems;  // per slot, per image (slots >= 2)
   std::vector<size_t> slot_off;   // byte offsets in the workspace
   size_t amax_bytes = 0;
@@ -39,6 +46,91 @@ ds_status layer_fail(ds_status st, int i) {
   char what[512];
   snprintf(what, sizeof(what), "%s", ds_last_error());
   return fail(st, "layer %d: %s", i, what);
+}
+
+// Dependencies through the slots: a layer waits for the last writer of each
+// slot it reads (in, aux) and, before it overwrites its output slot, for that
+// slot's last writer and every reader since.  A layer that does not depend on
+// its predecessor (and whose predecessor runs on the main stream) runs on the
+// side stream.
+void schedule(const ds_layer* L, int n, Plan& P) {
+  std::vector<int> last_writer(P.n_slots, -1);
+  std::vector<std::vector<int>> readers(P.n_slots);
+  P.side.assign(n, 0);
+  P.deps.assign(n, {});
+  P.signals.assign(n + 1, 0);
+  for (int i = 0; i < n; ++i) {
+    const ds_layer& l = L[i];
+    std::vector<int>& d = P.deps[i];
+    auto add = [&d](int j) {
+      if (std::find(d.begin(), d.end(), j) == d.end()) d.push_back(j);
+    };
+    add(last_writer[l.in]);
+    if (l.aux >= 0) add(last_writer[l.aux]);
+    add(last_writer[l.out]);
+    for (int j : readers[l.out]) add(j);
+    P.side[i] = i >= 1 && !P.side[i - 1] && std::find(d.begin(), d.end(), i - 1) == d.end();
+    readers[l.in].push_back(i);
+    if (l.aux >= 0) readers[l.aux].push_back(i);
+    last_writer[l.out] = i;
+    readers[l.out].clear();
+  }
+  for (int i = 0; i < n; ++i) {
+    if (P.side[i]) P.any_side = true;
+    for (int j : P.deps[i]) {
+      const bool j_side = j >= 0 && P.side[j];
+      if (j_side != (bool)P.side[i]) P.signals[j >= 0 ? j : n] = 1;
+    }
+    // a side layer whose dependencies all run on the side stream still waits for the reset of the workspace
+    if (P.side[i] && std::none_of(P.deps[i].begin(), P.deps[i].end(), [&](int j) { return j < 0 || !P.side[j]; })) {
+      P.deps[i].push_back(-1);
+      P.signals[n] = 1;
+    }
+  }
+  // the caller's stream waits for the last side layer before the call returns
+  for (int i = n - 1; i >= 0; --i)
+    if (P.side[i]) {
+      P.signals[i] = 1;
+      break;
+    }
+}
+
+// The side stream and the events of the two-stream schedule, one set per
+// host thread (created on first use, kept for the thread's lifetime).
+struct SideStream {
+  int dev = -1;
+  cudaStream_t s = nullptr;
+  std::vector<cudaEvent_t> ev;
+};
+thread_local SideStream t_side;
+
+// False when a resource cannot be created: the forward then runs on the caller's stream alone.
+bool side_resources(size_t n_events, SideStream*& out) {
+  SideStream& S = t_side;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return false;
+  }
+  if (S.dev != dev) {  // a new device for this thread: fresh objects (the old ones belong to the other device)
+    S = SideStream{};
+    if (cudaStreamCreateWithFlags(&S.s, cudaStreamNonBlocking) != cudaSuccess) {
+      (void)cudaGetLastError();
+      S = SideStream{};
+      return false;
+    }
+    S.dev = dev;
+  }
+  while (S.ev.size() < n_events) {
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) {
+      (void)cudaGetLastError();
+      return false;
+    }
+    S.ev.push_back(e);
+  }
+  out = &S;
+  return true;
 }
 
 ds_status plan_program(const ds_layer* L, int n, int batch, Plan& P) {
@@ -129,10 +221,12 @@ ds_status plan_program(const ds_layer* L, int n, int batch, Plan& P) {
     if (l.out >= 2) P.slot_elems[l.out] = std::max(P.slot_elems[l.out], out.elems());
   }
   if (!wrote_y) return fail(DS_ERR_INVALID_ARG, "no layer writes the output slot 1");
+  schedule(L, n, P);
   P.amax_bytes = ((size_t)(n + 1) * sizeof(uint32_t) + 255) / 256 * 256;
   P.split_bytes = (P.split_bytes + 255) / 256 * 256;
   P.slot_off.assign(P.n_slots, 0);
-  size_t off = P.amax_bytes + P.split_bytes;
+  // the side stream's layers split their reductions in a scratch region of their own
+  size_t off = P.amax_bytes + (P.any_side ? 2 : 1) * P.split_bytes;
   for (int s = 2; s < P.n_slots; ++s) {
     P.slot_off[s] = off;
     int64_t bytes = 0;
@@ -192,12 +286,25 @@ static ds_status shift_forward(const ds_layer* L, int n, const int32_t* x, int32
   // one reset per forward: the max|x| words and the split-reduction scratch (its
   // zero prefix is kept zero by the finalize kernels, larger regions are zeroed
   // before their layer)
-  r = cuda_check(cudaMemsetAsync(amax, 0, P.amax_bytes + P.split_bytes, st), "workspace reset");
+  const size_t split_regions = P.any_side ? 2 : 1;
+  r = cuda_check(cudaMemsetAsync(amax, 0, P.amax_bytes + split_regions * P.split_bytes, st), "workspace reset");
   if (r != DS_OK) return r;
   const Shape in0{L[0].C, L[0].H, L[0].W};
   r = cuda_check(launch_absmax(x, in0.elems() * batch, amax + n, st), "input max|x| pre-pass");
   if (r != DS_OK) return r;
   slot_amax[0] = amax + n;
+
+  // two-stream schedule (one stream when the program has no independent neighbours, or when the
+  // side stream's objects cannot be created)
+  SideStream* S = nullptr;
+  const bool two = P.any_side && side_resources((size_t)n + 1, S);
+  auto on_side = [&](int i) { return two && i >= 0 && P.side[i]; };
+  auto stream_of = [&](int i) { return on_side(i) ? S->s : st; };
+  auto event_of = [&](int i) { return S->ev[i >= 0 ? i : n]; };
+  if (two && P.signals[n]) {
+    r = cuda_check(cudaEventRecord(event_of(-1), st), "workspace reset event");
+    if (r != DS_OK) return r;
+  }
 
   static const char* const kOpName[] = {"layer", "conv", "fc", "maxpool", "avgpool"};
   for (int i = 0; i < n; ++i) {
@@ -205,33 +312,52 @@ static ds_status shift_forward(const ds_layer* L, int n, const int32_t* x, int32
     const int32_t* xin = slot_ptr[l.in];
     int32_t* yout = slot_ptr[l.out];
     NvtxRange nvtx_layer(kOpName[(l.op >= DS_OP_CONV && l.op <= DS_OP_AVGPOOL) ? l.op : 0], i);
+    const cudaStream_t ls = stream_of(i);
+    if (two)
+      for (int j : P.deps[i])
+        if (on_side(j) != on_side(i)) {
+          r = cuda_check(cudaStreamWaitEvent(ls, event_of(j), 0), "layer dependency");
+          if (r != DS_OK) return r;
+        }
+    unsigned char* split = base + P.amax_bytes + (on_side(i) ? P.split_bytes : 0);
     switch (l.op) {
       case DS_OP_CONV:
         r = conv_launch(xin, l.w, l.bias, l.aux >= 0 ? slot_ptr[l.aux] : nullptr, yout, batch, l.C, l.H, l.W,
-                        l.K, l.R, l.S, l.stride, l.pad, l.flags, slot_amax[l.in], amax + i, st,
-                        P.split_bytes ? reinterpret_cast<int64_t*>(base + P.amax_bytes) : nullptr, P.split_bytes);
+                        l.K, l.R, l.S, l.stride, l.pad, l.flags, slot_amax[l.in], amax + i, ls,
+                        P.split_bytes ? reinterpret_cast<int64_t*>(split) : nullptr, P.split_bytes);
         slot_amax[l.out] = amax + i;
         break;
       case DS_OP_FC:
         r = fc_launch(xin, l.w, l.bias, yout, batch, (int64_t)l.C * l.H * l.W, l.K, l.flags & DS_RELU,
-                      slot_amax[l.in], amax + i, st);
+                      slot_amax[l.in], amax + i, ls);
         slot_amax[l.out] = amax + i;
         break;
       case DS_OP_MAXPOOL:
         r = cuda_check(launch_maxpool(xin, yout, (int64_t)batch * l.C, l.H, l.W, P.out_shape[i].H,
-                                      P.out_shape[i].W, l.R, l.S, l.stride, l.pad, st),
+                                      P.out_shape[i].W, l.R, l.S, l.stride, l.pad, ls),
                        "maxpool launch");
         slot_amax[l.out] = slot_amax[l.in];
         break;
       default:
         r = cuda_check(launch_avgpool_floor(xin, yout, (int64_t)batch * l.C, l.H, l.W, P.out_shape[i].H,
-                                            P.out_shape[i].W, l.R, l.S, l.stride, st),
+                                            P.out_shape[i].W, l.R, l.S, l.stride, ls),
                        "avgpool launch");
         slot_amax[l.out] = slot_amax[l.in];
         break;
     }
     if (r != DS_OK) return r;
+    if (two && P.signals[i]) {
+      r = cuda_check(cudaEventRecord(event_of(i), ls), "layer event");
+      if (r != DS_OK) return r;
+    }
   }
+  if (two)
+    for (int i = n - 1; i >= 0; --i)
+      if (P.side[i]) {  // the caller's stream resumes after the side stream's last layer
+        r = cuda_check(cudaStreamWaitEvent(st, event_of(i), 0), "side stream join");
+        if (r != DS_OK) return r;
+        break;
+      }
   return DS_OK;
 }
 

@@ -114,8 +114,10 @@ def resnet_program(arch: str = "resnet18", H: int = 224, W: int = 224):
                 pds = b.reserve_param((out_c, b.shape[x][0], 1, 1)) if need_ds else None
                 t1 = b.conv(x, planes, 1, 1, 0, param=p1)
                 t2 = b.conv(t1, planes, 3, stride, 1, param=p2)
-                b.release(t1)
+                # the shortcut before t1's slot is freed: it then writes no slot the main branch still
+                # reads, so the executor can run it beside the main branch
                 sc = b.conv(x, out_c, 1, stride, 0, relu=False, param=pds) if need_ds else x
+                b.release(t1)
                 o = b.conv(t2, out_c, 1, 1, 0, residual=sc, param=p3)
                 b.release(t2)
             if need_ds:
