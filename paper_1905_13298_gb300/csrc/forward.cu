@@ -101,6 +101,19 @@ struct SideStream {
   int dev = -1;
   cudaStream_t s = nullptr;
   std::vector<cudaEvent_t> ev;
+  SideStream() = default;
+  SideStream(const SideStream&) = delete;
+  SideStream& operator=(const SideStream&) = delete;
+  ~SideStream() { release(); }
+  // at thread exit (errors ignored: at process exit the runtime may already be gone)
+  void release() {
+    for (cudaEvent_t e : ev) (void)cudaEventDestroy(e);
+    if (s != nullptr) (void)cudaStreamDestroy(s);
+    ev.clear();
+    s = nullptr;
+    dev = -1;
+    (void)cudaGetLastError();
+  }
 };
 thread_local SideStream t_side;
 
@@ -112,11 +125,11 @@ bool side_resources(size_t n_events, SideStream*& out) {
     (void)cudaGetLastError();
     return false;
   }
-  if (S.dev != dev) {  // a new device for this thread: fresh objects (the old ones belong to the other device)
-    S = SideStream{};
+  if (S.dev != dev) {  // a new device for this thread: fresh objects
+    S.release();
     if (cudaStreamCreateWithFlags(&S.s, cudaStreamNonBlocking) != cudaSuccess) {
       (void)cudaGetLastError();
-      S = SideStream{};
+      S.s = nullptr;
       return false;
     }
     S.dev = dev;

@@ -46,3 +46,36 @@ def test_two_host_threads(dslib):
     for seed, (y, want, yc, wantc) in out.items():
         assert np.array_equal(y, want), seed
         assert np.array_equal(yc, wantc), seed
+
+
+def _forward_work(seed, out, errors):
+    try:
+        from paper_1905_13298_gb300 import networks as PN
+        prog = PN.resnet_program("resnet18", 64, 64)
+        params = si.network_params(prog[1], 103)
+        x = si.image_batch(seed, 2, 3, 64, 64)
+        stream = torch.cuda.Stream()
+        with torch.cuda.stream(stream):
+            net = PN.ShiftNetwork(prog[0], params, batch=2)
+            xd = torch.from_numpy(x).cuda()
+            for _ in range(3):  # each thread's shortcut layers run on that thread's own side stream
+                y = net.forward(xd, stream=stream.cuda_stream)
+        stream.synchronize()
+        out[seed] = (y.cpu().numpy().reshape(2, -1), x, params)
+    except Exception as e:  # reported by the main thread
+        errors.append(e)
+
+
+def test_chained_forwards_on_four_host_threads(dslib):
+    """Four threads run the ResNet18 forward at once, each on its own stream (and its own side stream for the
+    shortcut layers): every result equals the oracle."""
+    from oracle import networks as ON
+    out, errors = {}, []
+    threads = [threading.Thread(target=_forward_work, args=(seed, out, errors)) for seed in (31, 32, 33, 34)]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    assert not errors, errors
+    for seed, (y, x, params) in out.items():
+        assert np.array_equal(y, ON.resnet_forward(x, params, "resnet18")), seed
