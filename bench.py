@@ -32,6 +32,7 @@ ALG_INT_OPS_PER_TERM = 2      # one shift + one add/subtract per term (Fig. 1a: 
 # DRAM bytes (read + write) of one conv_direct_kernel<1,3,7,0> launch on this workload, from one ncu capture
 # of the current kernel (dram__bytes_read.sum + dram__bytes_write.sum); y stays in L2 at kernel end.
 NCU_TRAFFIC_BYTES = 26.08e6
+HBM_NOMINAL_GBS = 7900.0  # GB300 HBM3e, nominal
 E2E_CHUNKS = 4  # chunks of the batch in the end-to-end measurement
 
 
@@ -867,7 +868,9 @@ def run_gpu(args, wl, rank, world, local_rank):
                                        f"(sm_max_mhz, {peak_kind})",
                          "alg_int_ops_per_launch": ALG_INT_OPS_PER_TERM * wl["terms"],
                          "hbm_gbs": alg_bytes / (kern_ms / 1e3) / 1e9,
-                         "hbm_frac": alg_bytes / (kern_ms / 1e3) / 1e9 / float(peaks.get("hbm_gbs", 6800.0))},
+                         "hbm_frac": alg_bytes / (kern_ms / 1e3) / 1e9 / float(peaks.get("hbm_gbs", 6800.0)),
+                         # against the nominal 7.9 TB/s of HBM3e as well as the measured copy bandwidth
+                         "hbm_frac_nominal": alg_bytes / (kern_ms / 1e3) / 1e9 / HBM_NOMINAL_GBS},
             "e2e": {"value": wl["terms"] * args.steps * world / (e2e_ms / 1e3) / 1e9, "unit": METRIC,
                     "h2d_bytes_per_step": int(x.nbytes), "d2h_bytes_per_step": int(x.nbytes // C * K),
                     "pipeline": f"{nch} chunks of {nb} images, one stream each", "parity_spot_check": e2e_parity},
