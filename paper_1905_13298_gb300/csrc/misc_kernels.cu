@@ -131,23 +131,26 @@ __global__ void pack_kernel_vec4(const int8_t* __restrict__ s, const int8_t* __r
     auto step = [&](int64_t b, uint32_t sw, uint32_t pw) {
       const int64_t k0 = b * 128 + 4 * lane;
       const bool in = k0 < k_red;  // k_red % 4 == 0: all 4 codes or none
-      uint32_t nb = 0u, zb = 0u, nib = 0u, a_sum = 0u;  // a lane adds at most 2^15 per code
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const int sv = (int)(int8_t)(sw >> (8 * i));
-        const int pv = (int)(int8_t)(pw >> (8 * i));
-        const bool bad = in && ((unsigned)(sv + 1) > 2u || (unsigned)(pv + 15) > 15u);
-        const bool ok = in && !bad;
-        invalid += bad ? 1u : 0u;
-        if (ok) {
-          nib |= (uint32_t)(-pv) << (4 * i);
-          if (sv != 0) {
-            zb |= 1u << i;
-            a_sum += 1u << (15 + pv);
-          }
-          if (sv == -1) nb |= 1u << i;
-        }
-      }
+      // the lane's 4 codes decoded a byte at a time with SIMD-in-word operations
+      const uint32_t inm = in ? 0xffffffffu : 0u;
+      const uint32_t bad = (__vcmpgtu4(__vadd4(sw, 0x01010101u), 0x02020202u) |   // s outside {-1, 0, 1}
+                            __vcmpgtu4(__vadd4(pw, 0x0f0f0f0fu), 0x0f0f0f0fu)) &  // p outside [-15, 0]
+                           inm;
+      const uint32_t okm = inm & ~bad;
+      invalid += (uint32_t)__popc(bad & 0x01010101u);
+      const uint32_t nzm = __vcmpne4(sw, 0u) & okm;              // s != 0
+      const uint32_t ngm = __vcmpeq4(sw, 0xffffffffu) & okm;     // s == -1
+      // byte masks (0x00 / 0xff) to 4 bits: (m & 0x01010101) * 0x10204080 >> 28
+      const uint32_t zb = ((nzm & 0x01010101u) * 0x10204080u) >> 28;
+      const uint32_t nb = ((ngm & 0x01010101u) * 0x10204080u) >> 28;
+      // shift nibbles k = -p: byte i of q holds k_i; packed as bits 4i .. 4i + 3
+      const uint32_t q = __vsub4(0u, pw) & okm;
+      const uint32_t nib = __byte_perm(q | (q >> 4), 0u, 0x4420u);  // bytes 0 and 2, then zeros
+      // A: sum of 2^(15 - k) over the nonzero codes, as 2^8 * sum 2^(7 - k) (k < 8) + sum 2^(15 - k) (k >= 8);
+      // each byte's power of two 2^(7 - (k & 7)) from a byte table selected by k & 7
+      const uint32_t pw2 = __byte_perm(0x10204080u, 0x01020408u, nib & 0x7777u) & nzm;
+      const uint32_t hi = __vcmpltu4(q, 0x08080808u);
+      const uint32_t a_sum = (__vsadu4(pw2 & hi, 0u) << 8) + __vsadu4(pw2 & ~hi, 0u);
       nnz += (uint32_t)__popc(zb);
       // planes of chunk q: lane 8q + jj holds bits 4 jj .. 4 jj + 3
       uint32_t np = nb << (4 * jj), zp = zb << (4 * jj);
@@ -190,6 +193,106 @@ __global__ void pack_kernel_vec4(const int8_t* __restrict__ s, const int8_t* __r
   }
 }
 
+// Decode of 4 codes held as the bytes of one word of s and one of p (SIMD
+// in word): the out-of-range count, the non-zero and negative bits (bit i for
+// byte i), the 4 shift nibbles (bits 4i .. 4i + 3) and the codes' share of A.
+struct Quad {
+  uint32_t bad, zb, nb, nib, a;
+};
+__device__ __forceinline__ Quad decode_quad(uint32_t sw, uint32_t pw) {
+  Quad r;
+  const uint32_t bad = __vcmpgtu4(__vadd4(sw, 0x01010101u), 0x02020202u) |  // s outside {-1, 0, 1}
+                       __vcmpgtu4(__vadd4(pw, 0x0f0f0f0fu), 0x0f0f0f0fu);   // p outside [-15, 0]
+  const uint32_t okm = ~bad;
+  const uint32_t nzm = __vcmpne4(sw, 0u) & okm;
+  const uint32_t ngm = __vcmpeq4(sw, 0xffffffffu) & okm;
+  r.bad = (uint32_t)__popc(bad & 0x01010101u);
+  r.zb = ((nzm & 0x01010101u) * 0x10204080u) >> 28;  // byte masks to 4 bits
+  r.nb = ((ngm & 0x01010101u) * 0x10204080u) >> 28;
+  const uint32_t q = __vsub4(0u, pw) & okm;            // k = -p per byte
+  r.nib = __byte_perm(q | (q >> 4), 0u, 0x4420u);
+  // 2^(15 - k) = 2^8 * 2^(7 - k) for k < 8, else 2^(7 - (k - 8)): a byte table selected by k & 7
+  const uint32_t pw2 = __byte_perm(0x10204080u, 0x01020408u, r.nib & 0x7777u) & nzm;
+  const uint32_t hi = __vcmpltu4(q, 0x08080808u);
+  r.a = (__vsadu4(pw2 & hi, 0u) << 8) + __vsadu4(pw2 & ~hi, 0u);
+  return r;
+}
+
+// Packing with 16 codes per lane (k_red a multiple of 16, 16-byte aligned
+// rows): one 16-byte load of s and one of p per lane; a 32-code chunk is a
+// lane pair, whose even lane writes the chunk's first two shift words and the
+// bit planes, the odd lane the last two shift words.  A warp covers 512
+// codes of one column per step.
+__global__ void pack_kernel_vec16(const int8_t* __restrict__ s, const int8_t* __restrict__ p, int64_t n_out,
+                                  int64_t k_red, uint8_t* __restrict__ blob, int64_t parts) {
+  const BlobLayout L = blob_layout(n_out, k_red);
+  BlobHeader* hdr = reinterpret_cast<BlobHeader*>(blob);
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    hdr->magic = DS_WEIGHTS_MAGIC;
+    hdr->format = DS_FORMAT_PLANES6;
+    hdr->n_out = n_out;
+    hdr->k_red = k_red;
+    hdr->n_chunks = L.n_chunks;
+  }
+  const unsigned full = 0xffffffffu;
+  const int lane = threadIdx.x & 31;
+  const int64_t steps = (k_red + 511) / 512;
+  const int64_t per = (steps + parts - 1) / parts;
+  const int64_t units = n_out * parts;
+  uint2* nibw = reinterpret_cast<uint2*>(blob + L.nib);
+  uint2* bits = reinterpret_cast<uint2*>(blob + L.bits);
+  for (int64_t u = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; u < units;
+       u += ((int64_t)gridDim.x * blockDim.x) >> 5) {
+    const int64_t n = u % n_out;
+    const int64_t b0 = (u / n_out) * per;
+    const int64_t b1 = b0 + per < steps ? b0 + per : steps;
+    const uint4* srow = reinterpret_cast<const uint4*>(s + n * k_red);
+    const uint4* prow = reinterpret_cast<const uint4*>(p + n * k_red);
+    uint32_t nnz = 0, invalid = 0;
+    unsigned long long a_col = 0;
+    for (int64_t b = b0; b < b1; b += 2) {  // two steps' loads in flight
+      uint4 sv[2], pv[2];
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        const bool in = b + q < b1 && (b + q) * 512 + 16 * lane < k_red;
+        sv[q] = in ? __ldg(srow + (b + q) * 32 + lane) : make_uint4(0u, 0u, 0u, 0u);
+        pv[q] = in ? __ldg(prow + (b + q) * 32 + lane) : make_uint4(0u, 0u, 0u, 0u);
+      }
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        if (b + q >= b1) break;
+        const Quad d0 = decode_quad(sv[q].x, pv[q].x), d1 = decode_quad(sv[q].y, pv[q].y);
+        const Quad d2 = decode_quad(sv[q].z, pv[q].z), d3 = decode_quad(sv[q].w, pv[q].w);
+        invalid += d0.bad + d1.bad + d2.bad + d3.bad;
+        const uint32_t zb = d0.zb | (d1.zb << 4) | (d2.zb << 8) | (d3.zb << 12);
+        const uint32_t nb = d0.nb | (d1.nb << 4) | (d2.nb << 8) | (d3.nb << 12);
+        nnz += (uint32_t)__popc(zb);
+        const uint32_t a_sum = d0.a + d1.a + d2.a + d3.a;  // at most 16 * 2^15
+        // planes of the lane pair's chunk: the even lane's 16 codes in bits 0..15, the odd lane's in 16..31
+        const int sh = 16 * (lane & 1);
+        uint32_t np = nb << sh, zp = zb << sh;
+        np |= __shfl_xor_sync(full, np, 1);
+        zp |= __shfl_xor_sync(full, zp, 1);
+        const int64_t g = (b + q) * 16 + (lane >> 1);  // this lane's chunk
+        if (g < L.n_chunks) {
+          // shift words 2 (lane & 1), 2 (lane & 1) + 1 of the chunk
+          nibw[((g * n_out + n) * 4 + 2 * (lane & 1)) >> 1] =
+              make_uint2(d0.nib | (d1.nib << 16), d2.nib | (d3.nib << 16));
+          if ((lane & 1) == 0) bits[g * n_out + n] = make_uint2(np, zp);
+        }
+        a_col += __reduce_add_sync(full, a_sum);  // a warp step adds at most 2^24
+      }
+    }
+    nnz = __reduce_add_sync(full, nnz);
+    invalid = __reduce_add_sync(full, invalid);
+    if (lane == 0) {
+      atomicAdd(reinterpret_cast<unsigned long long*>(blob + L.col_a) + n, a_col);
+      atomicAdd(reinterpret_cast<uint32_t*>(blob + L.nnz) + n, nnz);
+      if (invalid) atomicAdd(&hdr->invalid_count, invalid);
+    }
+  }
+}
+
 // Header maxima over the columns' A[n] and nnz[n].
 __global__ void pack_maxima_kernel(uint8_t* __restrict__ blob, int64_t n_out, int64_t k_red) {
   const BlobLayout L = blob_layout(n_out, k_red);
@@ -216,9 +319,6 @@ __global__ void pack_maxima_kernel(uint8_t* __restrict__ blob, int64_t n_out, in
 
 cudaError_t launch_pack(const int8_t* s, const int8_t* p, int64_t n_out, int64_t k_red,
                         uint8_t* blob, cudaStream_t st, const int* bwd) {
-  // zero the whole blob: header counters, column constants (added atomically), tail padding
-  cudaError_t e = cudaMemsetAsync(blob, 0, (size_t)blob_layout(n_out, k_red).total, st);
-  if (e != cudaSuccess) return e;
   const int sms = sm_count();
   if (sms <= 0) return cudaErrorNoDevice;
   BwdMap m{0, 0, 1, 1, 1, 1, 0, 0, 1, 1};
@@ -232,14 +332,29 @@ cudaError_t launch_pack(const int8_t* s, const int8_t* p, int64_t n_out, int64_t
   if (parts < 1) parts = 1;
   const bool vec4 = bwd == nullptr && (k_red % 4) == 0 && (reinterpret_cast<uintptr_t>(s) & 3) == 0 &&
                     (reinterpret_cast<uintptr_t>(p) & 3) == 0;
-  if (vec4) {  // 128-index steps: split a column's steps into parts the same way
-    const int64_t steps = (k_red + 127) / 128;
+  const bool vec16 = vec4 && (k_red % 16) == 0 && (reinterpret_cast<uintptr_t>(s) & 15) == 0 &&
+                     (reinterpret_cast<uintptr_t>(p) & 15) == 0;
+  // zero the header counters, the column constants (added atomically) and the tail padding; the vectorised
+  // kernels write every shift word and bit plane, the general one gets the whole blob zeroed
+  const BlobLayout L = blob_layout(n_out, k_red);
+  cudaError_t e;
+  if (vec4) {
+    e = cudaMemsetAsync(blob, 0, (size_t)L.nib, st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(blob + L.col_a, 0, (size_t)(L.total - L.col_a), st);
+  } else {
+    e = cudaMemsetAsync(blob, 0, (size_t)L.total, st);
+  }
+  if (e != cudaSuccess) return e;
+  if (vec4) {  // 128- or 512-index steps: split a column's steps into parts the same way
+    const int64_t steps = vec16 ? (k_red + 511) / 512 : (k_red + 127) / 128;
     if (parts > steps) parts = steps;
   }
   const int64_t units = n_out * parts;
   int64_t blocks = (units + threads / 32 - 1) / (threads / 32);
   if (blocks > (int64_t)sms * 32) blocks = (int64_t)sms * 32;  // grid-stride beyond
-  if (vec4) {
+  if (vec16) {
+    pack_kernel_vec16<<<(unsigned)blocks, threads, 0, st>>>(s, p, n_out, k_red, blob, parts);
+  } else if (vec4) {
     pack_kernel_vec4<<<(unsigned)blocks, threads, 0, st>>>(s, p, n_out, k_red, blob, parts);
   } else {
     pack_kernel<<<(unsigned)blocks, threads, 0, st>>>(s, p, n_out, k_red, blob, m, parts);

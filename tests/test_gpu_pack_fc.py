@@ -18,7 +18,7 @@ def _pack(ds, s, p, expand=False):
 
 
 @pytest.mark.parametrize("n_out,k_red", [(1, 1), (3, 31), (64, 576), (65, 33), (512, 784), (130, 100),
-                                         (3, 100000), (1024, 1152), (9, 4129)])
+                                         (3, 100000), (1024, 1152), (9, 4129), (7, 48), (5, 528)])
 def test_pack_blob_bitexact(dslib, n_out, k_red):
     seed = n_out * 7919 + k_red
     s = si.sign_codes(seed, (n_out, k_red))
@@ -60,6 +60,21 @@ def test_pack_rejects_bad_codes(dslib):
     p[1, 1] = -16
     with pytest.raises(dslib.DsError):
         _pack(dslib, s, p)
+
+
+@pytest.mark.parametrize("k_red", [10, 48, 100, 512])
+def test_pack_counts_every_bad_code(dslib, k_red):
+    """The out-of-range codes are counted exactly by every packing kernel (scalar, 4 and 16 codes per lane: k_red
+    10, 100 / 48, 512), including positions in a chunk's second half and a tail chunk."""
+    s = si.sign_codes(k_red, (5, k_red))
+    p = si.shift_codes_uniform(k_red, (5, k_red))
+    bad = [(0, 0, 2, 0), (1, k_red - 1, 1, 1), (3, k_red // 2, -2, -3), (4, k_red - 2, 0, -16), (2, 5, -1, 5)]
+    for n, k, sv, pv in bad:
+        s[n, k], p[n, k] = sv, pv
+    with pytest.raises(dslib.DsError) as e:
+        _pack(dslib, s, p)
+    assert e.value.status == dslib.DS_ERR_CODE_RANGE
+    assert str(e.value).split(": ", 1)[1].startswith(f"{len(bad)} codes"), str(e.value)
 
 
 def _run_fc(ds, x, s, p, b, flags=0, amax=True, expand=False):
