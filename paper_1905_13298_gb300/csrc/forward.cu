@@ -1,10 +1,14 @@
-// Chained forward: runs a program of shift layers and integer pools on one
-// stream (ResNet / VGG shaped networks built from the operators of Eq. 3).
+// Chained forward: runs a program of shift layers and integer pools (ResNet /
+// VGG shaped networks built from the operators of Eq. 3) on the caller's
+// stream, with the layers that do not depend on their predecessor on a side
+// stream beside it.
 //
 // Host side: one validation pass computes every slot's shape, the workspace
-// layout and the device max|x| word that bounds each layer's input.  Device
-// side: one memset of the max|x| words, one max|x| pre-pass over the network
-// input, then one launch per layer.  A shift layer reads the max|x| word of
+// layout, the device max|x| word that bounds each layer's input, and each
+// layer's stream and dependencies.  Device side: one memset of the max|x|
+// words and split scratch, one max|x| pre-pass over the network input, then
+// one launch per layer (plus a finalize for split reductions, and events
+// between the streams).  A shift layer reads the max|x| word of
 // its producer (pools pass their input's bound through, since max-pool and
 // floor-average never exceed it) and writes max|y| into its own word, so the
 // accumulator-width proof of every layer happens on the device.
